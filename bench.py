@@ -1,0 +1,359 @@
+#!/usr/bin/env python
+"""Benchmark of the masked-linear hot path on one GB300.
+
+Workload (one step): one Llama-3.2-3B-shaped decoder layer's outsourced
+linears at 128 prompt tokens, fp32, Gaussian noise at eps = 1 -- per input
+group noise + mask, then for each of Q, K, V, O, Gate, Up, Down the
+correction C = eta W^T and the masked product with the fused unmask
+Y = X~ W^T - C.  Weights (1.2 GB per layer incl. the TF32 split) are larger
+than L2, so no step reuses L2-resident weights.
+
+Prints one JSON line.  ``--impl reference`` times the fp64 CPU oracle on a
+bounded sample of the same workload instead.
+"""
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "masked-linear TFLOP/s & ms/prefill (Llama-3B shapes), % of roofline, oracle match"
+UNIT = "TFLOP/s"
+TF32_OVER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate on GB300
+WORKLOAD = "llama-3.2-3b-shaped layer (Q,K,V,O,gate,up,down), 128 tokens, fp32, gaussian eps=1"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--eps", type=float, default=1.0)
+    ap.add_argument("--path", default="auto")
+    ap.add_argument("--tokens", type=int, default=128)
+    ap.add_argument("--cpu-sample-rows", type=int, default=4)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    p = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            m = json.load(f)
+        p.update({k: float(m[k]) for k in ("hbm_gbs", "bf16_tflops", "bf16_tflops_sustained") if k in m})
+        p["source"] = "measured"
+    except (OSError, ValueError, KeyError):
+        pass
+    return p
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is None:
+            return
+        time.sleep(0.2)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        if self.proc is None or not getattr(self, "lines", None):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ----------------------------------------------------------------------------- reference arm
+def oracle_sample(model, M, rows, eps, mech, seed, deltas, weights_cpu, inputs_cpu):
+    """The oracle on the first ``rows`` tokens of every group: noise, mask, products, unmask."""
+    from oracle import linear, philox
+    out = {}
+    flops = 0
+    for gi, (g, K, names) in enumerate(model.input_groups()):
+        X = inputs_cpu[g][:rows]
+        eta = philox.noise((M, K), deltas[g], eps, mech, seed, stream_id=gi)[:rows]
+        Xt = linear.mask(X, eta)
+        for name in names:
+            W = weights_cpu[name]
+            r = linear.masked_linear(Xt, W)
+            C = linear.precompute_noise_product(eta, W)
+            out[name] = linear.unmask(r.astype("float32"), C.astype("float32"))
+            flops += 2 * 2 * rows * K * W.shape[0]
+    return out, flops
+
+
+def cpu_setup(model, M):
+    import numpy as np
+    from oracle import sensitivity as osens
+    from paper_2609_15039_gb300 import workloads as wl
+    weights = {name: wl.weight(N, K, seed=200 + pi).numpy() for pi, (name, K, N, g) in enumerate(model.projections())}
+    inputs = {g: wl.activations(M, K, seed=100 + gi).numpy() for gi, (g, K, _n) in enumerate(model.input_groups())}
+    ones = np.ones(model.d_model)
+    norms = {n: osens.spectral_norm(weights[n], iters=30) for n in ("v", "up", "gate")}
+    deltas = {"qkv": osens.delta_layernorm(ones), "gateup": osens.delta_layernorm(ones),
+              "o": osens.delta_attention(ones, norms["v"]),
+              "down": osens.delta_activation(ones, None, model.d_ff, norms["up"], norms["gate"])}
+    return weights, inputs, deltas
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2609_15039_gb300 import workloads as wl
+    model, M = wl.LLAMA_3_2_3B, args.tokens
+    weights, inputs, deltas = cpu_setup(model, M)
+    rows = args.cpu_sample_rows
+    for w in range(args.warmup):
+        oracle_sample(model, M, rows, args.eps, "gaussian", 1000 + w, deltas, weights, inputs)
+    t0 = time.perf_counter()
+    flops = 0
+    for s in range(args.steps):
+        _, f = oracle_sample(model, M, rows, args.eps, "gaussian", 2000 + s, deltas, weights, inputs)
+        flops += f
+    dt = time.perf_counter() - t0
+    value = flops / dt / 1e12
+    sample = f"first {rows} of {M} tokens of every input group, all 7 projections, per step"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "tokens": M, "eps": args.eps},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+# ----------------------------------------------------------------------------- our arm
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    from paper_2609_15039_gb300 import spl, workloads as wl
+    from paper_2609_15039_gb300.layer import MaskedLayer
+
+    world, rank, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    model, M, mech = wl.LLAMA_3_2_3B, args.tokens, "gaussian"
+
+    weights = {name: wl.weight(N, K, seed=200 + pi, device=dev) for pi, (name, K, N, g) in
+               enumerate(model.projections())}
+    layer = MaskedLayer.from_weights(model, weights, split=True, device=dev)
+    layer.sensitivities(power_iters=60)
+    inputs = {g: wl.activations(M, K, seed=100 + gi, device=dev) for gi, (g, K, _n) in
+              enumerate(model.input_groups())}
+    outputs, scratch = {}, {}
+    stream = torch.cuda.current_stream(dev)
+
+    # per-call events around the product calls (the dominant kernel)
+    prod_events = []
+
+    def timer(phase, kind):
+        if phase == "begin":
+            e = torch.cuda.Event(enable_timing=True)
+            e.record(stream)
+            prod_events.append([kind, e, None])
+        else:
+            e = torch.cuda.Event(enable_timing=True)
+            e.record(stream)
+            prod_events[-1][2] = e
+
+    def step(i, use_timer=False):
+        layer.step(inputs, args.eps, mech, 10_000 + i, outputs=outputs, scratch=scratch, path=args.path,
+                   timer=timer if use_timer else None)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    launches0 = spl.spl_launch_count()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(args.warmup + i, use_timer=True)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    gpu_launches = spl.spl_launch_count() - launches0
+    ms = t_start.elapsed_time(t_end) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    st = spl.spl_get_device_status()
+    if st != spl.SPL_OK:
+        raise RuntimeError("device status " + spl.status_string(st))
+
+    flops_step = layer.flops(M)
+    value = world * flops_step / (ms * 1e-3) / 1e12
+    resolved = spl.spl_resolve_path(M, model.d_model, model.d_model, args.path)
+    path_name = {1: "tf32x3", 2: "fp32"}.get(resolved, str(resolved))
+
+    # roofline of the dominant kernel (the product call)
+    pk = peaks()
+    durs = [(k, b.elapsed_time(e)) for k, b, e in prod_events]
+    prod_ms = sum(d for _, d in durs)
+    n_calls = len(durs)
+    flops_call = flops_step / (2 * len(layer.projections))
+    avg_ms = prod_ms / max(n_calls, 1)
+    achieved = flops_step * args.steps / (prod_ms * 1e-3) / 1e12
+    if path_name == "tf32x3":
+        peak = pk["bf16_tflops_sustained"] * TF32_OVER_BF16 / 3.0
+        peak_note = "measured sustained bf16 x nominal tf32/bf16 (1.1/2.25) / 3 products per term"
+    else:
+        peak = 152 * 128 * 2 * 2.07e9 / 1e12
+        peak_note = "fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2.07 GHz"
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None, "kernel": "product call (masked product / correction)",
+                "avg_call_ms": avg_ms, "calls_per_step": n_calls // max(args.steps, 1),
+                "share_of_step": prod_ms / (ms * args.steps), "peak_source": pk["source"], "peak_note": peak_note,
+                "flops_per_call_avg": flops_call}
+
+    # e2e: inputs from pinned host memory each step, outputs read back
+    host_in = {g: x.cpu().pin_memory() for g, x in inputs.items()}
+    host_out = {name: torch.empty(o.shape, dtype=o.dtype).pin_memory() for name, o in outputs.items()}
+    dev_in = {g: torch.empty_like(x) for g, x in inputs.items()}
+    h2d = sum(x.numel() * 4 for x in host_in.values())
+    d2h = sum(o.numel() * 4 for o in host_out.values())
+
+    def e2e_step(i):
+        for g in dev_in:
+            dev_in[g].copy_(host_in[g], non_blocking=True)
+        layer.step(dev_in, args.eps, mech, 50_000 + i, outputs=outputs, scratch=scratch, path=args.path)
+        for name in host_out:
+            host_out[name].copy_(outputs[name], non_blocking=True)
+
+    for i in range(2):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.steps):
+        e2e_step(10 + i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e = {"value": world * flops_step / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "path": path_name, "data": "synthetic",
+        "config": {"workload": WORKLOAD, "tokens": M, "eps": args.eps, "mech": mech, "layers_per_step": 1,
+                   "flops_per_step": flops_step, "l2": "weights 1.2 GB per step > 129 MB L2 (no flush needed)",
+                   "parallelism": "replicas" if world > 1 else "single"},
+        "ms_per_prefill_28_layers": 28 * ms,
+        "roofline": roofline,
+        "gpu_launches": gpu_launches,
+        "clocks": clocks.summary(),
+        "e2e": e2e,
+    }
+
+    # cpu baseline + oracle match on the first rows (rank 0, N = 1 only)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rows = args.cpu_sample_rows
+        w_cpu = {name: w.cpu().numpy() for name, w in weights.items()}
+        x_cpu = {g: x.cpu().numpy() for g, x in inputs.items()}
+        seed = 777
+        layer.step(inputs, args.eps, mech, seed, outputs=outputs, scratch=scratch, path=args.path)
+        torch.cuda.synchronize()
+        gpu_rows = {name: outputs[name][:rows].double().cpu().numpy() for name in outputs}
+        t0 = time.perf_counter()
+        ref, flops = oracle_sample(model, M, rows, args.eps, mech, seed, layer.deltas, w_cpu, x_cpu)
+        dt = time.perf_counter() - t0
+        result["cpu_baseline"] = {"value": flops / dt / 1e12, "unit": UNIT, "cores": os.cpu_count(),
+                                  "kind": "oracle", "sample": f"first {rows} of {M} tokens, all 7 projections",
+                                  "seconds": dt}
+        from oracle import bounds, linear, philox
+        worst = 0.0
+        for gi, (g, K, names) in enumerate(model.input_groups()):
+            X = x_cpu[g][:rows]
+            eta = philox.noise((M, K), layer.deltas[g], args.eps, mech, seed, stream_id=gi)[:rows]
+            Xt = linear.mask(X, eta)
+            for name in names:
+                S = linear.abs_products(X, Xt, eta, w_cpu[name])
+                err = np.abs(gpu_rows[name] - linear.reference_output(X, w_cpu[name]))
+                worst = max(worst, float(np.max(err / bounds.hard_bound(*S, K))))
+        result["oracle_match"] = {"rows_checked": rows, "max_err_over_hard_bound": worst, "pass": worst <= 1.0}
+
+    if rank == 0:
+        print(json.dumps(result))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,198 @@
+/*
+ * spl.h -- C ABI of the SpliTEE masked-linear hot path on GB300 (sm_103a).
+ *
+ * The method (arxiv 2609.15039, Sec. 3.3.1 and Eq. add-and-then-subtract):
+ * a trusted party masks the input x of a linear layer with differentially
+ * private noise eta, x~ = x + eta; the untrusted GPU computes r = W x~; the
+ * result is unmasked with the precomputed correction W eta,
+ * W x = r - W eta.  The noise follows the Gaussian mechanism with scale
+ * Delta f / eps (Prop. eps-GDP mechanism, Sec. 4.4); a Laplace variant with
+ * the same scale is also offered.  Delta f comes from Thms. 1-3 (Sec. 4.3).
+ *
+ * Conventions for every call
+ *  - Tensors are fp32, row-major and contiguous.  Rows are tokens.
+ *    X, X~ and the noise N are [M, K]; weights W are [N, K] (K contiguous,
+ *    the nn.Linear layout); outputs are [M, N].  The paper writes the same
+ *    product with column vectors (W x); here it is X W^T.
+ *  - Device pointers are owned by the caller.  Every base pointer must be
+ *    16-byte aligned and K must be a multiple of 4 (SPL_EALIGN otherwise).
+ *  - Work is enqueued asynchronously on `stream` (0 = legacy default stream);
+ *    no call synchronises the host except spl_get_device_status and
+ *    spl_spectral_norm.  A zero-sized problem returns SPL_OK and does nothing.
+ *  - Arguments are validated before anything is launched; an invalid call
+ *    launches nothing.  Launch failures return SPL_ECUDA.
+ *  - The library keeps no allocation of its own beyond one device status
+ *    word (set by kernels whose bounded waits expire, read by
+ *    spl_get_device_status).  Scratch memory is passed in as `workspace`.
+ */
+#ifndef SPL_H
+#define SPL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum spl_status {
+  SPL_OK = 0,
+  SPL_EINVAL = 1,       /* invalid value: NULL pointer, eps <= 0 or NaN, negative size, bad enum */
+  SPL_ESHAPE = 2,       /* sizes out of the supported range */
+  SPL_EALIGN = 3,       /* base pointer not 16-byte aligned, or K % 4 != 0 */
+  SPL_ECUDA = 4,        /* a CUDA runtime or driver call failed */
+  SPL_ETIMEOUT = 5,     /* a bounded device-side wait expired (see spl_get_device_status) */
+  SPL_EUNSUPPORTED = 6, /* the requested path cannot run on this device or with these operands */
+  SPL_EWORKSPACE = 7    /* workspace missing or smaller than spl_linear_workspace_bytes() */
+} spl_status;
+
+/* Noise law.  GAUSSIAN is the paper's mechanism (Sec. 4.4); LAPLACE uses the
+ * same scale b = Delta f / eps. */
+typedef enum spl_mech { SPL_MECH_LAPLACE = 0, SPL_MECH_GAUSSIAN = 1 } spl_mech;
+
+/* Arithmetic of the masked product.
+ *  FP32   -- fp32 FMA on the CUDA cores (each product exact before its
+ *            rounding, sequential summation per output).
+ *  TF32X3 -- tcgen05 tensor cores, three TF32 products per term
+ *            (hi*hi + hi*lo + lo*hi, fp32 accumulation in TMEM); needs the
+ *            weight split of spl_split_tf32.
+ *  AUTO   -- the library's choice (spl_resolve_path). */
+typedef enum spl_path { SPL_PATH_AUTO = 0, SPL_PATH_TF32X3 = 1, SPL_PATH_FP32 = 2 } spl_path;
+
+/* Philox4x32-10 stream (Salmon et al., SC'11).  Element e of a flat tensor
+ * uses lane e % 4 of block j = e / 4 + offset (64-bit, wrapping); the
+ * counter is (lo32 j, hi32 j, lo32 stream_id, hi32 stream_id) and the key
+ * (lo32 seed, hi32 seed).  Distinct (seed, stream_id, block) never share a
+ * counter, so draws with disjoint block ranges are independent. */
+typedef struct spl_rng {
+  uint64_t seed;
+  uint64_t stream_id;
+  uint64_t offset;
+} spl_rng;
+
+/* ---- a2: noise --------------------------------------------------------
+ * N[rows, cols] <- eta, scale b = fl32(sensitivity / eps) (Sec. 4.4).
+ *  Laplace: per element one word r; sign = bit 31, u = ((r & 0xFFFFFF)+1) 2^-24,
+ *           eta = +-b (-ln u).
+ *  Gaussian: Box-Muller on word pairs (0,1), (2,3) of a block:
+ *           u1 = ((r_a >> 8)+1) 2^-24, u2 = (r_b >> 8) 2^-24,
+ *           eta_a = b R cos(2 pi u2), eta_b = b R sin(2 pi u2), R = sqrt(-2 ln u1).
+ * eps = +INFINITY writes zeros (the noise-free T3 configuration).
+ * Errors: EINVAL if N is NULL, eps <= 0 or NaN, sensitivity < 0 or not finite,
+ * or mech unknown; EALIGN if N is not 16-byte aligned. */
+spl_status spl_noise(float* N, int64_t rows, int64_t cols, double sensitivity, double eps,
+                     spl_mech mech, spl_rng rng, cudaStream_t stream);
+
+/* The raw 32-bit words of the Philox stream above: out[e] is lane e % 4 of
+ * block e / 4 + rng.offset.  This is the integer stream spl_noise transforms.
+ * Errors: EINVAL for NULL out or count < 0, EALIGN if out is not 16-byte aligned. */
+spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng, cudaStream_t stream);
+
+/* ---- a3: mask ---------------------------------------------------------
+ * Xt = fl32(X + N) elementwise, round-to-nearest (Sec. 3.3.1).  Xt may alias X. */
+spl_status spl_mask(float* Xt, const float* X, const float* N, int64_t rows, int64_t cols,
+                    cudaStream_t stream);
+
+/* ---- a2 + a3 fused ----------------------------------------------------
+ * Draws eta exactly as spl_noise and writes Xt = fl32(X + eta) in one pass.
+ * N_out (may be NULL) receives eta for the correction precompute.
+ * Xt may alias X.  Same errors as spl_noise plus EINVAL for NULL X / Xt. */
+spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, int64_t rows, int64_t cols,
+                          double sensitivity, double eps, spl_mech mech, spl_rng rng,
+                          cudaStream_t stream);
+
+/* ---- weight preparation for TF32X3 ------------------------------------
+ * hi = src rounded to TF32 (10 explicit mantissa bits, ties away), lo = src - hi
+ * (exact in fp32).  Done once per weight; hi and lo are [count] like src. */
+spl_status spl_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream);
+
+/* Path that AUTO resolves to for an M x K x N product on the current device,
+ * assuming the weight split is passed (FP32 or TF32X3).  An explicit path
+ * is returned unchanged. */
+spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path);
+
+/* Bytes of device workspace the three product calls below need for this
+ * problem on the current device (0 if none; for AUTO the larger of the two
+ * paths).  It holds split-K partial sums, the arrival counters of the decode
+ * kernel and, for TF32X3, the TF32 split of the left operand.  It must be
+ * zero-filled before its first use; every call that returns SPL_OK leaves
+ * the counters at zero again.  One workspace must not be used by calls that
+ * can run concurrently. */
+size_t spl_linear_workspace_bytes(int64_t M, int64_t K, int64_t N, spl_path path);
+
+/* ---- a5: masked product -----------------------------------------------
+ * Yt[M, N] = Xt[M, K] W[N, K]^T, the GPU's r = W x~ (Sec. 5.1).
+ * W_hi / W_lo are the spl_split_tf32 halves of W (needed for TF32X3; may be
+ * NULL for FP32, in which case AUTO resolves to FP32).
+ * Errors: EINVAL for NULL operands, EALIGN, EUNSUPPORTED for TF32X3 without
+ * W_hi/W_lo or on a device that is not sm_103/sm_100, EWORKSPACE if the
+ * workspace is too small, ETIMEOUT never (waits are reported through
+ * spl_get_device_status). */
+spl_status spl_masked_linear(float* Yt, const float* Xt, const float* W, const float* W_hi,
+                             const float* W_lo, int64_t M, int64_t K, int64_t N, spl_path path,
+                             void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* ---- a4: correction precompute ----------------------------------------
+ * C[M, N] = Nz[M, K] W[N, K]^T, the correction W eta (Sec. 5.2).  Several
+ * noise draws may be stacked along M (rows are independent).  Same operands,
+ * paths and errors as spl_masked_linear. */
+spl_status spl_precompute_noise_product(float* C, const float* Nz, const float* W,
+                                        const float* W_hi, const float* W_lo, int64_t M, int64_t K,
+                                        int64_t N, spl_path path, void* workspace,
+                                        size_t workspace_bytes, cudaStream_t stream);
+
+/* ---- a6: unmask -------------------------------------------------------
+ * Y = fl32(Yt - C) elementwise (Eq. add-and-then-subtract).  Y may alias Yt. */
+spl_status spl_unmask(float* Y, const float* Yt, const float* C, int64_t rows, int64_t cols,
+                      cudaStream_t stream);
+
+/* ---- a5 + a6 fused ----------------------------------------------------
+ * Y[M, N] = fl32(fl32(Xt W^T) - C): the masked product with the unmask
+ * subtraction done in the product's epilogue.  M <= 16 runs the streaming
+ * decode kernel (W read once at HBM rate, FP32).  Same operands and errors as
+ * spl_masked_linear plus C. */
+spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const float* W, const float* W_hi,
+                                    const float* W_lo, const float* C, int64_t M, int64_t K,
+                                    int64_t N, spl_path path, void* workspace,
+                                    size_t workspace_bytes, cudaStream_t stream);
+
+/* ---- a1: noise scale ----------------------------------------------------
+ * Global l2 sensitivities (Sec. 4.3), evaluated in fp64 on the host from
+ * HOST arrays.  Return a negative value on invalid input.
+ *  Thm. 1: 2 sqrt(d) ||alpha||_4                         (input of Q, K, V, Gate, Up, LM head)
+ *  Thm. 2: 2 sqrt(d) ||W_val||_2 ||alpha||_4              (input of O)
+ *  Thm. 3: 2 sqrt(d_ff) (sqrt(d) ||alpha||_4 + ||beta||_2)^2 ||W_up||_2 ||W_gate||_2  (input of Down)
+ * beta may be NULL (zero). */
+double spl_delta_layernorm(const float* alpha, int64_t d);
+double spl_delta_attention(const float* alpha, int64_t d, double wval_spectral_norm);
+double spl_delta_activation(const float* alpha, const float* beta, int64_t d, int64_t d_ff,
+                            double wup_spectral_norm, double wgate_spectral_norm);
+
+/* ||W||_2 of a DEVICE matrix W[N, K] by power iteration on W^T W (fp32 products,
+ * fp64 norms), `iters` iterations from a fixed pseudo-random start vector.
+ * Needs a device workspace of at least 4 (N + 2 K) + 256 bytes; synchronises
+ * `stream` and writes the result to the HOST double *out. */
+spl_status spl_spectral_norm(double* out, const float* W, int64_t N, int64_t K, int iters,
+                             void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* ---- status -------------------------------------------------------------
+ * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last
+ * call gave up a bounded wait (and clears the flag), else SPL_ECUDA if the
+ * stream reports an error, else SPL_OK. */
+spl_status spl_get_device_status(cudaStream_t stream);
+
+/* Number of kernels this library has launched in this process so far
+ * (all devices, all threads).  Not part of the paper's method: it lets a
+ * caller count the library's launches inside a timed region. */
+uint64_t spl_launch_count(void);
+
+/* Static, NUL-terminated name of a status code. */
+const char* spl_status_string(spl_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPL_H */

@@ -1,0 +1,312 @@
+// a2 noise, a3 mask, a6 unmask and the TF32 split: bandwidth-bound elementwise
+// kernels over flat fp32 tensors.
+//
+// Noise follows the Gaussian mechanism N(0, (Delta f/eps)^2 I) of Sec. 4.4
+// (Prop. eps-GDP mechanism) or the Laplace variant at the same scale, drawn
+// from Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11, Sec. 3.3).  The mask
+// is x~ = x + eta (Sec. 3.3.1) and the unmask r - W eta (Eq.
+// add-and-then-subtract), each one fp32 round-to-nearest operation: the
+// explicit __fadd_rn/__fsub_rn/__fmul_rn keep the compiler from contracting
+// them into an FMA, so the eta written to N is exactly the eta added to x.
+//
+// Layout: one thread handles one Philox block (4 consecutive elements) per
+// step as a float4; two blocks are in flight per loop trip.  The grid is a
+// whole number of waves over the SMs (grid-stride loop).
+
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace spl {
+namespace {
+
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u;  // round multiplier for counter word 0
+constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;  // round multiplier for counter word 2
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;  // key increment, word 0
+constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;  // key increment, word 1
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k0 += kPhiloxW0;
+      k1 += kPhiloxW1;
+    }
+    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
+    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+enum { kLaplace = 0, kGaussian = 1, kZero = 2 };
+
+__device__ __forceinline__ float laplace1(uint32_t r, float b) {
+  const float u = __int2float_rn((int)((r & 0xFFFFFFu) + 1u)) * 0x1p-24f;  // (0, 1], exact
+  const float mag = __fmul_rn(b, -logf(u));
+  return (r >> 31) ? -mag : mag;
+}
+
+__device__ __forceinline__ void gauss2(uint32_t ra, uint32_t rb, float b, float& ea, float& eb) {
+  const float u1 = __int2float_rn((int)((ra >> 8) + 1u)) * 0x1p-24f;  // (0, 1]
+  const float u2 = __int2float_rn((int)(rb >> 8)) * 0x1p-24f;         // [0, 1)
+  const float R = sqrtf(__fmul_rn(-2.0f, logf(u1)));
+  float s, c;
+  sincospif(2.0f * u2, &s, &c);  // sin/cos of 2 pi u2; 2*u2 is exact
+  const float sr = __fmul_rn(b, R);
+  ea = __fmul_rn(sr, c);
+  eb = __fmul_rn(sr, s);
+}
+
+template <int MECH>
+__device__ __forceinline__ float4 draw_block(uint64_t j, uint32_t k0, uint32_t k1, uint32_t s0,
+                                             uint32_t s1, float b) {
+  if (MECH == kZero) return make_float4(0.f, 0.f, 0.f, 0.f);
+  const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
+  float4 e;
+  if (MECH == kLaplace) {
+    e = make_float4(laplace1(r.x, b), laplace1(r.y, b), laplace1(r.z, b), laplace1(r.w, b));
+  } else {
+    gauss2(r.x, r.y, b, e.x, e.y);
+    gauss2(r.z, r.w, b, e.z, e.w);
+  }
+  return e;
+}
+
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+  return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z), __fadd_rn(a.w, b.w));
+}
+
+// xt = x + eta (if xt), nout = eta (if nout).  n elements, nb = ceil(n/4) Philox blocks.
+template <int MECH>
+__global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* __restrict__ nout,
+                                                              const float* x, int64_t n, float b,
+                                                              uint32_t k0, uint32_t k1, uint32_t s0, uint32_t s1,
+                                                              uint64_t offset) {
+  const int64_t nb_full = n >> 2;  // blocks with all 4 elements in range
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  float4* xt4 = reinterpret_cast<float4*>(xt);
+  float4* n4 = reinterpret_cast<float4*>(nout);
+  // two blocks per trip: issue both loads first
+  for (; i + stride < nb_full; i += 2 * stride) {
+    float4 xa, xb;
+    if (xt) {
+      xa = __ldcs(x4 + i);
+      xb = __ldcs(x4 + i + stride);
+    }
+    const float4 ea = draw_block<MECH>((uint64_t)i + offset, k0, k1, s0, s1, b);
+    const float4 eb = draw_block<MECH>((uint64_t)(i + stride) + offset, k0, k1, s0, s1, b);
+    if (nout) {
+      __stcs(n4 + i, ea);
+      __stcs(n4 + i + stride, eb);
+    }
+    if (xt) {
+      __stcs(xt4 + i, add4(xa, ea));
+      __stcs(xt4 + i + stride, add4(xb, eb));
+    }
+  }
+  for (; i < nb_full; i += stride) {
+    const float4 e = draw_block<MECH>((uint64_t)i + offset, k0, k1, s0, s1, b);
+    if (nout) __stcs(n4 + i, e);
+    if (xt) __stcs(xt4 + i, add4(__ldcs(x4 + i), e));
+  }
+  // ragged tail: the last, partial Philox block
+  if (blockIdx.x == 0 && threadIdx.x == 0 && (n & 3)) {
+    const int64_t j = nb_full;
+    const float4 e = draw_block<MECH>((uint64_t)j + offset, k0, k1, s0, s1, b);
+    const float ev[4] = {e.x, e.y, e.z, e.w};
+    for (int l = 0; l < (int)(n & 3); ++l) {
+      const int64_t idx = 4 * j + l;
+      if (nout) nout[idx] = ev[l];
+      if (xt) xt[idx] = __fadd_rn(x[idx], ev[l]);
+    }
+  }
+}
+
+// The raw Philox words of the stream (element e = lane e % 4 of block e / 4 + offset).
+__global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restrict__ out, int64_t n, uint32_t k0,
+                                                               uint32_t k1, uint32_t s0, uint32_t s1,
+                                                               uint64_t offset) {
+  const int64_t nb = (n + 3) >> 2;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
+    const uint64_t j = (uint64_t)i + offset;
+    const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
+    if (4 * i + 3 < n) {
+      reinterpret_cast<uint4*>(out)[i] = r;
+    } else {
+      const uint32_t rv[4] = {r.x, r.y, r.z, r.w};
+      for (int l = 0; l < 4 && 4 * i + l < n; ++l) out[4 * i + l] = rv[l];
+    }
+  }
+}
+
+// out = a + s * b elementwise with s = +1 (mask) or -1 (unmask), one rounding.
+template <bool SUB>
+__global__ void __launch_bounds__(kThreads) addsub_kernel(float* out, const float* a,
+                                                          const float* __restrict__ b, int64_t n) {
+  const int64_t n4 = n >> 2;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const float4* a4 = reinterpret_cast<const float4*>(a);
+  const float4* b4 = reinterpret_cast<const float4*>(b);
+  float4* o4 = reinterpret_cast<float4*>(out);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
+    const float4 x = __ldcs(a4 + i), y = __ldcs(b4 + i);
+    float4 r;
+    if (SUB) {
+      r = make_float4(__fsub_rn(x.x, y.x), __fsub_rn(x.y, y.y), __fsub_rn(x.z, y.z), __fsub_rn(x.w, y.w));
+    } else {
+      r = add4(x, y);
+    }
+    __stcs(o4 + i, r);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < (n & 3)) {
+    const int64_t idx = 4 * n4 + threadIdx.x;
+    out[idx] = SUB ? __fsub_rn(a[idx], b[idx]) : __fadd_rn(a[idx], b[idx]);
+  }
+}
+
+__device__ __forceinline__ float tf32_rna(float v) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(v));
+  return __uint_as_float(r);
+}
+
+__global__ void __launch_bounds__(kThreads) split_tf32_kernel(float* __restrict__ hi, float* __restrict__ lo,
+                                                              const float* __restrict__ src, int64_t n) {
+  const int64_t n4 = n >> 2;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const float4* s4 = reinterpret_cast<const float4*>(src);
+  float4* h4 = reinterpret_cast<float4*>(hi);
+  float4* l4 = reinterpret_cast<float4*>(lo);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
+    const float4 v = __ldcs(s4 + i);
+    const float4 h = make_float4(tf32_rna(v.x), tf32_rna(v.y), tf32_rna(v.z), tf32_rna(v.w));
+    h4[i] = h;
+    l4[i] = make_float4(__fsub_rn(v.x, h.x), __fsub_rn(v.y, h.y), __fsub_rn(v.z, h.z), __fsub_rn(v.w, h.w));
+  }
+  if (blockIdx.x == 0 && threadIdx.x < (n & 3)) {
+    const int64_t idx = 4 * n4 + threadIdx.x;
+    const float h = tf32_rna(src[idx]);
+    hi[idx] = h;
+    lo[idx] = __fsub_rn(src[idx], h);
+  }
+}
+
+int grid_for(int64_t work_items, int blocks_per_sm) {
+  const int64_t want = ceil_div(work_items, kThreads);
+  const int64_t cap = (int64_t)device_sm_count() * blocks_per_sm;
+  return (int)std::max<int64_t>(1, std::min(want, cap));
+}
+
+spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech) {
+  if (rows < 0 || cols < 0) return SPL_EINVAL;
+  if (!(eps > 0.0)) return SPL_EINVAL;  // also rejects NaN
+  if (!(sensitivity >= 0.0) || std::isinf(sensitivity)) return SPL_EINVAL;
+  if (mech != SPL_MECH_LAPLACE && mech != SPL_MECH_GAUSSIAN) return SPL_EINVAL;
+  return SPL_OK;
+}
+
+spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, double sensitivity, double eps,
+                             spl_mech mech, spl_rng rng, cudaStream_t stream) {
+  const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
+  const int grid = grid_for(ceil_div(n, 4), 8);
+  const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
+  const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
+  if (b == 0.0f) {
+    noise_mask_kernel<kZero><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset);
+  } else if (mech == SPL_MECH_LAPLACE) {
+    noise_mask_kernel<kLaplace><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset);
+  } else {
+    noise_mask_kernel<kGaussian><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset);
+  }
+  return launch_status();
+}
+
+}  // namespace
+
+spl_status run_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {
+  if (count == 0) return SPL_OK;
+  split_tf32_kernel<<<grid_for(ceil_div(count, 4), 8), kThreads, 0, stream>>>(hi, lo, src, count);
+  return launch_status();
+}
+
+spl_status run_addsub(float* out, const float* a, const float* b, int64_t n, bool sub, cudaStream_t stream) {
+  if (n == 0) return SPL_OK;
+  const int grid = grid_for(ceil_div(n, 4), 8);
+  if (sub) {
+    addsub_kernel<true><<<grid, kThreads, 0, stream>>>(out, a, b, n);
+  } else {
+    addsub_kernel<false><<<grid, kThreads, 0, stream>>>(out, a, b, n);
+  }
+  return launch_status();
+}
+
+}  // namespace spl
+
+using namespace spl;
+
+extern "C" spl_status spl_noise(float* N, int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech,
+                                spl_rng rng, cudaStream_t stream) {
+  spl_status st = validate_noise(rows, cols, sensitivity, eps, mech);
+  if (st != SPL_OK) return st;
+  const int64_t n = rows * cols;
+  if (n == 0) return SPL_OK;
+  if (!N) return SPL_EINVAL;
+  if (!aligned16(N)) return SPL_EALIGN;
+  return launch_noise_mask(nullptr, N, nullptr, n, sensitivity, eps, mech, rng, stream);
+}
+
+extern "C" spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng, cudaStream_t stream) {
+  if (count < 0) return SPL_EINVAL;
+  if (count == 0) return SPL_OK;
+  if (!out) return SPL_EINVAL;
+  if (!aligned16(out)) return SPL_EALIGN;
+  random_bits_kernel<<<grid_for(ceil_div(count, 4), 8), kThreads, 0, stream>>>(
+      out, count, (uint32_t)rng.seed, (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id,
+      (uint32_t)(rng.stream_id >> 32), rng.offset);
+  return launch_status();
+}
+
+extern "C" spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, int64_t rows, int64_t cols,
+                                     double sensitivity, double eps, spl_mech mech, spl_rng rng,
+                                     cudaStream_t stream) {
+  spl_status st = validate_noise(rows, cols, sensitivity, eps, mech);
+  if (st != SPL_OK) return st;
+  const int64_t n = rows * cols;
+  if (n == 0) return SPL_OK;
+  if (!Xt || !X) return SPL_EINVAL;
+  if (!aligned16(Xt) || !aligned16(X) || (N_out && !aligned16(N_out))) return SPL_EALIGN;
+  return launch_noise_mask(Xt, N_out, X, n, sensitivity, eps, mech, rng, stream);
+}
+
+extern "C" spl_status spl_mask(float* Xt, const float* X, const float* N, int64_t rows, int64_t cols,
+                               cudaStream_t stream) {
+  if (rows < 0 || cols < 0) return SPL_EINVAL;
+  const int64_t n = rows * cols;
+  if (n == 0) return SPL_OK;
+  if (!Xt || !X || !N) return SPL_EINVAL;
+  if (!aligned16(Xt) || !aligned16(X) || !aligned16(N)) return SPL_EALIGN;
+  return run_addsub(Xt, X, N, n, false, stream);
+}
+
+extern "C" spl_status spl_unmask(float* Y, const float* Yt, const float* C, int64_t rows, int64_t cols,
+                                 cudaStream_t stream) {
+  if (rows < 0 || cols < 0) return SPL_EINVAL;
+  const int64_t n = rows * cols;
+  if (n == 0) return SPL_OK;
+  if (!Y || !Yt || !C) return SPL_EINVAL;
+  if (!aligned16(Y) || !aligned16(Yt) || !aligned16(C)) return SPL_EALIGN;
+  return run_addsub(Y, Yt, C, n, true, stream);
+}
+
+extern "C" spl_status spl_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {
+  if (count < 0) return SPL_EINVAL;
+  if (count == 0) return SPL_OK;
+  if (!hi || !lo || !src) return SPL_EINVAL;
+  if (!aligned16(hi) || !aligned16(lo) || !aligned16(src)) return SPL_EALIGN;
+  return run_split_tf32(hi, lo, src, count, stream);
+}

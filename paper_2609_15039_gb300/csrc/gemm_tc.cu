@@ -1,0 +1,431 @@
+// TF32X3 product on the 5th-generation tensor cores (tcgen05, sm_103a):
+//   out[M, N] = A[M, K] W[N, K]^T (- C)
+// with every operand split into a TF32 high part and an fp32 residual,
+// a = a_hi + a_lo, and three TF32 products per term accumulated in fp32:
+//   a w ~ a_lo w_hi + a_hi w_lo + a_hi w_hi     (the a_lo w_lo term is dropped).
+// The tensor core keeps 10 explicit mantissa bits of each operand; with
+// round-to-nearest hi parts the per-product error is about 2^-20 |a w|, so the
+// masked product r = W x~ (Sec. 5.1) and the correction W eta (Sec. 5.2) stay
+// inside the binary32 bound gamma_d <|w|,|x|> the paper's Thm. 4 is built on
+// for reduction lengths d >= 64, while running on the tensor pipe.  The paper
+// computes these products on a GPU in FP32 (Sec. 5, Sec. 6.3.2); this is the
+// GB300 way to get that accuracy.
+//
+// Kernel shape (one CTA per 128 x 256 output tile, one CTA per SM):
+//   warp 0      TMA producer: four tiles per stage (A_hi, A_lo, W_hi, W_lo),
+//               K step 16 fp32 = 64 bytes, 64-byte swizzle, 4-stage ring.
+//   warp 1      TMEM allocator and MMA issuer: per stage 2 k-steps x 3
+//               tcgen05.mma.kind::tf32 (M=128, N=256, K=8) into one fp32
+//               accumulator of 256 TMEM columns; tcgen05.commit frees the
+//               stage and finally signals the epilogue.
+//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns at a time,
+//               subtract C (the fused unmask of Eq. add-and-then-subtract)
+//               and store, or store split-K partials.
+// Every mbarrier wait is bounded (about 1 s of globaltimer); on expiry the
+// kernel raises the device status word, lets in-flight copies land (again
+// with a bound), frees its TMEM and returns.
+
+#include <algorithm>
+#include <cstring>
+
+#include <cuda.h>
+
+#include "common.cuh"
+
+namespace spl {
+
+__device__ unsigned int g_device_status = 0u;
+
+cudaError_t read_clear_device_status(unsigned int* word) {
+  cudaError_t e = cudaMemcpyFromSymbol(word, g_device_status, sizeof(unsigned int));
+  if (e != cudaSuccess) return e;
+  if (*word != 0u) {
+    const unsigned int zero = 0u;
+    e = cudaMemcpyToSymbol(g_device_status, &zero, sizeof(zero));
+  }
+  return e;
+}
+
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 16, STAGES = 4, THREADS = 192;
+constexpr int UMMA_K = 8;                                      // K of one kind::tf32 MMA
+constexpr uint32_t A_TILE_BYTES = BM * BK * 4;                 // 8 KB
+constexpr uint32_t B_TILE_BYTES = BN * BK * 4;                 // 16 KB
+constexpr uint32_t STAGE_BYTES = 2 * A_TILE_BYTES + 2 * B_TILE_BYTES;  // 48 KB
+constexpr uint32_t BAR_OFFSET = STAGES * STAGE_BYTES;          // barriers after the ring
+constexpr uint32_t SMEM_BYTES = BAR_OFFSET + 256 + 1024;       // + barriers + alignment slack
+constexpr uint32_t TMEM_COLS = 256;
+constexpr unsigned long long kWaitNs = 1000000000ull;          // 1 s per wait
+constexpr unsigned long long kDrainNs = 100000000ull;          // 0.1 s to drain on abort
+
+// ---- instruction and shared-memory descriptors (tcgen05) -------------------
+// Instruction descriptor, kind::tf32: D = F32 (bits 4-5 = 1), A = B = TF32
+// (bits 7-9 and 10-12 = 2), both K-major (bits 15, 16 = 0), N >> 3 at bits
+// 17-22, M >> 4 at bits 24-28.
+constexpr uint32_t make_idesc_tf32(int m, int n) {
+  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+constexpr uint32_t kIdesc = make_idesc_tf32(BM, BN);
+static_assert(kIdesc == 0x08400910u, "idesc encoding");
+
+// Shared-memory matrix descriptor for a K-major tile written by TMA with the
+// 64-byte swizzle: rows of 64 bytes, 8-row (512-byte) swizzle atoms stacked
+// along M/N.  start address >> 4 in bits 0-13, leading byte offset >> 4 in
+// 16-29 (not used by swizzled K-major layouts; 1), stride byte offset >> 4
+// (512 B between 8-row groups) in 32-45, descriptor version 1 at bit 46,
+// base offset 0 (atoms are 512-byte aligned), layout SWIZZLE_64B = 4 at 61-63.
+__device__ __forceinline__ uint64_t make_sdesc_sw64(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1u << 16;
+  d |= (uint64_t)(512u >> 4) << 32;
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)4u << 61;
+  return d;
+}
+
+// ---- PTX wrappers ----------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ unsigned long long now_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase of the given parity.  Returns false if it gave
+// up (deadline passed or another role raised *abort).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned long long budget_ns,
+                                          volatile int* abort) {
+  if (mbar_try(bar, parity)) return true;
+  const unsigned long long deadline = now_ns() + budget_ns;
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try(bar, parity)) return true;
+    if ((it & 63u) == 0u) {
+      if (abort && *abort) return false;
+      if (now_ns() > deadline) return false;
+    }
+  }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// 32 lanes x 32 columns of 32-bit words: thread t gets lane (base + t), columns col..col+31.
+__device__ __forceinline__ void tmem_ld_32x32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+struct TcMaps {
+  CUtensorMap a_hi, a_lo, w_hi, w_lo;
+};
+
+__global__ void __launch_bounds__(THREADS, 1)
+tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
+               int64_t M, int64_t K, int64_t N, int64_t k_per_split, int splits) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + BAR_OFFSET);  // full[S], empty[S], accum
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + BAR_OFFSET + 8 * (2 * STAGES + 1));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + BAR_OFFSET + 8 * (2 * STAGES + 1) + 8);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t m0 = (int64_t)blockIdx.y * BM, n0 = (int64_t)blockIdx.x * BN;
+  const int split = blockIdx.z;
+  const int64_t kbeg = (int64_t)split * k_per_split;
+  const int64_t kend = std::min<int64_t>(K, kbeg + k_per_split);
+  const int nk = (int)ceil_div(kend - kbeg, BK);
+
+  const uint32_t bar_base = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar_base + 8u * s; };
+  auto empty_bar = [&](int s) { return bar_base + 8u * (STAGES + s); };
+  const uint32_t accum_bar = bar_base + 8u * (2 * STAGES);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(accum_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(smem_u32(const_cast<uint32_t*>(tmem_slot)), TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      uint32_t issued_mask = 0u, phase_mask = 0u;  // per stage: a load was issued / its parity
+      bool ok = true;
+      for (int kb = 0; kb < nk && ok; ++kb) {
+        const int s = kb % STAGES;
+        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+        if (!mbar_wait(empty_bar(s), ph ^ 1u, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        const uint32_t st = smem_u32(smem + (size_t)s * STAGE_BYTES);
+        const int kx = (int)(kbeg + (int64_t)kb * BK);
+        mbar_expect_tx(full_bar(s), STAGE_BYTES);
+        tma_load_2d(st, &maps.a_hi, full_bar(s), kx, (int)m0);
+        tma_load_2d(st + A_TILE_BYTES, &maps.a_lo, full_bar(s), kx, (int)m0);
+        tma_load_2d(st + 2 * A_TILE_BYTES, &maps.w_hi, full_bar(s), kx, (int)n0);
+        tma_load_2d(st + 2 * A_TILE_BYTES + B_TILE_BYTES, &maps.w_lo, full_bar(s), kx, (int)n0);
+        issued_mask |= 1u << s;
+        phase_mask = (phase_mask & ~(1u << s)) | (ph << s);
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(&g_device_status, kStatusTimeout);
+        // let copies already issued land before the CTA exits
+        for (int s = 0; s < STAGES; ++s)
+          if (issued_mask & (1u << s)) mbar_wait(full_bar(s), (phase_mask >> s) & 1u, kDrainNs, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      bool ok = true;
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % STAGES;
+        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+        if (!mbar_wait(full_bar(s), ph, kWaitNs, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t st = smem_u32(smem + (size_t)s * STAGE_BYTES);
+        const uint32_t a_hi = st, a_lo = st + A_TILE_BYTES;
+        const uint32_t w_hi = st + 2 * A_TILE_BYTES, w_lo = w_hi + B_TILE_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+          const uint32_t koff = kk * UMMA_K * 4;  // 32 bytes along the swizzled row
+          const uint32_t first = (kb == 0 && kk == 0) ? 0u : 1u;
+          mma_tf32(tmem, make_sdesc_sw64(a_lo + koff), make_sdesc_sw64(w_hi + koff), kIdesc, first);
+          mma_tf32(tmem, make_sdesc_sw64(a_hi + koff), make_sdesc_sw64(w_lo + koff), kIdesc, 1u);
+          mma_tf32(tmem, make_sdesc_sw64(a_hi + koff), make_sdesc_sw64(w_hi + koff), kIdesc, 1u);
+        }
+        mma_commit(empty_bar(s));  // stage reusable once these MMAs have read it
+      }
+      if (ok) {
+        mma_commit(accum_bar);
+      } else {
+        *abort_flag = 1;
+        atomicOr(&g_device_status, kStatusTimeout);
+        // MMAs already issued must finish before TMEM is released
+        mma_commit(accum_bar);
+        mbar_wait(accum_bar, 0u, kDrainNs, nullptr);
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5) ----------------
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    bool ok = (nk > 0) ? mbar_wait(accum_bar, 0u, kWaitNs * 4, abort_flag) : true;
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok && !*abort_flag) {
+      tc_fence_after();
+      const int64_t m = m0 + 32 * q + lane;
+      float* dst = splits > 1 ? out + (int64_t)split * M * N : out;
+      const bool vec = (N & 3) == 0;
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        float v[32];
+        if (nk > 0) {
+          tmem_ld_32x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(32 * c), v);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = 0.f;
+        }
+        const int64_t nb = n0 + 32 * c;
+        if (m < M && nb < N) {
+          float* orow = dst + m * N;
+          const float* crow = (splits == 1 && C) ? C + m * N : nullptr;
+          if (vec && nb + 32 <= N) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              float4 r = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+              if (crow) {
+                const float4 cc = __ldcs(reinterpret_cast<const float4*>(crow + nb + j));
+                r = make_float4(__fsub_rn(r.x, cc.x), __fsub_rn(r.y, cc.y), __fsub_rn(r.z, cc.z),
+                                __fsub_rn(r.w, cc.w));
+              }
+              *reinterpret_cast<float4*>(orow + nb + j) = r;
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (nb + j < N) orow[nb + j] = crow ? __fsub_rn(v[j], crow[nb + j]) : v[j];
+          }
+        }
+      }
+    } else if (!ok) {
+      if (lane == 0) {
+        *abort_flag = 1;
+        atomicOr(&g_device_status, kStatusTimeout);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// ---- host side: tensor maps ---------------------------------------------------
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2-D fp32 map over a row-major [rows, K] matrix with a 16 x box_rows box, 64-byte swizzle.
+bool make_map(CUtensorMap* map, const float* base, int64_t rows, int64_t K, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)K * 4};
+  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
+  Plan p{};
+  p.kernel = kKernelTc;
+  const int64_t tiles = ceil_div(M, BM) * ceil_div(N, BN);
+  int64_t s = tiles >= sms ? 1 : std::max<int64_t>(1, sms / std::max<int64_t>(tiles, 1));
+  s = std::min<int64_t>(s, std::max<int64_t>(1, K / 256));  // at least 256 K per split
+  p.k_per_split = round_up(ceil_div(K, s), BK);
+  p.splits = (int)std::max<int64_t>(1, ceil_div(K, p.k_per_split));
+  p.ws_partials = p.splits > 1 ? (size_t)round_up((int64_t)p.splits * M * N * 4, 256) : 0;
+  p.ws_asplit = (size_t)round_up(M * K * 4, 256) * 2;
+  return p;
+}
+
+spl_status run_tc(const LinearArgs& a, const Plan& p) {
+  const int cc = device_cc();
+  if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
+  if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
+  if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
+  if (a.M > 0x7fffffffLL || a.N > 0x7fffffffLL || a.K > 0x7fffffffLL) return SPL_ESHAPE;
+  if (ceil_div(a.M, BM) > 65535 || p.splits > 65535) return SPL_ESHAPE;
+
+  // A operand split into the workspace: [hi | lo], each M*K fp32
+  char* ws = static_cast<char*>(a.ws);
+  float* part = reinterpret_cast<float*>(ws);
+  float* a_hi = reinterpret_cast<float*>(ws + p.ws_partials);
+  float* a_lo = reinterpret_cast<float*>(ws + p.ws_partials + p.ws_asplit / 2);
+  spl_status st = run_split_tf32(a_hi, a_lo, a.a, a.M * a.K, a.stream);
+  if (st != SPL_OK) return st;
+
+  TcMaps maps;
+  std::memset(&maps, 0, sizeof(maps));
+  if (!make_map(&maps.a_hi, a_hi, a.M, a.K, BM) || !make_map(&maps.a_lo, a_lo, a.M, a.K, BM) ||
+      !make_map(&maps.w_hi, a.w_hi, a.N, a.K, BN) || !make_map(&maps.w_lo, a.w_lo, a.N, a.K, BN))
+    return SPL_ECUDA;
+
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    if (cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) !=
+        cudaSuccess)
+      return SPL_ECUDA;
+    attr_set[dev] = true;
+  }
+  dim3 grid((unsigned)ceil_div(a.N, BN), (unsigned)ceil_div(a.M, BM), (unsigned)p.splits);
+  float* dst = p.splits > 1 ? part : a.out;
+  tc_gemm_kernel<<<grid, THREADS, SMEM_BYTES, a.stream>>>(maps, dst, p.splits > 1 ? nullptr : a.c, a.M, a.K, a.N,
+                                                          p.k_per_split, p.splits);
+  st = launch_status();
+  if (st != SPL_OK || p.splits == 1) return st;
+  return run_splitk_reduce(a.out, part, a.c, p.splits, a.M, a.N, a.stream);
+}
+
+}  // namespace spl

@@ -1,0 +1,204 @@
+// Streaming decode product for M <= 16 rows: out[M, N] = X~[M, K] W[N, K]^T (- C).
+//
+// At decode (one new token per step, Sec. 2.2; the paper's server batch is
+// 15 prompts, Sec. 6.1) the product reads every weight once and does only M
+// FMAs per weight, so it is bound by HBM bandwidth, not by arithmetic.  This
+// kernel streams W exactly once with 16-byte cache-streaming loads, keeps the
+// K-slice of X~ in shared memory, and fuses the unmask r - W eta (Eq.
+// add-and-then-subtract) into the final write.
+//
+// Work unit: a 256-thread block owns 32 (M <= 4) or 16 consecutive rows of W
+// over one K-slice; lanes stride the slice in float4 steps and every lane
+// keeps 4 x M partial dot products in registers, reduced across the warp
+// with shuffles at the end.  The K-split is a multiple of 128 elements and
+// is sized so the grid fills the SMs.  With more than one split, each block
+// writes fp32 partials to the workspace and bumps an arrival counter; the
+// last block of a row group sums the partials in split order (deterministic),
+// subtracts C, writes the result and resets the counter to zero.
+
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace spl {
+namespace {
+
+constexpr int THREADS = 256, WARPS = 8;
+constexpr int SMEM_FLOATS = 12000;  // just under 48 KB of X~ slice (static smem adds a few bytes)
+
+// Rows of W per warp: 4 for M <= 4, 2 for larger M (bounds the 4 x M accumulators).
+constexpr int rows_per_warp(int mt) { return mt >= 8 ? 2 : 4; }
+
+template <int MT, int ROWS_PER_WARP>
+__global__ void __launch_bounds__(THREADS)
+gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* __restrict__ W,
+            const float* __restrict__ C, float* __restrict__ part, unsigned int* __restrict__ counters, int M,
+            int64_t K, int64_t N, int64_t ks, int splits) {
+  constexpr int ROWS_PER_BLOCK = WARPS * ROWS_PER_WARP;
+  extern __shared__ __align__(16) float xs[];  // [MT][ks]
+  __shared__ int s_last;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.y;
+  const int64_t k0 = (int64_t)split * ks;
+  const int64_t klen = std::min<int64_t>(ks, K - k0);  // multiple of 4
+
+  // stage X~[:, k0:k0+klen] (rows >= M are zero)
+  const int64_t q_per_row = klen >> 2;
+  for (int64_t q = threadIdx.x; q < (int64_t)MT * q_per_row; q += THREADS) {
+    const int m = (int)(q / q_per_row);
+    const int64_t kq = (q - (int64_t)m * q_per_row) * 4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (m < M) v = __ldg(reinterpret_cast<const float4*>(X + (int64_t)m * K + k0 + kq));
+    *reinterpret_cast<float4*>(xs + (int64_t)m * ks + kq) = v;
+  }
+  __syncthreads();
+
+  const int64_t nbase = (int64_t)blockIdx.x * ROWS_PER_BLOCK + warp * ROWS_PER_WARP;
+  const float* wrow[ROWS_PER_WARP];
+  bool valid[ROWS_PER_WARP];
+#pragma unroll
+  for (int r = 0; r < ROWS_PER_WARP; ++r) {
+    valid[r] = nbase + r < N;
+    wrow[r] = W + (valid[r] ? (nbase + r) : 0) * K + k0;
+  }
+
+  float acc[ROWS_PER_WARP][MT];
+#pragma unroll
+  for (int r = 0; r < ROWS_PER_WARP; ++r)
+#pragma unroll
+    for (int m = 0; m < MT; ++m) acc[r][m] = 0.f;
+
+#pragma unroll 2
+  for (int64_t kk = lane * 4; kk < klen; kk += 128) {
+    float4 wv[ROWS_PER_WARP];
+#pragma unroll
+    for (int r = 0; r < ROWS_PER_WARP; ++r)
+      wv[r] = valid[r] ? __ldcs(reinterpret_cast<const float4*>(wrow[r] + kk)) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      const float4 xv = *reinterpret_cast<const float4*>(xs + (int64_t)m * ks + kk);
+#pragma unroll
+      for (int r = 0; r < ROWS_PER_WARP; ++r) {
+        float a = acc[r][m];
+        a = fmaf(wv[r].x, xv.x, a);
+        a = fmaf(wv[r].y, xv.y, a);
+        a = fmaf(wv[r].z, xv.z, a);
+        a = fmaf(wv[r].w, xv.w, a);
+        acc[r][m] = a;
+      }
+    }
+  }
+
+  // warp reduction: lane 0 ends with the full sums
+#pragma unroll
+  for (int r = 0; r < ROWS_PER_WARP; ++r)
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      float v = acc[r][m];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+      acc[r][m] = v;
+    }
+
+  if (splits == 1) {
+    if (lane == 0) {
+#pragma unroll
+      for (int r = 0; r < ROWS_PER_WARP; ++r) {
+        if (!valid[r]) continue;
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+          if (m >= M) break;
+          const int64_t o = (int64_t)m * N + nbase + r;
+          out[o] = C ? __fsub_rn(acc[r][m], C[o]) : acc[r][m];
+        }
+      }
+    }
+    return;
+  }
+
+  float* mypart = part + (int64_t)split * M * N;
+  if (lane == 0) {
+#pragma unroll
+    for (int r = 0; r < ROWS_PER_WARP; ++r) {
+      if (!valid[r]) continue;
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        if (m >= M) break;
+        __stcg(mypart + (int64_t)m * N + nbase + r, acc[r][m]);
+      }
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned int prev = atomicAdd(counters + blockIdx.x, 1u);
+    s_last = (prev == (unsigned int)(splits - 1));
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const int64_t n0 = (int64_t)blockIdx.x * ROWS_PER_BLOCK;
+  for (int idx = threadIdx.x; idx < ROWS_PER_BLOCK * M; idx += THREADS) {
+    const int m = idx / ROWS_PER_BLOCK;
+    const int64_t n = n0 + (idx % ROWS_PER_BLOCK);
+    if (n >= N) continue;
+    const int64_t o = (int64_t)m * N + n;
+    float s = __ldcg(part + o);
+    for (int sp = 1; sp < splits; ++sp) s = __fadd_rn(s, __ldcg(part + (int64_t)sp * M * N + o));
+    out[o] = C ? __fsub_rn(s, C[o]) : s;
+  }
+  if (threadIdx.x == 0) counters[blockIdx.x] = 0u;
+}
+
+int padded_m(int64_t M) { return M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : M <= 8 ? 8 : 16; }
+
+template <int MT>
+spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int* counters) {
+  constexpr int R = rows_per_warp(MT);
+  dim3 grid((unsigned)ceil_div(a.N, WARPS * R), (unsigned)p.splits);
+  const size_t smem = (size_t)MT * p.k_per_split * sizeof(float);
+  gemv_kernel<MT, R><<<grid, THREADS, smem, a.stream>>>(a.out, a.a, a.w, a.c, part, counters, (int)a.M, a.K, a.N,
+                                                      p.k_per_split, p.splits);
+  return launch_status();
+}
+
+}  // namespace
+
+Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
+  Plan p{};
+  p.kernel = kKernelGemv;
+  const int mt = padded_m(M);
+  const int64_t ks_max = (SMEM_FLOATS / mt) / 128 * 128;
+  const int64_t groups = ceil_div(N, WARPS * rows_per_warp(mt));
+  const int64_t target = (int64_t)sms * 4;  // about four 8-warp blocks per SM
+  int64_t s = std::max<int64_t>(1, ceil_div(target, groups));
+  s = std::min<int64_t>(s, std::max<int64_t>(1, K / 256));  // at least 256 K per split
+  int64_t ks = round_up(ceil_div(K, s), 128);
+  ks = std::min<int64_t>(ks, ks_max);
+  p.k_per_split = ks;
+  p.splits = (int)ceil_div(K, ks);
+  if (p.splits > 1) {
+    p.ws_partials = (size_t)round_up((int64_t)p.splits * M * N * 4, 256);
+    p.ws_counters = (size_t)round_up(groups * 4, 256);
+  }
+  return p;
+}
+
+spl_status run_gemv(const LinearArgs& a, const Plan& p) {
+  if (ceil_div(a.N, WARPS * 2) > 0x7fffffffLL || p.splits > 65535) return SPL_ESHAPE;
+  float* part = nullptr;
+  unsigned int* counters = nullptr;
+  if (p.splits > 1) {
+    part = static_cast<float*>(a.ws);
+    counters = reinterpret_cast<unsigned int*>(static_cast<char*>(a.ws) + p.ws_partials);
+  }
+  switch (padded_m(a.M)) {
+    case 1: return launch<1>(a, p, part, counters);
+    case 2: return launch<2>(a, p, part, counters);
+    case 4: return launch<4>(a, p, part, counters);
+    case 8: return launch<8>(a, p, part, counters);
+    default: return launch<16>(a, p, part, counters);
+  }
+}
+
+}  // namespace spl

@@ -1,0 +1,249 @@
+"""Thin ctypes binding of libspl.so (include/spl.h), same function names.
+
+Only argument marshalling happens here: shapes are read off the tensors,
+pointers and the current CUDA stream are passed through, and a non-OK
+status raises ``SplError``.  Every step of the path runs in the library's
+CUDA kernels; there is no fallback.  The library is loaded on first use and
+its absence is an error.
+"""
+
+import ctypes
+import math
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libspl.so")
+
+SPL_OK, SPL_EINVAL, SPL_ESHAPE, SPL_EALIGN, SPL_ECUDA, SPL_ETIMEOUT, SPL_EUNSUPPORTED, SPL_EWORKSPACE = range(8)
+SPL_MECH_LAPLACE, SPL_MECH_GAUSSIAN = 0, 1
+SPL_PATH_AUTO, SPL_PATH_TF32X3, SPL_PATH_FP32 = 0, 1, 2
+MECHS = {"laplace": SPL_MECH_LAPLACE, "gaussian": SPL_MECH_GAUSSIAN}
+PATHS = {"auto": SPL_PATH_AUTO, "tf32x3": SPL_PATH_TF32X3, "fp32": SPL_PATH_FP32}
+
+
+class SplError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__(f"{where} failed: {status_string(status)} ({status})")
+
+
+class spl_rng(ctypes.Structure):
+    _fields_ = [("seed", ctypes.c_uint64), ("stream_id", ctypes.c_uint64), ("offset", ctypes.c_uint64)]
+
+
+_P = ctypes.c_void_p
+_I64 = ctypes.c_int64
+_D = ctypes.c_double
+_I = ctypes.c_int
+_SZ = ctypes.c_size_t
+_SIGS = {
+    "spl_noise": (_I, [_P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
+    "spl_random_bits": (_I, [_P, _I64, spl_rng, _P]),
+    "spl_mask": (_I, [_P, _P, _P, _I64, _I64, _P]),
+    "spl_noise_mask": (_I, [_P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
+    "spl_split_tf32": (_I, [_P, _P, _P, _I64, _P]),
+    "spl_resolve_path": (_I, [_I64, _I64, _I64, _I]),
+    "spl_linear_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I]),
+    "spl_masked_linear": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_precompute_noise_product": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
+    "spl_masked_linear_unmask": (_I, [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_delta_layernorm": (_D, [_P, _I64]),
+    "spl_delta_attention": (_D, [_P, _I64, _D]),
+    "spl_delta_activation": (_D, [_P, _P, _I64, _I64, _D, _D]),
+    "spl_spectral_norm": (_I, [ctypes.POINTER(ctypes.c_double), _P, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_get_device_status": (_I, [_P]),
+    "spl_launch_count": (ctypes.c_uint64, []),
+    "spl_status_string": (ctypes.c_char_p, [_I]),
+}
+
+_lib = None
+
+
+def lib():
+    """Load libspl.so (once) and declare its signatures."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built; run `python -m paper_2609_15039_gb300.build`")
+        handle = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(handle, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = handle
+    return _lib
+
+
+def status_string(status):
+    return lib().spl_status_string(int(status)).decode()
+
+
+def _check(status, where):
+    if status != SPL_OK:
+        raise SplError(status, where)
+
+
+def _stream(stream):
+    if stream is None:
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _dev(t, name):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != torch.float32 and name != "workspace":
+        raise TypeError(f"{name} must be float32")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _rows_cols(t):
+    if t.dim() == 1:
+        return 1, t.shape[0]
+    return int(math.prod(t.shape[:-1])), int(t.shape[-1])
+
+
+def _mech(mech):
+    return MECHS[mech] if isinstance(mech, str) else int(mech)
+
+
+def _path(path):
+    return PATHS[path] if isinstance(path, str) else int(path)
+
+
+def _eps(eps):
+    return float("inf") if eps is None else float(eps)
+
+
+def spl_noise(N, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None):
+    rows, cols = _rows_cols(N)
+    _check(lib().spl_noise(_dev(N, "N"), rows, cols, float(sensitivity), _eps(eps), _mech(mech),
+                           spl_rng(seed % 2**64, stream_id % 2**64, offset % 2**64), _stream(stream)), "spl_noise")
+
+
+def spl_random_bits(out, seed, stream_id=0, offset=0, stream=None):
+    """Raw Philox words into a CUDA int32/uint32 tensor (bit pattern of the uint32 stream)."""
+    if not out.is_cuda or out.element_size() != 4 or not out.is_contiguous():
+        raise TypeError("out must be a contiguous 4-byte CUDA tensor")
+    _check(lib().spl_random_bits(ctypes.c_void_p(out.data_ptr()), out.numel(),
+                                 spl_rng(seed % 2**64, stream_id % 2**64, offset % 2**64), _stream(stream)),
+           "spl_random_bits")
+
+
+def spl_mask(Xt, X, N, stream=None):
+    rows, cols = _rows_cols(X)
+    _check(lib().spl_mask(_dev(Xt, "Xt"), _dev(X, "X"), _dev(N, "N"), rows, cols, _stream(stream)), "spl_mask")
+
+
+def spl_noise_mask(Xt, N_out, X, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None):
+    rows, cols = _rows_cols(X)
+    _check(lib().spl_noise_mask(_dev(Xt, "Xt"), _dev(N_out, "N_out"), _dev(X, "X"), rows, cols, float(sensitivity),
+                                _eps(eps), _mech(mech), spl_rng(seed % 2**64, stream_id % 2**64, offset % 2**64),
+                                _stream(stream)), "spl_noise_mask")
+
+
+def spl_split_tf32(hi, lo, src, stream=None):
+    _check(lib().spl_split_tf32(_dev(hi, "hi"), _dev(lo, "lo"), _dev(src, "src"), src.numel(), _stream(stream)),
+           "spl_split_tf32")
+
+
+def spl_resolve_path(M, K, N, path="auto"):
+    return lib().spl_resolve_path(M, K, N, _path(path))
+
+
+def spl_linear_workspace_bytes(M, K, N, path="auto"):
+    return int(lib().spl_linear_workspace_bytes(M, K, N, _path(path)))
+
+
+def workspace(nbytes, device=None):
+    """A zero-filled device workspace of at least nbytes (uint8 tensor)."""
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device or "cuda")
+
+
+def _ws(ws):
+    if ws is None:
+        return None, 0
+    return _dev(ws, "workspace"), ws.numel() * ws.element_size()
+
+
+def _linear(fn, name, out, a, W, W_hi, W_lo, C, path, ws, stream):
+    M, K = _rows_cols(a)
+    N = W.shape[0]
+    if W.shape[-1] != K or out.numel() != M * N or (C is not None and C.numel() != M * N):
+        raise ValueError(f"{name}: shape mismatch")
+    wsp, wsb = _ws(ws)
+    args = [_dev(out, "out"), _dev(a, "input"), _dev(W, "W"), _dev(W_hi, "W_hi"), _dev(W_lo, "W_lo")]
+    if C is not None or name == "spl_masked_linear_unmask":
+        args.append(_dev(C, "C"))
+    _check(fn(*args, M, K, N, _path(path), wsp, wsb, _stream(stream)), name)
+
+
+def spl_masked_linear(Yt, Xt, W, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
+    _linear(lib().spl_masked_linear, "spl_masked_linear", Yt, Xt, W, W_hi, W_lo, None, path, workspace, stream)
+
+
+def spl_precompute_noise_product(C, Nz, W, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
+    _linear(lib().spl_precompute_noise_product, "spl_precompute_noise_product", C, Nz, W, W_hi, W_lo, None, path,
+            workspace, stream)
+
+
+def spl_unmask(Y, Yt, C, stream=None):
+    rows, cols = _rows_cols(Yt)
+    _check(lib().spl_unmask(_dev(Y, "Y"), _dev(Yt, "Yt"), _dev(C, "C"), rows, cols, _stream(stream)), "spl_unmask")
+
+
+def spl_masked_linear_unmask(Y, Xt, W, C, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
+    _linear(lib().spl_masked_linear_unmask, "spl_masked_linear_unmask", Y, Xt, W, W_hi, W_lo, C, path, workspace,
+            stream)
+
+
+def _host_f32(t):
+    t = torch.as_tensor(t, dtype=torch.float32).contiguous().cpu()
+    return t, ctypes.c_void_p(t.data_ptr())
+
+
+def spl_delta_layernorm(alpha):
+    a, p = _host_f32(alpha)
+    return lib().spl_delta_layernorm(p, a.numel())
+
+
+def spl_delta_attention(alpha, wval_spectral_norm):
+    a, p = _host_f32(alpha)
+    return lib().spl_delta_attention(p, a.numel(), float(wval_spectral_norm))
+
+
+def spl_delta_activation(alpha, beta, d_ff, wup_spectral_norm, wgate_spectral_norm):
+    a, pa = _host_f32(alpha)
+    if beta is None:
+        pb = None
+    else:
+        b, pb = _host_f32(beta)
+    return lib().spl_delta_activation(pa, pb, a.numel(), int(d_ff), float(wup_spectral_norm),
+                                      float(wgate_spectral_norm))
+
+
+def spl_spectral_norm(W, iters=100, workspace=None, stream=None):
+    N, K = W.shape
+    ws = workspace if workspace is not None else globals()["workspace"](4 * (N + 2 * K) + 256, W.device)
+    wsp, wsb = _ws(ws)
+    out = ctypes.c_double(0.0)
+    _check(lib().spl_spectral_norm(ctypes.byref(out), _dev(W, "W"), N, K, int(iters), wsp, wsb, _stream(stream)),
+           "spl_spectral_norm")
+    return out.value
+
+
+def spl_launch_count():
+    return int(lib().spl_launch_count())
+
+
+def spl_get_device_status(stream=None):
+    return lib().spl_get_device_status(_stream(stream))

@@ -1,0 +1,111 @@
+"""The C-ABI library on the CPU: it loads without a GPU, exports every entry
+point include/spl.h declares, and its host-only logic agrees with the oracle.
+No kernel is launched here."""
+
+import ctypes
+import math
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import sensitivity as osens
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def spl():
+    from paper_2609_15039_gb300 import build, spl as binding
+    if not os.path.exists(binding.LIB_PATH):
+        build.build()
+    binding.lib()
+    return binding
+
+
+def declared_functions():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names += re.findall(r"^\s*(?:const\s+)?\w+\*?\s+\*?(spl_\w+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("spl_noise", "spl_mask", "spl_masked_linear", "spl_precompute_noise_product", "spl_unmask",
+                     "spl_noise_mask", "spl_masked_linear_unmask", "spl_random_bits"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(spl):
+    handle = ctypes.CDLL(spl.LIB_PATH)
+    missing = [n for n in declared_functions() if not hasattr(handle, n)]
+    assert not missing, missing
+    # the binding declares a signature for every exported entry point
+    assert set(declared_functions()) <= set(spl._SIGS)
+
+
+def test_status_strings(spl):
+    assert spl.status_string(0) == "SPL_OK"
+    assert spl.status_string(7) == "SPL_EWORKSPACE"
+    assert spl.status_string(99) == "SPL_UNKNOWN"
+
+
+def test_argument_validation_without_launch(spl):
+    L = spl.lib()
+    rng = spl.spl_rng(0, 0, 0)
+    # eps <= 0, NaN; negative sensitivity; bad mechanism -> EINVAL before any CUDA call
+    for eps in (0.0, -1.0, float("nan")):
+        assert L.spl_noise(None, 4, 4, 1.0, eps, 0, rng, None) == spl.SPL_EINVAL
+    assert L.spl_noise(None, 4, 4, -1.0, 1.0, 0, rng, None) == spl.SPL_EINVAL
+    assert L.spl_noise(None, 4, 4, float("inf"), 1.0, 0, rng, None) == spl.SPL_EINVAL
+    assert L.spl_noise(None, 4, 4, 1.0, 1.0, 7, rng, None) == spl.SPL_EINVAL
+    assert L.spl_noise(None, 4, 4, 1.0, 1.0, 0, rng, None) == spl.SPL_EINVAL  # NULL output
+    # zero-sized problems are no-ops
+    assert L.spl_noise(None, 0, 5, 1.0, 1.0, 0, rng, None) == spl.SPL_OK
+    assert L.spl_mask(None, None, None, 3, 0, None) == spl.SPL_OK
+    assert L.spl_unmask(None, None, None, 0, 0, None) == spl.SPL_OK
+    assert L.spl_masked_linear(None, None, None, None, None, 0, 8, 8, 0, None, 0, None) == spl.SPL_OK
+    # negative sizes, bad path, NULL operands, K % 4
+    assert L.spl_masked_linear(None, None, None, None, None, -1, 8, 8, 0, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_masked_linear(None, None, None, None, None, 4, 8, 8, 9, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_masked_linear(None, None, None, None, None, 4, 8, 8, 0, None, 0, None) == spl.SPL_EINVAL
+    buf = (ctypes.c_float * 64)()
+    p = ctypes.cast(buf, ctypes.c_void_p).value
+    base = p + (16 - p % 16) % 16
+    assert L.spl_masked_linear(base, base, base, None, None, 2, 6, 2, 2, None, 0, None) == spl.SPL_EALIGN
+    assert L.spl_masked_linear(base + 4, base, base, None, None, 2, 8, 2, 2, None, 0, None) == spl.SPL_EALIGN
+    assert L.spl_masked_linear_unmask(base, base, base, None, None, None, 2, 8, 2, 2, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_random_bits(None, -1, rng, None) == spl.SPL_EINVAL
+    assert L.spl_split_tf32(base + 4, base, base, 4, None) == spl.SPL_EALIGN
+
+
+def test_workspace_sizes_are_consistent(spl):
+    # decode shapes: split-K partials + counters; prefill TF32X3 adds the A split
+    for M, K, N in [(1, 3072, 3072), (16, 8192, 3072), (128, 3072, 1024), (2048, 2560, 9728)]:
+        auto = spl.spl_linear_workspace_bytes(M, K, N, "auto")
+        assert auto >= spl.spl_linear_workspace_bytes(M, K, N, "fp32")
+        assert auto >= spl.spl_linear_workspace_bytes(M, K, N, "tf32x3")
+        assert spl.spl_linear_workspace_bytes(M, K, N, "tf32x3") >= 2 * M * K * 4
+    assert spl.spl_linear_workspace_bytes(0, 8, 8) == 0
+
+
+def test_sensitivities_match_oracle(spl):
+    rng = np.random.default_rng(0)
+    for d, d_ff in ((256, 512), (3072, 8192)):
+        alpha = rng.standard_normal(d).astype(np.float32)
+        beta = rng.standard_normal(d).astype(np.float32) * 0.1
+        assert spl.spl_delta_layernorm(alpha) == pytest.approx(osens.delta_layernorm(alpha), rel=1e-12)
+        assert spl.spl_delta_attention(alpha, 1.7) == pytest.approx(osens.delta_attention(alpha, 1.7), rel=1e-12)
+        got = spl.spl_delta_activation(alpha, beta, d_ff, 2.9, 3.1)
+        assert got == pytest.approx(osens.delta_activation(alpha, beta, d_ff, 2.9, 3.1), rel=1e-12)
+        assert spl.spl_delta_activation(alpha, None, d_ff, 2.0, 2.0) == pytest.approx(
+            osens.delta_activation(alpha, None, d_ff, 2.0, 2.0), rel=1e-12)
+    ones = np.ones(3072, dtype=np.float32)
+    assert spl.spl_delta_layernorm(ones) == pytest.approx(2 * 3072 ** 0.75, rel=1e-12)
+    assert spl.lib().spl_delta_layernorm(None, 4) < 0
+    assert math.isfinite(spl.spl_delta_layernorm(ones))
