@@ -40,6 +40,7 @@ def parse():
     ap.add_argument("--tokens", type=int, default=128)
     ap.add_argument("--cpu-sample-rows", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
 
 
@@ -234,11 +235,13 @@ def main():
     t_end = torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clocks:
         torch.cuda.synchronize()
+        torch.cuda.nvtx.range_push("timed")
         t_start.record(stream)
         for i in range(args.steps):
             step(args.warmup + i, use_timer=True)
         t_end.record(stream)
         torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
     if world > 1:
         dist.barrier()
     gpu_launches = spl.spl_launch_count() - launches0
@@ -276,37 +279,38 @@ def main():
                 "share_of_step": prod_ms / (ms * args.steps), "peak_source": pk["source"], "peak_note": peak_note,
                 "flops_per_call_avg": flops_call}
 
-    # e2e: inputs from pinned host memory each step, outputs read back
-    host_in = {g: x.cpu().pin_memory() for g, x in inputs.items()}
-    host_out = {name: torch.empty(o.shape, dtype=o.dtype).pin_memory() for name, o in outputs.items()}
-    dev_in = {g: torch.empty_like(x) for g, x in inputs.items()}
-    h2d = sum(x.numel() * 4 for x in host_in.values())
-    d2h = sum(o.numel() * 4 for o in host_out.values())
+    e2e = None
+    if not args.no_e2e:
+        host_in = {g: x.cpu().pin_memory() for g, x in inputs.items()}
+        host_out = {name: torch.empty(o.shape, dtype=o.dtype).pin_memory() for name, o in outputs.items()}
+        dev_in = {g: torch.empty_like(x) for g, x in inputs.items()}
+        h2d = sum(x.numel() * 4 for x in host_in.values())
+        d2h = sum(o.numel() * 4 for o in host_out.values())
 
-    def e2e_step(i):
-        for g in dev_in:
-            dev_in[g].copy_(host_in[g], non_blocking=True)
-        layer.step(dev_in, args.eps, mech, 50_000 + i, outputs=outputs, scratch=scratch, path=args.path)
-        for name in host_out:
-            host_out[name].copy_(outputs[name], non_blocking=True)
+        def e2e_step(i):
+            for g in dev_in:
+                dev_in[g].copy_(host_in[g], non_blocking=True)
+            layer.step(dev_in, args.eps, mech, 50_000 + i, outputs=outputs, scratch=scratch, path=args.path)
+            for name in host_out:
+                host_out[name].copy_(outputs[name], non_blocking=True)
 
-    for i in range(2):
-        e2e_step(i)
-    torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for i in range(args.steps):
-        e2e_step(10 + i)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e = {"value": world * flops_step / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
-           "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+        for i in range(2):
+            e2e_step(i)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            e2e_step(10 + i)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1) / args.steps
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": world * flops_step / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
 
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -319,8 +323,9 @@ def main():
         "roofline": roofline,
         "gpu_launches": gpu_launches,
         "clocks": clocks.summary(),
-        "e2e": e2e,
     }
+    if e2e is not None:
+        result["e2e"] = e2e
 
     # cpu baseline + oracle match on the first rows (rank 0, N = 1 only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -42,9 +42,10 @@ spl_status run_linear(float* out, const float* a, const float* W, const float* W
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
   if (path != SPL_PATH_AUTO && path != SPL_PATH_TF32X3 && path != SPL_PATH_FP32) return SPL_EINVAL;
   if (M == 0 || N == 0) return SPL_OK;
-  if (!out || !a || !W || (need_c && !C)) return SPL_EINVAL;
+  if (!out || (need_c && !C)) return SPL_EINVAL;
   if ((K & 3) != 0) return SPL_EALIGN;
-  if (!aligned16(out) || !aligned16(a) || !aligned16(W) || (C && !aligned16(C))) return SPL_EALIGN;
+  if (K > 0 && (!a || !W)) return SPL_EINVAL;
+  if (!aligned16(out) || (a && !aligned16(a)) || (W && !aligned16(W)) || (C && !aligned16(C))) return SPL_EALIGN;
   if ((W_hi && !aligned16(W_hi)) || (W_lo && !aligned16(W_lo))) return SPL_EALIGN;
   if (M > (int64_t(1) << 31) || N > (int64_t(1) << 31) || K > (int64_t(1) << 31)) return SPL_ESHAPE;
   if (K == 0) {  // empty reduction: the product is zero

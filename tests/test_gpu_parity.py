@@ -145,7 +145,8 @@ def test_noise_mask_fused(spl, mech, shape):
 
 def test_split_tf32_properties(spl):
     W = wl.weight(257, 1028, seed=5).numpy()
-    W[0, :4] = [0.0, -0.0, 1.0 + 2.0 ** -12, -(1.0 + 3 * 2.0 ** -12)]
+    # ties: 1 + 2^-11 sits halfway between 1 and 1 + 2^-10 (TF32 ulp at 1)
+    W[0, :4] = [0.0, -0.0, 1.0 + 2.0 ** -11, -(1.0 + 3 * 2.0 ** -11)]
     hi = torch.empty_like(dev(W))
     lo = torch.empty_like(hi)
     spl.spl_split_tf32(hi, lo, dev(W))
@@ -280,7 +281,8 @@ def llama_layer(spl):
     weights = {name: wl.weight(N, K, seed=200 + pi) for pi, (name, K, N, g) in enumerate(model.projections())}
     layer = MaskedLayer.from_weights(model, weights)
     ones = np.ones(model.d_model)
-    norms = {n: osens.spectral_norm(weights[n].numpy(), iters=60) for n in ("v", "up", "gate")}
+    # ||W||_2 from LAPACK's singular values (a library routine), exact to rounding
+    norms = {n: float(np.linalg.svd(weights[n].double().numpy(), compute_uv=False)[0]) for n in ("v", "up", "gate")}
     deltas = {  # noise scales from the oracle: an input both sides get
         "qkv": osens.delta_layernorm(ones),
         "gateup": osens.delta_layernorm(ones),
@@ -292,9 +294,12 @@ def llama_layer(spl):
 
 def test_layer_sensitivities_match_oracle(llama_layer):
     layer, _weights_, deltas, norms = llama_layer
-    got = layer.sensitivities(power_iters=100)
+    # power iteration approaches ||W||_2 from below; 400 steps bring it within 0.3% on these
+    # Gaussian matrices, whose top singular values are close together
+    got = layer.sensitivities(power_iters=400)
     for g in deltas:
-        assert got[g] == pytest.approx(deltas[g], rel=2e-3), g
+        assert got[g] <= deltas[g] * (1 + 1e-5), g
+        assert got[g] == pytest.approx(deltas[g], rel=3e-3), g
     assert got["qkv"] == pytest.approx(2 * 3072 ** 0.75, rel=1e-9)
 
 
