@@ -115,11 +115,12 @@ spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path);
 
 /* Bytes of device workspace the three product calls below need for this
  * problem on the current device (0 if none; for AUTO the larger of the two
- * paths).  It holds split-K partial sums, the arrival counters of the decode
- * kernel and, for TF32X3, the TF32 split of the left operand.  It must be
- * zero-filled before its first use; every call that returns SPL_OK leaves
- * the counters at zero again.  One workspace must not be used by calls that
- * can run concurrently. */
+ * paths).  Layout: the first 64 KiB hold the decode kernel's arrival
+ * counters, then split-K partial sums and, for TF32X3, the TF32 split of the
+ * left operand.  It must be zero-filled before its first use; every call that
+ * returns SPL_OK leaves the counters at zero again, so one workspace (sized
+ * for the largest call) serves calls of any shape and path.  Calls that can
+ * run concurrently must not share a workspace. */
 size_t spl_linear_workspace_bytes(int64_t M, int64_t K, int64_t N, spl_path path);
 
 /* ---- a5: masked product -----------------------------------------------

@@ -49,15 +49,21 @@ struct LinearArgs {
   cudaStream_t stream;
 };
 
+// Workspace layout shared by every product call: the first kCounterBytes hold
+// the decode kernel's arrival counters (zero between calls); split-K partials
+// and the TF32 split of the left operand follow.  Keeping the counters at a
+// fixed place lets one workspace serve calls of any shape and path.
+constexpr size_t kCounterBytes = 64 * 1024;
+constexpr int64_t kMaxCounters = (int64_t)(kCounterBytes / sizeof(unsigned int));
+
 // Split-K plans: how many K-splits each kernel uses and the workspace it needs.
 struct Plan {
   int kernel;            // 0 = GEMV (decode), 1 = FP32 SIMT GEMM, 2 = TF32X3 tcgen05 GEMM
   int splits;            // K-splits (1 = none)
   int64_t k_per_split;   // multiple of the kernel's K granule
-  size_t ws_partials;    // bytes of split partials
-  size_t ws_counters;    // bytes of arrival counters (GEMV)
-  size_t ws_asplit;      // bytes of the A operand's hi/lo split (TF32X3)
-  size_t total() const { return ws_partials + ws_counters + ws_asplit; }
+  size_t ws_partials;    // bytes of split partials (at offset kCounterBytes)
+  size_t ws_asplit;      // bytes of the A operand's hi/lo split (TF32X3, after the partials)
+  size_t total() const { return (ws_partials + ws_asplit) ? kCounterBytes + ws_partials + ws_asplit : 0; }
 };
 
 constexpr int kGemvMaxM = 16;

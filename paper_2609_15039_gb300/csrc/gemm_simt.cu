@@ -184,7 +184,7 @@ spl_status run_simt(const LinearArgs& a, const Plan& p) {
     simt_gemm_kernel<<<grid, THREADS, 0, a.stream>>>(a.out, a.a, a.w, a.c, a.M, a.K, a.N, p.k_per_split, 1);
     return launch_status();
   }
-  float* part = static_cast<float*>(a.ws);
+  float* part = reinterpret_cast<float*>(static_cast<char*>(a.ws) + kCounterBytes);
   simt_gemm_kernel<<<grid, THREADS, 0, a.stream>>>(part, a.a, a.w, nullptr, a.M, a.K, a.N, p.k_per_split,
                                                    p.splits);
   spl_status st = launch_status();

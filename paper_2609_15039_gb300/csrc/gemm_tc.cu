@@ -397,7 +397,7 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
   if (ceil_div(a.M, BM) > 65535 || p.splits > 65535) return SPL_ESHAPE;
 
   // A operand split into the workspace: [hi | lo], each M*K fp32
-  char* ws = static_cast<char*>(a.ws);
+  char* ws = static_cast<char*>(a.ws) + kCounterBytes;
   float* part = reinterpret_cast<float*>(ws);
   float* a_hi = reinterpret_cast<float*>(ws + p.ws_partials);
   float* a_lo = reinterpret_cast<float*>(ws + p.ws_partials + p.ws_asplit / 2);

@@ -177,20 +177,18 @@ Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
   ks = std::min<int64_t>(ks, ks_max);
   p.k_per_split = ks;
   p.splits = (int)ceil_div(K, ks);
-  if (p.splits > 1) {
-    p.ws_partials = (size_t)round_up((int64_t)p.splits * M * N * 4, 256);
-    p.ws_counters = (size_t)round_up(groups * 4, 256);
-  }
+  if (p.splits > 1) p.ws_partials = (size_t)round_up((int64_t)p.splits * M * N * 4, 256);
   return p;
 }
 
 spl_status run_gemv(const LinearArgs& a, const Plan& p) {
-  if (ceil_div(a.N, WARPS * 2) > 0x7fffffffLL || p.splits > 65535) return SPL_ESHAPE;
+  if (p.splits > 65535) return SPL_ESHAPE;
   float* part = nullptr;
   unsigned int* counters = nullptr;
   if (p.splits > 1) {
-    part = static_cast<float*>(a.ws);
-    counters = reinterpret_cast<unsigned int*>(static_cast<char*>(a.ws) + p.ws_partials);
+    if (ceil_div(a.N, WARPS * rows_per_warp(padded_m(a.M))) > kMaxCounters) return SPL_ESHAPE;
+    counters = static_cast<unsigned int*>(a.ws);
+    part = reinterpret_cast<float*>(static_cast<char*>(a.ws) + kCounterBytes);
   }
   switch (padded_m(a.M)) {
     case 1: return launch<1>(a, p, part, counters);

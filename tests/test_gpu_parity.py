@@ -193,6 +193,23 @@ def test_products_match_oracle(spl, M, K, N, path):
     assert spl.spl_get_device_status() == 0
 
 
+def test_one_workspace_serves_every_shape_and_path(spl):
+    """Decode counters sit at a fixed place, so partials of other calls never land on them."""
+    cases = [(130, 1028, 600, "tf32x3"), (1, 3072, 3072, "fp32"), (17, 260, 300, "fp32"), (4, 8192, 1024, "fp32"),
+             (1, 3072, 3072, "fp32"), (300, 64, 257, "fp32"), (16, 2560, 3000, "fp32")]
+    need = max(spl.spl_linear_workspace_bytes(M, K, N, path) for M, K, N, path in cases)
+    ws = spl.workspace(need)
+    for i, (M, K, N, path) in enumerate(cases):
+        W, Wd, hi, lo = _weights(spl, N, K, seed=50 + i)
+        A = (wl.activations(M, K, seed=60 + i).numpy() * 300).astype(np.float32)
+        C = wl.activations(M, N, seed=70 + i).numpy()
+        Y = torch.empty((M, N), device="cuda")
+        spl.spl_masked_linear_unmask(Y, dev(A), Wd, dev(C), hi, lo, path=path, workspace=ws)
+        assert_product_close(f32(Y), A, W, path, C=C, what=f"case {i}")
+    # the counter region is back to zero after every call
+    assert torch.count_nonzero(ws[: 64 * 1024]).item() == 0
+
+
 def test_workspace_errors(spl):
     M, K, N = 4, 3072, 3072
     W, Wd, hi, lo = _weights(spl, N, K, seed=1)
