@@ -159,6 +159,31 @@ spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const float* W, c
                                     int64_t N, spl_path path, void* workspace,
                                     size_t workspace_bytes, cudaStream_t stream);
 
+/* ---- a5 + a6 for decode, without allocation ---------------------------
+ * The paper has no counterpart to this call; it exists for callers that
+ * cannot allocate device memory at the time of the product: a decode loop
+ * that must not stall on cudaMalloc/cudaFree (both synchronise the device),
+ * a process whose device memory is already fully reserved by another
+ * allocator, or a worker whose memory budget is fixed at start-up.
+ * Same result as spl_masked_linear_unmask on the FP32 decode kernel
+ * (Y = fl32(fl32(Xt W^T) - C), 1 <= M <= 16), but the kernel's scratch
+ * (arrival counters and split-K partials) is a fixed array inside the
+ * library: 64 KiB of counters plus 4 MiB of partials, which every GPU that
+ * loads the library holds until the process exits.  Nothing is allocated:
+ * no cudaMalloc, cudaFree or allocating library routine is called.
+ *  - The first call on a device (with that device current) looks up the
+ *    array's device address and clears its counters; make that first call
+ *    before any stream capture.
+ *  - All calls share the one array, which keeps the last call's contents;
+ *    each successful call leaves the counters at zero.  Calls that overlap on
+ *    the GPU (on different streams or threads) race on it: serialise them.
+ * Errors: EINVAL for NULL operands or negative sizes, ESHAPE for M > 16,
+ * EALIGN as for the other calls, EWORKSPACE when the problem needs more
+ * split-K partial storage than the built-in 4 MiB (splits x M x N x 4 bytes)
+ * or more than 16384 row groups. */
+spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt, const float* W, const float* C,
+                                            int64_t M, int64_t K, int64_t N, cudaStream_t stream);
+
 /* ---- a1: noise scale ----------------------------------------------------
  * Global l2 sensitivities (Sec. 4.3), evaluated in fp64 on the host from
  * HOST arrays.  Return a negative value on invalid input.

@@ -17,6 +17,7 @@
 // subtracts C, writes the result and resets the counter to zero.
 
 #include <algorithm>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -200,3 +201,66 @@ spl_status run_gemv(const LinearArgs& a, const Plan& p) {
 }
 
 }  // namespace spl
+
+// ---- variant without allocation ---------------------------------------------
+// Some callers cannot call cudaMalloc when they need this product: a decode
+// loop that must not stall (cudaMalloc and cudaFree synchronise the device),
+// a process whose device memory is already fully reserved by another
+// allocator, or a worker whose memory budget is fixed when it starts.  For
+// them the decode kernel's scratch (arrival counters + split-K partials, the
+// same layout as a workspace) lives in this fixed array instead.  Every GPU
+// that loads the library holds it until the process exits.
+namespace spl {
+namespace {
+
+constexpr size_t kStaticPartialBytes = size_t(4) << 20;  // 4 MiB of split-K partials
+constexpr size_t kStaticScratchBytes = kCounterBytes + kStaticPartialBytes;
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDev = 64;
+std::mutex g_static_mu;
+void* g_static_ptr[kMaxDev] = {nullptr};
+
+// Device address of g_static_scratch on the current device.  The first call on
+// a device looks it up (cudaGetSymbolAddress, with that device current) and
+// clears the counter region; later calls reuse the cached address.
+spl_status static_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return SPL_ECUDA;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) return SPL_ECUDA;
+    if (cudaMemset(p, 0, kCounterBytes) != cudaSuccess) return SPL_ECUDA;
+    g_static_ptr[dev] = p;
+  }
+  *out = g_static_ptr[dev];
+  return SPL_OK;
+}
+
+}  // namespace
+}  // namespace spl
+
+extern "C" spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt, const float* W, const float* C,
+                                                       int64_t M, int64_t K, int64_t N, cudaStream_t stream) {
+  using namespace spl;
+  if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
+  if (M == 0 || N == 0) return SPL_OK;
+  if (M > kGemvMaxM) return SPL_ESHAPE;
+  if (!Y || !C || (K > 0 && (!Xt || !W))) return SPL_EINVAL;
+  if ((K & 3) != 0) return SPL_EALIGN;
+  if (!aligned16(Y) || !aligned16(C) || (Xt && !aligned16(Xt)) || (W && !aligned16(W))) return SPL_EALIGN;
+  if (K > (int64_t(1) << 31) || N > (int64_t(1) << 31)) return SPL_ESHAPE;
+  if (K == 0) {
+    if (cudaMemsetAsync(Y, 0, (size_t)(M * N) * sizeof(float), stream) != cudaSuccess) return SPL_ECUDA;
+    return spl_unmask(Y, Y, C, M, N, stream);
+  }
+  const Plan plan = plan_gemv(M, K, N, device_sm_count());
+  if (plan.ws_partials > kStaticPartialBytes) return SPL_EWORKSPACE;  // beyond the built-in 4 MiB
+  if (plan.splits > 1 && ceil_div(N, WARPS * rows_per_warp(padded_m(M))) > kMaxCounters) return SPL_EWORKSPACE;
+  void* ws = nullptr;
+  spl_status st = static_scratch(&ws);
+  if (st != SPL_OK) return st;
+  LinearArgs args{Y, Xt, W, nullptr, nullptr, C, M, K, N, ws, kStaticScratchBytes, stream};
+  return run_gemv(args, plan);
+}

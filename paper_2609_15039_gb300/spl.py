@@ -50,6 +50,7 @@ _SIGS = {
     "spl_precompute_noise_product": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_masked_linear_unmask": (_I, [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_masked_linear_unmask_noalloc": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P]),
     "spl_delta_layernorm": (_D, [_P, _I64]),
     "spl_delta_attention": (_D, [_P, _I64, _D]),
     "spl_delta_activation": (_D, [_P, _P, _I64, _I64, _D, _D]),
@@ -204,6 +205,16 @@ def spl_unmask(Y, Yt, C, stream=None):
 def spl_masked_linear_unmask(Y, Xt, W, C, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
     _linear(lib().spl_masked_linear_unmask, "spl_masked_linear_unmask", Y, Xt, W, W_hi, W_lo, C, path, workspace,
             stream)
+
+
+def spl_masked_linear_unmask_noalloc(Y, Xt, W, C, stream=None):
+    """Decode product + unmask (M <= 16) using the library's built-in scratch array."""
+    M, K = _rows_cols(Xt)
+    N = W.shape[0]
+    if W.shape[-1] != K or Y.numel() != M * N or C.numel() != M * N:
+        raise ValueError("spl_masked_linear_unmask_noalloc: shape mismatch")
+    _check(lib().spl_masked_linear_unmask_noalloc(_dev(Y, "Y"), _dev(Xt, "Xt"), _dev(W, "W"), _dev(C, "C"), M, K,
+                                                  N, _stream(stream)), "spl_masked_linear_unmask_noalloc")
 
 
 def _host_f32(t):
