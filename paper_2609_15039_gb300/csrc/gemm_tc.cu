@@ -53,7 +53,7 @@ constexpr int UMMA_K = 8;                                      // K of one kind:
 constexpr uint32_t A_TILE_BYTES = BM * BK * 4;                 // 8 KB
 constexpr uint32_t B_TILE_BYTES = BN * BK * 4;                 // 16 KB
 constexpr uint32_t STAGE_BYTES = 2 * A_TILE_BYTES + 2 * B_TILE_BYTES;  // 48 KB
-constexpr uint32_t BAR_OFFSET = STAGES * STAGE_BYTES;          // barriers after the ring
+constexpr uint32_t BAR_OFFSET = STAGES * STAGE_BYTES;          // barriers after the ring (3S+1 of them)
 constexpr uint32_t SMEM_BYTES = BAR_OFFSET + 256 + 1024;       // + barriers + alignment slack
 constexpr uint32_t TMEM_COLS = 256;
 constexpr unsigned long long kWaitNs = 1000000000ull;          // 1 s per wait
@@ -86,6 +86,11 @@ __device__ __forceinline__ uint64_t make_sdesc_sw64(uint32_t saddr) {
 }
 
 // ---- PTX wrappers ----------------------------------------------------------
+__device__ __forceinline__ float tf32_rna(float v) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(v));
+  return __uint_as_float(r);
+}
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -177,33 +182,69 @@ __device__ __forceinline__ void tmem_ld_32x32(uint32_t taddr, float (&v)[32]) {
 }
 
 struct TcMaps {
-  CUtensorMap a_hi, a_lo, w_hi, w_lo;
+  CUtensorMap a, w_hi, w_lo;
 };
 
+constexpr int MAX_CLUSTER = 8;        // split-K CTAs of one output tile (portable cluster size)
+constexpr int RED_STRIDE = BN + 4;    // floats per row of the staged accumulator (pads bank conflicts)
+static_assert((size_t)BM * RED_STRIDE * 4 <= (size_t)STAGES * STAGE_BYTES, "staging fits in the stage ring");
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// One CTA computes a 128 x 256 tile of out over the K range of its split.
+// The `splits` CTAs of a tile form one thread-block cluster (z dimension);
+// their fp32 partial tiles are summed through distributed shared memory in
+// cluster-rank order, so the result does not depend on timing.
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
                int64_t M, int64_t K, int64_t N, int64_t k_per_split, int splits) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + BAR_OFFSET);  // full[S], empty[S], accum
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + BAR_OFFSET + 8 * (2 * STAGES + 1));
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + BAR_OFFSET + 8 * (2 * STAGES + 1) + 8);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + BAR_OFFSET);  // full[S], conv[S], empty[S], accum
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + BAR_OFFSET + 8 * (3 * STAGES + 1));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + BAR_OFFSET + 8 * (3 * STAGES + 1) + 8);
+  float* red = reinterpret_cast<float*>(smem);  // [BM][RED_STRIDE] staged accumulator, after the mainloop
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t m0 = (int64_t)blockIdx.y * BM, n0 = (int64_t)blockIdx.x * BN;
   const int split = blockIdx.z;
   const int64_t kbeg = (int64_t)split * k_per_split;
   const int64_t kend = std::min<int64_t>(K, kbeg + k_per_split);
-  const int nk = (int)ceil_div(kend - kbeg, BK);
+  const int nk = kend > kbeg ? (int)ceil_div(kend - kbeg, BK) : 0;
 
   const uint32_t bar_base = smem_u32(bars);
   auto full_bar = [&](int s) { return bar_base + 8u * s; };
-  auto empty_bar = [&](int s) { return bar_base + 8u * (STAGES + s); };
-  const uint32_t accum_bar = bar_base + 8u * (2 * STAGES);
+  auto conv_bar = [&](int s) { return bar_base + 8u * (STAGES + s); };
+  auto empty_bar = [&](int s) { return bar_base + 8u * (2 * STAGES + s); };
+  const uint32_t accum_bar = bar_base + 8u * (3 * STAGES);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full_bar(s), 1);
+      mbar_init(conv_bar(s), 4);  // one arrival per converter warp
       mbar_init(empty_bar(s), 1);
     }
     mbar_init(accum_bar, 1);
@@ -217,47 +258,47 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
+  // Every role loop is run by whole warps (lane 0 issues, all lanes wait), so no warp is
+  // ever diverged when it reaches a block- or cluster-wide barrier.
   if (warp == 0) {
-    if (lane == 0) {
-      // ---------------- TMA producer ----------------
-      uint32_t issued_mask = 0u, phase_mask = 0u;  // per stage: a load was issued / its parity
-      bool ok = true;
-      for (int kb = 0; kb < nk && ok; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-        if (!mbar_wait(empty_bar(s), ph ^ 1u, kWaitNs, abort_flag)) {
-          ok = false;
-          break;
-        }
+    // ---------------- TMA producer: raw A (into the A_hi slot), W_hi, W_lo ----------------
+    uint32_t issued_mask = 0u, phase_mask = 0u;  // per stage: a load was issued / its parity
+    bool ok = true;
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % STAGES;
+      const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+      ok = __all_sync(0xffffffffu, mbar_wait(empty_bar(s), ph ^ 1u, kWaitNs, abort_flag));
+      if (!ok) break;
+      if (lane == 0) {
         const uint32_t st = smem_u32(smem + (size_t)s * STAGE_BYTES);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
-        mbar_expect_tx(full_bar(s), STAGE_BYTES);
-        tma_load_2d(st, &maps.a_hi, full_bar(s), kx, (int)m0);
-        tma_load_2d(st + A_TILE_BYTES, &maps.a_lo, full_bar(s), kx, (int)m0);
+        mbar_expect_tx(full_bar(s), A_TILE_BYTES + 2 * B_TILE_BYTES);
+        tma_load_2d(st, &maps.a, full_bar(s), kx, (int)m0);
         tma_load_2d(st + 2 * A_TILE_BYTES, &maps.w_hi, full_bar(s), kx, (int)n0);
         tma_load_2d(st + 2 * A_TILE_BYTES + B_TILE_BYTES, &maps.w_lo, full_bar(s), kx, (int)n0);
-        issued_mask |= 1u << s;
-        phase_mask = (phase_mask & ~(1u << s)) | (ph << s);
       }
-      if (!ok) {
+      __syncwarp();
+      issued_mask |= 1u << s;
+      phase_mask = (phase_mask & ~(1u << s)) | (ph << s);
+    }
+    if (!ok) {
+      if (lane == 0) {
         *abort_flag = 1;
         atomicOr(&g_device_status, kStatusTimeout);
-        // let copies already issued land before the CTA exits
-        for (int s = 0; s < STAGES; ++s)
-          if (issued_mask & (1u << s)) mbar_wait(full_bar(s), (phase_mask >> s) & 1u, kDrainNs, nullptr);
       }
+      // let copies already issued land before the CTA exits
+      for (int s = 0; s < STAGES; ++s)
+        if (issued_mask & (1u << s)) mbar_wait(full_bar(s), (phase_mask >> s) & 1u, kDrainNs, nullptr);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------- MMA issuer ----------------
-      bool ok = true;
-      for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-        if (!mbar_wait(full_bar(s), ph, kWaitNs, abort_flag)) {
-          ok = false;
-          break;
-        }
+    // ---------------- MMA issuer ----------------
+    bool ok = true;
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % STAGES;
+      const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+      ok = __all_sync(0xffffffffu, mbar_wait(conv_bar(s), ph, kWaitNs, abort_flag));
+      if (!ok) break;
+      if (lane == 0) {
         tc_fence_after();
         const uint32_t st = smem_u32(smem + (size_t)s * STAGE_BYTES);
         const uint32_t a_hi = st, a_lo = st + A_TILE_BYTES;
@@ -272,26 +313,55 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
         }
         mma_commit(empty_bar(s));  // stage reusable once these MMAs have read it
       }
-      if (ok) {
-        mma_commit(accum_bar);
-      } else {
+      __syncwarp();
+    }
+    if (lane == 0) {
+      if (!ok) {
         *abort_flag = 1;
         atomicOr(&g_device_status, kStatusTimeout);
-        // MMAs already issued must finish before TMEM is released
-        mma_commit(accum_bar);
-        mbar_wait(accum_bar, 0u, kDrainNs, nullptr);
       }
+      mma_commit(accum_bar);  // MMAs already issued must finish before TMEM is read or released
     }
+    __syncwarp();
+    if (!ok) mbar_wait(accum_bar, 0u, kDrainNs, nullptr);
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
+    // ---------------- warps 2..5: split A during the mainloop, then the epilogue ----------------
+    const int t = threadIdx.x - 64;  // 0..127
+    bool ok = true;
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % STAGES;
+      const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+      ok = mbar_wait(full_bar(s), ph, kWaitNs, abort_flag);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      // The raw tile (8 KB, swizzled) sits in the hi slot; the hi and lo slots use the same
+      // swizzled positions, so the split is elementwise and in place (hi overwrites raw).
+      // Consecutive threads take consecutive 16-byte chunks: conflict-free shared accesses.
+      float4* hi = reinterpret_cast<float4*>(smem + (size_t)s * STAGE_BYTES);
+      float4* lo = reinterpret_cast<float4*>(smem + (size_t)s * STAGE_BYTES + A_TILE_BYTES);
+#pragma unroll
+      for (int j = 0; j < (int)(A_TILE_BYTES / 16) / 128; ++j) {
+        const int i = t + 128 * j;
+        const float4 v = hi[i];
+        const float4 h = make_float4(tf32_rna(v.x), tf32_rna(v.y), tf32_rna(v.z), tf32_rna(v.w));
+        hi[i] = h;
+        lo[i] = make_float4(__fsub_rn(v.x, h.x), __fsub_rn(v.y, h.y), __fsub_rn(v.z, h.z), __fsub_rn(v.w, h.w));
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
+      __syncwarp();
+      if (lane == 0) mbar_arrive(conv_bar(s));
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      atomicOr(&g_device_status, kStatusTimeout);
+    }
+    // stage this CTA's accumulator in shared memory (the ring is free once the MMAs are done)
+    bool have = ok && (nk == 0 || mbar_wait(accum_bar, 0u, kWaitNs * 4, abort_flag));
+    have = __all_sync(0xffffffffu, have) && !*abort_flag;
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    bool ok = (nk > 0) ? mbar_wait(accum_bar, 0u, kWaitNs * 4, abort_flag) : true;
-    ok = __all_sync(0xffffffffu, ok);
-    if (ok && !*abort_flag) {
+    if (have) {
       tc_fence_after();
-      const int64_t m = m0 + 32 * q + lane;
-      float* dst = splits > 1 ? out + (int64_t)split * M * N : out;
-      const bool vec = (N & 3) == 0;
+      float* row = red + (size_t)(32 * q + lane) * RED_STRIDE;
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         float v[32];
@@ -301,38 +371,91 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
-        const int64_t nb = n0 + 32 * c;
-        if (m < M && nb < N) {
-          float* orow = dst + m * N;
-          const float* crow = (splits == 1 && C) ? C + m * N : nullptr;
-          if (vec && nb + 32 <= N) {
 #pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              float4 r = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-              if (crow) {
-                const float4 cc = __ldcs(reinterpret_cast<const float4*>(crow + nb + j));
-                r = make_float4(__fsub_rn(r.x, cc.x), __fsub_rn(r.y, cc.y), __fsub_rn(r.z, cc.z),
-                                __fsub_rn(r.w, cc.w));
-              }
-              *reinterpret_cast<float4*>(orow + nb + j) = r;
-            }
-          } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-              if (nb + j < N) orow[nb + j] = crow ? __fsub_rn(v[j], crow[nb + j]) : v[j];
-          }
-        }
+        for (int j = 0; j < 32; j += 4)
+          *reinterpret_cast<float4*>(row + 32 * c + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
       }
-    } else if (!ok) {
-      if (lane == 0) {
-        *abort_flag = 1;
-        atomicOr(&g_device_status, kStatusTimeout);
-      }
+    } else if (lane == 0) {
+      *abort_flag = 1;
+      atomicOr(&g_device_status, kStatusTimeout);
     }
   }
 
+  // ---- sum the cluster's partial tiles in rank order, subtract C, store ----
+  __syncwarp();  // lane 0 of warps 0 and 1 ran the producer / MMA loops: reconverge before the barrier
   tc_fence_before();
-  __syncthreads();
+  if (splits > 1) {
+    cluster_sync_all();  // every rank's partial tile is staged
+  } else {
+    __syncthreads();
+  }
+  {
+    // Each thread keeps kUnroll float4 positions in flight (remote partials and C loads issued
+    // before any is used), so the epilogue streams instead of waiting one load at a time.
+    constexpr int kUnroll = 4;
+    const int rank = splits > 1 ? (int)cluster_rank() : 0;
+    const int rows_per_rank = (BM + splits - 1) / splits;
+    const int r0 = rank * rows_per_rank, r1 = (r0 + rows_per_rank < BM) ? r0 + rows_per_rank : BM;
+    const bool vec = (N & 3) == 0;
+    const uint32_t red_base = smem_u32(red);
+    const int total = (r1 - r0) * (BN / 4);
+    for (int base = threadIdx.x; base < total; base += THREADS * kUnroll) {
+      float4 acc[kUnroll], cc[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int idx = base + u * THREADS;
+        acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        cc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (idx >= total) continue;
+        const int r = r0 + idx / (BN / 4), c = 4 * (idx % (BN / 4));
+        const int64_t m = m0 + r, n = n0 + c;
+        if (m >= M || n >= N) continue;
+        const uint32_t off = red_base + (uint32_t)((r * RED_STRIDE + c) * 4);
+        if (splits > 1) {
+          float4 part[MAX_CLUSTER];
+#pragma unroll
+          for (int qr = 0; qr < MAX_CLUSTER; ++qr)  // all remote loads in flight at once
+            if (qr < splits) part[qr] = ld_cluster_f4(map_to_rank(off, (uint32_t)qr));
+          acc[u] = part[0];
+#pragma unroll
+          for (int qr = 1; qr < MAX_CLUSTER; ++qr)  // summed in rank order
+            if (qr < splits)
+              acc[u] = make_float4(__fadd_rn(acc[u].x, part[qr].x), __fadd_rn(acc[u].y, part[qr].y),
+                                   __fadd_rn(acc[u].z, part[qr].z), __fadd_rn(acc[u].w, part[qr].w));
+        } else {
+          acc[u] = *reinterpret_cast<const float4*>(red + r * RED_STRIDE + c);
+        }
+        if (C && vec && n + 4 <= N) cc[u] = __ldcs(reinterpret_cast<const float4*>(C + m * N + n));
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int idx = base + u * THREADS;
+        if (idx >= total) continue;
+        const int r = r0 + idx / (BN / 4), c = 4 * (idx % (BN / 4));
+        const int64_t m = m0 + r, n = n0 + c;
+        if (m >= M || n >= N) continue;
+        float* o = out + m * N + n;
+        if (vec && n + 4 <= N) {
+          float4 v = acc[u];
+          if (C)
+            v = make_float4(__fsub_rn(v.x, cc[u].x), __fsub_rn(v.y, cc[u].y), __fsub_rn(v.z, cc[u].z),
+                            __fsub_rn(v.w, cc[u].w));
+          *reinterpret_cast<float4*>(o) = v;
+        } else {
+          const float v[4] = {acc[u].x, acc[u].y, acc[u].z, acc[u].w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (n + j < N) o[j] = C ? __fsub_rn(v[j], C[m * N + n + j]) : v[j];
+        }
+      }
+    }
+  }
+  __syncwarp();
+  if (splits > 1) {
+    cluster_sync_all();  // no CTA leaves while others still read its shared memory
+  } else {
+    __syncthreads();
+  }
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
@@ -373,19 +496,64 @@ bool make_map(CUtensorMap* map, const float* base, int64_t rows, int64_t K, int 
   return r == CUDA_SUCCESS;
 }
 
+// Co-resident clusters of s CTAs (each one SM) on the current device; clusters
+// must fit inside one GPC, so this is not simply SMs / s.  Cached per device.
+int max_active_clusters(int s, int sms) {
+  static int cache[64][MAX_CLUSTER + 1] = {{0}};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return std::max(1, sms / s);
+  int& v = cache[dev][s];
+  if (v == 0) {
+    int n = 0;
+    if (cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) ==
+        cudaSuccess) {
+      cudaLaunchConfig_t cfg;
+      std::memset(&cfg, 0, sizeof(cfg));
+      cfg.gridDim = dim3(1, 1, (unsigned)s);
+      cfg.blockDim = dim3(THREADS, 1, 1);
+      cfg.dynamicSmemBytes = SMEM_BYTES;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 1;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = (unsigned)s;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();
+    v = n > 0 ? n : std::max(1, sms / s);
+  }
+  return v;
+}
+
 }  // namespace
 
 Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
+  // Split K across a cluster of up to 8 CTAs only when the output tiles alone
+  // leave SMs idle.  A CTA costs a fixed overhead (launch, pipeline fill, the
+  // staging and cross-CTA reduction of its 128 KB tile) worth about 450 of K
+  // on GB300 plus its K range, so time ~ waves x (450 + K / s), where waves
+  // counts the co-resident clusters of size s.  At least 256 of K per CTA;
+  // ties go to fewer splits.
+  constexpr double kFixedK = 450.0;
   Plan p{};
   p.kernel = kKernelTc;
   const int64_t tiles = ceil_div(M, BM) * ceil_div(N, BN);
-  int64_t s = tiles >= sms ? 1 : std::max<int64_t>(1, sms / std::max<int64_t>(tiles, 1));
-  s = std::min<int64_t>(s, std::max<int64_t>(1, K / 256));  // at least 256 K per split
-  p.k_per_split = round_up(ceil_div(K, s), BK);
+  const int64_t max_s = tiles >= sms ? 1 : std::max<int64_t>(1, std::min<int64_t>(MAX_CLUSTER, K / 256));
+  int64_t best = 1;
+  double best_cost = 1e300;
+  for (int64_t s = 1; s <= max_s; ++s) {
+    const int64_t clusters = max_active_clusters((int)s, sms);
+    const double cost = (double)ceil_div(tiles, clusters) * (kFixedK + (double)K / (double)s);
+    if (cost < best_cost * (1.0 - 1e-9)) {
+      best_cost = cost;
+      best = s;
+    }
+  }
+  p.k_per_split = round_up(ceil_div(K, best), BK);
   p.splits = (int)std::max<int64_t>(1, ceil_div(K, p.k_per_split));
-  p.ws_partials = p.splits > 1 ? (size_t)round_up((int64_t)p.splits * M * N * 4, 256) : 0;
-  p.ws_asplit = (size_t)round_up(M * K * 4, 256) * 2;
-  return p;
+  return p;  // no workspace: partials are reduced through distributed shared memory
 }
 
 spl_status run_tc(const LinearArgs& a, const Plan& p) {
@@ -394,20 +562,12 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
   if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
   if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
   if (a.M > 0x7fffffffLL || a.N > 0x7fffffffLL || a.K > 0x7fffffffLL) return SPL_ESHAPE;
-  if (ceil_div(a.M, BM) > 65535 || p.splits > 65535) return SPL_ESHAPE;
-
-  // A operand split into the workspace: [hi | lo], each M*K fp32
-  char* ws = static_cast<char*>(a.ws) + kCounterBytes;
-  float* part = reinterpret_cast<float*>(ws);
-  float* a_hi = reinterpret_cast<float*>(ws + p.ws_partials);
-  float* a_lo = reinterpret_cast<float*>(ws + p.ws_partials + p.ws_asplit / 2);
-  spl_status st = run_split_tf32(a_hi, a_lo, a.a, a.M * a.K, a.stream);
-  if (st != SPL_OK) return st;
+  if (ceil_div(a.M, BM) > 65535 || p.splits > MAX_CLUSTER) return SPL_ESHAPE;
 
   TcMaps maps;
   std::memset(&maps, 0, sizeof(maps));
-  if (!make_map(&maps.a_hi, a_hi, a.M, a.K, BM) || !make_map(&maps.a_lo, a_lo, a.M, a.K, BM) ||
-      !make_map(&maps.w_hi, a.w_hi, a.N, a.K, BN) || !make_map(&maps.w_lo, a.w_lo, a.N, a.K, BN))
+  if (!make_map(&maps.a, a.a, a.M, a.K, BM) || !make_map(&maps.w_hi, a.w_hi, a.N, a.K, BN) ||
+      !make_map(&maps.w_lo, a.w_lo, a.N, a.K, BN))
     return SPL_ECUDA;
 
   static bool attr_set[64] = {false};
@@ -419,13 +579,23 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
       return SPL_ECUDA;
     attr_set[dev] = true;
   }
-  dim3 grid((unsigned)ceil_div(a.N, BN), (unsigned)ceil_div(a.M, BM), (unsigned)p.splits);
-  float* dst = p.splits > 1 ? part : a.out;
-  tc_gemm_kernel<<<grid, THREADS, SMEM_BYTES, a.stream>>>(maps, dst, p.splits > 1 ? nullptr : a.c, a.M, a.K, a.N,
-                                                          p.k_per_split, p.splits);
-  st = launch_status();
-  if (st != SPL_OK || p.splits == 1) return st;
-  return run_splitk_reduce(a.out, part, a.c, p.splits, a.M, a.N, a.stream);
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3((unsigned)ceil_div(a.N, BN), (unsigned)ceil_div(a.M, BM), (unsigned)p.splits);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.stream = a.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = (unsigned)p.splits;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel, maps, a.out, a.c, a.M, a.K, a.N, p.k_per_split,
+                                           p.splits);
+  note_launches(1);
+  return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
 }
 
 }  // namespace spl

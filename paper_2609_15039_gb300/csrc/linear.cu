@@ -5,11 +5,11 @@
 //   spl_precompute_noise_product  C = N W^T             (Sec. 5.2)
 //   spl_masked_linear_unmask      Y = X~ W^T - C        (Eq. add-and-then-subtract, fused)
 //
-// Kernel choice: M <= 16 rows stream W once through the decode kernel (FP32);
-// larger M use the TF32X3 tcgen05 kernel when the weight split is available,
-// the device is sm_100/sm_103 and K >= 64 (below that the three-product error
-// of about 2^-20 per term is not small against gamma_K), otherwise the FP32
-// SIMT kernel.
+// Kernel choice: on the FP32 path M <= 16 rows stream W once through the decode
+// kernel and larger M use the SIMT kernel.  AUTO takes the TF32X3 tcgen05
+// kernel for M > 8 when the weight split is available, the device is
+// sm_100/sm_103 and K >= 64 (below that the three-product error of about
+// 2^-20 per term is not small against gamma_K), else FP32.
 
 #include <algorithm>
 
@@ -23,9 +23,14 @@ bool tc_capable() {
   return cc == 100 || cc == 103;
 }
 
+// AUTO: up to 8 rows the streaming decode kernel reads W once at HBM rate and
+// wins; from 9 rows on the tensor-core kernel is faster even with its 128-row
+// tile mostly empty (the decode kernel turns shared-memory bound as M grows).
+constexpr int64_t kAutoDecodeMaxM = 8;
+
 spl_path resolve(int64_t M, int64_t K, spl_path path, bool have_split) {
   if (path == SPL_PATH_FP32 || path == SPL_PATH_TF32X3) return path;
-  if (M > kGemvMaxM && K >= 64 && have_split && tc_capable()) return SPL_PATH_TF32X3;
+  if (M > kAutoDecodeMaxM && K >= 64 && have_split && tc_capable()) return SPL_PATH_TF32X3;
   return SPL_PATH_FP32;
 }
 

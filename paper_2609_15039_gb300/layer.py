@@ -1,16 +1,23 @@
 """One decoder layer's outsourced linears, run through the C ABI.
 
-Sec. 5.2: the inputs of Q, K and V are the same, so one mask serves all
-three (three corrections); Gate and Up likewise share one mask (two
-corrections); O (and Down, which the paper keeps in the TEE but this
-workload includes) get one each.  Per input group the step is
+Sec. 5.2 of the paper keeps a noise bank: masks and their corrections are
+precomputed, one mask serves every projection that shares an input (Q, K, V
+share one; Gate and Up share one; O and Down one each), and each entry is
+consumed once.  This module keeps that structure, GB300 style:
 
-    a2+a3  spl_noise_mask                 X~ = X + eta, eta kept for a4
-    a4     spl_precompute_noise_product   C_p = eta W_p^T   for each projection p
-    a5+a6  spl_masked_linear_unmask       Y_p = X~ W_p^T - C_p
+* weights that share an input are stored as one matrix (Q|K|V is [5120, d],
+  Gate|Up is [2 d_ff, d] for Llama), so one product call serves the group and
+  its output columns are the individual projections;
+* the bank holds only corrections.  ``refill`` draws D masks per group in
+  one pass (a2) and computes their corrections C = eta W^T as one product of
+  D*M rows (a4, "precomputed in a batch");
+* an ``online`` step regenerates its mask from the same Philox counters
+  (seed, group stream, block offset of draw d) instead of reading it back,
+  masks the input (a3) and runs the masked product with the unmask fused
+  into its epilogue, Y = X~ W^T - C_d (a5 + a6).
 
-with the noise scale b = Delta / eps from Thms. 1-3 (a1), evaluated once per
-layer by ``sensitivities``.  This module only sequences library calls.
+The noise scale Delta per group comes from Thms. 1-3 (a1, ``sensitivities``).
+This module only sequences library calls; all arithmetic is in libspl.
 """
 
 from dataclasses import dataclass, field
@@ -20,109 +27,150 @@ import torch
 from . import spl
 
 
-
 @dataclass
-class ProjectionWeights:
-    name: str
-    group: str
+class GroupWeights:
+    name: str            # qkv | o | gateup | down
     K: int
-    N: int
-    W: torch.Tensor
+    names: list          # projections in column order
+    widths: list         # output width of each projection
+    W: torch.Tensor      # [sum(widths), K]
     W_hi: torch.Tensor = None
     W_lo: torch.Tensor = None
+
+    @property
+    def N(self):
+        return self.W.shape[0]
+
+    def columns(self, name):
+        i = self.names.index(name)
+        off = sum(self.widths[:i])
+        return off, off + self.widths[i]
 
 
 @dataclass
 class MaskedLayer:
-    """Device-resident weights of one layer plus the per-group noise scales."""
+    """Device-resident fused weights of one layer, its noise scales and its correction bank."""
 
     model: object
-    projections: list
+    groups: list
     deltas: dict = field(default_factory=dict)
     workspace: torch.Tensor = None
-    M_max: int = 0
+    bank: dict = field(default_factory=dict)
+    draws: int = 0
+    M: int = 0
 
     @classmethod
     def from_weights(cls, model, weights, split=True, device="cuda"):
-        """weights: {name: [N, K] fp32 tensor}.  Splits each for TF32X3 when split=True."""
-        projs = []
-        for name, K, N, g in model.projections():
-            W = weights[name].to(device=device, dtype=torch.float32).contiguous()
-            pw = ProjectionWeights(name, g, K, N, W)
+        """weights: {projection: [N, K] fp32}.  Concatenates per input group; splits for TF32X3."""
+        groups = []
+        for g, K, names in model.input_groups():
+            parts = [weights[n].to(device=device, dtype=torch.float32) for n in names]
+            W = torch.cat(parts, dim=0).contiguous() if len(parts) > 1 else parts[0].contiguous()
+            gw = GroupWeights(g, K, list(names), [p.shape[0] for p in parts], W)
             if split:
-                pw.W_hi = torch.empty_like(W)
-                pw.W_lo = torch.empty_like(W)
-                spl.spl_split_tf32(pw.W_hi, pw.W_lo, W)
-            projs.append(pw)
-        return cls(model, projs)
+                gw.W_hi, gw.W_lo = torch.empty_like(W), torch.empty_like(W)
+                spl.spl_split_tf32(gw.W_hi, gw.W_lo, W)
+            groups.append(gw)
+        return cls(model, groups)
 
-    def proj(self, name):
-        return next(p for p in self.projections if p.name == name)
+    def group(self, name):
+        return next(g for g in self.groups if g.name == name)
 
-    def sensitivities(self, alpha=None, beta=None, power_iters=100):
-        """a1: Delta per input group (Thm. 1 for qkv/gateup, Thm. 2 for o, Thm. 3 for down)."""
+    def weight(self, proj):
+        """The [N, K] block of one projection (a view into its group's matrix)."""
+        for g in self.groups:
+            if proj in g.names:
+                a, b = g.columns(proj)
+                return g.W[a:b]
+        raise KeyError(proj)
+
+    def sensitivities(self, alpha=None, beta=None, power_iters=1000):
+        """a1: Delta per input group (Thm. 1 for qkv/gateup, Thm. 2 for o, Thm. 3 for down).
+
+        ||W||_2 comes from power iteration, which approaches it from below;
+        enough iterations make the shortfall negligible next to the noise scale.
+        """
         d = self.model.d_model
         a = torch.ones(d) if alpha is None else torch.as_tensor(alpha, dtype=torch.float32)
         d_ln = spl.spl_delta_layernorm(a)
-        wv = spl.spl_spectral_norm(self.proj("v").W, iters=power_iters)
-        wup = spl.spl_spectral_norm(self.proj("up").W, iters=power_iters)
-        wgate = spl.spl_spectral_norm(self.proj("gate").W, iters=power_iters)
+        norms = {p: spl.spl_spectral_norm(self.weight(p).contiguous(), iters=power_iters) for p in ("v", "up", "gate")}
         self.deltas = {
             "qkv": d_ln,
             "gateup": d_ln,
-            "o": spl.spl_delta_attention(a, wv),
-            "down": spl.spl_delta_activation(a, beta, self.model.d_ff, wup, wgate),
+            "o": spl.spl_delta_attention(a, norms["v"]),
+            "down": spl.spl_delta_activation(a, beta, self.model.d_ff, norms["up"], norms["gate"]),
         }
-        self.norms = {"v": wv, "up": wup, "gate": wgate}
+        self.norms = norms
         return self.deltas
 
-    def ensure_workspace(self, M, path="auto"):
-        need = max(spl.spl_linear_workspace_bytes(M, p.K, p.N, path) for p in self.projections)
+    # ------------------------------------------------------------------ bank
+    def allocate(self, M, draws, path="auto"):
+        """Buffers for M tokens and a bank of ``draws`` corrections per group."""
+        dev = self.groups[0].W.device
+        need = 0
+        for g in self.groups:
+            need = max(need, spl.spl_linear_workspace_bytes(M, g.K, g.N, path),
+                       spl.spl_linear_workspace_bytes(draws * M, g.K, g.N, path))
         if self.workspace is None or self.workspace.numel() < need:
-            self.workspace = spl.workspace(need, self.projections[0].W.device)
-        self.M_max = max(self.M_max, M)
-        return self.workspace
+            self.workspace = spl.workspace(need, dev)
+        self.M, self.draws = M, draws
+        self.bank = {}
+        for g in self.groups:
+            self.bank[g.name] = {
+                "eta": torch.empty((draws * M, g.K), device=dev),  # transient: the draws being precomputed
+                "C": torch.empty((draws * M, g.N), device=dev),
+                "xt": torch.empty((M, g.K), device=dev),
+                "Y": torch.empty((M, g.N), device=dev),
+            }
 
-    def step(self, inputs, eps, mech, seed, outputs=None, scratch=None, path="auto", stream=None, timer=None):
-        """Run every group of the layer once.
+    def block_offset(self, g, cycle, d):
+        """First Philox block of draw d of bank cycle ``cycle`` for group g."""
+        per_draw = self.M * g.K // 4  # K % 4 == 0, so a draw is a whole number of blocks
+        return (cycle * self.draws + d) * per_draw
 
-        inputs:  {group: X [M, K] device tensor}
-        outputs: {name: Y [M, N]} (allocated if None); scratch holds X~, eta, C.
-        Philox stream ids: one per group (0..3) under ``seed``, so no two groups
-        (and no two layers, if seeds differ) share a counter.  ``timer`` (if
-        given) is called as timer("begin"|"end", kind) around each product call.
+    def refill(self, eps, mech, seed, cycle, path="auto", stream=None, timer=None):
+        """a2 + a4: draw ``draws`` masks per group and precompute their corrections in one product."""
+        for gi, g in enumerate(self.groups):
+            b = self.bank[g.name]
+            spl.spl_noise(b["eta"], self.deltas[g.name], eps, mech, seed, stream_id=gi,
+                          offset=self.block_offset(g, cycle, 0), stream=stream)
+            if timer:
+                timer("begin", "precompute")
+            spl.spl_precompute_noise_product(b["C"], b["eta"], g.W, g.W_hi, g.W_lo, path=path,
+                                             workspace=self.workspace, stream=stream)
+            if timer:
+                timer("end", "precompute")
+
+    def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None):
+        """a3 + a5 + a6 for draw d: regenerate eta_d, mask, masked product with fused unmask.
+
+        inputs: {group: X [M, K]}.  Returns {group: Y [M, N_group]} (views of the layer's buffers).
         """
-        ws = self.ensure_workspace(max(x.shape[0] for x in inputs.values()), path)
-        outputs = {} if outputs is None else outputs
-        scratch = {} if scratch is None else scratch
-        for gi, (g, K, names) in enumerate(self.model.input_groups()):
-            X = inputs[g]
-            M = X.shape[0]
-            xt = scratch.get(("xt", g))
-            if xt is None or xt.shape != X.shape:
-                xt = scratch[("xt", g)] = torch.empty_like(X)
-                scratch[("eta", g)] = torch.empty_like(X)
-            eta = scratch[("eta", g)]
-            spl.spl_noise_mask(xt, eta, X, self.deltas[g], eps, mech, seed, stream_id=gi, stream=stream)
-            for name in names:
-                p = self.proj(name)
-                C = scratch.get(("c", name))
-                if C is None or C.shape[0] != M:
-                    C = scratch[("c", name)] = torch.empty((M, p.N), device=X.device)
-                Y = outputs.get(name)
-                if Y is None or Y.shape[0] != M:
-                    Y = outputs[name] = torch.empty((M, p.N), device=X.device)
-                if timer:
-                    timer("begin", "precompute")
-                spl.spl_precompute_noise_product(C, eta, p.W, p.W_hi, p.W_lo, path=path, workspace=ws, stream=stream)
-                if timer:
-                    timer("end", "precompute")
-                    timer("begin", "masked_linear_unmask")
-                spl.spl_masked_linear_unmask(Y, xt, p.W, C, p.W_hi, p.W_lo, path=path, workspace=ws, stream=stream)
-                if timer:
-                    timer("end", "masked_linear_unmask")
-        return outputs, scratch
+        M = self.M
+        out = {}
+        for gi, g in enumerate(self.groups):
+            b = self.bank[g.name]
+            spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
+                               offset=self.block_offset(g, cycle, d), stream=stream)
+            if timer:
+                timer("begin", "masked_linear_unmask")
+            spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M], g.W_hi, g.W_lo,
+                                         path=path, workspace=self.workspace, stream=stream)
+            if timer:
+                timer("end", "masked_linear_unmask")
+            out[g.name] = b["Y"]
+        return out
 
-    def flops(self, M):
-        """Algorithmic flops of one step: the masked product and the correction, 2 M K N each."""
-        return sum(2 * 2 * M * p.K * p.N for p in self.projections)
+    def flops_per_step(self):
+        """Algorithmic flops per online step: the masked product plus its share of the batched correction."""
+        return sum(2 * 2 * self.M * g.K * g.N for g in self.groups)
+
+
+def split_outputs(layer, outs):
+    """{projection: [M, N_p] view} from the per-group outputs."""
+    res = {}
+    for g in layer.groups:
+        for p in g.names:
+            a, b = g.columns(p)
+            res[p] = outs[g.name][:, a:b]
+    return res

@@ -292,8 +292,8 @@ def test_config_single_masked_linear(spl, path):
 # ------------------------------------------- end to end, one Llama layer (M=128)
 @pytest.fixture(scope="module")
 def llama_layer(spl):
-    from oracle import sensitivity as osens
     from paper_2609_15039_gb300.layer import MaskedLayer
+    from oracle import sensitivity as osens
     model = wl.LLAMA_3_2_3B
     weights = {name: wl.weight(N, K, seed=200 + pi) for pi, (name, K, N, g) in enumerate(model.projections())}
     layer = MaskedLayer.from_weights(model, weights)
@@ -311,32 +311,45 @@ def llama_layer(spl):
 
 def test_layer_sensitivities_match_oracle(llama_layer):
     layer, _weights_, deltas, norms = llama_layer
-    # power iteration approaches ||W||_2 from below; 400 steps bring it within 0.3% on these
+    # power iteration approaches ||W||_2 from below; 1000 steps bring it within 1e-5 on these
     # Gaussian matrices, whose top singular values are close together
-    got = layer.sensitivities(power_iters=400)
+    got = layer.sensitivities(power_iters=1000)
     for g in deltas:
         assert got[g] <= deltas[g] * (1 + 1e-5), g
-        assert got[g] == pytest.approx(deltas[g], rel=3e-3), g
+        assert got[g] == pytest.approx(deltas[g], rel=1e-4), g
     assert got["qkv"] == pytest.approx(2 * 3072 ** 0.75, rel=1e-9)
 
 
 @pytest.mark.parametrize("eps", [0.5, 1.0, 4.0])
-def test_config_llama_layer(llama_layer, eps):
+def test_config_llama_layer(spl, llama_layer, eps):
+    from paper_2609_15039_gb300.layer import split_outputs
     layer, weights, deltas, _norms = llama_layer
     layer.deltas = dict(deltas)
-    model, M, mech, seed = layer.model, wl.CONFIGS["llama_layer"]["M"], "gaussian", 31
+    model, M, mech, seed, draws = layer.model, wl.CONFIGS["llama_layer"]["M"], "gaussian", 31, 2
+    layer.allocate(M, draws)
     inputs_np = {g: wl.activations(M, K, seed=100 + gi).numpy() for gi, (g, K, _n) in enumerate(model.input_groups())}
-    outs, _scratch = layer.step({g: dev(x) for g, x in inputs_np.items()}, eps, mech, seed)
-    torch.cuda.synchronize()
-    for gi, (g, K, names) in enumerate(model.input_groups()):
-        X = inputs_np[g]
-        n_or = philox.noise((M, K), deltas[g], eps, mech, seed, stream_id=gi)
-        xt_or = linear.mask(X, n_or)
-        for name in names:
-            W = weights[name].numpy()
-            S = linear.abs_products(X, xt_or, n_or, W)
-            err = np.abs(f64(outs[name]) - linear.reference_output(X, W))
-            hb = bounds.hard_bound(*S, K) * (1 + 1e-5)
-            assert np.all(err <= hb), (name, float(np.max(err / hb)))
-            st = bounds.bound_statistics(err, bounds.log_bound(*S, K))
-            assert st["ratio"] > 1.0, (name, st)
+    inputs = {g: dev(x) for g, x in inputs_np.items()}
+    layer.refill(eps, mech, seed, cycle=3)
+    bank_eta = {g.name: layer.bank[g.name]["eta"].clone() for g in layer.groups}
+    for d in range(draws):
+        outs = split_outputs(layer, layer.online(inputs, eps, mech, seed, cycle=3, d=d))
+        torch.cuda.synchronize()
+        for gi, g in enumerate(layer.groups):
+            # the online step regenerates exactly the bank's mask of draw d
+            regen = torch.empty((M, g.K), device="cuda")
+            xt = torch.empty((M, g.K), device="cuda")
+            spl.spl_noise_mask(xt, regen, inputs[g.name], deltas[g.name], eps, mech, seed, stream_id=gi,
+                                   offset=layer.block_offset(g, 3, d))
+            assert torch.equal(regen, bank_eta[g.name][d * M:(d + 1) * M])
+            X = inputs_np[g.name]
+            n_or = philox.noise((M, g.K), deltas[g.name], eps, mech, seed, stream_id=gi,
+                                offset=layer.block_offset(g, 3, d))
+            xt_or = linear.mask(X, n_or)
+            for name in g.names:
+                W = weights[name].numpy()
+                S = linear.abs_products(X, xt_or, n_or, W)
+                err = np.abs(f64(outs[name]) - linear.reference_output(X, W))
+                hb = bounds.hard_bound(*S, g.K) * (1 + 1e-5)
+                assert np.all(err <= hb), (name, d, float(np.max(err / hb)))
+                st = bounds.bound_statistics(err, bounds.log_bound(*S, g.K))
+                assert st["ratio"] > 1.0, (name, st)
