@@ -214,13 +214,13 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
-// One CTA computes a 128 x 256 tile of out over the K range of its split.
+// One CTA computes a 128 x 256 tile of out over the K range of its split (blockIdx.z).
 // The `splits` CTAs of a tile form one thread-block cluster (z dimension);
 // their fp32 partial tiles are summed through distributed shared memory in
 // cluster-rank order, so the result does not depend on timing.
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
-               int64_t M, int64_t K, int64_t N, int64_t k_per_split, int splits) {
+               int64_t M, int64_t K, int64_t N, int64_t k_per_split, int splits, int tile_base, int m_tiles) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + BAR_OFFSET);  // full[S], conv[S], empty[S], accum
@@ -229,7 +229,9 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   float* red = reinterpret_cast<float*>(smem);  // [BM][RED_STRIDE] staged accumulator, after the mainloop
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t m0 = (int64_t)blockIdx.y * BM, n0 = (int64_t)blockIdx.x * BN;
+  // Linear tile id, M fastest: the CTAs that read the same weight tile run side by side and share it in L2.
+  const int tile = tile_base + (int)blockIdx.x;
+  const int64_t m0 = (int64_t)(tile % m_tiles) * BM, n0 = (int64_t)(tile / m_tiles) * BN;
   const int split = blockIdx.z;
   const int64_t kbeg = (int64_t)split * k_per_split;
   const int64_t kend = std::min<int64_t>(K, kbeg + k_per_split);
@@ -527,20 +529,15 @@ int max_active_clusters(int s, int sms) {
   return v;
 }
 
-}  // namespace
+// Split of the tiles into launches: full waves of unsplit tiles, then the remaining tiles with
+// K split across clusters so the last wave is not mostly idle.  Time of a launch ~ waves x
+// (kFixedK + K / s), waves counting co-resident clusters of size s; kFixedK is the fixed cost of
+// a CTA (launch, pipeline fill, staging and cross-CTA reduction of its 128 KB tile) measured on
+// GB300 in units of K.  At least 256 of K per CTA; ties go to fewer splits.
+constexpr double kFixedK = 450.0;
 
-Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
-  // Split K across a cluster of up to 8 CTAs only when the output tiles alone
-  // leave SMs idle.  A CTA costs a fixed overhead (launch, pipeline fill, the
-  // staging and cross-CTA reduction of its 128 KB tile) worth about 450 of K
-  // on GB300 plus its K range, so time ~ waves x (450 + K / s), where waves
-  // counts the co-resident clusters of size s.  At least 256 of K per CTA;
-  // ties go to fewer splits.
-  constexpr double kFixedK = 450.0;
-  Plan p{};
-  p.kernel = kKernelTc;
-  const int64_t tiles = ceil_div(M, BM) * ceil_div(N, BN);
-  const int64_t max_s = tiles >= sms ? 1 : std::max<int64_t>(1, std::min<int64_t>(MAX_CLUSTER, K / 256));
+int best_split(int64_t tiles, int64_t K, int sms) {
+  const int64_t max_s = std::max<int64_t>(1, std::min<int64_t>(MAX_CLUSTER, K / 256));
   int64_t best = 1;
   double best_cost = 1e300;
   for (int64_t s = 1; s <= max_s; ++s) {
@@ -551,8 +548,40 @@ Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
       best = s;
     }
   }
-  p.k_per_split = round_up(ceil_div(K, best), BK);
-  p.splits = (int)std::max<int64_t>(1, ceil_div(K, p.k_per_split));
+  return (int)best;
+}
+
+struct TcLaunches {
+  int64_t full_tiles;  // tiles of the first, unsplit launch (whole waves)
+  int64_t rest_tiles;  // tiles of the second launch
+  int rest_splits;
+};
+
+TcLaunches tc_launches(int64_t M, int64_t K, int64_t N, int sms) {
+  const int64_t tiles = ceil_div(M, BM) * ceil_div(N, BN);
+  TcLaunches t{0, tiles, 1};
+  const int64_t waves = tiles / sms;
+  if (waves >= 1) {
+    // keep the unsplit waves only if splitting the remainder beats one more unsplit wave
+    const int64_t rest = tiles - waves * sms;
+    if (rest == 0) return TcLaunches{tiles, 0, 1};
+    const int s = best_split(rest, K, sms);
+    const double split_cost = (double)ceil_div(rest, max_active_clusters(s, sms)) * (kFixedK + (double)K / s);
+    if (split_cost < kFixedK + (double)K) return TcLaunches{waves * sms, rest, s};
+    return TcLaunches{0, tiles, 1};
+  }
+  t.rest_splits = best_split(tiles, K, sms);
+  return t;
+}
+
+}  // namespace
+
+Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
+  Plan p{};
+  p.kernel = kKernelTc;
+  const TcLaunches t = tc_launches(M, K, N, sms);
+  p.splits = t.rest_splits;
+  p.k_per_split = round_up(ceil_div(K, t.rest_splits), BK);
   return p;  // no workspace: partials are reduced through distributed shared memory
 }
 
@@ -562,7 +591,7 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
   if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
   if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
   if (a.M > 0x7fffffffLL || a.N > 0x7fffffffLL || a.K > 0x7fffffffLL) return SPL_ESHAPE;
-  if (ceil_div(a.M, BM) > 65535 || p.splits > MAX_CLUSTER) return SPL_ESHAPE;
+  if (ceil_div(a.M, BM) * ceil_div(a.N, BN) > 0x7fffffffLL || p.splits > MAX_CLUSTER) return SPL_ESHAPE;
 
   TcMaps maps;
   std::memset(&maps, 0, sizeof(maps));
@@ -579,23 +608,32 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
       return SPL_ECUDA;
     attr_set[dev] = true;
   }
-  cudaLaunchConfig_t cfg;
-  std::memset(&cfg, 0, sizeof(cfg));
-  cfg.gridDim = dim3((unsigned)ceil_div(a.N, BN), (unsigned)ceil_div(a.M, BM), (unsigned)p.splits);
-  cfg.blockDim = dim3(THREADS, 1, 1);
-  cfg.dynamicSmemBytes = SMEM_BYTES;
-  cfg.stream = a.stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 1;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = (unsigned)p.splits;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel, maps, a.out, a.c, a.M, a.K, a.N, p.k_per_split,
-                                           p.splits);
-  note_launches(1);
-  return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
+  const int m_tiles = (int)ceil_div(a.M, BM);
+  const TcLaunches t = tc_launches(a.M, a.K, a.N, device_sm_count());
+  auto launch = [&](int64_t tiles, int64_t base, int splits) -> spl_status {
+    if (tiles <= 0) return SPL_OK;
+    const int64_t kps = round_up(ceil_div(a.K, splits), BK);
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof(cfg));
+    cfg.gridDim = dim3((unsigned)tiles, 1, (unsigned)splits);
+    cfg.blockDim = dim3(THREADS, 1, 1);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.stream = a.stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = (unsigned)splits;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel, maps, a.out, a.c, a.M, a.K, a.N, kps, splits,
+                                             (int)base, m_tiles);
+    note_launches(1);
+    return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
+  };
+  spl_status st = launch(t.full_tiles, 0, 1);
+  if (st != SPL_OK) return st;
+  return launch(t.rest_tiles, t.full_tiles, t.rest_splits);
 }
 
 }  // namespace spl
