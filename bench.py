@@ -211,6 +211,8 @@ def main():
     layer.allocate(M, DRAWS, args.path)
     inputs = {g: wl.activations(M, K, seed=100 + gi, device=dev) for gi, (g, K, _n) in
               enumerate(model.input_groups())}
+    if args.path == "auto":
+        layer.calibrate(inputs, args.eps, mech, seed)  # a8: bound-based path choice per group
     stream = torch.cuda.current_stream(dev)
 
     events = []  # (kind, begin, end) around every product call
@@ -342,6 +344,21 @@ def main():
     }
     if e2e is not None:
         result["e2e"] = e2e
+    if layer.calibration:
+        result["path_choice"] = {g: {"path": c["path"],
+                                     "tf32x3_max_err_over_hard": c["tf32x3"]["max_err_over_hard"],
+                                     "fp32_max_err_over_hard": c["fp32"]["max_err_over_hard"],
+                                     "tf32x3_mean_err": c["tf32x3"]["mean_err"], "fp32_mean_err": c["fp32"]["mean_err"]}
+                                 for g, c in layer.calibration.items()}
+    # the paper's bound over every output of one more online step, evaluated on the GPU in fp64
+    cycle, d = divmod(s, DRAWS)
+    outs = step(s)
+    s += 1
+    bc = layer.bound_check(inputs, outs, args.eps, mech, seed, cycle, d)
+    result["bound_check"] = {g: {"max_err_over_hard": v["max_err_over_hard"], "log_violation_pct": v["violation_pct"],
+                                 "mean_err": v["mean_err"], "mean_log_bound": v["mean_log_bound"],
+                                 "max_rel_err": v["max_err"] / v["max_abs_ref"] if v["max_abs_ref"] else 0.0}
+                             for g, v in bc.items()}
 
     # cpu baseline + oracle match on the first rows (rank 0, N = 1 only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

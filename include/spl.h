@@ -184,6 +184,37 @@ spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const float* W, c
 spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt, const float* W, const float* C,
                                             int64_t M, int64_t K, int64_t N, cudaStream_t stream);
 
+/* ---- a8: the cancellation bound on the GPU, and the path choice ----------
+ * The paper judges a configuration by evaluating its floating-point bound on
+ * sampled inputs and masks (Sec. 4.5 after Thm. 4; Sec. 6.3.2).
+ * spl_bound_check does this for `rows` rows: with u = 2^-24, gamma_n = n u/(1 - n u),
+ * S_x = <|w|,|x|>, S_xt = <|w|,|x~|>, S_n = <|w|,|eta|> and the exact Y* = X W^T (all fp64),
+ *   hard = gamma_K (S_x+S_xt+S_n) + u S_x + u S_xt (1+u)/(1-u) + u gamma_K (S_x+S_xt+S_n)
+ *          (Thm. 4 plus the rounding of the mask, second-order term written out)
+ *   log  = gamma_{ceil(log2 K)+1} (S_x+S_xt+S_n) + u S_x            (Eq. fp-log-bound)
+ * and writes SPL_BOUND_STATS doubles to the HOST array stats:
+ *   [0] max |Y-Y*|/hard  [1] max |Y-Y*|/log  [2] count |Y-Y*| > log  [3] sum |Y-Y*|
+ *   [4] sum log  [5] sum hard  [6] elements  [7] max |Y*|  [8] max |Y-Y*|.
+ * Y [rows, N] is the recovered output; X, Xt, Nz [rows, K]; W [N, K]; all device fp32.
+ * Needs a device workspace of >= 8 * SPL_BOUND_STATS bytes; synchronises `stream`. */
+#define SPL_BOUND_STATS 9
+spl_status spl_bound_check(double* stats, const float* Y, const float* X, const float* Xt, const float* Nz,
+                           const float* W, int64_t rows, int64_t K, int64_t N, void* workspace,
+                           size_t workspace_bytes, cudaStream_t stream);
+
+/* Bytes of device workspace spl_choose_path needs for a sample of `rows` rows. */
+size_t spl_choose_path_workspace_bytes(int64_t rows, int64_t K, int64_t N);
+
+/* a8: masks the sample X (+ Nz), computes the correction and the masked product with the
+ * unmask on each path (FP32, and TF32X3 if W_hi/W_lo are given and the device has tcgen05),
+ * checks both with spl_bound_check and sets *chosen to TF32X3 only if its max error over the
+ * hard bound is <= 1 and its log-bound violations and summed error are no worse than FP32's
+ * (within 1% of the elements and a factor 1.5), else FP32.  Both stats arrays (HOST,
+ * SPL_BOUND_STATS each) are filled; an unavailable path reports +inf in [0].  Synchronises. */
+spl_status spl_choose_path(spl_path* chosen, double* stats_tf32x3, double* stats_fp32, const float* X,
+                           const float* Nz, const float* W, const float* W_hi, const float* W_lo, int64_t rows,
+                           int64_t K, int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
 /* ---- a1: noise scale ----------------------------------------------------
  * Global l2 sensitivities (Sec. 4.3), evaluated in fp64 on the host from
  * HOST arrays.  Return a negative value on invalid input.
@@ -202,6 +233,16 @@ double spl_delta_activation(const float* alpha, const float* beta, int64_t d, in
  * `stream` and writes the result to the HOST double *out. */
 spl_status spl_spectral_norm(double* out, const float* W, int64_t N, int64_t K, int iters,
                              void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* Test hook for failure detection (the paper has no counterpart).  Runs one
+ * TF32X3 product (K <= 256, so each tile has a single K range) in which the
+ * copy of the first K stage is deliberately never issued: the kernel's bounded
+ * waits run out after about one second, it sets the device status word, lets
+ * the copies it did issue land, frees its tensor memory and returns.  The next
+ * spl_get_device_status returns SPL_ETIMEOUT and the context stays usable.
+ * `out` receives unspecified values. */
+spl_status spl_test_tc_wait_timeout(float* out, const float* A, const float* W, const float* W_hi,
+                                    const float* W_lo, int64_t M, int64_t K, int64_t N, cudaStream_t stream);
 
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last

@@ -220,7 +220,8 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 // cluster-rank order, so the result does not depend on timing.
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
-               int64_t M, int64_t K, int64_t N, int64_t k_per_split, int splits, int tile_base, int m_tiles) {
+               int64_t M, int64_t K, int64_t N, int64_t k_per_split, int splits, int tile_base, int m_tiles,
+               int skip_kblock) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + BAR_OFFSET);  // full[S], conv[S], empty[S], accum
@@ -271,6 +272,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
       ok = __all_sync(0xffffffffu, mbar_wait(empty_bar(s), ph ^ 1u, kWaitNs, abort_flag));
       if (!ok) break;
+      if (kb == skip_kblock) continue;  // failure-detection test only: this stage never arrives
       if (lane == 0) {
         const uint32_t st = smem_u32(smem + (size_t)s * STAGE_BYTES);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
@@ -585,7 +587,7 @@ Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
   return p;  // no workspace: partials are reduced through distributed shared memory
 }
 
-spl_status run_tc(const LinearArgs& a, const Plan& p) {
+spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock) {
   const int cc = device_cc();
   if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
   if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
@@ -627,7 +629,7 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel, maps, a.out, a.c, a.M, a.K, a.N, kps, splits,
-                                             (int)base, m_tiles);
+                                             (int)base, m_tiles, skip_kblock);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   };
@@ -636,4 +638,19 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
   return launch(t.rest_tiles, t.full_tiles, t.rest_splits);
 }
 
+spl_status run_tc(const LinearArgs& a, const Plan& p) { return run_tc_impl(a, p, -1); }
+
 }  // namespace spl
+
+// Failure-detection test hook: one TF32X3 product in which the copy of the first K stage is
+// never issued, so the kernel's bounded waits run out (about 1 s), it raises the device status
+// word and returns.  The paper has no counterpart.
+extern "C" spl_status spl_test_tc_wait_timeout(float* out, const float* A, const float* W, const float* W_hi,
+                                               const float* W_lo, int64_t M, int64_t K, int64_t N,
+                                               cudaStream_t stream) {
+  using namespace spl;
+  if (!out || !A || !W || !W_hi || !W_lo || M <= 0 || N <= 0 || K <= 0 || (K & 3)) return SPL_EINVAL;
+  if (K > 256) return SPL_ESHAPE;  // one K range per tile: the skipped stage belongs to every CTA
+  LinearArgs args{out, A, W, W_hi, W_lo, nullptr, M, K, N, nullptr, 0, stream};
+  return run_tc_impl(args, plan_tc(M, K, N, device_sm_count()), 0);
+}

@@ -58,6 +58,8 @@ class MaskedLayer:
     bank: dict = field(default_factory=dict)
     draws: int = 0
     M: int = 0
+    paths: dict = field(default_factory=dict)   # per group, from calibrate(); "auto" if not calibrated
+    calibration: dict = field(default_factory=dict)
 
     @classmethod
     def from_weights(cls, model, weights, split=True, device="cuda"):
@@ -103,6 +105,28 @@ class MaskedLayer:
         self.norms = norms
         return self.deltas
 
+    def calibrate(self, inputs, eps, mech, seed, rows=128):
+        """a8: choose TF32X3 or FP32 per group from the bound on a masked sample (spl_choose_path).
+
+        The sample is the first ``rows`` rows of each group's input with a fresh mask drawn
+        under a stream id no online step uses.
+        """
+        for gi, g in enumerate(self.groups):
+            X = inputs[g.name][:rows].contiguous()
+            eta = torch.empty_like(X)
+            spl.spl_noise(eta, self.deltas[g.name], eps, mech, seed, stream_id=1000 + gi)
+            name, st_tc, st_fp = spl.spl_choose_path(X, eta, g.W, g.W_hi, g.W_lo)
+            self.paths[g.name] = name
+            self.calibration[g.name] = {"path": name, "tf32x3": st_tc, "fp32": st_fp, "rows": X.shape[0]}
+        return self.paths
+
+    def path_of(self, g, path, rows):
+        """The calibrated path for products of more than 8 rows under AUTO (the range where AUTO
+        weighs the tensor-core path); smaller products keep AUTO's streaming decode kernel."""
+        if path == "auto" and rows > 8:
+            return self.paths.get(g.name, path)
+        return path
+
     # ------------------------------------------------------------------ bank
     def allocate(self, M, draws, path="auto"):
         """Buffers for M tokens and a bank of ``draws`` corrections per group."""
@@ -136,7 +160,7 @@ class MaskedLayer:
                           offset=self.block_offset(g, cycle, 0), stream=stream)
             if timer:
                 timer("begin", "precompute")
-            spl.spl_precompute_noise_product(b["C"], b["eta"], g.W, g.W_hi, g.W_lo, path=path,
+            spl.spl_precompute_noise_product(b["C"], b["eta"], g.W, g.W_hi, g.W_lo, path=self.path_of(g, path, b["eta"].shape[0]),
                                              workspace=self.workspace, stream=stream)
             if timer:
                 timer("end", "precompute")
@@ -155,11 +179,20 @@ class MaskedLayer:
             if timer:
                 timer("begin", "masked_linear_unmask")
             spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M], g.W_hi, g.W_lo,
-                                         path=path, workspace=self.workspace, stream=stream)
+                                         path=self.path_of(g, path, M), workspace=self.workspace, stream=stream)
             if timer:
                 timer("end", "masked_linear_unmask")
             out[g.name] = b["Y"]
         return out
+
+    def bound_check(self, inputs, outs, eps, mech, seed, cycle, d):
+        """The paper's bound on the GPU over every output of an online step (per group)."""
+        res = {}
+        for gi, g in enumerate(self.groups):
+            eta = torch.empty((self.M, g.K), device=g.W.device)
+            spl.spl_noise(eta, self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=self.block_offset(g, cycle, d))
+            res[g.name] = spl.spl_bound_check(outs[g.name], inputs[g.name], self.bank[g.name]["xt"], eta, g.W)
+        return res
 
     def flops_per_step(self):
         """Algorithmic flops per online step: the masked product plus its share of the batched correction."""

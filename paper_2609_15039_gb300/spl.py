@@ -55,6 +55,11 @@ _SIGS = {
     "spl_delta_attention": (_D, [_P, _I64, _D]),
     "spl_delta_activation": (_D, [_P, _P, _I64, _I64, _D, _D]),
     "spl_spectral_norm": (_I, [ctypes.POINTER(ctypes.c_double), _P, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_bound_check": (_I, [ctypes.POINTER(ctypes.c_double), _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
+    "spl_choose_path_workspace_bytes": (_SZ, [_I64, _I64, _I64]),
+    "spl_choose_path": (_I, [ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double),
+                             ctypes.POINTER(ctypes.c_double), _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
+    "spl_test_tc_wait_timeout": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _P]),
     "spl_get_device_status": (_I, [_P]),
     "spl_launch_count": (ctypes.c_uint64, []),
     "spl_status_string": (ctypes.c_char_p, [_I]),
@@ -250,6 +255,54 @@ def spl_spectral_norm(W, iters=100, workspace=None, stream=None):
     _check(lib().spl_spectral_norm(ctypes.byref(out), _dev(W, "W"), N, K, int(iters), wsp, wsb, _stream(stream)),
            "spl_spectral_norm")
     return out.value
+
+
+BOUND_STATS = ("max_err_over_hard", "max_err_over_log", "log_violations", "sum_err", "sum_log_bound",
+               "sum_hard_bound", "elements", "max_abs_ref", "max_err")
+
+
+def _stats_dict(arr):
+    d = {k: float(v) for k, v in zip(BOUND_STATS, arr)}
+    n = max(d["elements"], 1.0)
+    d["violation_pct"] = 100.0 * d["log_violations"] / n
+    d["mean_err"] = d["sum_err"] / n
+    d["mean_log_bound"] = d["sum_log_bound"] / n
+    d["log_bound_over_err"] = d["sum_log_bound"] / d["sum_err"] if d["sum_err"] > 0 else float("inf")
+    return d
+
+
+def spl_bound_check(Y, X, Xt, Nz, W, stream=None):
+    """The paper's bound on the GPU for every row of Y; returns a dict of statistics."""
+    rows, K = _rows_cols(X)
+    N = W.shape[0]
+    stats = (ctypes.c_double * 9)()
+    ws = workspace(256, X.device)
+    _check(lib().spl_bound_check(stats, _dev(Y, "Y"), _dev(X, "X"), _dev(Xt, "Xt"), _dev(Nz, "Nz"), _dev(W, "W"),
+                                 rows, K, N, _dev(ws, "workspace"), 256, _stream(stream)), "spl_bound_check")
+    return _stats_dict(stats)
+
+
+def spl_choose_path(X, Nz, W, W_hi=None, W_lo=None, stream=None):
+    """a8: returns (chosen path name, stats of TF32X3, stats of FP32) for the sample X + Nz."""
+    rows, K = _rows_cols(X)
+    N = W.shape[0]
+    nbytes = int(lib().spl_choose_path_workspace_bytes(rows, K, N))
+    ws = workspace(nbytes, X.device)
+    chosen = ctypes.c_int(0)
+    a = (ctypes.c_double * 9)()
+    b = (ctypes.c_double * 9)()
+    _check(lib().spl_choose_path(ctypes.byref(chosen), a, b, _dev(X, "X"), _dev(Nz, "Nz"), _dev(W, "W"),
+                                 _dev(W_hi, "W_hi"), _dev(W_lo, "W_lo"), rows, K, N, _dev(ws, "workspace"), nbytes,
+                                 _stream(stream)), "spl_choose_path")
+    name = {SPL_PATH_TF32X3: "tf32x3", SPL_PATH_FP32: "fp32"}.get(chosen.value, str(chosen.value))
+    return name, _stats_dict(a), _stats_dict(b)
+
+
+def spl_test_tc_wait_timeout(out, A, W, W_hi, W_lo, stream=None):
+    M, K = _rows_cols(A)
+    N = W.shape[0]
+    _check(lib().spl_test_tc_wait_timeout(_dev(out, "out"), _dev(A, "A"), _dev(W, "W"), _dev(W_hi, "W_hi"),
+                                          _dev(W_lo, "W_lo"), M, K, N, _stream(stream)), "spl_test_tc_wait_timeout")
 
 
 def spl_launch_count():

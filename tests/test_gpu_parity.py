@@ -237,6 +237,49 @@ def test_empty_reduction(spl):
     assert torch.equal(Y, -C)
 
 
+# ---------------------------------------------------------- a8: bound on the GPU, path choice
+def test_bound_check_matches_oracle(spl):
+    M, K, N = 24, 1028, 300
+    X = wl.activations(M, K, seed=3).numpy()
+    eta = philox.noise((M, K), 50.0, 1.0, "gaussian", 9)
+    Xt = linear.mask(X, eta)
+    W, Wd, hi, lo = _weights(spl, N, K, seed=4)
+    C = torch.empty((M, N), device="cuda")
+    Y = torch.empty((M, N), device="cuda")
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp32"))
+    spl.spl_precompute_noise_product(C, dev(eta), Wd, path="fp32", workspace=ws)
+    spl.spl_masked_linear_unmask(Y, dev(Xt), Wd, C, path="fp32", workspace=ws)
+    got = spl.spl_bound_check(Y, dev(X), dev(Xt), dev(eta), Wd)
+    S = linear.abs_products(X, Xt, eta, W)
+    err = np.abs(f64(Y) - linear.reference_output(X, W))
+    hard, logb = bounds.hard_bound(*S, K), bounds.log_bound(*S, K)
+    assert got["elements"] == M * N
+    assert got["max_err_over_hard"] == pytest.approx(float(np.max(err / hard)), rel=1e-9)
+    assert got["max_err_over_log"] == pytest.approx(float(np.max(err / logb)), rel=1e-9)
+    assert abs(got["log_violations"] - float(np.sum(err > logb))) <= 1
+    assert got["sum_err"] == pytest.approx(float(err.sum()), rel=1e-9)
+    assert got["sum_log_bound"] == pytest.approx(float(logb.sum()), rel=1e-12)
+    assert got["sum_hard_bound"] == pytest.approx(float(hard.sum()), rel=1e-12)
+    assert got["max_abs_ref"] == pytest.approx(float(np.max(np.abs(linear.reference_output(X, W)))), rel=1e-12)
+
+
+@pytest.mark.parametrize("K,N", [(3072, 3072), (8, 64)])
+def test_choose_path_follows_its_rule(spl, K, N):
+    rows = 128
+    X = dev(wl.activations(rows, K, seed=5).numpy())
+    eta = torch.empty((rows, K), device="cuda")
+    spl.spl_noise(eta, 2 * 3072 ** 0.75, 1.0, "gaussian", seed=6)
+    W, Wd, hi, lo = _weights(spl, N, K, seed=7)
+    name, st_tc, st_fp = spl.spl_choose_path(X, eta, Wd, hi, lo)
+    rule = (st_tc["max_err_over_hard"] <= 1.0
+            and st_tc["log_violations"] <= st_fp["log_violations"] + 0.01 * st_tc["elements"]
+            and st_tc["sum_err"] <= 1.5 * st_fp["sum_err"] + 1e-300)
+    assert name == ("tf32x3" if rule else "fp32")
+    assert st_fp["max_err_over_hard"] <= 1.0
+    if K >= 64:
+        assert name == "tf32x3"  # the three-product split stays inside the bound at Llama sizes
+
+
 # ---------------------------------------------------------- a1: ||W||_2
 def test_spectral_norm_matches_svd(spl):
     W = wl.weight(300, 200, seed=9).numpy()
