@@ -144,6 +144,23 @@ spl_status spl_precompute_noise_product(float* C, const float* Nz, const float* 
                                         int64_t N, spl_path path, void* workspace,
                                         size_t workspace_bytes, cudaStream_t stream);
 
+/* ---- a4, summed in the masked product's order ---------------------------
+ * C = Nz W^T like spl_precompute_noise_product, but every output element is
+ * summed in exactly the order spl_masked_linear_unmask uses for a call of
+ * `order_rows` rows with the same K, N, path and device: the same kernel, the
+ * same K-split boundaries and the same order of the cross-CTA reduction.
+ * When the noise dominates the input (x~ ~ eta), the rounding errors of
+ * fl(x~ W^T) and fl(eta W^T) then largely cancel in the unmask, so the
+ * recovered W x sits far inside the bound of Thm. 4.  Rows of Nz may stack
+ * several draws (a bank).  If the masked call's order cannot be reproduced
+ * (a launch whose tiles use different splits), this is spl_precompute_noise_product.
+ * Workspace: spl_precompute_matched_workspace_bytes(M, K, N, order_rows, path). */
+size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows, spl_path path);
+spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const float* W,
+                                                const float* W_hi, const float* W_lo, int64_t M, int64_t K,
+                                                int64_t N, int64_t order_rows, spl_path path, void* workspace,
+                                                size_t workspace_bytes, cudaStream_t stream);
+
 /* ---- a6: unmask -------------------------------------------------------
  * Y = fl32(Yt - C) elementwise (Eq. add-and-then-subtract).  Y may alias Yt. */
 spl_status spl_unmask(float* Y, const float* Yt, const float* C, int64_t rows, int64_t cols,

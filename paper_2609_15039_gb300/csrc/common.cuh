@@ -74,6 +74,9 @@ Plan plan_simt(int64_t M, int64_t K, int64_t N, int sms);
 Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms);
 
 spl_status run_gemv(const LinearArgs& a, const Plan& p);
+int64_t gemv_max_ks(int64_t M);                           // largest K-slice the decode kernel stages for M rows
+int tc_uniform_splits(int64_t M, int64_t K, int64_t N);    // K-split of a one-launch TF32X3 call, 0 if mixed
+spl_status run_tc_splits(const LinearArgs& a, int splits); // TF32X3 with the same K-split on every tile
 spl_status run_simt(const LinearArgs& a, const Plan& p);
 spl_status run_tc(const LinearArgs& a, const Plan& p);
 

@@ -587,7 +587,7 @@ Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
   return p;  // no workspace: partials are reduced through distributed shared memory
 }
 
-spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock) {
+spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock, int forced_splits = 0) {
   const int cc = device_cc();
   if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
   if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
@@ -611,7 +611,9 @@ spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock) {
     attr_set[dev] = true;
   }
   const int m_tiles = (int)ceil_div(a.M, BM);
-  const TcLaunches t = tc_launches(a.M, a.K, a.N, device_sm_count());
+  const TcLaunches t = forced_splits > 0
+                           ? TcLaunches{0, ceil_div(a.M, BM) * ceil_div(a.N, BN), forced_splits}
+                           : tc_launches(a.M, a.K, a.N, device_sm_count());
   auto launch = [&](int64_t tiles, int64_t base, int splits) -> spl_status {
     if (tiles <= 0) return SPL_OK;
     const int64_t kps = round_up(ceil_div(a.K, splits), BK);
@@ -639,6 +641,20 @@ spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock) {
 }
 
 spl_status run_tc(const LinearArgs& a, const Plan& p) { return run_tc_impl(a, p, -1); }
+
+int tc_uniform_splits(int64_t M, int64_t K, int64_t N) {
+  const TcLaunches t = tc_launches(M, K, N, device_sm_count());
+  return t.full_tiles > 0 && t.rest_tiles > 0 ? 0 : (t.full_tiles > 0 ? 1 : t.rest_splits);
+}
+
+spl_status run_tc_splits(const LinearArgs& a, int splits) {
+  if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
+  Plan p{};
+  p.kernel = kKernelTc;
+  p.splits = splits;
+  p.k_per_split = round_up(ceil_div(a.K, splits), BK);
+  return run_tc_impl(a, p, -1, splits);
+}
 
 }  // namespace spl
 

@@ -165,6 +165,8 @@ spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int*
 
 }  // namespace
 
+int64_t gemv_max_ks(int64_t M) { return (SMEM_FLOATS / padded_m(M)) / 128 * 128; }
+
 Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
   Plan p{};
   p.kernel = kKernelGemv;

@@ -70,10 +70,100 @@ spl_status run_linear(float* out, const float* a, const float* W, const float* W
   }
 }
 
+// The plan a correction of M rows must follow so that every output element is summed in the
+// order a masked product of `order_rows` rows uses (same kernel, same K-split boundaries, same
+// order of the cross-CTA reduction).  ok = false when that order cannot be reproduced.
+struct MatchedPlan {
+  bool ok;
+  int kernel;
+  int splits;
+  int64_t k_per_split;
+  int64_t chunk_rows;  // decode kernel: rows per launch (<= 16)
+  size_t ws;           // workspace bytes
+};
+
+MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, spl_path resolved) {
+  MatchedPlan mp{false, 0, 1, K, M, 0};
+  const Plan online = make_plan(order_rows, K, N, resolved);
+  mp.kernel = online.kernel;
+  if (online.kernel == kKernelTc) {
+    const int s = tc_uniform_splits(order_rows, K, N);
+    if (s <= 0) return mp;
+    mp.splits = s;
+    mp.ok = true;
+    return mp;  // no workspace
+  }
+  mp.splits = online.splits;
+  mp.k_per_split = online.k_per_split;
+  if (online.kernel == kKernelGemv) {
+    mp.chunk_rows = std::min<int64_t>(M, kGemvMaxM);
+    if (mp.k_per_split > gemv_max_ks(mp.chunk_rows)) return mp;
+    if (mp.splits > 1) mp.ws = kCounterBytes + (size_t)round_up((int64_t)mp.splits * mp.chunk_rows * N * 4, 256);
+  } else {
+    if (mp.splits > 1) mp.ws = kCounterBytes + (size_t)round_up((int64_t)mp.splits * M * N * 4, 256);
+  }
+  mp.ok = true;
+  return mp;
+}
+
 }  // namespace
 }  // namespace spl
 
 using namespace spl;
+
+extern "C" size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows,
+                                                         spl_path path) {
+  if (M <= 0 || K <= 0 || N <= 0 || order_rows <= 0) return 0;
+  size_t need = 0;
+  const spl_path paths[2] = {SPL_PATH_FP32, SPL_PATH_TF32X3};
+  for (spl_path p : paths) {
+    if (path != SPL_PATH_AUTO && path != p) continue;
+    const MatchedPlan mp = matched_plan(M, K, N, order_rows, p);
+    need = std::max(need, mp.ok ? mp.ws : make_plan(M, K, N, p).total());
+  }
+  return need;
+}
+
+extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const float* W,
+                                                           const float* W_hi, const float* W_lo, int64_t M, int64_t K,
+                                                           int64_t N, int64_t order_rows, spl_path path,
+                                                           void* workspace, size_t workspace_bytes,
+                                                           cudaStream_t stream) {
+  if (order_rows <= 0) return SPL_EINVAL;
+  if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
+  if (path != SPL_PATH_AUTO && path != SPL_PATH_TF32X3 && path != SPL_PATH_FP32) return SPL_EINVAL;
+  if (M == 0 || N == 0 || K == 0)
+    return run_linear(C, Nz, W, W_hi, W_lo, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
+  if (!C || !Nz || !W) return SPL_EINVAL;
+  if ((K & 3) != 0) return SPL_EALIGN;
+  if (!aligned16(C) || !aligned16(Nz) || !aligned16(W)) return SPL_EALIGN;
+  if ((W_hi && !aligned16(W_hi)) || (W_lo && !aligned16(W_lo))) return SPL_EALIGN;
+  const spl_path resolved = resolve(order_rows, K, path, W_hi && W_lo);
+  if (resolved == SPL_PATH_TF32X3 && (!W_hi || !W_lo || !tc_capable())) return SPL_EUNSUPPORTED;
+  const MatchedPlan mp = matched_plan(M, K, N, order_rows, resolved);
+  if (!mp.ok)  // the masked call's order cannot be reproduced: plain correction
+    return run_linear(C, Nz, W, W_hi, W_lo, nullptr, false, M, K, N, resolved, workspace, workspace_bytes, stream);
+  if (mp.ws > 0 && (!workspace || workspace_bytes < mp.ws)) return SPL_EWORKSPACE;
+  if (workspace && !aligned16(workspace)) return SPL_EALIGN;
+  LinearArgs args{C, Nz, W, W_hi, W_lo, nullptr, M, K, N, workspace, workspace_bytes, stream};
+  if (mp.kernel == kKernelTc) return run_tc_splits(args, mp.splits);
+  Plan p{};
+  p.kernel = mp.kernel;
+  p.splits = mp.splits;
+  p.k_per_split = mp.k_per_split;
+  if (mp.kernel == kKernelSimt) {
+    p.ws_partials = mp.splits > 1 ? (size_t)round_up((int64_t)mp.splits * M * N * 4, 256) : 0;
+    return run_simt(args, p);
+  }
+  for (int64_t r0 = 0; r0 < M; r0 += mp.chunk_rows) {  // decode kernel: at most 16 rows per launch
+    const int64_t rows = std::min<int64_t>(mp.chunk_rows, M - r0);
+    LinearArgs ca{C + r0 * N, Nz + r0 * K, W, W_hi, W_lo, nullptr, rows, K, N, workspace, workspace_bytes, stream};
+    p.ws_partials = mp.splits > 1 ? (size_t)round_up((int64_t)mp.splits * rows * N * 4, 256) : 0;
+    const spl_status st = run_gemv(ca, p);
+    if (st != SPL_OK) return st;
+  }
+  return SPL_OK;
+}
 
 extern "C" spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path) {
   (void)N;

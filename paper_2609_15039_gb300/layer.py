@@ -10,7 +10,9 @@ consumed once.  This module keeps that structure, GB300 style:
   its output columns are the individual projections;
 * the bank holds only corrections.  ``refill`` draws D masks per group in
   one pass (a2) and computes their corrections C = eta W^T as one product of
-  D*M rows (a4, "precomputed in a batch");
+  D*M rows (a4, "precomputed in a batch"), each output summed in the same
+  order as the online product of M rows, so the rounding errors of the two
+  products cancel in the unmask;
 * an ``online`` step regenerates its mask from the same Philox counters
   (seed, group stream, block offset of draw d) instead of reading it back,
   masks the input (a3) and runs the masked product with the unmask fused
@@ -134,7 +136,7 @@ class MaskedLayer:
         need = 0
         for g in self.groups:
             need = max(need, spl.spl_linear_workspace_bytes(M, g.K, g.N, path),
-                       spl.spl_linear_workspace_bytes(draws * M, g.K, g.N, path))
+                       spl.spl_precompute_matched_workspace_bytes(draws * M, g.K, g.N, M, path))
         if self.workspace is None or self.workspace.numel() < need:
             self.workspace = spl.workspace(need, dev)
         self.M, self.draws = M, draws
@@ -160,8 +162,10 @@ class MaskedLayer:
                           offset=self.block_offset(g, cycle, 0), stream=stream)
             if timer:
                 timer("begin", "precompute")
-            spl.spl_precompute_noise_product(b["C"], b["eta"], g.W, g.W_hi, g.W_lo, path=self.path_of(g, path, b["eta"].shape[0]),
-                                             workspace=self.workspace, stream=stream)
+            # summed in the order the online product of M rows uses, so their rounding cancels
+            spl.spl_precompute_noise_product_matched(b["C"], b["eta"], g.W, self.M, g.W_hi, g.W_lo,
+                                                     path=self.path_of(g, path, self.M), workspace=self.workspace,
+                                                     stream=stream)
             if timer:
                 timer("end", "precompute")
 

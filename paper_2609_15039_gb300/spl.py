@@ -48,6 +48,8 @@ _SIGS = {
     "spl_linear_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I]),
     "spl_masked_linear": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_precompute_noise_product": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_precompute_matched_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I64, _I]),
+    "spl_precompute_noise_product_matched": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_masked_linear_unmask": (_I, [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_masked_linear_unmask_noalloc": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P]),
@@ -200,6 +202,22 @@ def spl_masked_linear(Yt, Xt, W, W_hi=None, W_lo=None, path="auto", workspace=No
 def spl_precompute_noise_product(C, Nz, W, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
     _linear(lib().spl_precompute_noise_product, "spl_precompute_noise_product", C, Nz, W, W_hi, W_lo, None, path,
             workspace, stream)
+
+
+def spl_precompute_matched_workspace_bytes(M, K, N, order_rows, path="auto"):
+    return int(lib().spl_precompute_matched_workspace_bytes(M, K, N, order_rows, _path(path)))
+
+
+def spl_precompute_noise_product_matched(C, Nz, W, order_rows, W_hi=None, W_lo=None, path="auto", workspace=None,
+                                         stream=None):
+    M, K = _rows_cols(Nz)
+    N = W.shape[0]
+    if W.shape[-1] != K or C.numel() != M * N:
+        raise ValueError("spl_precompute_noise_product_matched: shape mismatch")
+    wsp, wsb = _ws(workspace)
+    _check(lib().spl_precompute_noise_product_matched(_dev(C, "C"), _dev(Nz, "Nz"), _dev(W, "W"), _dev(W_hi, "W_hi"),
+                                                      _dev(W_lo, "W_lo"), M, K, N, int(order_rows), _path(path), wsp,
+                                                      wsb, _stream(stream)), "spl_precompute_noise_product_matched")
 
 
 def spl_unmask(Y, Yt, C, stream=None):

@@ -237,6 +237,44 @@ def test_empty_reduction(spl):
     assert torch.equal(Y, -C)
 
 
+@pytest.mark.parametrize("M,K,N,path", [(128, 3072, 3072, "tf32x3"), (128, 3072, 3072, "fp32"),
+                                         (1, 3072, 3072, "fp32"), (128, 8192, 3072, "tf32x3")])
+def test_matched_correction_cancels_rounding(spl, M, K, N, path):
+    """A bank of 8 corrections summed in the online product's order: the same values up to
+    rounding, and on the tensor-core path a much smaller recovered error than a correction
+    computed with its own plan for 8 x M rows."""
+    draws, b = 8, 1443.0
+    W, Wd, hi, lo = _weights(spl, N, K, seed=K + N)
+    X = wl.activations(M, K, seed=21).numpy()
+    eta = philox.noise((draws * M, K), b, 1.0, "gaussian", seed=22)
+    Nd = dev(eta)
+    C_plain, C_matched = torch.empty((draws * M, N), device="cuda"), torch.empty((draws * M, N), device="cuda")
+    ws = spl.workspace(max(spl.spl_linear_workspace_bytes(draws * M, K, N, path),
+                           spl.spl_precompute_matched_workspace_bytes(draws * M, K, N, M, path),
+                           spl.spl_linear_workspace_bytes(M, K, N, path)))
+    spl.spl_precompute_noise_product(C_plain, Nd, Wd, hi, lo, path=path, workspace=ws)
+    spl.spl_precompute_noise_product_matched(C_matched, Nd, Wd, M, hi, lo, path=path, workspace=ws)
+    assert_product_close(f32(C_matched), eta, W, path, what="matched correction")
+    d = draws - 1
+    Xt = linear.mask(X, eta[d * M:(d + 1) * M])
+    errs = {}
+    for name, Cb in (("plain", C_plain), ("matched", C_matched)):
+        Y = torch.empty((M, N), device="cuda")
+        spl.spl_masked_linear_unmask(Y, dev(Xt), Wd, Cb[d * M:(d + 1) * M].contiguous(), hi, lo, path=path,
+                                     workspace=ws)
+        err = np.abs(f64(Y) - linear.reference_output(X, W))
+        S = linear.abs_products(X, Xt, eta[d * M:(d + 1) * M], W)
+        assert np.all(err <= bounds.hard_bound(*S, K)), name
+        errs[name] = float(err.mean())
+    if path == "tf32x3":
+        # the tensor-core bank at 8x the rows uses another K split and cluster order; matched, the
+        # errors of fl(x~ W^T) and fl(eta W^T) cancel
+        assert errs["matched"] * 3 < errs["plain"], errs
+    else:
+        # FMA chains in ascending k already keep the two roundings correlated; matching never hurts
+        assert errs["matched"] <= errs["plain"] * 1.1, errs
+
+
 # ---------------------------------------------------------- a8: bound on the GPU, path choice
 def test_bound_check_matches_oracle(spl):
     M, K, N = 24, 1028, 300
