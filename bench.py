@@ -8,8 +8,10 @@ then runs the masked product with the unmask fused into its epilogue
 (Y = X~ W^T - C).  Every 8 steps the correction bank is refilled: 8 masks
 per group are drawn and their corrections C = eta W^T computed as one
 product of 8 x 128 rows ("precomputed in a batch"), so each step carries an
-eighth of that work.  The weights (1.2 GB per layer incl. the TF32 split)
-are larger than L2, so no step reuses L2-resident weights.
+eighth of that work.  The weights (0.4 GB per layer in fp32, plus the TF32
+and fp16 splits) are larger than L2, so no step reuses L2-resident weights.
+The arithmetic path of each input group is chosen by the bound check on a
+masked sample (spl_choose_path) unless --path fixes it.
 
 Prints one JSON line.  ``--impl reference`` times the fp64 CPU oracle on a
 bounded sample of the same workload instead.
@@ -217,13 +219,13 @@ def main():
 
     events = []  # (kind, begin, end) around every product call
 
-    def timer(phase, kind):
+    def timer(phase, kind, group):
         e = torch.cuda.Event(enable_timing=True)
         e.record(stream)
         if phase == "begin":
-            events.append([kind, e, None])
+            events.append([kind, group, e, None])
         else:
-            events[-1][2] = e
+            events[-1][3] = e
 
     def step(s, use_timer=False, x=inputs):
         cycle, d = divmod(s, DRAWS)
@@ -266,31 +268,44 @@ def main():
 
     flops_step = layer.flops_per_step()
     value = world * flops_step / (ms * 1e-3) / 1e12
-    resolved = spl.spl_resolve_path(M, model.d_model, model.d_model, args.path)
-    path_name = {1: "tf32x3", 2: "fp32"}.get(resolved, str(resolved))
+    group_paths = {g.name: spl.PATH_NAMES[spl.spl_resolve_path(M, g.K, g.N, layer.path_of(g, args.path, M))]
+                   for g in layer.groups}
+    path_name = "+".join(sorted(set(group_paths.values())))
 
-    # roofline of the dominant kernel: the product calls (tcgen05 TF32X3 GEMM + its A split / reductions)
+    # roofline of the dominant kernel: the product calls (tcgen05 GEMM + its row exponents / reductions)
     pk = peaks()
-    by_kind = {}
-    for kind, b, e in events:
+    by_kind, by_group = {}, {}
+    for kind, group, b, e in events:
         by_kind.setdefault(kind, []).append(b.elapsed_time(e))
+        by_group.setdefault((kind, group), []).append(b.elapsed_time(e))
     prod_ms = sum(sum(v) for v in by_kind.values())
     achieved = flops_step * args.steps / (prod_ms * 1e-3) / 1e12
-    if path_name == "tf32x3":
-        peak = pk["bf16_tflops_sustained"] * TF32_OVER_BF16 / 3.0
-        peak_note = "measured sustained bf16 x nominal tf32/bf16 (1.1/2.25) / 3 products per term"
-    else:
-        peak = 152 * 128 * 2 * 2.07e9 / 1e12
-        peak_note = "fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2.07 GHz (derived)"
+    path_peak = {  # algorithmic flops (one product per term) per second at each path's instruction peak
+        "fp16x3": pk["bf16_tflops_sustained"] / 3.0,
+        "tf32x3": pk["bf16_tflops_sustained"] * TF32_OVER_BF16 / 3.0,
+        "fp32": 152 * 128 * 2 * 2.07e9 / 1e12,
+    }
+    # flop-weighted: the time the step's products would take with every group at its path's peak
+    t_peak = sum(2 * 2 * M * g.K * g.N / path_peak[group_paths[g.name]] for g in layer.groups)
+    peak = flops_step / t_peak
+    peak_note = ("per group: fp16x3 = measured sustained bf16 (fp16 runs at the bf16 rate) / 3 products per term; "
+                 "tf32x3 = that x nominal tf32/bf16 (1.1/2.25); fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2.07 GHz "
+                 "(derived); flop-weighted over the groups")
     per_kind = {}
     for kind, v in by_kind.items():
         rows = DRAWS * M if kind == "precompute" else M
         f = sum(2 * rows * g.K * g.N for g in layer.groups) * len(v) / len(layer.groups)
         per_kind[kind] = {"calls": len(v), "avg_ms": sum(v) / len(v), "tflops": f / (sum(v) * 1e-3) / 1e12,
                           "rows": rows}
+        for g in layer.groups:
+            t = by_group[(kind, g.name)]
+            avg = sum(t) / len(t)
+            per_kind[kind][g.name] = {"avg_us": 1e3 * avg, "tflops": 2 * rows * g.K * g.N / (avg * 1e-3) / 1e12,
+                                      "path": group_paths[g.name]}
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": None,
                 "kernel": "tc_gemm_kernel product calls (bank corrections at 1024 rows + online masked products)",
+                "group_paths": group_paths,
                 "share_of_step": prod_ms / (ms * args.steps), "per_call": per_kind,
                 "peak_source": pk["source"], "peak_note": peak_note}
 
@@ -346,9 +361,9 @@ def main():
         result["e2e"] = e2e
     if layer.calibration:
         result["path_choice"] = {g: {"path": c["path"],
-                                     "tf32x3_max_err_over_hard": c["tf32x3"]["max_err_over_hard"],
-                                     "fp32_max_err_over_hard": c["fp32"]["max_err_over_hard"],
-                                     "tf32x3_mean_err": c["tf32x3"]["mean_err"], "fp32_mean_err": c["fp32"]["mean_err"]}
+                                     **{f"{p}_max_err_over_hard": c[p]["max_err_over_hard"]
+                                        for p in ("fp32", "tf32x3", "fp16x3")},
+                                     **{f"{p}_mean_err": c[p]["mean_err"] for p in ("fp32", "tf32x3", "fp16x3")}}
                                  for g, c in layer.calibration.items()}
     # the paper's bound over every output of one more online step, evaluated on the GPU in fp64
     cycle, d = divmod(s, DRAWS)

@@ -57,9 +57,30 @@ typedef enum spl_mech { SPL_MECH_LAPLACE = 0, SPL_MECH_GAUSSIAN = 1 } spl_mech;
  *            rounding, sequential summation per output).
  *  TF32X3 -- tcgen05 tensor cores, three TF32 products per term
  *            (hi*hi + hi*lo + lo*hi, fp32 accumulation in TMEM); needs the
- *            weight split of spl_split_tf32.
+ *            weight split of spl_split_tf32 (8 bytes per weight).
+ *  FP16X3 -- the same three products in fp16 (kind::f16, twice the TF32 rate)
+ *            on rows scaled by powers of two, undone exactly in the epilogue;
+ *            needs the weight split of spl_split_fp16 (4 bytes per weight)
+ *            and K % 8 == 0.
  *  AUTO   -- the library's choice (spl_resolve_path). */
-typedef enum spl_path { SPL_PATH_AUTO = 0, SPL_PATH_TF32X3 = 1, SPL_PATH_FP32 = 2 } spl_path;
+typedef enum spl_path {
+  SPL_PATH_AUTO = 0,
+  SPL_PATH_TF32X3 = 1,
+  SPL_PATH_FP32 = 2,
+  SPL_PATH_FP16X3 = 3
+} spl_path;
+
+/* A weight W[N, K] (fp32, K contiguous) and the splits the tensor-core paths
+ * read.  Device pointers owned by the caller; any split may be NULL (the
+ * paths that need it then report SPL_EUNSUPPORTED and AUTO skips them). */
+typedef struct spl_weight {
+  const float* w;          /* [N, K] fp32, required */
+  const float* tf32_hi;    /* [N, K] from spl_split_tf32 */
+  const float* tf32_lo;
+  const uint16_t* f16_hi;  /* [N, K] binary16 bit patterns from spl_split_fp16 */
+  const uint16_t* f16_lo;
+  const int32_t* f16_exp;  /* [N] power-of-two row exponents of the fp16 split */
+} spl_weight;
 
 /* Philox4x32-10 stream (Salmon et al., SC'11).  Element e of a flat tensor
  * uses lane e % 4 of block j = e / 4 + offset (64-bit, wrapping); the
@@ -108,40 +129,49 @@ spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, int64_t rows,
  * (exact in fp32).  Done once per weight; hi and lo are [count] like src. */
 spl_status spl_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream);
 
+/* hi = fp16(src 2^e_r), lo = fp16(src 2^e_r - hi) per row r, with the power of
+ * two e_r (row_exp[r]) that brings the row's largest |entry| into [2^14, 2^15)
+ * (0 for an all-zero row); hi + lo = src 2^e_r to about 2^-22 relative.  Done
+ * once per weight; hi and lo are [rows, cols] binary16 bit patterns.
+ * cols % 8 == 0 (EALIGN otherwise). */
+spl_status spl_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows,
+                          int64_t cols, cudaStream_t stream);
+
 /* Path that AUTO resolves to for an M x K x N product on the current device,
- * assuming the weight split is passed (FP32 or TF32X3).  An explicit path
- * is returned unchanged. */
+ * assuming every split is passed: FP32 up to 8 rows (the streaming decode
+ * kernel), else FP16X3 when K % 8 == 0, else TF32X3 (K >= 64, tcgen05 device),
+ * else FP32.  An explicit path is returned unchanged. */
 spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path);
 
 /* Bytes of device workspace the three product calls below need for this
- * problem on the current device (0 if none; for AUTO the larger of the two
+ * problem on the current device (0 if none; for AUTO the largest over the
  * paths).  Layout: the first 64 KiB hold the decode kernel's arrival
- * counters, then split-K partial sums and, for TF32X3, the TF32 split of the
- * left operand.  It must be zero-filled before its first use; every call that
+ * counters, then either split-K partial sums (FP32 kernels) or, for FP16X3,
+ * one power-of-two exponent per row of the left operand (TF32X3 needs none:
+ * it reduces its K-split inside a thread-block cluster).  It must be
+ * zero-filled before its first use; every call that
  * returns SPL_OK leaves the counters at zero again, so one workspace (sized
  * for the largest call) serves calls of any shape and path.  Calls that can
  * run concurrently must not share a workspace. */
 size_t spl_linear_workspace_bytes(int64_t M, int64_t K, int64_t N, spl_path path);
 
 /* ---- a5: masked product -----------------------------------------------
- * Yt[M, N] = Xt[M, K] W[N, K]^T, the GPU's r = W x~ (Sec. 5.1).
- * W_hi / W_lo are the spl_split_tf32 halves of W (needed for TF32X3; may be
- * NULL for FP32, in which case AUTO resolves to FP32).
- * Errors: EINVAL for NULL operands, EALIGN, EUNSUPPORTED for TF32X3 without
- * W_hi/W_lo or on a device that is not sm_103/sm_100, EWORKSPACE if the
- * workspace is too small, ETIMEOUT never (waits are reported through
- * spl_get_device_status). */
-spl_status spl_masked_linear(float* Yt, const float* Xt, const float* W, const float* W_hi,
-                             const float* W_lo, int64_t M, int64_t K, int64_t N, spl_path path,
-                             void* workspace, size_t workspace_bytes, cudaStream_t stream);
+ * Yt[M, N] = Xt[M, K] W[N, K]^T, the GPU's r = W x~ (Sec. 5.1).  W carries the
+ * fp32 weight and whichever splits exist; AUTO uses only the ones present.
+ * Errors: EINVAL for NULL operands, EALIGN, EUNSUPPORTED for a tensor-core path
+ * whose split is missing or on a device that is not sm_103/sm_100, EALIGN for
+ * FP16X3 with K % 8 != 0, EWORKSPACE if the workspace is too small; a bounded
+ * device wait that runs out is reported by spl_get_device_status. */
+spl_status spl_masked_linear(float* Yt, const float* Xt, const spl_weight* W, int64_t M, int64_t K,
+                             int64_t N, spl_path path, void* workspace, size_t workspace_bytes,
+                             cudaStream_t stream);
 
 /* ---- a4: correction precompute ----------------------------------------
  * C[M, N] = Nz[M, K] W[N, K]^T, the correction W eta (Sec. 5.2).  Several
  * noise draws may be stacked along M (rows are independent).  Same operands,
  * paths and errors as spl_masked_linear. */
-spl_status spl_precompute_noise_product(float* C, const float* Nz, const float* W,
-                                        const float* W_hi, const float* W_lo, int64_t M, int64_t K,
-                                        int64_t N, spl_path path, void* workspace,
+spl_status spl_precompute_noise_product(float* C, const float* Nz, const spl_weight* W, int64_t M,
+                                        int64_t K, int64_t N, spl_path path, void* workspace,
                                         size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- a4, summed in the masked product's order ---------------------------
@@ -156,10 +186,9 @@ spl_status spl_precompute_noise_product(float* C, const float* Nz, const float* 
  * (a launch whose tiles use different splits), this is spl_precompute_noise_product.
  * Workspace: spl_precompute_matched_workspace_bytes(M, K, N, order_rows, path). */
 size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows, spl_path path);
-spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const float* W,
-                                                const float* W_hi, const float* W_lo, int64_t M, int64_t K,
-                                                int64_t N, int64_t order_rows, spl_path path, void* workspace,
-                                                size_t workspace_bytes, cudaStream_t stream);
+spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const spl_weight* W, int64_t M,
+                                                int64_t K, int64_t N, int64_t order_rows, spl_path path,
+                                                void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- a6: unmask -------------------------------------------------------
  * Y = fl32(Yt - C) elementwise (Eq. add-and-then-subtract).  Y may alias Yt. */
@@ -171,9 +200,8 @@ spl_status spl_unmask(float* Y, const float* Yt, const float* C, int64_t rows, i
  * subtraction done in the product's epilogue.  M <= 16 runs the streaming
  * decode kernel (W read once at HBM rate, FP32).  Same operands and errors as
  * spl_masked_linear plus C. */
-spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const float* W, const float* W_hi,
-                                    const float* W_lo, const float* C, int64_t M, int64_t K,
-                                    int64_t N, spl_path path, void* workspace,
+spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const spl_weight* W, const float* C,
+                                    int64_t M, int64_t K, int64_t N, spl_path path, void* workspace,
                                     size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- a5 + a6 for decode, without allocation ---------------------------
@@ -223,14 +251,16 @@ spl_status spl_bound_check(double* stats, const float* Y, const float* X, const 
 size_t spl_choose_path_workspace_bytes(int64_t rows, int64_t K, int64_t N);
 
 /* a8: masks the sample X (+ Nz), computes the correction and the masked product with the
- * unmask on each path (FP32, and TF32X3 if W_hi/W_lo are given and the device has tcgen05),
- * checks both with spl_bound_check and sets *chosen to TF32X3 only if its max error over the
- * hard bound is <= 1 and its log-bound violations and summed error are no worse than FP32's
- * (within 1% of the elements and a factor 1.5), else FP32.  Both stats arrays (HOST,
- * SPL_BOUND_STATS each) are filled; an unavailable path reports +inf in [0].  Synchronises. */
-spl_status spl_choose_path(spl_path* chosen, double* stats_tf32x3, double* stats_fp32, const float* X,
-                           const float* Nz, const float* W, const float* W_hi, const float* W_lo, int64_t rows,
-                           int64_t K, int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+ * unmask on each path (FP32, and the tensor-core paths whose splits W carries, on a
+ * tcgen05 device), checks each with spl_bound_check and sets *chosen to the fastest
+ * tensor-core path (FP16X3, then TF32X3) whose max error over the hard bound is <= 1 and
+ * whose log-bound violations and summed error are no worse than FP32's (within 1% of the
+ * elements and a factor 1.5), else FP32.  stats (HOST) receives 3 x SPL_BOUND_STATS doubles
+ * in the order FP32, TF32X3, FP16X3; an unavailable path reports +inf in its [0].
+ * Synchronises. */
+spl_status spl_choose_path(spl_path* chosen, double* stats, const float* X, const float* Nz,
+                           const spl_weight* W, int64_t rows, int64_t K, int64_t N, void* workspace,
+                           size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- a1: noise scale ----------------------------------------------------
  * Global l2 sensitivities (Sec. 4.3), evaluated in fp64 on the host from
@@ -258,8 +288,8 @@ spl_status spl_spectral_norm(double* out, const float* W, int64_t N, int64_t K, 
  * the copies it did issue land, frees its tensor memory and returns.  The next
  * spl_get_device_status returns SPL_ETIMEOUT and the context stays usable.
  * `out` receives unspecified values. */
-spl_status spl_test_tc_wait_timeout(float* out, const float* A, const float* W, const float* W_hi,
-                                    const float* W_lo, int64_t M, int64_t K, int64_t N, cudaStream_t stream);
+spl_status spl_test_tc_wait_timeout(float* out, const float* A, const spl_weight* W, int64_t M, int64_t K,
+                                    int64_t N, cudaStream_t stream);
 
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last

@@ -11,9 +11,10 @@
 //   log  = gamma_{ceil(log2 K)+1} (S_x + S_xt + S_n) + u S_x          (Eq. fp-log-bound)
 // with u = 2^-24 and gamma_n = n u / (1 - n u) (Def. u-and-theta).
 //
-// spl_choose_path masks a sample, runs the correction and the masked product with each path,
-// checks both against the bound and picks TF32X3 only when it stays inside the hard bound
-// and its log-bound violations and mean error are no worse than FP32's.
+// spl_choose_path masks a sample, runs the correction and the masked product with each path
+// (FP32, TF32X3, FP16X3), checks each against the bound and picks a tensor-core path only
+// when it stays inside the hard bound and its log-bound violations and mean error are no
+// worse than FP32's; FP16X3 is tried first.
 
 #include <algorithm>
 #include <cmath>
@@ -113,21 +114,19 @@ extern "C" spl_status spl_bound_check(double* stats, const float* Y, const float
 extern "C" size_t spl_choose_path_workspace_bytes(int64_t rows, int64_t K, int64_t N) {
   if (rows <= 0 || K <= 0 || N <= 0) return 0;
   const size_t f = sizeof(float);
-  const size_t prod = std::max(spl_linear_workspace_bytes(rows, K, N, SPL_PATH_FP32),
-                               spl_linear_workspace_bytes(rows, K, N, SPL_PATH_TF32X3));
+  const size_t prod = spl_linear_workspace_bytes(rows, K, N, SPL_PATH_AUTO);  // every path
   // Xt [rows, K], C [rows, N], Y [rows, N], stats, then the product workspace
   return (size_t)round_up((int64_t)(rows * K * f), 256) + 2 * (size_t)round_up((int64_t)(rows * N * f), 256) + 256 +
          prod;
 }
 
-extern "C" spl_status spl_choose_path(spl_path* chosen, double* stats_tf32x3, double* stats_fp32, const float* X,
-                                      const float* Nz, const float* W, const float* W_hi, const float* W_lo,
-                                      int64_t rows, int64_t K, int64_t N, void* workspace, size_t workspace_bytes,
-                                      cudaStream_t stream) {
-  if (!chosen || !stats_tf32x3 || !stats_fp32) return SPL_EINVAL;
+extern "C" spl_status spl_choose_path(spl_path* chosen, double* stats, const float* X, const float* Nz,
+                                      const spl_weight* W, int64_t rows, int64_t K, int64_t N, void* workspace,
+                                      size_t workspace_bytes, cudaStream_t stream) {
+  if (!chosen || !stats) return SPL_EINVAL;
   *chosen = SPL_PATH_FP32;
   if (rows <= 0 || K <= 0 || N <= 0) return SPL_EINVAL;
-  if (!X || !Nz || !W) return SPL_EINVAL;
+  if (!X || !Nz || !W || !W->w) return SPL_EINVAL;
   const size_t need = spl_choose_path_workspace_bytes(rows, K, N);
   if (!workspace || workspace_bytes < need) return SPL_EWORKSPACE;
   char* ws = static_cast<char*>(workspace);
@@ -143,31 +142,34 @@ extern "C" spl_status spl_choose_path(spl_path* chosen, double* stats_tf32x3, do
   const size_t pws_bytes = workspace_bytes - (size_t)(ws - static_cast<char*>(workspace));
   spl_status st = spl_mask(xt, X, Nz, rows, K, stream);
   if (st != SPL_OK) return st;
-  const bool tc = W_hi && W_lo && spl_resolve_path(rows, K, N, SPL_PATH_TF32X3) == SPL_PATH_TF32X3;
-  for (int pass = 0; pass < 2; ++pass) {
-    const spl_path path = pass == 0 ? SPL_PATH_FP32 : SPL_PATH_TF32X3;
-    double* out = pass == 0 ? stats_fp32 : stats_tf32x3;
-    if (path == SPL_PATH_TF32X3 && !tc) {
-      std::memset(out, 0, sizeof(double) * SPL_BOUND_STATS);
-      out[kMaxErrHard] = INFINITY;
-      continue;
-    }
-    st = spl_precompute_noise_product(c, Nz, W, W_hi, W_lo, rows, K, N, path, pws, pws_bytes, stream);
-    if (st == SPL_EUNSUPPORTED && path == SPL_PATH_TF32X3) {
-      std::memset(out, 0, sizeof(double) * SPL_BOUND_STATS);
-      out[kMaxErrHard] = INFINITY;
-      continue;
-    }
+  // stats blocks in the order FP32, TF32X3, FP16X3
+  const spl_path paths[3] = {SPL_PATH_FP32, SPL_PATH_TF32X3, SPL_PATH_FP16X3};
+  const int cc = device_cc();
+  const bool tc = cc == 100 || cc == 103;  // tcgen05 device
+  const bool have[3] = {true, tc && W->tf32_hi && W->tf32_lo,
+                        tc && W->f16_hi && W->f16_lo && W->f16_exp && (K & 7) == 0};
+  for (int p = 0; p < 3; ++p) {
+    double* out = stats + p * SPL_BOUND_STATS;
+    std::memset(out, 0, sizeof(double) * SPL_BOUND_STATS);
+    out[kMaxErrHard] = INFINITY;
+    if (!have[p]) continue;
+    st = spl_precompute_noise_product(c, Nz, W, rows, K, N, paths[p], pws, pws_bytes, stream);
+    if (st == SPL_EUNSUPPORTED && p > 0) continue;
     if (st != SPL_OK) return st;
-    st = spl_masked_linear_unmask(y, xt, W, W_hi, W_lo, c, rows, K, N, path, pws, pws_bytes, stream);
+    st = spl_masked_linear_unmask(y, xt, W, c, rows, K, N, paths[p], pws, pws_bytes, stream);
     if (st != SPL_OK) return st;
-    st = spl_bound_check(out, y, X, xt, Nz, W, rows, K, N, dstats, 256, stream);
+    st = spl_bound_check(out, y, X, xt, Nz, W->w, rows, K, N, dstats, 256, stream);
     if (st != SPL_OK) return st;
   }
-  const double* a = stats_tf32x3;
-  const double* b = stats_fp32;
-  const bool inside = a[kMaxErrHard] <= 1.0;
-  const bool no_worse = a[kViolLog] <= b[kViolLog] + 0.01 * a[kCount] && a[kSumErr] <= 1.5 * b[kSumErr] + 1e-300;
-  *chosen = (inside && no_worse) ? SPL_PATH_TF32X3 : SPL_PATH_FP32;
+  const double* b = stats;  // FP32
+  for (int p = 2; p >= 1; --p) {  // FP16X3 first (fewer weight bytes, twice the rate), then TF32X3
+    const double* a = stats + p * SPL_BOUND_STATS;
+    const bool inside = a[kMaxErrHard] <= 1.0;
+    const bool no_worse = a[kViolLog] <= b[kViolLog] + 0.01 * a[kCount] && a[kSumErr] <= 1.5 * b[kSumErr] + 1e-300;
+    if (inside && no_worse) {
+      *chosen = paths[p];
+      return SPL_OK;
+    }
+  }
   return SPL_OK;
 }

@@ -37,33 +37,68 @@ int device_cc();
 
 // ---- product dispatch shared by gemm_simt.cu, gemv.cu, gemm_tc.cu, linear.cu ----
 struct LinearArgs {
-  float* out;            // [M, N]
-  const float* a;        // [M, K]  (X~ or noise)
-  const float* w;        // [N, K]
-  const float* w_hi;     // [N, K] or null
-  const float* w_lo;     // [N, K] or null
-  const float* c;        // [M, N] correction subtracted in the epilogue, or null
+  float* out;               // [M, N]
+  const float* a;           // [M, K]  (X~ or noise)
+  const float* w;           // [N, K]  fp32
+  const float* w_hi;        // [N, K]  TF32 split, or null
+  const float* w_lo;
+  const uint16_t* w_h16;    // [N, K]  fp16 split (binary16 bits), or null
+  const uint16_t* w_l16;
+  const int32_t* w_exp;     // [N]     row exponents of the fp16 split
+  const float* c;           // [M, N]  correction subtracted in the epilogue, or null
   int64_t M, K, N;
-  void* ws;              // workspace (zero-filled), may be null
+  void* ws;                 // workspace (zero-filled), may be null
   size_t ws_bytes;
   cudaStream_t stream;
+  spl_path path;            // resolved arithmetic path
 };
 
 // Workspace layout shared by every product call: the first kCounterBytes hold
-// the decode kernel's arrival counters (zero between calls); split-K partials
-// and the TF32 split of the left operand follow.  Keeping the counters at a
-// fixed place lets one workspace serve calls of any shape and path.
+// the decode kernel's arrival counters (zero between calls); split-K partials,
+// or the FP16X3 row exponents of the left operand, follow.  Keeping the counters
+// at a fixed place lets one workspace serve calls of any shape and path.
 constexpr size_t kCounterBytes = 64 * 1024;
 constexpr int64_t kMaxCounters = (int64_t)(kCounterBytes / sizeof(unsigned int));
 
+inline LinearArgs make_args(float* out, const float* a, const spl_weight& W, const float* c, int64_t M, int64_t K,
+                            int64_t N, void* ws, size_t ws_bytes, cudaStream_t stream, spl_path path) {
+  LinearArgs r{};
+  r.out = out;
+  r.a = a;
+  r.w = W.w;
+  r.w_hi = W.tf32_hi;
+  r.w_lo = W.tf32_lo;
+  r.w_h16 = W.f16_hi;
+  r.w_l16 = W.f16_lo;
+  r.w_exp = W.f16_exp;
+  r.c = c;
+  r.M = M;
+  r.K = K;
+  r.N = N;
+  r.ws = ws;
+  r.ws_bytes = ws_bytes;
+  r.stream = stream;
+  r.path = path;
+  return r;
+}
+
+// Power-of-two exponent e that brings max |x| of a row into [2^14, 2^15) for the fp16 split
+// (0 for an all-zero row), clamped so 2^e and 2^-e stay normal floats.
+__device__ __forceinline__ int fp16_row_exponent(float amax) {
+  if (!(amax > 0.0f)) return 0;
+  const int e = ((__float_as_int(amax) >> 23) & 0xFF) - 127;  // amax in [2^e, 2^(e+1)) for normal amax
+  const int s = 14 - e;
+  return s < -126 ? -126 : (s > 126 ? 126 : s);
+}
+
 // Split-K plans: how many K-splits each kernel uses and the workspace it needs.
 struct Plan {
-  int kernel;            // 0 = GEMV (decode), 1 = FP32 SIMT GEMM, 2 = TF32X3 tcgen05 GEMM
+  int kernel;            // 0 = GEMV (decode), 1 = FP32 SIMT GEMM, 2 = tcgen05 GEMM (TF32X3 / FP16X3)
   int splits;            // K-splits (1 = none)
   int64_t k_per_split;   // multiple of the kernel's K granule
   size_t ws_partials;    // bytes of split partials (at offset kCounterBytes)
-  size_t ws_asplit;      // bytes of the A operand's hi/lo split (TF32X3, after the partials)
-  size_t total() const { return (ws_partials + ws_asplit) ? kCounterBytes + ws_partials + ws_asplit : 0; }
+  size_t ws_aexp;        // bytes of the FP16X3 row exponents of A (at offset kCounterBytes)
+  size_t total() const { return (ws_partials + ws_aexp) ? kCounterBytes + ws_partials + ws_aexp : 0; }
 };
 
 constexpr int kGemvMaxM = 16;
@@ -71,12 +106,13 @@ constexpr int kKernelGemv = 0, kKernelSimt = 1, kKernelTc = 2;
 
 Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms);
 Plan plan_simt(int64_t M, int64_t K, int64_t N, int sms);
-Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms);
+Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path);
 
 spl_status run_gemv(const LinearArgs& a, const Plan& p);
 int64_t gemv_max_ks(int64_t M);                           // largest K-slice the decode kernel stages for M rows
-int tc_uniform_splits(int64_t M, int64_t K, int64_t N);    // K-split of a one-launch TF32X3 call, 0 if mixed
-spl_status run_tc_splits(const LinearArgs& a, int splits); // TF32X3 with the same K-split on every tile
+int tc_uniform_splits(int64_t M, int64_t K, int64_t N);    // K-split of a one-launch tcgen05 call, 0 if mixed
+spl_status run_tc_splits(const LinearArgs& a, int splits); // tcgen05 product with the same K-split on every tile
+size_t tc_aexp_bytes(int64_t M, spl_path path);            // workspace of the FP16X3 row exponents (0 for TF32X3)
 spl_status run_simt(const LinearArgs& a, const Plan& p);
 spl_status run_tc(const LinearArgs& a, const Plan& p);
 

@@ -15,6 +15,8 @@
 
 #include <algorithm>
 
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 
 namespace spl {
@@ -196,6 +198,43 @@ __global__ void __launch_bounds__(kThreads) split_tf32_kernel(float* __restrict_
   }
 }
 
+// fp16 split of a weight, one warp per row: e = fp16_row_exponent(max |w|) brings the row's
+// largest entry into [2^14, 2^15); hi = fp16(w 2^e), lo = fp16(w 2^e - hi) (the difference
+// is exact in fp32).  cols % 8 == 0; each lane handles 8 consecutive entries at a time.
+__global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restrict__ hi, uint16_t* __restrict__ lo,
+                                                              int* __restrict__ row_exp, const float* __restrict__ src,
+                                                              int64_t rows, int64_t cols) {
+  const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const float4* row = reinterpret_cast<const float4*>(src + r * cols);
+  const int64_t q = cols >> 2;
+  float m = 0.f;
+  for (int64_t i = lane; i < q; i += 32) {
+    const float4 v = __ldg(row + i);
+    m = fmaxf(m, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
+  }
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  const int e = fp16_row_exponent(m);
+  if (lane == 0) row_exp[r] = e;
+  const float sc = __int_as_float((e + 127) << 23);
+  uint4* h8 = reinterpret_cast<uint4*>(hi + r * cols);
+  uint4* l8 = reinterpret_cast<uint4*>(lo + r * cols);
+  for (int64_t i = lane; i < (cols >> 3); i += 32) {
+    const float4 a = __ldg(row + 2 * i), b = __ldg(row + 2 * i + 1);
+    const float xs[8] = {a.x * sc, a.y * sc, a.z * sc, a.w * sc, b.x * sc, b.y * sc, b.z * sc, b.w * sc};
+    __align__(16) __half h[8];
+    __align__(16) __half l[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      h[k] = __float2half_rn(xs[k]);
+      l[k] = __float2half_rn(__fsub_rn(xs[k], __half2float(h[k])));
+    }
+    h8[i] = *reinterpret_cast<const uint4*>(h);
+    l8[i] = *reinterpret_cast<const uint4*>(l);
+  }
+}
+
 int grid_for(int64_t work_items, int blocks_per_sm) {
   const int64_t want = ceil_div(work_items, kThreads);
   const int64_t cap = (int64_t)device_sm_count() * blocks_per_sm;
@@ -301,6 +340,20 @@ extern "C" spl_status spl_unmask(float* Y, const float* Yt, const float* C, int6
   if (!Y || !Yt || !C) return SPL_EINVAL;
   if (!aligned16(Y) || !aligned16(Yt) || !aligned16(C)) return SPL_EALIGN;
   return run_addsub(Y, Yt, C, n, true, stream);
+}
+
+extern "C" spl_status spl_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows,
+                                     int64_t cols, cudaStream_t stream) {
+  if (rows < 0 || cols < 0) return SPL_EINVAL;
+  if (rows == 0) return SPL_OK;
+  if (!row_exp || (cols > 0 && (!hi || !lo || !src))) return SPL_EINVAL;
+  if ((cols & 7) != 0) return SPL_EALIGN;
+  if ((hi && !aligned16(hi)) || (lo && !aligned16(lo)) || (src && !aligned16(src))) return SPL_EALIGN;
+  if (cols == 0) return cudaMemsetAsync(row_exp, 0, (size_t)rows * sizeof(int32_t), stream) == cudaSuccess
+                            ? SPL_OK : SPL_ECUDA;
+  split_fp16_kernel<<<(unsigned)ceil_div(rows * 32, kThreads), kThreads, 0, stream>>>(hi, lo, row_exp, src, rows,
+                                                                                       cols);
+  return launch_status();
 }
 
 extern "C" spl_status spl_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {

@@ -1,34 +1,42 @@
-// TF32X3 product on the 5th-generation tensor cores (tcgen05, sm_103a):
+// Split-precision products on the 5th-generation tensor cores (tcgen05, sm_103a):
 //   out[M, N] = A[M, K] W[N, K]^T (- C)
-// with every operand split into a TF32 high part and an fp32 residual,
-// a = a_hi + a_lo, and three TF32 products per term accumulated in fp32:
-//   a w ~ a_lo w_hi + a_hi w_lo + a_hi w_hi     (the a_lo w_lo term is dropped).
-// The tensor core keeps 10 explicit mantissa bits of each operand; with
-// round-to-nearest hi parts the per-product error is about 2^-20 |a w|, so the
-// masked product r = W x~ (Sec. 5.1) and the correction W eta (Sec. 5.2) stay
-// inside the binary32 bound gamma_d <|w|,|x|> the paper's Thm. 4 is built on
-// for reduction lengths d >= 64, while running on the tensor pipe.  The paper
-// computes these products on a GPU in FP32 (Sec. 5, Sec. 6.3.2); this is the
-// GB300 way to get that accuracy.
+// Every operand is split into a high part and a residual, a = a_hi + a_lo, and
+// three products per term are accumulated in fp32 (the a_lo w_lo term is dropped):
+//   a w ~ a_lo w_hi + a_hi w_lo + a_hi w_hi.
+// Two encodings of the split:
+//   TF32X3  hi = a rounded to TF32 (11 significant bits), lo = a - hi kept in fp32;
+//           the tensor core truncates lo to TF32: per-term error ~2.5 x 2^-21 |a w|.
+//           kind::tf32, K = 8 per instruction; W split offline, 8 bytes per weight.
+//   FP16X3  each row is first scaled by a power of two so its largest entry lies in
+//           [2^14, 2^15); hi = fp16(a 2^e), lo = fp16(a 2^e - hi) (11 + 11 significant
+//           bits); per-term error ~2^-21 |a w|.  kind::f16 runs at twice the TF32 rate
+//           and the W split is 4 bytes per weight; the power-of-two scales are undone
+//           exactly in the epilogue.
+// Either way each term is within about 3 x 2^-21 of exact, below gamma_K = K 2^-24 for
+// K >= 64, so the masked product r = W x~ (Sec. 5.1) and the correction W eta (Sec. 5.2)
+// stay inside the binary32 error model the paper's Thm. 4 is built on while running on
+// the tensor pipe.
 //
-// Kernel shape (one CTA per 128 x 256 output tile, one CTA per SM):
-//   warp 0      TMA producer: four tiles per stage (A_hi, A_lo, W_hi, W_lo),
-//               K step 16 fp32 = 64 bytes, 64-byte swizzle, 4-stage ring.
-//   warp 1      TMEM allocator and MMA issuer: per stage 2 k-steps x 3
-//               tcgen05.mma.kind::tf32 (M=128, N=256, K=8) into one fp32
-//               accumulator of 256 TMEM columns; tcgen05.commit frees the
-//               stage and finally signals the epilogue.
-//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns at a time,
-//               subtract C (the fused unmask of Eq. add-and-then-subtract)
-//               and store, or store split-K partials.
-// Every mbarrier wait is bounded (about 1 s of globaltimer); on expiry the
-// kernel raises the device status word, lets in-flight copies land (again
-// with a bound), frees its TMEM and returns.
+// Kernel shape (one CTA per 128 x 256 output tile, one CTA per SM, 6 warps):
+//   warp 0      TMA producer: per stage the raw fp32 A tile and W_hi, W_lo.
+//   warps 2-5   split the raw A tile into the hi/lo operand tiles in shared memory
+//               (FP16X3: scaled by the per-row exponents a short pass over A wrote to
+//               the workspace before the product), then act as the epilogue.
+//   warp 1      TMEM allocator and MMA issuer: per stage 2 k-steps x 3 products into one
+//               fp32 accumulator of 256 TMEM columns; tcgen05.commit frees the stage.
+//   epilogue    tcgen05.ld 32 lanes x 32 columns, (FP16X3: descale), stage the tile in
+//               shared memory; the K-split CTAs of one tile (a thread-block cluster) sum
+//               their staged tiles through distributed shared memory in rank order;
+//               subtract C (the fused unmask of Eq. add-and-then-subtract) and store.
+// Every mbarrier wait is bounded (about 1 s of globaltimer); on expiry the kernel raises
+// the device status word, lets issued copies land (again bounded), frees its TMEM and
+// returns.  Role loops run warp-wide (lane 0 issues), so no warp is diverged at a barrier.
 
 #include <algorithm>
 #include <cstring>
 
 #include <cuda.h>
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 
@@ -48,33 +56,60 @@ cudaError_t read_clear_device_status(unsigned int* word) {
 
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 16, STAGES = 4, THREADS = 192;
-constexpr int UMMA_K = 8;                                      // K of one kind::tf32 MMA
-constexpr uint32_t A_TILE_BYTES = BM * BK * 4;                 // 8 KB
-constexpr uint32_t B_TILE_BYTES = BN * BK * 4;                 // 16 KB
-constexpr uint32_t STAGE_BYTES = 2 * A_TILE_BYTES + 2 * B_TILE_BYTES;  // 48 KB
-constexpr uint32_t BAR_OFFSET = STAGES * STAGE_BYTES;          // barriers after the ring (3S+1 of them)
-constexpr uint32_t SMEM_BYTES = BAR_OFFSET + 256 + 1024;       // + barriers + alignment slack
+constexpr int BM = 128, BN = 256, THREADS = 192;
 constexpr uint32_t TMEM_COLS = 256;
-constexpr unsigned long long kWaitNs = 1000000000ull;          // 1 s per wait
-constexpr unsigned long long kDrainNs = 100000000ull;          // 0.1 s to drain on abort
+constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
+constexpr unsigned long long kDrainNs = 100000000ull;  // 0.1 s to drain on abort
+constexpr int MAX_CLUSTER = 8;                         // split-K CTAs of one output tile (portable cluster)
+constexpr int RED_STRIDE = BN + 4;                     // floats per row of the staged accumulator
+constexpr uint32_t RING_BYTES = 192 * 1024;            // stage ring (both modes)
+constexpr uint32_t AUX_BYTES = 2048;                   // barriers, TMEM slot, abort flag, exponents
+constexpr uint32_t SMEM_BYTES = RING_BYTES + AUX_BYTES + 1024;  // + alignment slack
+static_assert((size_t)BM * RED_STRIDE * 4 <= RING_BYTES, "staging fits in the stage ring");
 
-// ---- instruction and shared-memory descriptors (tcgen05) -------------------
-// Instruction descriptor, kind::tf32: D = F32 (bits 4-5 = 1), A = B = TF32
-// (bits 7-9 and 10-12 = 2), both K-major (bits 15, 16 = 0), N >> 3 at bits
-// 17-22, M >> 4 at bits 24-28.
-constexpr uint32_t make_idesc_tf32(int m, int n) {
-  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+// ---- instruction descriptors (tcgen05.mma kind::tf32 / kind::f16) ---------------
+// D = F32 (bits 4-5 = 1); A and B formats at bits 7-9 and 10-12 (f16: 0, tf32: 2);
+// both K-major (bits 15, 16 = 0); N >> 3 at bits 17-22; M >> 4 at bits 24-28.
+constexpr uint32_t make_idesc(uint32_t ab_format, int m, int n) {
+  return (1u << 4) | (ab_format << 7) | (ab_format << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(m >> 4) << 24);
 }
-constexpr uint32_t kIdesc = make_idesc_tf32(BM, BN);
-static_assert(kIdesc == 0x08400910u, "idesc encoding");
+static_assert(make_idesc(2, BM, BN) == 0x08400910u, "tf32 idesc encoding");
+static_assert(make_idesc(0, BM, BN) == 0x08400010u, "f16 idesc encoding");
 
-// Shared-memory matrix descriptor for a K-major tile written by TMA with the
-// 64-byte swizzle: rows of 64 bytes, 8-row (512-byte) swizzle atoms stacked
-// along M/N.  start address >> 4 in bits 0-13, leading byte offset >> 4 in
-// 16-29 (not used by swizzled K-major layouts; 1), stride byte offset >> 4
-// (512 B between 8-row groups) in 32-45, descriptor version 1 at bit 46,
-// base offset 0 (atoms are 512-byte aligned), layout SWIZZLE_64B = 4 at 61-63.
+// The two modes.  Stage layout: [A_hi][A_lo][W_hi][W_lo][A_raw (FP16X3 only)]; in TF32X3
+// the raw A tile lands in the A_hi slot and is split in place.  Operand rows are 64 bytes
+// (64-byte swizzle) in both modes: 16 fp32 or 32 fp16 elements of K.
+struct Tf32x3 {
+  static constexpr bool kF16 = false;
+  static constexpr int BK = 16;  // K elements per stage
+  static constexpr int STAGES = 4;
+  static constexpr int UMMA_K = 8;
+  static constexpr uint32_t A_HALF = BM * BK * 4, B_HALF = BN * BK * 4, A_RAW = 0;
+  static constexpr uint32_t IDESC = make_idesc(2, BM, BN);
+};
+struct Fp16x3 {
+  static constexpr bool kF16 = true;
+  static constexpr int BK = 32;
+  static constexpr int STAGES = 3;
+  static constexpr int UMMA_K = 16;
+  static constexpr uint32_t A_HALF = BM * BK * 2, B_HALF = BN * BK * 2, A_RAW = BM * BK * 4;
+  static constexpr uint32_t IDESC = make_idesc(0, BM, BN);
+};
+template <class Md>
+struct Layout {
+  static constexpr uint32_t A_HI = 0, A_LO = Md::A_HALF, W_HI = 2 * Md::A_HALF, W_LO = W_HI + Md::B_HALF;
+  static constexpr uint32_t RAW = W_LO + Md::B_HALF;
+  static constexpr uint32_t STAGE = RAW + Md::A_RAW;
+  static constexpr uint32_t TX = (Md::kF16 ? Md::A_RAW : Md::A_HALF) + 2 * Md::B_HALF;  // bytes TMA brings
+  static_assert(STAGE * Md::STAGES <= RING_BYTES, "ring fits");
+  static_assert(RAW % 1024 == 0 && STAGE % 1024 == 0, "swizzle atoms aligned");
+};
+
+// Shared-memory matrix descriptor for a K-major operand tile with the 64-byte swizzle:
+// 64-byte rows, 8-row (512-byte) atoms stacked along M/N.  start >> 4 in bits 0-13, leading
+// byte offset >> 4 in 16-29 (unused by swizzled K-major layouts; 1), stride byte offset >> 4
+// (512) in 32-45, descriptor version 1 at bit 46, base offset 0, SWIZZLE_64B = 4 at 61-63.
 __device__ __forceinline__ uint64_t make_sdesc_sw64(uint32_t saddr) {
   uint64_t d = 0;
   d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
@@ -85,12 +120,13 @@ __device__ __forceinline__ uint64_t make_sdesc_sw64(uint32_t saddr) {
   return d;
 }
 
-// ---- PTX wrappers ----------------------------------------------------------
+// ---- PTX wrappers ----------------------------------------------------------------
 __device__ __forceinline__ float tf32_rna(float v) {
   uint32_t r;
   asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(v));
   return __uint_as_float(r);
 }
+__device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }  // e in [-126, 127]
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -105,6 +141,9 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
 __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -116,8 +155,8 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait for the phase of the given parity.  Returns false if it gave
-// up (deadline passed or another role raised *abort).
+// Bounded wait for the phase of the given parity; false if it gave up (deadline passed or
+// another role raised *abort).
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned long long budget_ns,
                                           volatile int* abort) {
   if (mbar_try(bar, parity)) return true;
@@ -145,14 +184,23 @@ __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
   asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
-__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                         uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
+template <class Md>
+__device__ __forceinline__ void mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+  if constexpr (Md::kF16) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(Md::IDESC), "r"(accumulate)
+        : "memory");
+  } else {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(Md::IDESC), "r"(accumulate)
+        : "memory");
+  }
 }
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
@@ -180,15 +228,6 @@ __device__ __forceinline__ void tmem_ld_32x32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
-
-struct TcMaps {
-  CUtensorMap a, w_hi, w_lo;
-};
-
-constexpr int MAX_CLUSTER = 8;        // split-K CTAs of one output tile (portable cluster size)
-constexpr int RED_STRIDE = BN + 4;    // floats per row of the staged accumulator (pads bank conflicts)
-static_assert((size_t)BM * RED_STRIDE * 4 <= (size_t)STAGES * STAGE_BYTES, "staging fits in the stage ring");
-
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
@@ -210,24 +249,60 @@ __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
                : "memory");
   return v;
 }
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+__device__ __forceinline__ void converter_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// FP16X3 row exponents of A: e_r = fp16_row_exponent(max_k |A[r, k]|), one warp per row,
+// each lane keeping several 16-byte loads in flight.  Scaling a row by 2^e_r is exact, so the
+// choice of e_r only has to keep every scaled entry inside the fp16 range.
+__global__ void __launch_bounds__(256) row_exponent_kernel(int* __restrict__ exps, const float* __restrict__ A,
+                                                           int64_t M, int64_t K) {
+  const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (r >= M) return;
+  const float4* row = reinterpret_cast<const float4*>(A + r * K);
+  const int64_t q = K >> 2;
+  float m0 = 0.f, m1 = 0.f, m2 = 0.f, m3 = 0.f;
+  int64_t i = lane;
+  for (; i + 96 < q; i += 128) {
+    const float4 a = __ldg(row + i), b = __ldg(row + i + 32), c = __ldg(row + i + 64), d = __ldg(row + i + 96);
+    m0 = fmaxf(m0, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
+    m1 = fmaxf(m1, fmaxf(fmaxf(fabsf(b.x), fabsf(b.y)), fmaxf(fabsf(b.z), fabsf(b.w))));
+    m2 = fmaxf(m2, fmaxf(fmaxf(fabsf(c.x), fabsf(c.y)), fmaxf(fabsf(c.z), fabsf(c.w))));
+    m3 = fmaxf(m3, fmaxf(fmaxf(fabsf(d.x), fabsf(d.y)), fmaxf(fabsf(d.z), fabsf(d.w))));
+  }
+  for (; i < q; i += 32) {
+    const float4 a = __ldg(row + i);
+    m0 = fmaxf(m0, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
+  }
+  float m = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if (lane == 0) exps[r] = fp16_row_exponent(m);
 }
 
+struct TcMaps {
+  CUtensorMap a, w_hi, w_lo;
+};
+
 // One CTA computes a 128 x 256 tile of out over the K range of its split (blockIdx.z).
-// The `splits` CTAs of a tile form one thread-block cluster (z dimension);
-// their fp32 partial tiles are summed through distributed shared memory in
-// cluster-rank order, so the result does not depend on timing.
+// The `splits` CTAs of a tile form one thread-block cluster (z dimension); their fp32
+// partial tiles are summed through distributed shared memory in cluster-rank order, so
+// the result does not depend on timing.
+template <class Md>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
-               int64_t M, int64_t K, int64_t N, int64_t k_per_split, int splits, int tile_base, int m_tiles,
-               int skip_kblock) {
+               const int* __restrict__ a_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
+               int64_t k_per_split, int splits, int tile_base, int m_tiles, int skip_kblock) {
+  using L = Layout<Md>;
+  constexpr int STAGES = Md::STAGES, BK = Md::BK;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + BAR_OFFSET);  // full[S], conv[S], empty[S], accum
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + BAR_OFFSET + 8 * (3 * STAGES + 1));
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + BAR_OFFSET + 8 * (3 * STAGES + 1) + 8);
-  float* red = reinterpret_cast<float*>(smem);  // [BM][RED_STRIDE] staged accumulator, after the mainloop
+  uint8_t* aux = smem + RING_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], conv[S], empty[S], accum
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (3 * STAGES + 1));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (3 * STAGES + 1) + 8);
+  int* ea = reinterpret_cast<int*>(aux + 512);    // [BM]  FP16X3: row exponents of A
+  int* ew = reinterpret_cast<int*>(aux + 1024);   // [BN]  FP16X3: row exponents of W (whole rows)
+  float* red = reinterpret_cast<float*>(smem);    // [BM][RED_STRIDE] staged accumulator, after the mainloop
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // Linear tile id, M fastest: the CTAs that read the same weight tile run side by side and share it in L2.
@@ -261,10 +336,8 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  // Every role loop is run by whole warps (lane 0 issues, all lanes wait), so no warp is
-  // ever diverged when it reaches a block- or cluster-wide barrier.
   if (warp == 0) {
-    // ---------------- TMA producer: raw A (into the A_hi slot), W_hi, W_lo ----------------
+    // ---------------- TMA producer: raw A, W_hi, W_lo ----------------
     uint32_t issued_mask = 0u, phase_mask = 0u;  // per stage: a load was issued / its parity
     bool ok = true;
     for (int kb = 0; kb < nk; ++kb) {
@@ -274,12 +347,12 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       if (!ok) break;
       if (kb == skip_kblock) continue;  // failure-detection test only: this stage never arrives
       if (lane == 0) {
-        const uint32_t st = smem_u32(smem + (size_t)s * STAGE_BYTES);
+        const uint32_t st = smem_u32(smem + (size_t)s * L::STAGE);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
-        mbar_expect_tx(full_bar(s), A_TILE_BYTES + 2 * B_TILE_BYTES);
-        tma_load_2d(st, &maps.a, full_bar(s), kx, (int)m0);
-        tma_load_2d(st + 2 * A_TILE_BYTES, &maps.w_hi, full_bar(s), kx, (int)n0);
-        tma_load_2d(st + 2 * A_TILE_BYTES + B_TILE_BYTES, &maps.w_lo, full_bar(s), kx, (int)n0);
+        mbar_expect_tx(full_bar(s), L::TX);
+        tma_load_2d(st + (Md::kF16 ? L::RAW : L::A_HI), &maps.a, full_bar(s), kx, (int)m0);
+        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(s), kx, (int)n0);
+        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(s), kx, (int)n0);
       }
       __syncwarp();
       issued_mask |= 1u << s;
@@ -304,16 +377,14 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       if (!ok) break;
       if (lane == 0) {
         tc_fence_after();
-        const uint32_t st = smem_u32(smem + (size_t)s * STAGE_BYTES);
-        const uint32_t a_hi = st, a_lo = st + A_TILE_BYTES;
-        const uint32_t w_hi = st + 2 * A_TILE_BYTES, w_lo = w_hi + B_TILE_BYTES;
+        const uint32_t st = smem_u32(smem + (size_t)s * L::STAGE);
 #pragma unroll
-        for (int kk = 0; kk < BK / UMMA_K; ++kk) {
-          const uint32_t koff = kk * UMMA_K * 4;  // 32 bytes along the swizzled row
+        for (int kk = 0; kk < BK / Md::UMMA_K; ++kk) {
+          const uint32_t koff = kk * 32u;  // one instruction's K is 32 bytes of the 64-byte swizzled row
           const uint32_t first = (kb == 0 && kk == 0) ? 0u : 1u;
-          mma_tf32(tmem, make_sdesc_sw64(a_lo + koff), make_sdesc_sw64(w_hi + koff), kIdesc, first);
-          mma_tf32(tmem, make_sdesc_sw64(a_hi + koff), make_sdesc_sw64(w_lo + koff), kIdesc, 1u);
-          mma_tf32(tmem, make_sdesc_sw64(a_hi + koff), make_sdesc_sw64(w_hi + koff), kIdesc, 1u);
+          mma<Md>(tmem, make_sdesc_sw64(st + L::A_LO + koff), make_sdesc_sw64(st + L::W_HI + koff), first);
+          mma<Md>(tmem, make_sdesc_sw64(st + L::A_HI + koff), make_sdesc_sw64(st + L::W_LO + koff), 1u);
+          mma<Md>(tmem, make_sdesc_sw64(st + L::A_HI + koff), make_sdesc_sw64(st + L::W_HI + koff), 1u);
         }
         mma_commit(empty_bar(s));  // stage reusable once these MMAs have read it
       }
@@ -331,6 +402,12 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   } else {
     // ---------------- warps 2..5: split A during the mainloop, then the epilogue ----------------
     const int t = threadIdx.x - 64;  // 0..127
+    if constexpr (Md::kF16) {
+      // power-of-two row exponents of A (whole rows, from the exponent pass) and of this tile's W rows
+      ea[t] = (m0 + t < M) ? a_exp[m0 + t] : 0;
+      for (int j = t; j < BN; j += 128) ew[j] = (n0 + j < N) ? w_exp[n0 + j] : 0;
+      converter_sync();
+    }
     bool ok = true;
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % STAGES;
@@ -338,18 +415,43 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       ok = mbar_wait(full_bar(s), ph, kWaitNs, abort_flag);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
-      // The raw tile (8 KB, swizzled) sits in the hi slot; the hi and lo slots use the same
-      // swizzled positions, so the split is elementwise and in place (hi overwrites raw).
-      // Consecutive threads take consecutive 16-byte chunks: conflict-free shared accesses.
-      float4* hi = reinterpret_cast<float4*>(smem + (size_t)s * STAGE_BYTES);
-      float4* lo = reinterpret_cast<float4*>(smem + (size_t)s * STAGE_BYTES + A_TILE_BYTES);
+      uint8_t* st = smem + (size_t)s * L::STAGE;
+      if constexpr (Md::kF16) {
+        // raw tile: 128 rows x 32 fp32 (128-byte rows, 128-byte swizzle); operand tiles: 128 rows x 32 fp16
+        // (64-byte rows, 64-byte swizzle).  Item (r, c): raw chunks 2c, 2c+1 -> one 16-byte chunk of hi and lo.
 #pragma unroll
-      for (int j = 0; j < (int)(A_TILE_BYTES / 16) / 128; ++j) {
-        const int i = t + 128 * j;
-        const float4 v = hi[i];
-        const float4 h = make_float4(tf32_rna(v.x), tf32_rna(v.y), tf32_rna(v.z), tf32_rna(v.w));
-        hi[i] = h;
-        lo[i] = make_float4(__fsub_rn(v.x, h.x), __fsub_rn(v.y, h.y), __fsub_rn(v.z, h.z), __fsub_rn(v.w, h.w));
+        for (int j = 0; j < 4; ++j) {
+          const int i = t + 128 * j;
+          const int r = i >> 2, c = i & 3;
+          const uint8_t* raw = st + L::RAW + r * 128;
+          const float4 x0 = *reinterpret_cast<const float4*>(raw + (((2 * c) ^ (r & 7)) << 4));
+          const float4 x1 = *reinterpret_cast<const float4*>(raw + (((2 * c + 1) ^ (r & 7)) << 4));
+          const float sc = pow2f(ea[r]);
+          const float xs[8] = {x0.x * sc, x0.y * sc, x0.z * sc, x0.w * sc, x1.x * sc, x1.y * sc, x1.z * sc, x1.w * sc};
+          __align__(16) __half h[8];
+          __align__(16) __half l[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            h[e] = __float2half_rn(xs[e]);
+            l[e] = __float2half_rn(__fsub_rn(xs[e], __half2float(h[e])));
+          }
+          const uint32_t dst = r * 64 + ((c ^ ((r >> 1) & 3)) << 4);
+          *reinterpret_cast<uint4*>(st + L::A_HI + dst) = *reinterpret_cast<const uint4*>(h);
+          *reinterpret_cast<uint4*>(st + L::A_LO + dst) = *reinterpret_cast<const uint4*>(l);
+        }
+      } else {
+        // The raw tile sits in the hi slot; hi and lo use the same swizzled positions, so the split is
+        // elementwise and in place.  Consecutive threads take consecutive 16-byte chunks.
+        float4* hi = reinterpret_cast<float4*>(st + L::A_HI);
+        float4* lo = reinterpret_cast<float4*>(st + L::A_LO);
+#pragma unroll
+        for (int j = 0; j < (int)(Md::A_HALF / 16) / 128; ++j) {
+          const int i = t + 128 * j;
+          const float4 v = hi[i];
+          const float4 h = make_float4(tf32_rna(v.x), tf32_rna(v.y), tf32_rna(v.z), tf32_rna(v.w));
+          hi[i] = h;
+          lo[i] = make_float4(__fsub_rn(v.x, h.x), __fsub_rn(v.y, h.y), __fsub_rn(v.z, h.z), __fsub_rn(v.w, h.w));
+        }
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
       __syncwarp();
@@ -365,7 +467,10 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     if (have) {
       tc_fence_after();
-      float* row = red + (size_t)(32 * q + lane) * RED_STRIDE;
+      const int r = 32 * q + lane;
+      float* row = red + (size_t)r * RED_STRIDE;
+      float sr = 1.0f;
+      if constexpr (Md::kF16) sr = pow2f(-ea[r]);
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         float v[32];
@@ -374,6 +479,10 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
         } else {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
+        }
+        if constexpr (Md::kF16) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = (v[i] * sr) * pow2f(-ew[32 * c + i]);  // exact power-of-two scaling
         }
 #pragma unroll
         for (int j = 0; j < 32; j += 4)
@@ -386,7 +495,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   }
 
   // ---- sum the cluster's partial tiles in rank order, subtract C, store ----
-  __syncwarp();  // lane 0 of warps 0 and 1 ran the producer / MMA loops: reconverge before the barrier
+  __syncwarp();
   tc_fence_before();
   if (splits > 1) {
     cluster_sync_all();  // every rank's partial tile is staged
@@ -466,7 +575,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   }
 }
 
-// ---- host side: tensor maps ---------------------------------------------------
+// ---- host side: tensor maps ------------------------------------------------------
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -486,22 +595,39 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D fp32 map over a row-major [rows, K] matrix with a 16 x box_rows box, 64-byte swizzle.
-bool make_map(CUtensorMap* map, const float* base, int64_t rows, int64_t K, int box_rows) {
+// 2-D map over a row-major [rows, K] matrix of fp32 or fp16 with a box_k x box_rows box.
+bool make_map(CUtensorMap* map, const void* base, bool f16, int64_t rows, int64_t K, int box_k, int box_rows,
+              CUtensorMapSwizzle swz) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
+  const int esize = f16 ? 2 : 4;
   cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)K * 4};
-  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+  cuuint64_t strides[1] = {(cuuint64_t)K * esize};
+  cuuint32_t box[2] = {(cuuint32_t)box_k, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(map, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
+                  const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
 
-// Co-resident clusters of s CTAs (each one SM) on the current device; clusters
-// must fit inside one GPC, so this is not simply SMs / s.  Cached per device.
+template <class Md>
+bool set_smem_attr() {
+  static bool done[64] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  if (!done[dev]) {
+    if (cudaFuncSetAttribute(tc_gemm_kernel<Md>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) !=
+        cudaSuccess)
+      return false;
+    done[dev] = true;
+  }
+  return true;
+}
+
+// Co-resident clusters of s CTAs (each one SM) on the current device; clusters must fit
+// inside one GPC, so this is not simply SMs / s.  Both modes use the same shared memory
+// and block shape, so one cache serves both.  Cached per device.
 int max_active_clusters(int s, int sms) {
   static int cache[64][MAX_CLUSTER + 1] = {{0}};
   int dev = 0;
@@ -509,8 +635,7 @@ int max_active_clusters(int s, int sms) {
   int& v = cache[dev][s];
   if (v == 0) {
     int n = 0;
-    if (cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) ==
-        cudaSuccess) {
+    if (set_smem_attr<Tf32x3>()) {
       cudaLaunchConfig_t cfg;
       std::memset(&cfg, 0, sizeof(cfg));
       cfg.gridDim = dim3(1, 1, (unsigned)s);
@@ -523,7 +648,7 @@ int max_active_clusters(int s, int sms) {
       attr[0].val.clusterDim.z = (unsigned)s;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
-      if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel, &cfg) != cudaSuccess) n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel<Tf32x3>, &cfg) != cudaSuccess) n = 0;
     }
     cudaGetLastError();
     v = n > 0 ? n : std::max(1, sms / s);
@@ -576,47 +701,31 @@ TcLaunches tc_launches(int64_t M, int64_t K, int64_t N, int sms) {
   return t;
 }
 
-}  // namespace
-
-Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms) {
-  Plan p{};
-  p.kernel = kKernelTc;
-  const TcLaunches t = tc_launches(M, K, N, sms);
-  p.splits = t.rest_splits;
-  p.k_per_split = round_up(ceil_div(K, t.rest_splits), BK);
-  return p;  // no workspace: partials are reduced through distributed shared memory
-}
-
-spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock, int forced_splits = 0) {
-  const int cc = device_cc();
-  if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
-  if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
-  if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
-  if (a.M > 0x7fffffffLL || a.N > 0x7fffffffLL || a.K > 0x7fffffffLL) return SPL_ESHAPE;
-  if (ceil_div(a.M, BM) * ceil_div(a.N, BN) > 0x7fffffffLL || p.splits > MAX_CLUSTER) return SPL_ESHAPE;
-
+template <class Md>
+spl_status launch_tc(const LinearArgs& a, int skip_kblock, int forced_splits) {
+  if (!set_smem_attr<Md>()) return SPL_ECUDA;
   TcMaps maps;
   std::memset(&maps, 0, sizeof(maps));
-  if (!make_map(&maps.a, a.a, a.M, a.K, BM) || !make_map(&maps.w_hi, a.w_hi, a.N, a.K, BN) ||
-      !make_map(&maps.w_lo, a.w_lo, a.N, a.K, BN))
+  const void* whi = Md::kF16 ? (const void*)a.w_h16 : (const void*)a.w_hi;
+  const void* wlo = Md::kF16 ? (const void*)a.w_l16 : (const void*)a.w_lo;
+  const CUtensorMapSwizzle a_swz = Md::kF16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+  if (!make_map(&maps.a, a.a, false, a.M, a.K, Md::BK, BM, a_swz) ||
+      !make_map(&maps.w_hi, whi, Md::kF16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
+      !make_map(&maps.w_lo, wlo, Md::kF16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
     return SPL_ECUDA;
-
-  static bool attr_set[64] = {false};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-    if (cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) !=
-        cudaSuccess)
-      return SPL_ECUDA;
-    attr_set[dev] = true;
+  int* a_exp = nullptr;
+  if constexpr (Md::kF16) {
+    a_exp = reinterpret_cast<int*>(static_cast<char*>(a.ws) + kCounterBytes);
+    row_exponent_kernel<<<(unsigned)ceil_div(a.M * 32, 256), 256, 0, a.stream>>>(a_exp, a.a, a.M, a.K);
+    const spl_status st = launch_status();
+    if (st != SPL_OK) return st;
   }
   const int m_tiles = (int)ceil_div(a.M, BM);
-  const TcLaunches t = forced_splits > 0
-                           ? TcLaunches{0, ceil_div(a.M, BM) * ceil_div(a.N, BN), forced_splits}
-                           : tc_launches(a.M, a.K, a.N, device_sm_count());
+  const TcLaunches t = forced_splits > 0 ? TcLaunches{0, ceil_div(a.M, BM) * ceil_div(a.N, BN), forced_splits}
+                                         : tc_launches(a.M, a.K, a.N, device_sm_count());
   auto launch = [&](int64_t tiles, int64_t base, int splits) -> spl_status {
     if (tiles <= 0) return SPL_OK;
-    const int64_t kps = round_up(ceil_div(a.K, splits), BK);
+    const int64_t kps = round_up(ceil_div(a.K, splits), Md::BK);
     cudaLaunchConfig_t cfg;
     std::memset(&cfg, 0, sizeof(cfg));
     cfg.gridDim = dim3((unsigned)tiles, 1, (unsigned)splits);
@@ -630,8 +739,9 @@ spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock, int 
     attr[0].val.clusterDim.z = (unsigned)splits;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel, maps, a.out, a.c, a.M, a.K, a.N, kps, splits,
-                                             (int)base, m_tiles, skip_kblock);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md>, maps, a.out, a.c, (const int*)a_exp,
+                                             (const int*)a.w_exp, a.M, a.K, a.N, kps, splits, (int)base, m_tiles,
+                                             skip_kblock);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   };
@@ -640,7 +750,44 @@ spl_status run_tc_impl(const LinearArgs& a, const Plan& p, int skip_kblock, int 
   return launch(t.rest_tiles, t.full_tiles, t.rest_splits);
 }
 
-spl_status run_tc(const LinearArgs& a, const Plan& p) { return run_tc_impl(a, p, -1); }
+spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_splits) {
+  const int cc = device_cc();
+  if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
+  const bool f16 = a.path == SPL_PATH_FP16X3;
+  if (f16) {
+    if (!a.w_h16 || !a.w_l16 || !a.w_exp) return SPL_EUNSUPPORTED;
+    if ((a.K & 7) != 0) return SPL_EALIGN;  // fp16 rows must be whole 16-byte units
+    if (!aligned16(a.w_h16) || !aligned16(a.w_l16)) return SPL_EALIGN;
+    if (!a.ws || a.ws_bytes < kCounterBytes + tc_aexp_bytes(a.M, a.path)) return SPL_EWORKSPACE;
+  } else {
+    if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
+    if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
+  }
+  if (a.M > 0x7fffffffLL || a.N > 0x7fffffffLL || a.K > 0x7fffffffLL) return SPL_ESHAPE;
+  if (ceil_div(a.M, BM) * ceil_div(a.N, BN) > 0x7fffffffLL || forced_splits > MAX_CLUSTER) return SPL_ESHAPE;
+  return f16 ? launch_tc<Fp16x3>(a, skip_kblock, forced_splits) : launch_tc<Tf32x3>(a, skip_kblock, forced_splits);
+}
+
+}  // namespace
+
+size_t tc_aexp_bytes(int64_t M, spl_path path) {
+  return path == SPL_PATH_FP16X3 ? (size_t)round_up(M * (int64_t)sizeof(int), 256) : 0;
+}
+
+Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path) {
+  Plan p{};
+  p.kernel = kKernelTc;
+  const TcLaunches t = tc_launches(M, K, N, sms);
+  p.splits = t.rest_splits;
+  p.k_per_split = ceil_div(K, t.rest_splits);
+  p.ws_aexp = tc_aexp_bytes(M, path);  // partials are reduced through distributed shared memory
+  return p;
+}
+
+spl_status run_tc(const LinearArgs& a, const Plan& p) {
+  (void)p;
+  return run_tc_impl(a, -1, 0);
+}
 
 int tc_uniform_splits(int64_t M, int64_t K, int64_t N) {
   const TcLaunches t = tc_launches(M, K, N, device_sm_count());
@@ -649,11 +796,7 @@ int tc_uniform_splits(int64_t M, int64_t K, int64_t N) {
 
 spl_status run_tc_splits(const LinearArgs& a, int splits) {
   if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
-  Plan p{};
-  p.kernel = kKernelTc;
-  p.splits = splits;
-  p.k_per_split = round_up(ceil_div(a.K, splits), BK);
-  return run_tc_impl(a, p, -1, splits);
+  return run_tc_impl(a, -1, splits);
 }
 
 }  // namespace spl
@@ -661,12 +804,22 @@ spl_status run_tc_splits(const LinearArgs& a, int splits) {
 // Failure-detection test hook: one TF32X3 product in which the copy of the first K stage is
 // never issued, so the kernel's bounded waits run out (about 1 s), it raises the device status
 // word and returns.  The paper has no counterpart.
-extern "C" spl_status spl_test_tc_wait_timeout(float* out, const float* A, const float* W, const float* W_hi,
-                                               const float* W_lo, int64_t M, int64_t K, int64_t N,
-                                               cudaStream_t stream) {
+extern "C" spl_status spl_test_tc_wait_timeout(float* out, const float* A, const spl_weight* W, int64_t M, int64_t K,
+                                               int64_t N, cudaStream_t stream) {
   using namespace spl;
-  if (!out || !A || !W || !W_hi || !W_lo || M <= 0 || N <= 0 || K <= 0 || (K & 3)) return SPL_EINVAL;
+  if (!out || !A || !W || !W->w || !W->tf32_hi || !W->tf32_lo || M <= 0 || N <= 0 || K <= 0 || (K & 3))
+    return SPL_EINVAL;
   if (K > 256) return SPL_ESHAPE;  // one K range per tile: the skipped stage belongs to every CTA
-  LinearArgs args{out, A, W, W_hi, W_lo, nullptr, M, K, N, nullptr, 0, stream};
-  return run_tc_impl(args, plan_tc(M, K, N, device_sm_count()), 0);
+  LinearArgs args{};
+  args.out = out;
+  args.a = A;
+  args.w = W->w;
+  args.w_hi = W->tf32_hi;
+  args.w_lo = W->tf32_lo;
+  args.M = M;
+  args.K = K;
+  args.N = N;
+  args.stream = stream;
+  args.path = SPL_PATH_TF32X3;
+  return run_tc_impl(args, 0, 0);
 }

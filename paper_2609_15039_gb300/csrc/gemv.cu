@@ -263,6 +263,17 @@ extern "C" spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt
   void* ws = nullptr;
   spl_status st = static_scratch(&ws);
   if (st != SPL_OK) return st;
-  LinearArgs args{Y, Xt, W, nullptr, nullptr, C, M, K, N, ws, kStaticScratchBytes, stream};
+  LinearArgs args{};
+  args.out = Y;
+  args.a = Xt;
+  args.w = W;
+  args.c = C;
+  args.M = M;
+  args.K = K;
+  args.N = N;
+  args.ws = ws;
+  args.ws_bytes = kStaticScratchBytes;
+  args.stream = stream;
+  args.path = SPL_PATH_FP32;
   return run_gemv(args, plan);
 }

@@ -6,10 +6,11 @@
 //   spl_masked_linear_unmask      Y = X~ W^T - C        (Eq. add-and-then-subtract, fused)
 //
 // Kernel choice: on the FP32 path M <= 16 rows stream W once through the decode
-// kernel and larger M use the SIMT kernel.  AUTO takes the TF32X3 tcgen05
-// kernel for M > 8 when the weight split is available, the device is
-// sm_100/sm_103 and K >= 64 (below that the three-product error of about
-// 2^-20 per term is not small against gamma_K), else FP32.
+// kernel and larger M use the SIMT kernel.  AUTO takes a tcgen05 kernel for M > 8
+// on an sm_100/sm_103 device with K >= 64 (below that the three-product error of
+// about 2^-20 per term is not small against gamma_K): FP16X3 when the weight
+// descriptor carries the fp16 split and K % 8 == 0, else TF32X3 when it carries the
+// TF32 split, else FP32.
 
 #include <algorithm>
 
@@ -23,46 +24,70 @@ bool tc_capable() {
   return cc == 100 || cc == 103;
 }
 
-// AUTO: up to 8 rows the streaming decode kernel reads W once at HBM rate and
-// wins; from 9 rows on the tensor-core kernel is faster even with its 128-row
-// tile mostly empty (the decode kernel turns shared-memory bound as M grows).
+// AUTO: up to 8 rows the streaming decode kernel reads W once at HBM rate and wins; from
+// 9 rows on a tensor-core path is faster even with its 128-row tile mostly empty (the
+// decode kernel turns shared-memory bound as M grows).  FP16X3 (4 bytes per weight, twice
+// the TF32 rate) is preferred over TF32X3 when its split is present and K % 8 == 0.
 constexpr int64_t kAutoDecodeMaxM = 8;
 
-spl_path resolve(int64_t M, int64_t K, spl_path path, bool have_split) {
-  if (path == SPL_PATH_FP32 || path == SPL_PATH_TF32X3) return path;
-  if (M > kAutoDecodeMaxM && K >= 64 && have_split && tc_capable()) return SPL_PATH_TF32X3;
+bool has_tf32(const spl_weight& w) { return w.tf32_hi && w.tf32_lo; }
+bool has_f16(const spl_weight& w) { return w.f16_hi && w.f16_lo && w.f16_exp; }
+
+spl_path resolve(int64_t M, int64_t K, spl_path path, bool tf32, bool f16) {
+  if (path != SPL_PATH_AUTO) return path;
+  if (M > kAutoDecodeMaxM && K >= 64 && tc_capable()) {
+    if (f16 && (K & 7) == 0) return SPL_PATH_FP16X3;
+    if (tf32) return SPL_PATH_TF32X3;
+  }
   return SPL_PATH_FP32;
 }
 
+bool is_tc(spl_path p) { return p == SPL_PATH_TF32X3 || p == SPL_PATH_FP16X3; }
+
 Plan make_plan(int64_t M, int64_t K, int64_t N, spl_path resolved) {
   const int sms = device_sm_count();
-  if (resolved == SPL_PATH_TF32X3) return plan_tc(M, K, N, sms);
+  if (is_tc(resolved)) return plan_tc(M, K, N, sms, resolved);
   if (M <= kGemvMaxM) return plan_gemv(M, K, N, sms);
   return plan_simt(M, K, N, sms);
 }
 
-spl_status run_linear(float* out, const float* a, const float* W, const float* W_hi, const float* W_lo,
-                      const float* C, bool need_c, int64_t M, int64_t K, int64_t N, spl_path path, void* ws,
-                      size_t ws_bytes, cudaStream_t stream) {
+bool valid_path(spl_path p) {
+  return p == SPL_PATH_AUTO || p == SPL_PATH_TF32X3 || p == SPL_PATH_FP32 || p == SPL_PATH_FP16X3;
+}
+
+spl_status check_weight(const spl_weight* W, int64_t K) {
+  if (!W) return SPL_EINVAL;
+  if (K > 0 && !W->w) return SPL_EINVAL;
+  if (W->w && !aligned16(W->w)) return SPL_EALIGN;
+  if ((W->tf32_hi && !aligned16(W->tf32_hi)) || (W->tf32_lo && !aligned16(W->tf32_lo))) return SPL_EALIGN;
+  if ((W->f16_hi && !aligned16(W->f16_hi)) || (W->f16_lo && !aligned16(W->f16_lo))) return SPL_EALIGN;
+  return SPL_OK;
+}
+
+spl_status run_linear(float* out, const float* a, const spl_weight* W, const float* C, bool need_c, int64_t M,
+                      int64_t K, int64_t N, spl_path path, void* ws, size_t ws_bytes, cudaStream_t stream) {
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
-  if (path != SPL_PATH_AUTO && path != SPL_PATH_TF32X3 && path != SPL_PATH_FP32) return SPL_EINVAL;
+  if (!valid_path(path)) return SPL_EINVAL;
   if (M == 0 || N == 0) return SPL_OK;
   if (!out || (need_c && !C)) return SPL_EINVAL;
   if ((K & 3) != 0) return SPL_EALIGN;
-  if (K > 0 && (!a || !W)) return SPL_EINVAL;
-  if (!aligned16(out) || (a && !aligned16(a)) || (W && !aligned16(W)) || (C && !aligned16(C))) return SPL_EALIGN;
-  if ((W_hi && !aligned16(W_hi)) || (W_lo && !aligned16(W_lo))) return SPL_EALIGN;
+  spl_status st = check_weight(W, K);
+  if (st != SPL_OK) return st;
+  if (K > 0 && !a) return SPL_EINVAL;
+  if (!aligned16(out) || (a && !aligned16(a)) || (C && !aligned16(C))) return SPL_EALIGN;
   if (M > (int64_t(1) << 31) || N > (int64_t(1) << 31) || K > (int64_t(1) << 31)) return SPL_ESHAPE;
   if (K == 0) {  // empty reduction: the product is zero
     if (cudaMemsetAsync(out, 0, (size_t)(M * N) * sizeof(float), stream) != cudaSuccess) return SPL_ECUDA;
     return C ? spl_unmask(out, out, C, M, N, stream) : SPL_OK;
   }
-  const spl_path resolved = resolve(M, K, path, W_hi && W_lo);
-  if (resolved == SPL_PATH_TF32X3 && (!W_hi || !W_lo || !tc_capable())) return SPL_EUNSUPPORTED;
+  const spl_path resolved = resolve(M, K, path, has_tf32(*W), has_f16(*W));
+  if (resolved == SPL_PATH_TF32X3 && (!has_tf32(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
+  if (resolved == SPL_PATH_FP16X3 && (!has_f16(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
+  if (resolved == SPL_PATH_FP16X3 && (K & 7) != 0) return SPL_EALIGN;
   const Plan plan = make_plan(M, K, N, resolved);
   if (plan.total() > 0 && (!ws || ws_bytes < plan.total())) return SPL_EWORKSPACE;
   if (ws && !aligned16(ws)) return SPL_EALIGN;
-  LinearArgs args{out, a, W, W_hi, W_lo, C, M, K, N, ws, ws_bytes, stream};
+  const LinearArgs args = make_args(out, a, *W, C, M, K, N, ws, ws_bytes, stream, resolved);
   switch (plan.kernel) {
     case kKernelTc: return run_tc(args, plan);
     case kKernelGemv: return run_gemv(args, plan);
@@ -90,8 +115,9 @@ MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, sp
     const int s = tc_uniform_splits(order_rows, K, N);
     if (s <= 0) return mp;
     mp.splits = s;
+    mp.ws = resolved == SPL_PATH_FP16X3 ? kCounterBytes + tc_aexp_bytes(M, resolved) : 0;
     mp.ok = true;
-    return mp;  // no workspace
+    return mp;
   }
   mp.splits = online.splits;
   mp.k_per_split = online.k_per_split;
@@ -106,16 +132,53 @@ MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, sp
   return mp;
 }
 
+// Workspace of a product call for every path it could take (AUTO: all of them).
+size_t linear_ws(int64_t M, int64_t K, int64_t N, spl_path path) {
+  size_t need = 0;
+  const spl_path paths[3] = {SPL_PATH_FP32, SPL_PATH_TF32X3, SPL_PATH_FP16X3};
+  for (spl_path p : paths)
+    if (path == SPL_PATH_AUTO || path == p) need = std::max(need, make_plan(M, K, N, p).total());
+  return need;
+}
+
 }  // namespace
 }  // namespace spl
 
 using namespace spl;
 
+extern "C" spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path) {
+  (void)N;
+  return resolve(M, K, path, true, true);
+}
+
+extern "C" size_t spl_linear_workspace_bytes(int64_t M, int64_t K, int64_t N, spl_path path) {
+  if (M <= 0 || K <= 0 || N <= 0) return 0;
+  return linear_ws(M, K, N, path);
+}
+
+extern "C" spl_status spl_masked_linear(float* Yt, const float* Xt, const spl_weight* W, int64_t M, int64_t K,
+                                        int64_t N, spl_path path, void* workspace, size_t workspace_bytes,
+                                        cudaStream_t stream) {
+  return run_linear(Yt, Xt, W, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
+}
+
+extern "C" spl_status spl_precompute_noise_product(float* C, const float* Nz, const spl_weight* W, int64_t M,
+                                                   int64_t K, int64_t N, spl_path path, void* workspace,
+                                                   size_t workspace_bytes, cudaStream_t stream) {
+  return run_linear(C, Nz, W, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
+}
+
+extern "C" spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const spl_weight* W, const float* C,
+                                               int64_t M, int64_t K, int64_t N, spl_path path, void* workspace,
+                                               size_t workspace_bytes, cudaStream_t stream) {
+  return run_linear(Y, Xt, W, C, true, M, K, N, path, workspace, workspace_bytes, stream);
+}
+
 extern "C" size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows,
                                                          spl_path path) {
   if (M <= 0 || K <= 0 || N <= 0 || order_rows <= 0) return 0;
   size_t need = 0;
-  const spl_path paths[2] = {SPL_PATH_FP32, SPL_PATH_TF32X3};
+  const spl_path paths[3] = {SPL_PATH_FP32, SPL_PATH_TF32X3, SPL_PATH_FP16X3};
   for (spl_path p : paths) {
     if (path != SPL_PATH_AUTO && path != p) continue;
     const MatchedPlan mp = matched_plan(M, K, N, order_rows, p);
@@ -124,28 +187,30 @@ extern "C" size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, i
   return need;
 }
 
-extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const float* W,
-                                                           const float* W_hi, const float* W_lo, int64_t M, int64_t K,
-                                                           int64_t N, int64_t order_rows, spl_path path,
+extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const spl_weight* W, int64_t M,
+                                                           int64_t K, int64_t N, int64_t order_rows, spl_path path,
                                                            void* workspace, size_t workspace_bytes,
                                                            cudaStream_t stream) {
   if (order_rows <= 0) return SPL_EINVAL;
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
-  if (path != SPL_PATH_AUTO && path != SPL_PATH_TF32X3 && path != SPL_PATH_FP32) return SPL_EINVAL;
+  if (!valid_path(path)) return SPL_EINVAL;
   if (M == 0 || N == 0 || K == 0)
-    return run_linear(C, Nz, W, W_hi, W_lo, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
-  if (!C || !Nz || !W) return SPL_EINVAL;
+    return run_linear(C, Nz, W, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
+  if (!C || !Nz) return SPL_EINVAL;
+  spl_status st = check_weight(W, K);
+  if (st != SPL_OK) return st;
   if ((K & 3) != 0) return SPL_EALIGN;
-  if (!aligned16(C) || !aligned16(Nz) || !aligned16(W)) return SPL_EALIGN;
-  if ((W_hi && !aligned16(W_hi)) || (W_lo && !aligned16(W_lo))) return SPL_EALIGN;
-  const spl_path resolved = resolve(order_rows, K, path, W_hi && W_lo);
-  if (resolved == SPL_PATH_TF32X3 && (!W_hi || !W_lo || !tc_capable())) return SPL_EUNSUPPORTED;
+  if (!aligned16(C) || !aligned16(Nz)) return SPL_EALIGN;
+  const spl_path resolved = resolve(order_rows, K, path, has_tf32(*W), has_f16(*W));
+  if (resolved == SPL_PATH_TF32X3 && (!has_tf32(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
+  if (resolved == SPL_PATH_FP16X3 && (!has_f16(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
+  if (resolved == SPL_PATH_FP16X3 && (K & 7) != 0) return SPL_EALIGN;
   const MatchedPlan mp = matched_plan(M, K, N, order_rows, resolved);
   if (!mp.ok)  // the masked call's order cannot be reproduced: plain correction
-    return run_linear(C, Nz, W, W_hi, W_lo, nullptr, false, M, K, N, resolved, workspace, workspace_bytes, stream);
+    return run_linear(C, Nz, W, nullptr, false, M, K, N, resolved, workspace, workspace_bytes, stream);
   if (mp.ws > 0 && (!workspace || workspace_bytes < mp.ws)) return SPL_EWORKSPACE;
   if (workspace && !aligned16(workspace)) return SPL_EALIGN;
-  LinearArgs args{C, Nz, W, W_hi, W_lo, nullptr, M, K, N, workspace, workspace_bytes, stream};
+  const LinearArgs args = make_args(C, Nz, *W, nullptr, M, K, N, workspace, workspace_bytes, stream, resolved);
   if (mp.kernel == kKernelTc) return run_tc_splits(args, mp.splits);
   Plan p{};
   p.kernel = mp.kernel;
@@ -157,44 +222,11 @@ extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float
   }
   for (int64_t r0 = 0; r0 < M; r0 += mp.chunk_rows) {  // decode kernel: at most 16 rows per launch
     const int64_t rows = std::min<int64_t>(mp.chunk_rows, M - r0);
-    LinearArgs ca{C + r0 * N, Nz + r0 * K, W, W_hi, W_lo, nullptr, rows, K, N, workspace, workspace_bytes, stream};
+    const LinearArgs ca = make_args(C + r0 * N, Nz + r0 * K, *W, nullptr, rows, K, N, workspace, workspace_bytes,
+                                    stream, resolved);
     p.ws_partials = mp.splits > 1 ? (size_t)round_up((int64_t)mp.splits * rows * N * 4, 256) : 0;
-    const spl_status st = run_gemv(ca, p);
+    st = run_gemv(ca, p);
     if (st != SPL_OK) return st;
   }
   return SPL_OK;
-}
-
-extern "C" spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path) {
-  (void)N;
-  return resolve(M, K, path, true);
-}
-
-extern "C" size_t spl_linear_workspace_bytes(int64_t M, int64_t K, int64_t N, spl_path path) {
-  if (M <= 0 || K <= 0 || N <= 0) return 0;
-  size_t need = 0;
-  if (path == SPL_PATH_AUTO || path == SPL_PATH_FP32) need = std::max(need, make_plan(M, K, N, SPL_PATH_FP32).total());
-  if (path == SPL_PATH_AUTO || path == SPL_PATH_TF32X3)
-    need = std::max(need, make_plan(M, K, N, SPL_PATH_TF32X3).total());
-  return need;
-}
-
-extern "C" spl_status spl_masked_linear(float* Yt, const float* Xt, const float* W, const float* W_hi,
-                                        const float* W_lo, int64_t M, int64_t K, int64_t N, spl_path path,
-                                        void* workspace, size_t workspace_bytes, cudaStream_t stream) {
-  return run_linear(Yt, Xt, W, W_hi, W_lo, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
-}
-
-extern "C" spl_status spl_precompute_noise_product(float* C, const float* Nz, const float* W, const float* W_hi,
-                                                   const float* W_lo, int64_t M, int64_t K, int64_t N,
-                                                   spl_path path, void* workspace, size_t workspace_bytes,
-                                                   cudaStream_t stream) {
-  return run_linear(C, Nz, W, W_hi, W_lo, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
-}
-
-extern "C" spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const float* W, const float* W_hi,
-                                               const float* W_lo, const float* C, int64_t M, int64_t K, int64_t N,
-                                               spl_path path, void* workspace, size_t workspace_bytes,
-                                               cudaStream_t stream) {
-  return run_linear(Y, Xt, W, W_hi, W_lo, C, true, M, K, N, path, workspace, workspace_bytes, stream);
 }

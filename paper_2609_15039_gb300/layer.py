@@ -36,8 +36,7 @@ class GroupWeights:
     names: list          # projections in column order
     widths: list         # output width of each projection
     W: torch.Tensor      # [sum(widths), K]
-    W_hi: torch.Tensor = None
-    W_lo: torch.Tensor = None
+    wt: spl.Weight = None  # W with the splits the tensor-core paths read
 
     @property
     def N(self):
@@ -65,15 +64,13 @@ class MaskedLayer:
 
     @classmethod
     def from_weights(cls, model, weights, split=True, device="cuda"):
-        """weights: {projection: [N, K] fp32}.  Concatenates per input group; splits for TF32X3."""
+        """weights: {projection: [N, K] fp32}.  Concatenates per input group; splits for TF32X3 and FP16X3."""
         groups = []
         for g, K, names in model.input_groups():
             parts = [weights[n].to(device=device, dtype=torch.float32) for n in names]
             W = torch.cat(parts, dim=0).contiguous() if len(parts) > 1 else parts[0].contiguous()
             gw = GroupWeights(g, K, list(names), [p.shape[0] for p in parts], W)
-            if split:
-                gw.W_hi, gw.W_lo = torch.empty_like(W), torch.empty_like(W)
-                spl.spl_split_tf32(gw.W_hi, gw.W_lo, W)
+            gw.wt = spl.Weight.prepare(W) if split else spl.Weight(W)
             groups.append(gw)
         return cls(model, groups)
 
@@ -108,7 +105,7 @@ class MaskedLayer:
         return self.deltas
 
     def calibrate(self, inputs, eps, mech, seed, rows=128):
-        """a8: choose TF32X3 or FP32 per group from the bound on a masked sample (spl_choose_path).
+        """a8: choose FP16X3, TF32X3 or FP32 per group from the bound on a masked sample (spl_choose_path).
 
         The sample is the first ``rows`` rows of each group's input with a fresh mask drawn
         under a stream id no online step uses.
@@ -117,9 +114,9 @@ class MaskedLayer:
             X = inputs[g.name][:rows].contiguous()
             eta = torch.empty_like(X)
             spl.spl_noise(eta, self.deltas[g.name], eps, mech, seed, stream_id=1000 + gi)
-            name, st_tc, st_fp = spl.spl_choose_path(X, eta, g.W, g.W_hi, g.W_lo)
+            name, stats = spl.spl_choose_path(X, eta, g.wt)
             self.paths[g.name] = name
-            self.calibration[g.name] = {"path": name, "tf32x3": st_tc, "fp32": st_fp, "rows": X.shape[0]}
+            self.calibration[g.name] = {"path": name, "rows": X.shape[0], **stats}
         return self.paths
 
     def path_of(self, g, path, rows):
@@ -161,13 +158,12 @@ class MaskedLayer:
             spl.spl_noise(b["eta"], self.deltas[g.name], eps, mech, seed, stream_id=gi,
                           offset=self.block_offset(g, cycle, 0), stream=stream)
             if timer:
-                timer("begin", "precompute")
+                timer("begin", "precompute", g.name)
             # summed in the order the online product of M rows uses, so their rounding cancels
-            spl.spl_precompute_noise_product_matched(b["C"], b["eta"], g.W, self.M, g.W_hi, g.W_lo,
-                                                     path=self.path_of(g, path, self.M), workspace=self.workspace,
-                                                     stream=stream)
+            spl.spl_precompute_noise_product_matched(b["C"], b["eta"], g.wt, self.M, path=self.path_of(g, path, self.M),
+                                                     workspace=self.workspace, stream=stream)
             if timer:
-                timer("end", "precompute")
+                timer("end", "precompute", g.name)
 
     def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None):
         """a3 + a5 + a6 for draw d: regenerate eta_d, mask, masked product with fused unmask.
@@ -181,11 +177,11 @@ class MaskedLayer:
             spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
                                offset=self.block_offset(g, cycle, d), stream=stream)
             if timer:
-                timer("begin", "masked_linear_unmask")
-            spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M], g.W_hi, g.W_lo,
-                                         path=self.path_of(g, path, M), workspace=self.workspace, stream=stream)
+                timer("begin", "masked_linear_unmask", g.name)
+            spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M], path=self.path_of(g, path, M),
+                                         workspace=self.workspace, stream=stream)
             if timer:
-                timer("end", "masked_linear_unmask")
+                timer("end", "masked_linear_unmask", g.name)
             out[g.name] = b["Y"]
         return out
 

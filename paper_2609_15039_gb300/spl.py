@@ -18,9 +18,10 @@ LIB_PATH = os.path.join(_HERE, "libspl.so")
 
 SPL_OK, SPL_EINVAL, SPL_ESHAPE, SPL_EALIGN, SPL_ECUDA, SPL_ETIMEOUT, SPL_EUNSUPPORTED, SPL_EWORKSPACE = range(8)
 SPL_MECH_LAPLACE, SPL_MECH_GAUSSIAN = 0, 1
-SPL_PATH_AUTO, SPL_PATH_TF32X3, SPL_PATH_FP32 = 0, 1, 2
+SPL_PATH_AUTO, SPL_PATH_TF32X3, SPL_PATH_FP32, SPL_PATH_FP16X3 = 0, 1, 2, 3
 MECHS = {"laplace": SPL_MECH_LAPLACE, "gaussian": SPL_MECH_GAUSSIAN}
-PATHS = {"auto": SPL_PATH_AUTO, "tf32x3": SPL_PATH_TF32X3, "fp32": SPL_PATH_FP32}
+PATHS = {"auto": SPL_PATH_AUTO, "tf32x3": SPL_PATH_TF32X3, "fp32": SPL_PATH_FP32, "fp16x3": SPL_PATH_FP16X3}
+PATH_NAMES = {v: k for k, v in PATHS.items()}
 
 
 class SplError(RuntimeError):
@@ -33,7 +34,13 @@ class spl_rng(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("stream_id", ctypes.c_uint64), ("offset", ctypes.c_uint64)]
 
 
+class spl_weight(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("tf32_hi", ctypes.c_void_p), ("tf32_lo", ctypes.c_void_p),
+                ("f16_hi", ctypes.c_void_p), ("f16_lo", ctypes.c_void_p), ("f16_exp", ctypes.c_void_p)]
+
+
 _P = ctypes.c_void_p
+_PW = ctypes.POINTER(spl_weight)
 _I64 = ctypes.c_int64
 _D = ctypes.c_double
 _I = ctypes.c_int
@@ -44,14 +51,15 @@ _SIGS = {
     "spl_mask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_noise_mask": (_I, [_P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_split_tf32": (_I, [_P, _P, _P, _I64, _P]),
+    "spl_split_fp16": (_I, [_P, _P, _P, _P, _I64, _I64, _P]),
     "spl_resolve_path": (_I, [_I64, _I64, _I64, _I]),
     "spl_linear_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I]),
-    "spl_masked_linear": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
-    "spl_precompute_noise_product": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_masked_linear": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_precompute_noise_product": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_precompute_matched_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I64, _I]),
-    "spl_precompute_noise_product_matched": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_precompute_noise_product_matched": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
-    "spl_masked_linear_unmask": (_I, [_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_masked_linear_unmask": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_masked_linear_unmask_noalloc": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P]),
     "spl_delta_layernorm": (_D, [_P, _I64]),
     "spl_delta_attention": (_D, [_P, _I64, _D]),
@@ -59,9 +67,9 @@ _SIGS = {
     "spl_spectral_norm": (_I, [ctypes.POINTER(ctypes.c_double), _P, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_bound_check": (_I, [ctypes.POINTER(ctypes.c_double), _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
     "spl_choose_path_workspace_bytes": (_SZ, [_I64, _I64, _I64]),
-    "spl_choose_path": (_I, [ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double),
-                             ctypes.POINTER(ctypes.c_double), _P, _P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
-    "spl_test_tc_wait_timeout": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _I64, _P]),
+    "spl_choose_path": (_I, [ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double), _P, _P, _PW, _I64,
+                             _I64, _I64, _P, _SZ, _P]),
+    "spl_test_tc_wait_timeout": (_I, [_P, _P, _PW, _I64, _I64, _I64, _P]),
     "spl_get_device_status": (_I, [_P]),
     "spl_launch_count": (ctypes.c_uint64, []),
     "spl_status_string": (ctypes.c_char_p, [_I]),
@@ -102,13 +110,13 @@ def _stream(stream):
     return ctypes.c_void_p(int(stream))
 
 
-def _dev(t, name):
+def _dev(t, name, dtype=torch.float32):
     if t is None:
         return None
     if not isinstance(t, torch.Tensor) or not t.is_cuda:
         raise TypeError(f"{name} must be a CUDA tensor")
-    if t.dtype != torch.float32 and name != "workspace":
-        raise TypeError(f"{name} must be float32")
+    if t.dtype != dtype and name != "workspace":
+        raise TypeError(f"{name} must be {dtype}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     return ctypes.c_void_p(t.data_ptr())
@@ -164,6 +172,60 @@ def spl_split_tf32(hi, lo, src, stream=None):
            "spl_split_tf32")
 
 
+def spl_split_fp16(hi, lo, row_exp, src, stream=None):
+    """hi, lo: int16 [rows, cols] (binary16 bit patterns); row_exp: int32 [rows]."""
+    rows, cols = _rows_cols(src)
+    if hi.numel() != rows * cols or lo.numel() != rows * cols or row_exp.numel() != rows:
+        raise ValueError("spl_split_fp16: shape mismatch")
+    _check(lib().spl_split_fp16(_dev(hi, "hi", torch.int16), _dev(lo, "lo", torch.int16),
+                                _dev(row_exp, "row_exp", torch.int32), _dev(src, "src"), rows, cols, _stream(stream)),
+           "spl_split_fp16")
+
+
+class Weight:
+    """A device weight W [N, K] (fp32) with the splits the tensor-core paths read (spl_weight).
+
+    ``Weight.prepare(W)`` runs the library's split kernels once; the splits live as long as
+    this object.  A plain tensor passed where a weight is expected carries no split (FP32
+    path only)."""
+
+    def __init__(self, w, tf32_hi=None, tf32_lo=None, f16_hi=None, f16_lo=None, f16_exp=None):
+        self.w, self.tf32_hi, self.tf32_lo = w, tf32_hi, tf32_lo
+        self.f16_hi, self.f16_lo, self.f16_exp = f16_hi, f16_lo, f16_exp
+
+    @classmethod
+    def prepare(cls, w, tf32=True, fp16=True, stream=None):
+        out = cls(w)
+        if tf32:
+            out.tf32_hi, out.tf32_lo = torch.empty_like(w), torch.empty_like(w)
+            spl_split_tf32(out.tf32_hi, out.tf32_lo, w, stream=stream)
+        if fp16 and w.shape[-1] % 8 == 0:
+            out.f16_hi = torch.empty(w.shape, dtype=torch.int16, device=w.device)
+            out.f16_lo = torch.empty_like(out.f16_hi)
+            out.f16_exp = torch.empty(w.shape[0], dtype=torch.int32, device=w.device)
+            spl_split_fp16(out.f16_hi, out.f16_lo, out.f16_exp, w, stream=stream)
+        return out
+
+    @property
+    def shape(self):
+        return self.w.shape
+
+    def rows(self, a, b):
+        """Rows a:b (output columns a:b of the product) as a Weight of views."""
+        sl = lambda t: None if t is None else t[a:b]
+        return Weight(self.w[a:b], sl(self.tf32_hi), sl(self.tf32_lo), sl(self.f16_hi), sl(self.f16_lo),
+                      sl(self.f16_exp))
+
+    def c_struct(self):
+        return spl_weight(_dev(self.w, "W"), _dev(self.tf32_hi, "W.tf32_hi"), _dev(self.tf32_lo, "W.tf32_lo"),
+                          _dev(self.f16_hi, "W.f16_hi", torch.int16), _dev(self.f16_lo, "W.f16_lo", torch.int16),
+                          _dev(self.f16_exp, "W.f16_exp", torch.int32))
+
+
+def _weight(W):
+    return W if isinstance(W, Weight) else Weight(W)
+
+
 def spl_resolve_path(M, K, N, path="auto"):
     return lib().spl_resolve_path(M, K, N, _path(path))
 
@@ -183,41 +245,45 @@ def _ws(ws):
     return _dev(ws, "workspace"), ws.numel() * ws.element_size()
 
 
-def _linear(fn, name, out, a, W, W_hi, W_lo, C, path, ws, stream):
+def _linear(fn, name, out, a, W, C, path, ws, stream):
+    W = _weight(W)
     M, K = _rows_cols(a)
     N = W.shape[0]
     if W.shape[-1] != K or out.numel() != M * N or (C is not None and C.numel() != M * N):
         raise ValueError(f"{name}: shape mismatch")
     wsp, wsb = _ws(ws)
-    args = [_dev(out, "out"), _dev(a, "input"), _dev(W, "W"), _dev(W_hi, "W_hi"), _dev(W_lo, "W_lo")]
-    if C is not None or name == "spl_masked_linear_unmask":
+    ws_ = W.c_struct()
+    args = [_dev(out, "out"), _dev(a, "input"), ctypes.byref(ws_)]
+    if name == "spl_masked_linear_unmask":
         args.append(_dev(C, "C"))
     _check(fn(*args, M, K, N, _path(path), wsp, wsb, _stream(stream)), name)
 
 
-def spl_masked_linear(Yt, Xt, W, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
-    _linear(lib().spl_masked_linear, "spl_masked_linear", Yt, Xt, W, W_hi, W_lo, None, path, workspace, stream)
+def spl_masked_linear(Yt, Xt, W, path="auto", workspace=None, stream=None):
+    """W: a Weight (or a plain fp32 tensor for the FP32 path)."""
+    _linear(lib().spl_masked_linear, "spl_masked_linear", Yt, Xt, W, None, path, workspace, stream)
 
 
-def spl_precompute_noise_product(C, Nz, W, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
-    _linear(lib().spl_precompute_noise_product, "spl_precompute_noise_product", C, Nz, W, W_hi, W_lo, None, path,
-            workspace, stream)
+def spl_precompute_noise_product(C, Nz, W, path="auto", workspace=None, stream=None):
+    _linear(lib().spl_precompute_noise_product, "spl_precompute_noise_product", C, Nz, W, None, path, workspace,
+            stream)
 
 
 def spl_precompute_matched_workspace_bytes(M, K, N, order_rows, path="auto"):
     return int(lib().spl_precompute_matched_workspace_bytes(M, K, N, order_rows, _path(path)))
 
 
-def spl_precompute_noise_product_matched(C, Nz, W, order_rows, W_hi=None, W_lo=None, path="auto", workspace=None,
-                                         stream=None):
+def spl_precompute_noise_product_matched(C, Nz, W, order_rows, path="auto", workspace=None, stream=None):
+    W = _weight(W)
     M, K = _rows_cols(Nz)
     N = W.shape[0]
     if W.shape[-1] != K or C.numel() != M * N:
         raise ValueError("spl_precompute_noise_product_matched: shape mismatch")
     wsp, wsb = _ws(workspace)
-    _check(lib().spl_precompute_noise_product_matched(_dev(C, "C"), _dev(Nz, "Nz"), _dev(W, "W"), _dev(W_hi, "W_hi"),
-                                                      _dev(W_lo, "W_lo"), M, K, N, int(order_rows), _path(path), wsp,
-                                                      wsb, _stream(stream)), "spl_precompute_noise_product_matched")
+    ws_ = W.c_struct()
+    _check(lib().spl_precompute_noise_product_matched(_dev(C, "C"), _dev(Nz, "Nz"), ctypes.byref(ws_), M, K, N,
+                                                      int(order_rows), _path(path), wsp, wsb, _stream(stream)),
+           "spl_precompute_noise_product_matched")
 
 
 def spl_unmask(Y, Yt, C, stream=None):
@@ -225,9 +291,8 @@ def spl_unmask(Y, Yt, C, stream=None):
     _check(lib().spl_unmask(_dev(Y, "Y"), _dev(Yt, "Yt"), _dev(C, "C"), rows, cols, _stream(stream)), "spl_unmask")
 
 
-def spl_masked_linear_unmask(Y, Xt, W, C, W_hi=None, W_lo=None, path="auto", workspace=None, stream=None):
-    _linear(lib().spl_masked_linear_unmask, "spl_masked_linear_unmask", Y, Xt, W, W_hi, W_lo, C, path, workspace,
-            stream)
+def spl_masked_linear_unmask(Y, Xt, W, C, path="auto", workspace=None, stream=None):
+    _linear(lib().spl_masked_linear_unmask, "spl_masked_linear_unmask", Y, Xt, W, C, path, workspace, stream)
 
 
 def spl_masked_linear_unmask_noalloc(Y, Xt, W, C, stream=None):
@@ -300,27 +365,29 @@ def spl_bound_check(Y, X, Xt, Nz, W, stream=None):
     return _stats_dict(stats)
 
 
-def spl_choose_path(X, Nz, W, W_hi=None, W_lo=None, stream=None):
-    """a8: returns (chosen path name, stats of TF32X3, stats of FP32) for the sample X + Nz."""
+def spl_choose_path(X, Nz, W, stream=None):
+    """a8: returns (chosen path name, {path name: stats}) for the sample X + Nz (W: a Weight)."""
+    W = _weight(W)
     rows, K = _rows_cols(X)
     N = W.shape[0]
     nbytes = int(lib().spl_choose_path_workspace_bytes(rows, K, N))
     ws = workspace(nbytes, X.device)
     chosen = ctypes.c_int(0)
-    a = (ctypes.c_double * 9)()
-    b = (ctypes.c_double * 9)()
-    _check(lib().spl_choose_path(ctypes.byref(chosen), a, b, _dev(X, "X"), _dev(Nz, "Nz"), _dev(W, "W"),
-                                 _dev(W_hi, "W_hi"), _dev(W_lo, "W_lo"), rows, K, N, _dev(ws, "workspace"), nbytes,
-                                 _stream(stream)), "spl_choose_path")
-    name = {SPL_PATH_TF32X3: "tf32x3", SPL_PATH_FP32: "fp32"}.get(chosen.value, str(chosen.value))
-    return name, _stats_dict(a), _stats_dict(b)
+    st = (ctypes.c_double * 27)()
+    ws_ = W.c_struct()
+    _check(lib().spl_choose_path(ctypes.byref(chosen), st, _dev(X, "X"), _dev(Nz, "Nz"), ctypes.byref(ws_), rows, K,
+                                 N, _dev(ws, "workspace"), nbytes, _stream(stream)), "spl_choose_path")
+    stats = {name: _stats_dict(st[9 * i:9 * (i + 1)]) for i, name in enumerate(("fp32", "tf32x3", "fp16x3"))}
+    return PATH_NAMES.get(chosen.value, str(chosen.value)), stats
 
 
-def spl_test_tc_wait_timeout(out, A, W, W_hi, W_lo, stream=None):
+def spl_test_tc_wait_timeout(out, A, W, stream=None):
+    W = _weight(W)
     M, K = _rows_cols(A)
     N = W.shape[0]
-    _check(lib().spl_test_tc_wait_timeout(_dev(out, "out"), _dev(A, "A"), _dev(W, "W"), _dev(W_hi, "W_hi"),
-                                          _dev(W_lo, "W_lo"), M, K, N, _stream(stream)), "spl_test_tc_wait_timeout")
+    ws_ = W.c_struct()
+    _check(lib().spl_test_tc_wait_timeout(_dev(out, "out"), _dev(A, "A"), ctypes.byref(ws_), M, K, N,
+                                          _stream(stream)), "spl_test_tc_wait_timeout")
 
 
 def spl_launch_count():

@@ -69,29 +69,44 @@ def test_argument_validation_without_launch(spl):
     assert L.spl_noise(None, 0, 5, 1.0, 1.0, 0, rng, None) == spl.SPL_OK
     assert L.spl_mask(None, None, None, 3, 0, None) == spl.SPL_OK
     assert L.spl_unmask(None, None, None, 0, 0, None) == spl.SPL_OK
-    assert L.spl_masked_linear(None, None, None, None, None, 0, 8, 8, 0, None, 0, None) == spl.SPL_OK
+    assert L.spl_masked_linear(None, None, None, 0, 8, 8, 0, None, 0, None) == spl.SPL_OK
     # negative sizes, bad path, NULL operands, K % 4
-    assert L.spl_masked_linear(None, None, None, None, None, -1, 8, 8, 0, None, 0, None) == spl.SPL_EINVAL
-    assert L.spl_masked_linear(None, None, None, None, None, 4, 8, 8, 9, None, 0, None) == spl.SPL_EINVAL
-    assert L.spl_masked_linear(None, None, None, None, None, 4, 8, 8, 0, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_masked_linear(None, None, None, -1, 8, 8, 0, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_masked_linear(None, None, None, 4, 8, 8, 9, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_masked_linear(None, None, None, 4, 8, 8, 0, None, 0, None) == spl.SPL_EINVAL
     buf = (ctypes.c_float * 64)()
     p = ctypes.cast(buf, ctypes.c_void_p).value
     base = p + (16 - p % 16) % 16
-    assert L.spl_masked_linear(base, base, base, None, None, 2, 6, 2, 2, None, 0, None) == spl.SPL_EALIGN
-    assert L.spl_masked_linear(base + 4, base, base, None, None, 2, 8, 2, 2, None, 0, None) == spl.SPL_EALIGN
-    assert L.spl_masked_linear_unmask(base, base, base, None, None, None, 2, 8, 2, 2, None, 0, None) == spl.SPL_EINVAL
+    w = spl.spl_weight(base, None, None, None, None, None)
+    assert L.spl_masked_linear(base, base, None, 2, 8, 2, 2, None, 0, None) == spl.SPL_EINVAL  # no weight
+    assert L.spl_masked_linear(base, base, ctypes.byref(w), 2, 6, 2, 2, None, 0, None) == spl.SPL_EALIGN
+    assert L.spl_masked_linear(base + 4, base, ctypes.byref(w), 2, 8, 2, 2, None, 0, None) == spl.SPL_EALIGN
+    w_bad = spl.spl_weight(base, None, None, base + 2, base, base)
+    assert L.spl_masked_linear(base, base, ctypes.byref(w_bad), 2, 8, 2, 2, None, 0, None) == spl.SPL_EALIGN
+    assert L.spl_masked_linear_unmask(base, base, ctypes.byref(w), None, 2, 8, 2, 2, None, 0, None) == spl.SPL_EINVAL
     assert L.spl_random_bits(None, -1, rng, None) == spl.SPL_EINVAL
     assert L.spl_split_tf32(base + 4, base, base, 4, None) == spl.SPL_EALIGN
+    assert L.spl_split_fp16(base, base, base, base, 2, 12, None) == spl.SPL_EALIGN  # cols % 8
+    assert L.spl_split_fp16(base, base, None, base, 2, 8, None) == spl.SPL_EINVAL
+    assert L.spl_split_fp16(None, None, None, None, 0, 8, None) == spl.SPL_OK
+    stats = (ctypes.c_double * 27)()
+    chosen = ctypes.c_int(5)
+    assert L.spl_choose_path(ctypes.byref(chosen), stats, base, base, None, 4, 8, 8, None, 0, None) == spl.SPL_EINVAL
+    assert chosen.value == spl.SPL_PATH_FP32
 
 
 def test_workspace_sizes_are_consistent(spl):
     # decode shapes need split-K partials after the 64 KiB counter region; the TF32X3 kernel
-    # splits its left operand in shared memory and reduces split-K in a cluster: no workspace
+    # splits its left operand in shared memory and reduces split-K in a cluster: no workspace;
+    # FP16X3 keeps one power-of-two exponent per row of the left operand after the counters
     for M, K, N in [(1, 3072, 3072), (16, 8192, 3072), (128, 3072, 1024), (2048, 2560, 9728)]:
         auto = spl.spl_linear_workspace_bytes(M, K, N, "auto")
         assert auto >= spl.spl_linear_workspace_bytes(M, K, N, "fp32")
         assert auto >= spl.spl_linear_workspace_bytes(M, K, N, "tf32x3")
+        assert auto >= spl.spl_linear_workspace_bytes(M, K, N, "fp16x3")
         assert spl.spl_linear_workspace_bytes(M, K, N, "tf32x3") == 0
+        assert spl.spl_linear_workspace_bytes(M, K, N, "fp16x3") >= 64 * 1024 + 4 * M
+        assert spl.spl_precompute_matched_workspace_bytes(8 * M, K, N, M, "fp16x3") >= 64 * 1024 + 32 * M
     assert spl.spl_linear_workspace_bytes(1, 3072, 3072, "fp32") > 64 * 1024
     assert spl.spl_linear_workspace_bytes(0, 8, 8) == 0
 

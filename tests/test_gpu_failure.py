@@ -32,12 +32,11 @@ def test_bounded_wait_times_out_and_context_survives(spl):
     W = wl.weight(N, K, seed=1).numpy()
     A = wl.activations(M, K, seed=2).numpy()
     Wd, Ad = torch.as_tensor(W).cuda(), torch.as_tensor(A).cuda()
-    hi, lo = torch.empty_like(Wd), torch.empty_like(Wd)
-    spl.spl_split_tf32(hi, lo, Wd)
+    Wt = spl.Weight.prepare(Wd)
     assert spl.spl_get_device_status() == spl.SPL_OK
     out = torch.empty((M, N), device="cuda")
     t0 = time.time()
-    spl.spl_test_tc_wait_timeout(out, Ad, Wd, hi, lo)
+    spl.spl_test_tc_wait_timeout(out, Ad, Wt)
     st = spl.spl_get_device_status()  # synchronises
     elapsed = time.time() - t0
     assert st == spl.SPL_ETIMEOUT, spl.status_string(st)
@@ -45,7 +44,7 @@ def test_bounded_wait_times_out_and_context_survives(spl):
     assert spl.spl_get_device_status() == spl.SPL_OK  # reading the status clears it
     # the context is still usable: a normal product is correct
     Y = torch.empty((M, N), device="cuda")
-    spl.spl_masked_linear(Y, Ad, Wd, hi, lo, path="tf32x3")
+    spl.spl_masked_linear(Y, Ad, Wt, path="tf32x3")
     torch.cuda.synchronize()
     assert_product_close(f32(Y), A, W, "tf32x3", what="after timeout")
     assert spl.spl_get_device_status() == spl.SPL_OK

@@ -150,3 +150,37 @@ def test_mask_alone_1e9_sampled(spl, mech):
         tol = 8 * 2.0 ** -24 * b * np.sqrt(-2 * np.log(u1)) + 2 * np.spacing(np.abs(eta.astype(np.float32)))
     exp = linear.mask(x, eta.astype(np.float32)).astype(np.float64)
     assert np.all(np.abs(xt - exp) <= tol + np.spacing(np.abs(exp.astype(np.float32))).astype(np.float64))
+
+
+@pytest.mark.parametrize("M", [512, 1])
+def test_llama_lm_head(spl, M):
+    """The LM head (3072 -> 128256, Sec. 5.1, after the final RMSNorm: Delta from Thm. 1) at
+    prefill and decode sizes, with a bank of 8 corrections summed in the online order."""
+    model = wl.LLAMA_3_2_3B
+    K, N, draws, eps, mech, seed = model.d_model, model.vocab, 8, 1.0, "gaussian", 606
+    W = wl.weight(N, K, seed=9001, device="cuda")
+    Wt = spl.Weight.prepare(W)
+    X = wl.activations(M, K, seed=9002, device="cuda")
+    delta = osens.delta_layernorm(np.ones(K))
+    eta = torch.empty((draws * M, K), device="cuda")
+    spl.spl_noise(eta, delta, eps, mech, seed)
+    C = torch.empty((draws * M, N), device="cuda")
+    ws = spl.workspace(max(spl.spl_precompute_matched_workspace_bytes(draws * M, K, N, M),
+                           spl.spl_linear_workspace_bytes(M, K, N)))
+    spl.spl_precompute_noise_product_matched(C, eta, Wt, M, workspace=ws)
+    d = 3
+    Xt = torch.empty_like(X)
+    spl.spl_noise_mask(Xt, None, X, delta, eps, mech, seed, offset=d * M * K // 4)
+    Y = torch.empty((M, N), device="cuda")
+    spl.spl_masked_linear_unmask(Y, Xt, Wt, C[d * M:(d + 1) * M], workspace=ws)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(M)
+    rows = np.sort(rng.choice(M, size=min(8, M), replace=False))
+    cols = np.sort(rng.choice(N, size=256, replace=False))
+    Xs = X[torch.as_tensor(rows, device="cuda")].cpu().numpy()
+    eta_s = np.stack([philox.noise((1, K), delta, eps, mech, seed, offset=(d * M + int(m)) * K // 4)[0] for m in rows])
+    Ws = W[torch.as_tensor(cols, device="cuda")].cpu().numpy()
+    S = linear.abs_products(Xs, linear.mask(Xs, eta_s), eta_s, Ws)
+    got = Y[torch.as_tensor(rows, device="cuda")][:, torch.as_tensor(cols, device="cuda")].double().cpu().numpy()
+    err = np.abs(got - linear.reference_output(Xs, Ws))
+    assert np.all(err <= bounds.hard_bound(*S, K) * (1 + 1e-5))

@@ -160,51 +160,106 @@ def test_split_tf32_properties(spl):
 
 # ------------------------------------------------ a4/a5/a6: products
 def _weights(spl, N, K, seed):
+    """Host W and the device Weight with both splits (the fp16 one when K % 8 == 0)."""
     W = wl.weight(N, K, seed=seed).numpy()
-    Wd = dev(W)
-    hi, lo = torch.empty_like(Wd), torch.empty_like(Wd)
-    spl.spl_split_tf32(hi, lo, Wd)
-    return W, Wd, hi, lo
+    return W, spl.Weight.prepare(dev(W))
+
+
+def _fp16_bits(x):
+    return np.asarray(x, dtype=np.float16).view(np.int16)
+
+
+def test_split_fp16_properties(spl):
+    """hi = fp16(w 2^e), lo = fp16(w 2^e - hi) per row; e puts the row's largest |w| in [2^14, 2^15)."""
+    W = wl.weight(37, 1032, seed=6).numpy()
+    W[1] = 0.0                                  # all-zero row: e = 0, hi = lo = 0
+    W[2] *= np.float32(1e-30)                   # tiny row (residuals below fp16's normal range)
+    W[3] *= np.float32(1e30)                    # huge row
+    W[4, :4] = [1.0, 1.0 + 2.0 ** -11, -(1.0 + 3 * 2.0 ** -11), 2.0 ** -30]  # fp16 ties at 1 (ulp 2^-10)
+    W[4, 4:] = 0.0
+    hi = torch.empty(W.shape, dtype=torch.int16, device="cuda")
+    lo = torch.empty_like(hi)
+    ex = torch.empty(W.shape[0], dtype=torch.int32, device="cuda")
+    spl.spl_split_fp16(hi, lo, ex, dev(W))
+    e = ex.cpu().numpy()
+    h = hi.cpu().numpy().view(np.float16).astype(np.float64)
+    l = lo.cpu().numpy().view(np.float16).astype(np.float64)
+    amax = np.abs(W.astype(np.float64)).max(axis=1)
+    assert e[1] == 0 and not h[1].any() and not l[1].any()
+    nz = amax > 0
+    scaled_max = amax[nz] * np.exp2(e[nz].astype(np.float64))
+    assert np.all((scaled_max >= 2.0 ** 14) & (scaled_max < 2.0 ** 15))
+    Ws = W.astype(np.float64) * np.exp2(e.astype(np.float64))[:, None]  # exact: power-of-two scaling
+    # numpy's float16 cast rounds to nearest even, the kernel's __float2half_rn too
+    np.testing.assert_array_equal(hi.cpu().numpy(), _fp16_bits(Ws))
+    np.testing.assert_array_equal(lo.cpu().numpy(), _fp16_bits(Ws - h))
+    assert np.all(np.abs(Ws - h - l) <= 2.0 ** -22 * np.abs(Ws) + 2.0 ** -25)
+    assert e[4] == 14 and h[4, 1] == 2.0 ** 14  # 2^14 (1 + 2^-11) ties to even (2^14)
 
 
 SHAPES = [(1, 4, 1), (3, 8, 5), (1, 256, 512), (16, 256, 512), (7, 3072, 1024), (17, 260, 300),
-          (130, 1028, 600), (128, 3072, 1024), (300, 64, 257)]
+          (130, 1028, 600), (128, 3072, 1024), (300, 64, 257), (130, 1032, 600), (17, 264, 300),
+          (257, 2056, 520)]
+
+
+def _skip(path, K):
+    if path != "fp32" and K < 64:
+        pytest.skip("the three-product split is not within gamma_K below K = 64 (the AUTO path picks FP32)")
+    if path == "fp16x3" and K % 8:
+        pytest.skip("FP16X3 needs K % 8 == 0 (whole 16-byte rows of fp16)")
 
 
 @pytest.mark.parametrize("M,K,N", SHAPES)
-@pytest.mark.parametrize("path", ["fp32", "tf32x3"])
+@pytest.mark.parametrize("path", ["fp32", "tf32x3", "fp16x3"])
 def test_products_match_oracle(spl, M, K, N, path):
-    if path == "tf32x3" and K < 64:
-        pytest.skip("the three-product split is not within gamma_K below K = 64 (the AUTO path picks FP32)")
-    W, Wd, hi, lo = _weights(spl, N, K, seed=M + K + N)
+    _skip(path, K)
+    W, Wt = _weights(spl, N, K, seed=M + K + N)
     A = (wl.activations(M, K, seed=M * 7 + 1).numpy() * 300).astype(np.float32)
     C = wl.activations(M, N, seed=11).numpy()
     ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, path))
     Yt = torch.empty((M, N), device="cuda")
     for _ in range(2):  # twice: the workspace must be reusable (counters reset)
-        spl.spl_masked_linear(Yt, dev(A), Wd, hi, lo, path=path, workspace=ws)
+        spl.spl_masked_linear(Yt, dev(A), Wt, path=path, workspace=ws)
         assert_product_close(f32(Yt), A, W, path, what="masked_linear")
     Cp = torch.empty((M, N), device="cuda")
-    spl.spl_precompute_noise_product(Cp, dev(A), Wd, hi, lo, path=path, workspace=ws)
+    spl.spl_precompute_noise_product(Cp, dev(A), Wt, path=path, workspace=ws)
     assert_product_close(f32(Cp), A, W, path, what="precompute")
     Y = torch.empty((M, N), device="cuda")
-    spl.spl_masked_linear_unmask(Y, dev(A), Wd, dev(C), hi, lo, path=path, workspace=ws)
+    spl.spl_masked_linear_unmask(Y, dev(A), Wt, dev(C), path=path, workspace=ws)
     assert_product_close(f32(Y), A, W, path, C=C, what="masked_linear_unmask")
     assert spl.spl_get_device_status() == 0
+
+
+@pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
+def test_products_with_extreme_row_scales(spl, path):
+    """Rows of A and W spread over 60 orders of magnitude, zero rows included: the power-of-two
+    row scaling of FP16X3 keeps every row inside fp16's range."""
+    M, K, N = 160, 1024, 300
+    A = wl.activations(M, K, seed=31).numpy().astype(np.float64)
+    A *= np.array([0.0, 1e-20, 1e-5, 1.0, 1e5, 1e20])[np.arange(M) % 6][:, None]
+    W = wl.weight(N, K, seed=32).numpy().astype(np.float64)
+    W *= np.array([1e-10, 1.0, 1e10])[np.arange(N) % 3][:, None]
+    A, W = A.astype(np.float32), W.astype(np.float32)
+    Wt = spl.Weight.prepare(dev(W))
+    Y = torch.empty((M, N), device="cuda")
+    spl.spl_masked_linear(Y, dev(A), Wt, path=path, workspace=spl.workspace(spl.spl_linear_workspace_bytes(M, K, N)))
+    assert_product_close(f32(Y), A, W, path, what=path)
+    assert not torch.any(Y[0::6]).item()  # zero rows give exact zeros
 
 
 def test_one_workspace_serves_every_shape_and_path(spl):
     """Decode counters sit at a fixed place, so partials of other calls never land on them."""
     cases = [(130, 1028, 600, "tf32x3"), (1, 3072, 3072, "fp32"), (17, 260, 300, "fp32"), (4, 8192, 1024, "fp32"),
-             (1, 3072, 3072, "fp32"), (300, 64, 257, "fp32"), (16, 2560, 3000, "fp32")]
+             (1, 3072, 3072, "fp32"), (1000, 1024, 256, "fp16x3"), (300, 64, 257, "fp32"), (16, 2560, 3000, "fp32"),
+             (1, 3072, 3072, "fp32")]
     need = max(spl.spl_linear_workspace_bytes(M, K, N, path) for M, K, N, path in cases)
     ws = spl.workspace(need)
     for i, (M, K, N, path) in enumerate(cases):
-        W, Wd, hi, lo = _weights(spl, N, K, seed=50 + i)
+        W, Wt = _weights(spl, N, K, seed=50 + i)
         A = (wl.activations(M, K, seed=60 + i).numpy() * 300).astype(np.float32)
         C = wl.activations(M, N, seed=70 + i).numpy()
         Y = torch.empty((M, N), device="cuda")
-        spl.spl_masked_linear_unmask(Y, dev(A), Wd, dev(C), hi, lo, path=path, workspace=ws)
+        spl.spl_masked_linear_unmask(Y, dev(A), Wt, dev(C), path=path, workspace=ws)
         assert_product_close(f32(Y), A, W, path, C=C, what=f"case {i}")
     # the counter region is back to zero after every call
     assert torch.count_nonzero(ws[: 64 * 1024]).item() == 0
@@ -212,7 +267,8 @@ def test_one_workspace_serves_every_shape_and_path(spl):
 
 def test_workspace_errors(spl):
     M, K, N = 4, 3072, 3072
-    W, Wd, hi, lo = _weights(spl, N, K, seed=1)
+    W, Wt = _weights(spl, N, K, seed=1)
+    Wd = Wt.w
     A = dev(wl.activations(M, K, seed=2).numpy())
     Y = torch.empty((M, N), device="cuda")
     need = spl.spl_linear_workspace_bytes(M, K, N, "fp32")
@@ -220,13 +276,29 @@ def test_workspace_errors(spl):
     with pytest.raises(spl.SplError) as e:
         spl.spl_masked_linear(Y, A, Wd, path="fp32", workspace=spl.workspace(16))
     assert e.value.status == spl.SPL_EWORKSPACE
-    with pytest.raises(spl.SplError) as e:
-        spl.spl_masked_linear(torch.empty((130, N), device="cuda"), dev(np.zeros((130, K), np.float32)), Wd,
-                              path="tf32x3", workspace=spl.workspace(spl.spl_linear_workspace_bytes(130, K, N)))
-    assert e.value.status == spl.SPL_EUNSUPPORTED  # no weight split given
+    A130, Y130 = dev(np.zeros((130, K), np.float32)), torch.empty((130, N), device="cuda")
+    for path in ("tf32x3", "fp16x3"):
+        with pytest.raises(spl.SplError) as e:
+            spl.spl_masked_linear(Y130, A130, Wd, path=path,
+                                  workspace=spl.workspace(spl.spl_linear_workspace_bytes(130, K, N)))
+        assert e.value.status == spl.SPL_EUNSUPPORTED  # no weight split given
+    with pytest.raises(spl.SplError) as e:  # FP16X3 keeps its row exponents in the workspace
+        spl.spl_masked_linear(Y130, A130, Wt, path="fp16x3", workspace=None)
+    assert e.value.status == spl.SPL_EWORKSPACE
     misaligned = torch.empty(M * K + 1, device="cuda")[1:].view(M, K)
     with pytest.raises(spl.SplError) as e:
         spl.spl_masked_linear(Y, misaligned, Wd, path="fp32", workspace=spl.workspace(need))
+    assert e.value.status == spl.SPL_EALIGN
+    # K % 8 != 0: no fp16 split is made, AUTO takes TF32X3, explicit FP16X3 is refused
+    K4 = 1028
+    W4 = spl.Weight.prepare(dev(wl.weight(64, K4, seed=3).numpy()))
+    assert W4.f16_hi is None
+    W4.f16_hi, W4.f16_lo = torch.zeros((64, K4), dtype=torch.int16, device="cuda"), torch.zeros(
+        (64, K4), dtype=torch.int16, device="cuda")
+    W4.f16_exp = torch.zeros(64, dtype=torch.int32, device="cuda")
+    with pytest.raises(spl.SplError) as e:
+        spl.spl_masked_linear(torch.empty((130, 64), device="cuda"), dev(np.zeros((130, K4), np.float32)), W4,
+                              path="fp16x3", workspace=spl.workspace(spl.spl_linear_workspace_bytes(130, K4, 64)))
     assert e.value.status == spl.SPL_EALIGN
 
 
@@ -238,13 +310,14 @@ def test_empty_reduction(spl):
 
 
 @pytest.mark.parametrize("M,K,N,path", [(128, 3072, 3072, "tf32x3"), (128, 3072, 3072, "fp32"),
-                                         (1, 3072, 3072, "fp32"), (128, 8192, 3072, "tf32x3")])
+                                         (1, 3072, 3072, "fp32"), (128, 8192, 3072, "tf32x3"),
+                                         (128, 3072, 3072, "fp16x3"), (128, 8192, 3072, "fp16x3")])
 def test_matched_correction_cancels_rounding(spl, M, K, N, path):
     """A bank of 8 corrections summed in the online product's order: the same values up to
     rounding, and on the tensor-core path a much smaller recovered error than a correction
     computed with its own plan for 8 x M rows."""
     draws, b = 8, 1443.0
-    W, Wd, hi, lo = _weights(spl, N, K, seed=K + N)
+    W, Wt = _weights(spl, N, K, seed=K + N)
     X = wl.activations(M, K, seed=21).numpy()
     eta = philox.noise((draws * M, K), b, 1.0, "gaussian", seed=22)
     Nd = dev(eta)
@@ -252,21 +325,20 @@ def test_matched_correction_cancels_rounding(spl, M, K, N, path):
     ws = spl.workspace(max(spl.spl_linear_workspace_bytes(draws * M, K, N, path),
                            spl.spl_precompute_matched_workspace_bytes(draws * M, K, N, M, path),
                            spl.spl_linear_workspace_bytes(M, K, N, path)))
-    spl.spl_precompute_noise_product(C_plain, Nd, Wd, hi, lo, path=path, workspace=ws)
-    spl.spl_precompute_noise_product_matched(C_matched, Nd, Wd, M, hi, lo, path=path, workspace=ws)
+    spl.spl_precompute_noise_product(C_plain, Nd, Wt, path=path, workspace=ws)
+    spl.spl_precompute_noise_product_matched(C_matched, Nd, Wt, M, path=path, workspace=ws)
     assert_product_close(f32(C_matched), eta, W, path, what="matched correction")
     d = draws - 1
     Xt = linear.mask(X, eta[d * M:(d + 1) * M])
     errs = {}
     for name, Cb in (("plain", C_plain), ("matched", C_matched)):
         Y = torch.empty((M, N), device="cuda")
-        spl.spl_masked_linear_unmask(Y, dev(Xt), Wd, Cb[d * M:(d + 1) * M].contiguous(), hi, lo, path=path,
-                                     workspace=ws)
+        spl.spl_masked_linear_unmask(Y, dev(Xt), Wt, Cb[d * M:(d + 1) * M].contiguous(), path=path, workspace=ws)
         err = np.abs(f64(Y) - linear.reference_output(X, W))
         S = linear.abs_products(X, Xt, eta[d * M:(d + 1) * M], W)
         assert np.all(err <= bounds.hard_bound(*S, K)), name
         errs[name] = float(err.mean())
-    if path == "tf32x3":
+    if path != "fp32":
         # the tensor-core bank at 8x the rows uses another K split and cluster order; matched, the
         # errors of fl(x~ W^T) and fl(eta W^T) cancel
         assert errs["matched"] * 3 < errs["plain"], errs
@@ -281,7 +353,8 @@ def test_bound_check_matches_oracle(spl):
     X = wl.activations(M, K, seed=3).numpy()
     eta = philox.noise((M, K), 50.0, 1.0, "gaussian", 9)
     Xt = linear.mask(X, eta)
-    W, Wd, hi, lo = _weights(spl, N, K, seed=4)
+    W, Wt = _weights(spl, N, K, seed=4)
+    Wd = Wt.w
     C = torch.empty((M, N), device="cuda")
     Y = torch.empty((M, N), device="cuda")
     ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp32"))
@@ -301,21 +374,28 @@ def test_bound_check_matches_oracle(spl):
     assert got["max_abs_ref"] == pytest.approx(float(np.max(np.abs(linear.reference_output(X, W)))), rel=1e-12)
 
 
-@pytest.mark.parametrize("K,N", [(3072, 3072), (8, 64)])
+@pytest.mark.parametrize("K,N", [(3072, 3072), (8, 64), (1028, 512)])
 def test_choose_path_follows_its_rule(spl, K, N):
     rows = 128
     X = dev(wl.activations(rows, K, seed=5).numpy())
     eta = torch.empty((rows, K), device="cuda")
     spl.spl_noise(eta, 2 * 3072 ** 0.75, 1.0, "gaussian", seed=6)
-    W, Wd, hi, lo = _weights(spl, N, K, seed=7)
-    name, st_tc, st_fp = spl.spl_choose_path(X, eta, Wd, hi, lo)
-    rule = (st_tc["max_err_over_hard"] <= 1.0
-            and st_tc["log_violations"] <= st_fp["log_violations"] + 0.01 * st_tc["elements"]
-            and st_tc["sum_err"] <= 1.5 * st_fp["sum_err"] + 1e-300)
-    assert name == ("tf32x3" if rule else "fp32")
-    assert st_fp["max_err_over_hard"] <= 1.0
+    W, Wt = _weights(spl, N, K, seed=7)
+    name, st = spl.spl_choose_path(X, eta, Wt)
+    fp = st["fp32"]
+
+    def ok(s):
+        return (s["max_err_over_hard"] <= 1.0 and s["log_violations"] <= fp["log_violations"] + 0.01 * s["elements"]
+                and s["sum_err"] <= 1.5 * fp["sum_err"] + 1e-300)
+
+    expect = "fp16x3" if ok(st["fp16x3"]) else ("tf32x3" if ok(st["tf32x3"]) else "fp32")
+    assert name == expect
+    assert fp["max_err_over_hard"] <= 1.0 and fp["elements"] == rows * N
+    if K % 8:
+        assert st["fp16x3"]["max_err_over_hard"] == float("inf")  # no fp16 split for K % 8 != 0
     if K >= 64:
-        assert name == "tf32x3"  # the three-product split stays inside the bound at Llama sizes
+        assert st["tf32x3"]["max_err_over_hard"] <= 1.0
+        assert name == ("fp16x3" if K % 8 == 0 else "tf32x3")  # the split paths stay inside the bound at Llama sizes
 
 
 # ---------------------------------------------------------- a1: ||W||_2
@@ -326,7 +406,7 @@ def test_spectral_norm_matches_svd(spl):
 
 
 # --------------------------------------------------- end to end, config "single"
-def _run_path(spl, X, W, Wd, hi, lo, sens, eps, mech, seed, path):
+def _run_path(spl, X, W, Wt, sens, eps, mech, seed, path):
     M, K = X.shape
     N = W.shape[0]
     Xt = torch.empty((M, K), device="cuda")
@@ -334,9 +414,9 @@ def _run_path(spl, X, W, Wd, hi, lo, sens, eps, mech, seed, path):
     spl.spl_noise_mask(Xt, Nz, dev(X), sens, eps, mech, seed=seed)
     ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, path))
     C = torch.empty((M, N), device="cuda")
-    spl.spl_precompute_noise_product(C, Nz, Wd, hi, lo, path=path, workspace=ws)
+    spl.spl_precompute_noise_product(C, Nz, Wt, path=path, workspace=ws)
     Y = torch.empty((M, N), device="cuda")
-    spl.spl_masked_linear_unmask(Y, Xt, Wd, C, hi, lo, path=path, workspace=ws)
+    spl.spl_masked_linear_unmask(Y, Xt, Wt, C, path=path, workspace=ws)
     return Y
 
 
@@ -352,20 +432,20 @@ def _hard_check(Y, X, W, sens, eps, mech, seed):
     return err, (S_x, S_xt, S_n)
 
 
-@pytest.mark.parametrize("path", ["fp32", "tf32x3"])
+@pytest.mark.parametrize("path", ["fp32", "tf32x3", "fp16x3"])
 def test_config_single_masked_linear(spl, path):
     cfg = wl.CONFIGS["single"]
     M, K, N = cfg["M"], cfg["K"], cfg["N"]
     X = wl.activations(M, K, seed=cfg["seed"], norm="unit").numpy()
-    W, Wd, hi, lo = _weights(spl, N, K, seed=cfg["seed"] + 1)
+    W, Wt = _weights(spl, N, K, seed=cfg["seed"] + 1)
     for eps in cfg["eps"]:
-        Y = _run_path(spl, X, W, Wd, hi, lo, cfg["sensitivity"], eps, cfg["mech"], cfg["seed"], path)
+        Y = _run_path(spl, X, W, Wt, cfg["sensitivity"], eps, cfg["mech"], cfg["seed"], path)
         _hard_check(Y, X, W, cfg["sensitivity"], eps, cfg["mech"], cfg["seed"])
         if math.isinf(eps):
             Yref = linear.reference_output(X, W)
             assert linear.max_relative_error(f64(Y), Yref) <= 1e-5
             plain = torch.empty((M, N), device="cuda")
-            spl.spl_masked_linear(plain, dev(X), Wd, hi, lo, path=path,
+            spl.spl_masked_linear(plain, dev(X), Wt, path=path,
                                   workspace=spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, path)))
             assert torch.equal(plain, Y)  # zero noise: C = 0 and X~ = X, so unmask(r) is the plain product
 
