@@ -55,7 +55,7 @@ struct LinearArgs {
 
 // Workspace layout shared by every product call: the first kCounterBytes hold
 // the decode kernel's arrival counters (zero between calls); split-K partials,
-// or the FP16X3 row exponents of the left operand, follow.  Keeping the counters
+// or the FP16X3 split of the left operand, follow.  Keeping the counters
 // at a fixed place lets one workspace serve calls of any shape and path.
 constexpr size_t kCounterBytes = 64 * 1024;
 constexpr int64_t kMaxCounters = (int64_t)(kCounterBytes / sizeof(unsigned int));
@@ -97,8 +97,8 @@ struct Plan {
   int splits;            // K-splits (1 = none)
   int64_t k_per_split;   // multiple of the kernel's K granule
   size_t ws_partials;    // bytes of split partials (at offset kCounterBytes)
-  size_t ws_aexp;        // bytes of the FP16X3 row exponents of A (at offset kCounterBytes)
-  size_t total() const { return (ws_partials + ws_aexp) ? kCounterBytes + ws_partials + ws_aexp : 0; }
+  size_t ws_asplit;      // bytes of the FP16X3 split of A: row exponents, hi, lo (at offset kCounterBytes)
+  size_t total() const { return (ws_partials + ws_asplit) ? kCounterBytes + ws_partials + ws_asplit : 0; }
 };
 
 constexpr int kGemvMaxM = 16;
@@ -112,7 +112,7 @@ spl_status run_gemv(const LinearArgs& a, const Plan& p);
 int64_t gemv_max_ks(int64_t M);                           // largest K-slice the decode kernel stages for M rows
 int tc_uniform_splits(int64_t M, int64_t K, int64_t N);    // K-split of a one-launch tcgen05 call, 0 if mixed
 spl_status run_tc_splits(const LinearArgs& a, int splits); // tcgen05 product with the same K-split on every tile
-size_t tc_aexp_bytes(int64_t M, spl_path path);            // workspace of the FP16X3 row exponents (0 for TF32X3)
+size_t tc_asplit_bytes(int64_t M, int64_t K, spl_path path);  // FP16X3 split of A in the workspace (0 for TF32X3)
 spl_status run_simt(const LinearArgs& a, const Plan& p);
 spl_status run_tc(const LinearArgs& a, const Plan& p);
 
@@ -120,8 +120,11 @@ spl_status run_tc(const LinearArgs& a, const Plan& p);
 spl_status run_splitk_reduce(float* out, const float* part, const float* c, int splits, int64_t M,
                              int64_t N, cudaStream_t stream);
 
-// Elementwise TF32 split (used for the A operand of TF32X3 inside the workspace).
+// Elementwise TF32 split (spl_split_tf32).
 spl_status run_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream);
+// Row-scaled fp16 split of a [rows, cols] matrix (spl_split_fp16; the left operand of FP16X3).
+spl_status run_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows, int64_t cols,
+                          cudaStream_t stream);
 
 __host__ __device__ inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 __host__ __device__ inline int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }

@@ -198,30 +198,42 @@ __global__ void __launch_bounds__(kThreads) split_tf32_kernel(float* __restrict_
   }
 }
 
-// fp16 split of a weight, one warp per row: e = fp16_row_exponent(max |w|) brings the row's
-// largest entry into [2^14, 2^15); hi = fp16(w 2^e), lo = fp16(w 2^e - hi) (the difference
-// is exact in fp32).  cols % 8 == 0; each lane handles 8 consecutive entries at a time.
+// fp16 split of a row-major matrix, one block per row: e = fp16_row_exponent(max |x|) brings the
+// row's largest entry into [2^14, 2^15); hi = fp16(x 2^e), lo = fp16(x 2^e - hi) (the difference
+// is exact in fp32).  cols % 8 == 0; each thread handles 8 consecutive entries at a time, and the
+// second pass re-reads the row from L1.
 __global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restrict__ hi, uint16_t* __restrict__ lo,
                                                               int* __restrict__ row_exp, const float* __restrict__ src,
-                                                              int64_t rows, int64_t cols) {
-  const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (r >= rows) return;
+                                                              int64_t cols) {
+  __shared__ float warp_max[kThreads / 32];
+  const int64_t r = blockIdx.x;
   const float4* row = reinterpret_cast<const float4*>(src + r * cols);
   const int64_t q = cols >> 2;
-  float m = 0.f;
-  for (int64_t i = lane; i < q; i += 32) {
-    const float4 v = __ldg(row + i);
-    m = fmaxf(m, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
+  float m0 = 0.f, m1 = 0.f;
+  int64_t i = threadIdx.x;
+  for (; i + kThreads < q; i += 2 * kThreads) {
+    const float4 a = row[i], b = row[i + kThreads];
+    m0 = fmaxf(m0, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
+    m1 = fmaxf(m1, fmaxf(fmaxf(fabsf(b.x), fabsf(b.y)), fmaxf(fabsf(b.z), fabsf(b.w))));
   }
+  if (i < q) {
+    const float4 a = row[i];
+    m0 = fmaxf(m0, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
+  }
+  float m = fmaxf(m0, m1);
   for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  m = warp_max[0];
+#pragma unroll
+  for (int w = 1; w < kThreads / 32; ++w) m = fmaxf(m, warp_max[w]);
   const int e = fp16_row_exponent(m);
-  if (lane == 0) row_exp[r] = e;
+  if (threadIdx.x == 0) row_exp[r] = e;
   const float sc = __int_as_float((e + 127) << 23);
   uint4* h8 = reinterpret_cast<uint4*>(hi + r * cols);
   uint4* l8 = reinterpret_cast<uint4*>(lo + r * cols);
-  for (int64_t i = lane; i < (cols >> 3); i += 32) {
-    const float4 a = __ldg(row + 2 * i), b = __ldg(row + 2 * i + 1);
+  for (int64_t c = threadIdx.x; c < (cols >> 3); c += kThreads) {
+    const float4 a = row[2 * c], b = row[2 * c + 1];
     const float xs[8] = {a.x * sc, a.y * sc, a.z * sc, a.w * sc, b.x * sc, b.y * sc, b.z * sc, b.w * sc};
     __align__(16) __half h[8];
     __align__(16) __half l[8];
@@ -230,8 +242,8 @@ __global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restri
       h[k] = __float2half_rn(xs[k]);
       l[k] = __float2half_rn(__fsub_rn(xs[k], __half2float(h[k])));
     }
-    h8[i] = *reinterpret_cast<const uint4*>(h);
-    l8[i] = *reinterpret_cast<const uint4*>(l);
+    h8[c] = *reinterpret_cast<const uint4*>(h);
+    l8[c] = *reinterpret_cast<const uint4*>(l);
   }
 }
 
@@ -266,6 +278,14 @@ spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, 
 }
 
 }  // namespace
+
+spl_status run_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows, int64_t cols,
+                          cudaStream_t stream) {
+  if (rows == 0) return SPL_OK;
+  if (rows > 0x7fffffffLL) return SPL_ESHAPE;
+  split_fp16_kernel<<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+  return launch_status();
+}
 
 spl_status run_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {
   if (count == 0) return SPL_OK;
@@ -351,9 +371,7 @@ extern "C" spl_status spl_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_ex
   if ((hi && !aligned16(hi)) || (lo && !aligned16(lo)) || (src && !aligned16(src))) return SPL_EALIGN;
   if (cols == 0) return cudaMemsetAsync(row_exp, 0, (size_t)rows * sizeof(int32_t), stream) == cudaSuccess
                             ? SPL_OK : SPL_ECUDA;
-  split_fp16_kernel<<<(unsigned)ceil_div(rows * 32, kThreads), kThreads, 0, stream>>>(hi, lo, row_exp, src, rows,
-                                                                                       cols);
-  return launch_status();
+  return run_split_fp16(hi, lo, row_exp, src, rows, cols, stream);
 }
 
 extern "C" spl_status spl_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {

@@ -10,18 +10,19 @@
 //   FP16X3  each row is first scaled by a power of two so its largest entry lies in
 //           [2^14, 2^15); hi = fp16(a 2^e), lo = fp16(a 2^e - hi) (11 + 11 significant
 //           bits); per-term error ~2^-21 |a w|.  kind::f16 runs at twice the TF32 rate
-//           and the W split is 4 bytes per weight; the power-of-two scales are undone
-//           exactly in the epilogue.
+//           and the split is 4 bytes per element; the power-of-two scales are undone
+//           exactly in the epilogue.  A is split by a pass before the product (into
+//           the workspace), so TMA lands every operand tile directly and the whole
+//           ring carries loads in flight.
 // Either way each term is within about 3 x 2^-21 of exact, below gamma_K = K 2^-24 for
 // K >= 64, so the masked product r = W x~ (Sec. 5.1) and the correction W eta (Sec. 5.2)
 // stay inside the binary32 error model the paper's Thm. 4 is built on while running on
 // the tensor pipe.
 //
 // Kernel shape (one CTA per 128 x 256 output tile, one CTA per SM, 6 warps):
-//   warp 0      TMA producer: per stage the raw fp32 A tile and W_hi, W_lo.
-//   warps 2-5   split the raw A tile into the hi/lo operand tiles in shared memory
-//               (FP16X3: scaled by the per-row exponents a short pass over A wrote to
-//               the workspace before the product), then act as the epilogue.
+//   warp 0      TMA producer: per stage the A tile(s) and W_hi, W_lo.
+//   warps 2-5   TF32X3: split the raw fp32 A tile into its hi/lo operand tiles in shared
+//               memory during the mainloop.  Both modes: the epilogue.
 //   warp 1      TMEM allocator and MMA issuer: per stage 2 k-steps x 3 products into one
 //               fp32 accumulator of 256 TMEM columns; tcgen05.commit frees the stage.
 //   epilogue    tcgen05.ld 32 lanes x 32 columns, (FP16X3: descale), stage the tile in
@@ -77,33 +78,32 @@ constexpr uint32_t make_idesc(uint32_t ab_format, int m, int n) {
 static_assert(make_idesc(2, BM, BN) == 0x08400910u, "tf32 idesc encoding");
 static_assert(make_idesc(0, BM, BN) == 0x08400010u, "f16 idesc encoding");
 
-// The two modes.  Stage layout: [A_hi][A_lo][W_hi][W_lo][A_raw (FP16X3 only)]; in TF32X3
-// the raw A tile lands in the A_hi slot and is split in place.  Operand rows are 64 bytes
-// (64-byte swizzle) in both modes: 16 fp32 or 32 fp16 elements of K.
+// The two modes.  Stage layout: [A_hi][A_lo][W_hi][W_lo]; in TF32X3 the raw A tile lands in
+// the A_hi slot and is split in place by warps 2-5; in FP16X3 TMA brings all four tiles.
+// Operand rows are 64 bytes (64-byte swizzle) in both modes: 16 fp32 or 32 fp16 elements of K.
 struct Tf32x3 {
   static constexpr bool kF16 = false;
   static constexpr int BK = 16;  // K elements per stage
   static constexpr int STAGES = 4;
   static constexpr int UMMA_K = 8;
-  static constexpr uint32_t A_HALF = BM * BK * 4, B_HALF = BN * BK * 4, A_RAW = 0;
+  static constexpr uint32_t A_HALF = BM * BK * 4, B_HALF = BN * BK * 4;
   static constexpr uint32_t IDESC = make_idesc(2, BM, BN);
 };
 struct Fp16x3 {
   static constexpr bool kF16 = true;
   static constexpr int BK = 32;
-  static constexpr int STAGES = 3;
+  static constexpr int STAGES = 4;
   static constexpr int UMMA_K = 16;
-  static constexpr uint32_t A_HALF = BM * BK * 2, B_HALF = BN * BK * 2, A_RAW = BM * BK * 4;
+  static constexpr uint32_t A_HALF = BM * BK * 2, B_HALF = BN * BK * 2;
   static constexpr uint32_t IDESC = make_idesc(0, BM, BN);
 };
 template <class Md>
 struct Layout {
   static constexpr uint32_t A_HI = 0, A_LO = Md::A_HALF, W_HI = 2 * Md::A_HALF, W_LO = W_HI + Md::B_HALF;
-  static constexpr uint32_t RAW = W_LO + Md::B_HALF;
-  static constexpr uint32_t STAGE = RAW + Md::A_RAW;
-  static constexpr uint32_t TX = (Md::kF16 ? Md::A_RAW : Md::A_HALF) + 2 * Md::B_HALF;  // bytes TMA brings
+  static constexpr uint32_t STAGE = W_LO + Md::B_HALF;
+  static constexpr uint32_t TX = (Md::kF16 ? 2 : 1) * Md::A_HALF + 2 * Md::B_HALF;  // bytes TMA brings
   static_assert(STAGE * Md::STAGES <= RING_BYTES, "ring fits");
-  static_assert(RAW % 1024 == 0 && STAGE % 1024 == 0, "swizzle atoms aligned");
+  static_assert(A_LO % 1024 == 0 && W_HI % 1024 == 0 && STAGE % 1024 == 0, "swizzle atoms aligned");
 };
 
 // Shared-memory matrix descriptor for a K-major operand tile with the 64-byte swizzle:
@@ -251,36 +251,8 @@ __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
 }
 __device__ __forceinline__ void converter_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// FP16X3 row exponents of A: e_r = fp16_row_exponent(max_k |A[r, k]|), one warp per row,
-// each lane keeping several 16-byte loads in flight.  Scaling a row by 2^e_r is exact, so the
-// choice of e_r only has to keep every scaled entry inside the fp16 range.
-__global__ void __launch_bounds__(256) row_exponent_kernel(int* __restrict__ exps, const float* __restrict__ A,
-                                                           int64_t M, int64_t K) {
-  const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (r >= M) return;
-  const float4* row = reinterpret_cast<const float4*>(A + r * K);
-  const int64_t q = K >> 2;
-  float m0 = 0.f, m1 = 0.f, m2 = 0.f, m3 = 0.f;
-  int64_t i = lane;
-  for (; i + 96 < q; i += 128) {
-    const float4 a = __ldg(row + i), b = __ldg(row + i + 32), c = __ldg(row + i + 64), d = __ldg(row + i + 96);
-    m0 = fmaxf(m0, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
-    m1 = fmaxf(m1, fmaxf(fmaxf(fabsf(b.x), fabsf(b.y)), fmaxf(fabsf(b.z), fabsf(b.w))));
-    m2 = fmaxf(m2, fmaxf(fmaxf(fabsf(c.x), fabsf(c.y)), fmaxf(fabsf(c.z), fabsf(c.w))));
-    m3 = fmaxf(m3, fmaxf(fmaxf(fabsf(d.x), fabsf(d.y)), fmaxf(fabsf(d.z), fabsf(d.w))));
-  }
-  for (; i < q; i += 32) {
-    const float4 a = __ldg(row + i);
-    m0 = fmaxf(m0, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
-  }
-  float m = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
-  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-  if (lane == 0) exps[r] = fp16_row_exponent(m);
-}
-
 struct TcMaps {
-  CUtensorMap a, w_hi, w_lo;
+  CUtensorMap a, a_lo, w_hi, w_lo;  // TF32X3: a = raw fp32 A (a_lo unused); FP16X3: a = A_hi, a_lo = A_lo
 };
 
 // One CTA computes a 128 x 256 tile of out over the K range of its split (blockIdx.z).
@@ -350,7 +322,8 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
         const uint32_t st = smem_u32(smem + (size_t)s * L::STAGE);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
         mbar_expect_tx(full_bar(s), L::TX);
-        tma_load_2d(st + (Md::kF16 ? L::RAW : L::A_HI), &maps.a, full_bar(s), kx, (int)m0);
+        tma_load_2d(st + L::A_HI, &maps.a, full_bar(s), kx, (int)m0);
+        if constexpr (Md::kF16) tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(s), kx, (int)m0);
         tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(s), kx, (int)n0);
         tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(s), kx, (int)n0);
       }
@@ -373,7 +346,8 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % STAGES;
       const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-      ok = __all_sync(0xffffffffu, mbar_wait(conv_bar(s), ph, kWaitNs, abort_flag));
+      // FP16X3: the operand tiles are ready when TMA lands them; TF32X3: when A is split
+      ok = __all_sync(0xffffffffu, mbar_wait(Md::kF16 ? full_bar(s) : conv_bar(s), ph, kWaitNs, abort_flag));
       if (!ok) break;
       if (lane == 0) {
         tc_fence_after();
@@ -409,39 +383,16 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       converter_sync();
     }
     bool ok = true;
-    for (int kb = 0; kb < nk; ++kb) {
-      const int s = kb % STAGES;
-      const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-      ok = mbar_wait(full_bar(s), ph, kWaitNs, abort_flag);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      uint8_t* st = smem + (size_t)s * L::STAGE;
-      if constexpr (Md::kF16) {
-        // raw tile: 128 rows x 32 fp32 (128-byte rows, 128-byte swizzle); operand tiles: 128 rows x 32 fp16
-        // (64-byte rows, 64-byte swizzle).  Item (r, c): raw chunks 2c, 2c+1 -> one 16-byte chunk of hi and lo.
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int i = t + 128 * j;
-          const int r = i >> 2, c = i & 3;
-          const uint8_t* raw = st + L::RAW + r * 128;
-          const float4 x0 = *reinterpret_cast<const float4*>(raw + (((2 * c) ^ (r & 7)) << 4));
-          const float4 x1 = *reinterpret_cast<const float4*>(raw + (((2 * c + 1) ^ (r & 7)) << 4));
-          const float sc = pow2f(ea[r]);
-          const float xs[8] = {x0.x * sc, x0.y * sc, x0.z * sc, x0.w * sc, x1.x * sc, x1.y * sc, x1.z * sc, x1.w * sc};
-          __align__(16) __half h[8];
-          __align__(16) __half l[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            h[e] = __float2half_rn(xs[e]);
-            l[e] = __float2half_rn(__fsub_rn(xs[e], __half2float(h[e])));
-          }
-          const uint32_t dst = r * 64 + ((c ^ ((r >> 1) & 3)) << 4);
-          *reinterpret_cast<uint4*>(st + L::A_HI + dst) = *reinterpret_cast<const uint4*>(h);
-          *reinterpret_cast<uint4*>(st + L::A_LO + dst) = *reinterpret_cast<const uint4*>(l);
-        }
-      } else {
+    if constexpr (!Md::kF16) {
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % STAGES;
+        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+        ok = mbar_wait(full_bar(s), ph, kWaitNs, abort_flag);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
         // The raw tile sits in the hi slot; hi and lo use the same swizzled positions, so the split is
         // elementwise and in place.  Consecutive threads take consecutive 16-byte chunks.
+        uint8_t* st = smem + (size_t)s * L::STAGE;
         float4* hi = reinterpret_cast<float4*>(st + L::A_HI);
         float4* lo = reinterpret_cast<float4*>(st + L::A_LO);
 #pragma unroll
@@ -452,10 +403,10 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
           hi[i] = h;
           lo[i] = make_float4(__fsub_rn(v.x, h.x), __fsub_rn(v.y, h.y), __fsub_rn(v.z, h.z), __fsub_rn(v.w, h.w));
         }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
+        __syncwarp();
+        if (lane == 0) mbar_arrive(conv_bar(s));
       }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
-      __syncwarp();
-      if (lane == 0) mbar_arrive(conv_bar(s));
     }
     if (!ok && lane == 0) {
       *abort_flag = 1;
@@ -706,19 +657,26 @@ spl_status launch_tc(const LinearArgs& a, int skip_kblock, int forced_splits) {
   if (!set_smem_attr<Md>()) return SPL_ECUDA;
   TcMaps maps;
   std::memset(&maps, 0, sizeof(maps));
-  const void* whi = Md::kF16 ? (const void*)a.w_h16 : (const void*)a.w_hi;
-  const void* wlo = Md::kF16 ? (const void*)a.w_l16 : (const void*)a.w_lo;
-  const CUtensorMapSwizzle a_swz = Md::kF16 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
-  if (!make_map(&maps.a, a.a, false, a.M, a.K, Md::BK, BM, a_swz) ||
-      !make_map(&maps.w_hi, whi, Md::kF16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
-      !make_map(&maps.w_lo, wlo, Md::kF16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
-    return SPL_ECUDA;
-  int* a_exp = nullptr;
+  const int* a_exp = nullptr;
   if constexpr (Md::kF16) {
-    a_exp = reinterpret_cast<int*>(static_cast<char*>(a.ws) + kCounterBytes);
-    row_exponent_kernel<<<(unsigned)ceil_div(a.M * 32, 256), 256, 0, a.stream>>>(a_exp, a.a, a.M, a.K);
-    const spl_status st = launch_status();
+    // split A (row exponents, hi, lo) into the workspace, then map the two fp16 halves
+    char* base = static_cast<char*>(a.ws) + kCounterBytes;
+    int* exps = reinterpret_cast<int*>(base);
+    uint16_t* a_hi = reinterpret_cast<uint16_t*>(base + round_up(a.M * 4, 256));
+    uint16_t* a_lo = reinterpret_cast<uint16_t*>(base + round_up(a.M * 4, 256) + round_up(a.M * a.K * 2, 256));
+    const spl_status st = run_split_fp16(a_hi, a_lo, exps, a.a, a.M, a.K, a.stream);
     if (st != SPL_OK) return st;
+    a_exp = exps;
+    if (!make_map(&maps.a, a_hi, true, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
+        !make_map(&maps.a_lo, a_lo, true, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
+        !make_map(&maps.w_hi, a.w_h16, true, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
+        !make_map(&maps.w_lo, a.w_l16, true, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
+      return SPL_ECUDA;
+  } else {
+    if (!make_map(&maps.a, a.a, false, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
+        !make_map(&maps.w_hi, a.w_hi, false, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
+        !make_map(&maps.w_lo, a.w_lo, false, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
+      return SPL_ECUDA;
   }
   const int m_tiles = (int)ceil_div(a.M, BM);
   const TcLaunches t = forced_splits > 0 ? TcLaunches{0, ceil_div(a.M, BM) * ceil_div(a.N, BN), forced_splits}
@@ -739,7 +697,7 @@ spl_status launch_tc(const LinearArgs& a, int skip_kblock, int forced_splits) {
     attr[0].val.clusterDim.z = (unsigned)splits;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md>, maps, a.out, a.c, (const int*)a_exp,
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md>, maps, a.out, a.c, a_exp,
                                              (const int*)a.w_exp, a.M, a.K, a.N, kps, splits, (int)base, m_tiles,
                                              skip_kblock);
     note_launches(1);
@@ -758,7 +716,8 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_splits) 
     if (!a.w_h16 || !a.w_l16 || !a.w_exp) return SPL_EUNSUPPORTED;
     if ((a.K & 7) != 0) return SPL_EALIGN;  // fp16 rows must be whole 16-byte units
     if (!aligned16(a.w_h16) || !aligned16(a.w_l16)) return SPL_EALIGN;
-    if (!a.ws || a.ws_bytes < kCounterBytes + tc_aexp_bytes(a.M, a.path)) return SPL_EWORKSPACE;
+    if (!a.ws || a.ws_bytes < kCounterBytes + tc_asplit_bytes(a.M, a.K, a.path)) return SPL_EWORKSPACE;
+    if (!aligned16(a.ws)) return SPL_EALIGN;
   } else {
     if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
     if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
@@ -770,8 +729,9 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_splits) 
 
 }  // namespace
 
-size_t tc_aexp_bytes(int64_t M, spl_path path) {
-  return path == SPL_PATH_FP16X3 ? (size_t)round_up(M * (int64_t)sizeof(int), 256) : 0;
+size_t tc_asplit_bytes(int64_t M, int64_t K, spl_path path) {
+  if (path != SPL_PATH_FP16X3) return 0;
+  return (size_t)(round_up(M * 4, 256) + 2 * round_up(M * K * 2, 256));  // exponents, hi, lo
 }
 
 Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path) {
@@ -780,7 +740,7 @@ Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path) {
   const TcLaunches t = tc_launches(M, K, N, sms);
   p.splits = t.rest_splits;
   p.k_per_split = ceil_div(K, t.rest_splits);
-  p.ws_aexp = tc_aexp_bytes(M, path);  // partials are reduced through distributed shared memory
+  p.ws_asplit = tc_asplit_bytes(M, K, path);  // partials are reduced through distributed shared memory
   return p;
 }
 

@@ -115,7 +115,7 @@ MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, sp
     const int s = tc_uniform_splits(order_rows, K, N);
     if (s <= 0) return mp;
     mp.splits = s;
-    mp.ws = resolved == SPL_PATH_FP16X3 ? kCounterBytes + tc_aexp_bytes(M, resolved) : 0;
+    mp.ws = resolved == SPL_PATH_FP16X3 ? kCounterBytes + tc_asplit_bytes(M, K, resolved) : 0;
     mp.ok = true;
     return mp;
   }
