@@ -146,9 +146,9 @@ spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path);
 /* Bytes of device workspace the three product calls below need for this
  * problem on the current device (0 if none; for AUTO the largest over the
  * paths).  Layout: the first 64 KiB hold the decode kernel's arrival
- * counters, then either split-K partial sums (FP32 kernels) or, for FP16X3,
- * one power-of-two exponent per row of the left operand (TF32X3 needs none:
- * it reduces its K-split inside a thread-block cluster).  It must be
+ * counters, then either split-K partial sums (FP32 kernels) or the split of
+ * the left operand for the tensor-core paths (TF32X3: hi and lo in fp32;
+ * FP16X3: one power-of-two exponent per row, hi and lo in fp16).  It must be
  * zero-filled before its first use; every call that
  * returns SPL_OK leaves the counters at zero again, so one workspace (sized
  * for the largest call) serves calls of any shape and path.  Calls that can
@@ -287,9 +287,22 @@ spl_status spl_spectral_norm(double* out, const float* W, int64_t N, int64_t K, 
  * waits run out after about one second, it sets the device status word, lets
  * the copies it did issue land, frees its tensor memory and returns.  The next
  * spl_get_device_status returns SPL_ETIMEOUT and the context stays usable.
- * `out` receives unspecified values. */
+ * `out` receives unspecified values.  Workspace: spl_linear_workspace_bytes(M,
+ * K, N, SPL_PATH_TF32X3). */
 spl_status spl_test_tc_wait_timeout(float* out, const float* A, const spl_weight* W, int64_t M, int64_t K,
-                                    int64_t N, cudaStream_t stream);
+                                    int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* Test hook (the paper has no counterpart): Y = Xt W^T (- C if C is not NULL)
+ * on the tcgen05 kernel with a fixed launch variant -- tile width tile_n and a
+ * stage ring of ring_kb KB: (256, 192), (128, 192) or (128, 96) -- and every
+ * tile's K range split `splits` ways (1..8) across a thread-block cluster,
+ * instead of the shape the library would choose.  path is SPL_PATH_TF32X3 or
+ * SPL_PATH_FP16X3.  Same operands, workspace and errors as
+ * spl_masked_linear_unmask; EINVAL for another path or variant, ESHAPE for a
+ * split outside 1..8. */
+spl_status spl_test_tc_product(float* Y, const float* Xt, const spl_weight* W, const float* C, int64_t M,
+                               int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
+                               void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last

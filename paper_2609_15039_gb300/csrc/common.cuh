@@ -110,8 +110,11 @@ Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path);
 
 spl_status run_gemv(const LinearArgs& a, const Plan& p);
 int64_t gemv_max_ks(int64_t M);                           // largest K-slice the decode kernel stages for M rows
-int tc_uniform_splits(int64_t M, int64_t K, int64_t N);    // K-split of a one-launch tcgen05 call, 0 if mixed
-spl_status run_tc_splits(const LinearArgs& a, int splits); // tcgen05 product with the same K-split on every tile
+// Launch variant and K-split of a one-launch tcgen05 call (false if the call makes two launches).
+bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, int* variant, int* splits);
+// One unsplit tcgen05 launch whose every output is summed in the order of a `splits`-way K-split
+// (partials of the K ranges added in rank order): the correction bank in the masked product's order.
+spl_status run_tc_segmented(const LinearArgs& a, int splits);
 size_t tc_asplit_bytes(int64_t M, int64_t K, spl_path path);  // FP16X3 split of A in the workspace (0 for TF32X3)
 spl_status run_simt(const LinearArgs& a, const Plan& p);
 spl_status run_tc(const LinearArgs& a, const Plan& p);

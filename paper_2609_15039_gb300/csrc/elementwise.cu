@@ -179,6 +179,7 @@ __device__ __forceinline__ float tf32_rna(float v) {
 
 __global__ void __launch_bounds__(kThreads) split_tf32_kernel(float* __restrict__ hi, float* __restrict__ lo,
                                                               const float* __restrict__ src, int64_t n) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int64_t n4 = n >> 2;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const float4* s4 = reinterpret_cast<const float4*>(src);
@@ -247,6 +248,63 @@ __global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restri
   }
 }
 
+// The same split with the row held in registers: one block per row, CH chunks of 8 entries per
+// thread, all loads issued before any is used, so a row costs one memory round trip.  The
+// kernel lets a dependent grid (the product that reads the split) start launching at once.
+template <int CH>
+__global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __restrict__ hi,
+                                                                   uint16_t* __restrict__ lo,
+                                                                   int* __restrict__ row_exp,
+                                                                   const float* __restrict__ src, int64_t cols) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  __shared__ float warp_max[kThreads / 32];
+  const int64_t r = blockIdx.x;
+  const float4* row = reinterpret_cast<const float4*>(src + r * cols);
+  const int64_t n8 = cols >> 3;
+  float4 v[2 * CH];
+#pragma unroll
+  for (int c = 0; c < CH; ++c) {
+    const int64_t i = threadIdx.x + (int64_t)c * kThreads;
+    if (i < n8) {
+      v[2 * c] = __ldg(row + 2 * i);
+      v[2 * c + 1] = __ldg(row + 2 * i + 1);
+    } else {
+      v[2 * c] = v[2 * c + 1] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  float m = 0.f;
+#pragma unroll
+  for (int c = 0; c < 2 * CH; ++c)
+    m = fmaxf(m, fmaxf(fmaxf(fabsf(v[c].x), fabsf(v[c].y)), fmaxf(fabsf(v[c].z), fabsf(v[c].w))));
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  m = warp_max[0];
+#pragma unroll
+  for (int w = 1; w < kThreads / 32; ++w) m = fmaxf(m, warp_max[w]);
+  const int e = fp16_row_exponent(m);
+  if (threadIdx.x == 0) row_exp[r] = e;
+  const float sc = __int_as_float((e + 127) << 23);
+  uint4* h8 = reinterpret_cast<uint4*>(hi + r * cols);
+  uint4* l8 = reinterpret_cast<uint4*>(lo + r * cols);
+#pragma unroll
+  for (int c = 0; c < CH; ++c) {
+    const int64_t i = threadIdx.x + (int64_t)c * kThreads;
+    if (i >= n8) break;
+    const float4 a = v[2 * c], b = v[2 * c + 1];
+    const float xs[8] = {a.x * sc, a.y * sc, a.z * sc, a.w * sc, b.x * sc, b.y * sc, b.z * sc, b.w * sc};
+    __align__(16) __half h[8];
+    __align__(16) __half l[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      h[k] = __float2half_rn(xs[k]);
+      l[k] = __float2half_rn(__fsub_rn(xs[k], __half2float(h[k])));
+    }
+    h8[i] = *reinterpret_cast<const uint4*>(h);
+    l8[i] = *reinterpret_cast<const uint4*>(l);
+  }
+}
+
 int grid_for(int64_t work_items, int blocks_per_sm) {
   const int64_t want = ceil_div(work_items, kThreads);
   const int64_t cap = (int64_t)device_sm_count() * blocks_per_sm;
@@ -283,7 +341,18 @@ spl_status run_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const fl
                           cudaStream_t stream) {
   if (rows == 0) return SPL_OK;
   if (rows > 0x7fffffffLL) return SPL_ESHAPE;
-  split_fp16_kernel<<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+  const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
+  if (per_thread <= 1) {
+    split_fp16_regs_kernel<1><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+  } else if (per_thread <= 2) {
+    split_fp16_regs_kernel<2><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+  } else if (per_thread <= 4) {
+    split_fp16_regs_kernel<4><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+  } else if (per_thread <= 8) {
+    split_fp16_regs_kernel<8><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+  } else {
+    split_fp16_kernel<<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+  }
   return launch_status();
 }
 

@@ -6,28 +6,27 @@
 // Two encodings of the split:
 //   TF32X3  hi = a rounded to TF32 (11 significant bits), lo = a - hi kept in fp32;
 //           the tensor core truncates lo to TF32: per-term error ~2.5 x 2^-21 |a w|.
-//           kind::tf32, K = 8 per instruction; W split offline, 8 bytes per weight.
+//           kind::tf32, K = 8 per instruction, 8 bytes per element.
 //   FP16X3  each row is first scaled by a power of two so its largest entry lies in
 //           [2^14, 2^15); hi = fp16(a 2^e), lo = fp16(a 2^e - hi) (11 + 11 significant
 //           bits); per-term error ~2^-21 |a w|.  kind::f16 runs at twice the TF32 rate
 //           and the split is 4 bytes per element; the power-of-two scales are undone
-//           exactly in the epilogue.  A is split by a pass before the product (into
-//           the workspace), so TMA lands every operand tile directly and the whole
-//           ring carries loads in flight.
+//           exactly in the epilogue.
 // Either way each term is within about 3 x 2^-21 of exact, below gamma_K = K 2^-24 for
 // K >= 64, so the masked product r = W x~ (Sec. 5.1) and the correction W eta (Sec. 5.2)
 // stay inside the binary32 error model the paper's Thm. 4 is built on while running on
-// the tensor pipe.
+// the tensor pipe.  W is split once, offline; A is split by a pass before the product
+// into the workspace, so TMA lands every operand tile directly.
 //
-// Kernel shape (one CTA per 128 x 256 output tile, one CTA per SM, 6 warps):
-//   warp 0      TMA producer: per stage the A tile(s) and W_hi, W_lo.
-//   warps 2-5   TF32X3: split the raw fp32 A tile into its hi/lo operand tiles in shared
-//               memory during the mainloop.  Both modes: the epilogue.
-//   warp 1      TMEM allocator and MMA issuer: per stage 2 k-steps x 3 products into one
-//               fp32 accumulator of 256 TMEM columns; tcgen05.commit frees the stage.
-//   epilogue    tcgen05.ld 32 lanes x 32 columns, (FP16X3: descale), stage the tile in
-//               shared memory; the K-split CTAs of one tile (a thread-block cluster) sum
-//               their staged tiles through distributed shared memory in rank order;
+// Kernel shape (one CTA per 128 x BN output tile, 6 warps; BN = 256 with a 192 KB ring and
+// one CTA per SM, or BN = 128 with a 96 KB ring and two CTAs per SM, so that one CTA's
+// epilogue overlaps the other's mainloop):
+//   warp 0      TMA producer: per stage A_hi, A_lo, W_hi, W_lo.
+//   warp 1      TMEM allocator and MMA issuer: per stage 3 products per k-step into one
+//               fp32 accumulator of BN TMEM columns; tcgen05.commit frees the stage.
+//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns, (FP16X3: descale), stage the
+//               tile in shared memory; the K-split CTAs of one tile (a thread-block cluster)
+//               sum their staged tiles through distributed shared memory in rank order;
 //               subtract C (the fused unmask of Eq. add-and-then-subtract) and store.
 // Every mbarrier wait is bounded (about 1 s of globaltimer); on expiry the kernel raises
 // the device status word, lets issued copies land (again bounded), frees its TMEM and
@@ -57,16 +56,11 @@ cudaError_t read_clear_device_status(unsigned int* word) {
 
 namespace {
 
-constexpr int BM = 128, BN = 256, THREADS = 192;
-constexpr uint32_t TMEM_COLS = 256;
+constexpr int BM = 128, THREADS = 192;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
 constexpr unsigned long long kDrainNs = 100000000ull;  // 0.1 s to drain on abort
 constexpr int MAX_CLUSTER = 8;                         // split-K CTAs of one output tile (portable cluster)
-constexpr int RED_STRIDE = BN + 4;                     // floats per row of the staged accumulator
-constexpr uint32_t RING_BYTES = 192 * 1024;            // stage ring (both modes)
-constexpr uint32_t AUX_BYTES = 2048;                   // barriers, TMEM slot, abort flag, exponents
-constexpr uint32_t SMEM_BYTES = RING_BYTES + AUX_BYTES + 1024;  // + alignment slack
-static_assert((size_t)BM * RED_STRIDE * 4 <= RING_BYTES, "staging fits in the stage ring");
+constexpr uint32_t AUX_BYTES = 1024;                   // barriers, TMEM slot, abort flag
 
 // ---- instruction descriptors (tcgen05.mma kind::tf32 / kind::f16) ---------------
 // D = F32 (bits 4-5 = 1); A and B formats at bits 7-9 and 10-12 (f16: 0, tf32: 2);
@@ -75,35 +69,42 @@ constexpr uint32_t make_idesc(uint32_t ab_format, int m, int n) {
   return (1u << 4) | (ab_format << 7) | (ab_format << 10) | ((uint32_t)(n >> 3) << 17) |
          ((uint32_t)(m >> 4) << 24);
 }
-static_assert(make_idesc(2, BM, BN) == 0x08400910u, "tf32 idesc encoding");
-static_assert(make_idesc(0, BM, BN) == 0x08400010u, "f16 idesc encoding");
+static_assert(make_idesc(2, 128, 256) == 0x08400910u, "tf32 idesc encoding");
+static_assert(make_idesc(0, 128, 256) == 0x08400010u, "f16 idesc encoding");
 
-// The two modes.  Stage layout: [A_hi][A_lo][W_hi][W_lo]; in TF32X3 the raw A tile lands in
-// the A_hi slot and is split in place by warps 2-5; in FP16X3 TMA brings all four tiles.
-// Operand rows are 64 bytes (64-byte swizzle) in both modes: 16 fp32 or 32 fp16 elements of K.
+// The two encodings.  Operand rows are 64 bytes (64-byte swizzle) in both: 16 fp32 or
+// 32 fp16 elements of K per stage.
 struct Tf32x3 {
   static constexpr bool kF16 = false;
-  static constexpr int BK = 16;  // K elements per stage
-  static constexpr int STAGES = 4;
-  static constexpr int UMMA_K = 8;
-  static constexpr uint32_t A_HALF = BM * BK * 4, B_HALF = BN * BK * 4;
-  static constexpr uint32_t IDESC = make_idesc(2, BM, BN);
+  static constexpr int BK = 16, UMMA_K = 8, ESZ = 4;
+  static constexpr uint32_t FMT = 2;
 };
 struct Fp16x3 {
   static constexpr bool kF16 = true;
-  static constexpr int BK = 32;
-  static constexpr int STAGES = 4;
-  static constexpr int UMMA_K = 16;
-  static constexpr uint32_t A_HALF = BM * BK * 2, B_HALF = BN * BK * 2;
-  static constexpr uint32_t IDESC = make_idesc(0, BM, BN);
+  static constexpr int BK = 32, UMMA_K = 16, ESZ = 2;
+  static constexpr uint32_t FMT = 0;
 };
-template <class Md>
-struct Layout {
-  static constexpr uint32_t A_HI = 0, A_LO = Md::A_HALF, W_HI = 2 * Md::A_HALF, W_LO = W_HI + Md::B_HALF;
-  static constexpr uint32_t STAGE = W_LO + Md::B_HALF;
-  static constexpr uint32_t TX = (Md::kF16 ? 2 : 1) * Md::A_HALF + 2 * Md::B_HALF;  // bytes TMA brings
-  static_assert(STAGE * Md::STAGES <= RING_BYTES, "ring fits");
-  static_assert(A_LO % 1024 == 0 && W_HI % 1024 == 0 && STAGE % 1024 == 0, "swizzle atoms aligned");
+// Shared-memory layout of one configuration: tile width BN and a stage ring of RK KB.
+// Stage: [A_hi][A_lo][W_hi][W_lo].  A 192 KB ring keeps the most bytes in flight with one CTA
+// per SM; a 96 KB ring lets two CTAs share an SM, one streaming while the other finishes.
+template <class Md, int BN, int RK>
+struct Cfg {
+  static_assert(BN == 128 || BN == 256, "tile width");
+  static_assert(RK == 96 || RK == 192, "ring size");
+  static constexpr uint32_t A_HALF = BM * Md::BK * Md::ESZ, B_HALF = BN * Md::BK * Md::ESZ;
+  static constexpr uint32_t A_HI = 0, A_LO = A_HALF, W_HI = 2 * A_HALF, W_LO = W_HI + B_HALF;
+  static constexpr uint32_t STAGE = W_LO + B_HALF;  // bytes TMA brings per stage
+  static constexpr uint32_t RING = RK * 1024;
+  static constexpr int STAGES = (int)(RING / STAGE);
+  static constexpr int CTAS_PER_SM = RK == 96 ? 2 : 1;
+  static constexpr uint32_t SMEM = RING + AUX_BYTES + 1024;  // + alignment slack
+  static constexpr int RED_STRIDE = BN + 4;                  // floats per row of the staged accumulator
+  static constexpr uint32_t IDESC = make_idesc(Md::FMT, BM, BN);
+  static_assert(A_LO % 1024 == 0 && W_HI % 1024 == 0 && W_LO % 1024 == 0 && STAGE % 1024 == 0,
+                "swizzle atoms aligned");
+  static_assert(STAGES >= 3 && STAGES <= 8, "ring depth");
+  static_assert((size_t)BM * RED_STRIDE * 4 <= RING, "staging fits in the stage ring");
+  static_assert(8 * (2 * STAGES + 3) + 16 <= AUX_BYTES, "aux fits");
 };
 
 // Shared-memory matrix descriptor for a K-major operand tile with the 64-byte swizzle:
@@ -121,11 +122,6 @@ __device__ __forceinline__ uint64_t make_sdesc_sw64(uint32_t saddr) {
 }
 
 // ---- PTX wrappers ----------------------------------------------------------------
-__device__ __forceinline__ float tf32_rna(float v) {
-  uint32_t r;
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(v));
-  return __uint_as_float(r);
-}
 __device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }  // e in [-126, 127]
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -184,21 +180,21 @@ __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
   asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
-template <class Md>
+template <class Md, uint32_t IDESC>
 __device__ __forceinline__ void mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
   if constexpr (Md::kF16) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(Md::IDESC), "r"(accumulate)
+        "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate)
         : "memory");
   } else {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(Md::IDESC), "r"(accumulate)
+        "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate)
         : "memory");
   }
 }
@@ -228,6 +224,27 @@ __device__ __forceinline__ void tmem_ld_32x32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
+// Programmatic dependent launch: wait until the grid this one depends on has completed and its
+// memory is visible (returns at once when the launch did not use programmatic serialization).
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// 32 lanes x 32 columns of 32-bit words back to TMEM (thread t writes lane base + t).
+__device__ __forceinline__ void tmem_st_32x32(uint32_t taddr, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
+      "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
+      "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
@@ -249,32 +266,35 @@ __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
                : "memory");
   return v;
 }
-__device__ __forceinline__ void converter_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 struct TcMaps {
-  CUtensorMap a, a_lo, w_hi, w_lo;  // TF32X3: a = raw fp32 A (a_lo unused); FP16X3: a = A_hi, a_lo = A_lo
+  CUtensorMap a_hi, a_lo, w_hi, w_lo;
 };
 
-// One CTA computes a 128 x 256 tile of out over the K range of its split (blockIdx.z).
+// One CTA computes a 128 x BN tile of out over the K range of its split (blockIdx.z).
 // The `splits` CTAs of a tile form one thread-block cluster (z dimension); their fp32
 // partial tiles are summed through distributed shared memory in cluster-rank order, so
 // the result does not depend on timing.
-template <class Md>
-__global__ void __launch_bounds__(THREADS, 1)
+// Segmented mode (seg_blocks > 0, one CTA per tile over all of K): the K range is cut into
+// segments of seg_blocks stages, the same boundaries a K-split of the same problem uses; the
+// first segment accumulates into R (TMEM columns 0..BN-1), every later one into P (columns
+// BN..2BN-1), which the epilogue warps fold into R (R = fl(R + P)) before the next segment
+// starts.  Each output is then summed in exactly the order of the split launch -- the partials
+// of the splits added in rank order -- while one CTA streams its whole K range.
+template <class Md, int BN, int RK>
+__global__ void __launch_bounds__(THREADS, Cfg<Md, BN, RK>::CTAS_PER_SM)
 tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
                const int* __restrict__ a_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
-               int64_t k_per_split, int splits, int tile_base, int m_tiles, int skip_kblock) {
-  using L = Layout<Md>;
-  constexpr int STAGES = Md::STAGES, BK = Md::BK;
+               int64_t k_per_split, int splits, int tile_base, int m_tiles, int skip_kblock, int seg_blocks) {
+  using L = Cfg<Md, BN, RK>;
+  constexpr int STAGES = L::STAGES, BK = Md::BK, RED_STRIDE = L::RED_STRIDE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* aux = smem + RING_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], conv[S], empty[S], accum
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (3 * STAGES + 1));
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (3 * STAGES + 1) + 8);
-  int* ea = reinterpret_cast<int*>(aux + 512);    // [BM]  FP16X3: row exponents of A
-  int* ew = reinterpret_cast<int*>(aux + 1024);   // [BN]  FP16X3: row exponents of W (whole rows)
-  float* red = reinterpret_cast<float*>(smem);    // [BM][RED_STRIDE] staged accumulator, after the mainloop
+  uint8_t* aux = smem + L::RING;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], empty[S], accum, seg, fold
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (2 * STAGES + 3));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (2 * STAGES + 3) + 8);
+  float* red = reinterpret_cast<float*>(smem);  // [BM][RED_STRIDE] staged accumulator, after the mainloop
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // Linear tile id, M fastest: the CTAs that read the same weight tile run side by side and share it in L2.
@@ -287,43 +307,74 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
 
   const uint32_t bar_base = smem_u32(bars);
   auto full_bar = [&](int s) { return bar_base + 8u * s; };
-  auto conv_bar = [&](int s) { return bar_base + 8u * (STAGES + s); };
-  auto empty_bar = [&](int s) { return bar_base + 8u * (2 * STAGES + s); };
-  const uint32_t accum_bar = bar_base + 8u * (3 * STAGES);
+  auto empty_bar = [&](int s) { return bar_base + 8u * (STAGES + s); };
+  const uint32_t accum_bar = bar_base + 8u * (2 * STAGES);
+  const uint32_t seg_bar = bar_base + 8u * (2 * STAGES + 1);   // segmented: a later segment is in P
+  const uint32_t fold_bar = bar_base + 8u * (2 * STAGES + 2);  // segmented: P folded into R
+  const int seg_len = seg_blocks > 0 ? seg_blocks : nk + 1;    // stages per segment
+  const int nseg = seg_blocks > 0 ? (int)ceil_div(nk, seg_blocks) : 1;
+  const uint32_t tmem_cols = seg_blocks > 0 ? 2u * BN : (uint32_t)BN;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(conv_bar(s), 4);  // one arrival per converter warp
       mbar_init(empty_bar(s), 1);
     }
     mbar_init(accum_bar, 1);
+    mbar_init(seg_bar, 1);
+    mbar_init(fold_bar, 4);  // one arrival per epilogue warp
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(smem_u32(const_cast<uint32_t*>(tmem_slot)), TMEM_COLS);
+  if (warp == 1) tmem_alloc(smem_u32(const_cast<uint32_t*>(tmem_slot)), tmem_cols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    // ---------------- TMA producer: raw A, W_hi, W_lo ----------------
+    // ---------------- TMA producer: A_hi, A_lo, W_hi, W_lo ----------------
+    // The weight tiles of the first stages do not depend on the kernel before this one (the split
+    // of A, which may still be running under programmatic dependent launch): issue them first,
+    // then wait for that kernel's results and issue the A tiles.
     uint32_t issued_mask = 0u, phase_mask = 0u;  // per stage: a load was issued / its parity
     bool ok = true;
-    for (int kb = 0; kb < nk; ++kb) {
+    const int pre = nk < STAGES ? nk : STAGES;
+    for (int kb = 0; kb < pre; ++kb) {  // fresh ring: every stage is free
+      if (kb == skip_kblock) continue;  // failure-detection test only: this stage never arrives
+      if (lane == 0) {
+        const uint32_t st = smem_u32(smem + (size_t)kb * L::STAGE);
+        const int kx = (int)(kbeg + (int64_t)kb * BK);
+        mbar_expect_tx(full_bar(kb), L::STAGE);
+        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(kb), kx, (int)n0);
+        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(kb), kx, (int)n0);
+      }
+      issued_mask |= 1u << kb;
+    }
+    grid_dependency_wait();
+    for (int kb = 0; kb < pre; ++kb) {
+      if (kb == skip_kblock) continue;
+      if (lane == 0) {
+        const uint32_t st = smem_u32(smem + (size_t)kb * L::STAGE);
+        const int kx = (int)(kbeg + (int64_t)kb * BK);
+        tma_load_2d(st + L::A_HI, &maps.a_hi, full_bar(kb), kx, (int)m0);
+        tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(kb), kx, (int)m0);
+      }
+    }
+    __syncwarp();
+    for (int kb = pre; kb < nk; ++kb) {
       const int s = kb % STAGES;
       const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
       ok = __all_sync(0xffffffffu, mbar_wait(empty_bar(s), ph ^ 1u, kWaitNs, abort_flag));
       if (!ok) break;
-      if (kb == skip_kblock) continue;  // failure-detection test only: this stage never arrives
+      if (kb == skip_kblock) continue;
       if (lane == 0) {
         const uint32_t st = smem_u32(smem + (size_t)s * L::STAGE);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
-        mbar_expect_tx(full_bar(s), L::TX);
-        tma_load_2d(st + L::A_HI, &maps.a, full_bar(s), kx, (int)m0);
-        if constexpr (Md::kF16) tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(s), kx, (int)m0);
+        mbar_expect_tx(full_bar(s), L::STAGE);
+        tma_load_2d(st + L::A_HI, &maps.a_hi, full_bar(s), kx, (int)m0);
+        tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(s), kx, (int)m0);
         tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(s), kx, (int)n0);
         tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(s), kx, (int)n0);
       }
@@ -346,21 +397,27 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % STAGES;
       const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-      // FP16X3: the operand tiles are ready when TMA lands them; TF32X3: when A is split
-      ok = __all_sync(0xffffffffu, mbar_wait(Md::kF16 ? full_bar(s) : conv_bar(s), ph, kWaitNs, abort_flag));
+      const int seg = kb / seg_len, in_seg = kb % seg_len;
+      if (in_seg == 0 && seg >= 2) {  // P is free once the previous segment has been folded into R
+        ok = __all_sync(0xffffffffu, mbar_wait(fold_bar, (uint32_t)(seg - 2) & 1u, kWaitNs, abort_flag));
+        if (!ok) break;
+      }
+      ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), ph, kWaitNs, abort_flag));
       if (!ok) break;
       if (lane == 0) {
         tc_fence_after();
         const uint32_t st = smem_u32(smem + (size_t)s * L::STAGE);
+        const uint32_t acc = tmem + (seg >= 1 ? (uint32_t)BN : 0u);
 #pragma unroll
         for (int kk = 0; kk < BK / Md::UMMA_K; ++kk) {
           const uint32_t koff = kk * 32u;  // one instruction's K is 32 bytes of the 64-byte swizzled row
-          const uint32_t first = (kb == 0 && kk == 0) ? 0u : 1u;
-          mma<Md>(tmem, make_sdesc_sw64(st + L::A_LO + koff), make_sdesc_sw64(st + L::W_HI + koff), first);
-          mma<Md>(tmem, make_sdesc_sw64(st + L::A_HI + koff), make_sdesc_sw64(st + L::W_LO + koff), 1u);
-          mma<Md>(tmem, make_sdesc_sw64(st + L::A_HI + koff), make_sdesc_sw64(st + L::W_HI + koff), 1u);
+          const uint32_t first = (in_seg == 0 && kk == 0) ? 0u : 1u;
+          mma<Md, L::IDESC>(acc, make_sdesc_sw64(st + L::A_LO + koff), make_sdesc_sw64(st + L::W_HI + koff), first);
+          mma<Md, L::IDESC>(acc, make_sdesc_sw64(st + L::A_HI + koff), make_sdesc_sw64(st + L::W_LO + koff), 1u);
+          mma<Md, L::IDESC>(acc, make_sdesc_sw64(st + L::A_HI + koff), make_sdesc_sw64(st + L::W_HI + koff), 1u);
         }
         mma_commit(empty_bar(s));  // stage reusable once these MMAs have read it
+        if (seg >= 1 && (in_seg == seg_len - 1 || kb == nk - 1)) mma_commit(seg_bar);  // P complete
       }
       __syncwarp();
     }
@@ -374,54 +431,37 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     __syncwarp();
     if (!ok) mbar_wait(accum_bar, 0u, kDrainNs, nullptr);
   } else {
-    // ---------------- warps 2..5: split A during the mainloop, then the epilogue ----------------
-    const int t = threadIdx.x - 64;  // 0..127
-    if constexpr (Md::kF16) {
-      // power-of-two row exponents of A (whole rows, from the exponent pass) and of this tile's W rows
-      ea[t] = (m0 + t < M) ? a_exp[m0 + t] : 0;
-      for (int j = t; j < BN; j += 128) ew[j] = (n0 + j < N) ? w_exp[n0 + j] : 0;
-      converter_sync();
-    }
+    // ---------------- warps 2..5: stage the accumulator in shared memory ----------------
+    // (the ring is free once the MMAs are done)
+    grid_dependency_wait();  // the row exponents of A come from the kernel before this one
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
     bool ok = true;
-    if constexpr (!Md::kF16) {
-      for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-        ok = mbar_wait(full_bar(s), ph, kWaitNs, abort_flag);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok) break;
-        // The raw tile sits in the hi slot; hi and lo use the same swizzled positions, so the split is
-        // elementwise and in place.  Consecutive threads take consecutive 16-byte chunks.
-        uint8_t* st = smem + (size_t)s * L::STAGE;
-        float4* hi = reinterpret_cast<float4*>(st + L::A_HI);
-        float4* lo = reinterpret_cast<float4*>(st + L::A_LO);
+    for (int f = 0; f + 1 < nseg; ++f) {  // segmented: fold segment f + 1 (in P) into R
+      ok = __all_sync(0xffffffffu, mbar_wait(seg_bar, (uint32_t)f & 1u, kWaitNs * 4, abort_flag));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t lane_base = tmem + ((uint32_t)(32 * q) << 16);
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        float r[32], p[32];
+        tmem_ld_32x32(lane_base + (uint32_t)(32 * c), r);
+        tmem_ld_32x32(lane_base + (uint32_t)(BN + 32 * c), p);
 #pragma unroll
-        for (int j = 0; j < (int)(Md::A_HALF / 16) / 128; ++j) {
-          const int i = t + 128 * j;
-          const float4 v = hi[i];
-          const float4 h = make_float4(tf32_rna(v.x), tf32_rna(v.y), tf32_rna(v.z), tf32_rna(v.w));
-          hi[i] = h;
-          lo[i] = make_float4(__fsub_rn(v.x, h.x), __fsub_rn(v.y, h.y), __fsub_rn(v.z, h.z), __fsub_rn(v.w, h.w));
-        }
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic writes -> tensor core reads
-        __syncwarp();
-        if (lane == 0) mbar_arrive(conv_bar(s));
+        for (int i = 0; i < 32; ++i) r[i] = __fadd_rn(r[i], p[i]);
+        tmem_st_32x32(lane_base + (uint32_t)(32 * c), r);
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(fold_bar);
     }
-    if (!ok && lane == 0) {
-      *abort_flag = 1;
-      atomicOr(&g_device_status, kStatusTimeout);
-    }
-    // stage this CTA's accumulator in shared memory (the ring is free once the MMAs are done)
     bool have = ok && (nk == 0 || mbar_wait(accum_bar, 0u, kWaitNs * 4, abort_flag));
     have = __all_sync(0xffffffffu, have) && !*abort_flag;
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
     if (have) {
       tc_fence_after();
       const int r = 32 * q + lane;
       float* row = red + (size_t)r * RED_STRIDE;
       float sr = 1.0f;
-      if constexpr (Md::kF16) sr = pow2f(-ea[r]);
+      if constexpr (Md::kF16) sr = pow2f(-((m0 + r < M) ? __ldg(a_exp + m0 + r) : 0));
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         float v[32];
@@ -432,8 +472,10 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
         if constexpr (Md::kF16) {
+          // exact power-of-two scaling; the 32 column exponents are the same for every lane
+          const int64_t nc = n0 + 32 * c;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = (v[i] * sr) * pow2f(-ew[32 * c + i]);  // exact power-of-two scaling
+          for (int i = 0; i < 32; ++i) v[i] = (v[i] * sr) * pow2f(-((nc + i < N) ? __ldg(w_exp + nc + i) : 0));
         }
 #pragma unroll
         for (int j = 0; j < 32; j += 4)
@@ -522,7 +564,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   }
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, TMEM_COLS);
+    tmem_dealloc(tmem, tmem_cols);
   }
 }
 
@@ -562,125 +604,149 @@ bool make_map(CUtensorMap* map, const void* base, bool f16, int64_t rows, int64_
   return r == CUDA_SUCCESS;
 }
 
-template <class Md>
+template <class Md, int BN, int RK>
 bool set_smem_attr() {
   static bool done[64] = {false};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
   if (!done[dev]) {
-    if (cudaFuncSetAttribute(tc_gemm_kernel<Md>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES) !=
-        cudaSuccess)
+    if (cudaFuncSetAttribute(tc_gemm_kernel<Md, BN, RK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)Cfg<Md, BN, RK>::SMEM) != cudaSuccess)
       return false;
     done[dev] = true;
   }
   return true;
 }
 
-// Co-resident clusters of s CTAs (each one SM) on the current device; clusters must fit
-// inside one GPC, so this is not simply SMs / s.  Both modes use the same shared memory
-// and block shape, so one cache serves both.  Cached per device.
-int max_active_clusters(int s, int sms) {
-  static int cache[64][MAX_CLUSTER + 1] = {{0}};
+// The launch variants: tile width, ring size, CTAs per SM, and the cost constants of the
+// launch model below (F: fixed cost of a CTA -- launch, pipeline fill, staging and cross-CTA
+// reduction of its tile; b: cost per unit of K, i.e. bytes per K over the bytes the ring keeps
+// in flight, relative to the 256-wide tile with the 192 KB ring).  Measured on GB300.
+struct Variant {
+  int bn, rk, cps;
+  double F, b;
+};
+constexpr int kVariants = 3;
+constexpr Variant kVariant[kVariants] = {{256, 192, 1, 450.0, 1.0}, {128, 192, 1, 300.0, 0.667},
+                                         {128, 96, 2, 300.0, 1.333}};
+
+// Co-resident clusters of s CTAs of variant v on the current device; clusters must fit inside
+// one GPC, so this is not simply (SMs x CTAs per SM) / s.  Both encodings use the same shared
+// memory and block shape for a given variant, so one query serves both.  Cached per device.
+template <int BN, int RK>
+int query_active_clusters(int s) {
+  int n = 0;
+  if (!set_smem_attr<Tf32x3, BN, RK>()) return 0;
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(1, 1, (unsigned)s);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = Cfg<Tf32x3, BN, RK>::SMEM;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = (unsigned)s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel<Tf32x3, BN, RK>, &cfg) != cudaSuccess) n = 0;
+  cudaGetLastError();
+  return n;
+}
+
+int max_active_clusters(int v, int s, int sms) {
+  static int cache[64][kVariants][MAX_CLUSTER + 1] = {{{0}}};
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return std::max(1, sms / s);
-  int& v = cache[dev][s];
-  if (v == 0) {
-    int n = 0;
-    if (set_smem_attr<Tf32x3>()) {
-      cudaLaunchConfig_t cfg;
-      std::memset(&cfg, 0, sizeof(cfg));
-      cfg.gridDim = dim3(1, 1, (unsigned)s);
-      cfg.blockDim = dim3(THREADS, 1, 1);
-      cfg.dynamicSmemBytes = SMEM_BYTES;
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = 1;
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = (unsigned)s;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      if (cudaOccupancyMaxActiveClusters(&n, tc_gemm_kernel<Tf32x3>, &cfg) != cudaSuccess) n = 0;
-    }
-    cudaGetLastError();
-    v = n > 0 ? n : std::max(1, sms / s);
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return std::max(1, sms * kVariant[v].cps / s);
+  int& c = cache[dev][v][s];
+  if (c == 0) {
+    const int n = v == 0 ? query_active_clusters<256, 192>(s)
+                         : (v == 1 ? query_active_clusters<128, 192>(s) : query_active_clusters<128, 96>(s));
+    c = n > 0 ? n : std::max(1, sms * kVariant[v].cps / s);
   }
-  return v;
+  return c;
 }
 
-// Split of the tiles into launches: full waves of unsplit tiles, then the remaining tiles with
-// K split across clusters so the last wave is not mostly idle.  Time of a launch ~ waves x
-// (kFixedK + K / s), waves counting co-resident clusters of size s; kFixedK is the fixed cost of
-// a CTA (launch, pipeline fill, staging and cross-CTA reduction of its 128 KB tile) measured on
-// GB300 in units of K.  At least 256 of K per CTA; ties go to fewer splits.
-constexpr double kFixedK = 450.0;
-
-int best_split(int64_t tiles, int64_t K, int sms) {
-  const int64_t max_s = std::max<int64_t>(1, std::min<int64_t>(MAX_CLUSTER, K / 256));
-  int64_t best = 1;
-  double best_cost = 1e300;
-  for (int64_t s = 1; s <= max_s; ++s) {
-    const int64_t clusters = max_active_clusters((int)s, sms);
-    const double cost = (double)ceil_div(tiles, clusters) * (kFixedK + (double)K / (double)s);
-    if (cost < best_cost * (1.0 - 1e-9)) {
-      best_cost = cost;
-      best = s;
-    }
-  }
-  return (int)best;
-}
-
-struct TcLaunches {
+// Launch shape: a variant, then either one launch with every tile's K split s ways over a
+// cluster, or whole waves of unsplit tiles followed by the remaining tiles split (so the last
+// wave is not mostly idle).  Cost of a launch in units of K: rounds x (F + b K / s), rounds
+// counting co-resident CTAs.  At least 256 of K per CTA; ties go to the earlier variant and to
+// fewer splits.
+struct TcShape {
+  int v;
   int64_t full_tiles;  // tiles of the first, unsplit launch (whole waves)
   int64_t rest_tiles;  // tiles of the second launch
   int rest_splits;
+  double cost;
 };
 
-TcLaunches tc_launches(int64_t M, int64_t K, int64_t N, int sms) {
-  const int64_t tiles = ceil_div(M, BM) * ceil_div(N, BN);
-  TcLaunches t{0, tiles, 1};
-  const int64_t waves = tiles / sms;
-  if (waves >= 1) {
-    // keep the unsplit waves only if splitting the remainder beats one more unsplit wave
-    const int64_t rest = tiles - waves * sms;
-    if (rest == 0) return TcLaunches{tiles, 0, 1};
-    const int s = best_split(rest, K, sms);
-    const double split_cost = (double)ceil_div(rest, max_active_clusters(s, sms)) * (kFixedK + (double)K / s);
-    if (split_cost < kFixedK + (double)K) return TcLaunches{waves * sms, rest, s};
-    return TcLaunches{0, tiles, 1};
-  }
-  t.rest_splits = best_split(tiles, K, sms);
-  return t;
+double launch_cost(int v, int64_t tiles, int64_t K, int s, int sms) {
+  if (tiles <= 0) return 0.0;
+  const int64_t capacity = (int64_t)max_active_clusters(v, s, sms) * s;
+  const int64_t rounds = ceil_div(tiles * s, capacity);
+  return (double)rounds * (kVariant[v].F + kVariant[v].b * (double)K / (double)s);
 }
 
-template <class Md>
-spl_status launch_tc(const LinearArgs& a, int skip_kblock, int forced_splits) {
-  if (!set_smem_attr<Md>()) return SPL_ECUDA;
+TcShape tc_shape_for(int v, int64_t M, int64_t K, int64_t N, int sms) {
+  const int64_t tiles = ceil_div(M, BM) * ceil_div(N, kVariant[v].bn);
+  const int max_s = (int)std::max<int64_t>(1, std::min<int64_t>(MAX_CLUSTER, K / 256));
+  TcShape best{v, 0, tiles, 1, 1e300};
+  for (int s = 1; s <= max_s; ++s) {
+    const double c = launch_cost(v, tiles, K, s, sms);
+    if (c < best.cost * (1.0 - 1e-9)) best = TcShape{v, 0, tiles, s, c};
+  }
+  const int64_t wave = max_active_clusters(v, 1, sms);
+  const int64_t full = (tiles / wave) * wave, rest = tiles - full;
+  if (full > 0 && rest > 0) {
+    const double cf = launch_cost(v, full, K, 1, sms);
+    for (int s = 1; s <= max_s; ++s) {
+      const double c = cf + launch_cost(v, rest, K, s, sms);
+      if (c < best.cost * (1.0 - 1e-9)) best = TcShape{v, full, rest, s, c};
+    }
+  }
+  return best;
+}
+
+// Best variant for one unsplit launch (segmented mode).
+TcShape tc_unsplit_shape(int64_t M, int64_t K, int64_t N, int sms) {
+  TcShape best{0, 0, 0, 1, 1e300};
+  for (int v = 0; v < kVariants; ++v) {
+    const int64_t tiles = ceil_div(M, BM) * ceil_div(N, kVariant[v].bn);
+    const double c = launch_cost(v, tiles, K, 1, sms);
+    if (c < best.cost * (1.0 - 1e-9)) best = TcShape{v, 0, tiles, 1, c};
+  }
+  return best;
+}
+
+TcShape tc_shape(int64_t M, int64_t K, int64_t N, int sms) {
+  TcShape best = tc_shape_for(0, M, K, N, sms);
+  for (int v = 1; v < kVariants; ++v) {
+    const TcShape t = tc_shape_for(v, M, K, N, sms);
+    if (t.cost < best.cost * (1.0 - 1e-9)) best = t;
+  }
+  return best;
+}
+
+template <class Md, int BN, int RK>
+spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* a_lo, const int* a_exp,
+                     const TcShape& shape, int skip_kblock, int seg_splits) {
+  // segmented mode: one CTA per tile over all of K, cut where a seg_splits-way split would cut it
+  const int seg_blocks = seg_splits > 0 ? (int)(round_up(ceil_div(a.K, seg_splits), Md::BK) / Md::BK) : 0;
+  if (!set_smem_attr<Md, BN, RK>()) return SPL_ECUDA;
   TcMaps maps;
   std::memset(&maps, 0, sizeof(maps));
-  const int* a_exp = nullptr;
-  if constexpr (Md::kF16) {
-    // split A (row exponents, hi, lo) into the workspace, then map the two fp16 halves
-    char* base = static_cast<char*>(a.ws) + kCounterBytes;
-    int* exps = reinterpret_cast<int*>(base);
-    uint16_t* a_hi = reinterpret_cast<uint16_t*>(base + round_up(a.M * 4, 256));
-    uint16_t* a_lo = reinterpret_cast<uint16_t*>(base + round_up(a.M * 4, 256) + round_up(a.M * a.K * 2, 256));
-    const spl_status st = run_split_fp16(a_hi, a_lo, exps, a.a, a.M, a.K, a.stream);
-    if (st != SPL_OK) return st;
-    a_exp = exps;
-    if (!make_map(&maps.a, a_hi, true, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
-        !make_map(&maps.a_lo, a_lo, true, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
-        !make_map(&maps.w_hi, a.w_h16, true, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
-        !make_map(&maps.w_lo, a.w_l16, true, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
-      return SPL_ECUDA;
-  } else {
-    if (!make_map(&maps.a, a.a, false, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
-        !make_map(&maps.w_hi, a.w_hi, false, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
-        !make_map(&maps.w_lo, a.w_lo, false, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
-      return SPL_ECUDA;
-  }
+  const bool f16 = Md::kF16;
+  const void* whi = f16 ? (const void*)a.w_h16 : (const void*)a.w_hi;
+  const void* wlo = f16 ? (const void*)a.w_l16 : (const void*)a.w_lo;
+  if (!make_map(&maps.a_hi, a_hi, f16, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
+      !make_map(&maps.a_lo, a_lo, f16, a.M, a.K, Md::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
+      !make_map(&maps.w_hi, whi, f16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
+      !make_map(&maps.w_lo, wlo, f16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
+    return SPL_ECUDA;
   const int m_tiles = (int)ceil_div(a.M, BM);
-  const TcLaunches t = forced_splits > 0 ? TcLaunches{0, ceil_div(a.M, BM) * ceil_div(a.N, BN), forced_splits}
-                                         : tc_launches(a.M, a.K, a.N, device_sm_count());
+  // The first launch follows the split of A under programmatic dependent launch: its CTAs start
+  // (barriers, TMEM, weight tiles) while the split finishes.
+  bool first = true;
   auto launch = [&](int64_t tiles, int64_t base, int splits) -> spl_status {
     if (tiles <= 0) return SPL_OK;
     const int64_t kps = round_up(ceil_div(a.K, splits), Md::BK);
@@ -688,27 +754,42 @@ spl_status launch_tc(const LinearArgs& a, int skip_kblock, int forced_splits) {
     std::memset(&cfg, 0, sizeof(cfg));
     cfg.gridDim = dim3((unsigned)tiles, 1, (unsigned)splits);
     cfg.blockDim = dim3(THREADS, 1, 1);
-    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.dynamicSmemBytes = Cfg<Md, BN, RK>::SMEM;
     cfg.stream = a.stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 1;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = (unsigned)splits;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md>, maps, a.out, a.c, a_exp,
+    cfg.numAttrs = first ? 2 : 1;
+    first = false;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md, BN, RK>, maps, a.out, a.c, a_exp,
                                              (const int*)a.w_exp, a.M, a.K, a.N, kps, splits, (int)base, m_tiles,
-                                             skip_kblock);
+                                             skip_kblock, seg_blocks);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   };
-  spl_status st = launch(t.full_tiles, 0, 1);
+  spl_status st = launch(shape.full_tiles, 0, 1);
   if (st != SPL_OK) return st;
-  return launch(t.rest_tiles, t.full_tiles, t.rest_splits);
+  return launch(shape.rest_tiles, shape.full_tiles, shape.rest_splits);
 }
 
-spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_splits) {
+template <class Md>
+spl_status launch_variant(const LinearArgs& a, const uint16_t* hi, const uint16_t* lo, const int* a_exp,
+                          const TcShape& shape, int skip_kblock, int seg_splits) {
+  switch (shape.v) {
+    case 0: return launch_tc<Md, 256, 192>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    case 1: return launch_tc<Md, 128, 192>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    default: return launch_tc<Md, 128, 96>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+  }
+}
+
+// forced_v >= 0: every tile with that variant and K-split (forced_splits) in one launch.
+// seg_splits > 0: segmented mode, one unsplit launch whose sums follow a seg_splits-way split.
+spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int forced_splits, int seg_splits = 0) {
   const int cc = device_cc();
   if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
   const bool f16 = a.path == SPL_PATH_FP16X3;
@@ -716,28 +797,55 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_splits) 
     if (!a.w_h16 || !a.w_l16 || !a.w_exp) return SPL_EUNSUPPORTED;
     if ((a.K & 7) != 0) return SPL_EALIGN;  // fp16 rows must be whole 16-byte units
     if (!aligned16(a.w_h16) || !aligned16(a.w_l16)) return SPL_EALIGN;
-    if (!a.ws || a.ws_bytes < kCounterBytes + tc_asplit_bytes(a.M, a.K, a.path)) return SPL_EWORKSPACE;
-    if (!aligned16(a.ws)) return SPL_EALIGN;
   } else {
     if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
     if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
   }
+  if (!a.ws || a.ws_bytes < kCounterBytes + tc_asplit_bytes(a.M, a.K, a.path)) return SPL_EWORKSPACE;
+  if (!aligned16(a.ws)) return SPL_EALIGN;
   if (a.M > 0x7fffffffLL || a.N > 0x7fffffffLL || a.K > 0x7fffffffLL) return SPL_ESHAPE;
-  if (ceil_div(a.M, BM) * ceil_div(a.N, BN) > 0x7fffffffLL || forced_splits > MAX_CLUSTER) return SPL_ESHAPE;
-  return f16 ? launch_tc<Fp16x3>(a, skip_kblock, forced_splits) : launch_tc<Tf32x3>(a, skip_kblock, forced_splits);
+  if (ceil_div(a.M, BM) * ceil_div(a.N, 128) > 0x7fffffffLL || forced_splits > MAX_CLUSTER) return SPL_ESHAPE;
+  if (forced_v >= kVariants) return SPL_EINVAL;
+  // split A into the workspace: [counters][FP16X3: row exponents][hi][lo]
+  char* base = static_cast<char*>(a.ws) + kCounterBytes;
+  const int64_t esz = f16 ? 2 : 4;
+  int* a_exp = nullptr;
+  if (f16) {
+    a_exp = reinterpret_cast<int*>(base);
+    base += round_up(a.M * 4, 256);
+  }
+  void* a_hi = base;
+  void* a_lo = base + round_up(a.M * a.K * esz, 256);
+  const spl_status st =
+      f16 ? run_split_fp16(static_cast<uint16_t*>(a_hi), static_cast<uint16_t*>(a_lo), a_exp, a.a, a.M, a.K, a.stream)
+          : run_split_tf32(static_cast<float*>(a_hi), static_cast<float*>(a_lo), a.a, a.M * a.K, a.stream);
+  if (st != SPL_OK) return st;
+  TcShape shape;
+  if (forced_v >= 0) {
+    shape = TcShape{forced_v, 0, ceil_div(a.M, BM) * ceil_div(a.N, kVariant[forced_v].bn), forced_splits, 0.0};
+  } else if (seg_splits > 0) {
+    shape = tc_unsplit_shape(a.M, a.K, a.N, device_sm_count());
+  } else {
+    shape = tc_shape(a.M, a.K, a.N, device_sm_count());
+  }
+  const uint16_t* hi = static_cast<const uint16_t*>(a_hi);
+  const uint16_t* lo = static_cast<const uint16_t*>(a_lo);
+  return f16 ? launch_variant<Fp16x3>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits)
+             : launch_variant<Tf32x3>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
 }
 
 }  // namespace
 
 size_t tc_asplit_bytes(int64_t M, int64_t K, spl_path path) {
-  if (path != SPL_PATH_FP16X3) return 0;
-  return (size_t)(round_up(M * 4, 256) + 2 * round_up(M * K * 2, 256));  // exponents, hi, lo
+  if (path == SPL_PATH_FP16X3) return (size_t)(round_up(M * 4, 256) + 2 * round_up(M * K * 2, 256));
+  if (path == SPL_PATH_TF32X3) return (size_t)(2 * round_up(M * K * 4, 256));
+  return 0;
 }
 
 Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path) {
   Plan p{};
   p.kernel = kKernelTc;
-  const TcLaunches t = tc_launches(M, K, N, sms);
+  const TcShape t = tc_shape(M, K, N, sms);
   p.splits = t.rest_splits;
   p.k_per_split = ceil_div(K, t.rest_splits);
   p.ws_asplit = tc_asplit_bytes(M, K, path);  // partials are reduced through distributed shared memory
@@ -746,17 +854,20 @@ Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path) {
 
 spl_status run_tc(const LinearArgs& a, const Plan& p) {
   (void)p;
-  return run_tc_impl(a, -1, 0);
+  return run_tc_impl(a, -1, -1, 0);
 }
 
-int tc_uniform_splits(int64_t M, int64_t K, int64_t N) {
-  const TcLaunches t = tc_launches(M, K, N, device_sm_count());
-  return t.full_tiles > 0 && t.rest_tiles > 0 ? 0 : (t.full_tiles > 0 ? 1 : t.rest_splits);
+bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, int* variant, int* splits) {
+  const TcShape t = tc_shape(M, K, N, device_sm_count());
+  if (t.full_tiles > 0 && t.rest_tiles > 0) return false;
+  *variant = t.v;
+  *splits = t.full_tiles > 0 ? 1 : t.rest_splits;
+  return true;
 }
 
-spl_status run_tc_splits(const LinearArgs& a, int splits) {
+spl_status run_tc_segmented(const LinearArgs& a, int splits) {
   if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
-  return run_tc_impl(a, -1, splits);
+  return run_tc_impl(a, -1, -1, 0, splits);
 }
 
 }  // namespace spl
@@ -765,21 +876,31 @@ spl_status run_tc_splits(const LinearArgs& a, int splits) {
 // never issued, so the kernel's bounded waits run out (about 1 s), it raises the device status
 // word and returns.  The paper has no counterpart.
 extern "C" spl_status spl_test_tc_wait_timeout(float* out, const float* A, const spl_weight* W, int64_t M, int64_t K,
-                                               int64_t N, cudaStream_t stream) {
+                                               int64_t N, void* workspace, size_t workspace_bytes,
+                                               cudaStream_t stream) {
   using namespace spl;
   if (!out || !A || !W || !W->w || !W->tf32_hi || !W->tf32_lo || M <= 0 || N <= 0 || K <= 0 || (K & 3))
     return SPL_EINVAL;
   if (K > 256) return SPL_ESHAPE;  // one K range per tile: the skipped stage belongs to every CTA
-  LinearArgs args{};
-  args.out = out;
-  args.a = A;
-  args.w = W->w;
-  args.w_hi = W->tf32_hi;
-  args.w_lo = W->tf32_lo;
-  args.M = M;
-  args.K = K;
-  args.N = N;
-  args.stream = stream;
-  args.path = SPL_PATH_TF32X3;
-  return run_tc_impl(args, 0, 0);
+  LinearArgs args = make_args(out, A, *W, nullptr, M, K, N, workspace, workspace_bytes, stream, SPL_PATH_TF32X3);
+  return run_tc_impl(args, 0, 0, 1);
+}
+
+// Test hook: the tensor-core product with a fixed tile width and K-split, so that tests cover
+// every kernel instance and a sweep can time each launch shape.  The paper has no counterpart.
+extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_weight* W, const float* C, int64_t M,
+                                          int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
+                                          void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  using namespace spl;
+  if (!out || !A || !W || !W->w || M <= 0 || N <= 0 || K <= 0) return SPL_EINVAL;
+  if (path != SPL_PATH_TF32X3 && path != SPL_PATH_FP16X3) return SPL_EINVAL;
+  int v = -1;
+  for (int i = 0; i < kVariants; ++i)
+    if (kVariant[i].bn == tile_n && kVariant[i].rk == ring_kb) v = i;
+  if (v < 0) return SPL_EINVAL;
+  if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
+  if ((K & 3) != 0) return SPL_EALIGN;
+  if (!aligned16(out) || !aligned16(A) || (C && !aligned16(C))) return SPL_EALIGN;
+  const LinearArgs args = make_args(out, A, *W, C, M, K, N, workspace, workspace_bytes, stream, path);
+  return run_tc_impl(args, -1, v, splits);
 }

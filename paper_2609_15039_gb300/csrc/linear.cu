@@ -112,10 +112,9 @@ MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, sp
   const Plan online = make_plan(order_rows, K, N, resolved);
   mp.kernel = online.kernel;
   if (online.kernel == kKernelTc) {
-    const int s = tc_uniform_splits(order_rows, K, N);
-    if (s <= 0) return mp;
-    mp.splits = s;
-    mp.ws = resolved == SPL_PATH_FP16X3 ? kCounterBytes + tc_asplit_bytes(M, K, resolved) : 0;
+    int variant = 0;  // the bank runs its own launch shape; only the K-split order carries over
+    if (!tc_uniform_shape(order_rows, K, N, &variant, &mp.splits)) return mp;
+    mp.ws = kCounterBytes + tc_asplit_bytes(M, K, resolved);
     mp.ok = true;
     return mp;
   }
@@ -211,7 +210,7 @@ extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float
   if (mp.ws > 0 && (!workspace || workspace_bytes < mp.ws)) return SPL_EWORKSPACE;
   if (workspace && !aligned16(workspace)) return SPL_EALIGN;
   const LinearArgs args = make_args(C, Nz, *W, nullptr, M, K, N, workspace, workspace_bytes, stream, resolved);
-  if (mp.kernel == kKernelTc) return run_tc_splits(args, mp.splits);
+  if (mp.kernel == kKernelTc) return run_tc_segmented(args, mp.splits);
   Plan p{};
   p.kernel = mp.kernel;
   p.splits = mp.splits;

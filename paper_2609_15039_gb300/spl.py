@@ -69,7 +69,8 @@ _SIGS = {
     "spl_choose_path_workspace_bytes": (_SZ, [_I64, _I64, _I64]),
     "spl_choose_path": (_I, [ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double), _P, _P, _PW, _I64,
                              _I64, _I64, _P, _SZ, _P]),
-    "spl_test_tc_wait_timeout": (_I, [_P, _P, _PW, _I64, _I64, _I64, _P]),
+    "spl_test_tc_wait_timeout": (_I, [_P, _P, _PW, _I64, _I64, _I64, _P, _SZ, _P]),
+    "spl_test_tc_product": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _I, _I, _I, _P, _SZ, _P]),
     "spl_get_device_status": (_I, [_P]),
     "spl_launch_count": (ctypes.c_uint64, []),
     "spl_status_string": (ctypes.c_char_p, [_I]),
@@ -381,13 +382,33 @@ def spl_choose_path(X, Nz, W, stream=None):
     return PATH_NAMES.get(chosen.value, str(chosen.value)), stats
 
 
-def spl_test_tc_wait_timeout(out, A, W, stream=None):
+def spl_test_tc_wait_timeout(out, A, W, workspace=None, stream=None):
     W = _weight(W)
     M, K = _rows_cols(A)
     N = W.shape[0]
     ws_ = W.c_struct()
-    _check(lib().spl_test_tc_wait_timeout(_dev(out, "out"), _dev(A, "A"), ctypes.byref(ws_), M, K, N,
+    if workspace is None:
+        workspace = globals()["workspace"](spl_linear_workspace_bytes(M, K, N, "tf32x3"), A.device)
+    wsp, wsb = _ws(workspace)
+    _check(lib().spl_test_tc_wait_timeout(_dev(out, "out"), _dev(A, "A"), ctypes.byref(ws_), M, K, N, wsp, wsb,
                                           _stream(stream)), "spl_test_tc_wait_timeout")
+
+
+def spl_test_tc_product(Y, Xt, W, C=None, path="fp16x3", tile_n=256, ring_kb=192, splits=1, workspace=None,
+                        stream=None):
+    """The tensor-core product with a fixed launch variant and K-split (a test hook)."""
+    W = _weight(W)
+    M, K = _rows_cols(Xt)
+    N = W.shape[0]
+    if W.shape[-1] != K or Y.numel() != M * N or (C is not None and C.numel() != M * N):
+        raise ValueError("spl_test_tc_product: shape mismatch")
+    if workspace is None:
+        workspace = globals()["workspace"](spl_linear_workspace_bytes(M, K, N, path), Xt.device)
+    wsp, wsb = _ws(workspace)
+    ws_ = W.c_struct()
+    _check(lib().spl_test_tc_product(_dev(Y, "Y"), _dev(Xt, "Xt"), ctypes.byref(ws_), _dev(C, "C"), M, K, N,
+                                     _path(path), int(tile_n), int(ring_kb), int(splits), wsp, wsb, _stream(stream)),
+           "spl_test_tc_product")
 
 
 def spl_launch_count():

@@ -44,7 +44,8 @@ def test_bounded_wait_times_out_and_context_survives(spl):
     assert spl.spl_get_device_status() == spl.SPL_OK  # reading the status clears it
     # the context is still usable: a normal product is correct
     Y = torch.empty((M, N), device="cuda")
-    spl.spl_masked_linear(Y, Ad, Wt, path="tf32x3")
+    spl.spl_masked_linear(Y, Ad, Wt, path="tf32x3",
+                          workspace=spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "tf32x3")))
     torch.cuda.synchronize()
     assert_product_close(f32(Y), A, W, "tf32x3", what="after timeout")
     assert spl.spl_get_device_status() == spl.SPL_OK

@@ -231,6 +231,25 @@ def test_products_match_oracle(spl, M, K, N, path):
 
 
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
+@pytest.mark.parametrize("tile_n,ring_kb", [(256, 192), (128, 192), (128, 96)])
+@pytest.mark.parametrize("splits", [1, 3, 8])
+def test_tc_every_launch_shape(spl, path, tile_n, ring_kb, splits):
+    """Each kernel instance (encoding x tile width x ring) with each cluster K-split, on a ragged
+    problem: M, N and K not multiples of the tile, and at 8 splits an empty last K range."""
+    M, K, N = 130, 1032, 600
+    W, Wt = _weights(spl, N, K, seed=41)
+    A = (wl.activations(M, K, seed=42).numpy() * 300).astype(np.float32)
+    C = wl.activations(M, N, seed=43).numpy()
+    Y = torch.empty((M, N), device="cuda")
+    spl.spl_test_tc_product(Y, dev(A), Wt, dev(C), path=path, tile_n=tile_n, ring_kb=ring_kb, splits=splits)
+    assert_product_close(f32(Y), A, W, path, C=C, what=f"{path} tile {tile_n} split {splits}")
+    Y2 = torch.empty((M, N), device="cuda")
+    spl.spl_test_tc_product(Y2, dev(A), Wt, None, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=splits)
+    assert_product_close(f32(Y2), A, W, path, what="without C")
+    assert spl.spl_get_device_status() == 0
+
+
+@pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 def test_products_with_extreme_row_scales(spl, path):
     """Rows of A and W spread over 60 orders of magnitude, zero rows included: the power-of-two
     row scaling of FP16X3 keeps every row inside fp16's range."""
@@ -345,6 +364,28 @@ def test_matched_correction_cancels_rounding(spl, M, K, N, path):
     else:
         # FMA chains in ascending k already keep the two roundings correlated; matching never hurts
         assert errs["matched"] <= errs["plain"] * 1.1, errs
+
+
+@pytest.mark.parametrize("M,K,N,path", [(128, 3072, 3072, "fp16x3"), (128, 3072, 5120, "fp16x3"),
+                                         (128, 8192, 3072, "fp16x3"), (128, 3072, 16384, "fp16x3"),
+                                         (128, 3072, 3072, "tf32x3"), (100, 1032, 600, "fp16x3"),
+                                         (128, 3072, 3072, "fp32"), (1, 3072, 3072, "fp32"), (512, 3072, 3072, "fp16x3")])
+def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path):
+    """The bank's correction of draw d is, bit for bit, what the online product computes when
+    its input is that draw's noise: the same K ranges, partials summed in the same order."""
+    draws = 4
+    W, Wt = _weights(spl, N, K, seed=K + N + 1)
+    eta = torch.empty((draws * M, K), device="cuda")
+    spl.spl_noise(eta, 1443.0, 1.0, "gaussian", seed=23)
+    C = torch.empty((draws * M, N), device="cuda")
+    ws = spl.workspace(max(spl.spl_precompute_matched_workspace_bytes(draws * M, K, N, M, path),
+                           spl.spl_linear_workspace_bytes(M, K, N, path)))
+    spl.spl_precompute_noise_product_matched(C, eta, Wt, M, path=path, workspace=ws)
+    for d in range(draws):
+        Y = torch.empty((M, N), device="cuda")
+        spl.spl_masked_linear(Y, eta[d * M:(d + 1) * M].contiguous(), Wt, path=path, workspace=ws)
+        assert torch.equal(Y, C[d * M:(d + 1) * M]), (d, float((Y - C[d * M:(d + 1) * M]).abs().max()))
+    assert spl.spl_get_device_status() == 0
 
 
 # ---------------------------------------------------------- a8: bound on the GPU, path choice
