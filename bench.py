@@ -217,31 +217,60 @@ def main():
         layer.calibrate(inputs, args.eps, mech, seed)  # a8: bound-based path choice per group
     stream = torch.cuda.current_stream(dev)
 
-    events = []  # (kind, begin, end) around every product call
-
-    def timer(phase, kind, group):
-        e = torch.cuda.Event(enable_timing=True)
-        e.record(stream)
-        if phase == "begin":
-            events.append([kind, group, e, None])
-        else:
-            events[-1][3] = e
-
-    def step(s, use_timer=False, x=inputs):
+    def step(s, x=inputs):
+        """One eager step through the library calls (host-side Philox offsets)."""
         cycle, d = divmod(s, DRAWS)
-        t = timer if use_timer else None
         if d == 0:
-            layer.refill(args.eps, mech, seed, cycle, path=args.path, timer=t)
-        return layer.online(x, args.eps, mech, seed, cycle, d, path=args.path, timer=t)
+            layer.refill(args.eps, mech, seed, cycle, path=args.path)
+        return layer.online(x, args.eps, mech, seed, cycle, d, path=args.path)
 
-    s = 0
+    # One eager step sets up every library call (tensor maps, shared-memory attributes, occupancy
+    # queries); then the steps of one bank cycle are captured as CUDA graphs, with CUDA events
+    # around every product call (external event nodes, timestamped at each replay).
+    step(0)
+    torch.cuda.synchronize()
+    gevents = {}  # (draw, kind, group) -> [begin, end] of the latest replay
+    cur = {"d": 0}
+
+    def gtimer(phase, kind, group):
+        e = torch.cuda.Event(enable_timing=True, external=True)
+        e.record()
+        if phase == "begin":
+            gevents[(cur["d"], kind, group)] = [e, None]
+        else:
+            gevents[(cur["d"], kind, group)][1] = e
+
+    graphs, graph_launches = layer.capture(inputs, args.eps, mech, seed, path=args.path, timer=gtimer,
+                                           before=lambda d: cur.update(d=d))
+    # end to end: the same steps with the inputs copied in from pinned host memory and the outputs
+    # copied back inside each graph
+    host_in = {g: x.cpu().pin_memory() for g, x in inputs.items()}
+    dev_in = {g: torch.empty_like(x) for g, x in inputs.items()}
+    host_out = {g.name: torch.empty((M, g.N)).pin_memory() for g in layer.groups}
+    h2d = sum(x.numel() * 4 for x in host_in.values())
+    d2h = sum(o.numel() * 4 for o in host_out.values())
+
+    def copy_in(d):
+        for g in dev_in:
+            dev_in[g].copy_(host_in[g], non_blocking=True)
+
+    def copy_out(d):
+        for g in host_out:
+            host_out[g].copy_(layer.bank[g]["Y"], non_blocking=True)
+
+    e2e_graphs = None
+    if not args.no_e2e:
+        e2e_graphs, _ = layer.capture(dev_in, args.eps, mech, seed, path=args.path, before=copy_in, after=copy_out)
+
+    s = DRAWS  # the graphs start at a bank cycle
+    layer.set_cycle(s // DRAWS)
     for _ in range(args.warmup):
-        step(s)
+        graphs[s % DRAWS].replay()
         s += 1
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    launches0 = spl.spl_launch_count()
+    s_timed = s
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clocks:
@@ -249,14 +278,14 @@ def main():
         torch.cuda.nvtx.range_push("timed")
         t_start.record(stream)
         for _ in range(args.steps):
-            step(s, use_timer=True)
+            graphs[s % DRAWS].replay()
             s += 1
         t_end.record(stream)
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()
     if world > 1:
         dist.barrier()
-    gpu_launches = spl.spl_launch_count() - launches0
+    gpu_launches = sum(graph_launches[(s_timed + i) % DRAWS] for i in range(args.steps))
     ms = t_start.elapsed_time(t_end) / args.steps
     if world > 1:
         t = torch.tensor([ms], device=dev)
@@ -274,12 +303,13 @@ def main():
 
     # roofline of the dominant kernel: the product calls (tcgen05 GEMM + its row exponents / reductions)
     pk = peaks()
+    # per product call: the latest replay of each graph (the last bank cycle of the timed region)
     by_kind, by_group = {}, {}
-    for kind, group, b, e in events:
+    for (d, kind, group), (b, e) in gevents.items():
         by_kind.setdefault(kind, []).append(b.elapsed_time(e))
         by_group.setdefault((kind, group), []).append(b.elapsed_time(e))
-    prod_ms = sum(sum(v) for v in by_kind.values())
-    achieved = flops_step * args.steps / (prod_ms * 1e-3) / 1e12
+    prod_ms = sum(sum(v) for v in by_kind.values())  # one bank cycle: DRAWS online steps, one refill
+    achieved = flops_step * DRAWS / (prod_ms * 1e-3) / 1e12
     path_peak = {  # algorithmic flops (one product per term) per second at each path's instruction peak
         "fp16x3": pk["bf16_tflops_sustained"] / 3.0,
         "tf32x3": pk["bf16_tflops_sustained"] * TF32_OVER_BF16 / 3.0,
@@ -310,29 +340,16 @@ def main():
                 "peak_source": pk["source"], "peak_note": peak_note}
 
     e2e = None
-    if not args.no_e2e:
-        host_in = {g: x.cpu().pin_memory() for g, x in inputs.items()}
-        dev_in = {g: torch.empty_like(x) for g, x in inputs.items()}
-        host_out = {g.name: torch.empty((M, g.N)).pin_memory() for g in layer.groups}
-        h2d = sum(x.numel() * 4 for x in host_in.values())
-        d2h = sum(o.numel() * 4 for o in host_out.values())
-
-        def e2e_step(s):
-            for g in dev_in:
-                dev_in[g].copy_(host_in[g], non_blocking=True)
-            outs = step(s, x=dev_in)
-            for g in host_out:
-                host_out[g].copy_(outs[g], non_blocking=True)
-
+    if e2e_graphs is not None:
         for _ in range(2):
-            e2e_step(s)
+            e2e_graphs[s % DRAWS].replay()
             s += 1
         torch.cuda.synchronize()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(args.steps):
-            e2e_step(s)
+            e2e_graphs[s % DRAWS].replay()
             s += 1
         e1.record(stream)
         torch.cuda.synchronize()

@@ -91,6 +91,10 @@ typedef struct spl_rng {
   uint64_t seed;
   uint64_t stream_id;
   uint64_t offset;
+  /* Optional DEVICE pointer (8-byte aligned) or NULL: the kernel adds the value it
+   * finds there, when it runs, to `offset`.  A CUDA graph captured with it draws
+   * fresh noise on every replay once the value is moved on (spl_rng_advance). */
+  const uint64_t* offset_dev;
 } spl_rng;
 
 /* ---- a2: noise --------------------------------------------------------
@@ -110,6 +114,11 @@ spl_status spl_noise(float* N, int64_t rows, int64_t cols, double sensitivity, d
  * block e / 4 + rng.offset.  This is the integer stream spl_noise transforms.
  * Errors: EINVAL for NULL out or count < 0, EALIGN if out is not 16-byte aligned. */
 spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng, cudaStream_t stream);
+
+/* *offset_dev += delta, on the device, in stream order (one thread).  The step a
+ * captured graph ends with to move its draws to the next blocks of the stream.
+ * Errors: EINVAL for NULL, EALIGN if not 8-byte aligned. */
+spl_status spl_rng_advance(uint64_t* offset_dev, uint64_t delta, cudaStream_t stream);
 
 /* ---- a3: mask ---------------------------------------------------------
  * Xt = fl32(X + N) elementwise, round-to-nearest (Sec. 3.3.1).  Xt may alias X. */

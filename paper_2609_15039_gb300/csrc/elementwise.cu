@@ -85,7 +85,8 @@ template <int MECH>
 __global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* __restrict__ nout,
                                                               const float* x, int64_t n, float b,
                                                               uint32_t k0, uint32_t k1, uint32_t s0, uint32_t s1,
-                                                              uint64_t offset) {
+                                                              uint64_t offset_host, const uint64_t* offset_dev) {
+  const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
   const int64_t nb_full = n >> 2;  // blocks with all 4 elements in range
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -128,10 +129,13 @@ __global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* 
   }
 }
 
+__global__ void rng_advance_kernel(uint64_t* offset_dev, uint64_t delta) { *offset_dev += delta; }
+
 // The raw Philox words of the stream (element e = lane e % 4 of block e / 4 + offset).
 __global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restrict__ out, int64_t n, uint32_t k0,
                                                                uint32_t k1, uint32_t s0, uint32_t s1,
-                                                               uint64_t offset) {
+                                                               uint64_t offset_host, const uint64_t* offset_dev) {
+  const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
   const int64_t nb = (n + 3) >> 2;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
@@ -321,16 +325,20 @@ spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double
 
 spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, double sensitivity, double eps,
                              spl_mech mech, spl_rng rng, cudaStream_t stream) {
+  if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
   const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
   const int grid = grid_for(ceil_div(n, 4), 8);
   const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
   const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
   if (b == 0.0f) {
-    noise_mask_kernel<kZero><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset);
+    noise_mask_kernel<kZero><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset,
+                                                                 rng.offset_dev);
   } else if (mech == SPL_MECH_LAPLACE) {
-    noise_mask_kernel<kLaplace><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset);
+    noise_mask_kernel<kLaplace><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset,
+                                                                 rng.offset_dev);
   } else {
-    noise_mask_kernel<kGaussian><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset);
+    noise_mask_kernel<kGaussian><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset,
+                                                                 rng.offset_dev);
   }
   return launch_status();
 }
@@ -390,12 +398,20 @@ extern "C" spl_status spl_noise(float* N, int64_t rows, int64_t cols, double sen
 
 extern "C" spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng, cudaStream_t stream) {
   if (count < 0) return SPL_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
   if (count == 0) return SPL_OK;
   if (!out) return SPL_EINVAL;
   if (!aligned16(out)) return SPL_EALIGN;
   random_bits_kernel<<<grid_for(ceil_div(count, 4), 8), kThreads, 0, stream>>>(
       out, count, (uint32_t)rng.seed, (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id,
-      (uint32_t)(rng.stream_id >> 32), rng.offset);
+      (uint32_t)(rng.stream_id >> 32), rng.offset, rng.offset_dev);
+  return launch_status();
+}
+
+extern "C" spl_status spl_rng_advance(uint64_t* offset_dev, uint64_t delta, cudaStream_t stream) {
+  if (!offset_dev) return SPL_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(offset_dev) & 7u) != 0) return SPL_EALIGN;
+  rng_advance_kernel<<<1, 1, 0, stream>>>(offset_dev, delta);
   return launch_status();
 }
 

@@ -16,7 +16,11 @@ consumed once.  This module keeps that structure, GB300 style:
 * an ``online`` step regenerates its mask from the same Philox counters
   (seed, group stream, block offset of draw d) instead of reading it back,
   masks the input (a3) and runs the masked product with the unmask fused
-  into its epilogue, Y = X~ W^T - C_d (a5 + a6).
+  into its epilogue, Y = X~ W^T - C_d (a5 + a6);
+* ``capture`` records the steps of one bank cycle as CUDA graphs (draw 0
+  with the refill): the Philox block offset of each group then lives on the
+  device and the last graph moves it to the next cycle, so the same graphs
+  replay cycle after cycle with fresh noise and no host work per kernel.
 
 The noise scale Delta per group comes from Thms. 1-3 (a1, ``sensitivities``).
 This module only sequences library calls; all arithmetic is in libspl.
@@ -61,6 +65,7 @@ class MaskedLayer:
     M: int = 0
     paths: dict = field(default_factory=dict)   # per group, from calibrate(); "auto" if not calibrated
     calibration: dict = field(default_factory=dict)
+    rng_base: torch.Tensor = None               # [groups] int64 on the device: Philox block offset of the cycle
 
     @classmethod
     def from_weights(cls, model, weights, split=True, device="cuda"):
@@ -137,6 +142,7 @@ class MaskedLayer:
         if self.workspace is None or self.workspace.numel() < need:
             self.workspace = spl.workspace(need, dev)
         self.M, self.draws = M, draws
+        self.rng_base = torch.zeros(len(self.groups), dtype=torch.int64, device=dev)
         self.bank = {}
         for g in self.groups:
             self.bank[g.name] = {
@@ -151,12 +157,24 @@ class MaskedLayer:
         per_draw = self.M * g.K // 4  # K % 4 == 0, so a draw is a whole number of blocks
         return (cycle * self.draws + d) * per_draw
 
-    def refill(self, eps, mech, seed, cycle, path="auto", stream=None, timer=None):
+    def _offset(self, gi, g, cycle, d, device_base):
+        """(host offset, device offset tensor or None) of draw d of cycle ``cycle``."""
+        if device_base:  # the cycle's base is on the device (set_cycle / the last captured graph)
+            return d * (self.M * g.K // 4), self.rng_base[gi:gi + 1]
+        return self.block_offset(g, cycle, d), None
+
+    def set_cycle(self, cycle):
+        """Put the device-side Philox bases at bank cycle ``cycle`` (for captured graphs)."""
+        base = torch.tensor([self.block_offset(g, cycle, 0) for g in self.groups], dtype=torch.int64)
+        self.rng_base.copy_(base)
+
+    def refill(self, eps, mech, seed, cycle, path="auto", stream=None, timer=None, device_base=False):
         """a2 + a4: draw ``draws`` masks per group and precompute their corrections in one product."""
         for gi, g in enumerate(self.groups):
             b = self.bank[g.name]
-            spl.spl_noise(b["eta"], self.deltas[g.name], eps, mech, seed, stream_id=gi,
-                          offset=self.block_offset(g, cycle, 0), stream=stream)
+            off, off_dev = self._offset(gi, g, cycle, 0, device_base)
+            spl.spl_noise(b["eta"], self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off, stream=stream,
+                          offset_dev=off_dev)
             if timer:
                 timer("begin", "precompute", g.name)
             # summed in the order the online product of M rows uses, so their rounding cancels
@@ -165,7 +183,7 @@ class MaskedLayer:
             if timer:
                 timer("end", "precompute", g.name)
 
-    def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None):
+    def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None, device_base=False):
         """a3 + a5 + a6 for draw d: regenerate eta_d, mask, masked product with fused unmask.
 
         inputs: {group: X [M, K]}.  Returns {group: Y [M, N_group]} (views of the layer's buffers).
@@ -174,8 +192,9 @@ class MaskedLayer:
         out = {}
         for gi, g in enumerate(self.groups):
             b = self.bank[g.name]
+            off, off_dev = self._offset(gi, g, cycle, d, device_base)
             spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
-                               offset=self.block_offset(g, cycle, d), stream=stream)
+                               offset=off, stream=stream, offset_dev=off_dev)
             if timer:
                 timer("begin", "masked_linear_unmask", g.name)
             spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M], path=self.path_of(g, path, M),
@@ -184,6 +203,33 @@ class MaskedLayer:
                 timer("end", "masked_linear_unmask", g.name)
             out[g.name] = b["Y"]
         return out
+
+    def capture(self, inputs, eps, mech, seed, path="auto", timer=None, before=None, after=None):
+        """CUDA graphs of the ``draws`` steps of one bank cycle: graph d runs online step d (graph 0
+        refills the bank first); the last graph moves every group's Philox base on by one cycle.
+        Replay graphs[s % draws] for step s after set_cycle(s // draws) -- the graphs read their
+        offsets on the device, so they replay cycle after cycle.  ``before(d)`` / ``after(d)`` run
+        inside the capture around the step (host-to-device input copies, device-to-host result
+        copies).  Every library call must have run once before (warm-up), so nothing is set up
+        during capture.  Returns the graphs and the number of library kernels in each."""
+        graphs, launches = [], []
+        for d in range(self.draws):
+            graph = torch.cuda.CUDAGraph()
+            n0 = spl.spl_launch_count()
+            with torch.cuda.graph(graph):
+                if before:
+                    before(d)
+                if d == 0:
+                    self.refill(eps, mech, seed, 0, path=path, timer=timer, device_base=True)
+                self.online(inputs, eps, mech, seed, 0, d, path=path, timer=timer, device_base=True)
+                if after:
+                    after(d)
+                if d == self.draws - 1:
+                    for gi, g in enumerate(self.groups):
+                        spl.spl_rng_advance(self.rng_base[gi:gi + 1], self.draws * (self.M * g.K // 4))
+            graphs.append(graph)
+            launches.append(spl.spl_launch_count() - n0)
+        return graphs, launches
 
     def bound_check(self, inputs, outs, eps, mech, seed, cycle, d):
         """The paper's bound on the GPU over every output of an online step (per group)."""

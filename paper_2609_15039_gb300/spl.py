@@ -31,7 +31,8 @@ class SplError(RuntimeError):
 
 
 class spl_rng(ctypes.Structure):
-    _fields_ = [("seed", ctypes.c_uint64), ("stream_id", ctypes.c_uint64), ("offset", ctypes.c_uint64)]
+    _fields_ = [("seed", ctypes.c_uint64), ("stream_id", ctypes.c_uint64), ("offset", ctypes.c_uint64),
+                ("offset_dev", ctypes.c_void_p)]
 
 
 class spl_weight(ctypes.Structure):
@@ -48,6 +49,7 @@ _SZ = ctypes.c_size_t
 _SIGS = {
     "spl_noise": (_I, [_P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_random_bits": (_I, [_P, _I64, spl_rng, _P]),
+    "spl_rng_advance": (_I, [_P, ctypes.c_uint64, _P]),
     "spl_mask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_noise_mask": (_I, [_P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_split_tf32": (_I, [_P, _P, _P, _I64, _P]),
@@ -141,19 +143,33 @@ def _eps(eps):
     return float("inf") if eps is None else float(eps)
 
 
-def spl_noise(N, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None):
+def _rng(seed, stream_id, offset, offset_dev):
+    """offset_dev: None or a one-element int64 CUDA tensor added on the device to offset."""
+    if offset_dev is not None and (offset_dev.dtype != torch.int64 or not offset_dev.is_cuda):
+        raise TypeError("offset_dev must be an int64 CUDA tensor")
+    return spl_rng(seed % 2**64, stream_id % 2**64, offset % 2**64,
+                   None if offset_dev is None else offset_dev.data_ptr())
+
+
+def spl_noise(N, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None, offset_dev=None):
     rows, cols = _rows_cols(N)
     _check(lib().spl_noise(_dev(N, "N"), rows, cols, float(sensitivity), _eps(eps), _mech(mech),
-                           spl_rng(seed % 2**64, stream_id % 2**64, offset % 2**64), _stream(stream)), "spl_noise")
+                           _rng(seed, stream_id, offset, offset_dev), _stream(stream)), "spl_noise")
 
 
-def spl_random_bits(out, seed, stream_id=0, offset=0, stream=None):
+def spl_random_bits(out, seed, stream_id=0, offset=0, stream=None, offset_dev=None):
     """Raw Philox words into a CUDA int32/uint32 tensor (bit pattern of the uint32 stream)."""
     if not out.is_cuda or out.element_size() != 4 or not out.is_contiguous():
         raise TypeError("out must be a contiguous 4-byte CUDA tensor")
-    _check(lib().spl_random_bits(ctypes.c_void_p(out.data_ptr()), out.numel(),
-                                 spl_rng(seed % 2**64, stream_id % 2**64, offset % 2**64), _stream(stream)),
-           "spl_random_bits")
+    _check(lib().spl_random_bits(ctypes.c_void_p(out.data_ptr()), out.numel(), _rng(seed, stream_id, offset, offset_dev),
+                                 _stream(stream)), "spl_random_bits")
+
+
+def spl_rng_advance(offset_dev, delta, stream=None):
+    if offset_dev.dtype != torch.int64 or not offset_dev.is_cuda:
+        raise TypeError("offset_dev must be an int64 CUDA tensor")
+    _check(lib().spl_rng_advance(ctypes.c_void_p(offset_dev.data_ptr()), int(delta) % 2**64, _stream(stream)),
+           "spl_rng_advance")
 
 
 def spl_mask(Xt, X, N, stream=None):
@@ -161,11 +177,11 @@ def spl_mask(Xt, X, N, stream=None):
     _check(lib().spl_mask(_dev(Xt, "Xt"), _dev(X, "X"), _dev(N, "N"), rows, cols, _stream(stream)), "spl_mask")
 
 
-def spl_noise_mask(Xt, N_out, X, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None):
+def spl_noise_mask(Xt, N_out, X, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None, offset_dev=None):
     rows, cols = _rows_cols(X)
     _check(lib().spl_noise_mask(_dev(Xt, "Xt"), _dev(N_out, "N_out"), _dev(X, "X"), rows, cols, float(sensitivity),
-                                _eps(eps), _mech(mech), spl_rng(seed % 2**64, stream_id % 2**64, offset % 2**64),
-                                _stream(stream)), "spl_noise_mask")
+                                _eps(eps), _mech(mech), _rng(seed, stream_id, offset, offset_dev), _stream(stream)),
+           "spl_noise_mask")
 
 
 def spl_split_tf32(hi, lo, src, stream=None):

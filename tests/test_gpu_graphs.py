@@ -1,0 +1,79 @@
+"""CUDA graphs of a bank cycle: replayed graphs compute, bit for bit, what the eager library
+calls compute for the same steps, across bank refills (the Philox offsets then come from the
+device and the last graph of a cycle moves them on)."""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_15039_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def spl():
+    from paper_2609_15039_gb300 import spl as binding
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    binding.lib()
+    return binding
+
+
+def make_layer(model, M, draws):
+    from paper_2609_15039_gb300.layer import MaskedLayer
+    weights = {name: wl.weight(N, K, seed=300 + pi, device="cuda")
+               for pi, (name, K, N, g) in enumerate(model.projections())}
+    layer = MaskedLayer.from_weights(model, weights)
+    layer.deltas = {"qkv": 90.0, "gateup": 90.0, "o": 45.0, "down": 700.0}
+    layer.allocate(M, draws)
+    inputs = {g: wl.activations(M, K, seed=400 + gi, device="cuda")
+              for gi, (g, K, _n) in enumerate(model.input_groups())}
+    return layer, inputs
+
+
+@pytest.mark.parametrize("M", [128, 4])
+def test_graph_replay_equals_eager_steps(spl, M):
+    model = wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)
+    draws, eps, mech, seed = 3, 1.0, "laplace", 77
+    layer, inputs = make_layer(model, M, draws)
+
+    def eager(s):
+        cycle, d = divmod(s, draws)
+        if d == 0:
+            layer.refill(eps, mech, seed, cycle)
+        return {g: y.clone() for g, y in layer.online(inputs, eps, mech, seed, cycle, d).items()}
+
+    first, steps = 2 * draws, 2 * draws + 2  # from cycle 2 into cycle 4
+    expected = [eager(s) for s in range(first, first + steps)]
+    torch.cuda.synchronize()
+    graphs, launches = layer.capture(inputs, eps, mech, seed)
+    assert len(graphs) == draws and all(n > 0 for n in launches)
+    layer.set_cycle(first // draws)
+    for i, s in enumerate(range(first, first + steps)):
+        graphs[s % draws].replay()
+        torch.cuda.synchronize()
+        for g in expected[i]:
+            assert torch.equal(layer.bank[g]["Y"], expected[i][g]), (s, g)
+    # the device bases moved on by one cycle per completed cycle
+    exp_base = [layer.block_offset(g, (first + steps) // draws, 0) for g in layer.groups]
+    assert layer.rng_base.cpu().tolist() == exp_base
+    assert spl.spl_get_device_status() == 0
+
+
+def test_device_offset_equals_host_offset(spl):
+    n, seed, sid = 4096 + 3, 5, 2
+    base = torch.tensor([12345], dtype=torch.int64, device="cuda")
+    a = torch.empty(n, dtype=torch.int32, device="cuda")
+    b = torch.empty_like(a)
+    spl.spl_random_bits(a, seed, sid, offset=12345 + 7)
+    spl.spl_random_bits(b, seed, sid, offset=7, offset_dev=base)
+    assert torch.equal(a, b)
+    X = torch.randn(33, 64, device="cuda")
+    x1, x2 = torch.empty_like(X), torch.empty_like(X)
+    spl.spl_noise_mask(x1, None, X, 3.0, 1.0, "gaussian", seed, sid, offset=12345 + 9)
+    spl.spl_noise_mask(x2, None, X, 3.0, 1.0, "gaussian", seed, sid, offset=9, offset_dev=base)
+    assert torch.equal(x1, x2)
+    spl.spl_rng_advance(base, 2 ** 40)
+    assert base.item() == 12345 + 2 ** 40
+    # an offset word must be 8-byte aligned: refused before anything is launched
+    assert spl.lib().spl_rng_advance(base.data_ptr() + 4, 1, None) == spl.SPL_EALIGN
