@@ -30,6 +30,31 @@ inline spl_status launch_status() {
   return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
 }
 
+// Programmatic dependent launch.  A kernel launched with launch_pdl may start while the kernel
+// before it in the stream is still running; it calls pdl_wait() before it touches memory that
+// kernel writes (or any memory at all, when in doubt), and pdl_trigger() once it has waited, so
+// that the next kernel can be scheduled early in turn (a chain never runs more than one kernel
+// ahead, and no kernel holds SM resources while waiting on a kernel that is not yet resident).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline spl_status launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+  note_launches(1);
+  return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
+}
+
 // Number of SMs of the current device (cached per device).
 int device_sm_count();
 // Compute capability major*10+minor of the current device.

@@ -86,6 +86,8 @@ __global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* 
                                                               const float* x, int64_t n, float b,
                                                               uint32_t k0, uint32_t k1, uint32_t s0, uint32_t s1,
                                                               uint64_t offset_host, const uint64_t* offset_dev) {
+  pdl_wait();
+  pdl_trigger();
   const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
   const int64_t nb_full = n >> 2;  // blocks with all 4 elements in range
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -129,12 +131,18 @@ __global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* 
   }
 }
 
-__global__ void rng_advance_kernel(uint64_t* offset_dev, uint64_t delta) { *offset_dev += delta; }
+__global__ void rng_advance_kernel(uint64_t* offset_dev, uint64_t delta) {
+  pdl_wait();
+  pdl_trigger();
+  *offset_dev += delta;
+}
 
 // The raw Philox words of the stream (element e = lane e % 4 of block e / 4 + offset).
 __global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restrict__ out, int64_t n, uint32_t k0,
                                                                uint32_t k1, uint32_t s0, uint32_t s1,
                                                                uint64_t offset_host, const uint64_t* offset_dev) {
+  pdl_wait();
+  pdl_trigger();
   const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
   const int64_t nb = (n + 3) >> 2;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -183,7 +191,8 @@ __device__ __forceinline__ float tf32_rna(float v) {
 
 __global__ void __launch_bounds__(kThreads) split_tf32_kernel(float* __restrict__ hi, float* __restrict__ lo,
                                                               const float* __restrict__ src, int64_t n) {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  pdl_wait();
+  pdl_trigger();
   const int64_t n4 = n >> 2;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const float4* s4 = reinterpret_cast<const float4*>(src);
@@ -253,14 +262,14 @@ __global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restri
 }
 
 // The same split with the row held in registers: one block per row, CH chunks of 8 entries per
-// thread, all loads issued before any is used, so a row costs one memory round trip.  The
-// kernel lets a dependent grid (the product that reads the split) start launching at once.
+// thread, all loads issued before any is used, so a row costs one memory round trip.
 template <int CH>
 __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __restrict__ hi,
                                                                    uint16_t* __restrict__ lo,
                                                                    int* __restrict__ row_exp,
                                                                    const float* __restrict__ src, int64_t cols) {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  pdl_wait();
+  pdl_trigger();
   __shared__ float warp_max[kThreads / 32];
   const int64_t r = blockIdx.x;
   const float4* row = reinterpret_cast<const float4*>(src + r * cols);
@@ -331,16 +340,15 @@ spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, 
   const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
   const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
   if (b == 0.0f) {
-    noise_mask_kernel<kZero><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset,
-                                                                 rng.offset_dev);
+    return launch_pdl(noise_mask_kernel<kZero>, dim3(grid), dim3(kThreads), stream, xt, nout, x, n, b, k0, k1, s0,
+                      s1, rng.offset, rng.offset_dev);
   } else if (mech == SPL_MECH_LAPLACE) {
-    noise_mask_kernel<kLaplace><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset,
-                                                                 rng.offset_dev);
+    return launch_pdl(noise_mask_kernel<kLaplace>, dim3(grid), dim3(kThreads), stream, xt, nout, x, n, b, k0, k1, s0,
+                      s1, rng.offset, rng.offset_dev);
   } else {
-    noise_mask_kernel<kGaussian><<<grid, kThreads, 0, stream>>>(xt, nout, x, n, b, k0, k1, s0, s1, rng.offset,
-                                                                 rng.offset_dev);
+    return launch_pdl(noise_mask_kernel<kGaussian>, dim3(grid), dim3(kThreads), stream, xt, nout, x, n, b, k0, k1, s0,
+                      s1, rng.offset, rng.offset_dev);
   }
-  return launch_status();
 }
 
 }  // namespace
@@ -351,23 +359,22 @@ spl_status run_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const fl
   if (rows > 0x7fffffffLL) return SPL_ESHAPE;
   const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
   if (per_thread <= 1) {
-    split_fp16_regs_kernel<1><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<1>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
   } else if (per_thread <= 2) {
-    split_fp16_regs_kernel<2><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<2>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
   } else if (per_thread <= 4) {
-    split_fp16_regs_kernel<4><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<4>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
   } else if (per_thread <= 8) {
-    split_fp16_regs_kernel<8><<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<8>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
   } else {
-    split_fp16_kernel<<<(unsigned)rows, kThreads, 0, stream>>>(hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_kernel, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
   }
-  return launch_status();
 }
 
 spl_status run_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {
   if (count == 0) return SPL_OK;
-  split_tf32_kernel<<<grid_for(ceil_div(count, 4), 8), kThreads, 0, stream>>>(hi, lo, src, count);
-  return launch_status();
+  return launch_pdl(split_tf32_kernel, dim3(grid_for(ceil_div(count, 4), 8)), dim3(kThreads), stream, hi, lo, src,
+                    count);
 }
 
 spl_status run_addsub(float* out, const float* a, const float* b, int64_t n, bool sub, cudaStream_t stream) {
@@ -402,17 +409,15 @@ extern "C" spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng,
   if (count == 0) return SPL_OK;
   if (!out) return SPL_EINVAL;
   if (!aligned16(out)) return SPL_EALIGN;
-  random_bits_kernel<<<grid_for(ceil_div(count, 4), 8), kThreads, 0, stream>>>(
-      out, count, (uint32_t)rng.seed, (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id,
-      (uint32_t)(rng.stream_id >> 32), rng.offset, rng.offset_dev);
-  return launch_status();
+  return launch_pdl(random_bits_kernel, dim3(grid_for(ceil_div(count, 4), 8)), dim3(kThreads), stream, out, count,
+                    (uint32_t)rng.seed, (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id,
+                    (uint32_t)(rng.stream_id >> 32), rng.offset, rng.offset_dev);
 }
 
 extern "C" spl_status spl_rng_advance(uint64_t* offset_dev, uint64_t delta, cudaStream_t stream) {
   if (!offset_dev) return SPL_EINVAL;
   if ((reinterpret_cast<uintptr_t>(offset_dev) & 7u) != 0) return SPL_EALIGN;
-  rng_advance_kernel<<<1, 1, 0, stream>>>(offset_dev, delta);
-  return launch_status();
+  return launch_pdl(rng_advance_kernel, dim3(1), dim3(1), stream, offset_dev, delta);
 }
 
 extern "C" spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, int64_t rows, int64_t cols,

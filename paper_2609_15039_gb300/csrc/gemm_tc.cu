@@ -60,7 +60,7 @@ constexpr int BM = 128, THREADS = 192;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
 constexpr unsigned long long kDrainNs = 100000000ull;  // 0.1 s to drain on abort
 constexpr int MAX_CLUSTER = 8;                         // split-K CTAs of one output tile (portable cluster)
-constexpr uint32_t AUX_BYTES = 1024;                   // barriers, TMEM slot, abort flag
+constexpr uint32_t AUX_BYTES = 2048;                   // barriers, TMEM slot, abort flag; column scales at +1024
 
 // ---- instruction descriptors (tcgen05.mma kind::tf32 / kind::f16) ---------------
 // D = F32 (bits 4-5 = 1); A and B formats at bits 7-9 and 10-12 (f16: 0, tf32: 2);
@@ -104,7 +104,7 @@ struct Cfg {
                 "swizzle atoms aligned");
   static_assert(STAGES >= 3 && STAGES <= 8, "ring depth");
   static_assert((size_t)BM * RED_STRIDE * 4 <= RING, "staging fits in the stage ring");
-  static_assert(8 * (2 * STAGES + 3) + 16 <= AUX_BYTES, "aux fits");
+  static_assert(8 * (2 * STAGES + 3) + 16 <= 1024 && 1024 + 4 * BN <= AUX_BYTES, "aux fits");
 };
 
 // Shared-memory matrix descriptor for a K-major operand tile with the 64-byte swizzle:
@@ -224,9 +224,6 @@ __device__ __forceinline__ void tmem_ld_32x32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
-// Programmatic dependent launch: wait until the grid this one depends on has completed and its
-// memory is visible (returns at once when the launch did not use programmatic serialization).
-__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 // 32 lanes x 32 columns of 32-bit words back to TMEM (thread t writes lane base + t).
 __device__ __forceinline__ void tmem_st_32x32(uint32_t taddr, const float (&v)[32]) {
   asm volatile(
@@ -245,6 +242,8 @@ __device__ __forceinline__ void tmem_st_32x32(uint32_t taddr, const float (&v)[3
       : "memory");
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
+__device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+__device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
@@ -295,6 +294,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (2 * STAGES + 3));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (2 * STAGES + 3) + 8);
   float* red = reinterpret_cast<float*>(smem);  // [BM][RED_STRIDE] staged accumulator, after the mainloop
+  float* col_scale = reinterpret_cast<float*>(aux + 1024);  // [BN] FP16X3: 2^-e of the tile's W rows
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // Linear tile id, M fastest: the CTAs that read the same weight tile run side by side and share it in L2.
@@ -352,7 +352,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       }
       issued_mask |= 1u << kb;
     }
-    grid_dependency_wait();
+    pdl_wait();
     for (int kb = 0; kb < pre; ++kb) {
       if (kb == skip_kblock) continue;
       if (lane == 0) {
@@ -382,6 +382,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       issued_mask |= 1u << s;
       phase_mask = (phase_mask & ~(1u << s)) | (ph << s);
     }
+    pdl_trigger();  // this CTA's loads are issued: the next kernel may be scheduled
     if (!ok) {
       if (lane == 0) {
         *abort_flag = 1;
@@ -421,6 +422,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       }
       __syncwarp();
     }
+    pdl_trigger();
     if (lane == 0) {
       if (!ok) {
         *abort_flag = 1;
@@ -433,8 +435,27 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   } else {
     // ---------------- warps 2..5: stage the accumulator in shared memory ----------------
     // (the ring is free once the MMAs are done)
-    grid_dependency_wait();  // the row exponents of A come from the kernel before this one
+    // While the mainloop runs: the column scales of the tile into shared memory, and the rows of
+    // C this CTA will subtract into L2, so that the epilogue does not wait on DRAM for them.
+    const int t = threadIdx.x - 64;  // 0..127
+    if constexpr (Md::kF16)
+      for (int j = t; j < BN; j += 128) col_scale[j] = pow2f(-((n0 + j < N) ? __ldg(w_exp + n0 + j) : 0));
+    if (C && (N & 3) == 0) {
+      const int rows_per_rank = (BM + splits - 1) / splits;
+      const int rank = splits > 1 ? (int)cluster_rank() : 0;
+      const int r0 = rank * rows_per_rank, r1 = (r0 + rows_per_rank < BM) ? r0 + rows_per_rank : BM;
+      const int64_t ncols = std::min<int64_t>(BN, N - n0);
+      const int lines = (int)ceil_div(ncols * 4, 128);
+      for (int i = t; i < (r1 - r0) * lines; i += 128) {
+        const int64_t m = m0 + r0 + i / lines;
+        if (m < M) prefetch_l2(C + m * N + n0 + (int64_t)(i % lines) * 32);
+      }
+    }
+    pdl_wait();  // the row exponents of A come from the kernel before this one
     const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int r_own = 32 * q + lane;
+    const int e_row = (Md::kF16 && m0 + r_own < M) ? __ldg(a_exp + m0 + r_own) : 0;
+    epilogue_sync();  // col_scale is complete
     bool ok = true;
     for (int f = 0; f + 1 < nseg; ++f) {  // segmented: fold segment f + 1 (in P) into R
       ok = __all_sync(0xffffffffu, mbar_wait(seg_bar, (uint32_t)f & 1u, kWaitNs * 4, abort_flag));
@@ -456,12 +477,12 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     }
     bool have = ok && (nk == 0 || mbar_wait(accum_bar, 0u, kWaitNs * 4, abort_flag));
     have = __all_sync(0xffffffffu, have) && !*abort_flag;
+    pdl_trigger();
     if (have) {
       tc_fence_after();
       const int r = 32 * q + lane;
       float* row = red + (size_t)r * RED_STRIDE;
-      float sr = 1.0f;
-      if constexpr (Md::kF16) sr = pow2f(-((m0 + r < M) ? __ldg(a_exp + m0 + r) : 0));
+      const float sr = pow2f(-e_row);
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         float v[32];
@@ -472,10 +493,8 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
         if constexpr (Md::kF16) {
-          // exact power-of-two scaling; the 32 column exponents are the same for every lane
-          const int64_t nc = n0 + 32 * c;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = (v[i] * sr) * pow2f(-((nc + i < N) ? __ldg(w_exp + nc + i) : 0));
+          for (int i = 0; i < 32; ++i) v[i] = (v[i] * sr) * col_scale[32 * c + i];  // exact power-of-two scaling
         }
 #pragma unroll
         for (int j = 0; j < 32; j += 4)
