@@ -48,6 +48,10 @@ def parse():
     ap.add_argument("--cpu-sample-rows", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--workload", default="llama_layer",
+                    choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep"],
+                    help="llama_layer (default): the headline line; the others measure the stack and sweep "
+                         "workloads and print their own line")
     return ap.parse_args()
 
 
@@ -189,10 +193,35 @@ def run_reference(args):
 
 
 # ----------------------------------------------------------------------------- our arm
+def run_workload(args):
+    """bench.py --workload llama_stack | qwen_stack | qwen_sweep: one JSON line of that workload."""
+    import torch
+    from paper_2609_15039_gb300 import measure
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    with ClockSampler(local) as clocks:
+        res = measure.WORKLOADS[args.workload]()
+    if args.workload == "llama_stack":
+        value, unit, ms = res["prefill"]["tflops"], UNIT, res["prefill"]["ms_per_prefill"]
+    elif args.workload == "qwen_stack":
+        first = next(iter(res["prefill"].values()))
+        value, unit, ms = first["tflops"], UNIT, first["ms_per_prefill"]
+    else:
+        last = list(res["sweep"].values())[-1]
+        value, unit, ms = last["tflops"], UNIT, last["online_ms"]
+    if rank == 0:
+        print(json.dumps({"metric": METRIC, "value": value, "unit": unit, "n_gpus": world, "ms_per_step": ms,
+                          "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                          "data": "synthetic", "config": {"workload": res.pop("workload")}, "clocks": clocks.summary(),
+                          **res}))
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload != "llama_layer":
+        return run_workload(args)
     import numpy as np
     import torch
     import torch.distributed as dist

@@ -132,14 +132,23 @@ class MaskedLayer:
         return path
 
     # ------------------------------------------------------------------ bank
-    def allocate(self, M, draws, path="auto"):
-        """Buffers for M tokens and a bank of ``draws`` corrections per group."""
-        dev = self.groups[0].W.device
+    def workspace_bytes(self, M, draws, path="auto"):
+        """Workspace for products of M rows and a bank refill of draws x M rows, every group."""
         need = 0
         for g in self.groups:
             need = max(need, spl.spl_linear_workspace_bytes(M, g.K, g.N, path),
                        spl.spl_precompute_matched_workspace_bytes(draws * M, g.K, g.N, M, path))
-        if self.workspace is None or self.workspace.numel() < need:
+        return need
+
+    def allocate(self, M, draws, path="auto", workspace=None):
+        """Buffers for M tokens and a bank of ``draws`` corrections per group.  ``workspace`` may be
+        shared with other layers whose calls run on the same stream."""
+        dev = self.groups[0].W.device
+        need = self.workspace_bytes(M, draws, path)
+        if workspace is not None:
+            assert workspace.numel() >= need, "shared workspace too small"
+            self.workspace = workspace
+        elif self.workspace is None or self.workspace.numel() < need:
             self.workspace = spl.workspace(need, dev)
         self.M, self.draws = M, draws
         self.rng_base = torch.zeros(len(self.groups), dtype=torch.int64, device=dev)
@@ -243,6 +252,79 @@ class MaskedLayer:
     def flops_per_step(self):
         """Algorithmic flops per online step: the masked product plus its share of the batched correction."""
         return sum(2 * 2 * self.M * g.K * g.N for g in self.groups)
+
+
+class MaskedStack:
+    """The linear layers of a decoder stack, each a MaskedLayer with its own weights, noise scales,
+    Philox seed and correction bank, run in order on one stream with one shared workspace."""
+
+    def __init__(self, layers, seeds):
+        self.layers, self.seeds = layers, seeds
+
+    @classmethod
+    def build(cls, model, n_layers, M, draws, base_seed, device="cuda", split=True, power_iters=1000, path="auto"):
+        """Seeded synthetic weights per layer (workloads.layer_seed), Delta per layer (Thms. 1-3)."""
+        from . import workloads as wl
+        layers = []
+        for li in range(n_layers):
+            weights = {name: wl.weight(N, K, seed=wl.layer_seed(base_seed, li, pi), device=device)
+                       for pi, (name, K, N, _g) in enumerate(model.projections())}
+            layer = MaskedLayer.from_weights(model, weights, split=split, device=device)
+            del weights
+            layer.sensitivities(power_iters=power_iters)
+            layers.append(layer)
+        need = max(l.workspace_bytes(M, draws, path) for l in layers)
+        ws = spl.workspace(need, device)
+        for layer in layers:
+            layer.allocate(M, draws, path, workspace=ws)
+        return cls(layers, [wl.layer_seed(base_seed, li, 99) for li in range(n_layers)])
+
+    @property
+    def draws(self):
+        return self.layers[0].draws
+
+    def inputs(self, base_seed, device="cuda"):
+        """Seeded synthetic activations per layer and group (the enclave-side ops between the
+        linears -- attention, norms, activation -- are not part of this path)."""
+        from . import workloads as wl
+        return [{g: wl.activations(layer.M, K, seed=wl.layer_seed(base_seed, li, 50 + gi), device=device)
+                 for gi, (g, K, _n) in enumerate(layer.model.input_groups())} for li, layer in enumerate(self.layers)]
+
+    def step(self, inputs, eps, mech, s, path="auto", refill=True):
+        """Eager step s (draw s % draws of bank cycle s // draws) through every layer."""
+        cycle, d = divmod(s, self.draws)
+        for layer, x, seed in zip(self.layers, inputs, self.seeds):
+            if d == 0 and refill:
+                layer.refill(eps, mech, seed, cycle, path=path)
+            layer.online(x, eps, mech, seed, cycle, d, path=path)
+
+    def set_cycle(self, cycle):
+        for layer in self.layers:
+            layer.set_cycle(cycle)
+
+    def capture(self, inputs, eps, mech, path="auto", refill=True):
+        """CUDA graphs of one bank cycle for the whole stack (see MaskedLayer.capture); graph 0
+        refills every layer's bank first unless ``refill`` is False."""
+        graphs, launches = [], []
+        D = self.draws
+        for d in range(D):
+            graph = torch.cuda.CUDAGraph()
+            n0 = spl.spl_launch_count()
+            with torch.cuda.graph(graph):
+                for layer, x, seed in zip(self.layers, inputs, self.seeds):
+                    if d == 0 and refill:
+                        layer.refill(eps, mech, seed, 0, path=path, device_base=True)
+                    layer.online(x, eps, mech, seed, 0, d, path=path, device_base=True)
+                if d == D - 1:
+                    for layer in self.layers:
+                        for gi, g in enumerate(layer.groups):
+                            spl.spl_rng_advance(layer.rng_base[gi:gi + 1], D * (layer.M * g.K // 4))
+            graphs.append(graph)
+            launches.append(spl.spl_launch_count() - n0)
+        return graphs, launches
+
+    def flops_per_step(self):
+        return sum(l.flops_per_step() for l in self.layers)
 
 
 def split_outputs(layer, outs):

@@ -1,0 +1,226 @@
+"""Measurements of the stack and sweep workloads (bench.py --workload ...).
+
+Each function runs one workload on the current CUDA device through the library (MaskedStack /
+MaskedLayer sequencing ABI calls, replayed as CUDA graphs) and returns a dict that bench.py
+prints as its JSON line.  Times are CUDA events on the launching stream around graph replays;
+inputs are resident in HBM.  The workloads:
+
+* llama_stack -- 28 Llama-3.2-3B-shaped layers: prefill of 512 tokens (banks of 8 draws), then
+  decode at one token per step for 256 steps (its own banks of 8 one-row draws); Laplace, eps = 1.
+* qwen_stack  -- 36 Qwen3-4B-shaped layers, prefill of 2048 tokens at eps in {0.1, 1, 10} with
+  the cancellation error of every output of the first and last layer checked against the bound.
+* qwen_sweep  -- one Qwen3-4B-shaped layer at M in {1, 4, 16, 64, 256, 1024} tokens, and the
+  noise + mask kernel alone on 10^9 elements.
+"""
+
+import torch
+
+from . import spl, workloads as wl
+from .layer import MaskedStack
+
+
+def _peaks():
+    import json
+    import os
+    p = {"hbm_gbs": 6800.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+    path = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            m = json.load(f)
+        p.update({k: float(m[k]) for k in ("hbm_gbs", "bf16_tflops_sustained") if k in m})
+        p["source"] = "measured"
+    except (OSError, ValueError, KeyError):
+        pass
+    return p
+
+
+def _path_peak(path, pk):
+    """Algorithmic TFLOP/s at each path's instruction peak (see bench.py)."""
+    return {"fp16x3": pk["bf16_tflops_sustained"] / 3.0,
+            "tf32x3": pk["bf16_tflops_sustained"] * (1.1 / 2.25) / 3.0,
+            "fp32": 152 * 128 * 2 * 2.07e9 / 1e12}[path]
+
+
+def _group_paths(stack_or_layer, M):
+    layers = getattr(stack_or_layer, "layers", [stack_or_layer])
+    out = {}
+    for g in layers[0].groups:
+        out[g.name] = spl.PATH_NAMES[spl.spl_resolve_path(M, g.K, g.N, layers[0].path_of(g, "auto", M))]
+    return out
+
+
+def _weight_bytes(layer, M, paths):
+    """HBM bytes of one online step of a layer: the weight in the format its path reads, x~ in,
+    C in, Y out (fp32)."""
+    per_w = {"fp32": 4, "tf32x3": 8, "fp16x3": 4}
+    total = 0
+    for g in layer.groups:
+        total += per_w[paths[g.name]] * g.K * g.N + 4 * M * g.K + 8 * M * g.N
+    return total
+
+
+def _time_replays(graphs, start, n, stream):
+    """Replays graphs[(start + i) % D] for i < n; returns per-replay ms (events around each)."""
+    D = len(graphs)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    ev[0].record(stream)
+    for i in range(n):
+        graphs[(start + i) % D].replay()
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize()
+    return [ev[i].elapsed_time(ev[i + 1]) for i in range(n)]
+
+
+def _calibrate(stack, inputs, eps, mech):
+    for layer, x, seed in zip(stack.layers, inputs, stack.seeds):
+        layer.calibrate(x, eps, mech, seed)
+
+
+def _bound(stack, inputs, eps, mech, s, layers):
+    """The bound over every output of layers ``layers`` for eager step s (its bank cycle is
+    refilled first, whatever the bank held before)."""
+    cycle, d = divmod(s, stack.draws)
+    res = {}
+    for li in layers:
+        layer, x, seed = stack.layers[li], inputs[li], stack.seeds[li]
+        layer.refill(eps, mech, seed, cycle)
+        outs = layer.online(x, eps, mech, seed, cycle, d)
+        bc = layer.bound_check(x, outs, eps, mech, seed, cycle, d)
+        res[f"layer{li}"] = {g: {"max_err_over_hard": v["max_err_over_hard"], "log_violation_pct": v["violation_pct"],
+                                 "mean_err": v["mean_err"], "mean_log_bound": v["mean_log_bound"]}
+                             for g, v in bc.items()}
+    return res
+
+
+def _prefill(stack, inputs, eps, mech, cycles=2):
+    """Graph-replayed prefill: online-only steps (draws 1..D-1) and the draw-0 step that also
+    refills every bank; returns ms per online pass and per refill."""
+    stream = torch.cuda.current_stream()
+    D = stack.draws
+    stack.step(inputs, eps, mech, 0)  # sets up every library call before capture
+    torch.cuda.synchronize()
+    graphs, launches = stack.capture(inputs, eps, mech)
+    stack.set_cycle(1)
+    _time_replays(graphs, 0, D, stream)  # warm-up cycle
+    times = _time_replays(graphs, 0, cycles * D, stream)
+    online = [t for i, t in enumerate(times) if i % D != 0]
+    with_refill = [t for i, t in enumerate(times) if i % D == 0]
+    on = sum(online) / len(online) if online else float("nan")
+    rf = sum(with_refill) / len(with_refill) - (on if online else 0.0)
+    del graphs
+    torch.cuda.synchronize()
+    return on, rf, launches
+
+
+def llama_stack(layers=28, tokens=512, decode_steps=256, eps=1.0, mech="laplace", draws=8):
+    model = wl.LLAMA_3_2_3B
+    pk = _peaks()
+    stack = MaskedStack.build(model, layers, tokens, draws, base_seed=7)
+    inputs = stack.inputs(11)
+    _calibrate(stack, inputs, eps, mech)
+    paths = _group_paths(stack, tokens)
+    on_ms, refill_ms, launches = _prefill(stack, inputs, eps, mech)
+    flops = 2 * tokens * model.weights_per_layer() * layers
+    peak = flops / sum(2 * tokens * g.K * g.N * layers / _path_peak(paths[g.name], pk) for g in stack.layers[0].groups)
+    prefill = {"ms_per_prefill": on_ms, "tflops": flops / (on_ms * 1e-3) / 1e12, "tokens_per_s": tokens / (on_ms * 1e-3),
+               "roofline_peak_tflops": peak, "frac": flops / (on_ms * 1e-3) / 1e12 / peak,
+               "bank_refill_ms": refill_ms, "bank_refill_ms_per_draw": refill_ms / draws,
+               "bank_refill_tflops": draws * flops / (refill_ms * 1e-3) / 1e12, "paths": paths,
+               "kernels_per_online_step": launches[1] if len(launches) > 1 else launches[0]}
+    bound = _bound(stack, inputs, eps, mech, 3 * draws + 1, [0, layers - 1])
+    # decode: the same layers re-allocated for one token per step, banks of `draws` one-row draws
+    ws = spl.workspace(max(l.workspace_bytes(1, draws) for l in stack.layers))
+    for layer in stack.layers:
+        layer.allocate(1, draws, workspace=ws)
+    inputs1 = stack.inputs(13)
+    stream = torch.cuda.current_stream()
+    stack.step(inputs1, eps, mech, 0)
+    torch.cuda.synchronize()
+    graphs, dl = stack.capture(inputs1, eps, mech)
+    stack.set_cycle(1)
+    _time_replays(graphs, 0, draws, stream)
+    times = _time_replays(graphs, 0, decode_steps, stream)
+    step_ms = sum(times) / len(times)
+    dpaths = _group_paths(stack, 1)
+    step_bytes = sum(_weight_bytes(l, 1, dpaths) for l in stack.layers) * (1 + 1.0 / draws)  # + the bank's share
+    decode = {"steps": decode_steps, "ms_per_token": step_ms, "tokens_per_s": 1e3 / step_ms,
+              "gbs": step_bytes / (step_ms * 1e-3) / 1e9, "hbm_peak_gbs": pk["hbm_gbs"],
+              "frac": step_bytes / (step_ms * 1e-3) / 1e9 / pk["hbm_gbs"], "bytes_per_step": step_bytes,
+              "paths": dpaths, "kernels_per_step": sum(dl) / len(dl)}
+    del graphs
+    return {"workload": f"llama-3.2-3b-shaped stack, {layers} layers, prefill {tokens} tokens + decode "
+                        f"{decode_steps} steps at 1 token, {mech} eps={eps}, banks of {draws} draws",
+            "prefill": prefill, "decode": decode, "bound_check": bound, "peak_source": pk["source"]}
+
+
+def qwen_stack(layers=36, tokens=2048, eps_list=(0.1, 1.0, 10.0), mech="gaussian", draws=2):
+    model = wl.QWEN3_4B
+    pk = _peaks()
+    stack = MaskedStack.build(model, layers, tokens, draws, base_seed=11)
+    inputs = stack.inputs(17)
+    res = {}
+    flops = 2 * tokens * model.weights_per_layer() * layers
+    for eps in eps_list:
+        _calibrate(stack, inputs, eps, mech)
+        paths = _group_paths(stack, tokens)
+        on_ms, refill_ms, _ = _prefill(stack, inputs, eps, mech, cycles=2)
+        peak = flops / sum(2 * tokens * g.K * g.N * layers / _path_peak(paths[g.name], pk)
+                           for g in stack.layers[0].groups)
+        res[f"eps={eps}"] = {
+            "ms_per_prefill": on_ms, "tflops": flops / (on_ms * 1e-3) / 1e12, "tokens_per_s": tokens / (on_ms * 1e-3),
+            "roofline_peak_tflops": peak, "frac": flops / (on_ms * 1e-3) / 1e12 / peak,
+            "bank_refill_ms_per_draw": refill_ms / draws, "paths": paths,
+            "bound_check": _bound(stack, inputs, eps, mech, 5 * draws + 1, [0, layers - 1])}
+    return {"workload": f"qwen3-4b-shaped stack, {layers} layers, prefill {tokens} tokens, {mech}, "
+                        f"banks of {draws} draws", "prefill": res, "peak_source": pk["source"]}
+
+
+def qwen_sweep(Ms=(1, 4, 16, 64, 256, 1024), eps=1.0, mech="gaussian", draws=8, mask_elements=10 ** 9):
+    model = wl.QWEN3_4B
+    pk = _peaks()
+    stack = MaskedStack.build(model, 1, Ms[0], draws, base_seed=13)
+    layer = stack.layers[0]
+    out = {}
+    for M in Ms:
+        ws = spl.workspace(layer.workspace_bytes(M, draws))
+        layer.allocate(M, draws, workspace=ws)
+        inputs = stack.inputs(19)
+        _calibrate(stack, inputs, eps, mech)
+        paths = _group_paths(stack, M)
+        on_ms, refill_ms, _ = _prefill(stack, inputs, eps, mech, cycles=4)
+        flops = 2 * M * model.weights_per_layer()
+        nbytes = _weight_bytes(layer, M, paths)
+        peak_t = flops / sum(2 * M * g.K * g.N / _path_peak(paths[g.name], pk) for g in layer.groups)
+        t_hbm = nbytes / (pk["hbm_gbs"] * 1e9)
+        t_tc = flops / (peak_t * 1e12)
+        out[f"M={M}"] = {"online_ms": on_ms, "tflops": flops / (on_ms * 1e-3) / 1e12,
+                         "gbs": nbytes / (on_ms * 1e-3) / 1e9, "bound": "hbm" if t_hbm >= t_tc else "tensor",
+                         "roofline_ms": max(t_hbm, t_tc) * 1e3, "frac": max(t_hbm, t_tc) * 1e3 / on_ms,
+                         "bank_refill_ms_per_draw": refill_ms / draws, "paths": paths}
+        del ws
+    # the noise + mask kernel alone (eta regenerated, not stored): 8 bytes per element
+    n = mask_elements
+    X = torch.empty(n, device="cuda")
+    X.normal_(generator=torch.Generator(device="cuda").manual_seed(3))
+    Xt = torch.empty_like(X)
+    stream = torch.cuda.current_stream()
+    mask = {}
+    for m in ("laplace", "gaussian"):
+        for _ in range(2):
+            spl.spl_noise_mask(Xt, None, X, 719.8, 1.0, m, 5)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 10
+        e0.record(stream)
+        for r in range(reps):
+            spl.spl_noise_mask(Xt, None, X, 719.8, 1.0, m, 5, offset=r * (n // 4))
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        mask[m] = {"ms": ms, "gbs": 8 * n / (ms * 1e-3) / 1e9, "frac": 8 * n / (ms * 1e-3) / 1e9 / pk["hbm_gbs"]}
+    return {"workload": f"qwen3-4b-shaped layer, M sweep {list(Ms)}, {mech} eps={eps}, banks of {draws} draws; "
+                        f"noise + mask alone on {n} elements", "sweep": out, "mask": mask,
+            "hbm_peak_gbs": pk["hbm_gbs"], "peak_source": pk["source"]}
+
+
+WORKLOADS = {"llama_stack": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep}
