@@ -340,13 +340,13 @@ spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, 
   const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
   const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
   if (b == 0.0f) {
-    return launch_pdl(noise_mask_kernel<kZero>, dim3(grid), dim3(kThreads), stream, xt, nout, x, n, b, k0, k1, s0,
+    return launch_pdl(noise_mask_kernel<kZero>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, k0, k1, s0,
                       s1, rng.offset, rng.offset_dev);
   } else if (mech == SPL_MECH_LAPLACE) {
-    return launch_pdl(noise_mask_kernel<kLaplace>, dim3(grid), dim3(kThreads), stream, xt, nout, x, n, b, k0, k1, s0,
+    return launch_pdl(noise_mask_kernel<kLaplace>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, k0, k1, s0,
                       s1, rng.offset, rng.offset_dev);
   } else {
-    return launch_pdl(noise_mask_kernel<kGaussian>, dim3(grid), dim3(kThreads), stream, xt, nout, x, n, b, k0, k1, s0,
+    return launch_pdl(noise_mask_kernel<kGaussian>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, k0, k1, s0,
                       s1, rng.offset, rng.offset_dev);
   }
 }
@@ -359,21 +359,21 @@ spl_status run_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const fl
   if (rows > 0x7fffffffLL) return SPL_ESHAPE;
   const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
   if (per_thread <= 1) {
-    return launch_pdl(split_fp16_regs_kernel<1>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<1>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
   } else if (per_thread <= 2) {
-    return launch_pdl(split_fp16_regs_kernel<2>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<2>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
   } else if (per_thread <= 4) {
-    return launch_pdl(split_fp16_regs_kernel<4>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<4>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
   } else if (per_thread <= 8) {
-    return launch_pdl(split_fp16_regs_kernel<8>, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_regs_kernel<8>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
   } else {
-    return launch_pdl(split_fp16_kernel, dim3((unsigned)rows), dim3(kThreads), stream, hi, lo, row_exp, src, cols);
+    return launch_pdl(split_fp16_kernel, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
   }
 }
 
 spl_status run_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {
   if (count == 0) return SPL_OK;
-  return launch_pdl(split_tf32_kernel, dim3(grid_for(ceil_div(count, 4), 8)), dim3(kThreads), stream, hi, lo, src,
+  return launch_pdl(split_tf32_kernel, dim3(grid_for(ceil_div(count, 4), 8)), dim3(kThreads), 0, stream, hi, lo, src,
                     count);
 }
 
@@ -409,7 +409,7 @@ extern "C" spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng,
   if (count == 0) return SPL_OK;
   if (!out) return SPL_EINVAL;
   if (!aligned16(out)) return SPL_EALIGN;
-  return launch_pdl(random_bits_kernel, dim3(grid_for(ceil_div(count, 4), 8)), dim3(kThreads), stream, out, count,
+  return launch_pdl(random_bits_kernel, dim3(grid_for(ceil_div(count, 4), 8)), dim3(kThreads), 0, stream, out, count,
                     (uint32_t)rng.seed, (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id,
                     (uint32_t)(rng.stream_id >> 32), rng.offset, rng.offset_dev);
 }
@@ -417,7 +417,7 @@ extern "C" spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng,
 extern "C" spl_status spl_rng_advance(uint64_t* offset_dev, uint64_t delta, cudaStream_t stream) {
   if (!offset_dev) return SPL_EINVAL;
   if ((reinterpret_cast<uintptr_t>(offset_dev) & 7u) != 0) return SPL_EALIGN;
-  return launch_pdl(rng_advance_kernel, dim3(1), dim3(1), stream, offset_dev, delta);
+  return launch_pdl(rng_advance_kernel, dim3(1), dim3(1), 0, stream, offset_dev, delta);
 }
 
 extern "C" spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, int64_t rows, int64_t cols,

@@ -27,14 +27,15 @@ namespace {
 constexpr int THREADS = 256, WARPS = 8;
 constexpr int SMEM_FLOATS = 12000;  // just under 48 KB of X~ slice (static smem adds a few bytes)
 
-// Rows of W per warp: 4 for M <= 4, 2 for larger M (bounds the 4 x M accumulators).
+// Rows of W per warp: 4 for M <= 4, 2 for larger M (bounds the rows x M accumulators and keeps
+// four blocks resident per SM).
 constexpr int rows_per_warp(int mt) { return mt >= 8 ? 2 : 4; }
 
 template <int MT, int ROWS_PER_WARP>
 __global__ void __launch_bounds__(THREADS)
 gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* __restrict__ W,
             const float* __restrict__ C, float* __restrict__ part, unsigned int* __restrict__ counters, int M,
-            int64_t K, int64_t N, int64_t ks, int splits) {
+            int64_t K, int64_t N, int64_t ks, int splits, int64_t prefetch_bytes) {
   constexpr int ROWS_PER_BLOCK = WARPS * ROWS_PER_WARP;
   extern __shared__ __align__(16) float xs[];  // [MT][ks]
   __shared__ int s_last;
@@ -42,6 +43,18 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
   const int split = blockIdx.y;
   const int64_t k0 = (int64_t)split * ks;
   const int64_t klen = std::min<int64_t>(ks, K - k0);  // multiple of 4
+
+  // the first prefetch_bytes of each of this warp's W rows (slice k0..k0+klen) into L2
+  {
+    const int64_t n_first = (int64_t)blockIdx.x * ROWS_PER_BLOCK + warp * ROWS_PER_WARP;
+    const int64_t lines = std::min<int64_t>(prefetch_bytes, klen * 4) >> 7;  // 128-byte lines per row
+    for (int r = 0; r < ROWS_PER_WARP; ++r) {
+      if (n_first + r >= N) break;
+      const char* base = reinterpret_cast<const char*>(W + (n_first + r) * K + k0);
+      for (int64_t l = lane; l < lines; l += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(base + 128 * l));
+    }
+  }
+  pdl_wait();
 
   // stage X~[:, k0:k0+klen] (rows >= M are zero)
   const int64_t q_per_row = klen >> 2;
@@ -89,6 +102,8 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
       }
     }
   }
+
+  pdl_trigger();  // W is streamed: the next kernel may be scheduled
 
   // warp reduction: lane 0 ends with the full sums
 #pragma unroll
@@ -158,14 +173,49 @@ spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int*
   constexpr int R = rows_per_warp(MT);
   dim3 grid((unsigned)ceil_div(a.N, WARPS * R), (unsigned)p.splits);
   const size_t smem = (size_t)MT * p.k_per_split * sizeof(float);
-  gemv_kernel<MT, R><<<grid, THREADS, smem, a.stream>>>(a.out, a.a, a.w, a.c, part, counters, (int)a.M, a.K, a.N,
-                                                      p.k_per_split, p.splits);
-  return launch_status();
+  // L2 budget of the early prefetch: about 32 MB over the whole grid
+  const int64_t rows = (int64_t)grid.x * WARPS * R * p.splits;
+  const int64_t prefetch = std::max<int64_t>(0, (int64_t(32) << 20) / std::max<int64_t>(rows, 1));
+  return launch_pdl(gemv_kernel<MT, R>, grid, dim3(THREADS), smem, a.stream, a.out, a.a, a.w, a.c, part, counters,
+                    (int)a.M, a.K, a.N, p.k_per_split, p.splits, prefetch);
+}
+
+// Resident blocks per SM of the decode kernel for MT rows and a K-slice of ks (cached).
+int blocks_per_sm(int mt, int64_t ks) {
+  static std::mutex mu;
+  static int cache[64][5][128] = {{{0}}};  // device, log2(mt), ks / 128 (ks <= 12000 / mt)
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  const int mi = mt == 1 ? 0 : mt == 2 ? 1 : mt == 4 ? 2 : mt == 8 ? 3 : 4;
+  const int ki = (int)std::min<int64_t>(127, ks / 128);
+  std::lock_guard<std::mutex> lock(mu);
+  int& v = cache[dev][mi][ki];
+  if (v == 0) {
+    const size_t smem = (size_t)mt * ks * sizeof(float);
+    int n = 0;
+    cudaError_t e = cudaErrorInvalidValue;
+    switch (mt) {
+      case 1: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<1, rows_per_warp(1)>, THREADS, smem); break;
+      case 2: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<2, rows_per_warp(2)>, THREADS, smem); break;
+      case 4: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<4, rows_per_warp(4)>, THREADS, smem); break;
+      case 8: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<8, rows_per_warp(8)>, THREADS, smem); break;
+      default: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<16, rows_per_warp(16)>, THREADS, smem);
+    }
+    if (e != cudaSuccess) cudaGetLastError();
+    v = (e == cudaSuccess && n > 0) ? n : 1;
+  }
+  return v;
 }
 
 }  // namespace
 
 int64_t gemv_max_ks(int64_t M) { return (SMEM_FLOATS / padded_m(M)) / 128 * 128; }
+
+// K-split of the decode kernel: the number of splits s minimises waves(s) x (K/s + F), waves
+// counting the resident block slots of all SMs, with K/s a multiple of 128 that fits the shared-
+// memory slice and at least 256; F (the fixed cost of a block -- staging X~, the warp reduction,
+// the split-K reduction -- in units of K) measured on GB300.
+constexpr double kGemvFixedK = 512.0;
 
 Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
   Plan p{};
@@ -173,13 +223,20 @@ Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
   const int mt = padded_m(M);
   const int64_t ks_max = (SMEM_FLOATS / mt) / 128 * 128;
   const int64_t groups = ceil_div(N, WARPS * rows_per_warp(mt));
-  const int64_t target = (int64_t)sms * 4;  // about four 8-warp blocks per SM
-  int64_t s = std::max<int64_t>(1, ceil_div(target, groups));
-  s = std::min<int64_t>(s, std::max<int64_t>(1, K / 256));  // at least 256 K per split
-  int64_t ks = round_up(ceil_div(K, s), 128);
-  ks = std::min<int64_t>(ks, ks_max);
-  p.k_per_split = ks;
-  p.splits = (int)ceil_div(K, ks);
+  const int64_t s_min = ceil_div(K, ks_max);
+  const int64_t s_max = std::max<int64_t>(s_min, std::min<int64_t>(64, K / 256));
+  double best = 1e300;
+  for (int64_t s = s_min; s <= s_max; ++s) {
+    const int64_t ks = std::min<int64_t>(round_up(ceil_div(K, s), 128), ks_max);
+    const int64_t splits = ceil_div(K, ks);
+    const int64_t slots = (int64_t)sms * blocks_per_sm(mt, ks);
+    const double cost = (double)ceil_div(groups * splits, slots) * ((double)ks + kGemvFixedK);
+    if (cost < best * (1.0 - 1e-9)) {
+      best = cost;
+      p.k_per_split = ks;
+      p.splits = (int)splits;
+    }
+  }
   if (p.splits > 1) p.ws_partials = (size_t)round_up((int64_t)p.splits * M * N * 4, 256);
   return p;
 }

@@ -121,8 +121,12 @@ MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, sp
   mp.splits = online.splits;
   mp.k_per_split = online.k_per_split;
   if (online.kernel == kKernelGemv) {
-    mp.chunk_rows = std::min<int64_t>(M, kGemvMaxM);
-    if (mp.k_per_split > gemv_max_ks(mp.chunk_rows)) return mp;
+    // rows per launch: the most (a power of two up to 16) whose shared-memory K-slice still holds
+    // the online K-split; a row's sum does not depend on how many rows a launch carries
+    mp.chunk_rows = 0;
+    for (int64_t c = kGemvMaxM; c >= 1 && mp.chunk_rows == 0; c /= 2)
+      if (c <= std::max<int64_t>(M, 1) && gemv_max_ks(c) >= mp.k_per_split) mp.chunk_rows = std::min<int64_t>(c, M);
+    if (mp.chunk_rows == 0) return mp;
     if (mp.splits > 1) mp.ws = kCounterBytes + (size_t)round_up((int64_t)mp.splits * mp.chunk_rows * N * 4, 256);
   } else {
     if (mp.splits > 1) mp.ws = kCounterBytes + (size_t)round_up((int64_t)mp.splits * M * N * 4, 256);

@@ -369,7 +369,9 @@ def test_matched_correction_cancels_rounding(spl, M, K, N, path):
 @pytest.mark.parametrize("M,K,N,path", [(128, 3072, 3072, "fp16x3"), (128, 3072, 5120, "fp16x3"),
                                          (128, 8192, 3072, "fp16x3"), (128, 3072, 16384, "fp16x3"),
                                          (128, 3072, 3072, "tf32x3"), (100, 1032, 600, "fp16x3"),
-                                         (128, 3072, 3072, "fp32"), (1, 3072, 3072, "fp32"), (512, 3072, 3072, "fp16x3")])
+                                         (128, 3072, 3072, "fp32"), (1, 3072, 3072, "fp32"), (512, 3072, 3072, "fp16x3"),
+                                         (1, 3072, 5120, "fp32"), (1, 3072, 16384, "fp32"), (1, 8192, 3072, "fp32"),
+                                         (4, 3072, 5120, "fp32"), (3, 1028, 600, "fp32")])
 def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path):
     """The bank's correction of draw d is, bit for bit, what the online product computes when
     its input is that draw's noise: the same K ranges, partials summed in the same order."""
