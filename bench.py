@@ -124,6 +124,23 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def profiled_traffic():
+    """DRAM bytes per step of the online product launches from the committed ncu summary, if it
+    was taken on the current tensor-core kernel source (else None)."""
+    import hashlib
+    prof = os.path.join(ROOT, "profiles", "tc_gemm_fp16x3_llama_online_and_bank.md")
+    src = os.path.join(ROOT, "paper_2609_15039_gb300", "csrc", "gemm_tc.cu")
+    try:
+        fields = dict(line.split(":", 1) for line in open(prof).read().splitlines()
+                      if line.startswith(("traffic_bytes_per_step:", "kernel_source_sha256_prefix:")))
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    except (OSError, ValueError):
+        return None, "no profile"
+    if not digest.startswith(fields.get("kernel_source_sha256_prefix", "-").strip()):
+        return None, "kernel changed since the ncu capture"
+    return float(fields["traffic_bytes_per_step"]), "ncu capture of the same kernel source (profiles/)"
+
+
 def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -351,19 +368,11 @@ def main():
     for (d, kind, group), (b, e) in gevents.items():
         by_kind.setdefault(kind, []).append(b.elapsed_time(e))
         by_group.setdefault((kind, group), []).append(b.elapsed_time(e))
-    prod_ms = sum(sum(v) for v in by_kind.values())  # one bank cycle: DRAWS online steps, one refill
-    achieved = flops_step * DRAWS / (prod_ms * 1e-3) / 1e12
     path_peak = {  # algorithmic flops (one product per term) per second at each path's instruction peak
         "fp16x3": pk["bf16_tflops_sustained"] / 3.0,
         "tf32x3": pk["bf16_tflops_sustained"] * TF32_OVER_BF16 / 3.0,
         "fp32": 152 * 128 * 2 * 2.07e9 / 1e12,
     }
-    # flop-weighted: the time the step's products would take with every group at its path's peak
-    t_peak = sum(2 * 2 * M * g.K * g.N / path_peak[group_paths[g.name]] for g in layer.groups)
-    peak = flops_step / t_peak
-    peak_note = ("per group: fp16x3 = measured sustained bf16 (fp16 runs at the bf16 rate) / 3 products per term; "
-                 "tf32x3 = that x nominal tf32/bf16 (1.1/2.25); fp32 FMA: 152 SMs x 128 lanes x 2 flop x 2.07 GHz "
-                 "(derived); flop-weighted over the groups")
     per_kind = {}
     for kind, v in by_kind.items():
         rows = DRAWS * M if kind == "precompute" else M
@@ -375,14 +384,34 @@ def main():
             avg = sum(t) / len(t)
             per_kind[kind][g.name] = {"avg_us": 1e3 * avg, "tflops": 2 * rows * g.K * g.N / (avg * 1e-3) / 1e12,
                                       "path": group_paths[g.name]}
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": None,
-                "kernel": "tc_gemm_kernel product calls (bank corrections at 1024 rows + online masked products)",
-                "group_paths": group_paths,
-                "share_of_step": prod_ms / (ms_with_events * DRAWS), "per_call": per_kind,
+    # The dominant kernel: the online masked products (a5 + a6), four calls per step.  At 128 rows
+    # they do 64 algorithmic flops per byte, below the FP16X3 ridge (~84), so HBM bounds them:
+    # achieved = algorithmic bytes per step (weight split 4 B per weight or the path's format,
+    # X~ in, C in, Y out) / their measured time per step.
+    online_ms = sum(by_kind["masked_linear_unmask"]) / DRAWS
+    wbytes = {"fp16x3": 4, "tf32x3": 8, "fp32": 4}
+    online_bytes = sum(wbytes[group_paths[g.name]] * g.K * g.N + 4 * M * g.K + 8 * M * g.N for g in layer.groups)
+    achieved = online_bytes / (online_ms * 1e-3) / 1e9
+    bank_ms = sum(by_kind["precompute"])
+    bank_flops = sum(2 * DRAWS * M * g.K * g.N for g in layer.groups)
+    bank_peak = bank_flops / sum(2 * DRAWS * M * g.K * g.N / path_peak[group_paths[g.name]] for g in layer.groups)
+    traffic, traffic_note = profiled_traffic()
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / pk["hbm_gbs"], "traffic": traffic,
+                "kernel": "tc_gemm_kernel online masked products with fused unmask (4 calls per step, 128 rows)",
+                "algorithmic_bytes_per_step": online_bytes, "ms_per_step": online_ms,
+                "traffic_note": traffic_note, "group_paths": group_paths,
+                "share_of_step": (online_ms + bank_ms / DRAWS) / ms_with_events,
+                "bank": {"bound": "tensor", "kernel": "tc_gemm_kernel bank refill, 1024 rows, segmented K",
+                         "achieved": bank_flops / (bank_ms * 1e-3) / 1e12, "peak": bank_peak, "unit": "TFLOP/s",
+                         "frac": bank_flops / (bank_ms * 1e-3) / 1e12 / bank_peak, "ms_per_refill": bank_ms},
+                "per_call": per_kind,
                 "timing": "per-call CUDA events (external event nodes) in a second pass over the same steps; "
                           f"that pass ran at {ms_with_events:.4f} ms/step",
-                "peak_source": pk["source"], "peak_note": peak_note}
+                "peak_source": pk["source"],
+                "peak_note": "hbm: measured copy bandwidth; bank: per group fp16x3 = measured sustained bf16 "
+                             "(fp16 runs at the bf16 rate) / 3 products per term, tf32x3 = that x nominal "
+                             "tf32/bf16 (1.1/2.25), fp32 FMA = 152 SMs x 128 lanes x 2 flop x 2.07 GHz (derived)"}
 
     e2e = None
     if e2e_graphs is not None:
