@@ -165,11 +165,24 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigne
     }
   }
 }
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+// L2 eviction policies: weight tiles are streamed (first out), A tiles are re-read by every
+// output tile of the row block and the rows of C are wanted again in the epilogue (last out).
+__device__ __forceinline__ uint64_t l2_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y,
+                                            uint64_t policy) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-          dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
       : "memory");
 }
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
@@ -243,7 +256,9 @@ __device__ __forceinline__ void tmem_st_32x32(uint32_t taddr, const float (&v)[3
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
-__device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2::evict_last [%0];" ::"l"(p));
+}
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
@@ -269,6 +284,65 @@ __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
 struct TcMaps {
   CUtensorMap a_hi, a_lo, w_hi, w_lo;
 };
+
+// Rows r0..r1 of the staged tile: the S partial tiles of the cluster summed in rank order (S = 1:
+// this CTA's own), minus C, stored.  A thread takes P float4 positions per batch and issues every
+// load of the batch -- S partials and C for each -- before it adds anything, about 16 loads in
+// flight per thread whatever S is, so the epilogue streams instead of waiting load by load.
+template <int S, int BN>
+__device__ __forceinline__ void reduce_store(const float* red, int r0, int r1, int64_t m0, int64_t n0, int64_t M,
+                                             int64_t N, const float* __restrict__ C, float* __restrict__ out) {
+  constexpr int RS = BN + 4;
+  constexpr int P = S >= 8 ? 2 : (S >= 4 ? 4 : 8);
+  const bool vec = (N & 3) == 0;
+  const uint32_t red_base = smem_u32(red);
+  const int total = (r1 - r0) * (BN / 4);
+  for (int base = threadIdx.x; base < total; base += THREADS * P) {
+    float4 part[P][S], cc[P];
+    bool live[P];
+#pragma unroll
+    for (int u = 0; u < P; ++u) {
+      const int idx = base + u * THREADS;
+      const int r = r0 + idx / (BN / 4), c = 4 * (idx % (BN / 4));
+      const int64_t m = m0 + r, n = n0 + c;
+      live[u] = idx < total && m < M && n < N;
+      cc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (!live[u]) continue;
+      if constexpr (S == 1) {
+        part[u][0] = *reinterpret_cast<const float4*>(red + r * RS + c);
+      } else {
+        const uint32_t off = red_base + (uint32_t)((r * RS + c) * 4);
+#pragma unroll
+        for (int q = 0; q < S; ++q) part[u][q] = ld_cluster_f4(map_to_rank(off, (uint32_t)q));
+      }
+      if (C && vec && n + 4 <= N) cc[u] = __ldcs(reinterpret_cast<const float4*>(C + m * N + n));
+    }
+#pragma unroll
+    for (int u = 0; u < P; ++u) {
+      if (!live[u]) continue;
+      const int idx = base + u * THREADS;
+      const int r = r0 + idx / (BN / 4), c = 4 * (idx % (BN / 4));
+      const int64_t m = m0 + r, n = n0 + c;
+      float4 v = part[u][0];
+#pragma unroll
+      for (int q = 1; q < S; ++q)  // summed in rank order
+        v = make_float4(__fadd_rn(v.x, part[u][q].x), __fadd_rn(v.y, part[u][q].y), __fadd_rn(v.z, part[u][q].z),
+                        __fadd_rn(v.w, part[u][q].w));
+      float* o = out + m * N + n;
+      if (vec && n + 4 <= N) {
+        if (C)
+          v = make_float4(__fsub_rn(v.x, cc[u].x), __fsub_rn(v.y, cc[u].y), __fsub_rn(v.z, cc[u].z),
+                          __fsub_rn(v.w, cc[u].w));
+        *reinterpret_cast<float4*>(o) = v;
+      } else {
+        const float vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (n + j < N) o[j] = C ? __fsub_rn(vv[j], C[m * N + n + j]) : vv[j];
+      }
+    }
+  }
+}
 
 // One CTA computes a 128 x BN tile of out over the K range of its split (blockIdx.z).
 // The `splits` CTAs of a tile form one thread-block cluster (z dimension); their fp32
@@ -340,6 +414,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     // then wait for that kernel's results and issue the A tiles.
     uint32_t issued_mask = 0u, phase_mask = 0u;  // per stage: a load was issued / its parity
     bool ok = true;
+    const uint64_t pol_w = l2_evict_first(), pol_a = l2_evict_last();
     const int pre = nk < STAGES ? nk : STAGES;
     for (int kb = 0; kb < pre; ++kb) {  // fresh ring: every stage is free
       if (kb == skip_kblock) continue;  // failure-detection test only: this stage never arrives
@@ -347,8 +422,8 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
         const uint32_t st = smem_u32(smem + (size_t)kb * L::STAGE);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
         mbar_expect_tx(full_bar(kb), L::STAGE);
-        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(kb), kx, (int)n0);
-        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(kb), kx, (int)n0);
+        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(kb), kx, (int)n0, pol_w);
+        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(kb), kx, (int)n0, pol_w);
       }
       issued_mask |= 1u << kb;
     }
@@ -358,8 +433,8 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       if (lane == 0) {
         const uint32_t st = smem_u32(smem + (size_t)kb * L::STAGE);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
-        tma_load_2d(st + L::A_HI, &maps.a_hi, full_bar(kb), kx, (int)m0);
-        tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(kb), kx, (int)m0);
+        tma_load_2d(st + L::A_HI, &maps.a_hi, full_bar(kb), kx, (int)m0, pol_a);
+        tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(kb), kx, (int)m0, pol_a);
       }
     }
     __syncwarp();
@@ -373,10 +448,10 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
         const uint32_t st = smem_u32(smem + (size_t)s * L::STAGE);
         const int kx = (int)(kbeg + (int64_t)kb * BK);
         mbar_expect_tx(full_bar(s), L::STAGE);
-        tma_load_2d(st + L::A_HI, &maps.a_hi, full_bar(s), kx, (int)m0);
-        tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(s), kx, (int)m0);
-        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(s), kx, (int)n0);
-        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(s), kx, (int)n0);
+        tma_load_2d(st + L::A_HI, &maps.a_hi, full_bar(s), kx, (int)m0, pol_a);
+        tma_load_2d(st + L::A_LO, &maps.a_lo, full_bar(s), kx, (int)m0, pol_a);
+        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(s), kx, (int)n0, pol_w);
+        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(s), kx, (int)n0, pol_w);
       }
       __syncwarp();
       issued_mask |= 1u << s;
@@ -515,64 +590,18 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     __syncthreads();
   }
   {
-    // Each thread keeps kUnroll float4 positions in flight (remote partials and C loads issued
-    // before any is used), so the epilogue streams instead of waiting one load at a time.
-    constexpr int kUnroll = 4;
     const int rank = splits > 1 ? (int)cluster_rank() : 0;
     const int rows_per_rank = (BM + splits - 1) / splits;
     const int r0 = rank * rows_per_rank, r1 = (r0 + rows_per_rank < BM) ? r0 + rows_per_rank : BM;
-    const bool vec = (N & 3) == 0;
-    const uint32_t red_base = smem_u32(red);
-    const int total = (r1 - r0) * (BN / 4);
-    for (int base = threadIdx.x; base < total; base += THREADS * kUnroll) {
-      float4 acc[kUnroll], cc[kUnroll];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int idx = base + u * THREADS;
-        acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        cc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (idx >= total) continue;
-        const int r = r0 + idx / (BN / 4), c = 4 * (idx % (BN / 4));
-        const int64_t m = m0 + r, n = n0 + c;
-        if (m >= M || n >= N) continue;
-        const uint32_t off = red_base + (uint32_t)((r * RED_STRIDE + c) * 4);
-        if (splits > 1) {
-          float4 part[MAX_CLUSTER];
-#pragma unroll
-          for (int qr = 0; qr < MAX_CLUSTER; ++qr)  // all remote loads in flight at once
-            if (qr < splits) part[qr] = ld_cluster_f4(map_to_rank(off, (uint32_t)qr));
-          acc[u] = part[0];
-#pragma unroll
-          for (int qr = 1; qr < MAX_CLUSTER; ++qr)  // summed in rank order
-            if (qr < splits)
-              acc[u] = make_float4(__fadd_rn(acc[u].x, part[qr].x), __fadd_rn(acc[u].y, part[qr].y),
-                                   __fadd_rn(acc[u].z, part[qr].z), __fadd_rn(acc[u].w, part[qr].w));
-        } else {
-          acc[u] = *reinterpret_cast<const float4*>(red + r * RED_STRIDE + c);
-        }
-        if (C && vec && n + 4 <= N) cc[u] = __ldcs(reinterpret_cast<const float4*>(C + m * N + n));
-      }
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int idx = base + u * THREADS;
-        if (idx >= total) continue;
-        const int r = r0 + idx / (BN / 4), c = 4 * (idx % (BN / 4));
-        const int64_t m = m0 + r, n = n0 + c;
-        if (m >= M || n >= N) continue;
-        float* o = out + m * N + n;
-        if (vec && n + 4 <= N) {
-          float4 v = acc[u];
-          if (C)
-            v = make_float4(__fsub_rn(v.x, cc[u].x), __fsub_rn(v.y, cc[u].y), __fsub_rn(v.z, cc[u].z),
-                            __fsub_rn(v.w, cc[u].w));
-          *reinterpret_cast<float4*>(o) = v;
-        } else {
-          const float v[4] = {acc[u].x, acc[u].y, acc[u].z, acc[u].w};
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            if (n + j < N) o[j] = C ? __fsub_rn(v[j], C[m * N + n + j]) : v[j];
-        }
-      }
+    switch (splits) {
+      case 1: reduce_store<1, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      case 2: reduce_store<2, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      case 3: reduce_store<3, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      case 4: reduce_store<4, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      case 5: reduce_store<5, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      case 6: reduce_store<6, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      case 7: reduce_store<7, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      default: reduce_store<8, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
     }
   }
   __syncwarp();
