@@ -213,6 +213,30 @@ spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const spl_weight*
                                     int64_t M, int64_t K, int64_t N, spl_path path, void* workspace,
                                     size_t workspace_bytes, cudaStream_t stream);
 
+/* ---- binary64 path (Sec. 5.5, the Down projection) ----------------------
+ * The input of Down is masked with noise scaled by the activation bound of Thm. 3,
+ * so large that in binary32 the cancellation error of Eq. fp-log-bound swamps the
+ * output; Sec. 5.5 notes that binary64 (p = 53) resolves it.  These calls do the
+ * whole computation in binary64:
+ *   spl_noise_mask_f64:   Xt = fl64(X + eta), eta drawn exactly as spl_noise
+ *                         (same rng): one binary64 rounding; Xt [rows, cols]
+ *                         binary64, X fp32.
+ *   spl_precompute_noise_product_f64: C[M, N] = Nz W^T, Nz and W fp32, every
+ *                         product exact, binary64 sums; C binary64.
+ *   spl_masked_linear_unmask_f64: Y = fl32(fl64(Xt W^T) - C), Xt and C binary64,
+ *                         W fp32, products rounded once in binary64, binary64 sums.
+ * Bound by the FP64 rate.  Workspace: spl_f64_workspace_bytes(M, K, N) (the
+ * first 64 KiB are left untouched, so the product workspace can be shared).
+ * Errors as spl_masked_linear (all base pointers 16-byte aligned, K % 4 == 0). */
+spl_status spl_noise_mask_f64(double* Xt, const float* X, int64_t rows, int64_t cols, double sensitivity,
+                              double eps, spl_mech mech, spl_rng rng, cudaStream_t stream);
+size_t spl_f64_workspace_bytes(int64_t M, int64_t K, int64_t N);
+spl_status spl_precompute_noise_product_f64(double* C, const float* Nz, const float* W, int64_t M, int64_t K,
+                                            int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+spl_status spl_masked_linear_unmask_f64(float* Y, const double* Xt, const float* W, const double* C, int64_t M,
+                                        int64_t K, int64_t N, void* workspace, size_t workspace_bytes,
+                                        cudaStream_t stream);
+
 /* ---- a5 + a6 for decode, without allocation ---------------------------
  * The paper has no counterpart to this call; it exists for callers that
  * cannot allocate device memory at the time of the product: a decode loop

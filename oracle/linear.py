@@ -30,6 +30,11 @@ def mask(X, N):
     return (_f64(X) + _f64(N)).astype(np.float32)
 
 
+def mask_f64(X, N):
+    """x~ = fl64(x + eta), the mask in binary64 (Sec. 5.5): one rounding of at most 2^-53 |x~|."""
+    return _f64(X) + _f64(N)
+
+
 def matmul_exact(A, W):
     """A W^T in fp64 for fp32 A [M, K] and W [N, K] (the plain definition of the product)."""
     return _f64(A) @ _f64(W).T

@@ -137,6 +137,32 @@ __global__ void rng_advance_kernel(uint64_t* offset_dev, uint64_t delta) {
   *offset_dev += delta;
 }
 
+// Binary64 mask (Sec. 5.5): xt = fl64((double)x + (double)eta) with eta drawn exactly as above:
+// one rounding of at most 2^-53 |xt| (none at all while the exponents of x and eta are within 29).
+template <int MECH>
+__global__ void __launch_bounds__(kThreads) noise_mask_f64_kernel(double* __restrict__ xt, const float* __restrict__ x,
+                                                                  int64_t n, float b, uint32_t k0, uint32_t k1,
+                                                                  uint32_t s0, uint32_t s1, uint64_t offset_host,
+                                                                  const uint64_t* offset_dev) {
+  pdl_wait();
+  pdl_trigger();
+  const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
+  const int64_t nb = (n + 3) >> 2;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
+    const float4 e = draw_block<MECH>((uint64_t)i + offset, k0, k1, s0, s1, b);
+    const float ev[4] = {e.x, e.y, e.z, e.w};
+    if (4 * i + 3 < n) {
+      const float4 xv = __ldcs(reinterpret_cast<const float4*>(x) + i);
+      double2* o = reinterpret_cast<double2*>(xt + 4 * i);
+      __stcs(o, make_double2((double)xv.x + (double)ev[0], (double)xv.y + (double)ev[1]));
+      __stcs(o + 1, make_double2((double)xv.z + (double)ev[2], (double)xv.w + (double)ev[3]));
+    } else {
+      for (int l = 0; l < 4 && 4 * i + l < n; ++l) xt[4 * i + l] = (double)x[4 * i + l] + (double)ev[l];
+    }
+  }
+}
+
 // The raw Philox words of the stream (element e = lane e % 4 of block e / 4 + offset).
 __global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restrict__ out, int64_t n, uint32_t k0,
                                                                uint32_t k1, uint32_t s0, uint32_t s1,
@@ -430,6 +456,29 @@ extern "C" spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, in
   if (!Xt || !X) return SPL_EINVAL;
   if (!aligned16(Xt) || !aligned16(X) || (N_out && !aligned16(N_out))) return SPL_EALIGN;
   return launch_noise_mask(Xt, N_out, X, n, sensitivity, eps, mech, rng, stream);
+}
+
+extern "C" spl_status spl_noise_mask_f64(double* Xt, const float* X, int64_t rows, int64_t cols, double sensitivity,
+                                         double eps, spl_mech mech, spl_rng rng, cudaStream_t stream) {
+  spl_status st = validate_noise(rows, cols, sensitivity, eps, mech);
+  if (st != SPL_OK) return st;
+  const int64_t n = rows * cols;
+  if (n == 0) return SPL_OK;
+  if (!Xt || !X) return SPL_EINVAL;
+  if (!aligned16(Xt) || !aligned16(X)) return SPL_EALIGN;
+  if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
+  const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
+  const int grid = grid_for(ceil_div(n, 4), 8);
+  const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
+  const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
+  if (b == 0.0f)
+    return launch_pdl(noise_mask_f64_kernel<kZero>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, k0, k1, s0, s1,
+                      rng.offset, rng.offset_dev);
+  if (mech == SPL_MECH_LAPLACE)
+    return launch_pdl(noise_mask_f64_kernel<kLaplace>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, k0, k1, s0,
+                      s1, rng.offset, rng.offset_dev);
+  return launch_pdl(noise_mask_f64_kernel<kGaussian>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, k0, k1, s0,
+                    s1, rng.offset, rng.offset_dev);
 }
 
 extern "C" spl_status spl_mask(float* Xt, const float* X, const float* N, int64_t rows, int64_t cols,

@@ -66,6 +66,7 @@ class MaskedLayer:
     paths: dict = field(default_factory=dict)   # per group, from calibrate(); "auto" if not calibrated
     calibration: dict = field(default_factory=dict)
     rng_base: torch.Tensor = None               # [groups] int64 on the device: Philox block offset of the cycle
+    fp64: set = field(default_factory=set)      # groups computed in binary64 (Sec. 5.5; normally {"down"})
 
     @classmethod
     def from_weights(cls, model, weights, split=True, device="cuda"):
@@ -138,6 +139,9 @@ class MaskedLayer:
         for g in self.groups:
             need = max(need, spl.spl_linear_workspace_bytes(M, g.K, g.N, path),
                        spl.spl_precompute_matched_workspace_bytes(draws * M, g.K, g.N, M, path))
+            if g.name in self.fp64:
+                need = max(need, spl.spl_f64_workspace_bytes(M, g.K, g.N),
+                           spl.spl_f64_workspace_bytes(draws * M, g.K, g.N))
         return need
 
     def allocate(self, M, draws, path="auto", workspace=None):
@@ -154,10 +158,11 @@ class MaskedLayer:
         self.rng_base = torch.zeros(len(self.groups), dtype=torch.int64, device=dev)
         self.bank = {}
         for g in self.groups:
+            wide = torch.float64 if g.name in self.fp64 else torch.float32  # binary64 mask and correction
             self.bank[g.name] = {
                 "eta": torch.empty((draws * M, g.K), device=dev),  # transient: the draws being precomputed
-                "C": torch.empty((draws * M, g.N), device=dev),
-                "xt": torch.empty((M, g.K), device=dev),
+                "C": torch.empty((draws * M, g.N), device=dev, dtype=wide),
+                "xt": torch.empty((M, g.K), device=dev, dtype=wide),
                 "Y": torch.empty((M, g.N), device=dev),
             }
 
@@ -186,9 +191,13 @@ class MaskedLayer:
                           offset_dev=off_dev)
             if timer:
                 timer("begin", "precompute", g.name)
-            # summed in the order the online product of M rows uses, so their rounding cancels
-            spl.spl_precompute_noise_product_matched(b["C"], b["eta"], g.wt, self.M, path=self.path_of(g, path, self.M),
-                                                     workspace=self.workspace, stream=stream)
+            if g.name in self.fp64:
+                spl.spl_precompute_noise_product_f64(b["C"], b["eta"], g.W, workspace=self.workspace, stream=stream)
+            else:
+                # summed in the order the online product of M rows uses, so their rounding cancels
+                spl.spl_precompute_noise_product_matched(b["C"], b["eta"], g.wt, self.M,
+                                                         path=self.path_of(g, path, self.M), workspace=self.workspace,
+                                                         stream=stream)
             if timer:
                 timer("end", "precompute", g.name)
 
@@ -202,12 +211,21 @@ class MaskedLayer:
         for gi, g in enumerate(self.groups):
             b = self.bank[g.name]
             off, off_dev = self._offset(gi, g, cycle, d, device_base)
-            spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
-                               offset=off, stream=stream, offset_dev=off_dev)
+            fp64 = g.name in self.fp64
+            if fp64:
+                spl.spl_noise_mask_f64(b["xt"], inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
+                                       offset=off, stream=stream, offset_dev=off_dev)
+            else:
+                spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
+                                   offset=off, stream=stream, offset_dev=off_dev)
             if timer:
                 timer("begin", "masked_linear_unmask", g.name)
-            spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M], path=self.path_of(g, path, M),
-                                         workspace=self.workspace, stream=stream)
+            if fp64:
+                spl.spl_masked_linear_unmask_f64(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M],
+                                                 workspace=self.workspace, stream=stream)
+            else:
+                spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M],
+                                             path=self.path_of(g, path, M), workspace=self.workspace, stream=stream)
             if timer:
                 timer("end", "masked_linear_unmask", g.name)
             out[g.name] = b["Y"]
@@ -241,12 +259,15 @@ class MaskedLayer:
         return graphs, launches
 
     def bound_check(self, inputs, outs, eps, mech, seed, cycle, d):
-        """The paper's bound on the GPU over every output of an online step (per group)."""
+        """The paper's bound on the GPU over every output of an online step (per group).  For a
+        binary64 group the errors are measured the same way against the binary32 bound (its mask
+        is passed rounded to fp32, which moves S_xt by at most 2^-24 relative)."""
         res = {}
         for gi, g in enumerate(self.groups):
             eta = torch.empty((self.M, g.K), device=g.W.device)
             spl.spl_noise(eta, self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=self.block_offset(g, cycle, d))
-            res[g.name] = spl.spl_bound_check(outs[g.name], inputs[g.name], self.bank[g.name]["xt"], eta, g.W)
+            xt = self.bank[g.name]["xt"]
+            res[g.name] = spl.spl_bound_check(outs[g.name], inputs[g.name], xt.float().contiguous(), eta, g.W)
         return res
 
     def flops_per_step(self):

@@ -223,4 +223,48 @@ def qwen_sweep(Ms=(1, 4, 16, 64, 256, 1024), eps=1.0, mech="gaussian", draws=8, 
             "hbm_peak_gbs": pk["hbm_gbs"], "peak_source": pk["source"]}
 
 
-WORKLOADS = {"llama_stack": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep}
+def down_fp64(tokens=(128, 1), eps=1.0, mech="laplace", draws=8, steps=8):
+    """The Down projection of a Llama layer in binary32-family arithmetic (the calibrated path)
+    and in binary64 (Sec. 5.5): time per online product call and the recovered error over every
+    output of one step, against the exact product."""
+    model = wl.LLAMA_3_2_3B
+    out = {}
+    for M in tokens:
+        stack = MaskedStack.build(model, 1, M, draws, base_seed=23)
+        layer = stack.layers[0]
+        inputs = stack.inputs(29)
+        _calibrate(stack, inputs, eps, mech)
+        res = {}
+        for mode in ("binary32", "binary64"):
+            layer.fp64 = {"down"} if mode == "binary64" else set()
+            ws = spl.workspace(layer.workspace_bytes(M, draws))
+            layer.allocate(M, draws, workspace=ws)
+            events = []
+
+            def timer(phase, kind, group):
+                if group != "down" or kind != "masked_linear_unmask":
+                    return
+                e = torch.cuda.Event(enable_timing=True)
+                e.record()
+                events.append(e)
+
+            seed = stack.seeds[0]
+            layer.refill(eps, mech, seed, 0)
+            for d in range(min(steps, draws)):
+                layer.online(inputs[0], eps, mech, seed, 0, d, timer=timer)
+            torch.cuda.synchronize()
+            times = [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
+            outs = layer.online(inputs[0], eps, mech, seed, 0, 0)
+            bc = layer.bound_check(inputs[0], outs, eps, mech, seed, 0, 0)["down"]
+            path = "fp64" if mode == "binary64" else _group_paths(layer, M)["down"]
+            res[mode] = {"path": path, "us_per_call": 1e3 * sum(times[1:]) / max(1, len(times) - 1),
+                         "mean_err": bc["mean_err"], "max_err": bc["max_err"], "max_abs_ref": bc["max_abs_ref"],
+                         "max_err_over_hard_binary32": bc["max_err_over_hard"]}
+        out[f"M={M}"] = res
+        del stack, layer
+        torch.cuda.empty_cache()
+    return {"workload": f"llama-3.2-3b-shaped Down projection (8192 -> 3072) in binary32 and binary64, {mech} "
+                        f"eps={eps}, M in {list(tokens)}", "down": out}
+
+
+WORKLOADS = {"llama_stack": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep, "down_fp64": down_fp64}

@@ -51,6 +51,10 @@ _SIGS = {
     "spl_random_bits": (_I, [_P, _I64, spl_rng, _P]),
     "spl_rng_advance": (_I, [_P, ctypes.c_uint64, _P]),
     "spl_mask": (_I, [_P, _P, _P, _I64, _I64, _P]),
+    "spl_noise_mask_f64": (_I, [_P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
+    "spl_f64_workspace_bytes": (_SZ, [_I64, _I64, _I64]),
+    "spl_precompute_noise_product_f64": (_I, [_P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
+    "spl_masked_linear_unmask_f64": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
     "spl_noise_mask": (_I, [_P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_split_tf32": (_I, [_P, _P, _P, _I64, _P]),
     "spl_split_fp16": (_I, [_P, _P, _P, _P, _I64, _I64, _P]),
@@ -182,6 +186,47 @@ def spl_noise_mask(Xt, N_out, X, sensitivity, eps, mech, seed, stream_id=0, offs
     _check(lib().spl_noise_mask(_dev(Xt, "Xt"), _dev(N_out, "N_out"), _dev(X, "X"), rows, cols, float(sensitivity),
                                 _eps(eps), _mech(mech), _rng(seed, stream_id, offset, offset_dev), _stream(stream)),
            "spl_noise_mask")
+
+
+def spl_noise_mask_f64(Xt, X, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None, offset_dev=None):
+    """Binary64 mask (Sec. 5.5): Xt float64 = X + eta, eta as spl_noise draws it."""
+    rows, cols = _rows_cols(X)
+    if Xt.numel() != rows * cols:
+        raise ValueError("spl_noise_mask_f64: shape mismatch")
+    _check(lib().spl_noise_mask_f64(_dev(Xt, "Xt", torch.float64), _dev(X, "X"), rows, cols, float(sensitivity),
+                                    _eps(eps), _mech(mech), _rng(seed, stream_id, offset, offset_dev),
+                                    _stream(stream)), "spl_noise_mask_f64")
+
+
+def spl_f64_workspace_bytes(M, K, N):
+    return int(lib().spl_f64_workspace_bytes(M, K, N))
+
+
+def spl_precompute_noise_product_f64(C, Nz, W, workspace=None, stream=None):
+    """C float64 [M, N] = Nz W^T in binary64 (Nz, W fp32)."""
+    M, K = _rows_cols(Nz)
+    N = W.shape[0]
+    if W.shape[-1] != K or C.numel() != M * N:
+        raise ValueError("spl_precompute_noise_product_f64: shape mismatch")
+    if workspace is None:
+        workspace = globals()["workspace"](spl_f64_workspace_bytes(M, K, N), Nz.device)
+    wsp, wsb = _ws(workspace)
+    _check(lib().spl_precompute_noise_product_f64(_dev(C, "C", torch.float64), _dev(Nz, "Nz"), _dev(W, "W"), M, K, N,
+                                                  wsp, wsb, _stream(stream)), "spl_precompute_noise_product_f64")
+
+
+def spl_masked_linear_unmask_f64(Y, Xt, W, C, workspace=None, stream=None):
+    """Y fp32 = fl32(Xt W^T - C) with Xt and C float64 (binary64 sums)."""
+    M, K = _rows_cols(Xt)
+    N = W.shape[0]
+    if W.shape[-1] != K or Y.numel() != M * N or C.numel() != M * N:
+        raise ValueError("spl_masked_linear_unmask_f64: shape mismatch")
+    if workspace is None:
+        workspace = globals()["workspace"](spl_f64_workspace_bytes(M, K, N), Xt.device)
+    wsp, wsb = _ws(workspace)
+    _check(lib().spl_masked_linear_unmask_f64(_dev(Y, "Y"), _dev(Xt, "Xt", torch.float64), _dev(W, "W"),
+                                              _dev(C, "C", torch.float64), M, K, N, wsp, wsb, _stream(stream)),
+           "spl_masked_linear_unmask_f64")
 
 
 def spl_split_tf32(hi, lo, src, stream=None):

@@ -89,6 +89,10 @@ def test_argument_validation_without_launch(spl):
     assert L.spl_split_fp16(base, base, base, base, 2, 12, None) == spl.SPL_EALIGN  # cols % 8
     assert L.spl_split_fp16(base, base, None, base, 2, 8, None) == spl.SPL_EINVAL
     assert L.spl_split_fp16(None, None, None, None, 0, 8, None) == spl.SPL_OK
+    assert L.spl_noise_mask_f64(None, None, 4, 4, 1.0, 1.0, 0, rng, None) == spl.SPL_EINVAL
+    assert L.spl_masked_linear_unmask_f64(base, base, base, base, 2, 6, 2, None, 0, None) == spl.SPL_EALIGN
+    assert L.spl_precompute_noise_product_f64(None, base, base, 2, 8, 2, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_precompute_noise_product_f64(None, None, None, 0, 8, 2, None, 0, None) == spl.SPL_OK
     stats = (ctypes.c_double * 27)()
     chosen = ctypes.c_int(5)
     assert L.spl_choose_path(ctypes.byref(chosen), stats, base, base, None, 4, 8, 8, None, 0, None) == spl.SPL_EINVAL

@@ -390,6 +390,76 @@ def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path):
     assert spl.spl_get_device_status() == 0
 
 
+# ------------------------------------------------ binary64 path (Sec. 5.5, the Down projection)
+U53 = 2.0 ** -53
+
+
+def test_noise_mask_f64_matches_oracle(spl):
+    X = dev(wl.activations(37, 1028, seed=61).numpy())
+    eta = torch.empty_like(X)
+    spl.spl_noise(eta, 2.6e8, 1.0, "laplace", seed=62, stream_id=3, offset=17)
+    Xt = torch.empty(X.shape, dtype=torch.float64, device="cuda")
+    spl.spl_noise_mask_f64(Xt, X, 2.6e8, 1.0, "laplace", seed=62, stream_id=3, offset=17)
+    np.testing.assert_array_equal(Xt.cpu().numpy(), linear.mask_f64(f32(X), f32(eta)))
+
+
+@pytest.mark.parametrize("M,K,N", [(1, 256, 64), (3, 1028, 300), (8, 8192, 512), (13, 3072, 700), (128, 3072, 256)])
+def test_f64_products_match_oracle(spl, M, K, N):
+    """C = eta W^T and Y = fl32(X~ W^T - C) in binary64 against the exact products (oracle)."""
+    W = wl.weight(N, K, seed=M + K).numpy()
+    X = wl.activations(M, K, seed=M + 1).numpy()
+    eta = philox.noise((M, K), 2.6e8, 1.0, "gaussian", seed=M + 2)
+    Wd = dev(W)
+    C = torch.empty((M, N), dtype=torch.float64, device="cuda")
+    ws = spl.workspace(spl.spl_f64_workspace_bytes(M, K, N) + 64 * 1024)
+    spl.spl_precompute_noise_product_f64(C, dev(eta), Wd, workspace=ws)
+    Cref = linear.precompute_noise_product(eta, W)
+    S_n = np.abs(eta.astype(np.float64)) @ np.abs(W.astype(np.float64)).T
+    assert np.all(np.abs(C.cpu().numpy() - Cref) <= 2 * bounds.gamma(K, U53) * S_n)
+    Xt = dev(linear.mask_f64(X, eta))
+    Y = torch.empty((M, N), device="cuda")
+    spl.spl_masked_linear_unmask_f64(Y, Xt, Wd, C, workspace=ws)
+    ref = linear.reference_output(X, W)
+    S = linear.abs_products(X, linear.mask_f64(X, eta), eta, W)
+    tol = bounds.hard_bound(*S, K, u=U53) + bounds.gamma(K, U53) * S[0] + 2.0 ** -24 * np.abs(ref) * (1 + 2.0 ** -20)
+    assert np.all(np.abs(f64(Y) - ref) <= tol)
+    assert torch.count_nonzero(ws[: 64 * 1024]).item() == 0  # the decode counters stay untouched
+    assert spl.spl_get_device_status() == 0
+
+
+def test_f64_down_recovers_what_binary32_cannot(spl):
+    """Llama Down shapes, Delta from Thm. 3 (~2.6e8): in binary32 the mask alone rounds away the
+    input; the binary64 path recovers X W^T to a few ulps of fp32."""
+    M, K, N = 4, 8192, 512
+    W = wl.weight(N, K, seed=71).numpy()
+    X = wl.activations(M, K, seed=72).numpy()
+    delta, eps = 2.6e8, 1.0
+    eta = torch.empty((M, K), device="cuda")
+    spl.spl_noise(eta, delta, eps, "laplace", seed=73)
+    Xd, Wd = dev(X), dev(W)
+    ref = linear.reference_output(X, W)
+    # binary64
+    C64 = torch.empty((M, N), dtype=torch.float64, device="cuda")
+    Xt64 = torch.empty((M, K), dtype=torch.float64, device="cuda")
+    spl.spl_precompute_noise_product_f64(C64, eta, Wd)
+    spl.spl_noise_mask_f64(Xt64, Xd, delta, eps, "laplace", seed=73)
+    Y64 = torch.empty((M, N), device="cuda")
+    spl.spl_masked_linear_unmask_f64(Y64, Xt64, Wd, C64)
+    err64 = np.abs(f64(Y64) - ref)
+    assert np.max(err64) <= 4 * 2.0 ** -24 * np.max(np.abs(ref))
+    # binary32, same noise
+    Wt = spl.Weight.prepare(Wd)
+    C32 = torch.empty((M, N), device="cuda")
+    Xt32 = torch.empty((M, K), device="cuda")
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp32"))
+    spl.spl_precompute_noise_product(C32, eta, Wt, path="fp32", workspace=ws)
+    spl.spl_noise_mask(Xt32, None, Xd, delta, eps, "laplace", seed=73)
+    Y32 = torch.empty((M, N), device="cuda")
+    spl.spl_masked_linear_unmask(Y32, Xt32, Wt, C32, path="fp32", workspace=ws)
+    err32 = np.abs(f64(Y32) - ref)
+    assert np.mean(err32) > 1e4 * np.mean(err64)
+
+
 # ---------------------------------------------------------- a8: bound on the GPU, path choice
 def test_bound_check_matches_oracle(spl):
     M, K, N = 24, 1028, 300

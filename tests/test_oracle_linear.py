@@ -83,3 +83,19 @@ def test_max_relative_error_definition():
     Yr = np.array([[1.0, 2.5], [3.0, -4.0]])
     assert linear.max_relative_error(Y, Yr) == pytest.approx(0.5 / 4.0)
     assert linear.max_relative_error(np.zeros((0, 3)), np.zeros((0, 3))) == 0.0
+
+
+def test_binary64_mask_rounds_once():
+    """The binary64 mask of Sec. 5.5 is x + eta rounded once to binary64 (within half an ulp of the
+    exact rational sum), 2^29 times finer than the binary32 mask, which loses x almost entirely
+    when eta is 10^8 times larger."""
+    g = np.random.default_rng(5)
+    x = g.standard_normal(2000).astype(np.float32)
+    eta = (g.standard_normal(2000) * 2.6e8).astype(np.float32)
+    xt = linear.mask_f64(x, eta)
+    assert xt.dtype == np.float64
+    for a, b, s in zip(x[:300], eta[:300], xt[:300]):
+        exact = Fraction(float(a)) + Fraction(float(b))
+        assert abs(Fraction(float(s)) - exact) <= Fraction(np.spacing(abs(float(s)))) / 2
+    assert np.max(np.abs(xt - eta.astype(np.float64) - x)) <= 2.0 ** -53 * np.max(np.abs(xt))
+    assert np.max(np.abs(linear.mask(x, eta).astype(np.float64) - eta.astype(np.float64) - x)) > 1.0
