@@ -49,7 +49,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", default="llama_layer",
-                    choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep", "down_fp64"],
+                    choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep", "down_fp64", "slalom"],
                     help="llama_layer (default): the headline line; the others measure the stack and sweep "
                          "workloads and print their own line")
     return ap.parse_args()
@@ -223,6 +223,10 @@ def run_workload(args):
     elif args.workload == "qwen_stack":
         first = next(iter(res["prefill"].values()))
         value, unit, ms = first["tflops"], UNIT, first["ms_per_prefill"]
+    elif args.workload == "slalom":
+        first = next(iter(res["compare"].values()))["qkv"]
+        value, unit, ms = first["slalom_us"] / first["ours_us"], "slalom time / this path's time (QKV)", \
+            first["ours_us"] / 1e3
     elif args.workload == "down_fp64":
         first = next(iter(res["down"].values()))["binary64"]
         value, unit, ms = first["mean_err"], "mean abs error of the recovered Down output", first["us_per_call"] / 1e3

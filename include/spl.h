@@ -237,6 +237,29 @@ spl_status spl_masked_linear_unmask_f64(float* Y, const double* Xt, const float*
                                         int64_t K, int64_t N, void* workspace, size_t workspace_bytes,
                                         cudaStream_t stream);
 
+/* ---- Slalom comparator (Sec. 6.2) ------------------------------------------
+ * The paper compares its noise masking with Slalom's one-time pad over Z_q,
+ * q = 2^23 + 2^21 + 7, with inputs and weights in fixed point with 8 fractional
+ * bits.  Field elements are integers below 2^24, carried exactly as fp32.
+ *   spl_slalom_quantize: out = rint(v 2^8) (round half to even), fp32 integers;
+ *                        for the weights (done once).
+ *   spl_slalom_mask:     Xt_q = (rint(X 2^8) mod q + eta) mod q; eta uniform in Z_q,
+ *                        element e from Philox block e / 2 + rng.offset, words
+ *                        2 (e % 2), 2 (e % 2) + 1 as lo + 2^32 hi, eta = that mod q;
+ *                        eta_out (may be NULL) receives eta.  rng.offset_dev must
+ *                        be NULL.
+ *   correction:          spl_precompute_noise_product_f64(C, eta, W_q): exact.
+ *   spl_slalom_linear_unmask: Y = ((Xt_q W_q^T - C) mod q, taken in (-q/2, q/2])
+ *                        2^-16, the product exact in binary64 (while every partial
+ *                        sum of |Xt_q| |W_q| stays below 2^53: |W| < 0.5 and
+ *                        K < 2^22, else ESHAPE for K).  Workspace:
+ *                        spl_f64_workspace_bytes(M, K, N). */
+spl_status spl_slalom_quantize(float* out, const float* v, int64_t count, cudaStream_t stream);
+spl_status spl_slalom_mask(float* Xt_q, float* eta_out, const float* X, int64_t rows, int64_t cols, spl_rng rng,
+                           cudaStream_t stream);
+spl_status spl_slalom_linear_unmask(float* Y, const float* Xt_q, const float* W_q, const double* C, int64_t M,
+                                    int64_t K, int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
 /* ---- a5 + a6 for decode, without allocation ---------------------------
  * The paper has no counterpart to this call; it exists for callers that
  * cannot allocate device memory at the time of the product: a decode loop

@@ -163,6 +163,45 @@ __global__ void __launch_bounds__(kThreads) noise_mask_f64_kernel(double* __rest
   }
 }
 
+// Slalom comparator (Sec. 6.2): fixed point with 8 fractional bits, mask uniform in Z_q,
+// q = 2^23 + 2^21 + 7.  Element e draws block e / 2 + offset and takes words 2 (e % 2) and
+// 2 (e % 2) + 1 as the 64-bit integer lo + 2^32 hi; eta = that mod q.  Values below 2^24 are
+// exact in fp32, so the field elements travel as fp32.
+constexpr int64_t kSlalomQ = (1 << 23) + (1 << 21) + 7;
+
+__device__ __forceinline__ float slalom_mask1(float x, uint32_t lo, uint32_t hi, float* eta_out) {
+  const int64_t eta = (int64_t)((((uint64_t)hi << 32) | lo) % (uint64_t)kSlalomQ);
+  const int64_t xq = ((int64_t)llrintf(x * 256.0f) % kSlalomQ + kSlalomQ) % kSlalomQ;
+  if (eta_out) *eta_out = (float)eta;
+  return (float)((xq + eta) % kSlalomQ);
+}
+
+__global__ void __launch_bounds__(kThreads) slalom_mask_kernel(float* __restrict__ xt, float* __restrict__ eta,
+                                                               const float* __restrict__ x, int64_t n, uint32_t k0,
+                                                               uint32_t k1, uint32_t s0, uint32_t s1,
+                                                               uint64_t offset) {
+  pdl_wait();
+  pdl_trigger();
+  const int64_t nb = (n + 1) >> 1;  // two elements per Philox block
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
+    const uint64_t j = (uint64_t)i + offset;
+    const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
+    const int64_t e = 2 * i;
+    xt[e] = slalom_mask1(x[e], r.x, r.y, eta ? eta + e : nullptr);
+    if (e + 1 < n) xt[e + 1] = slalom_mask1(x[e + 1], r.z, r.w, eta ? eta + e + 1 : nullptr);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) slalom_quantize_kernel(float* __restrict__ out,
+                                                                   const float* __restrict__ v, int64_t n) {
+  pdl_wait();
+  pdl_trigger();
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+    out[i] = rintf(v[i] * 256.0f);  // v 2^8 is exact; rint rounds half to even
+}
+
 // The raw Philox words of the stream (element e = lane e % 4 of block e / 4 + offset).
 __global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restrict__ out, int64_t n, uint32_t k0,
                                                                uint32_t k1, uint32_t s0, uint32_t s1,
@@ -479,6 +518,25 @@ extern "C" spl_status spl_noise_mask_f64(double* Xt, const float* X, int64_t row
                       s1, rng.offset, rng.offset_dev);
   return launch_pdl(noise_mask_f64_kernel<kGaussian>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, k0, k1, s0,
                     s1, rng.offset, rng.offset_dev);
+}
+
+extern "C" spl_status spl_slalom_mask(float* Xt, float* eta, const float* X, int64_t rows, int64_t cols, spl_rng rng,
+                                      cudaStream_t stream) {
+  if (rows < 0 || cols < 0) return SPL_EINVAL;
+  const int64_t n = rows * cols;
+  if (n == 0) return SPL_OK;
+  if (!Xt || !X) return SPL_EINVAL;
+  if (rng.offset_dev) return SPL_EINVAL;  // host offsets only
+  const int grid = grid_for(ceil_div(n, 2), 8);
+  return launch_pdl(slalom_mask_kernel, dim3(grid), dim3(kThreads), 0, stream, Xt, eta, X, n, (uint32_t)rng.seed,
+                    (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id, (uint32_t)(rng.stream_id >> 32), rng.offset);
+}
+
+extern "C" spl_status spl_slalom_quantize(float* out, const float* v, int64_t count, cudaStream_t stream) {
+  if (count < 0) return SPL_EINVAL;
+  if (count == 0) return SPL_OK;
+  if (!out || !v) return SPL_EINVAL;
+  return launch_pdl(slalom_quantize_kernel, dim3(grid_for(count, 8)), dim3(kThreads), 0, stream, out, v, count);
 }
 
 extern "C" spl_status spl_mask(float* Xt, const float* X, const float* N, int64_t rows, int64_t cols,

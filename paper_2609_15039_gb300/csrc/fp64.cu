@@ -39,13 +39,35 @@ __device__ __forceinline__ double2 load_a2<double>(const double* p) {
   return __ldg(reinterpret_cast<const double2*>(p));
 }
 
-// part[split][m][n] (splits > 1) or, with one split, the final value: C64 (c == nullptr, out64)
-// or Y = fl32(acc - c) (out32).
+// Final value of an output (one split, or after the split-order reduction):
+//   kOut64  out64 = acc (the correction C, binary64)
+//   kUnmask out32 = fl32(acc - c)
+//   kSlalom out32 = ((acc - c) mod q, taken in (-q/2, q/2]) 2^-16: the Slalom comparator's unmask
+//           and de-quantization (Sec. 6.2); acc and c are exact integers in binary64.
+enum { kOut64 = 0, kUnmask = 1, kSlalom = 2 };
+constexpr double kSlalomQ = 10485767.0;  // 2^23 + 2^21 + 7
+
+__device__ __forceinline__ void finish(double* out64, float* out32, int64_t o, double acc, const double* c, int mode) {
+  if (mode == kOut64) {
+    out64[o] = acc;
+  } else if (mode == kUnmask) {
+    out32[o] = (float)(acc - c[o]);
+  } else {
+    const double t = acc - c[o];  // exact integer, |t| < 2^53
+    double m = t - kSlalomQ * floor(t / kSlalomQ);
+    if (m < 0.0) m += kSlalomQ;
+    if (m >= kSlalomQ) m -= kSlalomQ;
+    if (m > (kSlalomQ - 1.0) * 0.5) m -= kSlalomQ;
+    out32[o] = (float)(m * 0x1p-16);
+  }
+}
+
+// part[split][m][n] (splits > 1) or, with one split, the final value (see finish).
 template <typename TA, int MT>
 __global__ void __launch_bounds__(THREADS) gemv_f64_kernel(double* __restrict__ out64, float* __restrict__ out32,
                                                            const TA* __restrict__ A, const float* __restrict__ W,
                                                            const double* __restrict__ c, int64_t M, int64_t K,
-                                                           int64_t N, int64_t ks, int splits) {
+                                                           int64_t N, int64_t ks, int splits, int mode) {
   extern __shared__ __align__(16) double as[];  // [MT][ks]
   pdl_wait();
   pdl_trigger();
@@ -109,13 +131,10 @@ __global__ void __launch_bounds__(THREADS) gemv_f64_kernel(double* __restrict__ 
       const int64_t row = mbase + m;
       if (row >= M) continue;
       const int64_t o = row * N + n;
-      if (splits > 1) {
+      if (splits > 1)
         out64[(int64_t)split * M * N + o] = acc[r][m];
-      } else if (out32) {
-        out32[o] = (float)(acc[r][m] - c[o]);
-      } else {
-        out64[o] = acc[r][m];
-      }
+      else
+        finish(out64, out32, o, acc[r][m], c, mode);
     }
   }
 }
@@ -123,17 +142,14 @@ __global__ void __launch_bounds__(THREADS) gemv_f64_kernel(double* __restrict__ 
 // Sum of the split partials in split order; then C64 (out64) or Y = fl32(sum - c) (out32).
 __global__ void __launch_bounds__(256) reduce_f64_kernel(double* __restrict__ out64, float* __restrict__ out32,
                                                          const double* __restrict__ part, const double* __restrict__ c,
-                                                         int splits, int64_t total) {
+                                                         int splits, int64_t total, int mode) {
   pdl_wait();
   pdl_trigger();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
     double s = part[i];
     for (int sp = 1; sp < splits; ++sp) s += part[(int64_t)sp * total + i];
-    if (out32)
-      out32[i] = (float)(s - c[i]);
-    else
-      out64[i] = s;
+    finish(out64, out32, i, s, c, mode);
   }
 }
 
@@ -160,26 +176,26 @@ PlanF64 plan_f64(int64_t M, int64_t K, int64_t N) {
 
 template <typename TA, int MT>
 spl_status launch_f64(const PlanF64& p, double* out64, float* out32, const TA* A, const float* W, const double* c,
-                      int64_t M, int64_t K, int64_t N, void* ws, cudaStream_t stream) {
+                      int64_t M, int64_t K, int64_t N, void* ws, cudaStream_t stream, int mode) {
   const dim3 grid((unsigned)ceil_div(N, WARPS * ROWS), (unsigned)p.splits, (unsigned)ceil_div(M, MT));
   if (grid.y > 65535u || grid.z > 65535u) return SPL_ESHAPE;
   const size_t smem = (size_t)MT * p.ks * sizeof(double);
   if (p.splits == 1)
     return launch_pdl(gemv_f64_kernel<TA, MT>, grid, dim3(THREADS), smem, stream, out64, out32, A, W, c, M, K, N, p.ks,
-                      1);
+                      1, mode);
   double* part = reinterpret_cast<double*>(static_cast<char*>(ws) + kCounterBytes);
   spl_status st = launch_pdl(gemv_f64_kernel<TA, MT>, grid, dim3(THREADS), smem, stream, part, (float*)nullptr, A, W,
-                             (const double*)nullptr, M, K, N, p.ks, p.splits);
+                             (const double*)nullptr, M, K, N, p.ks, p.splits, (int)kOut64);
   if (st != SPL_OK) return st;
   const int64_t total = M * N;
   const int rgrid = (int)std::max<int64_t>(1, std::min<int64_t>(ceil_div(total, 256), (int64_t)device_sm_count() * 8));
   return launch_pdl(reduce_f64_kernel, dim3(rgrid), dim3(256), 0, stream, out64, out32, (const double*)part, c,
-                    p.splits, total);
+                    p.splits, total, mode);
 }
 
 template <typename TA>
 spl_status run_f64(double* out64, float* out32, const TA* A, const float* W, const double* c, int64_t M, int64_t K,
-                   int64_t N, void* ws, size_t ws_bytes, cudaStream_t stream) {
+                   int64_t N, void* ws, size_t ws_bytes, cudaStream_t stream, int mode) {
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
   if (M == 0 || N == 0) return SPL_OK;
   if ((!out64 && !out32) || (out32 && !c) || (K > 0 && (!A || !W))) return SPL_EINVAL;
@@ -192,10 +208,10 @@ spl_status run_f64(double* out64, float* out32, const TA* A, const float* W, con
   if (p.ws > 0 && (!ws || ws_bytes < p.ws)) return SPL_EWORKSPACE;
   if (ws && !aligned16(ws)) return SPL_EALIGN;
   switch (p.mt) {
-    case 1: return launch_f64<TA, 1>(p, out64, out32, A, W, c, M, K, N, ws, stream);
-    case 2: return launch_f64<TA, 2>(p, out64, out32, A, W, c, M, K, N, ws, stream);
-    case 4: return launch_f64<TA, 4>(p, out64, out32, A, W, c, M, K, N, ws, stream);
-    default: return launch_f64<TA, 8>(p, out64, out32, A, W, c, M, K, N, ws, stream);
+    case 1: return launch_f64<TA, 1>(p, out64, out32, A, W, c, M, K, N, ws, stream, mode);
+    case 2: return launch_f64<TA, 2>(p, out64, out32, A, W, c, M, K, N, ws, stream, mode);
+    case 4: return launch_f64<TA, 4>(p, out64, out32, A, W, c, M, K, N, ws, stream, mode);
+    default: return launch_f64<TA, 8>(p, out64, out32, A, W, c, M, K, N, ws, stream, mode);
   }
 }
 
@@ -212,11 +228,18 @@ extern "C" size_t spl_f64_workspace_bytes(int64_t M, int64_t K, int64_t N) {
 extern "C" spl_status spl_precompute_noise_product_f64(double* C, const float* Nz, const float* W, int64_t M,
                                                        int64_t K, int64_t N, void* workspace, size_t workspace_bytes,
                                                        cudaStream_t stream) {
-  return run_f64<float>(C, nullptr, Nz, W, nullptr, M, K, N, workspace, workspace_bytes, stream);
+  return run_f64<float>(C, nullptr, Nz, W, nullptr, M, K, N, workspace, workspace_bytes, stream, kOut64);
 }
 
 extern "C" spl_status spl_masked_linear_unmask_f64(float* Y, const double* Xt, const float* W, const double* C,
                                                    int64_t M, int64_t K, int64_t N, void* workspace,
                                                    size_t workspace_bytes, cudaStream_t stream) {
-  return run_f64<double>(nullptr, Y, Xt, W, C, M, K, N, workspace, workspace_bytes, stream);
+  return run_f64<double>(nullptr, Y, Xt, W, C, M, K, N, workspace, workspace_bytes, stream, kUnmask);
+}
+
+extern "C" spl_status spl_slalom_linear_unmask(float* Y, const float* Xt_q, const float* W_q, const double* C,
+                                               int64_t M, int64_t K, int64_t N, void* workspace, size_t workspace_bytes,
+                                               cudaStream_t stream) {
+  if (K >= (int64_t(1) << 22)) return SPL_ESHAPE;  // keeps every integer sum below 2^53
+  return run_f64<float>(nullptr, Y, Xt_q, W_q, C, M, K, N, workspace, workspace_bytes, stream, kSlalom);
 }

@@ -267,4 +267,71 @@ def down_fp64(tokens=(128, 1), eps=1.0, mech="laplace", draws=8, steps=8):
                         f"eps={eps}, M in {list(tokens)}", "down": out}
 
 
-WORKLOADS = {"llama_stack": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep, "down_fp64": down_fp64}
+def slalom_compare(tokens=(128, 1), eps=1.0, mech="gaussian", reps=10):
+    """Slalom's masking (Sec. 6.2: 8-bit fixed point, one-time pad over Z_q, exact integer product,
+    modular unmask) beside this path on the outsourced projections of one Llama layer: time per
+    product call and the error of the recovered output against the exact product."""
+    model = wl.LLAMA_3_2_3B
+    out = {}
+    for M in tokens:
+        stack = MaskedStack.build(model, 1, M, 2, base_seed=31)
+        layer = stack.layers[0]
+        inputs = stack.inputs(37)[0]
+        _calibrate(stack, [inputs], eps, mech)
+        seed = stack.seeds[0]
+        layer.refill(eps, mech, seed, 0)
+        outs = layer.online(inputs, eps, mech, seed, 0, 0)
+        bc = layer.bound_check(inputs, outs, eps, mech, seed, 0, 0)
+        res = {}
+        for gi, g in enumerate(layer.groups):
+            if g.name == "down":
+                continue  # kept in the enclave by both systems (Sec. 5.5)
+            X = inputs[g.name]
+            Wq = torch.empty_like(g.W)
+            spl.spl_slalom_quantize(Wq, g.W)
+            Xt = torch.empty_like(X)
+            eta = torch.empty_like(X)
+            spl.spl_slalom_mask(Xt, eta, X, seed, stream_id=gi)
+            ws = spl.workspace(spl.spl_f64_workspace_bytes(M, g.K, g.N))
+            C = torch.empty((M, g.N), dtype=torch.float64, device=X.device)
+            spl.spl_precompute_noise_product_f64(C, eta, Wq, workspace=ws)
+            Y = torch.empty((M, g.N), device=X.device)
+            call = lambda: spl.spl_slalom_linear_unmask(Y, Xt, Wq, C, workspace=ws)
+            call()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                call()
+            e1.record()
+            torch.cuda.synchronize()
+            slalom_us = 1e3 * e0.elapsed_time(e1) / reps
+            # error of each against the exact product (computed on the device in binary64)
+            ref = X.double() @ g.W.double().T
+            scale = float(ref.abs().max())
+            ours_ev = []
+
+            def timer(phase, kind, group, _g=g.name):
+                if group == _g and kind == "masked_linear_unmask":
+                    e = torch.cuda.Event(enable_timing=True)
+                    e.record()
+                    ours_ev.append(e)
+
+            for d in range(reps + 1):
+                layer.online(inputs, eps, mech, seed, 0, d % 2, timer=timer)
+            torch.cuda.synchronize()
+            ours_us = 1e3 * sum(ours_ev[i].elapsed_time(ours_ev[i + 1]) for i in range(2, len(ours_ev), 2)) / reps
+            res[g.name] = {"slalom_us": slalom_us, "ours_us": ours_us,
+                           "slalom_max_rel_err": float((Y.double() - ref).abs().max()) / scale,
+                           "slalom_mean_abs_err": float((Y.double() - ref).abs().mean()),
+                           "ours_max_rel_err": bc[g.name]["max_err"] / scale, "ours_mean_abs_err": bc[g.name]["mean_err"],
+                           "ours_path": _group_paths(layer, M)[g.name]}
+        out[f"M={M}"] = res
+        del stack, layer
+        torch.cuda.empty_cache()
+    return {"workload": f"llama-3.2-3b-shaped layer, Q|K|V, O, Gate|Up: Slalom's one-time pad over Z_q (8-bit fixed "
+                        f"point) vs this path ({mech} eps={eps}), M in {list(tokens)}", "compare": out}
+
+
+WORKLOADS = {"llama_stack": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep, "down_fp64": down_fp64,
+             "slalom": slalom_compare}

@@ -53,6 +53,9 @@ _SIGS = {
     "spl_mask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_noise_mask_f64": (_I, [_P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_f64_workspace_bytes": (_SZ, [_I64, _I64, _I64]),
+    "spl_slalom_quantize": (_I, [_P, _P, _I64, _P]),
+    "spl_slalom_mask": (_I, [_P, _P, _P, _I64, _I64, spl_rng, _P]),
+    "spl_slalom_linear_unmask": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
     "spl_precompute_noise_product_f64": (_I, [_P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
     "spl_masked_linear_unmask_f64": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
     "spl_noise_mask": (_I, [_P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
@@ -227,6 +230,32 @@ def spl_masked_linear_unmask_f64(Y, Xt, W, C, workspace=None, stream=None):
     _check(lib().spl_masked_linear_unmask_f64(_dev(Y, "Y"), _dev(Xt, "Xt", torch.float64), _dev(W, "W"),
                                               _dev(C, "C", torch.float64), M, K, N, wsp, wsb, _stream(stream)),
            "spl_masked_linear_unmask_f64")
+
+
+def spl_slalom_quantize(out, v, stream=None):
+    """Slalom fixed point (Sec. 6.2): out = rint(v 2^8) as fp32 integers."""
+    _check(lib().spl_slalom_quantize(_dev(out, "out"), _dev(v, "v"), v.numel(), _stream(stream)), "spl_slalom_quantize")
+
+
+def spl_slalom_mask(Xt_q, eta_out, X, seed, stream_id=0, offset=0, stream=None):
+    """Slalom mask: Xt_q = (rint(X 2^8) mod q + eta) mod q, eta uniform in Z_q (fp32 integers)."""
+    rows, cols = _rows_cols(X)
+    _check(lib().spl_slalom_mask(_dev(Xt_q, "Xt_q"), _dev(eta_out, "eta_out"), _dev(X, "X"), rows, cols,
+                                 _rng(seed, stream_id, offset, None), _stream(stream)), "spl_slalom_mask")
+
+
+def spl_slalom_linear_unmask(Y, Xt_q, W_q, C, workspace=None, stream=None):
+    """Y = de-quantized ((Xt_q W_q^T - C) mod q), the product exact in binary64."""
+    M, K = _rows_cols(Xt_q)
+    N = W_q.shape[0]
+    if W_q.shape[-1] != K or Y.numel() != M * N or C.numel() != M * N:
+        raise ValueError("spl_slalom_linear_unmask: shape mismatch")
+    if workspace is None:
+        workspace = globals()["workspace"](spl_f64_workspace_bytes(M, K, N), Xt_q.device)
+    wsp, wsb = _ws(workspace)
+    _check(lib().spl_slalom_linear_unmask(_dev(Y, "Y"), _dev(Xt_q, "Xt_q"), _dev(W_q, "W_q"),
+                                          _dev(C, "C", torch.float64), M, K, N, wsp, wsb, _stream(stream)),
+           "spl_slalom_linear_unmask")
 
 
 def spl_split_tf32(hi, lo, src, stream=None):

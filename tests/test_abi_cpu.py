@@ -93,6 +93,9 @@ def test_argument_validation_without_launch(spl):
     assert L.spl_masked_linear_unmask_f64(base, base, base, base, 2, 6, 2, None, 0, None) == spl.SPL_EALIGN
     assert L.spl_precompute_noise_product_f64(None, base, base, 2, 8, 2, None, 0, None) == spl.SPL_EINVAL
     assert L.spl_precompute_noise_product_f64(None, None, None, 0, 8, 2, None, 0, None) == spl.SPL_OK
+    assert L.spl_slalom_quantize(None, None, -1, None) == spl.SPL_EINVAL
+    assert L.spl_slalom_mask(None, None, None, 0, 3, rng, None) == spl.SPL_OK
+    assert L.spl_slalom_linear_unmask(base, base, base, base, 1, 1 << 22, 1, None, 0, None) == spl.SPL_ESHAPE
     stats = (ctypes.c_double * 27)()
     chosen = ctypes.c_int(5)
     assert L.spl_choose_path(ctypes.byref(chosen), stats, base, base, None, 4, 8, 8, None, 0, None) == spl.SPL_EINVAL

@@ -12,7 +12,7 @@ import numpy as np
 import pytest
 import torch
 
-from oracle import bounds, linear, philox, stats
+from oracle import bounds, linear, philox, slalom, stats
 from paper_2609_15039_gb300 import workloads as wl
 from _util import U, assert_product_close, f32, f64, ulp32
 
@@ -458,6 +458,31 @@ def test_f64_down_recovers_what_binary32_cannot(spl):
     spl.spl_masked_linear_unmask(Y32, Xt32, Wt, C32, path="fp32", workspace=ws)
     err32 = np.abs(f64(Y32) - ref)
     assert np.mean(err32) > 1e4 * np.mean(err64)
+
+
+# ------------------------------------------------ Slalom comparator (Sec. 6.2)
+@pytest.mark.parametrize("M,K,N", [(1, 256, 64), (5, 1028, 300), (16, 3072, 512), (128, 8192, 256)])
+def test_slalom_matches_oracle_bitwise(spl, M, K, N):
+    """Integer work end to end: quantized weights, the masked field elements, the exact
+    correction and the de-quantized result all equal the oracle's bit for bit."""
+    W = wl.weight(N, K, seed=K + 5).numpy()
+    X = wl.activations(M, K, seed=M + 6).numpy()
+    Wq = torch.empty((N, K), device="cuda")
+    spl.spl_slalom_quantize(Wq, dev(W))
+    np.testing.assert_array_equal(f64(Wq), slalom.quantize(W).astype(np.float64))
+    Xt = torch.empty((M, K), device="cuda")
+    eta = torch.empty((M, K), device="cuda")
+    spl.spl_slalom_mask(Xt, eta, dev(X), seed=77, stream_id=2, offset=5)
+    eta_or = slalom.mask_noise((M, K), seed=77, stream_id=2, offset=5)
+    np.testing.assert_array_equal(f64(eta), eta_or.astype(np.float64))
+    np.testing.assert_array_equal(f64(Xt), slalom.mask(X, eta_or).astype(np.float64))
+    ws = spl.workspace(spl.spl_f64_workspace_bytes(M, K, N) + 64 * 1024)
+    C = torch.empty((M, N), dtype=torch.float64, device="cuda")
+    spl.spl_precompute_noise_product_f64(C, eta, Wq, workspace=ws)
+    np.testing.assert_array_equal(C.cpu().numpy(), slalom.product(eta_or, slalom.quantize(W)).astype(np.float64))
+    Y = torch.empty((M, N), device="cuda")
+    spl.spl_slalom_linear_unmask(Y, Xt, Wq, C, workspace=ws)
+    np.testing.assert_array_equal(f64(Y), slalom.masked_linear(X, W, eta_or))
 
 
 # ---------------------------------------------------------- a8: bound on the GPU, path choice
