@@ -350,7 +350,7 @@ spl_status spl_test_tc_wait_timeout(float* out, const float* A, const spl_weight
 
 /* Test hook (the paper has no counterpart): Y = Xt W^T (- C if C is not NULL)
  * on the tcgen05 kernel with a fixed launch variant -- tile width tile_n and a
- * stage ring of ring_kb KB: (256, 192), (128, 192) or (128, 96) -- and every
+ * stage ring of ring_kb KB: (256, 192), (128, 224) or (128, 96) -- and every
  * tile's K range split `splits` ways (1..8) across a thread-block cluster,
  * instead of the shape the library would choose.  path is SPL_PATH_TF32X3 or
  * SPL_PATH_FP16X3.  Same operands, workspace and errors as

@@ -90,7 +90,7 @@ struct Fp16x3 {
 template <class Md, int BN, int RK>
 struct Cfg {
   static_assert(BN == 128 || BN == 256, "tile width");
-  static_assert(RK == 96 || RK == 192, "ring size");
+  static_assert(RK == 96 || RK == 192 || RK == 224, "ring size");
   static constexpr uint32_t A_HALF = BM * Md::BK * Md::ESZ, B_HALF = BN * Md::BK * Md::ESZ;
   static constexpr uint32_t A_HI = 0, A_LO = A_HALF, W_HI = 2 * A_HALF, W_LO = W_HI + B_HALF;
   static constexpr uint32_t STAGE = W_LO + B_HALF;  // bytes TMA brings per stage
@@ -103,6 +103,7 @@ struct Cfg {
   static_assert(A_LO % 1024 == 0 && W_HI % 1024 == 0 && W_LO % 1024 == 0 && STAGE % 1024 == 0,
                 "swizzle atoms aligned");
   static_assert(STAGES >= 3 && STAGES <= 8, "ring depth");
+  static_assert(SMEM <= 232448, "227 KB of dynamic shared memory per block");
   static_assert((size_t)BM * RED_STRIDE * 4 <= RING, "staging fits in the stage ring");
   static_assert(8 * (2 * STAGES + 3) + 16 <= 1024 && 1024 + 4 * BN <= AUX_BYTES, "aux fits");
 };
@@ -675,7 +676,7 @@ struct Variant {
   double F, b;
 };
 constexpr int kVariants = 3;
-constexpr Variant kVariant[kVariants] = {{256, 192, 1, 450.0, 1.0}, {128, 192, 1, 300.0, 0.667},
+constexpr Variant kVariant[kVariants] = {{256, 192, 1, 450.0, 1.0}, {128, 224, 1, 300.0, 0.667},
                                          {128, 96, 2, 300.0, 1.333}};
 
 // Co-resident clusters of s CTAs of variant v on the current device; clusters must fit inside
@@ -709,7 +710,7 @@ int max_active_clusters(int v, int s, int sms) {
   int& c = cache[dev][v][s];
   if (c == 0) {
     const int n = v == 0 ? query_active_clusters<256, 192>(s)
-                         : (v == 1 ? query_active_clusters<128, 192>(s) : query_active_clusters<128, 96>(s));
+                         : (v == 1 ? query_active_clusters<128, 224>(s) : query_active_clusters<128, 96>(s));
     c = n > 0 ? n : std::max(1, sms * kVariant[v].cps / s);
   }
   return c;
@@ -830,7 +831,7 @@ spl_status launch_variant(const LinearArgs& a, const uint16_t* hi, const uint16_
                           const TcShape& shape, int skip_kblock, int seg_splits) {
   switch (shape.v) {
     case 0: return launch_tc<Md, 256, 192>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
-    case 1: return launch_tc<Md, 128, 192>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    case 1: return launch_tc<Md, 128, 224>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
     default: return launch_tc<Md, 128, 96>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
   }
 }

@@ -231,7 +231,7 @@ def test_products_match_oracle(spl, M, K, N, path):
 
 
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
-@pytest.mark.parametrize("tile_n,ring_kb", [(256, 192), (128, 192), (128, 96)])
+@pytest.mark.parametrize("tile_n,ring_kb", [(256, 192), (128, 224), (128, 96)])
 @pytest.mark.parametrize("splits", [1, 3, 8])
 def test_tc_every_launch_shape(spl, path, tile_n, ring_kb, splits):
     """Each kernel instance (encoding x tile width x ring) with each cluster K-split, on a ragged
