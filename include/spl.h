@@ -133,6 +133,16 @@ spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, int64_t rows,
                           double sensitivity, double eps, spl_mech mech, spl_rng rng,
                           cudaStream_t stream);
 
+/* ---- a2 + a3 fused with the fp16 split of X~ ----------------------------
+ * Draws eta exactly as spl_noise, forms Xt = fl32(X + eta) (written to Xt
+ * unless it is NULL) and writes its FP16X3 split as spl_split_fp16 would:
+ * hi, lo [rows, cols] binary16 and row_exp [rows].  One pass, one block per
+ * row; cols % 8 == 0 and cols <= 16384 (EALIGN / ESHAPE otherwise).  The split
+ * is what spl_masked_linear_unmask_split consumes.  Errors as spl_noise_mask. */
+spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,
+                                int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech,
+                                spl_rng rng, cudaStream_t stream);
+
 /* ---- weight preparation for TF32X3 ------------------------------------
  * hi = src rounded to TF32 (10 explicit mantissa bits, ties away), lo = src - hi
  * (exact in fp32).  Done once per weight; hi and lo are [count] like src. */
@@ -259,6 +269,17 @@ spl_status spl_slalom_mask(float* Xt_q, float* eta_out, const float* X, int64_t 
                            cudaStream_t stream);
 spl_status spl_slalom_linear_unmask(float* Y, const float* Xt_q, const float* W_q, const double* C, int64_t M,
                                     int64_t K, int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* ---- a5 + a6 with the left operand already split ---------------------------
+ * As spl_masked_linear_unmask, with X~ given as a descriptor: Xt->w the fp32
+ * X~ (may be NULL when the call runs FP16X3) and Xt->f16_hi / f16_lo / f16_exp
+ * its fp16 split (from spl_noise_mask_split or spl_split_fp16).  On the FP16X3
+ * path the product reads the split and skips its own split pass (no workspace
+ * needed); other paths read Xt->w (EINVAL if it is NULL).  The result equals
+ * spl_masked_linear_unmask's bit for bit. */
+spl_status spl_masked_linear_unmask_split(float* Y, const spl_weight* Xt, const spl_weight* W, const float* C,
+                                          int64_t M, int64_t K, int64_t N, spl_path path, void* workspace,
+                                          size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- a5 + a6 for decode, without allocation ---------------------------
  * The paper has no counterpart to this call; it exists for callers that

@@ -77,6 +77,9 @@ struct LinearArgs {
   size_t ws_bytes;
   cudaStream_t stream;
   spl_path path;            // resolved arithmetic path
+  const uint16_t* a_h16;    // [M, K]  fp16 split of a, made by the caller (FP16X3), or null
+  const uint16_t* a_l16;
+  const int32_t* a_exp;     // [M]
 };
 
 // Workspace layout shared by every product call: the first kCounterBytes hold

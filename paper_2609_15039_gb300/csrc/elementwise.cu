@@ -328,11 +328,19 @@ __global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restri
 
 // The same split with the row held in registers: one block per row, CH chunks of 8 entries per
 // thread, all loads issued before any is used, so a row costs one memory round trip.
-template <int CH>
+// MECH >= 0: the row is first masked (a2 + a3 fused into the split): xt = fl32(x + eta) with eta
+// drawn exactly as noise_mask_kernel draws it (element e: lane e % 4 of Philox block e / 4 +
+// offset), written to xt_out when it is not NULL, then split.
+constexpr int kNoMask = -1;
+
+template <int CH, int MECH>
 __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __restrict__ hi,
                                                                    uint16_t* __restrict__ lo,
                                                                    int* __restrict__ row_exp,
-                                                                   const float* __restrict__ src, int64_t cols) {
+                                                                   const float* __restrict__ src, int64_t cols,
+                                                                   float* __restrict__ xt_out, float b, uint32_t k0,
+                                                                   uint32_t k1, uint32_t s0, uint32_t s1,
+                                                                   uint64_t offset_host, const uint64_t* offset_dev) {
   pdl_wait();
   pdl_trigger();
   __shared__ float warp_max[kThreads / 32];
@@ -348,6 +356,23 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
       v[2 * c + 1] = __ldg(row + 2 * i + 1);
     } else {
       v[2 * c] = v[2 * c + 1] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  if constexpr (MECH != kNoMask) {
+    const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
+    const uint64_t j0 = (uint64_t)((r * cols) >> 2) + offset;  // cols % 8 == 0: rows start on a block
+#pragma unroll
+    for (int c = 0; c < CH; ++c) {
+      const int64_t i = threadIdx.x + (int64_t)c * kThreads;
+      if (i >= n8) break;
+      const uint64_t j = j0 + 2 * (uint64_t)i;
+      v[2 * c] = add4(v[2 * c], draw_block<MECH>(j, k0, k1, s0, s1, b));
+      v[2 * c + 1] = add4(v[2 * c + 1], draw_block<MECH>(j + 1, k0, k1, s0, s1, b));
+      if (xt_out) {
+        float4* o = reinterpret_cast<float4*>(xt_out + r * cols);
+        __stcs(o + 2 * i, v[2 * c]);
+        __stcs(o + 2 * i + 1, v[2 * c + 1]);
+      }
     }
   }
   float m = 0.f;
@@ -369,8 +394,8 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
   for (int c = 0; c < CH; ++c) {
     const int64_t i = threadIdx.x + (int64_t)c * kThreads;
     if (i >= n8) break;
-    const float4 a = v[2 * c], b = v[2 * c + 1];
-    const float xs[8] = {a.x * sc, a.y * sc, a.z * sc, a.w * sc, b.x * sc, b.y * sc, b.z * sc, b.w * sc};
+    const float4 a = v[2 * c], bb = v[2 * c + 1];
+    const float xs[8] = {a.x * sc, a.y * sc, a.z * sc, a.w * sc, bb.x * sc, bb.y * sc, bb.z * sc, bb.w * sc};
     __align__(16) __half h[8];
     __align__(16) __half l[8];
 #pragma unroll
@@ -418,22 +443,36 @@ spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, 
 
 }  // namespace
 
+// Row split with an optional fused mask (mech < 0: none).  Rows whose register copy does not fit
+// (more than 16384 entries) and no mask take the two-pass kernel.
+template <int MECH>
+spl_status launch_split_rows(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows,
+                             int64_t cols, float* xt_out, float b, const spl_rng& rng, cudaStream_t stream) {
+  const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
+  const dim3 grid((unsigned)rows), block(kThreads);
+  const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
+  const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
+  if (per_thread <= 1)
+    return launch_pdl(split_fp16_regs_kernel<1, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
+                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+  if (per_thread <= 2)
+    return launch_pdl(split_fp16_regs_kernel<2, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
+                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+  if (per_thread <= 4)
+    return launch_pdl(split_fp16_regs_kernel<4, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
+                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+  if (per_thread <= 8)
+    return launch_pdl(split_fp16_regs_kernel<8, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
+                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+  if (MECH != kNoMask) return SPL_ESHAPE;
+  return launch_pdl(split_fp16_kernel, grid, block, 0, stream, hi, lo, row_exp, src, cols);
+}
+
 spl_status run_split_fp16(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows, int64_t cols,
                           cudaStream_t stream) {
   if (rows == 0) return SPL_OK;
   if (rows > 0x7fffffffLL) return SPL_ESHAPE;
-  const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
-  if (per_thread <= 1) {
-    return launch_pdl(split_fp16_regs_kernel<1>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
-  } else if (per_thread <= 2) {
-    return launch_pdl(split_fp16_regs_kernel<2>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
-  } else if (per_thread <= 4) {
-    return launch_pdl(split_fp16_regs_kernel<4>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
-  } else if (per_thread <= 8) {
-    return launch_pdl(split_fp16_regs_kernel<8>, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
-  } else {
-    return launch_pdl(split_fp16_kernel, dim3((unsigned)rows), dim3(kThreads), 0, stream, hi, lo, row_exp, src, cols);
-  }
+  return launch_split_rows<kNoMask>(hi, lo, row_exp, src, rows, cols, nullptr, 0.f, spl_rng{}, stream);
 }
 
 spl_status run_split_tf32(float* hi, float* lo, const float* src, int64_t count, cudaStream_t stream) {
@@ -537,6 +576,23 @@ extern "C" spl_status spl_slalom_quantize(float* out, const float* v, int64_t co
   if (count == 0) return SPL_OK;
   if (!out || !v) return SPL_EINVAL;
   return launch_pdl(slalom_quantize_kernel, dim3(grid_for(count, 8)), dim3(kThreads), 0, stream, out, v, count);
+}
+
+extern "C" spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,
+                                           int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech,
+                                           spl_rng rng, cudaStream_t stream) {
+  spl_status st = validate_noise(rows, cols, sensitivity, eps, mech);
+  if (st != SPL_OK) return st;
+  if (rows == 0 || cols == 0) return SPL_OK;
+  if (!X || !hi || !lo || !row_exp) return SPL_EINVAL;
+  if ((cols & 7) != 0) return SPL_EALIGN;
+  if (!aligned16(X) || !aligned16(hi) || !aligned16(lo) || (Xt && !aligned16(Xt))) return SPL_EALIGN;
+  if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
+  if (rows > 0x7fffffffLL) return SPL_ESHAPE;
+  const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
+  if (b == 0.0f) return launch_split_rows<kZero>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
+  if (mech == SPL_MECH_LAPLACE) return launch_split_rows<kLaplace>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
+  return launch_split_rows<kGaussian>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
 }
 
 extern "C" spl_status spl_mask(float* Xt, const float* X, const float* N, int64_t rows, int64_t cols,

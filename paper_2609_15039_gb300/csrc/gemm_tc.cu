@@ -850,25 +850,42 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int f
     if (!a.w_hi || !a.w_lo) return SPL_EUNSUPPORTED;
     if (!aligned16(a.w_hi) || !aligned16(a.w_lo)) return SPL_EALIGN;
   }
-  if (!a.ws || a.ws_bytes < kCounterBytes + tc_asplit_bytes(a.M, a.K, a.path)) return SPL_EWORKSPACE;
-  if (!aligned16(a.ws)) return SPL_EALIGN;
+  const bool presplit = f16 && a.a_h16 && a.a_l16 && a.a_exp;  // the caller passed the split of A
+  if (presplit) {
+    if (!aligned16(a.a_h16) || !aligned16(a.a_l16)) return SPL_EALIGN;
+  } else {
+    if (!a.ws || a.ws_bytes < kCounterBytes + tc_asplit_bytes(a.M, a.K, a.path)) return SPL_EWORKSPACE;
+    if (!aligned16(a.ws)) return SPL_EALIGN;
+  }
   if (a.M > 0x7fffffffLL || a.N > 0x7fffffffLL || a.K > 0x7fffffffLL) return SPL_ESHAPE;
   if (ceil_div(a.M, BM) * ceil_div(a.N, 128) > 0x7fffffffLL || forced_splits > MAX_CLUSTER) return SPL_ESHAPE;
   if (forced_v >= kVariants) return SPL_EINVAL;
-  // split A into the workspace: [counters][FP16X3: row exponents][hi][lo]
-  char* base = static_cast<char*>(a.ws) + kCounterBytes;
-  const int64_t esz = f16 ? 2 : 4;
-  int* a_exp = nullptr;
-  if (f16) {
-    a_exp = reinterpret_cast<int*>(base);
-    base += round_up(a.M * 4, 256);
+  // split A into the workspace: [counters][FP16X3: row exponents][hi][lo] (unless passed in)
+  const int* a_exp = nullptr;
+  const void* a_hi = nullptr;
+  const void* a_lo = nullptr;
+  if (presplit) {
+    a_exp = a.a_exp;
+    a_hi = a.a_h16;
+    a_lo = a.a_l16;
+  } else {
+    char* base = static_cast<char*>(a.ws) + kCounterBytes;
+    const int64_t esz = f16 ? 2 : 4;
+    int* exps = nullptr;
+    if (f16) {
+      exps = reinterpret_cast<int*>(base);
+      base += round_up(a.M * 4, 256);
+    }
+    void* hi_ = base;
+    void* lo_ = base + round_up(a.M * a.K * esz, 256);
+    const spl_status st =
+        f16 ? run_split_fp16(static_cast<uint16_t*>(hi_), static_cast<uint16_t*>(lo_), exps, a.a, a.M, a.K, a.stream)
+            : run_split_tf32(static_cast<float*>(hi_), static_cast<float*>(lo_), a.a, a.M * a.K, a.stream);
+    if (st != SPL_OK) return st;
+    a_exp = exps;
+    a_hi = hi_;
+    a_lo = lo_;
   }
-  void* a_hi = base;
-  void* a_lo = base + round_up(a.M * a.K * esz, 256);
-  const spl_status st =
-      f16 ? run_split_fp16(static_cast<uint16_t*>(a_hi), static_cast<uint16_t*>(a_lo), a_exp, a.a, a.M, a.K, a.stream)
-          : run_split_tf32(static_cast<float*>(a_hi), static_cast<float*>(a_lo), a.a, a.M * a.K, a.stream);
-  if (st != SPL_OK) return st;
   TcShape shape;
   if (forced_v >= 0) {
     shape = TcShape{forced_v, 0, ceil_div(a.M, BM) * ceil_div(a.N, kVariant[forced_v].bn), forced_splits, 0.0};

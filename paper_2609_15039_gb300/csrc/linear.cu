@@ -65,7 +65,8 @@ spl_status check_weight(const spl_weight* W, int64_t K) {
 }
 
 spl_status run_linear(float* out, const float* a, const spl_weight* W, const float* C, bool need_c, int64_t M,
-                      int64_t K, int64_t N, spl_path path, void* ws, size_t ws_bytes, cudaStream_t stream) {
+                      int64_t K, int64_t N, spl_path path, void* ws, size_t ws_bytes, cudaStream_t stream,
+                      const spl_weight* A = nullptr) {
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
   if (!valid_path(path)) return SPL_EINVAL;
   if (M == 0 || N == 0) return SPL_OK;
@@ -73,7 +74,9 @@ spl_status run_linear(float* out, const float* a, const spl_weight* W, const flo
   if ((K & 3) != 0) return SPL_EALIGN;
   spl_status st = check_weight(W, K);
   if (st != SPL_OK) return st;
-  if (K > 0 && !a) return SPL_EINVAL;
+  // a pre-split left operand (FP16X3): its fp32 values may be absent when that path runs
+  const bool a_split = A && A->f16_hi && A->f16_lo && A->f16_exp;
+  if (K > 0 && !a && !a_split) return SPL_EINVAL;
   if (!aligned16(out) || (a && !aligned16(a)) || (C && !aligned16(C))) return SPL_EALIGN;
   if (M > (int64_t(1) << 31) || N > (int64_t(1) << 31) || K > (int64_t(1) << 31)) return SPL_ESHAPE;
   if (K == 0) {  // empty reduction: the product is zero
@@ -84,10 +87,17 @@ spl_status run_linear(float* out, const float* a, const spl_weight* W, const flo
   if (resolved == SPL_PATH_TF32X3 && (!has_tf32(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
   if (resolved == SPL_PATH_FP16X3 && (!has_f16(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
   if (resolved == SPL_PATH_FP16X3 && (K & 7) != 0) return SPL_EALIGN;
+  if (!a && resolved != SPL_PATH_FP16X3) return SPL_EINVAL;  // only FP16X3 reads the split alone
+  const bool use_split = a_split && resolved == SPL_PATH_FP16X3;
   const Plan plan = make_plan(M, K, N, resolved);
-  if (plan.total() > 0 && (!ws || ws_bytes < plan.total())) return SPL_EWORKSPACE;
+  if (!use_split && plan.total() > 0 && (!ws || ws_bytes < plan.total())) return SPL_EWORKSPACE;
   if (ws && !aligned16(ws)) return SPL_EALIGN;
-  const LinearArgs args = make_args(out, a, *W, C, M, K, N, ws, ws_bytes, stream, resolved);
+  LinearArgs args = make_args(out, a, *W, C, M, K, N, ws, ws_bytes, stream, resolved);
+  if (use_split) {
+    args.a_h16 = A->f16_hi;
+    args.a_l16 = A->f16_lo;
+    args.a_exp = A->f16_exp;
+  }
   switch (plan.kernel) {
     case kKernelTc: return run_tc(args, plan);
     case kKernelGemv: return run_gemv(args, plan);
@@ -175,6 +185,13 @@ extern "C" spl_status spl_masked_linear_unmask(float* Y, const float* Xt, const 
                                                int64_t M, int64_t K, int64_t N, spl_path path, void* workspace,
                                                size_t workspace_bytes, cudaStream_t stream) {
   return run_linear(Y, Xt, W, C, true, M, K, N, path, workspace, workspace_bytes, stream);
+}
+
+extern "C" spl_status spl_masked_linear_unmask_split(float* Y, const spl_weight* Xt, const spl_weight* W,
+                                                     const float* C, int64_t M, int64_t K, int64_t N, spl_path path,
+                                                     void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  if (!Xt) return SPL_EINVAL;
+  return run_linear(Y, Xt->w, W, C, true, M, K, N, path, workspace, workspace_bytes, stream, Xt);
 }
 
 extern "C" size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows,

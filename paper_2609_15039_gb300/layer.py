@@ -165,6 +165,18 @@ class MaskedLayer:
                 "xt": torch.empty((M, g.K), device=dev, dtype=wide),
                 "Y": torch.empty((M, g.N), device=dev),
             }
+            if self._fused_split(g, path, M):  # X~ with its fp16 split, written by the mask kernel
+                b = self.bank[g.name]
+                b["xs"] = spl.Weight(b["xt"], f16_hi=torch.empty((M, g.K), dtype=torch.int16, device=dev),
+                                     f16_lo=torch.empty((M, g.K), dtype=torch.int16, device=dev),
+                                     f16_exp=torch.empty(M, dtype=torch.int32, device=dev))
+
+    def _fused_split(self, g, path, M):
+        """True when the online product of group g runs FP16X3: then the mask kernel also writes the
+        fp16 split of X~ and the product skips its own split pass."""
+        if g.name in self.fp64 or g.wt is None or g.wt.f16_hi is None or g.K % 8 or g.K > 16384:
+            return False
+        return spl.spl_resolve_path(M, g.K, g.N, self.path_of(g, path, M)) == spl.SPL_PATH_FP16X3
 
     def block_offset(self, g, cycle, d):
         """First Philox block of draw d of bank cycle ``cycle`` for group g."""
@@ -212,9 +224,13 @@ class MaskedLayer:
             b = self.bank[g.name]
             off, off_dev = self._offset(gi, g, cycle, d, device_base)
             fp64 = g.name in self.fp64
+            xs = b.get("xs") if self._fused_split(g, path, M) else None
             if fp64:
                 spl.spl_noise_mask_f64(b["xt"], inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
                                        offset=off, stream=stream, offset_dev=off_dev)
+            elif xs is not None:
+                spl.spl_noise_mask_split(b["xt"], xs.f16_hi, xs.f16_lo, xs.f16_exp, inputs[g.name], self.deltas[g.name],
+                                         eps, mech, seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
             else:
                 spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
                                    offset=off, stream=stream, offset_dev=off_dev)
@@ -223,6 +239,10 @@ class MaskedLayer:
             if fp64:
                 spl.spl_masked_linear_unmask_f64(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M],
                                                  workspace=self.workspace, stream=stream)
+            elif xs is not None:
+                spl.spl_masked_linear_unmask_split(b["Y"], xs, g.wt, b["C"][d * M:(d + 1) * M],
+                                                   path=self.path_of(g, path, M), workspace=self.workspace,
+                                                   stream=stream)
             else:
                 spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M],
                                              path=self.path_of(g, path, M), workspace=self.workspace, stream=stream)

@@ -60,6 +60,8 @@ _SIGS = {
     "spl_masked_linear_unmask_f64": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P, _SZ, _P]),
     "spl_noise_mask": (_I, [_P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_split_tf32": (_I, [_P, _P, _P, _I64, _P]),
+    "spl_noise_mask_split": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
+    "spl_masked_linear_unmask_split": (_I, [_P, _PW, _PW, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_split_fp16": (_I, [_P, _P, _P, _P, _I64, _I64, _P]),
     "spl_resolve_path": (_I, [_I64, _I64, _I64, _I]),
     "spl_linear_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I]),
@@ -232,6 +234,33 @@ def spl_masked_linear_unmask_f64(Y, Xt, W, C, workspace=None, stream=None):
            "spl_masked_linear_unmask_f64")
 
 
+def spl_noise_mask_split(Xt, hi, lo, row_exp, X, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None,
+                         offset_dev=None):
+    """a2 + a3 + the fp16 split of X~ in one pass (Xt may be None)."""
+    rows, cols = _rows_cols(X)
+    if hi.numel() != rows * cols or lo.numel() != rows * cols or row_exp.numel() != rows:
+        raise ValueError("spl_noise_mask_split: shape mismatch")
+    _check(lib().spl_noise_mask_split(_dev(Xt, "Xt"), _dev(hi, "hi", torch.int16), _dev(lo, "lo", torch.int16),
+                                      _dev(row_exp, "row_exp", torch.int32), _dev(X, "X"), rows, cols,
+                                      float(sensitivity), _eps(eps), _mech(mech),
+                                      _rng(seed, stream_id, offset, offset_dev), _stream(stream)),
+           "spl_noise_mask_split")
+
+
+def spl_masked_linear_unmask_split(Y, Xt, W, C, path="auto", workspace=None, stream=None):
+    """Xt: a Weight holding X~ (w, may be None on FP16X3) and its fp16 split; W: a Weight."""
+    W = _weight(W)
+    M, K = Xt.shape
+    N = W.shape[0]
+    if W.shape[-1] != K or Y.numel() != M * N or C.numel() != M * N:
+        raise ValueError("spl_masked_linear_unmask_split: shape mismatch")
+    wsp, wsb = _ws(workspace)
+    xs, ws_ = Xt.c_struct(), W.c_struct()
+    _check(lib().spl_masked_linear_unmask_split(_dev(Y, "Y"), ctypes.byref(xs), ctypes.byref(ws_), _dev(C, "C"), M, K,
+                                                N, _path(path), wsp, wsb, _stream(stream)),
+           "spl_masked_linear_unmask_split")
+
+
 def spl_slalom_quantize(out, v, stream=None):
     """Slalom fixed point (Sec. 6.2): out = rint(v 2^8) as fp32 integers."""
     _check(lib().spl_slalom_quantize(_dev(out, "out"), _dev(v, "v"), v.numel(), _stream(stream)), "spl_slalom_quantize")
@@ -299,7 +328,7 @@ class Weight:
 
     @property
     def shape(self):
-        return self.w.shape
+        return self.w.shape if self.w is not None else self.f16_hi.shape
 
     def rows(self, a, b):
         """Rows a:b (output columns a:b of the product) as a Weight of views."""

@@ -390,6 +390,48 @@ def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path):
     assert spl.spl_get_device_status() == 0
 
 
+# ------------------------------------------------ a2 + a3 fused with the split of X~
+@pytest.mark.parametrize("rows,cols,mech,eps", [(5, 8, "laplace", 1.0), (130, 3072, "gaussian", 0.5),
+                                                (3, 16384, "laplace", 2.0), (17, 1032, "gaussian", None)])
+def test_noise_mask_split_equals_separate_calls(spl, rows, cols, mech, eps):
+    X = dev(wl.activations(rows, cols, seed=rows + cols).numpy())
+    base = torch.tensor([3000], dtype=torch.int64, device="cuda")
+    xt_ref = torch.empty_like(X)
+    spl.spl_noise_mask(xt_ref, None, X, 825.3, eps, mech, seed=19, stream_id=2, offset=3000 + 40)
+    hi_ref = torch.empty(X.shape, dtype=torch.int16, device="cuda")
+    lo_ref, ex_ref = torch.empty_like(hi_ref), torch.empty(rows, dtype=torch.int32, device="cuda")
+    spl.spl_split_fp16(hi_ref, lo_ref, ex_ref, xt_ref)
+    xt = torch.empty_like(X)
+    hi, lo, ex = torch.empty_like(hi_ref), torch.empty_like(lo_ref), torch.empty_like(ex_ref)
+    spl.spl_noise_mask_split(xt, hi, lo, ex, X, 825.3, eps, mech, seed=19, stream_id=2, offset=40, offset_dev=base)
+    assert torch.equal(xt, xt_ref) and torch.equal(hi, hi_ref) and torch.equal(lo, lo_ref) and torch.equal(ex, ex_ref)
+    spl.spl_noise_mask_split(None, hi, lo, ex, X, 825.3, eps, mech, seed=19, stream_id=2, offset=3040)  # no X~ out
+    assert torch.equal(hi, hi_ref) and torch.equal(ex, ex_ref)
+
+
+@pytest.mark.parametrize("M,K,N", [(128, 3072, 3072), (130, 1032, 600), (512, 3072, 5120), (9, 256, 512)])
+def test_presplit_product_equals_plain(spl, M, K, N):
+    W, Wt = _weights(spl, N, K, seed=N + 3)
+    X = dev(wl.activations(M, K, seed=M + 4).numpy())
+    C = dev(wl.activations(M, N, seed=5).numpy())
+    xt = torch.empty_like(X)
+    hi = torch.empty(X.shape, dtype=torch.int16, device="cuda")
+    lo, ex = torch.empty_like(hi), torch.empty(M, dtype=torch.int32, device="cuda")
+    spl.spl_noise_mask_split(xt, hi, lo, ex, X, 825.3, 1.0, "gaussian", seed=7)
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N))
+    Y_plain, Y_split, Y_none = (torch.empty((M, N), device="cuda") for _ in range(3))
+    spl.spl_masked_linear_unmask(Y_plain, xt, Wt, C, path="fp16x3", workspace=ws)
+    spl.spl_masked_linear_unmask_split(Y_split, spl.Weight(xt, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, C,
+                                       path="fp16x3", workspace=ws)
+    spl.spl_masked_linear_unmask_split(Y_none, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, C,
+                                       path="fp16x3", workspace=None)
+    assert torch.equal(Y_plain, Y_split) and torch.equal(Y_plain, Y_none)
+    with pytest.raises(spl.SplError) as e:  # FP32 reads the fp32 X~, which is absent
+        spl.spl_masked_linear_unmask_split(Y_none, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, C,
+                                           path="fp32", workspace=ws)
+    assert e.value.status == spl.SPL_EINVAL
+
+
 # ------------------------------------------------ binary64 path (Sec. 5.5, the Down projection)
 U53 = 2.0 ** -53
 
