@@ -7,14 +7,23 @@
 // K-slice of X~ in shared memory, and fuses the unmask r - W eta (Eq.
 // add-and-then-subtract) into the final write.
 //
-// Work unit: a 256-thread block owns 32 (M <= 4) or 16 consecutive rows of W
-// over one K-slice; lanes stride the slice in float4 steps and every lane
-// keeps 4 x M partial dot products in registers, reduced across the warp
-// with shuffles at the end.  The K-split is a multiple of 128 elements and
-// is sized so the grid fills the SMs.  With more than one split, each block
-// writes fp32 partials to the workspace and bumps an arrival counter; the
-// last block of a row group sums the partials in split order (deterministic),
-// subtracts C, writes the result and resets the counter to zero.
+// Work unit: a 256-thread block owns RB consecutive rows of W over one
+// K-slice.  Each quarter-warp (8 lanes) reads one row at a time, 32 floats
+// (one 128-byte line) per step, so a warp-wide load covers four rows and a
+// shared-memory read of X~ is one 128-byte line broadcast to the four
+// quarters.  A lane holds RQ rows (rows q, q+4, ... of its warp's 4 RQ) x MT
+// partial dot products; at the end each quarter-warp sums its 8 lanes with a
+// reduce-scatter butterfly (V - 1 shuffles for V = RQ MT values, not 3 V).
+// Every output element is summed in one order whatever MT and RQ are: the
+// lane's own k positions in increasing order, then the fixed xor-4/2/1 tree
+// over the 8 lanes, then the K-slices in split order; so a correction
+// computed with a different number of rows per launch cancels exactly.
+//
+// The K-split is a multiple of 128 elements and is sized so the grid fills the
+// SMs.  With more than one split, each block writes fp32 partials to the
+// workspace and bumps an arrival counter; the last block of a row group sums
+// the partials in split order (deterministic), subtracts C, writes the result
+// and resets the counter to zero.
 
 #include <algorithm>
 #include <mutex>
@@ -25,107 +34,161 @@ namespace spl {
 namespace {
 
 constexpr int THREADS = 256, WARPS = 8;
-constexpr int SMEM_FLOATS = 12000;  // just under 48 KB of X~ slice (static smem adds a few bytes)
+constexpr int kStep = 32;                    // K elements a quarter-warp covers per step
+constexpr int kSliceAlign = 128;             // K-slices are multiples of this
+constexpr int kXsBytes = 96 * 1024;          // largest X~ slice a block stages (two blocks per SM)
+constexpr int kMaxKs = kXsBytes / (4 * kGemvMaxM) / kSliceAlign * kSliceAlign;  // 1536: every MT fits it
 
-// Rows of W per warp: 4 for M <= 4, 2 for larger M (bounds the rows x M accumulators and keeps
-// four blocks resident per SM).
-constexpr int rows_per_warp(int mt) { return mt >= 8 ? 2 : 4; }
+// Rows per lane: 4 while the accumulators are few (MT <= 2), else 2 (RQ x MT accumulators).
+__host__ __device__ constexpr int rows_per_lane(int mt) { return mt <= 2 ? 4 : 2; }
+__host__ __device__ constexpr int rows_per_block(int mt) { return WARPS * 4 * rows_per_lane(mt); }
+// Steps of 32 per unrolled iteration: 8 float4 loads of W in flight per lane per buffer.
+__host__ __device__ constexpr int unroll_steps(int mt) { return 8 / rows_per_lane(mt); }
 
-template <int MT, int ROWS_PER_WARP>
+// Reduce-scatter over the 8 lanes of a quarter-warp (xor offsets 4, 2, 1).  While C >= 2 values
+// remain, the lane with bit O set keeps the upper half and sends the lower half; afterwards the
+// single value left is summed with a plain xor exchange.  Each step adds (own, partner), so every
+// element gets the same tree whatever C is.
+template <int C, int O, int V>
+__device__ __forceinline__ void quarter_reduce(float (&v)[V], int lane) {
+  if constexpr (O >= 1) {
+    if constexpr (C >= 2) {
+      const bool up = (lane & O) != 0;
+#pragma unroll
+      for (int i = 0; i < C / 2; ++i) {
+        const float send = up ? v[i] : v[i + C / 2];
+        const float keep = up ? v[i + C / 2] : v[i];
+        v[i] = __fadd_rn(keep, __shfl_xor_sync(0xffffffffu, send, O));
+      }
+      quarter_reduce<C / 2, O / 2, V>(v, lane);
+    } else {
+      v[0] = __fadd_rn(v[0], __shfl_xor_sync(0xffffffffu, v[0], O));
+      quarter_reduce<1, O / 2, V>(v, lane);
+    }
+  }
+}
+
+// Index (in the lane's original V values) of the first value the lane holds after quarter_reduce,
+// and the mask of lane bits whose partners hold the same values.
+template <int V>
+__device__ __forceinline__ int reduced_base(int lane, int* dup_mask) {
+  int base = 0, c = V, dup = 0;
+#pragma unroll
+  for (int o = 4; o >= 1; o >>= 1) {
+    if (c >= 2) {
+      if (lane & o) base += c / 2;
+      c /= 2;
+    } else {
+      dup |= o;
+    }
+  }
+  *dup_mask = dup;
+  return base;
+}
+
+template <int MT>
 __global__ void __launch_bounds__(THREADS)
 gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* __restrict__ W,
             const float* __restrict__ C, float* __restrict__ part, unsigned int* __restrict__ counters, int M,
-            int64_t K, int64_t N, int64_t ks, int splits, int64_t prefetch_bytes) {
-  constexpr int ROWS_PER_BLOCK = WARPS * ROWS_PER_WARP;
-  extern __shared__ __align__(16) float xs[];  // [MT][ks]
+            int64_t K, int64_t N, int ks, int splits, int prefetch_lines) {
+  constexpr int RQ = rows_per_lane(MT), RB = rows_per_block(MT), U = unroll_steps(MT);
+  constexpr int V = RQ * MT;
+  extern __shared__ __align__(16) float4 xs[];  // [MT][ks / 4]
   __shared__ int s_last;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int quarter = lane >> 3, kl = (lane & 7) * 4;
   const int split = blockIdx.y;
   const int64_t k0 = (int64_t)split * ks;
-  const int64_t klen = std::min<int64_t>(ks, K - k0);  // multiple of 4
+  const int klen = (int)(K - k0 < ks ? K - k0 : (int64_t)ks);  // multiple of 4
+  const int64_t row0 = (int64_t)blockIdx.x * RB + warp * 4 * RQ + quarter;  // lane's rows: row0 + 4 r
 
-  // the first prefetch_bytes of each of this warp's W rows (slice k0..k0+klen) into L2
-  {
-    const int64_t n_first = (int64_t)blockIdx.x * ROWS_PER_BLOCK + warp * ROWS_PER_WARP;
-    const int64_t lines = std::min<int64_t>(prefetch_bytes, klen * 4) >> 7;  // 128-byte lines per row
-    for (int r = 0; r < ROWS_PER_WARP; ++r) {
-      if (n_first + r >= N) break;
-      const char* base = reinterpret_cast<const char*>(W + (n_first + r) * K + k0);
-      for (int64_t l = lane; l < lines; l += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(base + 128 * l));
-    }
+  const float* wp[RQ];
+  bool valid[RQ];
+#pragma unroll
+  for (int r = 0; r < RQ; ++r) {
+    valid[r] = row0 + 4 * r < N;
+    wp[r] = W + (valid[r] ? row0 + 4 * r : 0) * K + k0 + kl;
   }
+
+  // W never changes, so its first lines are fetched before waiting on the kernel that writes X~
+  // and C: the first U steps into registers, the next prefetch_lines lines of each row into L2.
+  float4 w[U][RQ];
+#pragma unroll
+  for (int u = 0; u < U; ++u)
+#pragma unroll
+    for (int r = 0; r < RQ; ++r)
+      w[u][r] = (valid[r] && u * kStep + kl < klen) ? __ldcs(reinterpret_cast<const float4*>(wp[r] + u * kStep))
+                                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int l = U + (lane & 7); l < prefetch_lines && l * kStep < klen; l += 8)
+#pragma unroll
+    for (int r = 0; r < RQ; ++r)
+      if (valid[r]) asm volatile("prefetch.global.L2 [%0];" ::"l"(wp[r] - kl + l * kStep));
   pdl_wait();
 
-  // stage X~[:, k0:k0+klen] (rows >= M are zero)
-  const int64_t q_per_row = klen >> 2;
-  for (int64_t q = threadIdx.x; q < (int64_t)MT * q_per_row; q += THREADS) {
-    const int m = (int)(q / q_per_row);
-    const int64_t kq = (q - (int64_t)m * q_per_row) * 4;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (m < M) v = __ldg(reinterpret_cast<const float4*>(X + (int64_t)m * K + k0 + kq));
-    *reinterpret_cast<float4*>(xs + (int64_t)m * ks + kq) = v;
+  // stage X~[:, k0:k0+ks] (rows >= M and columns >= klen are zero)
+  const int q_row = ks >> 2, q_len = klen >> 2;
+#pragma unroll
+  for (int m = 0; m < MT; ++m) {
+    const float4* src = reinterpret_cast<const float4*>(X + (int64_t)m * K + k0);
+    for (int q = threadIdx.x; q < q_row; q += THREADS)
+      xs[m * q_row + q] = (m < M && q < q_len) ? __ldg(src + q) : make_float4(0.f, 0.f, 0.f, 0.f);
   }
   __syncthreads();
 
-  const int64_t nbase = (int64_t)blockIdx.x * ROWS_PER_BLOCK + warp * ROWS_PER_WARP;
-  const float* wrow[ROWS_PER_WARP];
-  bool valid[ROWS_PER_WARP];
+  float acc[V];
 #pragma unroll
-  for (int r = 0; r < ROWS_PER_WARP; ++r) {
-    valid[r] = nbase + r < N;
-    wrow[r] = W + (valid[r] ? (nbase + r) : 0) * K + k0;
-  }
+  for (int i = 0; i < V; ++i) acc[i] = 0.f;
 
-  float acc[ROWS_PER_WARP][MT];
+  const float4* xl = xs + (kl >> 2);
+  for (int kb = 0; kb < klen; kb += U * kStep) {
+    // the next U steps of W while this one is summed
+    float4 wn[U][RQ];
+    const int kn = kb + U * kStep;
 #pragma unroll
-  for (int r = 0; r < ROWS_PER_WARP; ++r)
+    for (int u = 0; u < U; ++u)
 #pragma unroll
-    for (int m = 0; m < MT; ++m) acc[r][m] = 0.f;
-
-#pragma unroll 2
-  for (int64_t kk = lane * 4; kk < klen; kk += 128) {
-    float4 wv[ROWS_PER_WARP];
+      for (int r = 0; r < RQ; ++r)
+        wn[u][r] = (valid[r] && kn + u * kStep + kl < klen)
+                       ? __ldcs(reinterpret_cast<const float4*>(wp[r] + kn + u * kStep))
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int r = 0; r < ROWS_PER_WARP; ++r)
-      wv[r] = valid[r] ? __ldcs(reinterpret_cast<const float4*>(wrow[r] + kk)) : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int u = 0; u < U; ++u)
 #pragma unroll
-    for (int m = 0; m < MT; ++m) {
-      const float4 xv = *reinterpret_cast<const float4*>(xs + (int64_t)m * ks + kk);
+      for (int m = 0; m < MT; ++m) {
+        const float4 x = xl[m * q_row + ((kb + u * kStep) >> 2)];
 #pragma unroll
-      for (int r = 0; r < ROWS_PER_WARP; ++r) {
-        float a = acc[r][m];
-        a = fmaf(wv[r].x, xv.x, a);
-        a = fmaf(wv[r].y, xv.y, a);
-        a = fmaf(wv[r].z, xv.z, a);
-        a = fmaf(wv[r].w, xv.w, a);
-        acc[r][m] = a;
+        for (int r = 0; r < RQ; ++r) {
+          float a = acc[r * MT + m];
+          a = fmaf(w[u][r].x, x.x, a);
+          a = fmaf(w[u][r].y, x.y, a);
+          a = fmaf(w[u][r].z, x.z, a);
+          a = fmaf(w[u][r].w, x.w, a);
+          acc[r * MT + m] = a;
+        }
       }
-    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+#pragma unroll
+      for (int r = 0; r < RQ; ++r) w[u][r] = wn[u][r];
   }
 
   pdl_trigger();  // W is streamed: the next kernel may be scheduled
 
-  // warp reduction: lane 0 ends with the full sums
-#pragma unroll
-  for (int r = 0; r < ROWS_PER_WARP; ++r)
-#pragma unroll
-    for (int m = 0; m < MT; ++m) {
-      float v = acc[r][m];
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
-      acc[r][m] = v;
-    }
+  quarter_reduce<V, 4, V>(acc, lane);
+  int dup = 0;
+  const int base = reduced_base<V>(lane, &dup);
+  constexpr int HELD = V >= 8 ? V / 8 : 1;
+  const bool writer = (lane & dup) == 0;
 
   if (splits == 1) {
-    if (lane == 0) {
+    if (writer) {
 #pragma unroll
-      for (int r = 0; r < ROWS_PER_WARP; ++r) {
-        if (!valid[r]) continue;
-#pragma unroll
-        for (int m = 0; m < MT; ++m) {
-          if (m >= M) break;
-          const int64_t o = (int64_t)m * N + nbase + r;
-          out[o] = C ? __fsub_rn(acc[r][m], C[o]) : acc[r][m];
+      for (int i = 0; i < HELD; ++i) {
+        const int idx = base + i, r = idx / MT, m = idx - r * MT;
+        const int64_t n = row0 + 4 * r;
+        if (m < M && n < N) {
+          const int64_t o = (int64_t)m * N + n;
+          out[o] = C ? __fsub_rn(acc[i], C[o]) : acc[i];
         }
       }
     }
@@ -133,15 +196,12 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
   }
 
   float* mypart = part + (int64_t)split * M * N;
-  if (lane == 0) {
+  if (writer) {
 #pragma unroll
-    for (int r = 0; r < ROWS_PER_WARP; ++r) {
-      if (!valid[r]) continue;
-#pragma unroll
-      for (int m = 0; m < MT; ++m) {
-        if (m >= M) break;
-        __stcg(mypart + (int64_t)m * N + nbase + r, acc[r][m]);
-      }
+    for (int i = 0; i < HELD; ++i) {
+      const int idx = base + i, r = idx / MT, m = idx - r * MT;
+      const int64_t n = row0 + 4 * r;
+      if (m < M && n < N) __stcg(mypart + (int64_t)m * N + n, acc[i]);
     }
   }
   __threadfence();
@@ -153,10 +213,10 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  const int64_t n0 = (int64_t)blockIdx.x * ROWS_PER_BLOCK;
-  for (int idx = threadIdx.x; idx < ROWS_PER_BLOCK * M; idx += THREADS) {
-    const int m = idx / ROWS_PER_BLOCK;
-    const int64_t n = n0 + (idx % ROWS_PER_BLOCK);
+  const int64_t n0 = (int64_t)blockIdx.x * RB;
+  for (int idx = threadIdx.x; idx < RB * M; idx += THREADS) {
+    const int m = idx / RB;
+    const int64_t n = n0 + (idx - m * RB);
     if (n >= N) continue;
     const int64_t o = (int64_t)m * N + n;
     float s = __ldcg(part + o);
@@ -169,38 +229,64 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 int padded_m(int64_t M) { return M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : M <= 8 ? 8 : 16; }
 
 template <int MT>
+void* kernel_ptr() { return reinterpret_cast<void*>(gemv_kernel<MT>); }
+
+void* kernel_for(int mt) {
+  switch (mt) {
+    case 1: return kernel_ptr<1>();
+    case 2: return kernel_ptr<2>();
+    case 4: return kernel_ptr<4>();
+    case 8: return kernel_ptr<8>();
+    default: return kernel_ptr<16>();
+  }
+}
+
+// Opt every instantiation into the shared memory of the largest X~ slice (once per device).
+bool smem_attr_set() {
+  static std::mutex mu;
+  static bool done[64] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev]) {
+    for (int mt : {1, 2, 4, 8, 16})
+      if (cudaFuncSetAttribute(kernel_for(mt), cudaFuncAttributeMaxDynamicSharedMemorySize, kXsBytes) !=
+          cudaSuccess) {
+        cudaGetLastError();
+        return false;
+      }
+    done[dev] = true;
+  }
+  return true;
+}
+
+template <int MT>
 spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int* counters) {
-  constexpr int R = rows_per_warp(MT);
-  dim3 grid((unsigned)ceil_div(a.N, WARPS * R), (unsigned)p.splits);
+  if (!smem_attr_set()) return SPL_ECUDA;
+  dim3 grid((unsigned)ceil_div(a.N, rows_per_block(MT)), (unsigned)p.splits);
   const size_t smem = (size_t)MT * p.k_per_split * sizeof(float);
-  // L2 budget of the early prefetch: about 32 MB over the whole grid
-  const int64_t rows = (int64_t)grid.x * WARPS * R * p.splits;
-  const int64_t prefetch = std::max<int64_t>(0, (int64_t(32) << 20) / std::max<int64_t>(rows, 1));
-  return launch_pdl(gemv_kernel<MT, R>, grid, dim3(THREADS), smem, a.stream, a.out, a.a, a.w, a.c, part, counters,
-                    (int)a.M, a.K, a.N, p.k_per_split, p.splits, prefetch);
+  // L2 budget of the early prefetch: about 32 MB over the whole grid, in 128-byte lines per row
+  const int64_t rows = (int64_t)grid.x * rows_per_block(MT) * p.splits;
+  const int lines = (int)std::min<int64_t>(p.k_per_split / kStep, ((int64_t(32) << 20) / std::max<int64_t>(rows, 1)) >> 7);
+  return launch_pdl(gemv_kernel<MT>, grid, dim3(THREADS), smem, a.stream, a.out, a.a, a.w, a.c, part, counters,
+                    (int)a.M, a.K, a.N, (int)p.k_per_split, p.splits, lines);
 }
 
 // Resident blocks per SM of the decode kernel for MT rows and a K-slice of ks (cached).
 int blocks_per_sm(int mt, int64_t ks) {
   static std::mutex mu;
-  static int cache[64][5][128] = {{{0}}};  // device, log2(mt), ks / 128 (ks <= 12000 / mt)
+  static int cache[64][5][kMaxKs / kSliceAlign + 1] = {{{0}}};  // device, log2(mt), ks / 128
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (!smem_attr_set()) return 1;
   const int mi = mt == 1 ? 0 : mt == 2 ? 1 : mt == 4 ? 2 : mt == 8 ? 3 : 4;
-  const int ki = (int)std::min<int64_t>(127, ks / 128);
+  const int ki = (int)std::min<int64_t>(kMaxKs / kSliceAlign, ks / kSliceAlign);
   std::lock_guard<std::mutex> lock(mu);
   int& v = cache[dev][mi][ki];
   if (v == 0) {
-    const size_t smem = (size_t)mt * ks * sizeof(float);
     int n = 0;
-    cudaError_t e = cudaErrorInvalidValue;
-    switch (mt) {
-      case 1: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<1, rows_per_warp(1)>, THREADS, smem); break;
-      case 2: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<2, rows_per_warp(2)>, THREADS, smem); break;
-      case 4: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<4, rows_per_warp(4)>, THREADS, smem); break;
-      case 8: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<8, rows_per_warp(8)>, THREADS, smem); break;
-      default: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<16, rows_per_warp(16)>, THREADS, smem);
-    }
+    const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel_for(mt), THREADS,
+                                                                         (size_t)mt * ks * sizeof(float));
     if (e != cudaSuccess) cudaGetLastError();
     v = (e == cudaSuccess && n > 0) ? n : 1;
   }
@@ -209,25 +295,28 @@ int blocks_per_sm(int mt, int64_t ks) {
 
 }  // namespace
 
-int64_t gemv_max_ks(int64_t M) { return (SMEM_FLOATS / padded_m(M)) / 128 * 128; }
+int64_t gemv_max_ks(int64_t M) {
+  return std::min<int64_t>(kMaxKs, (int64_t)kXsBytes / (4 * padded_m(M)) / kSliceAlign * kSliceAlign);
+}
 
 // K-split of the decode kernel: the number of splits s minimises waves(s) x (K/s + F), waves
-// counting the resident block slots of all SMs, with K/s a multiple of 128 that fits the shared-
-// memory slice and at least 256; F (the fixed cost of a block -- staging X~, the warp reduction,
-// the split-K reduction -- in units of K) measured on GB300.
+// counting the resident block slots of all SMs, with K/s a multiple of 128 no larger than 1536
+// (the slice 16 rows can stage, so a correction of up to 16 rows per launch reproduces the
+// online order); F (the fixed cost of a block -- staging X~, the warp reduction, the split-K
+// reduction -- in units of K) measured on GB300.
 constexpr double kGemvFixedK = 512.0;
 
 Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
   Plan p{};
   p.kernel = kKernelGemv;
   const int mt = padded_m(M);
-  const int64_t ks_max = (SMEM_FLOATS / mt) / 128 * 128;
-  const int64_t groups = ceil_div(N, WARPS * rows_per_warp(mt));
+  const int64_t ks_max = kMaxKs;
+  const int64_t groups = ceil_div(N, rows_per_block(mt));
   const int64_t s_min = ceil_div(K, ks_max);
   const int64_t s_max = std::max<int64_t>(s_min, std::min<int64_t>(64, K / 256));
   double best = 1e300;
   for (int64_t s = s_min; s <= s_max; ++s) {
-    const int64_t ks = std::min<int64_t>(round_up(ceil_div(K, s), 128), ks_max);
+    const int64_t ks = std::min<int64_t>(round_up(ceil_div(K, s), kSliceAlign), ks_max);
     const int64_t splits = ceil_div(K, ks);
     const int64_t slots = (int64_t)sms * blocks_per_sm(mt, ks);
     const double cost = (double)ceil_div(groups * splits, slots) * ((double)ks + kGemvFixedK);
@@ -246,7 +335,7 @@ spl_status run_gemv(const LinearArgs& a, const Plan& p) {
   float* part = nullptr;
   unsigned int* counters = nullptr;
   if (p.splits > 1) {
-    if (ceil_div(a.N, WARPS * rows_per_warp(padded_m(a.M))) > kMaxCounters) return SPL_ESHAPE;
+    if (ceil_div(a.N, rows_per_block(padded_m(a.M))) > kMaxCounters) return SPL_ESHAPE;
     counters = static_cast<unsigned int*>(a.ws);
     part = reinterpret_cast<float*>(static_cast<char*>(a.ws) + kCounterBytes);
   }
@@ -316,7 +405,7 @@ extern "C" spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt
   }
   const Plan plan = plan_gemv(M, K, N, device_sm_count());
   if (plan.ws_partials > kStaticPartialBytes) return SPL_EWORKSPACE;  // beyond the built-in 4 MiB
-  if (plan.splits > 1 && ceil_div(N, WARPS * rows_per_warp(padded_m(M))) > kMaxCounters) return SPL_EWORKSPACE;
+  if (plan.splits > 1 && ceil_div(N, rows_per_block(padded_m(M))) > kMaxCounters) return SPL_EWORKSPACE;
   void* ws = nullptr;
   spl_status st = static_scratch(&ws);
   if (st != SPL_OK) return st;

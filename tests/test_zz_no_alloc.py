@@ -62,8 +62,9 @@ def test_noalloc_rejects_what_it_cannot_hold(spl):
         spl.spl_masked_linear_unmask_noalloc(torch.empty((17, 8), device="cuda"), X, W, torch.zeros((17, 8),
                                                                                                   device="cuda"))
     assert e.value.status == spl.SPL_ESHAPE  # only the decode kernel (M <= 16) has this variant
-    # 16 tokens x 1024 outputs x 103 K-splits of partials (6.75 MB) is more than the 4 MiB array holds
-    N, K = 1024, 65536
+    # K = 65536 takes at least 43 K-slices (a slice holds at most 1536 columns), so 16 tokens x 4096
+    # outputs of partials per slice (11.3 MB and more) is more than the 4 MiB array holds
+    N, K = 4096, 65536
     W = torch.zeros((N, K), device="cuda")
     X = torch.zeros((16, K), device="cuda")
     with pytest.raises(spl.SplError) as e:
