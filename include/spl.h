@@ -281,6 +281,22 @@ spl_status spl_masked_linear_unmask_split(float* Y, const spl_weight* Xt, const 
                                           int64_t M, int64_t K, int64_t N, spl_path path, void* workspace,
                                           size_t workspace_bytes, cudaStream_t stream);
 
+/* ---- a2 + a3 + a5 + a6 in one call ------------------------------------------
+ * Y = fl32(fl32(Xt W^T) - C) with Xt = fl32(X + eta) (Sec. 3.3.1, Eq.
+ * add-and-then-subtract): the noise is drawn exactly as spl_noise_mask draws it
+ * with the same arguments (rows = M, cols = K, rng), Xt [M, K] is written, and Y
+ * equals spl_noise_mask followed by spl_masked_linear_unmask bit for bit.  For
+ * 1 <= M <= 4 rows on the FP32 path (AUTO resolves to it there) one launch of the
+ * decode kernel does all of it: every block draws the noise of its own K-slice
+ * while staging X~, so no separate mask kernel sits between two products; other
+ * calls run the two steps.  Xt and X must not overlap (EINVAL).  Workspace and errors as
+ * spl_masked_linear_unmask, plus spl_noise_mask's checks on sensitivity, eps,
+ * mech and rng; on an error after the mask ran, Xt may have been written. */
+spl_status spl_noise_mask_linear_unmask(float* Y, float* Xt, const float* X, const spl_weight* W, const float* C,
+                                        int64_t M, int64_t K, int64_t N, double sensitivity, double eps,
+                                        spl_mech mech, spl_rng rng, spl_path path, void* workspace,
+                                        size_t workspace_bytes, cudaStream_t stream);
+
 /* ---- a5 + a6 for decode, without allocation ---------------------------
  * The paper has no counterpart to this call; it exists for callers that
  * cannot allocate device memory at the time of the product: a decode loop

@@ -138,6 +138,21 @@ Plan plan_simt(int64_t M, int64_t K, int64_t N, int sms);
 Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path);
 
 spl_status run_gemv(const LinearArgs& a, const Plan& p);
+// The decode product with the mask fused into its staging of X~ (a2 + a3 + a5 + a6 in one launch):
+// a.a is the unmasked X; X~ = fl32(X + eta) is drawn exactly as spl_noise_mask draws it, used for
+// the product and written to nz.xt.  Same plan, same order, same result as the separate calls.
+struct MaskNoise {
+  float* xt;                   // [M, K] X~ out
+  float b;                     // scale Delta f / eps (0: eps = inf, no noise)
+  int mech;                    // spl_mech
+  uint32_t k0, k1, s0, s1;     // Philox key, counter words 2-3
+  uint64_t offset;             // Philox block offset (host part)
+  const uint64_t* offset_dev;  // device part of the offset (may be null)
+};
+constexpr int kGemvMaskMaxM = 4;  // rows up to which every block draws its slice's noise itself
+spl_status run_gemv_masked(const LinearArgs& a, const Plan& p, const MaskNoise& nz);
+// Argument check shared by the noise entries.
+spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech);
 int64_t gemv_max_ks(int64_t M);                           // largest K-slice the decode kernel stages for M rows
 // Launch variant and K-split of a one-launch tcgen05 call (false if the call makes two launches).
 bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, int* variant, int* splits);

@@ -18,67 +18,12 @@
 #include <cuda_fp16.h>
 
 #include "common.cuh"
+#include "noise.cuh"
 
 namespace spl {
 namespace {
 
-constexpr uint32_t kPhiloxM0 = 0xD2511F53u;  // round multiplier for counter word 0
-constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;  // round multiplier for counter word 2
-constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;  // key increment, word 0
-constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;  // key increment, word 1
 constexpr int kThreads = 256;
-
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    if (r > 0) {
-      k0 += kPhiloxW0;
-      k1 += kPhiloxW1;
-    }
-    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
-    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-  }
-  return c;
-}
-
-enum { kLaplace = 0, kGaussian = 1, kZero = 2 };
-
-__device__ __forceinline__ float laplace1(uint32_t r, float b) {
-  const float u = __int2float_rn((int)((r & 0xFFFFFFu) + 1u)) * 0x1p-24f;  // (0, 1], exact
-  const float mag = __fmul_rn(b, -logf(u));
-  return (r >> 31) ? -mag : mag;
-}
-
-__device__ __forceinline__ void gauss2(uint32_t ra, uint32_t rb, float b, float& ea, float& eb) {
-  const float u1 = __int2float_rn((int)((ra >> 8) + 1u)) * 0x1p-24f;  // (0, 1]
-  const float u2 = __int2float_rn((int)(rb >> 8)) * 0x1p-24f;         // [0, 1)
-  const float R = sqrtf(__fmul_rn(-2.0f, logf(u1)));
-  float s, c;
-  sincospif(2.0f * u2, &s, &c);  // sin/cos of 2 pi u2; 2*u2 is exact
-  const float sr = __fmul_rn(b, R);
-  ea = __fmul_rn(sr, c);
-  eb = __fmul_rn(sr, s);
-}
-
-template <int MECH>
-__device__ __forceinline__ float4 draw_block(uint64_t j, uint32_t k0, uint32_t k1, uint32_t s0,
-                                             uint32_t s1, float b) {
-  if (MECH == kZero) return make_float4(0.f, 0.f, 0.f, 0.f);
-  const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
-  float4 e;
-  if (MECH == kLaplace) {
-    e = make_float4(laplace1(r.x, b), laplace1(r.y, b), laplace1(r.z, b), laplace1(r.w, b));
-  } else {
-    gauss2(r.x, r.y, b, e.x, e.y);
-    gauss2(r.z, r.w, b, e.z, e.w);
-  }
-  return e;
-}
-
-__device__ __forceinline__ float4 add4(float4 a, float4 b) {
-  return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z), __fadd_rn(a.w, b.w));
-}
 
 // xt = x + eta (if xt), nout = eta (if nout).  n elements, nb = ceil(n/4) Philox blocks.
 template <int MECH>
@@ -414,14 +359,6 @@ int grid_for(int64_t work_items, int blocks_per_sm) {
   return (int)std::max<int64_t>(1, std::min(want, cap));
 }
 
-spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech) {
-  if (rows < 0 || cols < 0) return SPL_EINVAL;
-  if (!(eps > 0.0)) return SPL_EINVAL;  // also rejects NaN
-  if (!(sensitivity >= 0.0) || std::isinf(sensitivity)) return SPL_EINVAL;
-  if (mech != SPL_MECH_LAPLACE && mech != SPL_MECH_GAUSSIAN) return SPL_EINVAL;
-  return SPL_OK;
-}
-
 spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, double sensitivity, double eps,
                              spl_mech mech, spl_rng rng, cudaStream_t stream) {
   if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
@@ -442,6 +379,14 @@ spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, 
 }
 
 }  // namespace
+
+spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech) {
+  if (rows < 0 || cols < 0) return SPL_EINVAL;
+  if (!(eps > 0.0)) return SPL_EINVAL;  // also rejects NaN
+  if (!(sensitivity >= 0.0) || std::isinf(sensitivity)) return SPL_EINVAL;
+  if (mech != SPL_MECH_LAPLACE && mech != SPL_MECH_GAUSSIAN) return SPL_EINVAL;
+  return SPL_OK;
+}
 
 // Row split with an optional fused mask (mech < 0: none).  Rows whose register copy does not fit
 // (more than 16384 entries) and no mask take the two-pass kernel.

@@ -29,6 +29,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "noise.cuh"
 
 namespace spl {
 namespace {
@@ -86,11 +87,22 @@ __device__ __forceinline__ int reduced_base(int lane, int* dup_mask) {
   return base;
 }
 
-template <int MT>
+constexpr int kNoMask = -1;
+
+// Noise of the fused mask, as the kernel receives it (MASK != kNoMask).
+struct KernelNoise {
+  float* xt;
+  float b;
+  uint32_t k0, k1, s0, s1;
+  uint64_t offset;
+  const uint64_t* offset_dev;
+};
+
+template <int MT, int MASK>
 __global__ void __launch_bounds__(THREADS)
 gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* __restrict__ W,
             const float* __restrict__ C, float* __restrict__ part, unsigned int* __restrict__ counters, int M,
-            int64_t K, int64_t N, int ks, int splits, int prefetch_lines) {
+            int64_t K, int64_t N, int ks, int splits, int prefetch_lines, KernelNoise nz) {
   constexpr int RQ = rows_per_lane(MT), RB = rows_per_block(MT), U = unroll_steps(MT);
   constexpr int V = RQ * MT;
   extern __shared__ __align__(16) float4 xs[];  // [MT][ks / 4]
@@ -111,15 +123,19 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
   }
 
   // W never changes, so its first lines are fetched before waiting on the kernel that writes X~
-  // and C: the first U steps into registers, the next prefetch_lines lines of each row into L2.
+  // and C: the first U steps into registers (after the staging when it draws noise, which needs
+  // the registers), the next prefetch_lines lines of each row into L2.
   float4 w[U][RQ];
+  auto load_first = [&]() {
 #pragma unroll
-  for (int u = 0; u < U; ++u)
+    for (int u = 0; u < U; ++u)
 #pragma unroll
-    for (int r = 0; r < RQ; ++r)
-      w[u][r] = (valid[r] && u * kStep + kl < klen) ? __ldcs(reinterpret_cast<const float4*>(wp[r] + u * kStep))
-                                                     : make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int l = U + (lane & 7); l < prefetch_lines && l * kStep < klen; l += 8)
+      for (int r = 0; r < RQ; ++r)
+        w[u][r] = (valid[r] && u * kStep + kl < klen) ? __ldcs(reinterpret_cast<const float4*>(wp[r] + u * kStep))
+                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+  };
+  if constexpr (MASK == kNoMask) load_first();
+  for (int l = (MASK == kNoMask ? U : 0) + (lane & 7); l < prefetch_lines && l * kStep < klen; l += 8)
 #pragma unroll
     for (int r = 0; r < RQ; ++r)
       if (valid[r]) asm volatile("prefetch.global.L2 [%0];" ::"l"(wp[r] - kl + l * kStep));
@@ -127,11 +143,34 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 
   // stage X~[:, k0:k0+ks] (rows >= M and columns >= klen are zero)
   const int q_row = ks >> 2, q_len = klen >> 2;
+  if constexpr (MASK == kNoMask) {
 #pragma unroll
-  for (int m = 0; m < MT; ++m) {
-    const float4* src = reinterpret_cast<const float4*>(X + (int64_t)m * K + k0);
-    for (int q = threadIdx.x; q < q_row; q += THREADS)
-      xs[m * q_row + q] = (m < M && q < q_len) ? __ldg(src + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int m = 0; m < MT; ++m) {
+      const float4* src = reinterpret_cast<const float4*>(X + (int64_t)m * K + k0);
+      for (int q = threadIdx.x; q < q_row; q += THREADS)
+        xs[m * q_row + q] = (m < M && q < q_len) ? __ldg(src + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  } else {
+    // fused mask: X~ = fl32(X + eta), eta of element (m, k) being lane k % 4 of Philox block
+    // (m K + k) / 4 + offset, as the mask kernel draws it; the blocks of the first row group
+    // also write X~ out
+    const uint64_t off = nz.offset + (nz.offset_dev ? *nz.offset_dev : 0ull);
+    const bool write_xt = blockIdx.x == 0;
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      const float4* src = reinterpret_cast<const float4*>(X + (int64_t)m * K + k0);
+      float4* dst = reinterpret_cast<float4*>(nz.xt + (int64_t)m * K + k0);
+      const uint64_t j0 = (uint64_t)(((int64_t)m * K + k0) >> 2) + off;
+      for (int q = threadIdx.x; q < q_row; q += THREADS) {
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (m < M && q < q_len) {
+          v = add4(__ldg(src + q), draw_block<MASK>(j0 + (uint64_t)q, nz.k0, nz.k1, nz.s0, nz.s1, nz.b));
+          if (write_xt) __stcs(dst + q, v);
+        }
+        xs[m * q_row + q] = v;
+      }
+    }
+    load_first();
   }
   __syncthreads();
 
@@ -228,8 +267,8 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 
 int padded_m(int64_t M) { return M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : M <= 8 ? 8 : 16; }
 
-template <int MT>
-void* kernel_ptr() { return reinterpret_cast<void*>(gemv_kernel<MT>); }
+template <int MT, int MASK = kNoMask>
+void* kernel_ptr() { return reinterpret_cast<void*>(gemv_kernel<MT, MASK>); }
 
 void* kernel_for(int mt) {
   switch (mt) {
@@ -249,9 +288,12 @@ bool smem_attr_set() {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
   std::lock_guard<std::mutex> lock(mu);
   if (!done[dev]) {
-    for (int mt : {1, 2, 4, 8, 16})
-      if (cudaFuncSetAttribute(kernel_for(mt), cudaFuncAttributeMaxDynamicSharedMemorySize, kXsBytes) !=
-          cudaSuccess) {
+    void* const kernels[] = {kernel_ptr<1>(), kernel_ptr<2>(), kernel_ptr<4>(), kernel_ptr<8>(), kernel_ptr<16>(),
+                             kernel_ptr<1, kZero>(), kernel_ptr<2, kZero>(), kernel_ptr<4, kZero>(),
+                             kernel_ptr<1, kLaplace>(), kernel_ptr<2, kLaplace>(), kernel_ptr<4, kLaplace>(),
+                             kernel_ptr<1, kGaussian>(), kernel_ptr<2, kGaussian>(), kernel_ptr<4, kGaussian>()};
+    for (void* k : kernels)
+      if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kXsBytes) != cudaSuccess) {
         cudaGetLastError();
         return false;
       }
@@ -260,16 +302,27 @@ bool smem_attr_set() {
   return true;
 }
 
-template <int MT>
-spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int* counters) {
+template <int MT, int MASK = kNoMask>
+spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int* counters,
+                  const KernelNoise& nz = KernelNoise{}) {
   if (!smem_attr_set()) return SPL_ECUDA;
   dim3 grid((unsigned)ceil_div(a.N, rows_per_block(MT)), (unsigned)p.splits);
   const size_t smem = (size_t)MT * p.k_per_split * sizeof(float);
   // L2 budget of the early prefetch: about 32 MB over the whole grid, in 128-byte lines per row
   const int64_t rows = (int64_t)grid.x * rows_per_block(MT) * p.splits;
   const int lines = (int)std::min<int64_t>(p.k_per_split / kStep, ((int64_t(32) << 20) / std::max<int64_t>(rows, 1)) >> 7);
-  return launch_pdl(gemv_kernel<MT>, grid, dim3(THREADS), smem, a.stream, a.out, a.a, a.w, a.c, part, counters,
-                    (int)a.M, a.K, a.N, (int)p.k_per_split, p.splits, lines);
+  return launch_pdl(gemv_kernel<MT, MASK>, grid, dim3(THREADS), smem, a.stream, a.out, a.a, a.w, a.c, part, counters,
+                    (int)a.M, a.K, a.N, (int)p.k_per_split, p.splits, lines, nz);
+}
+
+template <int MASK>
+spl_status launch_masked(const LinearArgs& a, const Plan& p, float* part, unsigned int* counters,
+                         const KernelNoise& nz) {
+  switch (padded_m(a.M)) {
+    case 1: return launch<1, MASK>(a, p, part, counters, nz);
+    case 2: return launch<2, MASK>(a, p, part, counters, nz);
+    default: return launch<4, MASK>(a, p, part, counters, nz);
+  }
 }
 
 // Resident blocks per SM of the decode kernel for MT rows and a K-slice of ks (cached).
@@ -330,15 +383,37 @@ Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
   return p;
 }
 
-spl_status run_gemv(const LinearArgs& a, const Plan& p) {
+namespace {
+spl_status scratch(const LinearArgs& a, const Plan& p, float** part, unsigned int** counters) {
+  *part = nullptr;
+  *counters = nullptr;
   if (p.splits > 65535) return SPL_ESHAPE;
-  float* part = nullptr;
-  unsigned int* counters = nullptr;
   if (p.splits > 1) {
     if (ceil_div(a.N, rows_per_block(padded_m(a.M))) > kMaxCounters) return SPL_ESHAPE;
-    counters = static_cast<unsigned int*>(a.ws);
-    part = reinterpret_cast<float*>(static_cast<char*>(a.ws) + kCounterBytes);
+    *counters = static_cast<unsigned int*>(a.ws);
+    *part = reinterpret_cast<float*>(static_cast<char*>(a.ws) + kCounterBytes);
   }
+  return SPL_OK;
+}
+}  // namespace
+
+spl_status run_gemv_masked(const LinearArgs& a, const Plan& p, const MaskNoise& nz) {
+  if (a.M > kGemvMaskMaxM || !nz.xt) return SPL_EINVAL;
+  float* part;
+  unsigned int* counters;
+  spl_status st = scratch(a, p, &part, &counters);
+  if (st != SPL_OK) return st;
+  const KernelNoise kn{nz.xt, nz.b, nz.k0, nz.k1, nz.s0, nz.s1, nz.offset, nz.offset_dev};
+  if (nz.b == 0.0f) return launch_masked<kZero>(a, p, part, counters, kn);
+  if (nz.mech == SPL_MECH_LAPLACE) return launch_masked<kLaplace>(a, p, part, counters, kn);
+  return launch_masked<kGaussian>(a, p, part, counters, kn);
+}
+
+spl_status run_gemv(const LinearArgs& a, const Plan& p) {
+  float* part;
+  unsigned int* counters;
+  spl_status st = scratch(a, p, &part, &counters);
+  if (st != SPL_OK) return st;
   switch (padded_m(a.M)) {
     case 1: return launch<1>(a, p, part, counters);
     case 2: return launch<2>(a, p, part, counters);

@@ -66,7 +66,7 @@ spl_status check_weight(const spl_weight* W, int64_t K) {
 
 spl_status run_linear(float* out, const float* a, const spl_weight* W, const float* C, bool need_c, int64_t M,
                       int64_t K, int64_t N, spl_path path, void* ws, size_t ws_bytes, cudaStream_t stream,
-                      const spl_weight* A = nullptr) {
+                      const spl_weight* A = nullptr, const MaskNoise* noise = nullptr) {
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
   if (!valid_path(path)) return SPL_EINVAL;
   if (M == 0 || N == 0) return SPL_OK;
@@ -98,9 +98,10 @@ spl_status run_linear(float* out, const float* a, const spl_weight* W, const flo
     args.a_l16 = A->f16_lo;
     args.a_exp = A->f16_exp;
   }
+  if (noise && (plan.kernel != kKernelGemv || M > kGemvMaskMaxM)) return SPL_EUNSUPPORTED;
   switch (plan.kernel) {
     case kKernelTc: return run_tc(args, plan);
-    case kKernelGemv: return run_gemv(args, plan);
+    case kKernelGemv: return noise ? run_gemv_masked(args, plan, *noise) : run_gemv(args, plan);
     default: return run_simt(args, plan);
   }
 }
@@ -192,6 +193,42 @@ extern "C" spl_status spl_masked_linear_unmask_split(float* Y, const spl_weight*
                                                      void* workspace, size_t workspace_bytes, cudaStream_t stream) {
   if (!Xt) return SPL_EINVAL;
   return run_linear(Y, Xt->w, W, C, true, M, K, N, path, workspace, workspace_bytes, stream, Xt);
+}
+
+extern "C" spl_status spl_noise_mask_linear_unmask(float* Y, float* Xt, const float* X, const spl_weight* W,
+                                                   const float* C, int64_t M, int64_t K, int64_t N,
+                                                   double sensitivity, double eps, spl_mech mech, spl_rng rng,
+                                                   spl_path path, void* workspace, size_t workspace_bytes,
+                                                   cudaStream_t stream) {
+  spl_status st = validate_noise(M, K, sensitivity, eps, mech);
+  if (st != SPL_OK) return st;
+  if (N < 0 || !valid_path(path)) return SPL_EINVAL;
+  if (M > 0 && K > 0 && (!Xt || !X)) return SPL_EINVAL;
+  if ((Xt && !aligned16(Xt)) || (X && !aligned16(X))) return SPL_EALIGN;
+  if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
+  if (M > 0 && K > 0) {  // X~ is written while other blocks still read X
+    const uintptr_t x0 = reinterpret_cast<uintptr_t>(X), t0 = reinterpret_cast<uintptr_t>(Xt);
+    const uintptr_t bytes = (uintptr_t)(M * K) * sizeof(float);
+    if (x0 < t0 + bytes && t0 < x0 + bytes) return SPL_EINVAL;
+  }
+  const bool fused = M > 0 && M <= kGemvMaskMaxM && K > 0 && N > 0 && W &&
+                     resolve(M, K, path, has_tf32(*W), has_f16(*W)) == SPL_PATH_FP32;
+  if (!fused) {  // mask, then the product: two launches with the same results
+    st = spl_noise_mask(Xt, nullptr, X, M, K, sensitivity, eps, mech, rng, stream);
+    if (st != SPL_OK) return st;
+    return run_linear(Y, Xt, W, C, true, M, K, N, path, workspace, workspace_bytes, stream);
+  }
+  MaskNoise nz{};
+  nz.xt = Xt;
+  nz.b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
+  nz.mech = (int)mech;
+  nz.k0 = (uint32_t)rng.seed;
+  nz.k1 = (uint32_t)(rng.seed >> 32);
+  nz.s0 = (uint32_t)rng.stream_id;
+  nz.s1 = (uint32_t)(rng.stream_id >> 32);
+  nz.offset = rng.offset;
+  nz.offset_dev = rng.offset_dev;
+  return run_linear(Y, X, W, C, true, M, K, N, path, workspace, workspace_bytes, stream, nullptr, &nz);
 }
 
 extern "C" size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows,

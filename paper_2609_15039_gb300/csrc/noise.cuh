@@ -1,0 +1,99 @@
+// Noise draw shared by the mask kernels (elementwise.cu) and the decode product's fused mask
+// (gemv.cu): Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11, Sec. 3.3) and the Laplace /
+// Gaussian transforms at scale Delta f / eps (Sec. 4.4).  Element e of a flat [rows, cols]
+// tensor is lane e % 4 of Philox block e / 4 + offset, key = seed, counter words 2-3 =
+// stream_id.  The mask is one fp32 round-to-nearest addition x + eta (Sec. 3.3.1).
+#pragma once
+
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace spl {
+namespace {
+
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u;  // round multiplier for counter word 0
+constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;  // round multiplier for counter word 2
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;  // key increment, word 0
+constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;  // key increment, word 1
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k0 += kPhiloxW0;
+      k1 += kPhiloxW1;
+    }
+    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
+    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+enum { kLaplace = 0, kGaussian = 1, kZero = 2 };
+
+__device__ __forceinline__ float laplace1(uint32_t r, float b) {
+  const float u = __int2float_rn((int)((r & 0xFFFFFFu) + 1u)) * 0x1p-24f;  // (0, 1], exact
+  const float mag = __fmul_rn(b, -logf(u));
+  return (r >> 31) ? -mag : mag;
+}
+
+// sin(pi x) and cos(pi x) for x = 2 u2 in [0, 2), x a multiple of 2^-23: x = q / 2 + r with
+// q = rint(2 x) (quarter turns) and |r| <= 1/4, both exact; sin(pi r) and cos(pi r) from their
+// Taylor series to degree 9 and 10 (truncation below 3e-9 at |pi r| <= pi / 4), evaluated by
+// Horner's rule in r^2; then the rotation by q quarter turns.  Error at most 1.7 ulp (checked
+// against binary64 sin and cos over all 2^24 inputs), with the exact zeros of sin and cos exact.
+__device__ __forceinline__ void sincospi_turns(float x, float* s, float* c) {
+  const float q = rintf(2.0f * x);
+  const float r = fmaf(q, -0.5f, x);
+  const float r2 = __fmul_rn(r, r);
+  float ps = 0.08214588661112819f;        //  pi^9 / 9!
+  ps = fmaf(ps, r2, -0.5992645293207919f);  // -pi^7 / 7!
+  ps = fmaf(ps, r2, 2.550164039877345f);    //  pi^5 / 5!
+  ps = fmaf(ps, r2, -5.167712780049969f);   // -pi^3 / 3!
+  ps = fmaf(ps, r2, 3.141592653589793f);    //  pi
+  const float sr = __fmul_rn(ps, r);
+  float pc = -0.02580689139001405f;         // -pi^10 / 10!
+  pc = fmaf(pc, r2, 0.23533063035889312f);  //  pi^8 / 8!
+  pc = fmaf(pc, r2, -1.3352627688545893f);  // -pi^6 / 6!
+  pc = fmaf(pc, r2, 4.058712126416768f);    //  pi^4 / 4!
+  pc = fmaf(pc, r2, -4.934802200544679f);   // -pi^2 / 2!
+  pc = fmaf(pc, r2, 1.0f);
+  const int t = (int)q & 3;  // (sin, cos)(pi (r + t / 2))
+  *s = t == 0 ? sr : t == 1 ? pc : t == 2 ? -sr : -pc;
+  *c = t == 0 ? pc : t == 1 ? -sr : t == 2 ? -pc : sr;
+}
+
+__device__ __forceinline__ void gauss2(uint32_t ra, uint32_t rb, float b, float& ea, float& eb) {
+  const float u1 = __int2float_rn((int)((ra >> 8) + 1u)) * 0x1p-24f;  // (0, 1]
+  const float u2 = __int2float_rn((int)(rb >> 8)) * 0x1p-24f;         // [0, 1)
+  const float R = sqrtf(__fmul_rn(-2.0f, logf(u1)));
+  float s, c;
+  sincospi_turns(2.0f * u2, &s, &c);  // sin/cos of 2 pi u2; 2*u2 is exact
+  const float sr = __fmul_rn(b, R);
+  ea = __fmul_rn(sr, c);
+  eb = __fmul_rn(sr, s);
+}
+
+template <int MECH>
+__device__ __forceinline__ float4 draw_block(uint64_t j, uint32_t k0, uint32_t k1, uint32_t s0,
+                                             uint32_t s1, float b) {
+  if (MECH == kZero) return make_float4(0.f, 0.f, 0.f, 0.f);
+  const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
+  float4 e;
+  if (MECH == kLaplace) {
+    e = make_float4(laplace1(r.x, b), laplace1(r.y, b), laplace1(r.z, b), laplace1(r.w, b));
+  } else {
+    gauss2(r.x, r.y, b, e.x, e.y);
+    gauss2(r.z, r.w, b, e.z, e.w);
+  }
+  return e;
+}
+
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+  return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z), __fadd_rn(a.w, b.w));
+}
+
+}  // namespace
+}  // namespace spl

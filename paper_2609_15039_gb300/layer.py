@@ -178,6 +178,13 @@ class MaskedLayer:
             return False
         return spl.spl_resolve_path(M, g.K, g.N, self.path_of(g, path, M)) == spl.SPL_PATH_FP16X3
 
+    def _fused_mask(self, g, path, M):
+        """True when the online product of group g is the FP32 decode kernel at M <= 4 rows: then one
+        launch draws the noise, masks and multiplies (spl_noise_mask_linear_unmask)."""
+        if g.name in self.fp64 or M > 4:
+            return False
+        return spl.spl_resolve_path(M, g.K, g.N, self.path_of(g, path, M)) == spl.SPL_PATH_FP32
+
     def block_offset(self, g, cycle, d):
         """First Philox block of draw d of bank cycle ``cycle`` for group g."""
         per_draw = self.M * g.K // 4  # K % 4 == 0, so a draw is a whole number of blocks
@@ -225,6 +232,17 @@ class MaskedLayer:
             off, off_dev = self._offset(gi, g, cycle, d, device_base)
             fp64 = g.name in self.fp64
             xs = b.get("xs") if self._fused_split(g, path, M) else None
+            if self._fused_mask(g, path, M):
+                if timer:
+                    timer("begin", "masked_linear_unmask", g.name)
+                spl.spl_noise_mask_linear_unmask(b["Y"], b["xt"], inputs[g.name], g.wt, b["C"][d * M:(d + 1) * M],
+                                                 self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off,
+                                                 path=self.path_of(g, path, M), workspace=self.workspace,
+                                                 stream=stream, offset_dev=off_dev)
+                if timer:
+                    timer("end", "masked_linear_unmask", g.name)
+                out[g.name] = b["Y"]
+                continue
             if fp64:
                 spl.spl_noise_mask_f64(b["xt"], inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
                                        offset=off, stream=stream, offset_dev=off_dev)

@@ -72,6 +72,8 @@ _SIGS = {
     "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_masked_linear_unmask": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_masked_linear_unmask_noalloc": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P]),
+    "spl_noise_mask_linear_unmask": (_I, [_P, _P, _P, _PW, _P, _I64, _I64, _I64, _D, _D, _I, spl_rng, _I, _P, _SZ,
+                                          _P]),
     "spl_delta_layernorm": (_D, [_P, _I64]),
     "spl_delta_attention": (_D, [_P, _I64, _D]),
     "spl_delta_activation": (_D, [_P, _P, _I64, _I64, _D, _D]),
@@ -413,6 +415,23 @@ def spl_unmask(Y, Yt, C, stream=None):
 
 def spl_masked_linear_unmask(Y, Xt, W, C, path="auto", workspace=None, stream=None):
     _linear(lib().spl_masked_linear_unmask, "spl_masked_linear_unmask", Y, Xt, W, C, path, workspace, stream)
+
+
+def spl_noise_mask_linear_unmask(Y, Xt, X, W, C, sensitivity, eps, mech, seed, stream_id=0, offset=0, path="auto",
+                                 workspace=None, stream=None, offset_dev=None):
+    """a2 + a3 + a5 + a6: Xt = X + eta (written), Y = Xt W^T - C; one launch for M <= 4 on FP32."""
+    W = _weight(W)
+    M, K = _rows_cols(X)
+    N = W.shape[0]
+    if W.shape[-1] != K or Xt.numel() != M * K or Y.numel() != M * N or C.numel() != M * N:
+        raise ValueError("spl_noise_mask_linear_unmask: shape mismatch")
+    wsp, wsb = _ws(workspace)
+    ws_ = W.c_struct()
+    _check(lib().spl_noise_mask_linear_unmask(_dev(Y, "Y"), _dev(Xt, "Xt"), _dev(X, "X"), ctypes.byref(ws_),
+                                              _dev(C, "C"), M, K, N, float(sensitivity), _eps(eps), _mech(mech),
+                                              _rng(seed, stream_id, offset, offset_dev), _path(path), wsp, wsb,
+                                              _stream(stream)),
+           "spl_noise_mask_linear_unmask")
 
 
 def spl_masked_linear_unmask_noalloc(Y, Xt, W, C, stream=None):

@@ -409,6 +409,42 @@ def test_noise_mask_split_equals_separate_calls(spl, rows, cols, mech, eps):
     assert torch.equal(hi, hi_ref) and torch.equal(ex, ex_ref)
 
 
+@pytest.mark.parametrize("M,K,N,mech,eps", [(1, 3072, 3072, "laplace", 1.0), (2, 1028, 600, "gaussian", 0.5),
+                                             (3, 8192, 520, "laplace", None), (4, 2560, 2056, "gaussian", 1.0),
+                                             (5, 516, 300, "laplace", 1.0), (16, 3072, 512, "gaussian", 1.0)])
+def test_noise_mask_linear_unmask_equals_separate_calls(spl, M, K, N, mech, eps):
+    """The decode call with the mask drawn inside the product (M <= 4; two launches beyond) gives
+    the X~ of spl_noise_mask and the Y of spl_masked_linear_unmask bit for bit, and both match the
+    oracle: X~ within the noise tolerance, Y within the FP32 product bound of that X~."""
+    W, Wt = _weights(spl, N, K, seed=N + K)
+    X = wl.activations(M, K, seed=M + 21).numpy()
+    C = dev(wl.activations(M, N, seed=M + 22).numpy())
+    base = torch.tensor([500], dtype=torch.int64, device="cuda")
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp32"))
+    xt_ref, Y_ref = torch.empty((M, K), device="cuda"), torch.empty((M, N), device="cuda")
+    spl.spl_noise_mask(xt_ref, None, dev(X), 825.3, eps, mech, seed=23, stream_id=1, offset=500 + 12)
+    spl.spl_masked_linear_unmask(Y_ref, xt_ref, Wt, C, path="fp32", workspace=ws)
+    xt, Y = torch.full((M, K), 7.0, device="cuda"), torch.full((M, N), 7.0, device="cuda")
+    n0 = spl.spl_launch_count()
+    spl.spl_noise_mask_linear_unmask(Y, xt, dev(X), Wt, C, 825.3, eps, mech, seed=23, stream_id=1, offset=12,
+                                     path="fp32", workspace=ws, offset_dev=base)
+    torch.cuda.synchronize()
+    assert spl.spl_launch_count() - n0 == (1 if M <= 4 else 2)
+    assert torch.equal(xt, xt_ref) and torch.equal(Y, Y_ref)
+    # against the oracle: X~ = fl32(X + eta) with the oracle's eta (a few ulps of the transcendentals)
+    n_exp = philox.noise((M, K), 825.3, math.inf if eps is None else eps, mech, 23, 1, 512).astype(np.float64)
+    xt_exp = linear.mask(X, n_exp.astype(np.float32)).astype(np.float64)
+    tol = 2 * ulp32(xt_exp) + 8 * ulp32(n_exp)
+    if mech == "gaussian" and eps is not None:
+        tol = tol + 8 * U * float(np.float32(825.3 / eps)) * philox.radius_fp64((M, K), 23, 1, 512)
+    assert np.all(np.abs(f64(xt) - xt_exp) <= tol)
+    assert_product_close(f32(Y), f32(xt), W, "fp32", C=f32(C), what="fused decode call")
+    Xd = dev(X)
+    with pytest.raises(spl.SplError) as e:  # X~ may not overwrite X: other blocks still read it
+        spl.spl_noise_mask_linear_unmask(Y, Xd, Xd, Wt, C, 825.3, eps, mech, seed=23, path="fp32", workspace=ws)
+    assert e.value.status == spl.SPL_EINVAL
+
+
 @pytest.mark.parametrize("M,K,N", [(128, 3072, 3072), (130, 1032, 600), (512, 3072, 5120), (9, 256, 512)])
 def test_presplit_product_equals_plain(spl, M, K, N):
     W, Wt = _weights(spl, N, K, seed=N + 3)
