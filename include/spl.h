@@ -385,6 +385,21 @@ spl_status spl_spectral_norm(double* out, const float* W, int64_t N, int64_t K, 
 spl_status spl_test_tc_wait_timeout(float* out, const float* A, const spl_weight* W, int64_t M, int64_t K,
                                     int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
+/* Test hook (no counterpart in the paper): the launch shape the tensor-core
+ * product of M x K by N x K takes (seg_splits = 0), or a correction whose sums
+ * follow a seg_splits-way split of K (the bank, seg_splits >= 1).  out[5]
+ * (host) receives {tile width, ring KB, tiles of the unsplit launch, tiles of the
+ * split launch, its K-split}.  EINVAL for non-positive sizes, seg_splits outside
+ * [0, 8] or a NULL out.  No GPU work; needs a current CUDA device for the
+ * occupancy queries. */
+spl_status spl_test_tc_shape(int64_t M, int64_t K, int64_t N, int64_t seg_splits, int64_t* out);
+
+/* Test hook (no counterpart in the paper): *out (host) = the number of clusters
+ * of `cluster` CTAs (1..8) of the launch variant (tile_n, ring_kb) -- (256, 192),
+ * (128, 224) or (128, 96) -- that can be resident at once on the current device.
+ * EINVAL for another variant, cluster outside [1, 8] or a NULL out. */
+spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int64_t cluster, int64_t* out);
+
 /* Test hook (the paper has no counterpart): Y = Xt W^T (- C if C is not NULL)
  * on the tcgen05 kernel with a fixed launch variant -- tile width tile_n and a
  * stage ring of ring_kb KB: (256, 192), (128, 224) or (128, 96) -- and every

@@ -756,13 +756,22 @@ TcShape tc_shape_for(int v, int64_t M, int64_t K, int64_t N, int sms) {
   return best;
 }
 
-// Best variant for one unsplit launch (segmented mode).
-TcShape tc_unsplit_shape(int64_t M, int64_t K, int64_t N, int sms) {
+// Shape of a correction whose sums must follow a seg_splits-way split of K (the bank): whole
+// waves of unsplit tiles that fold the K ranges in TMEM (segmented mode), then the remaining
+// tiles with K split seg_splits ways over a cluster, whose rank-order sum is the same fold; or
+// every tile segmented.  The cheapest variant and form.
+TcShape tc_bank_shape(int64_t M, int64_t K, int64_t N, int seg_splits, int sms) {
   TcShape best{0, 0, 0, 1, 1e300};
   for (int v = 0; v < kVariants; ++v) {
     const int64_t tiles = ceil_div(M, BM) * ceil_div(N, kVariant[v].bn);
     const double c = launch_cost(v, tiles, K, 1, sms);
     if (c < best.cost * (1.0 - 1e-9)) best = TcShape{v, 0, tiles, 1, c};
+    if (seg_splits < 2 || seg_splits > MAX_CLUSTER) continue;
+    const int64_t wave = max_active_clusters(v, 1, sms);
+    const int64_t full = (tiles / wave) * wave, rest = tiles - full;
+    if (rest == 0) continue;
+    const double c2 = launch_cost(v, full, K, 1, sms) + launch_cost(v, rest, K, seg_splits, sms);
+    if (c2 < best.cost * (1.0 - 1e-9)) best = TcShape{v, full, rest, seg_splits, c2};
   }
   return best;
 }
@@ -796,7 +805,7 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
   // The first launch follows the split of A under programmatic dependent launch: its CTAs start
   // (barriers, TMEM, weight tiles) while the split finishes.
   bool first = true;
-  auto launch = [&](int64_t tiles, int64_t base, int splits) -> spl_status {
+  auto launch = [&](int64_t tiles, int64_t base, int splits, int seg) -> spl_status {
     if (tiles <= 0) return SPL_OK;
     const int64_t kps = round_up(ceil_div(a.K, splits), Md::BK);
     cudaLaunchConfig_t cfg;
@@ -817,13 +826,15 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
     first = false;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md, BN, RK>, maps, a.out, a.c, a_exp,
                                              (const int*)a.w_exp, a.M, a.K, a.N, kps, splits, (int)base, m_tiles,
-                                             skip_kblock, seg_blocks);
+                                             skip_kblock, seg);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   };
-  spl_status st = launch(shape.full_tiles, 0, 1);
+  // segmented mode: unsplit tiles fold the K ranges in TMEM; tiles split over a cluster (the same
+  // K ranges) sum them in rank order, which is the same fold
+  spl_status st = launch(shape.full_tiles, 0, 1, seg_blocks);
   if (st != SPL_OK) return st;
-  return launch(shape.rest_tiles, shape.full_tiles, shape.rest_splits);
+  return launch(shape.rest_tiles, shape.full_tiles, shape.rest_splits, shape.rest_splits > 1 ? 0 : seg_blocks);
 }
 
 template <class Md>
@@ -890,7 +901,7 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int f
   if (forced_v >= 0) {
     shape = TcShape{forced_v, 0, ceil_div(a.M, BM) * ceil_div(a.N, kVariant[forced_v].bn), forced_splits, 0.0};
   } else if (seg_splits > 0) {
-    shape = tc_unsplit_shape(a.M, a.K, a.N, device_sm_count());
+    shape = tc_bank_shape(a.M, a.K, a.N, seg_splits, device_sm_count());
   } else {
     shape = tc_shape(a.M, a.K, a.N, device_sm_count());
   }
@@ -950,6 +961,36 @@ extern "C" spl_status spl_test_tc_wait_timeout(float* out, const float* A, const
   if (K > 256) return SPL_ESHAPE;  // one K range per tile: the skipped stage belongs to every CTA
   LinearArgs args = make_args(out, A, *W, nullptr, M, K, N, workspace, workspace_bytes, stream, SPL_PATH_TF32X3);
   return run_tc_impl(args, 0, 0, 1);
+}
+
+// Test hook: the launch shape the tensor-core product (seg_splits = 0) or a correction in the order
+// of a seg_splits-way split (seg_splits > 0) takes: out = {tile width, ring KB, tiles of the
+// unsplit launch, tiles of the split launch, its K-split}.  The paper has no counterpart.
+extern "C" spl_status spl_test_tc_shape(int64_t M, int64_t K, int64_t N, int64_t seg_splits, int64_t* out) {
+  using namespace spl;
+  if (!out || M <= 0 || K <= 0 || N <= 0 || seg_splits < 0 || seg_splits > MAX_CLUSTER) return SPL_EINVAL;
+  const int sms = device_sm_count();
+  const TcShape t = seg_splits > 0 ? tc_bank_shape(M, K, N, (int)seg_splits, sms) : tc_shape(M, K, N, sms);
+  out[0] = kVariant[t.v].bn;
+  out[1] = kVariant[t.v].rk;
+  out[2] = t.full_tiles;
+  out[3] = t.rest_tiles;
+  out[4] = t.rest_splits;
+  return SPL_OK;
+}
+
+// Test hook: co-resident clusters of `cluster` CTAs of the launch variant (tile_n, ring_kb) on the
+// current device (the occupancy query the launch shapes are planned with).  The paper has no
+// counterpart.
+extern "C" spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int64_t cluster, int64_t* out) {
+  using namespace spl;
+  if (!out || cluster < 1 || cluster > MAX_CLUSTER) return SPL_EINVAL;
+  for (int v = 0; v < kVariants; ++v)
+    if (kVariant[v].bn == tile_n && kVariant[v].rk == ring_kb) {
+      *out = max_active_clusters(v, (int)cluster, device_sm_count());
+      return SPL_OK;
+    }
+  return SPL_EINVAL;
 }
 
 // Test hook: the tensor-core product with a fixed tile width and K-split, so that tests cover

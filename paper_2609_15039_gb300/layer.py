@@ -179,9 +179,12 @@ class MaskedLayer:
         return spl.spl_resolve_path(M, g.K, g.N, self.path_of(g, path, M)) == spl.SPL_PATH_FP16X3
 
     def _fused_mask(self, g, path, M):
-        """True when the online product of group g is the FP32 decode kernel at M <= 4 rows: then one
-        launch draws the noise, masks and multiplies (spl_noise_mask_linear_unmask)."""
-        if g.name in self.fp64 or M > 4:
+        """True when the online product of group g is the FP32 decode kernel at 2 <= M <= 4 rows: then
+        one launch draws the noise, masks and multiplies (spl_noise_mask_linear_unmask).  At one row
+        the two-launch form is faster on GB300 (Llama shapes: 76 against 79 us per layer): there the
+        product's blocks load their first W lines while the small mask kernel runs, whereas the
+        fused blocks can only start on W after drawing their noise."""
+        if g.name in self.fp64 or not 2 <= M <= 4:
             return False
         return spl.spl_resolve_path(M, g.K, g.N, self.path_of(g, path, M)) == spl.SPL_PATH_FP32
 

@@ -83,6 +83,8 @@ _SIGS = {
     "spl_choose_path": (_I, [ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double), _P, _P, _PW, _I64,
                              _I64, _I64, _P, _SZ, _P]),
     "spl_test_tc_wait_timeout": (_I, [_P, _P, _PW, _I64, _I64, _I64, _P, _SZ, _P]),
+    "spl_test_tc_capacity": (_I, [_I64, _I64, _I64, ctypes.POINTER(ctypes.c_int64)]),
+    "spl_test_tc_shape": (_I, [_I64, _I64, _I64, _I64, ctypes.POINTER(ctypes.c_int64)]),
     "spl_test_tc_product": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _I, _I, _I, _P, _SZ, _P]),
     "spl_get_device_status": (_I, [_P]),
     "spl_launch_count": (ctypes.c_uint64, []),
@@ -530,6 +532,22 @@ def spl_test_tc_wait_timeout(out, A, W, workspace=None, stream=None):
     wsp, wsb = _ws(workspace)
     _check(lib().spl_test_tc_wait_timeout(_dev(out, "out"), _dev(A, "A"), ctypes.byref(ws_), M, K, N, wsp, wsb,
                                           _stream(stream)), "spl_test_tc_wait_timeout")
+
+
+def spl_test_tc_shape(M, K, N, seg_splits=0):
+    """Launch shape of the tensor-core product (or of a correction in a seg_splits-way order):
+    (tile width, ring KB, unsplit tiles, split tiles, K-split)."""
+    out = (ctypes.c_int64 * 5)()
+    _check(lib().spl_test_tc_shape(int(M), int(K), int(N), int(seg_splits), out), "spl_test_tc_shape")
+    return tuple(int(v) for v in out)
+
+
+def spl_test_tc_capacity(tile_n, ring_kb, cluster):
+    """Co-resident clusters of `cluster` CTAs of the launch variant (tile_n, ring_kb)."""
+    out = ctypes.c_int64(0)
+    _check(lib().spl_test_tc_capacity(int(tile_n), int(ring_kb), int(cluster), ctypes.byref(out)),
+           "spl_test_tc_capacity")
+    return int(out.value)
 
 
 def spl_test_tc_product(Y, Xt, W, C=None, path="fp16x3", tile_n=256, ring_kb=192, splits=1, workspace=None,

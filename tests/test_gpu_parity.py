@@ -372,10 +372,12 @@ def test_matched_correction_cancels_rounding(spl, M, K, N, path):
                                          (128, 3072, 3072, "fp32"), (1, 3072, 3072, "fp32"), (512, 3072, 3072, "fp16x3"),
                                          (1, 3072, 5120, "fp32"), (1, 3072, 16384, "fp32"), (1, 8192, 3072, "fp32"),
                                          (4, 3072, 5120, "fp32"), (3, 1028, 600, "fp32")])
-def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path):
+@pytest.mark.parametrize("draws", [4, 8])
+def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path, draws):
     """The bank's correction of draw d is, bit for bit, what the online product computes when
-    its input is that draw's noise: the same K ranges, partials summed in the same order."""
-    draws = 4
+    its input is that draw's noise: the same K ranges, partials summed in the same order (with 8
+    draws of 128 rows the bank mixes whole waves of tiles that fold the K ranges in TMEM and
+    tiles split over a cluster)."""
     W, Wt = _weights(spl, N, K, seed=K + N + 1)
     eta = torch.empty((draws * M, K), device="cuda")
     spl.spl_noise(eta, 1443.0, 1.0, "gaussian", seed=23)
@@ -388,6 +390,16 @@ def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path):
         spl.spl_masked_linear(Y, eta[d * M:(d + 1) * M].contiguous(), Wt, path=path, workspace=ws)
         assert torch.equal(Y, C[d * M:(d + 1) * M]), (d, float((Y - C[d * M:(d + 1) * M]).abs().max()))
     assert spl.spl_get_device_status() == 0
+
+
+def test_bank_shape_mixes_folded_and_split_tiles(spl):
+    """A correction of 8 x 128 rows for the Llama Q|K|V shape: 160 tiles of 256 columns, one wave
+    of them folded in TMEM and the rest split over a cluster the way the online product splits K."""
+    online = spl.spl_test_tc_shape(128, 3072, 5120)
+    assert online[2] == 0  # the online product is one split launch
+    bank = spl.spl_test_tc_shape(1024, 3072, 5120, seg_splits=online[4])
+    assert bank[2] + bank[3] == (1024 // 128) * (5120 // bank[0])
+    assert bank[3] == 0 or bank[4] == online[4]
 
 
 # ------------------------------------------------ a2 + a3 fused with the split of X~
