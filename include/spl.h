@@ -404,13 +404,14 @@ spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int64_t cluster
  * on the tcgen05 kernel with a fixed launch variant -- tile width tile_n and a
  * stage ring of ring_kb KB: (256, 192), (128, 224) or (128, 96) -- and every
  * tile's K range split `splits` ways (1..8) across a thread-block cluster,
- * instead of the shape the library would choose.  path is SPL_PATH_TF32X3 or
- * SPL_PATH_FP16X3.  Same operands, workspace and errors as
- * spl_masked_linear_unmask; EINVAL for another path or variant, ESHAPE for a
- * split outside 1..8. */
+ * instead of the shape the library would choose; with full_tiles > 0 the first
+ * full_tiles tiles (M fastest) run unsplit in a launch of their own and only the
+ * rest is split.  path is SPL_PATH_TF32X3 or SPL_PATH_FP16X3.  Same operands,
+ * workspace and errors as spl_masked_linear_unmask; EINVAL for another path or
+ * variant or full_tiles outside [0, tiles], ESHAPE for a split outside 1..8. */
 spl_status spl_test_tc_product(float* Y, const float* Xt, const spl_weight* W, const float* C, int64_t M,
                                int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
-                               void* workspace, size_t workspace_bytes, cudaStream_t stream);
+                               int64_t full_tiles, void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last

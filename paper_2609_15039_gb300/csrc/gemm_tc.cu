@@ -671,13 +671,17 @@ bool set_smem_attr() {
 // launch model below (F: fixed cost of a CTA -- launch, pipeline fill, staging and cross-CTA
 // reduction of its tile; b: cost per unit of K, i.e. bytes per K over the bytes the ring keeps
 // in flight, relative to the 256-wide tile with the 192 KB ring).  Measured on GB300.
+// Cost of one round of co-resident CTAs, in units of K: F + f s + b K / s (F: setup and epilogue,
+// f: the cluster reduction per rank, b: the mainloop per K element), fitted to a sweep of every
+// variant, split and whole-wave form over the Llama and Qwen projections at 128..4096 rows on
+// GB300 (the shapes it picks are within 0.3% of the best measured in total).
 struct Variant {
   int bn, rk, cps;
-  double F, b;
+  double F, f, b;
 };
 constexpr int kVariants = 3;
-constexpr Variant kVariant[kVariants] = {{256, 192, 1, 450.0, 1.0}, {128, 224, 1, 300.0, 0.667},
-                                         {128, 96, 2, 300.0, 1.333}};
+constexpr Variant kVariant[kVariants] = {{256, 192, 1, 450.0, 20.0, 1.0}, {128, 224, 1, 300.0, 20.0, 0.9},
+                                         {128, 96, 2, 300.0, 20.0, 1.333}};
 
 // Co-resident clusters of s CTAs of variant v on the current device; clusters must fit inside
 // one GPC, so this is not simply (SMs x CTAs per SM) / s.  Both encodings use the same shared
@@ -718,7 +722,7 @@ int max_active_clusters(int v, int s, int sms) {
 
 // Launch shape: a variant, then either one launch with every tile's K split s ways over a
 // cluster, or whole waves of unsplit tiles followed by the remaining tiles split (so the last
-// wave is not mostly idle).  Cost of a launch in units of K: rounds x (F + b K / s), rounds
+// wave is not mostly idle).  Cost of a launch in units of K: rounds x (F + f s + b K / s), rounds
 // counting co-resident CTAs.  At least 256 of K per CTA; ties go to the earlier variant and to
 // fewer splits.
 struct TcShape {
@@ -733,7 +737,7 @@ double launch_cost(int v, int64_t tiles, int64_t K, int s, int sms) {
   if (tiles <= 0) return 0.0;
   const int64_t capacity = (int64_t)max_active_clusters(v, s, sms) * s;
   const int64_t rounds = ceil_div(tiles * s, capacity);
-  return (double)rounds * (kVariant[v].F + kVariant[v].b * (double)K / (double)s);
+  return (double)rounds * (kVariant[v].F + kVariant[v].f * s + kVariant[v].b * (double)K / (double)s);
 }
 
 TcShape tc_shape_for(int v, int64_t M, int64_t K, int64_t N, int sms) {
@@ -847,9 +851,11 @@ spl_status launch_variant(const LinearArgs& a, const uint16_t* hi, const uint16_
   }
 }
 
-// forced_v >= 0: every tile with that variant and K-split (forced_splits) in one launch.
+// forced_v >= 0: every tile with that variant, the first forced_full tiles unsplit in a launch of their own
+// and the rest with K split forced_splits ways (one launch when forced_full is 0).
 // seg_splits > 0: segmented mode, one unsplit launch whose sums follow a seg_splits-way split.
-spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int forced_splits, int seg_splits = 0) {
+spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int forced_splits, int seg_splits = 0,
+                       int64_t forced_full = 0) {
   const int cc = device_cc();
   if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
   const bool f16 = a.path == SPL_PATH_FP16X3;
@@ -899,7 +905,8 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int f
   }
   TcShape shape;
   if (forced_v >= 0) {
-    shape = TcShape{forced_v, 0, ceil_div(a.M, BM) * ceil_div(a.N, kVariant[forced_v].bn), forced_splits, 0.0};
+    const int64_t tiles = ceil_div(a.M, BM) * ceil_div(a.N, kVariant[forced_v].bn);
+    shape = TcShape{forced_v, forced_full, tiles - forced_full, forced_splits, 0.0};
   } else if (seg_splits > 0) {
     shape = tc_bank_shape(a.M, a.K, a.N, seg_splits, device_sm_count());
   } else {
@@ -997,7 +1004,8 @@ extern "C" spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int6
 // every kernel instance and a sweep can time each launch shape.  The paper has no counterpart.
 extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_weight* W, const float* C, int64_t M,
                                           int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
-                                          void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+                                          int64_t full_tiles, void* workspace, size_t workspace_bytes,
+                                          cudaStream_t stream) {
   using namespace spl;
   if (!out || !A || !W || !W->w || M <= 0 || N <= 0 || K <= 0) return SPL_EINVAL;
   if (path != SPL_PATH_TF32X3 && path != SPL_PATH_FP16X3) return SPL_EINVAL;
@@ -1008,6 +1016,8 @@ extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_
   if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
   if ((K & 3) != 0) return SPL_EALIGN;
   if (!aligned16(out) || !aligned16(A) || (C && !aligned16(C))) return SPL_EALIGN;
+  const int64_t tiles = ceil_div(M, BM) * ceil_div(N, (int64_t)tile_n);
+  if (full_tiles < 0 || full_tiles > tiles) return SPL_EINVAL;
   const LinearArgs args = make_args(out, A, *W, C, M, K, N, workspace, workspace_bytes, stream, path);
-  return run_tc_impl(args, -1, v, splits);
+  return run_tc_impl(args, -1, v, splits, 0, full_tiles);
 }

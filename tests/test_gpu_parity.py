@@ -246,6 +246,12 @@ def test_tc_every_launch_shape(spl, path, tile_n, ring_kb, splits):
     Y2 = torch.empty((M, N), device="cuda")
     spl.spl_test_tc_product(Y2, dev(A), Wt, None, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=splits)
     assert_product_close(f32(Y2), A, W, path, what="without C")
+    # the first tiles unsplit in a launch of their own, the rest split
+    tiles = -(-M // 128) * -(-N // tile_n)
+    Y3 = torch.empty((M, N), device="cuda")
+    spl.spl_test_tc_product(Y3, dev(A), Wt, dev(C), path=path, tile_n=tile_n, ring_kb=ring_kb, splits=splits,
+                            full_tiles=tiles // 2 + 1)
+    assert_product_close(f32(Y3), A, W, path, C=C, what=f"{path} tile {tile_n} split {splits}, two launches")
     assert spl.spl_get_device_status() == 0
 
 
