@@ -223,63 +223,75 @@ class MaskedLayer:
             if timer:
                 timer("end", "precompute", g.name)
 
-    def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None, device_base=False):
+    def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None, device_base=False,
+               group_hooks=None):
         """a3 + a5 + a6 for draw d: regenerate eta_d, mask, masked product with fused unmask.
 
         inputs: {group: X [M, K]}.  Returns {group: Y [M, N_group]} (views of the layer's buffers).
+        group_hooks: (before(gi, name), after(gi, name)) called around each group's calls (e.g. to
+        wait for its input copy and to start copying its result out).
         """
         M = self.M
         out = {}
         for gi, g in enumerate(self.groups):
-            b = self.bank[g.name]
-            off, off_dev = self._offset(gi, g, cycle, d, device_base)
-            fp64 = g.name in self.fp64
-            xs = b.get("xs") if self._fused_split(g, path, M) else None
-            if self._fused_mask(g, path, M):
-                if timer:
-                    timer("begin", "masked_linear_unmask", g.name)
-                spl.spl_noise_mask_linear_unmask(b["Y"], b["xt"], inputs[g.name], g.wt, b["C"][d * M:(d + 1) * M],
-                                                 self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off,
-                                                 path=self.path_of(g, path, M), workspace=self.workspace,
-                                                 stream=stream, offset_dev=off_dev)
-                if timer:
-                    timer("end", "masked_linear_unmask", g.name)
-                out[g.name] = b["Y"]
-                continue
-            if fp64:
-                spl.spl_noise_mask_f64(b["xt"], inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
-                                       offset=off, stream=stream, offset_dev=off_dev)
-            elif xs is not None:
-                spl.spl_noise_mask_split(b["xt"], xs.f16_hi, xs.f16_lo, xs.f16_exp, inputs[g.name], self.deltas[g.name],
-                                         eps, mech, seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
-            else:
-                spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
-                                   offset=off, stream=stream, offset_dev=off_dev)
+            if group_hooks:
+                group_hooks[0](gi, g.name)
+            self._online_group(gi, g, inputs, eps, mech, seed, cycle, d, path, stream, timer, device_base, out)
+            if group_hooks:
+                group_hooks[1](gi, g.name)
+        return out
+
+    def _online_group(self, gi, g, inputs, eps, mech, seed, cycle, d, path, stream, timer, device_base, out):
+        M = self.M
+        b = self.bank[g.name]
+        off, off_dev = self._offset(gi, g, cycle, d, device_base)
+        fp64 = g.name in self.fp64
+        xs = b.get("xs") if self._fused_split(g, path, M) else None
+        if self._fused_mask(g, path, M):
             if timer:
                 timer("begin", "masked_linear_unmask", g.name)
-            if fp64:
-                spl.spl_masked_linear_unmask_f64(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M],
-                                                 workspace=self.workspace, stream=stream)
-            elif xs is not None:
-                spl.spl_masked_linear_unmask_split(b["Y"], xs, g.wt, b["C"][d * M:(d + 1) * M],
-                                                   path=self.path_of(g, path, M), workspace=self.workspace,
-                                                   stream=stream)
-            else:
-                spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M],
-                                             path=self.path_of(g, path, M), workspace=self.workspace, stream=stream)
+            spl.spl_noise_mask_linear_unmask(b["Y"], b["xt"], inputs[g.name], g.wt, b["C"][d * M:(d + 1) * M],
+                                             self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off,
+                                             path=self.path_of(g, path, M), workspace=self.workspace,
+                                             stream=stream, offset_dev=off_dev)
             if timer:
                 timer("end", "masked_linear_unmask", g.name)
             out[g.name] = b["Y"]
-        return out
+            return
+        if fp64:
+            spl.spl_noise_mask_f64(b["xt"], inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
+                                   offset=off, stream=stream, offset_dev=off_dev)
+        elif xs is not None:
+            spl.spl_noise_mask_split(b["xt"], xs.f16_hi, xs.f16_lo, xs.f16_exp, inputs[g.name], self.deltas[g.name],
+                                     eps, mech, seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
+        else:
+            spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
+                               offset=off, stream=stream, offset_dev=off_dev)
+        if timer:
+            timer("begin", "masked_linear_unmask", g.name)
+        if fp64:
+            spl.spl_masked_linear_unmask_f64(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M],
+                                             workspace=self.workspace, stream=stream)
+        elif xs is not None:
+            spl.spl_masked_linear_unmask_split(b["Y"], xs, g.wt, b["C"][d * M:(d + 1) * M],
+                                               path=self.path_of(g, path, M), workspace=self.workspace,
+                                               stream=stream)
+        else:
+            spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M],
+                                         path=self.path_of(g, path, M), workspace=self.workspace, stream=stream)
+        if timer:
+            timer("end", "masked_linear_unmask", g.name)
+        out[g.name] = b["Y"]
 
-    def capture(self, inputs, eps, mech, seed, path="auto", timer=None, before=None, after=None):
+    def capture(self, inputs, eps, mech, seed, path="auto", timer=None, before=None, after=None, group_hooks=None):
         """CUDA graphs of the ``draws`` steps of one bank cycle: graph d runs online step d (graph 0
         refills the bank first); the last graph moves every group's Philox base on by one cycle.
         Replay graphs[s % draws] for step s after set_cycle(s // draws) -- the graphs read their
         offsets on the device, so they replay cycle after cycle.  ``before(d)`` / ``after(d)`` run
         inside the capture around the step (host-to-device input copies, device-to-host result
-        copies).  Every library call must have run once before (warm-up), so nothing is set up
-        during capture.  Returns the graphs and the number of library kernels in each."""
+        copies), ``group_hooks`` around each group's calls (see online).  Every library call must
+        have run once before (warm-up), so nothing is set up during capture.  Returns the graphs and
+        the number of library kernels in each."""
         graphs, launches = [], []
         for d in range(self.draws):
             graph = torch.cuda.CUDAGraph()
@@ -289,7 +301,8 @@ class MaskedLayer:
                     before(d)
                 if d == 0:
                     self.refill(eps, mech, seed, 0, path=path, timer=timer, device_base=True)
-                self.online(inputs, eps, mech, seed, 0, d, path=path, timer=timer, device_base=True)
+                self.online(inputs, eps, mech, seed, 0, d, path=path, timer=timer, device_base=True,
+                            group_hooks=group_hooks)
                 if after:
                     after(d)
                 if d == self.draws - 1:
