@@ -145,7 +145,7 @@ struct MaskNoise {
   float* xt;                   // [M, K] X~ out
   float b;                     // scale Delta f / eps (0: eps = inf, no noise)
   int mech;                    // spl_mech
-  uint32_t k0, k1, s0, s1;     // Philox key, counter words 2-3
+  uint64_t seed, stream_id;    // Philox key, counter words 2-3
   uint64_t offset;             // Philox block offset (host part)
   const uint64_t* offset_dev;  // device part of the offset (may be null)
 };

@@ -29,7 +29,7 @@ constexpr int kThreads = 256;
 template <int MECH>
 __global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* __restrict__ nout,
                                                               const float* x, int64_t n, float b,
-                                                              uint32_t k0, uint32_t k1, uint32_t s0, uint32_t s1,
+                                                              const __grid_constant__ PhiloxKey key,
                                                               uint64_t offset_host, const uint64_t* offset_dev) {
   pdl_wait();
   pdl_trigger();
@@ -47,8 +47,8 @@ __global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* 
       xa = __ldcs(x4 + i);
       xb = __ldcs(x4 + i + stride);
     }
-    const float4 ea = draw_block<MECH>((uint64_t)i + offset, k0, k1, s0, s1, b);
-    const float4 eb = draw_block<MECH>((uint64_t)(i + stride) + offset, k0, k1, s0, s1, b);
+    const float4 ea = draw_block<MECH>((uint64_t)i + offset, key, b);
+    const float4 eb = draw_block<MECH>((uint64_t)(i + stride) + offset, key, b);
     if (nout) {
       __stcs(n4 + i, ea);
       __stcs(n4 + i + stride, eb);
@@ -59,14 +59,14 @@ __global__ void __launch_bounds__(kThreads) noise_mask_kernel(float* xt, float* 
     }
   }
   for (; i < nb_full; i += stride) {
-    const float4 e = draw_block<MECH>((uint64_t)i + offset, k0, k1, s0, s1, b);
+    const float4 e = draw_block<MECH>((uint64_t)i + offset, key, b);
     if (nout) __stcs(n4 + i, e);
     if (xt) __stcs(xt4 + i, add4(__ldcs(x4 + i), e));
   }
   // ragged tail: the last, partial Philox block
   if (blockIdx.x == 0 && threadIdx.x == 0 && (n & 3)) {
     const int64_t j = nb_full;
-    const float4 e = draw_block<MECH>((uint64_t)j + offset, k0, k1, s0, s1, b);
+    const float4 e = draw_block<MECH>((uint64_t)j + offset, key, b);
     const float ev[4] = {e.x, e.y, e.z, e.w};
     for (int l = 0; l < (int)(n & 3); ++l) {
       const int64_t idx = 4 * j + l;
@@ -86,8 +86,7 @@ __global__ void rng_advance_kernel(uint64_t* offset_dev, uint64_t delta) {
 // one rounding of at most 2^-53 |xt| (none at all while the exponents of x and eta are within 29).
 template <int MECH>
 __global__ void __launch_bounds__(kThreads) noise_mask_f64_kernel(double* __restrict__ xt, const float* __restrict__ x,
-                                                                  int64_t n, float b, uint32_t k0, uint32_t k1,
-                                                                  uint32_t s0, uint32_t s1, uint64_t offset_host,
+                                                                  int64_t n, float b, const __grid_constant__ PhiloxKey key, uint64_t offset_host,
                                                                   const uint64_t* offset_dev) {
   pdl_wait();
   pdl_trigger();
@@ -95,7 +94,7 @@ __global__ void __launch_bounds__(kThreads) noise_mask_f64_kernel(double* __rest
   const int64_t nb = (n + 3) >> 2;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
-    const float4 e = draw_block<MECH>((uint64_t)i + offset, k0, k1, s0, s1, b);
+    const float4 e = draw_block<MECH>((uint64_t)i + offset, key, b);
     const float ev[4] = {e.x, e.y, e.z, e.w};
     if (4 * i + 3 < n) {
       const float4 xv = __ldcs(reinterpret_cast<const float4*>(x) + i);
@@ -122,8 +121,7 @@ __device__ __forceinline__ float slalom_mask1(float x, uint32_t lo, uint32_t hi,
 }
 
 __global__ void __launch_bounds__(kThreads) slalom_mask_kernel(float* __restrict__ xt, float* __restrict__ eta,
-                                                               const float* __restrict__ x, int64_t n, uint32_t k0,
-                                                               uint32_t k1, uint32_t s0, uint32_t s1,
+                                                               const float* __restrict__ x, int64_t n, const __grid_constant__ PhiloxKey key,
                                                                uint64_t offset) {
   pdl_wait();
   pdl_trigger();
@@ -131,7 +129,7 @@ __global__ void __launch_bounds__(kThreads) slalom_mask_kernel(float* __restrict
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
     const uint64_t j = (uint64_t)i + offset;
-    const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
+    const uint4 r = philox_block(j, key);
     const int64_t e = 2 * i;
     xt[e] = slalom_mask1(x[e], r.x, r.y, eta ? eta + e : nullptr);
     if (e + 1 < n) xt[e + 1] = slalom_mask1(x[e + 1], r.z, r.w, eta ? eta + e + 1 : nullptr);
@@ -148,8 +146,7 @@ __global__ void __launch_bounds__(kThreads) slalom_quantize_kernel(float* __rest
 }
 
 // The raw Philox words of the stream (element e = lane e % 4 of block e / 4 + offset).
-__global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restrict__ out, int64_t n, uint32_t k0,
-                                                               uint32_t k1, uint32_t s0, uint32_t s1,
+__global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restrict__ out, int64_t n, const __grid_constant__ PhiloxKey key,
                                                                uint64_t offset_host, const uint64_t* offset_dev) {
   pdl_wait();
   pdl_trigger();
@@ -158,7 +155,7 @@ __global__ void __launch_bounds__(kThreads) random_bits_kernel(uint32_t* __restr
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nb; i += stride) {
     const uint64_t j = (uint64_t)i + offset;
-    const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
+    const uint4 r = philox_block(j, key);
     if (4 * i + 3 < n) {
       reinterpret_cast<uint4*>(out)[i] = r;
     } else {
@@ -283,8 +280,7 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
                                                                    uint16_t* __restrict__ lo,
                                                                    int* __restrict__ row_exp,
                                                                    const float* __restrict__ src, int64_t cols,
-                                                                   float* __restrict__ xt_out, float b, uint32_t k0,
-                                                                   uint32_t k1, uint32_t s0, uint32_t s1,
+                                                                   float* __restrict__ xt_out, float b, const __grid_constant__ PhiloxKey key,
                                                                    uint64_t offset_host, const uint64_t* offset_dev) {
   pdl_wait();
   pdl_trigger();
@@ -311,8 +307,8 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
       const int64_t i = threadIdx.x + (int64_t)c * kThreads;
       if (i >= n8) break;
       const uint64_t j = j0 + 2 * (uint64_t)i;
-      v[2 * c] = add4(v[2 * c], draw_block<MECH>(j, k0, k1, s0, s1, b));
-      v[2 * c + 1] = add4(v[2 * c + 1], draw_block<MECH>(j + 1, k0, k1, s0, s1, b));
+      v[2 * c] = add4(v[2 * c], draw_block<MECH>(j, key, b));
+      v[2 * c + 1] = add4(v[2 * c + 1], draw_block<MECH>(j + 1, key, b));
       if (xt_out) {
         float4* o = reinterpret_cast<float4*>(xt_out + r * cols);
         __stcs(o + 2 * i, v[2 * c]);
@@ -364,17 +360,13 @@ spl_status launch_noise_mask(float* xt, float* nout, const float* x, int64_t n, 
   if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
   const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
   const int grid = grid_for(ceil_div(n, 4), 8);
-  const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
-  const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
+  const PhiloxKey key = make_philox_key(rng.seed, rng.stream_id);
   if (b == 0.0f) {
-    return launch_pdl(noise_mask_kernel<kZero>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, k0, k1, s0,
-                      s1, rng.offset, rng.offset_dev);
+    return launch_pdl(noise_mask_kernel<kZero>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, key, rng.offset, rng.offset_dev);
   } else if (mech == SPL_MECH_LAPLACE) {
-    return launch_pdl(noise_mask_kernel<kLaplace>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, k0, k1, s0,
-                      s1, rng.offset, rng.offset_dev);
+    return launch_pdl(noise_mask_kernel<kLaplace>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, key, rng.offset, rng.offset_dev);
   } else {
-    return launch_pdl(noise_mask_kernel<kGaussian>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, k0, k1, s0,
-                      s1, rng.offset, rng.offset_dev);
+    return launch_pdl(noise_mask_kernel<kGaussian>, dim3(grid), dim3(kThreads), 0, stream, xt, nout, x, n, b, key, rng.offset, rng.offset_dev);
   }
 }
 
@@ -395,20 +387,19 @@ spl_status launch_split_rows(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const
                              int64_t cols, float* xt_out, float b, const spl_rng& rng, cudaStream_t stream) {
   const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
   const dim3 grid((unsigned)rows), block(kThreads);
-  const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
-  const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
+  const PhiloxKey key = make_philox_key(rng.seed, rng.stream_id);
   if (per_thread <= 1)
     return launch_pdl(split_fp16_regs_kernel<1, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev);
   if (per_thread <= 2)
     return launch_pdl(split_fp16_regs_kernel<2, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev);
   if (per_thread <= 4)
     return launch_pdl(split_fp16_regs_kernel<4, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev);
   if (per_thread <= 8)
     return launch_pdl(split_fp16_regs_kernel<8, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      k0, k1, s0, s1, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev);
   if (MECH != kNoMask) return SPL_ESHAPE;
   return launch_pdl(split_fp16_kernel, grid, block, 0, stream, hi, lo, row_exp, src, cols);
 }
@@ -459,8 +450,7 @@ extern "C" spl_status spl_random_bits(uint32_t* out, int64_t count, spl_rng rng,
   if (!out) return SPL_EINVAL;
   if (!aligned16(out)) return SPL_EALIGN;
   return launch_pdl(random_bits_kernel, dim3(grid_for(ceil_div(count, 4), 8)), dim3(kThreads), 0, stream, out, count,
-                    (uint32_t)rng.seed, (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id,
-                    (uint32_t)(rng.stream_id >> 32), rng.offset, rng.offset_dev);
+                    make_philox_key(rng.seed, rng.stream_id), rng.offset, rng.offset_dev);
 }
 
 extern "C" spl_status spl_rng_advance(uint64_t* offset_dev, uint64_t delta, cudaStream_t stream) {
@@ -492,16 +482,12 @@ extern "C" spl_status spl_noise_mask_f64(double* Xt, const float* X, int64_t row
   if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
   const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
   const int grid = grid_for(ceil_div(n, 4), 8);
-  const uint32_t k0 = (uint32_t)rng.seed, k1 = (uint32_t)(rng.seed >> 32);
-  const uint32_t s0 = (uint32_t)rng.stream_id, s1 = (uint32_t)(rng.stream_id >> 32);
+  const PhiloxKey key = make_philox_key(rng.seed, rng.stream_id);
   if (b == 0.0f)
-    return launch_pdl(noise_mask_f64_kernel<kZero>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, k0, k1, s0, s1,
-                      rng.offset, rng.offset_dev);
+    return launch_pdl(noise_mask_f64_kernel<kZero>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, key, rng.offset, rng.offset_dev);
   if (mech == SPL_MECH_LAPLACE)
-    return launch_pdl(noise_mask_f64_kernel<kLaplace>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, k0, k1, s0,
-                      s1, rng.offset, rng.offset_dev);
-  return launch_pdl(noise_mask_f64_kernel<kGaussian>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, k0, k1, s0,
-                    s1, rng.offset, rng.offset_dev);
+    return launch_pdl(noise_mask_f64_kernel<kLaplace>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, key, rng.offset, rng.offset_dev);
+  return launch_pdl(noise_mask_f64_kernel<kGaussian>, dim3(grid), dim3(kThreads), 0, stream, Xt, X, n, b, key, rng.offset, rng.offset_dev);
 }
 
 extern "C" spl_status spl_slalom_mask(float* Xt, float* eta, const float* X, int64_t rows, int64_t cols, spl_rng rng,
@@ -512,8 +498,8 @@ extern "C" spl_status spl_slalom_mask(float* Xt, float* eta, const float* X, int
   if (!Xt || !X) return SPL_EINVAL;
   if (rng.offset_dev) return SPL_EINVAL;  // host offsets only
   const int grid = grid_for(ceil_div(n, 2), 8);
-  return launch_pdl(slalom_mask_kernel, dim3(grid), dim3(kThreads), 0, stream, Xt, eta, X, n, (uint32_t)rng.seed,
-                    (uint32_t)(rng.seed >> 32), (uint32_t)rng.stream_id, (uint32_t)(rng.stream_id >> 32), rng.offset);
+  return launch_pdl(slalom_mask_kernel, dim3(grid), dim3(kThreads), 0, stream, Xt, eta, X, n,
+                    make_philox_key(rng.seed, rng.stream_id), rng.offset);
 }
 
 extern "C" spl_status spl_slalom_quantize(float* out, const float* v, int64_t count, cudaStream_t stream) {

@@ -43,8 +43,9 @@ constexpr int kMaxKs = kXsBytes / (4 * kGemvMaxM) / kSliceAlign * kSliceAlign;  
 // Rows per lane: 4 while the accumulators are few (MT <= 2), else 2 (RQ x MT accumulators).
 __host__ __device__ constexpr int rows_per_lane(int mt) { return mt <= 2 ? 4 : 2; }
 __host__ __device__ constexpr int rows_per_block(int mt) { return WARPS * 4 * rows_per_lane(mt); }
-// Steps of 32 per unrolled iteration: 8 float4 loads of W in flight per lane per buffer.
-__host__ __device__ constexpr int unroll_steps(int mt) { return 8 / rows_per_lane(mt); }
+// Steps of 32 per unrolled iteration: 8 float4 loads of W in flight per lane per buffer, but 4 at 8
+// rows (then 80 registers give 3 blocks per SM instead of 2; measured faster at 8 rows, slower at 16).
+__host__ __device__ constexpr int unroll_steps(int mt) { return mt == 8 ? 2 : 8 / rows_per_lane(mt); }
 
 // Reduce-scatter over the 8 lanes of a quarter-warp (xor offsets 4, 2, 1).  While C >= 2 values
 // remain, the lane with bit O set keeps the upper half and sends the lower half; afterwards the
@@ -93,7 +94,7 @@ constexpr int kNoMask = -1;
 struct KernelNoise {
   float* xt;
   float b;
-  uint32_t k0, k1, s0, s1;
+  PhiloxKey key;
   uint64_t offset;
   const uint64_t* offset_dev;
 };
@@ -102,7 +103,7 @@ template <int MT, int MASK>
 __global__ void __launch_bounds__(THREADS)
 gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* __restrict__ W,
             const float* __restrict__ C, float* __restrict__ part, unsigned int* __restrict__ counters, int M,
-            int64_t K, int64_t N, int ks, int splits, int prefetch_lines, KernelNoise nz) {
+            int64_t K, int64_t N, int ks, int splits, int prefetch_lines, const __grid_constant__ KernelNoise nz) {
   constexpr int RQ = rows_per_lane(MT), RB = rows_per_block(MT), U = unroll_steps(MT);
   constexpr int V = RQ * MT;
   extern __shared__ __align__(16) float4 xs[];  // [MT][ks / 4]
@@ -164,7 +165,7 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
       for (int q = threadIdx.x; q < q_row; q += THREADS) {
         float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
         if (m < M && q < q_len) {
-          v = add4(__ldg(src + q), draw_block<MASK>(j0 + (uint64_t)q, nz.k0, nz.k1, nz.s0, nz.s1, nz.b));
+          v = add4(__ldg(src + q), draw_block<MASK>(j0 + (uint64_t)q, nz.key, nz.b));
           if (write_xt) __stcs(dst + q, v);
         }
         xs[m * q_row + q] = v;
@@ -403,7 +404,12 @@ spl_status run_gemv_masked(const LinearArgs& a, const Plan& p, const MaskNoise& 
   unsigned int* counters;
   spl_status st = scratch(a, p, &part, &counters);
   if (st != SPL_OK) return st;
-  const KernelNoise kn{nz.xt, nz.b, nz.k0, nz.k1, nz.s0, nz.s1, nz.offset, nz.offset_dev};
+  KernelNoise kn{};
+  kn.xt = nz.xt;
+  kn.b = nz.b;
+  kn.key = make_philox_key(nz.seed, nz.stream_id);
+  kn.offset = nz.offset;
+  kn.offset_dev = nz.offset_dev;
   if (nz.b == 0.0f) return launch_masked<kZero>(a, p, part, counters, kn);
   if (nz.mech == SPL_MECH_LAPLACE) return launch_masked<kLaplace>(a, p, part, counters, kn);
   return launch_masked<kGaussian>(a, p, part, counters, kn);

@@ -222,10 +222,8 @@ extern "C" spl_status spl_noise_mask_linear_unmask(float* Y, float* Xt, const fl
   nz.xt = Xt;
   nz.b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
   nz.mech = (int)mech;
-  nz.k0 = (uint32_t)rng.seed;
-  nz.k1 = (uint32_t)(rng.seed >> 32);
-  nz.s0 = (uint32_t)rng.stream_id;
-  nz.s1 = (uint32_t)(rng.stream_id >> 32);
+  nz.seed = rng.seed;
+  nz.stream_id = rng.stream_id;
   nz.offset = rng.offset;
   nz.offset_dev = rng.offset_dev;
   return run_linear(Y, X, W, C, true, M, K, N, path, workspace, workspace_bytes, stream, nullptr, &nz);

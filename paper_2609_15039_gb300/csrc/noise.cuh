@@ -17,16 +17,37 @@ constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;  // round multiplier for counter wor
 constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;  // key increment, word 0
 constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;  // key increment, word 1
 
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+// The round keys and counter words 2-3 of one (seed, stream_id), computed once on the host:
+// round r uses the key (lo(seed) + r W0, hi(seed) + r W1) mod 2^32.  A kernel receives them as a
+// __grid_constant__ parameter, so every round's key enters its XOR straight from the constant
+// bank, with no addition per round.
+struct PhiloxKey {
+  uint32_t k0[10], k1[10];
+  uint32_t s0, s1;
+};
+
+inline PhiloxKey make_philox_key(uint64_t seed, uint64_t stream_id) {
+  PhiloxKey k;
+  uint32_t a = (uint32_t)seed, b = (uint32_t)(seed >> 32);
+  for (int r = 0; r < 10; ++r) {
+    k.k0[r] = a;
+    k.k1[r] = b;
+    a += kPhiloxW0;
+    b += kPhiloxW1;
+  }
+  k.s0 = (uint32_t)stream_id;
+  k.s1 = (uint32_t)(stream_id >> 32);
+  return k;
+}
+
+// Philox4x32-10 of counter (lo j, hi j, s0, s1).
+__device__ __forceinline__ uint4 philox_block(uint64_t j, const PhiloxKey& key) {
+  uint4 c = make_uint4((uint32_t)j, (uint32_t)(j >> 32), key.s0, key.s1);
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
-    if (r > 0) {
-      k0 += kPhiloxW0;
-      k1 += kPhiloxW1;
-    }
     const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
     const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    c = make_uint4(hi1 ^ c.y ^ key.k0[r], lo1, hi0 ^ c.w ^ key.k1[r], lo0);
   }
   return c;
 }
@@ -77,10 +98,9 @@ __device__ __forceinline__ void gauss2(uint32_t ra, uint32_t rb, float b, float&
 }
 
 template <int MECH>
-__device__ __forceinline__ float4 draw_block(uint64_t j, uint32_t k0, uint32_t k1, uint32_t s0,
-                                             uint32_t s1, float b) {
+__device__ __forceinline__ float4 draw_block(uint64_t j, const PhiloxKey& key, float b) {
   if (MECH == kZero) return make_float4(0.f, 0.f, 0.f, 0.f);
-  const uint4 r = philox4x32_10(make_uint4((uint32_t)j, (uint32_t)(j >> 32), s0, s1), k0, k1);
+  const uint4 r = philox_block(j, key);
   float4 e;
   if (MECH == kLaplace) {
     e = make_float4(laplace1(r.x, b), laplace1(r.y, b), laplace1(r.z, b), laplace1(r.w, b));

@@ -165,9 +165,9 @@ class MaskedLayer:
                 "xt": torch.empty((M, g.K), device=dev, dtype=wide),
                 "Y": torch.empty((M, g.N), device=dev),
             }
-            if self._fused_split(g, path, M):  # X~ with its fp16 split, written by the mask kernel
+            if self._fused_split(g, path, M):  # the fp16 split of X~, written by the mask kernel
                 b = self.bank[g.name]
-                b["xs"] = spl.Weight(b["xt"], f16_hi=torch.empty((M, g.K), dtype=torch.int16, device=dev),
+                b["xs"] = spl.Weight(None, f16_hi=torch.empty((M, g.K), dtype=torch.int16, device=dev),
                                      f16_lo=torch.empty((M, g.K), dtype=torch.int16, device=dev),
                                      f16_exp=torch.empty(M, dtype=torch.int32, device=dev))
 
@@ -261,8 +261,8 @@ class MaskedLayer:
         if fp64:
             spl.spl_noise_mask_f64(b["xt"], inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
                                    offset=off, stream=stream, offset_dev=off_dev)
-        elif xs is not None:
-            spl.spl_noise_mask_split(b["xt"], xs.f16_hi, xs.f16_lo, xs.f16_exp, inputs[g.name], self.deltas[g.name],
+        elif xs is not None:  # the FP16X3 product reads only the split: X~ itself is not written
+            spl.spl_noise_mask_split(None, xs.f16_hi, xs.f16_lo, xs.f16_exp, inputs[g.name], self.deltas[g.name],
                                      eps, mech, seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
         else:
             spl.spl_noise_mask(b["xt"], None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
@@ -319,9 +319,15 @@ class MaskedLayer:
         res = {}
         for gi, g in enumerate(self.groups):
             eta = torch.empty((self.M, g.K), device=g.W.device)
-            spl.spl_noise(eta, self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=self.block_offset(g, cycle, d))
-            xt = self.bank[g.name]["xt"]
-            res[g.name] = spl.spl_bound_check(outs[g.name], inputs[g.name], xt.float().contiguous(), eta, g.W)
+            off = self.block_offset(g, cycle, d)
+            spl.spl_noise(eta, self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off)
+            if g.name in self.fp64:
+                xt = self.bank[g.name]["xt"].float().contiguous()
+            else:  # the step's X~, drawn again (online steps that feed the split do not keep it)
+                xt = torch.empty_like(eta)
+                spl.spl_noise_mask(xt, None, inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
+                                   offset=off)
+            res[g.name] = spl.spl_bound_check(outs[g.name], inputs[g.name], xt, eta, g.W)
         return res
 
     def flops_per_step(self):
