@@ -54,9 +54,36 @@ __device__ __forceinline__ uint4 philox_block(uint64_t j, const PhiloxKey& key) 
 
 enum { kLaplace = 0, kGaussian = 1, kZero = 2 };
 
+// ln u for u = k 2^-24, k = 1 .. 2^24: u = 2^e m with m in [sqrt(1/2), sqrt(2)) and s = m - 1
+// (both exact), ln(1 + s) = s P(s) with P of degree 9 fitted to the relative error on that interval
+// (least squares on Chebyshev nodes, then Lawson's reweighting toward the minimax), and
+// ln u = e ln 2 + s P(s).  At most 1.6 ulp from ln u over all 2^24 inputs (checked against
+// binary64), and exact (0) at u = 1.
+__device__ __forceinline__ float log_unit(float u) {
+  const int bits = __float_as_int(u);
+  int e = (bits >> 23) - 127;
+  float m = __int_as_float((bits & 0x7FFFFF) | 0x3F800000);
+  if (m > 1.41421356f) {
+    m = __fmul_rn(m, 0.5f);
+    e += 1;
+  }
+  const float s = __fsub_rn(m, 1.0f);
+  float p = -0.07830669730901718f;
+  p = fmaf(p, s, 0.13019075989723206f);
+  p = fmaf(p, s, -0.13212285935878754f);
+  p = fmaf(p, s, 0.1416073590517044f);
+  p = fmaf(p, s, -0.16610340774059296f);
+  p = fmaf(p, s, 0.2000320553779602f);
+  p = fmaf(p, s, -0.2500157058238983f);
+  p = fmaf(p, s, 0.33333301544189453f);
+  p = fmaf(p, s, -0.49999988079071045f);
+  p = fmaf(p, s, 1.0f);
+  return fmaf((float)e, 0.6931471824645996f, __fmul_rn(p, s));
+}
+
 __device__ __forceinline__ float laplace1(uint32_t r, float b) {
   const float u = __int2float_rn((int)((r & 0xFFFFFFu) + 1u)) * 0x1p-24f;  // (0, 1], exact
-  const float mag = __fmul_rn(b, -logf(u));
+  const float mag = __fmul_rn(b, -log_unit(u));
   return (r >> 31) ? -mag : mag;
 }
 
@@ -89,7 +116,7 @@ __device__ __forceinline__ void sincospi_turns(float x, float* s, float* c) {
 __device__ __forceinline__ void gauss2(uint32_t ra, uint32_t rb, float b, float& ea, float& eb) {
   const float u1 = __int2float_rn((int)((ra >> 8) + 1u)) * 0x1p-24f;  // (0, 1]
   const float u2 = __int2float_rn((int)(rb >> 8)) * 0x1p-24f;         // [0, 1)
-  const float R = sqrtf(__fmul_rn(-2.0f, logf(u1)));
+  const float R = sqrtf(__fmul_rn(-2.0f, log_unit(u1)));
   float s, c;
   sincospi_turns(2.0f * u2, &s, &c);  // sin/cos of 2 pi u2; 2*u2 is exact
   const float sr = __fmul_rn(b, R);
