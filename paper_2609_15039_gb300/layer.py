@@ -289,9 +289,10 @@ class MaskedLayer:
         Replay graphs[s % draws] for step s after set_cycle(s // draws) -- the graphs read their
         offsets on the device, so they replay cycle after cycle.  ``before(d)`` / ``after(d)`` run
         inside the capture around the step (host-to-device input copies, device-to-host result
-        copies), ``group_hooks`` around each group's calls (see online).  Every library call must
-        have run once before (warm-up), so nothing is set up during capture.  Returns the graphs and
-        the number of library kernels in each."""
+        copies), ``group_hooks`` around each group's calls (see online).  ``inputs`` may be a list
+        of input dicts: graph d then reads inputs[d % len(inputs)].  Every library call must have run
+        once before (warm-up), so nothing is set up during capture.  Returns the graphs and the
+        number of library kernels in each."""
         graphs, launches = [], []
         for d in range(self.draws):
             graph = torch.cuda.CUDAGraph()
@@ -301,7 +302,8 @@ class MaskedLayer:
                     before(d)
                 if d == 0:
                     self.refill(eps, mech, seed, 0, path=path, timer=timer, device_base=True)
-                self.online(inputs, eps, mech, seed, 0, d, path=path, timer=timer, device_base=True,
+                inp = inputs[d % len(inputs)] if isinstance(inputs, (list, tuple)) else inputs
+                self.online(inp, eps, mech, seed, 0, d, path=path, timer=timer, device_base=True,
                             group_hooks=group_hooks)
                 if after:
                     after(d)
