@@ -136,9 +136,12 @@ spl_status spl_noise_mask(float* Xt, float* N_out, const float* X, int64_t rows,
 /* ---- a2 + a3 fused with the fp16 split of X~ ----------------------------
  * Draws eta exactly as spl_noise, forms Xt = fl32(X + eta) (written to Xt
  * unless it is NULL) and writes its FP16X3 split as spl_split_fp16 would:
- * hi, lo [rows, cols] binary16 and row_exp [rows].  One pass, one block per
- * row; cols % 8 == 0 and cols <= 16384 (EALIGN / ESHAPE otherwise).  The split
- * is what spl_masked_linear_unmask_split consumes.  Errors as spl_noise_mask. */
+ * hi, lo [rows, cols] binary16 and row_exp [rows].  With X NULL the split is
+ * that of eta itself (and Xt, if given, receives eta): a bank of noise draws
+ * split in one pass for spl_precompute_noise_product_matched_split.  One pass,
+ * one block per row; cols % 8 == 0 and cols <= 16384 (EALIGN / ESHAPE
+ * otherwise).  The split is what spl_masked_linear_unmask_split consumes.
+ * Errors as spl_noise_mask, except that X may be NULL. */
 spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,
                                 int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech,
                                 spl_rng rng, cudaStream_t stream);
@@ -296,6 +299,17 @@ spl_status spl_noise_mask_linear_unmask(float* Y, float* Xt, const float* X, con
                                         int64_t M, int64_t K, int64_t N, double sensitivity, double eps,
                                         spl_mech mech, spl_rng rng, spl_path path, void* workspace,
                                         size_t workspace_bytes, cudaStream_t stream);
+
+/* ---- a4 with the noise already split ------------------------------------
+ * As spl_precompute_noise_product_matched, with the noise given as a
+ * descriptor: Nz->w the fp32 noise (may be NULL when the call runs FP16X3) and
+ * Nz->f16_hi / f16_lo / f16_exp its fp16 split (from spl_noise_mask_split with
+ * X NULL).  On the FP16X3 path the tensor-core kernel reads the split and skips
+ * its own split pass; other paths read Nz->w (EINVAL if it is NULL).  The
+ * result equals spl_precompute_noise_product_matched's bit for bit. */
+spl_status spl_precompute_noise_product_matched_split(float* C, const spl_weight* Nz, const spl_weight* W, int64_t M,
+                                                      int64_t K, int64_t N, int64_t order_rows, spl_path path,
+                                                      void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- a5 + a6 for decode, without allocation ---------------------------
  * The paper has no counterpart to this call; it exists for callers that

@@ -286,13 +286,14 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
   pdl_trigger();
   __shared__ float warp_max[kThreads / 32];
   const int64_t r = blockIdx.x;
-  const float4* row = reinterpret_cast<const float4*>(src + r * cols);
+  // src NULL (with a mechanism): the row is the noise alone
+  const float4* row = src ? reinterpret_cast<const float4*>(src + r * cols) : nullptr;
   const int64_t n8 = cols >> 3;
   float4 v[2 * CH];
 #pragma unroll
   for (int c = 0; c < CH; ++c) {
     const int64_t i = threadIdx.x + (int64_t)c * kThreads;
-    if (i < n8) {
+    if (row && i < n8) {
       v[2 * c] = __ldg(row + 2 * i);
       v[2 * c + 1] = __ldg(row + 2 * i + 1);
     } else {
@@ -307,8 +308,9 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
       const int64_t i = threadIdx.x + (int64_t)c * kThreads;
       if (i >= n8) break;
       const uint64_t j = j0 + 2 * (uint64_t)i;
-      v[2 * c] = add4(v[2 * c], draw_block<MECH>(j, key, b));
-      v[2 * c + 1] = add4(v[2 * c + 1], draw_block<MECH>(j + 1, key, b));
+      const float4 e0 = draw_block<MECH>(j, key, b), e1 = draw_block<MECH>(j + 1, key, b);
+      v[2 * c] = row ? add4(v[2 * c], e0) : e0;
+      v[2 * c + 1] = row ? add4(v[2 * c + 1], e1) : e1;
       if (xt_out) {
         float4* o = reinterpret_cast<float4*>(xt_out + r * cols);
         __stcs(o + 2 * i, v[2 * c]);
@@ -515,9 +517,9 @@ extern "C" spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo
   spl_status st = validate_noise(rows, cols, sensitivity, eps, mech);
   if (st != SPL_OK) return st;
   if (rows == 0 || cols == 0) return SPL_OK;
-  if (!X || !hi || !lo || !row_exp) return SPL_EINVAL;
+  if (!hi || !lo || !row_exp) return SPL_EINVAL;  // X NULL: the split of the noise itself
   if ((cols & 7) != 0) return SPL_EALIGN;
-  if (!aligned16(X) || !aligned16(hi) || !aligned16(lo) || (Xt && !aligned16(Xt))) return SPL_EALIGN;
+  if ((X && !aligned16(X)) || !aligned16(hi) || !aligned16(lo) || (Xt && !aligned16(Xt))) return SPL_EALIGN;
   if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
   if (rows > 0x7fffffffLL) return SPL_ESHAPE;
   const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);

@@ -242,30 +242,40 @@ extern "C" size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, i
   return need;
 }
 
-extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const spl_weight* W, int64_t M,
-                                                           int64_t K, int64_t N, int64_t order_rows, spl_path path,
-                                                           void* workspace, size_t workspace_bytes,
-                                                           cudaStream_t stream) {
+namespace spl {
+namespace {
+// The correction in the online order; A (may be NULL) carries the fp16 split of the noise.
+spl_status precompute_matched(float* C, const float* Nz, const spl_weight* A, const spl_weight* W, int64_t M,
+                              int64_t K, int64_t N, int64_t order_rows, spl_path path, void* workspace,
+                              size_t workspace_bytes, cudaStream_t stream) {
   if (order_rows <= 0) return SPL_EINVAL;
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
   if (!valid_path(path)) return SPL_EINVAL;
   if (M == 0 || N == 0 || K == 0)
-    return run_linear(C, Nz, W, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream);
-  if (!C || !Nz) return SPL_EINVAL;
+    return run_linear(C, Nz, W, nullptr, false, M, K, N, path, workspace, workspace_bytes, stream, A);
+  const bool a_split = A && A->f16_hi && A->f16_lo && A->f16_exp;
+  if (!C || (!Nz && !a_split)) return SPL_EINVAL;
   spl_status st = check_weight(W, K);
   if (st != SPL_OK) return st;
   if ((K & 3) != 0) return SPL_EALIGN;
-  if (!aligned16(C) || !aligned16(Nz)) return SPL_EALIGN;
+  if (!aligned16(C) || (Nz && !aligned16(Nz))) return SPL_EALIGN;
   const spl_path resolved = resolve(order_rows, K, path, has_tf32(*W), has_f16(*W));
   if (resolved == SPL_PATH_TF32X3 && (!has_tf32(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
   if (resolved == SPL_PATH_FP16X3 && (!has_f16(*W) || !tc_capable())) return SPL_EUNSUPPORTED;
   if (resolved == SPL_PATH_FP16X3 && (K & 7) != 0) return SPL_EALIGN;
+  const bool use_split = a_split && resolved == SPL_PATH_FP16X3;
+  if (!Nz && !use_split) return SPL_EINVAL;  // only FP16X3 reads the split alone
   const MatchedPlan mp = matched_plan(M, K, N, order_rows, resolved);
   if (!mp.ok)  // the masked call's order cannot be reproduced: plain correction
-    return run_linear(C, Nz, W, nullptr, false, M, K, N, resolved, workspace, workspace_bytes, stream);
+    return run_linear(C, Nz, W, nullptr, false, M, K, N, resolved, workspace, workspace_bytes, stream, A);
   if (mp.ws > 0 && (!workspace || workspace_bytes < mp.ws)) return SPL_EWORKSPACE;
   if (workspace && !aligned16(workspace)) return SPL_EALIGN;
-  const LinearArgs args = make_args(C, Nz, *W, nullptr, M, K, N, workspace, workspace_bytes, stream, resolved);
+  LinearArgs args = make_args(C, Nz, *W, nullptr, M, K, N, workspace, workspace_bytes, stream, resolved);
+  if (use_split) {
+    args.a_h16 = A->f16_hi;
+    args.a_l16 = A->f16_lo;
+    args.a_exp = A->f16_exp;
+  }
   if (mp.kernel == kKernelTc) return run_tc_segmented(args, mp.splits);
   Plan p{};
   p.kernel = mp.kernel;
@@ -284,4 +294,22 @@ extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float
     if (st != SPL_OK) return st;
   }
   return SPL_OK;
+}
+}  // namespace
+}  // namespace spl
+
+extern "C" spl_status spl_precompute_noise_product_matched(float* C, const float* Nz, const spl_weight* W, int64_t M,
+                                                           int64_t K, int64_t N, int64_t order_rows, spl_path path,
+                                                           void* workspace, size_t workspace_bytes,
+                                                           cudaStream_t stream) {
+  if (M > 0 && K > 0 && N > 0 && !Nz) return SPL_EINVAL;
+  return precompute_matched(C, Nz, nullptr, W, M, K, N, order_rows, path, workspace, workspace_bytes, stream);
+}
+
+extern "C" spl_status spl_precompute_noise_product_matched_split(float* C, const spl_weight* Nz, const spl_weight* W,
+                                                                 int64_t M, int64_t K, int64_t N, int64_t order_rows,
+                                                                 spl_path path, void* workspace,
+                                                                 size_t workspace_bytes, cudaStream_t stream) {
+  if (!Nz) return SPL_EINVAL;
+  return precompute_matched(C, Nz->w, Nz, W, M, K, N, order_rows, path, workspace, workspace_bytes, stream);
 }

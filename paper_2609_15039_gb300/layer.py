@@ -165,11 +165,14 @@ class MaskedLayer:
                 "xt": torch.empty((M, g.K), device=dev, dtype=wide),
                 "Y": torch.empty((M, g.N), device=dev),
             }
-            if self._fused_split(g, path, M):  # the fp16 split of X~, written by the mask kernel
+            if self._fused_split(g, path, M):  # the fp16 splits of X~ and of the bank's noise
                 b = self.bank[g.name]
                 b["xs"] = spl.Weight(None, f16_hi=torch.empty((M, g.K), dtype=torch.int16, device=dev),
                                      f16_lo=torch.empty((M, g.K), dtype=torch.int16, device=dev),
                                      f16_exp=torch.empty(M, dtype=torch.int32, device=dev))
+                b["es"] = spl.Weight(None, f16_hi=torch.empty((draws * M, g.K), dtype=torch.int16, device=dev),
+                                     f16_lo=torch.empty((draws * M, g.K), dtype=torch.int16, device=dev),
+                                     f16_exp=torch.empty(draws * M, dtype=torch.int32, device=dev))
 
     def _fused_split(self, g, path, M):
         """True when the online product of group g runs FP16X3: then the mask kernel also writes the
@@ -209,6 +212,18 @@ class MaskedLayer:
         for gi, g in enumerate(self.groups):
             b = self.bank[g.name]
             off, off_dev = self._offset(gi, g, cycle, 0, device_base)
+            es = b.get("es") if self._fused_split(g, path, self.M) else None
+            if es is not None:  # the FP16X3 correction reads only the split: the noise is split as drawn
+                spl.spl_noise_mask_split(None, es.f16_hi, es.f16_lo, es.f16_exp, None, self.deltas[g.name], eps, mech,
+                                         seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
+                if timer:
+                    timer("begin", "precompute", g.name)
+                spl.spl_precompute_noise_product_matched_split(b["C"], es, g.wt, self.M,
+                                                               path=self.path_of(g, path, self.M),
+                                                               workspace=self.workspace, stream=stream)
+                if timer:
+                    timer("end", "precompute", g.name)
+                continue
             spl.spl_noise(b["eta"], self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off, stream=stream,
                           offset_dev=off_dev)
             if timer:

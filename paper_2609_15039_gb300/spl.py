@@ -69,6 +69,7 @@ _SIGS = {
     "spl_precompute_noise_product": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_precompute_matched_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I64, _I]),
     "spl_precompute_noise_product_matched": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
+    "spl_precompute_noise_product_matched_split": (_I, [_P, _PW, _PW, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_masked_linear_unmask": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_masked_linear_unmask_noalloc": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P]),
@@ -240,8 +241,9 @@ def spl_masked_linear_unmask_f64(Y, Xt, W, C, workspace=None, stream=None):
 
 def spl_noise_mask_split(Xt, hi, lo, row_exp, X, sensitivity, eps, mech, seed, stream_id=0, offset=0, stream=None,
                          offset_dev=None):
-    """a2 + a3 + the fp16 split of X~ in one pass (Xt may be None)."""
-    rows, cols = _rows_cols(X)
+    """a2 + a3 + the fp16 split of X~ in one pass (Xt may be None; X None: the split of the noise
+    itself, of hi's shape)."""
+    rows, cols = _rows_cols(X if X is not None else hi)
     if hi.numel() != rows * cols or lo.numel() != rows * cols or row_exp.numel() != rows:
         raise ValueError("spl_noise_mask_split: shape mismatch")
     _check(lib().spl_noise_mask_split(_dev(Xt, "Xt"), _dev(hi, "hi", torch.int16), _dev(lo, "lo", torch.int16),
@@ -408,6 +410,20 @@ def spl_precompute_noise_product_matched(C, Nz, W, order_rows, path="auto", work
     _check(lib().spl_precompute_noise_product_matched(_dev(C, "C"), _dev(Nz, "Nz"), ctypes.byref(ws_), M, K, N,
                                                       int(order_rows), _path(path), wsp, wsb, _stream(stream)),
            "spl_precompute_noise_product_matched")
+
+
+def spl_precompute_noise_product_matched_split(C, Nz, W, order_rows, path="auto", workspace=None, stream=None):
+    """Nz: a Weight holding the noise (w, may be None on FP16X3) and its fp16 split."""
+    W = _weight(W)
+    M, K = Nz.shape
+    N = W.shape[0]
+    if W.shape[-1] != K or C.numel() != M * N:
+        raise ValueError("spl_precompute_noise_product_matched_split: shape mismatch")
+    wsp, wsb = _ws(workspace)
+    ns, ws_ = Nz.c_struct(), W.c_struct()
+    _check(lib().spl_precompute_noise_product_matched_split(_dev(C, "C"), ctypes.byref(ns), ctypes.byref(ws_), M, K, N,
+                                                            int(order_rows), _path(path), wsp, wsb, _stream(stream)),
+           "spl_precompute_noise_product_matched_split")
 
 
 def spl_unmask(Y, Yt, C, stream=None):

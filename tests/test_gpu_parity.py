@@ -463,6 +463,54 @@ def test_noise_mask_linear_unmask_equals_separate_calls(spl, M, K, N, mech, eps)
     assert e.value.status == spl.SPL_EINVAL
 
 
+@pytest.mark.parametrize("rows,cols,mech,eps", [(1024, 3072, "gaussian", 1.0), (37, 1032, "laplace", 0.5),
+                                                (8, 8192, "laplace", None)])
+def test_noise_split_is_the_split_of_the_noise(spl, rows, cols, mech, eps):
+    """With no input the fused kernel splits the noise itself: the same bits as spl_noise then
+    spl_split_fp16 (eps = inf: the split of zeros)."""
+    eta = torch.empty((rows, cols), device="cuda")
+    spl.spl_noise(eta, 825.3, eps, mech, seed=5, stream_id=3, offset=77)
+    hi_ref = torch.empty((rows, cols), dtype=torch.int16, device="cuda")
+    lo_ref, ex_ref = torch.empty_like(hi_ref), torch.empty(rows, dtype=torch.int32, device="cuda")
+    spl.spl_split_fp16(hi_ref, lo_ref, ex_ref, eta)
+    hi, lo, ex = torch.empty_like(hi_ref), torch.empty_like(lo_ref), torch.empty_like(ex_ref)
+    xt = torch.full((rows, cols), 3.0, device="cuda")
+    spl.spl_noise_mask_split(xt, hi, lo, ex, None, 825.3, eps, mech, seed=5, stream_id=3, offset=77)
+    assert torch.equal(hi, hi_ref) and torch.equal(lo, lo_ref) and torch.equal(ex, ex_ref)
+    assert torch.equal(xt, eta)  # X~ of no input is the noise
+
+
+@pytest.mark.parametrize("M,K,N,order", [(1024, 3072, 5120, 128), (1024, 8192, 3072, 128), (400, 1032, 600, 100),
+                                         (4096, 3072, 3072, 512)])
+def test_matched_correction_from_the_split_noise(spl, M, K, N, order):
+    """The bank's correction from the noise split as drawn equals the one from the fp32 noise, bit
+    for bit, and so the online order."""
+    W, Wt = _weights(spl, N, K, seed=K + N + 5)
+    eta = torch.empty((M, K), device="cuda")
+    spl.spl_noise(eta, 1443.0, 1.0, "gaussian", seed=29)
+    hi = torch.empty((M, K), dtype=torch.int16, device="cuda")
+    lo, ex = torch.empty_like(hi), torch.empty(M, dtype=torch.int32, device="cuda")
+    spl.spl_noise_mask_split(None, hi, lo, ex, None, 1443.0, 1.0, "gaussian", seed=29)
+    ws = spl.workspace(spl.spl_precompute_matched_workspace_bytes(M, K, N, order, "fp16x3"))
+    C_ref, C, C_w = (torch.empty((M, N), device="cuda") for _ in range(3))
+    spl.spl_precompute_noise_product_matched(C_ref, eta, Wt, order, path="fp16x3", workspace=ws)
+    spl.spl_precompute_noise_product_matched_split(C, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, order,
+                                                   path="fp16x3", workspace=ws)
+    assert torch.equal(C, C_ref)
+    # the FP32 path reads the fp32 noise of the descriptor
+    ws32 = spl.workspace(spl.spl_precompute_matched_workspace_bytes(M, K, N, 1, "fp32"))
+    C32_ref = torch.empty((M, N), device="cuda")
+    spl.spl_precompute_noise_product_matched(C32_ref, eta, Wt, 1, path="fp32", workspace=ws32)
+    spl.spl_precompute_noise_product_matched_split(C_w, spl.Weight(eta, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, 1,
+                                                   path="fp32", workspace=ws32)
+    assert torch.equal(C_w, C32_ref)
+    with pytest.raises(spl.SplError) as e:  # ... and refuses a descriptor without it
+        spl.spl_precompute_noise_product_matched_split(C_w, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, 1,
+                                                       path="fp32", workspace=ws32)
+    assert e.value.status == spl.SPL_EINVAL
+    assert spl.spl_get_device_status() == 0
+
+
 @pytest.mark.parametrize("M,K,N", [(128, 3072, 3072), (130, 1032, 600), (512, 3072, 5120), (9, 256, 512)])
 def test_presplit_product_equals_plain(spl, M, K, N):
     W, Wt = _weights(spl, N, K, seed=N + 3)
@@ -725,7 +773,9 @@ def test_config_llama_layer(spl, llama_layer, eps):
     inputs_np = {g: wl.activations(M, K, seed=100 + gi).numpy() for gi, (g, K, _n) in enumerate(model.input_groups())}
     inputs = {g: dev(x) for g, x in inputs_np.items()}
     layer.refill(eps, mech, seed, cycle=3)
-    bank_eta = {g.name: layer.bank[g.name]["eta"].clone() for g in layer.groups}
+    # the bank keeps the noise (or, for an FP16X3 group, only its fp16 split)
+    bank = {g.name: (layer.bank[g.name]["es"].f16_hi.clone() if "es" in layer.bank[g.name]
+                     else layer.bank[g.name]["eta"].clone()) for g in layer.groups}
     for d in range(draws):
         outs = split_outputs(layer, layer.online(inputs, eps, mech, seed, cycle=3, d=d))
         torch.cuda.synchronize()
@@ -735,7 +785,13 @@ def test_config_llama_layer(spl, llama_layer, eps):
             xt = torch.empty((M, g.K), device="cuda")
             spl.spl_noise_mask(xt, regen, inputs[g.name], deltas[g.name], eps, mech, seed, stream_id=gi,
                                    offset=layer.block_offset(g, 3, d))
-            assert torch.equal(regen, bank_eta[g.name][d * M:(d + 1) * M])
+            if "es" in layer.bank[g.name]:
+                hi, lo = torch.empty((M, g.K), dtype=torch.int16, device="cuda"), None
+                lo, ex = torch.empty_like(hi), torch.empty(M, dtype=torch.int32, device="cuda")
+                spl.spl_split_fp16(hi, lo, ex, regen)
+                assert torch.equal(hi, bank[g.name][d * M:(d + 1) * M])
+            else:
+                assert torch.equal(regen, bank[g.name][d * M:(d + 1) * M])
             X = inputs_np[g.name]
             n_or = philox.noise((M, g.K), deltas[g.name], eps, mech, seed, stream_id=gi,
                                 offset=layer.block_offset(g, 3, d))
