@@ -47,6 +47,34 @@ __host__ __device__ constexpr int rows_per_block(int mt) { return WARPS * 4 * ro
 // rows (then 80 registers give 3 blocks per SM instead of 2; measured faster at 8 rows, slower at 16).
 __host__ __device__ constexpr int unroll_steps(int mt) { return mt == 8 ? 2 : 8 / rows_per_lane(mt); }
 
+// Packed pairs of fp32 (two rows of X~): one fma.rn.f32x2 does the two round-to-nearest FMAs the
+// scalar loop would, so the sums are the same bit for bit with half the FMA instructions.
+__device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpack2(unsigned long long v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b,
+                                                    unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ void lds_v2b64(uint32_t addr, unsigned long long& a, unsigned long long& b) {
+  asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(addr));
+}
+
+// Paired layout of the staged X~ (MT >= 4): rows 2p and 2p + 1 interleaved, and within each step of
+// 32 columns the 16-byte group that lane i reads first holds columns 4i, 4i + 1 of both rows and
+// the second one columns 4i + 2, 4i + 3: a quarter-warp reads 128 contiguous bytes per access.
+// Offset (in floats) of the group holding columns k, k + 1 (k = 4q + 2h) of pair p.
+__device__ __forceinline__ int pair_off(int p, int ks, int q, int h) {
+  return p * 2 * ks + (q >> 3) * 64 + h * 32 + (q & 7) * 4;
+}
+
 // Reduce-scatter over the 8 lanes of a quarter-warp (xor offsets 4, 2, 1).  While C >= 2 values
 // remain, the lane with bit O set keeps the upper half and sends the lower half; afterwards the
 // single value left is summed with a plain xor exchange.  Each step adds (own, partner), so every
@@ -144,7 +172,36 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 
   // stage X~[:, k0:k0+ks] (rows >= M and columns >= klen are zero)
   const int q_row = ks >> 2, q_len = klen >> 2;
-  if constexpr (MASK == kNoMask) {
+  float* xsf = reinterpret_cast<float*>(xs);
+  // X~ of rows m, columns 4q..4q+3 (stored as given, or with the noise drawn here)
+  auto x4 = [&](int m, int q, float4* dst_out) -> float4 {
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (m < M && q < q_len) {
+      v = __ldg(reinterpret_cast<const float4*>(X + (int64_t)m * K + k0) + q);
+      if constexpr (MASK != kNoMask) {
+        const uint64_t j = (uint64_t)(((int64_t)m * K + k0) >> 2) + (uint64_t)q + nz.offset +
+                           (nz.offset_dev ? *nz.offset_dev : 0ull);
+        v = add4(v, draw_block<MASK>(j, nz.key, nz.b));
+        if (dst_out) __stcs(dst_out, v);
+      }
+    }
+    return v;
+  };
+  if constexpr (MT >= 4) {
+    // fused mask: X~ = fl32(X + eta), eta of element (m, k) being lane k % 4 of Philox block
+    // (m K + k) / 4 + offset, as the mask kernel draws it; the first row group writes X~ out
+    const bool write_xt = MASK != kNoMask && blockIdx.x == 0;
+#pragma unroll
+    for (int p = 0; p < MT / 2; ++p)
+      for (int q = threadIdx.x; q < q_row; q += THREADS) {
+        float4* d0 = write_xt && 2 * p < M && q < q_len ? reinterpret_cast<float4*>(nz.xt + (int64_t)(2 * p) * K + k0) + q : nullptr;
+        float4* d1 = write_xt && 2 * p + 1 < M && q < q_len ? reinterpret_cast<float4*>(nz.xt + (int64_t)(2 * p + 1) * K + k0) + q : nullptr;
+        const float4 a = x4(2 * p, q, d0), b = x4(2 * p + 1, q, d1);
+        *reinterpret_cast<float4*>(xsf + pair_off(p, ks, q, 0)) = make_float4(a.x, b.x, a.y, b.y);
+        *reinterpret_cast<float4*>(xsf + pair_off(p, ks, q, 1)) = make_float4(a.z, b.z, a.w, b.w);
+      }
+    if constexpr (MASK != kNoMask) load_first();
+  } else if constexpr (MASK == kNoMask) {
 #pragma unroll
     for (int m = 0; m < MT; ++m) {
       const float4* src = reinterpret_cast<const float4*>(X + (int64_t)m * K + k0);
@@ -179,8 +236,64 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 #pragma unroll
   for (int i = 0; i < V; ++i) acc[i] = 0.f;
 
+  if constexpr (MT >= 4) {
+    // acc2[r][p]: rows 2p, 2p + 1 of X~ against the lane's row r of W, as packed pairs
+    unsigned long long acc2[RQ][MT / 2];
+#pragma unroll
+    for (int r = 0; r < RQ; ++r)
+#pragma unroll
+      for (int p = 0; p < MT / 2; ++p) acc2[r][p] = 0ull;
+    const uint32_t xbase = static_cast<uint32_t>(__cvta_generic_to_shared(xsf));
+    for (int kb = 0; kb < klen; kb += U * kStep) {
+      float4 wn[U][RQ];
+      const int kn = kb + U * kStep;
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int r = 0; r < RQ; ++r)
+          wn[u][r] = (valid[r] && kn + u * kStep + kl < klen)
+                         ? __ldcs(reinterpret_cast<const float4*>(wp[r] + kn + u * kStep))
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        unsigned long long wx[RQ], wy[RQ], wz[RQ], ww[RQ];
+#pragma unroll
+        for (int r = 0; r < RQ; ++r) {
+          wx[r] = pack2(w[u][r].x, w[u][r].x);
+          wy[r] = pack2(w[u][r].y, w[u][r].y);
+          wz[r] = pack2(w[u][r].z, w[u][r].z);
+          ww[r] = pack2(w[u][r].w, w[u][r].w);
+        }
+        const int q = (kb + u * kStep + kl) >> 2;
+#pragma unroll
+        for (int p = 0; p < MT / 2; ++p) {
+          unsigned long long x0, x1, x2, x3;  // columns k, k+1, k+2, k+3 of rows 2p, 2p+1
+          lds_v2b64(xbase + 4u * (uint32_t)pair_off(p, ks, q, 0), x0, x1);
+          lds_v2b64(xbase + 4u * (uint32_t)pair_off(p, ks, q, 1), x2, x3);
+#pragma unroll
+          for (int r = 0; r < RQ; ++r) {
+            unsigned long long a = acc2[r][p];
+            a = ffma2(wx[r], x0, a);
+            a = ffma2(wy[r], x1, a);
+            a = ffma2(wz[r], x2, a);
+            a = ffma2(ww[r], x3, a);
+            acc2[r][p] = a;
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int r = 0; r < RQ; ++r) w[u][r] = wn[u][r];
+    }
+#pragma unroll
+    for (int r = 0; r < RQ; ++r)
+#pragma unroll
+      for (int p = 0; p < MT / 2; ++p) unpack2(acc2[r][p], acc[r * MT + 2 * p], acc[r * MT + 2 * p + 1]);
+  }
+
   const float4* xl = xs + (kl >> 2);
-  for (int kb = 0; kb < klen; kb += U * kStep) {
+  for (int kb = 0; kb < (MT >= 4 ? 0 : klen); kb += U * kStep) {
     // the next U steps of W while this one is summed
     float4 wn[U][RQ];
     const int kn = kb + U * kStep;
