@@ -47,22 +47,9 @@ __host__ __device__ constexpr int rows_per_block(int mt) { return WARPS * 4 * ro
 // rows (then 80 registers give 3 blocks per SM instead of 2; measured faster at 8 rows, slower at 16).
 __host__ __device__ constexpr int unroll_steps(int mt) { return mt == 8 ? 2 : 8 / rows_per_lane(mt); }
 
-// Packed pairs of fp32 (two rows of X~): one fma.rn.f32x2 does the two round-to-nearest FMAs the
-// scalar loop would, so the sums are the same bit for bit with half the FMA instructions.
-__device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
-  unsigned long long r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-  return r;
-}
-__device__ __forceinline__ void unpack2(unsigned long long v, float& lo, float& hi) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-}
-__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b,
-                                                    unsigned long long c) {
-  unsigned long long d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
+// Rows of X~ are summed in packed pairs (p2 / fma2 / up2 of noise.cuh): one fma.rn.f32x2 does the
+// two round-to-nearest FMAs the scalar loop would, so the sums are the same bit for bit with half
+// the FMA instructions.
 __device__ __forceinline__ void lds_v2b64(uint32_t addr, unsigned long long& a, unsigned long long& b) {
   asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(addr));
 }
@@ -259,10 +246,10 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
         unsigned long long wx[RQ], wy[RQ], wz[RQ], ww[RQ];
 #pragma unroll
         for (int r = 0; r < RQ; ++r) {
-          wx[r] = pack2(w[u][r].x, w[u][r].x);
-          wy[r] = pack2(w[u][r].y, w[u][r].y);
-          wz[r] = pack2(w[u][r].z, w[u][r].z);
-          ww[r] = pack2(w[u][r].w, w[u][r].w);
+          wx[r] = p2(w[u][r].x, w[u][r].x);
+          wy[r] = p2(w[u][r].y, w[u][r].y);
+          wz[r] = p2(w[u][r].z, w[u][r].z);
+          ww[r] = p2(w[u][r].w, w[u][r].w);
         }
         const int q = (kb + u * kStep + kl) >> 2;
 #pragma unroll
@@ -273,10 +260,10 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 #pragma unroll
           for (int r = 0; r < RQ; ++r) {
             unsigned long long a = acc2[r][p];
-            a = ffma2(wx[r], x0, a);
-            a = ffma2(wy[r], x1, a);
-            a = ffma2(wz[r], x2, a);
-            a = ffma2(ww[r], x3, a);
+            a = fma2(wx[r], x0, a);
+            a = fma2(wy[r], x1, a);
+            a = fma2(wz[r], x2, a);
+            a = fma2(ww[r], x3, a);
             acc2[r][p] = a;
           }
         }
@@ -289,7 +276,7 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 #pragma unroll
     for (int r = 0; r < RQ; ++r)
 #pragma unroll
-      for (int p = 0; p < MT / 2; ++p) unpack2(acc2[r][p], acc[r * MT + 2 * p], acc[r * MT + 2 * p + 1]);
+      for (int p = 0; p < MT / 2; ++p) up2(acc2[r][p], acc[r * MT + 2 * p], acc[r * MT + 2 * p + 1]);
   }
 
   const float4* xl = xs + (kl >> 2);

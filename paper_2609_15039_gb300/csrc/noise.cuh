@@ -54,37 +54,58 @@ __device__ __forceinline__ uint4 philox_block(uint64_t j, const PhiloxKey& key) 
 
 enum { kLaplace = 0, kGaussian = 1, kZero = 2 };
 
+// Packed pairs of fp32: one fma.rn.f32x2 does the two round-to-nearest FMAs that two fmaf calls
+// would, so a pair of uniforms (or angles) runs its polynomial in one chain, same results.
+__device__ __forceinline__ unsigned long long p2(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void up2(unsigned long long v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ unsigned long long fma2(unsigned long long a, unsigned long long b, unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ unsigned long long fma2c(unsigned long long a, unsigned long long b, float c) {
+  return fma2(a, b, p2(c, c));
+}
+
 // ln u for u = k 2^-24, k = 1 .. 2^24: u = 2^e m with m in [sqrt(1/2), sqrt(2)) and s = m - 1
 // (both exact), ln(1 + s) = s P(s) with P of degree 9 fitted to the relative error on that interval
 // (least squares on Chebyshev nodes, then Lawson's reweighting toward the minimax), and
 // ln u = e ln 2 + s P(s).  At most 1.6 ulp from ln u over all 2^24 inputs (checked against
 // binary64), and exact (0) at u = 1.
-__device__ __forceinline__ float log_unit(float u) {
-  const int bits = __float_as_int(u);
-  int e = (bits >> 23) - 127;
-  float m = __int_as_float((bits & 0x7FFFFF) | 0x3F800000);
-  if (m > 1.41421356f) {
-    m = __fmul_rn(m, 0.5f);
-    e += 1;
+// Two uniforms at once: ln u0 and ln u1.
+__device__ __forceinline__ void log_unit2(float u0, float u1, float& l0, float& l1) {
+  const int b0 = __float_as_int(u0), b1 = __float_as_int(u1);
+  int e0 = (b0 >> 23) - 127, e1 = (b1 >> 23) - 127;
+  float m0 = __int_as_float((b0 & 0x7FFFFF) | 0x3F800000), m1 = __int_as_float((b1 & 0x7FFFFF) | 0x3F800000);
+  if (m0 > 1.41421356f) {
+    m0 = __fmul_rn(m0, 0.5f);
+    e0 += 1;
   }
-  const float s = __fsub_rn(m, 1.0f);
-  float p = -0.07830669730901718f;
-  p = fmaf(p, s, 0.13019075989723206f);
-  p = fmaf(p, s, -0.13212285935878754f);
-  p = fmaf(p, s, 0.1416073590517044f);
-  p = fmaf(p, s, -0.16610340774059296f);
-  p = fmaf(p, s, 0.2000320553779602f);
-  p = fmaf(p, s, -0.2500157058238983f);
-  p = fmaf(p, s, 0.33333301544189453f);
-  p = fmaf(p, s, -0.49999988079071045f);
-  p = fmaf(p, s, 1.0f);
-  return fmaf((float)e, 0.6931471824645996f, __fmul_rn(p, s));
-}
-
-__device__ __forceinline__ float laplace1(uint32_t r, float b) {
-  const float u = __int2float_rn((int)((r & 0xFFFFFFu) + 1u)) * 0x1p-24f;  // (0, 1], exact
-  const float mag = __fmul_rn(b, -log_unit(u));
-  return (r >> 31) ? -mag : mag;
+  if (m1 > 1.41421356f) {
+    m1 = __fmul_rn(m1, 0.5f);
+    e1 += 1;
+  }
+  const unsigned long long s = p2(__fsub_rn(m0, 1.0f), __fsub_rn(m1, 1.0f));
+  unsigned long long p = p2(-0.07830669730901718f, -0.07830669730901718f);
+  p = fma2c(p, s, 0.13019075989723206f);
+  p = fma2c(p, s, -0.13212285935878754f);
+  p = fma2c(p, s, 0.1416073590517044f);
+  p = fma2c(p, s, -0.16610340774059296f);
+  p = fma2c(p, s, 0.2000320553779602f);
+  p = fma2c(p, s, -0.2500157058238983f);
+  p = fma2c(p, s, 0.33333301544189453f);
+  p = fma2c(p, s, -0.49999988079071045f);
+  p = fma2c(p, s, 1.0f);
+  float ps0, ps1;
+  up2(fma2c(p, s, -0.0f), ps0, ps1);  // fl(p s): adding -0 changes no rounding
+  l0 = fmaf((float)e0, 0.6931471824645996f, ps0);
+  l1 = fmaf((float)e1, 0.6931471824645996f, ps1);
 }
 
 // sin(pi x) and cos(pi x) for x = 2 u2 in [0, 2), x a multiple of 2^-23: x = q / 2 + r with
@@ -92,36 +113,31 @@ __device__ __forceinline__ float laplace1(uint32_t r, float b) {
 // Taylor series to degree 9 and 10 (truncation below 3e-9 at |pi r| <= pi / 4), evaluated by
 // Horner's rule in r^2; then the rotation by q quarter turns.  Error at most 1.7 ulp (checked
 // against binary64 sin and cos over all 2^24 inputs), with the exact zeros of sin and cos exact.
-__device__ __forceinline__ void sincospi_turns(float x, float* s, float* c) {
-  const float q = rintf(2.0f * x);
-  const float r = fmaf(q, -0.5f, x);
-  const float r2 = __fmul_rn(r, r);
-  float ps = 0.08214588661112819f;        //  pi^9 / 9!
-  ps = fmaf(ps, r2, -0.5992645293207919f);  // -pi^7 / 7!
-  ps = fmaf(ps, r2, 2.550164039877345f);    //  pi^5 / 5!
-  ps = fmaf(ps, r2, -5.167712780049969f);   // -pi^3 / 3!
-  ps = fmaf(ps, r2, 3.141592653589793f);    //  pi
-  const float sr = __fmul_rn(ps, r);
-  float pc = -0.02580689139001405f;         // -pi^10 / 10!
-  pc = fmaf(pc, r2, 0.23533063035889312f);  //  pi^8 / 8!
-  pc = fmaf(pc, r2, -1.3352627688545893f);  // -pi^6 / 6!
-  pc = fmaf(pc, r2, 4.058712126416768f);    //  pi^4 / 4!
-  pc = fmaf(pc, r2, -4.934802200544679f);   // -pi^2 / 2!
-  pc = fmaf(pc, r2, 1.0f);
-  const int t = (int)q & 3;  // (sin, cos)(pi (r + t / 2))
-  *s = t == 0 ? sr : t == 1 ? pc : t == 2 ? -sr : -pc;
-  *c = t == 0 ? pc : t == 1 ? -sr : t == 2 ? -pc : sr;
-}
-
-__device__ __forceinline__ void gauss2(uint32_t ra, uint32_t rb, float b, float& ea, float& eb) {
-  const float u1 = __int2float_rn((int)((ra >> 8) + 1u)) * 0x1p-24f;  // (0, 1]
-  const float u2 = __int2float_rn((int)(rb >> 8)) * 0x1p-24f;         // [0, 1)
-  const float R = sqrtf(__fmul_rn(-2.0f, log_unit(u1)));
-  float s, c;
-  sincospi_turns(2.0f * u2, &s, &c);  // sin/cos of 2 pi u2; 2*u2 is exact
-  const float sr = __fmul_rn(b, R);
-  ea = __fmul_rn(sr, c);
-  eb = __fmul_rn(sr, s);
+// Two angles at once.
+__device__ __forceinline__ void sincospi_turns2(float x0, float x1, float* s0, float* c0, float* s1, float* c1) {
+  const float q0 = rintf(2.0f * x0), q1 = rintf(2.0f * x1);
+  const float r0 = fmaf(q0, -0.5f, x0), r1 = fmaf(q1, -0.5f, x1);
+  const unsigned long long r = p2(r0, r1), r2 = p2(__fmul_rn(r0, r0), __fmul_rn(r1, r1));
+  unsigned long long ps = p2(0.08214588661112819f, 0.08214588661112819f);
+  ps = fma2c(ps, r2, -0.5992645293207919f);
+  ps = fma2c(ps, r2, 2.550164039877345f);
+  ps = fma2c(ps, r2, -5.167712780049969f);
+  ps = fma2c(ps, r2, 3.141592653589793f);
+  float sr0, sr1;
+  up2(fma2c(ps, r, -0.0f), sr0, sr1);  // fl(ps r)
+  unsigned long long pc = p2(-0.02580689139001405f, -0.02580689139001405f);
+  pc = fma2c(pc, r2, 0.23533063035889312f);
+  pc = fma2c(pc, r2, -1.3352627688545893f);
+  pc = fma2c(pc, r2, 4.058712126416768f);
+  pc = fma2c(pc, r2, -4.934802200544679f);
+  pc = fma2c(pc, r2, 1.0f);
+  float pc0, pc1;
+  up2(pc, pc0, pc1);
+  const int t0 = (int)q0 & 3, t1 = (int)q1 & 3;
+  *s0 = t0 == 0 ? sr0 : t0 == 1 ? pc0 : t0 == 2 ? -sr0 : -pc0;
+  *c0 = t0 == 0 ? pc0 : t0 == 1 ? -sr0 : t0 == 2 ? -pc0 : sr0;
+  *s1 = t1 == 0 ? sr1 : t1 == 1 ? pc1 : t1 == 2 ? -sr1 : -pc1;
+  *c1 = t1 == 0 ? pc1 : t1 == 1 ? -sr1 : t1 == 2 ? -pc1 : sr1;
 }
 
 template <int MECH>
@@ -130,10 +146,30 @@ __device__ __forceinline__ float4 draw_block(uint64_t j, const PhiloxKey& key, f
   const uint4 r = philox_block(j, key);
   float4 e;
   if (MECH == kLaplace) {
-    e = make_float4(laplace1(r.x, b), laplace1(r.y, b), laplace1(r.z, b), laplace1(r.w, b));
-  } else {
-    gauss2(r.x, r.y, b, e.x, e.y);
-    gauss2(r.z, r.w, b, e.z, e.w);
+    const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+    float u[4], l[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) u[i] = __int2float_rn((int)((w[i] & 0xFFFFFFu) + 1u)) * 0x1p-24f;
+    log_unit2(u[0], u[1], l[0], l[1]);
+    log_unit2(u[2], u[3], l[2], l[3]);
+    float v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float mag = __fmul_rn(b, -l[i]);
+      v[i] = (w[i] >> 31) ? -mag : mag;
+    }
+    e = make_float4(v[0], v[1], v[2], v[3]);
+  } else {  // Box-Muller on the pairs (x, y) and (z, w), the two done side by side
+    const float ua = __int2float_rn((int)((r.x >> 8) + 1u)) * 0x1p-24f;  // (0, 1]
+    const float ub = __int2float_rn((int)((r.z >> 8) + 1u)) * 0x1p-24f;
+    const float va = __int2float_rn((int)(r.y >> 8)) * 0x1p-24f;         // [0, 1)
+    const float vb = __int2float_rn((int)(r.w >> 8)) * 0x1p-24f;
+    float la, lb, sa, ca, sb, cb;
+    log_unit2(ua, ub, la, lb);
+    sincospi_turns2(2.0f * va, 2.0f * vb, &sa, &ca, &sb, &cb);  // sin/cos of 2 pi v; 2 v is exact
+    const float ra_ = __fmul_rn(b, sqrtf(__fmul_rn(-2.0f, la)));
+    const float rb_ = __fmul_rn(b, sqrtf(__fmul_rn(-2.0f, lb)));
+    e = make_float4(__fmul_rn(ra_, ca), __fmul_rn(ra_, sa), __fmul_rn(rb_, cb), __fmul_rn(rb_, sb));
   }
   return e;
 }
