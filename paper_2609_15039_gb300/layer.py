@@ -207,22 +207,35 @@ class MaskedLayer:
         base = torch.tensor([self.block_offset(g, cycle, 0) for g in self.groups], dtype=torch.int64)
         self.rng_base.copy_(base)
 
-    def refill(self, eps, mech, seed, cycle, path="auto", stream=None, timer=None, device_base=False):
-        """a2 + a4: draw ``draws`` masks per group and precompute their corrections in one product."""
+    def refill(self, eps, mech, seed, cycle, path="auto", stream=None, timer=None, device_base=False,
+               parallel=False):
+        """a2 + a4: draw ``draws`` masks per group and precompute their corrections in one product.
+
+        parallel: the FP16X3 groups' corrections (which use no workspace: the noise comes split and
+        the tensor-core kernel reduces on chip) run side by side on streams of their own, so the
+        tiles of one fill the SMs another leaves idle; the current stream waits for all of them."""
+        main = torch.cuda.current_stream() if stream is None else stream
+        forks = []
         for gi, g in enumerate(self.groups):
             b = self.bank[g.name]
             off, off_dev = self._offset(gi, g, cycle, 0, device_base)
             es = b.get("es") if self._fused_split(g, path, self.M) else None
             if es is not None:  # the FP16X3 correction reads only the split: the noise is split as drawn
-                spl.spl_noise_mask_split(None, es.f16_hi, es.f16_lo, es.f16_exp, None, self.deltas[g.name], eps, mech,
-                                         seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
-                if timer:
-                    timer("begin", "precompute", g.name)
-                spl.spl_precompute_noise_product_matched_split(b["C"], es, g.wt, self.M,
-                                                               path=self.path_of(g, path, self.M),
-                                                               workspace=self.workspace, stream=stream)
-                if timer:
-                    timer("end", "precompute", g.name)
+                side = main
+                if parallel:
+                    side = self._side_stream(gi)
+                    side.wait_stream(main)
+                    forks.append(side)
+                with torch.cuda.stream(side):
+                    spl.spl_noise_mask_split(None, es.f16_hi, es.f16_lo, es.f16_exp, None, self.deltas[g.name], eps,
+                                             mech, seed, stream_id=gi, offset=off, stream=side, offset_dev=off_dev)
+                    if timer:
+                        timer("begin", "precompute", g.name)
+                    spl.spl_precompute_noise_product_matched_split(b["C"], es, g.wt, self.M,
+                                                                   path=self.path_of(g, path, self.M),
+                                                                   workspace=self.workspace, stream=side)
+                    if timer:
+                        timer("end", "precompute", g.name)
                 continue
             spl.spl_noise(b["eta"], self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off, stream=stream,
                           offset_dev=off_dev)
@@ -237,6 +250,16 @@ class MaskedLayer:
                                                          stream=stream)
             if timer:
                 timer("end", "precompute", g.name)
+        for side in forks:
+            main.wait_stream(side)
+
+    def _side_stream(self, gi):
+        """A stream of this layer for group gi's correction (created once)."""
+        if not hasattr(self, "_sides"):
+            self._sides = {}
+        if gi not in self._sides:
+            self._sides[gi] = torch.cuda.Stream()
+        return self._sides[gi]
 
     def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None, device_base=False,
                group_hooks=None):
@@ -316,7 +339,7 @@ class MaskedLayer:
                 if before:
                     before(d)
                 if d == 0:
-                    self.refill(eps, mech, seed, 0, path=path, timer=timer, device_base=True)
+                    self.refill(eps, mech, seed, 0, path=path, timer=timer, device_base=True, parallel=timer is None)
                 inp = inputs[d % len(inputs)] if isinstance(inputs, (list, tuple)) else inputs
                 self.online(inp, eps, mech, seed, 0, d, path=path, timer=timer, device_base=True,
                             group_hooks=group_hooks)
@@ -411,7 +434,7 @@ class MaskedStack:
             with torch.cuda.graph(graph):
                 for layer, x, seed in zip(self.layers, inputs, self.seeds):
                     if d == 0 and refill:
-                        layer.refill(eps, mech, seed, 0, path=path, device_base=True)
+                        layer.refill(eps, mech, seed, 0, path=path, device_base=True, parallel=True)
                     layer.online(x, eps, mech, seed, 0, d, path=path, device_base=True)
                 if d == D - 1:
                     for layer in self.layers:
