@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--cpu-sample-rows", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-overlap", action="store_true",
+                    help="compute each bank cycle's corrections before its steps instead of during the previous cycle")
     ap.add_argument("--workload", default="llama_layer",
                     choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep", "down_fp64", "slalom"],
                     help="llama_layer (default): the headline line; the others measure the stack and sweep "
@@ -347,11 +349,34 @@ def main():
         e2e_graphs, _ = layer.capture(dev_in, args.eps, mech, seed, path=args.path, before=copy_in, after=copy_out,
                                       group_hooks=(group_in, group_out))
 
+    # The corrections of the next bank cycle need nothing from this one: whole-cycle graphs compute
+    # them during this cycle's steps, on streams of lower priority (MaskedLayer.capture_overlapped).
+    # Used when every group takes the fused fp16 split and the step count is whole cycles.
+    use_ov = (not args.no_overlap and args.steps % DRAWS == 0 and
+              all(layer._fused_split(g, args.path, M) for g in layer.groups))
+    if use_ov:
+        ov_graphs, ov_launches = layer.capture_overlapped(inputs, args.eps, mech, seed, path=args.path)
+        e2e_ov = None
+        if e2e_graphs is not None:
+            e2e_ov, _ = layer.capture_overlapped(dev_in, args.eps, mech, seed, path=args.path, before=copy_in,
+                                                 after=copy_out, group_hooks=(group_in, group_out))
+
+    def start_overlapped(cycle):
+        """Bank buffer cycle % 2 holds the corrections of ``cycle``; the bases are at ``cycle``."""
+        layer.set_cycle(cycle)
+        layer.refill(args.eps, mech, seed, 0, path=args.path, device_base=True, parallel=True, parity=cycle % 2)
+
     s = DRAWS  # the graphs start at a bank cycle
-    layer.set_cycle(s // DRAWS)
-    for _ in range(args.warmup):
-        graphs[s % DRAWS].replay()
-        s += 1
+    if use_ov:
+        start_overlapped(s // DRAWS)
+        for _ in range(-(-args.warmup // DRAWS)):  # warm-up: whole cycles, at least the W steps
+            ov_graphs[(s // DRAWS) % 2].replay()
+            s += DRAWS
+    else:
+        layer.set_cycle(s // DRAWS)
+        for _ in range(args.warmup):
+            graphs[s % DRAWS].replay()
+            s += 1
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -362,16 +387,25 @@ def main():
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_push("timed")
         t_start.record(stream)
-        for _ in range(args.steps):
-            graphs[s % DRAWS].replay()
-            s += 1
+        if use_ov:
+            for _ in range(args.steps // DRAWS):
+                ov_graphs[(s // DRAWS) % 2].replay()
+                s += DRAWS
+        else:
+            for _ in range(args.steps):
+                graphs[s % DRAWS].replay()
+                s += 1
         t_end.record(stream)
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()
     if world > 1:
         dist.barrier()
-    gpu_launches = sum(graph_launches[(s_timed + i) % DRAWS] for i in range(args.steps))
+    if use_ov:
+        gpu_launches = sum(ov_launches[(s_timed // DRAWS + i) % 2] for i in range(args.steps // DRAWS))
+    else:
+        gpu_launches = sum(graph_launches[(s_timed + i) % DRAWS] for i in range(args.steps))
     ms = t_start.elapsed_time(t_end) / args.steps
+    layer.set_cycle(s // DRAWS)  # the per-step graphs below start at a bank cycle
     # second pass: per-call events (the last replay of each draw's graph holds its times)
     p_start = torch.cuda.Event(enable_timing=True)
     p_end = torch.cuda.Event(enable_timing=True)
@@ -450,16 +484,27 @@ def main():
 
     e2e = None
     if e2e_graphs is not None:
-        for _ in range(2):
-            e2e_graphs[s % DRAWS].replay()
-            s += 1
+        if use_ov:
+            s = -(-s // DRAWS) * DRAWS
+            start_overlapped(s // DRAWS)
+            e2e_ov[(s // DRAWS) % 2].replay()  # warm-up cycle
+            s += DRAWS
+        else:
+            for _ in range(2):
+                e2e_graphs[s % DRAWS].replay()
+                s += 1
         torch.cuda.synchronize()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for _ in range(args.steps):
-            e2e_graphs[s % DRAWS].replay()
-            s += 1
+        if use_ov:
+            for _ in range(args.steps // DRAWS):
+                e2e_ov[(s // DRAWS) % 2].replay()
+                s += DRAWS
+        else:
+            for _ in range(args.steps):
+                e2e_graphs[s % DRAWS].replay()
+                s += 1
         host_out[last].copy_(layer.bank[last]["Y"], non_blocking=True)  # the last step's, in the region
         e1.record(stream)
         torch.cuda.synchronize()
@@ -480,6 +525,9 @@ def main():
         "vs_baseline": None, "dtype": "f32", "path": path_name, "data": "synthetic",
         "config": {"workload": WORKLOAD, "tokens": M, "eps": args.eps, "mech": mech, "layers_per_step": 1,
                    "bank_draws": DRAWS, "flops_per_step": flops_step,
+                   "bank_schedule": ("each cycle's corrections computed during the previous cycle's steps, on "
+                                     "lower-priority streams (whole-cycle graphs)") if use_ov else
+                                    "each cycle's corrections computed before its first step",
                    "l2": "weights 1.2 GB per step > 129 MB L2 (no flush needed)",
                    "parallelism": "replicas" if world > 1 else "single"},
         "ms_per_prefill_28_layers": 28 * ms,

@@ -174,6 +174,18 @@ class MaskedLayer:
                                      f16_lo=torch.empty((draws * M, g.K), dtype=torch.int16, device=dev),
                                      f16_exp=torch.empty(draws * M, dtype=torch.int32, device=dev))
 
+    def enable_overlap(self):
+        """A second correction buffer per group, so that a bank cycle can run its online steps on one
+        while the next cycle's corrections are computed into the other (capture_overlapped)."""
+        for g in self.groups:
+            b = self.bank[g.name]
+            if "Cs" not in b:
+                b["Cs"] = [b["C"], torch.empty_like(b["C"])]
+
+    def _C(self, g, parity):
+        b = self.bank[g.name]
+        return b["Cs"][parity] if "Cs" in b else b["C"]
+
     def _fused_split(self, g, path, M):
         """True when the online product of group g runs FP16X3: then the mask kernel also writes the
         fp16 split of X~ and the product skips its own split pass."""
@@ -208,17 +220,22 @@ class MaskedLayer:
         self.rng_base.copy_(base)
 
     def refill(self, eps, mech, seed, cycle, path="auto", stream=None, timer=None, device_base=False,
-               parallel=False):
+               parallel=False, parity=0, ahead=0):
         """a2 + a4: draw ``draws`` masks per group and precompute their corrections in one product.
 
         parallel: the FP16X3 groups' corrections (which use no workspace: the noise comes split and
         the tensor-core kernel reduces on chip) run side by side on streams of their own, so the
-        tiles of one fill the SMs another leaves idle; the current stream waits for all of them."""
+        tiles of one fill the SMs another leaves idle; the current stream waits for all of them.
+        parity: the correction buffer to fill (see enable_overlap); ahead: the draws of cycle
+        ``cycle + ahead`` (with device_base: that many cycles past the device-side base)."""
         main = torch.cuda.current_stream() if stream is None else stream
         forks = []
         for gi, g in enumerate(self.groups):
             b = self.bank[g.name]
-            off, off_dev = self._offset(gi, g, cycle, 0, device_base)
+            off, off_dev = self._offset(gi, g, cycle + (0 if device_base else ahead), 0, device_base)
+            if device_base:
+                off += ahead * self.draws * (self.M * g.K // 4)
+            C = self._C(g, parity)
             es = b.get("es") if self._fused_split(g, path, self.M) else None
             if es is not None:  # the FP16X3 correction reads only the split: the noise is split as drawn
                 side = main
@@ -231,7 +248,7 @@ class MaskedLayer:
                                              mech, seed, stream_id=gi, offset=off, stream=side, offset_dev=off_dev)
                     if timer:
                         timer("begin", "precompute", g.name)
-                    spl.spl_precompute_noise_product_matched_split(b["C"], es, g.wt, self.M,
+                    spl.spl_precompute_noise_product_matched_split(C, es, g.wt, self.M,
                                                                    path=self.path_of(g, path, self.M),
                                                                    workspace=self.workspace, stream=side)
                     if timer:
@@ -242,10 +259,10 @@ class MaskedLayer:
             if timer:
                 timer("begin", "precompute", g.name)
             if g.name in self.fp64:
-                spl.spl_precompute_noise_product_f64(b["C"], b["eta"], g.W, workspace=self.workspace, stream=stream)
+                spl.spl_precompute_noise_product_f64(C, b["eta"], g.W, workspace=self.workspace, stream=stream)
             else:
                 # summed in the order the online product of M rows uses, so their rounding cancels
-                spl.spl_precompute_noise_product_matched(b["C"], b["eta"], g.wt, self.M,
+                spl.spl_precompute_noise_product_matched(C, b["eta"], g.wt, self.M,
                                                          path=self.path_of(g, path, self.M), workspace=self.workspace,
                                                          stream=stream)
             if timer:
@@ -262,7 +279,7 @@ class MaskedLayer:
         return self._sides[gi]
 
     def online(self, inputs, eps, mech, seed, cycle, d, path="auto", stream=None, timer=None, device_base=False,
-               group_hooks=None):
+               group_hooks=None, parity=0):
         """a3 + a5 + a6 for draw d: regenerate eta_d, mask, masked product with fused unmask.
 
         inputs: {group: X [M, K]}.  Returns {group: Y [M, N_group]} (views of the layer's buffers).
@@ -274,21 +291,22 @@ class MaskedLayer:
         for gi, g in enumerate(self.groups):
             if group_hooks:
                 group_hooks[0](gi, g.name)
-            self._online_group(gi, g, inputs, eps, mech, seed, cycle, d, path, stream, timer, device_base, out)
+            self._online_group(gi, g, inputs, eps, mech, seed, cycle, d, path, stream, timer, device_base, out, parity)
             if group_hooks:
                 group_hooks[1](gi, g.name)
         return out
 
-    def _online_group(self, gi, g, inputs, eps, mech, seed, cycle, d, path, stream, timer, device_base, out):
+    def _online_group(self, gi, g, inputs, eps, mech, seed, cycle, d, path, stream, timer, device_base, out, parity):
         M = self.M
         b = self.bank[g.name]
+        Cd = self._C(g, parity)[d * M:(d + 1) * M]
         off, off_dev = self._offset(gi, g, cycle, d, device_base)
         fp64 = g.name in self.fp64
         xs = b.get("xs") if self._fused_split(g, path, M) else None
         if self._fused_mask(g, path, M):
             if timer:
                 timer("begin", "masked_linear_unmask", g.name)
-            spl.spl_noise_mask_linear_unmask(b["Y"], b["xt"], inputs[g.name], g.wt, b["C"][d * M:(d + 1) * M],
+            spl.spl_noise_mask_linear_unmask(b["Y"], b["xt"], inputs[g.name], g.wt, Cd,
                                              self.deltas[g.name], eps, mech, seed, stream_id=gi, offset=off,
                                              path=self.path_of(g, path, M), workspace=self.workspace,
                                              stream=stream, offset_dev=off_dev)
@@ -308,14 +326,14 @@ class MaskedLayer:
         if timer:
             timer("begin", "masked_linear_unmask", g.name)
         if fp64:
-            spl.spl_masked_linear_unmask_f64(b["Y"], b["xt"], g.W, b["C"][d * M:(d + 1) * M],
+            spl.spl_masked_linear_unmask_f64(b["Y"], b["xt"], g.W, Cd,
                                              workspace=self.workspace, stream=stream)
         elif xs is not None:
-            spl.spl_masked_linear_unmask_split(b["Y"], xs, g.wt, b["C"][d * M:(d + 1) * M],
+            spl.spl_masked_linear_unmask_split(b["Y"], xs, g.wt, Cd,
                                                path=self.path_of(g, path, M), workspace=self.workspace,
                                                stream=stream)
         else:
-            spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, b["C"][d * M:(d + 1) * M],
+            spl.spl_masked_linear_unmask(b["Y"], b["xt"], g.wt, Cd,
                                          path=self.path_of(g, path, M), workspace=self.workspace, stream=stream)
         if timer:
             timer("end", "masked_linear_unmask", g.name)
@@ -348,6 +366,48 @@ class MaskedLayer:
                 if d == self.draws - 1:
                     for gi, g in enumerate(self.groups):
                         spl.spl_rng_advance(self.rng_base[gi:gi + 1], self.draws * (self.M * g.K // 4))
+            graphs.append(graph)
+            launches.append(spl.spl_launch_count() - n0)
+        return graphs, launches
+
+    def capture_overlapped(self, inputs, eps, mech, seed, path="auto", before=None, after=None, group_hooks=None):
+        """Two CUDA graphs, each a whole bank cycle: graph p runs the ``draws`` online steps on
+        correction buffer p while, on streams of lower priority, the next cycle's corrections are
+        computed into buffer 1 - p, filling the SMs and the bandwidth the online products leave
+        idle; the graph ends when both are done and moves the Philox bases on by one cycle.  Replay
+        graphs[c % 2] for cycle c after set_cycle(c) and a refill of buffer c % 2 for cycle c.
+        ``before(d)`` / ``after(d)`` / ``group_hooks`` as in capture; ``inputs`` may be a list
+        (step d reads inputs[d % len(inputs)]).  Returns the graphs and their kernel counts."""
+        # the two sides must not share the workspace: every group's online product and correction
+        # take the fp16 split (on-chip reductions, no workspace)
+        if not all(self._fused_split(g, path, self.M) for g in self.groups):
+            raise ValueError("capture_overlapped needs every group on FP16X3 with the fused split")
+        self.enable_overlap()
+        lo, hi = torch.cuda.Stream.priority_range()
+        if not hasattr(self, "_bank_stream"):
+            self._bank_stream = torch.cuda.Stream(priority=lo)
+            self._online_stream = torch.cuda.Stream(priority=hi)
+        graphs, launches = [], []
+        for parity in range(2):
+            graph = torch.cuda.CUDAGraph()
+            n0 = spl.spl_launch_count()
+            with torch.cuda.graph(graph, stream=self._online_stream):
+                main = torch.cuda.current_stream()
+                self._bank_stream.wait_stream(main)
+                with torch.cuda.stream(self._bank_stream):
+                    self.refill(eps, mech, seed, 0, path=path, device_base=True, parallel=True, parity=1 - parity,
+                                ahead=1)
+                for d in range(self.draws):
+                    if before:
+                        before(d)
+                    inp = inputs[d % len(inputs)] if isinstance(inputs, (list, tuple)) else inputs
+                    self.online(inp, eps, mech, seed, 0, d, path=path, device_base=True, group_hooks=group_hooks,
+                                parity=parity)
+                    if after:
+                        after(d)
+                main.wait_stream(self._bank_stream)
+                for gi, g in enumerate(self.groups):
+                    spl.spl_rng_advance(self.rng_base[gi:gi + 1], self.draws * (self.M * g.K // 4))
             graphs.append(graph)
             launches.append(spl.spl_launch_count() - n0)
         return graphs, launches

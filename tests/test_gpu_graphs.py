@@ -77,3 +77,44 @@ def test_device_offset_equals_host_offset(spl):
     assert base.item() == 12345 + 2 ** 40
     # an offset word must be 8-byte aligned: refused before anything is launched
     assert spl.lib().spl_rng_advance(base.data_ptr() + 4, 1, None) == spl.SPL_EALIGN
+
+
+def test_overlapped_cycle_graphs_equal_eager_steps(spl):
+    """Whole-cycle graphs that compute the next cycle's corrections during this cycle's steps (on
+    streams of their own) give, step by step, the eager results -- across three cycles, so both
+    correction buffers are filled by a graph and read by the other."""
+    model = wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)
+    draws, eps, mech, seed, M = 3, 1.0, "gaussian", 78, 128
+    layer, inputs = make_layer(model, M, draws)
+    assert all(layer._fused_split(g, "auto", M) for g in layer.groups)
+
+    def eager(s):
+        cycle, d = divmod(s, draws)
+        if d == 0:
+            layer.refill(eps, mech, seed, cycle)
+        return {g: y.clone() for g, y in layer.online(inputs, eps, mech, seed, cycle, d).items()}
+
+    first, cycles = 2, 3
+    expected = [eager(s) for s in range(first * draws, (first + cycles) * draws)]
+    torch.cuda.synchronize()
+    outs = []
+
+    def after(d):  # each step's results, kept inside the graph
+        outs.append({g.name: layer.bank[g.name]["Y"].clone() for g in layer.groups})
+
+    graphs, launches = layer.capture_overlapped(inputs, eps, mech, seed, after=after)
+    assert len(graphs) == 2 and all(n > 0 for n in launches)
+    captured = list(outs)  # the tensors each graph writes its step results into
+    layer.set_cycle(first)
+    layer.refill(eps, mech, seed, 0, device_base=True, parallel=True, parity=first % 2)
+    for i in range(cycles):
+        c = first + i
+        graphs[c % 2].replay()
+        torch.cuda.synchronize()
+        for d in range(draws):
+            got = captured[(c % 2) * draws + d]
+            for g in got:
+                assert torch.equal(got[g], expected[i * draws + d][g]), (c, d, g)
+    exp_base = [layer.block_offset(g, first + cycles, 0) for g in layer.groups]
+    assert layer.rng_base.cpu().tolist() == exp_base
+    assert spl.spl_get_device_status() == 0
