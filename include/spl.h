@@ -410,22 +410,29 @@ spl_status spl_test_tc_shape(int64_t M, int64_t K, int64_t N, int64_t seg_splits
 
 /* Test hook (no counterpart in the paper): *out (host) = the number of clusters
  * of `cluster` CTAs (1..8) of the launch variant (tile_n, ring_kb) -- (256, 192),
- * (128, 224) or (128, 96) -- that can be resident at once on the current device.
+ * (128, 224), (128, 96), (160, 224), (192, 224) or (224, 224) -- that can be
+ * resident at once on the current device.
  * EINVAL for another variant, cluster outside [1, 8] or a NULL out. */
 spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int64_t cluster, int64_t* out);
 
 /* Test hook (the paper has no counterpart): Y = Xt W^T (- C if C is not NULL)
  * on the tcgen05 kernel with a fixed launch variant -- tile width tile_n and a
- * stage ring of ring_kb KB: (256, 192), (128, 224) or (128, 96) -- and every
- * tile's K range split `splits` ways (1..8) across a thread-block cluster,
- * instead of the shape the library would choose; with full_tiles > 0 the first
- * full_tiles tiles (M fastest) run unsplit in a launch of their own and only the
- * rest is split.  path is SPL_PATH_TF32X3 or SPL_PATH_FP16X3.  Same operands,
- * workspace and errors as spl_masked_linear_unmask; EINVAL for another path or
- * variant or full_tiles outside [0, tiles], ESHAPE for a split outside 1..8. */
+ * stage ring of ring_kb KB: (256, 192), (128, 224), (128, 96), (160, 224),
+ * (192, 224) or (224, 224) -- and every tile's K range split `splits` ways
+ * (1..8) across a thread-block cluster, instead of the shape the library would
+ * choose; with full_tiles > 0 the first full_tiles tiles (M fastest) run unsplit
+ * in a launch of their own and only the rest is split.  seg_splits > 0: the
+ * unsplit tiles run in segmented mode (the bank's form: one CTA over all of K,
+ * the partial sums of a seg_splits-way split of K folded in order), so the
+ * result equals the seg_splits-way split product bit for bit; splits must then
+ * be 1 or seg_splits.  path is SPL_PATH_TF32X3 or SPL_PATH_FP16X3.  Same
+ * operands, workspace and errors as spl_masked_linear_unmask; EINVAL for another
+ * path or variant, full_tiles outside [0, tiles], seg_splits outside [0, 8] or
+ * a splits other than 1 or seg_splits, ESHAPE for a split outside 1..8. */
 spl_status spl_test_tc_product(float* Y, const float* Xt, const spl_weight* W, const float* C, int64_t M,
                                int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
-                               int64_t full_tiles, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+                               int64_t full_tiles, int seg_splits, void* workspace, size_t workspace_bytes,
+                               cudaStream_t stream);
 
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last

@@ -89,7 +89,7 @@ struct Fp16x3 {
 // per SM; a 96 KB ring lets two CTAs share an SM, one streaming while the other finishes.
 template <class Md, int BN, int RK>
 struct Cfg {
-  static_assert(BN == 128 || BN == 256, "tile width");
+  static_assert(BN % 32 == 0 && BN >= 128 && BN <= 256, "tile width: whole 32-column TMEM loads, one MMA wide");
   static_assert(RK == 96 || RK == 192 || RK == 224, "ring size");
   static constexpr uint32_t A_HALF = BM * Md::BK * Md::ESZ, B_HALF = BN * Md::BK * Md::ESZ;
   static constexpr uint32_t A_HI = 0, A_LO = A_HALF, W_HI = 2 * A_HALF, W_LO = W_HI + B_HALF;
@@ -100,6 +100,10 @@ struct Cfg {
   static constexpr uint32_t SMEM = RING + AUX_BYTES + 1024;  // + alignment slack
   static constexpr int RED_STRIDE = BN + 4;                  // floats per row of the staged accumulator
   static constexpr uint32_t IDESC = make_idesc(Md::FMT, BM, BN);
+  // TMEM: the accumulator R at column 0 and, in segmented mode, P at column P_OFF (allocations
+  // are powers of two of at least 32 columns).
+  static constexpr uint32_t P_OFF = BN <= 128 ? 128u : 256u;
+  static constexpr uint32_t TMEM_COLS = P_OFF, TMEM_COLS_SEG = 2u * P_OFF;
   static_assert(A_LO % 1024 == 0 && W_HI % 1024 == 0 && W_LO % 1024 == 0 && STAGE % 1024 == 0,
                 "swizzle atoms aligned");
   static_assert(STAGES >= 3 && STAGES <= 8, "ring depth");
@@ -352,7 +356,7 @@ __device__ __forceinline__ void reduce_store(const float* red, int r0, int r1, i
 // Segmented mode (seg_blocks > 0, one CTA per tile over all of K): the K range is cut into
 // segments of seg_blocks stages, the same boundaries a K-split of the same problem uses; the
 // first segment accumulates into R (TMEM columns 0..BN-1), every later one into P (columns
-// BN..2BN-1), which the epilogue warps fold into R (R = fl(R + P)) before the next segment
+// P_OFF..P_OFF+BN-1), which the epilogue warps fold into R (R = fl(R + P)) before the next segment
 // starts.  Each output is then summed in exactly the order of the split launch -- the partials
 // of the splits added in rank order -- while one CTA streams its whole K range.
 template <class Md, int BN, int RK>
@@ -388,7 +392,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   const uint32_t fold_bar = bar_base + 8u * (2 * STAGES + 2);  // segmented: P folded into R
   const int seg_len = seg_blocks > 0 ? seg_blocks : nk + 1;    // stages per segment
   const int nseg = seg_blocks > 0 ? (int)ceil_div(nk, seg_blocks) : 1;
-  const uint32_t tmem_cols = seg_blocks > 0 ? 2u * BN : (uint32_t)BN;
+  const uint32_t tmem_cols = seg_blocks > 0 ? L::TMEM_COLS_SEG : L::TMEM_COLS;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -484,7 +488,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       if (lane == 0) {
         tc_fence_after();
         const uint32_t st = smem_u32(smem + (size_t)s * L::STAGE);
-        const uint32_t acc = tmem + (seg >= 1 ? (uint32_t)BN : 0u);
+        const uint32_t acc = tmem + (seg >= 1 ? L::P_OFF : 0u);
 #pragma unroll
         for (int kk = 0; kk < BK / Md::UMMA_K; ++kk) {
           const uint32_t koff = kk * 32u;  // one instruction's K is 32 bytes of the 64-byte swizzled row
@@ -542,7 +546,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       for (int c = 0; c < BN / 32; ++c) {
         float r[32], p[32];
         tmem_ld_32x32(lane_base + (uint32_t)(32 * c), r);
-        tmem_ld_32x32(lane_base + (uint32_t)(BN + 32 * c), p);
+        tmem_ld_32x32(lane_base + L::P_OFF + (uint32_t)(32 * c), p);
 #pragma unroll
         for (int i = 0; i < 32; ++i) r[i] = __fadd_rn(r[i], p[i]);
         tmem_st_32x32(lane_base + (uint32_t)(32 * c), r);
@@ -668,20 +672,23 @@ bool set_smem_attr() {
 }
 
 // The launch variants: tile width, ring size, CTAs per SM, and the cost constants of the
-// launch model below (F: fixed cost of a CTA -- launch, pipeline fill, staging and cross-CTA
-// reduction of its tile; b: cost per unit of K, i.e. bytes per K over the bytes the ring keeps
-// in flight, relative to the 256-wide tile with the 192 KB ring).  Measured on GB300.
-// Cost of one round of co-resident CTAs, in units of K: F + f s + b K / s (F: setup and epilogue,
-// f: the cluster reduction per rank, b: the mainloop per K element), fitted to a sweep of every
-// variant, split and whole-wave form over the Llama and Qwen projections at 128..4096 rows on
-// GB300 (the shapes it picks are within 0.3% of the best measured in total).
+// launch model below.  Cost of one round of co-resident CTAs, in units of K: F + f s + b K / s
+// (F: setup, pipeline fill and epilogue of a CTA; f: the cluster reduction per rank; b: the
+// mainloop per K element, relative to the 256-wide tile with the 192 KB ring), fitted to a sweep
+// of every variant, split and whole-wave form over the eight Llama and Qwen projections at 128,
+// 512, 1024, 2048 and 4096 rows on GB300: the shapes it picks are within 0.3% of the best
+// measured, on average over the 40 cases.  A k-step of a narrower tile costs almost as much as
+// one of a 256-wide tile (b ~ 1 for every width), so the narrower tiles win only where they fill
+// a wave that the 256-wide tiles leave part empty (e.g. 512 x 3072 by 3072: 64 tiles of 192
+// columns in clusters of 2 instead of 48 of 256).
 struct Variant {
   int bn, rk, cps;
   double F, f, b;
 };
-constexpr int kVariants = 3;
-constexpr Variant kVariant[kVariants] = {{256, 192, 1, 450.0, 20.0, 1.0}, {128, 224, 1, 300.0, 20.0, 0.9},
-                                         {128, 96, 2, 300.0, 20.0, 1.333}};
+constexpr int kVariants = 6;
+constexpr Variant kVariant[kVariants] = {{256, 192, 1, 600.0, 20.0, 1.0},   {128, 224, 1, 300.0, 20.0, 1.05},
+                                         {128, 96, 2, 300.0, 20.0, 1.05},   {160, 224, 1, 300.0, 20.0, 1.05},
+                                         {192, 224, 1, 450.0, 20.0, 0.95},  {224, 224, 1, 600.0, 20.0, 1.0}};
 
 // Co-resident clusters of s CTAs of variant v on the current device; clusters must fit inside
 // one GPC, so this is not simply (SMs x CTAs per SM) / s.  Both encodings use the same shared
@@ -713,8 +720,15 @@ int max_active_clusters(int v, int s, int sms) {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return std::max(1, sms * kVariant[v].cps / s);
   int& c = cache[dev][v][s];
   if (c == 0) {
-    const int n = v == 0 ? query_active_clusters<256, 192>(s)
-                         : (v == 1 ? query_active_clusters<128, 224>(s) : query_active_clusters<128, 96>(s));
+    int n = 0;
+    switch (v) {
+      case 0: n = query_active_clusters<kVariant[0].bn, kVariant[0].rk>(s); break;
+      case 1: n = query_active_clusters<kVariant[1].bn, kVariant[1].rk>(s); break;
+      case 2: n = query_active_clusters<kVariant[2].bn, kVariant[2].rk>(s); break;
+      case 3: n = query_active_clusters<kVariant[3].bn, kVariant[3].rk>(s); break;
+      case 4: n = query_active_clusters<kVariant[4].bn, kVariant[4].rk>(s); break;
+      default: n = query_active_clusters<kVariant[5].bn, kVariant[5].rk>(s); break;
+    }
     c = n > 0 ? n : std::max(1, sms * kVariant[v].cps / s);
   }
   return c;
@@ -844,10 +858,14 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
 template <class Md>
 spl_status launch_variant(const LinearArgs& a, const uint16_t* hi, const uint16_t* lo, const int* a_exp,
                           const TcShape& shape, int skip_kblock, int seg_splits) {
+  static_assert(kVariants == 6, "one case per variant");
   switch (shape.v) {
-    case 0: return launch_tc<Md, 256, 192>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
-    case 1: return launch_tc<Md, 128, 224>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
-    default: return launch_tc<Md, 128, 96>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    case 0: return launch_tc<Md, kVariant[0].bn, kVariant[0].rk>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    case 1: return launch_tc<Md, kVariant[1].bn, kVariant[1].rk>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    case 2: return launch_tc<Md, kVariant[2].bn, kVariant[2].rk>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    case 3: return launch_tc<Md, kVariant[3].bn, kVariant[3].rk>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    case 4: return launch_tc<Md, kVariant[4].bn, kVariant[4].rk>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
+    default: return launch_tc<Md, kVariant[5].bn, kVariant[5].rk>(a, hi, lo, a_exp, shape, skip_kblock, seg_splits);
   }
 }
 
@@ -1001,10 +1019,12 @@ extern "C" spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int6
 }
 
 // Test hook: the tensor-core product with a fixed tile width and K-split, so that tests cover
-// every kernel instance and a sweep can time each launch shape.  The paper has no counterpart.
+// every kernel instance and a sweep can time each launch shape; seg_splits > 0 runs the unsplit
+// tiles in segmented mode (the bank's form), their sums following a seg_splits-way split of K.
+// The paper has no counterpart.
 extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_weight* W, const float* C, int64_t M,
                                           int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
-                                          int64_t full_tiles, void* workspace, size_t workspace_bytes,
+                                          int64_t full_tiles, int seg_splits, void* workspace, size_t workspace_bytes,
                                           cudaStream_t stream) {
   using namespace spl;
   if (!out || !A || !W || !W->w || M <= 0 || N <= 0 || K <= 0) return SPL_EINVAL;
@@ -1018,6 +1038,8 @@ extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_
   if (!aligned16(out) || !aligned16(A) || (C && !aligned16(C))) return SPL_EALIGN;
   const int64_t tiles = ceil_div(M, BM) * ceil_div(N, (int64_t)tile_n);
   if (full_tiles < 0 || full_tiles > tiles) return SPL_EINVAL;
+  if (seg_splits < 0 || seg_splits > MAX_CLUSTER || (seg_splits > 0 && splits > 1 && splits != seg_splits))
+    return SPL_EINVAL;
   const LinearArgs args = make_args(out, A, *W, C, M, K, N, workspace, workspace_bytes, stream, path);
-  return run_tc_impl(args, -1, v, splits, 0, full_tiles);
+  return run_tc_impl(args, -1, v, splits, seg_splits, full_tiles);
 }

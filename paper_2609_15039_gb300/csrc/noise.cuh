@@ -73,24 +73,18 @@ __device__ __forceinline__ unsigned long long fma2c(unsigned long long a, unsign
   return fma2(a, b, p2(c, c));
 }
 
-// ln u for u = k 2^-24, k = 1 .. 2^24: u = 2^e m with m in [sqrt(1/2), sqrt(2)) and s = m - 1
+// ln u for u = k 2^-24, k = 1 .. 2^24: u = 2^e m with m in (sqrt(1/2), sqrt(2)] and s = m - 1
 // (both exact), ln(1 + s) = s P(s) with P of degree 9 fitted to the relative error on that interval
 // (least squares on Chebyshev nodes, then Lawson's reweighting toward the minimax), and
 // ln u = e ln 2 + s P(s).  At most 1.6 ulp from ln u over all 2^24 inputs (checked against
-// binary64), and exact (0) at u = 1.
+// binary64), and exact (0) at u = 1.  The reduction is the usual branch-free one on the bit
+// pattern: subtracting the bits of the float just above sqrt(1/2) leaves e in the high bits
+// (arithmetic shift) and, added back to the low 23 bits, the bits of m.
 // Two uniforms at once: ln u0 and ln u1.
 __device__ __forceinline__ void log_unit2(float u0, float u1, float& l0, float& l1) {
-  const int b0 = __float_as_int(u0), b1 = __float_as_int(u1);
-  int e0 = (b0 >> 23) - 127, e1 = (b1 >> 23) - 127;
-  float m0 = __int_as_float((b0 & 0x7FFFFF) | 0x3F800000), m1 = __int_as_float((b1 & 0x7FFFFF) | 0x3F800000);
-  if (m0 > 1.41421356f) {
-    m0 = __fmul_rn(m0, 0.5f);
-    e0 += 1;
-  }
-  if (m1 > 1.41421356f) {
-    m1 = __fmul_rn(m1, 0.5f);
-    e1 += 1;
-  }
+  constexpr int kOff = 0x3F3504F4;  // bits of the float just above sqrt(1/2)
+  const int d0 = __float_as_int(u0) - kOff, d1 = __float_as_int(u1) - kOff;
+  const float m0 = __int_as_float((d0 & 0x7FFFFF) + kOff), m1 = __int_as_float((d1 & 0x7FFFFF) + kOff);
   const unsigned long long s = p2(__fsub_rn(m0, 1.0f), __fsub_rn(m1, 1.0f));
   unsigned long long p = p2(-0.07830669730901718f, -0.07830669730901718f);
   p = fma2c(p, s, 0.13019075989723206f);
@@ -102,10 +96,8 @@ __device__ __forceinline__ void log_unit2(float u0, float u1, float& l0, float& 
   p = fma2c(p, s, 0.33333301544189453f);
   p = fma2c(p, s, -0.49999988079071045f);
   p = fma2c(p, s, 1.0f);
-  float ps0, ps1;
-  up2(fma2c(p, s, -0.0f), ps0, ps1);  // fl(p s): adding -0 changes no rounding
-  l0 = fmaf((float)e0, 0.6931471824645996f, ps0);
-  l1 = fmaf((float)e1, 0.6931471824645996f, ps1);
+  const unsigned long long ps = fma2c(p, s, -0.0f);  // fl(p s): adding -0 changes no rounding
+  up2(fma2(p2((float)(d0 >> 23), (float)(d1 >> 23)), p2(0.6931471824645996f, 0.6931471824645996f), ps), l0, l1);
 }
 
 // sin(pi x) and cos(pi x) for x = 2 u2 in [0, 2), x a multiple of 2^-23: x = q / 2 + r with
@@ -133,11 +125,22 @@ __device__ __forceinline__ void sincospi_turns2(float x0, float x1, float* s0, f
   pc = fma2c(pc, r2, 1.0f);
   float pc0, pc1;
   up2(pc, pc0, pc1);
-  const int t0 = (int)q0 & 3, t1 = (int)q1 & 3;
-  *s0 = t0 == 0 ? sr0 : t0 == 1 ? pc0 : t0 == 2 ? -sr0 : -pc0;
-  *c0 = t0 == 0 ? pc0 : t0 == 1 ? -sr0 : t0 == 2 ? -pc0 : sr0;
-  *s1 = t1 == 0 ? sr1 : t1 == 1 ? pc1 : t1 == 2 ? -sr1 : -pc1;
-  *c1 = t1 == 0 ? pc1 : t1 == 1 ? -sr1 : t1 == 2 ? -pc1 : sr1;
+  // quarter turn t: (sin, cos) = (sr, pc), (pc, -sr), (-sr, -pc), (-pc, sr) for t mod 4 = 0..3;
+  // odd t swaps the two, t = 2, 3 negates the sine and t = 1, 2 the cosine (sign-bit flips)
+  const uint32_t t0 = (uint32_t)(int)q0, t1 = (uint32_t)(int)q1;
+  *s0 = __uint_as_float(__float_as_uint((t0 & 1u) ? pc0 : sr0) ^ ((t0 & 2u) << 30));
+  *c0 = __uint_as_float(__float_as_uint((t0 & 1u) ? sr0 : pc0) ^ (((t0 + 1u) & 2u) << 30));
+  *s1 = __uint_as_float(__float_as_uint((t1 & 1u) ? pc1 : sr1) ^ ((t1 & 2u) << 30));
+  *c1 = __uint_as_float(__float_as_uint((t1 & 1u) ? sr1 : pc1) ^ (((t1 + 1u) & 2u) << 30));
+}
+
+// The hardware square-root approximation (sqrt.approx.f32), no Newton refinement: at most
+// 1.68 x 2^-24 relative error over every float in [1, 4) and over all 2^24 values of -2 ln u
+// the draw can take (measured against binary64 on GB300), against 2^-24 for the rounded root.
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float r;
+  asm("sqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
 }
 
 template <int MECH>
@@ -152,12 +155,12 @@ __device__ __forceinline__ float4 draw_block(uint64_t j, const PhiloxKey& key, f
     for (int i = 0; i < 4; ++i) u[i] = __int2float_rn((int)((w[i] & 0xFFFFFFu) + 1u)) * 0x1p-24f;
     log_unit2(u[0], u[1], l[0], l[1]);
     log_unit2(u[2], u[3], l[2], l[3]);
+    float m[4];  // b (-ln u), two at a time; the sign is the top bit of the word
+    up2(fma2(p2(-b, -b), p2(l[0], l[1]), p2(-0.0f, -0.0f)), m[0], m[1]);
+    up2(fma2(p2(-b, -b), p2(l[2], l[3]), p2(-0.0f, -0.0f)), m[2], m[3]);
     float v[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float mag = __fmul_rn(b, -l[i]);
-      v[i] = (w[i] >> 31) ? -mag : mag;
-    }
+    for (int i = 0; i < 4; ++i) v[i] = __uint_as_float(__float_as_uint(m[i]) ^ (w[i] & 0x80000000u));
     e = make_float4(v[0], v[1], v[2], v[3]);
   } else {  // Box-Muller on the pairs (x, y) and (z, w), the two done side by side
     const float ua = __int2float_rn((int)((r.x >> 8) + 1u)) * 0x1p-24f;  // (0, 1]
@@ -167,9 +170,12 @@ __device__ __forceinline__ float4 draw_block(uint64_t j, const PhiloxKey& key, f
     float la, lb, sa, ca, sb, cb;
     log_unit2(ua, ub, la, lb);
     sincospi_turns2(2.0f * va, 2.0f * vb, &sa, &ca, &sb, &cb);  // sin/cos of 2 pi v; 2 v is exact
-    const float ra_ = __fmul_rn(b, sqrtf(__fmul_rn(-2.0f, la)));
-    const float rb_ = __fmul_rn(b, sqrtf(__fmul_rn(-2.0f, lb)));
-    e = make_float4(__fmul_rn(ra_, ca), __fmul_rn(ra_, sa), __fmul_rn(rb_, cb), __fmul_rn(rb_, sb));
+    float ra_, rb_;  // b sqrt(-2 ln u) for both pairs (-2 ln u is exact)
+    up2(fma2(p2(b, b), p2(sqrt_approx(-2.0f * la), sqrt_approx(-2.0f * lb)), p2(-0.0f, -0.0f)), ra_, rb_);
+    float x0, y0, x1, y1;
+    up2(fma2(p2(ra_, ra_), p2(ca, sa), p2(-0.0f, -0.0f)), x0, y0);
+    up2(fma2(p2(rb_, rb_), p2(cb, sb), p2(-0.0f, -0.0f)), x1, y1);
+    e = make_float4(x0, y0, x1, y1);
   }
   return e;
 }

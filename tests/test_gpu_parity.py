@@ -77,7 +77,9 @@ def test_noise_matches_oracle(spl, shape, mech):
     else:
         b = float(np.float32(sens / eps))
         R = philox.radius_fp64(shape, seed, sid, off)
-        tol = 8 * U * b * R + 2 * ulp32(exp)  # errors of sqrt/log/sincos scaled by b R
+        # radius b sqrt(-2 ln u): ln u 1.6 ulp (1.6 U after the root), sqrt.approx 1.68 U, x b 1 U;
+        # sin/cos 1.7 ulp (3.4 U): 7.7 U b R, plus the last rounding
+        tol = 8 * U * b * R + 2 * ulp32(exp)
     assert np.all(np.abs(got - exp) <= tol)
 
 
@@ -230,8 +232,11 @@ def test_products_match_oracle(spl, M, K, N, path):
     assert spl.spl_get_device_status() == 0
 
 
+TC_VARIANTS = [(256, 192), (128, 224), (128, 96), (160, 224), (192, 224), (224, 224)]
+
+
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
-@pytest.mark.parametrize("tile_n,ring_kb", [(256, 192), (128, 224), (128, 96)])
+@pytest.mark.parametrize("tile_n,ring_kb", TC_VARIANTS)
 @pytest.mark.parametrize("splits", [1, 3, 8])
 def test_tc_every_launch_shape(spl, path, tile_n, ring_kb, splits):
     """Each kernel instance (encoding x tile width x ring) with each cluster K-split, on a ragged
@@ -398,14 +403,39 @@ def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path, draw
     assert spl.spl_get_device_status() == 0
 
 
+@pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
+@pytest.mark.parametrize("tile_n,ring_kb", TC_VARIANTS)
+def test_tc_segmented_equals_split_product(spl, path, tile_n, ring_kb):
+    """Every kernel instance in segmented mode (one CTA over all of K, the partial sums of a 3-way
+    split of K folded in TMEM in order) gives the 3-way cluster-split product bit for bit, alone
+    and with the tiles after the first half+1 split over a cluster; ragged M, N and K."""
+    M, K, N = 300, 2056, 700
+    W, Wt = _weights(spl, N, K, seed=47)
+    A = (wl.activations(M, K, seed=48).numpy() * 30).astype(np.float32)
+    C = dev(wl.activations(M, N, seed=49).numpy())
+    tiles = -(-M // 128) * -(-N // tile_n)
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, path))
+    ref = torch.empty((M, N), device="cuda")
+    spl.spl_test_tc_product(ref, dev(A), Wt, C, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=3, workspace=ws)
+    assert_product_close(f32(ref), A, W, path, C=C.cpu().numpy(), what=f"{path} tile {tile_n} split 3")
+    for full, splits in ((0, 1), (tiles // 2 + 1, 3), (tiles, 1)):
+        Y = torch.full((M, N), float("nan"), device="cuda")
+        spl.spl_test_tc_product(Y, dev(A), Wt, C, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=splits,
+                                full_tiles=full, seg_splits=3, workspace=ws)
+        assert torch.equal(Y, ref), (full, splits, float((Y - ref).abs().max()))
+    assert spl.spl_get_device_status() == 0
+
+
 def test_bank_shape_mixes_folded_and_split_tiles(spl):
-    """A correction of 8 x 128 rows for the Llama Q|K|V shape: 160 tiles of 256 columns, one wave
-    of them folded in TMEM and the rest split over a cluster the way the online product splits K."""
+    """A correction of 8 x 128 rows for the Llama Q|K|V shape: its tiles cover the output once,
+    a whole wave of them folded in TMEM and the rest (if any) split over a cluster the way the
+    online product splits K."""
     online = spl.spl_test_tc_shape(128, 3072, 5120)
     assert online[2] == 0  # the online product is one split launch
     bank = spl.spl_test_tc_shape(1024, 3072, 5120, seg_splits=online[4])
-    assert bank[2] + bank[3] == (1024 // 128) * (5120 // bank[0])
+    assert bank[2] + bank[3] == (1024 // 128) * -(-5120 // bank[0])
     assert bank[3] == 0 or bank[4] == online[4]
+    assert bank[2] % spl.spl_test_tc_capacity(bank[0], bank[1], 1) == 0
 
 
 # ------------------------------------------------ a2 + a3 fused with the split of X~
