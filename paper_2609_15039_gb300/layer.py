@@ -220,15 +220,18 @@ class MaskedLayer:
         self.rng_base.copy_(base)
 
     def refill(self, eps, mech, seed, cycle, path="auto", stream=None, timer=None, device_base=False,
-               parallel=False, parity=0, ahead=0):
+               parallel=False, parity=0, ahead=0, workspace=None):
         """a2 + a4: draw ``draws`` masks per group and precompute their corrections in one product.
 
         parallel: the FP16X3 groups' corrections (which use no workspace: the noise comes split and
         the tensor-core kernel reduces on chip) run side by side on streams of their own, so the
         tiles of one fill the SMs another leaves idle; the current stream waits for all of them.
         parity: the correction buffer to fill (see enable_overlap); ahead: the draws of cycle
-        ``cycle + ahead`` (with device_base: that many cycles past the device-side base)."""
+        ``cycle + ahead`` (with device_base: that many cycles past the device-side base).
+        workspace: the workspace of the corrections that take one (default: the layer's), e.g. a
+        second one while online steps run beside them."""
         main = torch.cuda.current_stream() if stream is None else stream
+        ws = self.workspace if workspace is None else workspace
         forks = []
         for gi, g in enumerate(self.groups):
             b = self.bank[g.name]
@@ -259,11 +262,11 @@ class MaskedLayer:
             if timer:
                 timer("begin", "precompute", g.name)
             if g.name in self.fp64:
-                spl.spl_precompute_noise_product_f64(C, b["eta"], g.W, workspace=self.workspace, stream=stream)
+                spl.spl_precompute_noise_product_f64(C, b["eta"], g.W, workspace=ws, stream=stream)
             else:
                 # summed in the order the online product of M rows uses, so their rounding cancels
                 spl.spl_precompute_noise_product_matched(C, b["eta"], g.wt, self.M,
-                                                         path=self.path_of(g, path, self.M), workspace=self.workspace,
+                                                         path=self.path_of(g, path, self.M), workspace=ws,
                                                          stream=stream)
             if timer:
                 timer("end", "precompute", g.name)
@@ -503,6 +506,53 @@ class MaskedStack:
             graphs.append(graph)
             launches.append(spl.spl_launch_count() - n0)
         return graphs, launches
+
+    def capture_overlapped(self, inputs, eps, mech, bank_workspace, path="auto", after=None):
+        """Two CUDA graphs, each a whole bank cycle of the stack: graph p runs the ``draws`` steps
+        through every layer on correction buffers p while, on a stream of lower priority, the next
+        cycle's corrections of every layer are computed into buffers 1 - p, with a workspace of their
+        own (``bank_workspace``, at least max(layer.workspace_bytes(M, draws))).  The graph ends when
+        both are done and moves every Philox base on by one cycle.  Replay graphs[c % 2] for cycle
+        c after set_cycle(c) and a refill of buffers c % 2 for cycle c (start_overlapped).
+        ``after(d)`` is called after step d's launches (e.g. to copy its results inside the graph).
+        Returns the graphs and their kernel counts."""
+        lo, hi = torch.cuda.Stream.priority_range()
+        if not hasattr(self, "_bank_stream"):
+            self._bank_stream = torch.cuda.Stream(priority=lo)
+            self._online_stream = torch.cuda.Stream(priority=hi)
+        for layer in self.layers:
+            layer.enable_overlap()
+        D = self.draws
+        graphs, launches = [], []
+        for parity in range(2):
+            graph = torch.cuda.CUDAGraph()
+            n0 = spl.spl_launch_count()
+            with torch.cuda.graph(graph, stream=self._online_stream):
+                main = torch.cuda.current_stream()
+                self._bank_stream.wait_stream(main)
+                with torch.cuda.stream(self._bank_stream):
+                    for layer, seed in zip(self.layers, self.seeds):
+                        layer.refill(eps, mech, seed, 0, path=path, device_base=True, parity=1 - parity, ahead=1,
+                                     workspace=bank_workspace)
+                for d in range(D):
+                    for layer, x, seed in zip(self.layers, inputs, self.seeds):
+                        layer.online(x, eps, mech, seed, 0, d, path=path, device_base=True, parity=parity)
+                    if after:
+                        after(d)
+                main.wait_stream(self._bank_stream)
+                for layer in self.layers:
+                    for gi, g in enumerate(layer.groups):
+                        spl.spl_rng_advance(layer.rng_base[gi:gi + 1], D * (layer.M * g.K // 4))
+            graphs.append(graph)
+            launches.append(spl.spl_launch_count() - n0)
+        return graphs, launches
+
+    def start_overlapped(self, cycle, eps, mech, path="auto"):
+        """Before replaying the overlapped graphs from bank cycle ``cycle``: the device-side Philox
+        bases at ``cycle`` and that cycle's corrections in buffers cycle % 2."""
+        self.set_cycle(cycle)
+        for layer, seed in zip(self.layers, self.seeds):
+            layer.refill(eps, mech, seed, 0, path=path, device_base=True, parity=cycle % 2)
 
     def flops_per_step(self):
         return sum(l.flops_per_step() for l in self.layers)

@@ -118,3 +118,50 @@ def test_overlapped_cycle_graphs_equal_eager_steps(spl):
     exp_base = [layer.block_offset(g, first + cycles, 0) for g in layer.groups]
     assert layer.rng_base.cpu().tolist() == exp_base
     assert spl.spl_get_device_status() == 0
+
+
+def test_stack_overlapped_decode_graphs_equal_eager_steps(spl):
+    """The stack's whole-cycle graphs -- every layer's next-cycle corrections on a stream of lower
+    priority with a workspace of their own -- give the eager steps' results bit for bit on the FP32
+    decode path (one row), where both the products and the corrections use a workspace: across
+    three cycles, so each correction buffer is filled by one graph and read by the other."""
+    from paper_2609_15039_gb300.layer import MaskedStack
+    model = wl.ModelShape("small", 2, 512, 1024, 512, 256, 1000)
+    draws, eps, mech, M = 3, 1.0, "laplace", 1
+    stack = MaskedStack.build(model, 2, M, draws, base_seed=5, power_iters=50)
+    inputs = stack.inputs(6)
+
+    def eager(s):
+        cycle, d = divmod(s, draws)
+        res = []
+        for layer, x, seed in zip(stack.layers, inputs, stack.seeds):
+            if d == 0:
+                layer.refill(eps, mech, seed, cycle)
+            res.append({g: y.clone() for g, y in layer.online(x, eps, mech, seed, cycle, d).items()})
+        return res
+
+    first, cycles = 2, 3
+    expected = [eager(s) for s in range(first * draws, (first + cycles) * draws)]
+    torch.cuda.synchronize()
+    outs = []
+
+    def after(d):
+        outs.append([{g.name: l.bank[g.name]["Y"].clone() for g in l.groups} for l in stack.layers])
+
+    bank_ws = spl.workspace(max(l.workspace_bytes(M, draws) for l in stack.layers))
+    graphs, launches = stack.capture_overlapped(inputs, eps, mech, bank_ws, after=after)
+    assert len(graphs) == 2 and all(n > 0 for n in launches)
+    captured = list(outs)
+    stack.start_overlapped(first, eps, mech)
+    for i in range(cycles):
+        c = first + i
+        graphs[c % 2].replay()
+        torch.cuda.synchronize()
+        for d in range(draws):
+            got = captured[(c % 2) * draws + d]
+            for li in range(len(stack.layers)):
+                for g in got[li]:
+                    assert torch.equal(got[li][g], expected[i * draws + d][li][g]), (c, d, li, g)
+    for layer in stack.layers:
+        assert layer.rng_base.cpu().tolist() == [layer.block_offset(g, first + cycles, 0) for g in layer.groups]
+    assert spl.spl_get_device_status() == 0
