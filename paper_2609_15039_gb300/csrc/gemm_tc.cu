@@ -109,7 +109,11 @@ struct Cfg {
   static_assert(STAGES >= 3 && STAGES <= 8, "ring depth");
   static_assert(SMEM <= 232448, "227 KB of dynamic shared memory per block");
   static_assert((size_t)BM * RED_STRIDE * 4 <= RING, "staging fits in the stage ring");
-  static_assert(8 * (2 * STAGES + 3) + 16 <= 1024 && 1024 + 4 * BN <= AUX_BYTES, "aux fits");
+  static_assert(8 * (2 * STAGES + 4) + 16 <= 1024 && 1024 + 4 * BN <= AUX_BYTES, "aux fits");
+  // TMA epilogue (unsplit tiles): the tile as BN / 32 chunks of 128 rows x 32 fp32 (128-byte
+  // swizzle), C loaded into them and the result stored from them, in the ring once the MMAs are done
+  static constexpr uint32_t EPI_CHUNK = BM * 32 * 4;
+  static_assert(BN % 32 == 0 && (BN / 32) * EPI_CHUNK <= RING, "epilogue chunks fit in the ring");
 };
 
 // Shared-memory matrix descriptor for a K-major operand tile with the 64-byte swizzle:
@@ -189,6 +193,19 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
       : "memory");
+}
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void tma_store_commit_wait() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");  // the writes are done, not only the reads
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
@@ -288,6 +305,7 @@ __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
 
 struct TcMaps {
   CUtensorMap a_hi, a_lo, w_hi, w_lo;
+  CUtensorMap y, c;  // TMA epilogue: the output and C as [M, N] fp32, 32 x 128 boxes, 128-byte swizzle
 };
 
 // Rows r0..r1 of the staged tile: the S partial tiles of the cluster summed in rank order (S = 1:
@@ -352,7 +370,10 @@ __device__ __forceinline__ void reduce_store(const float* red, int r0, int r1, i
 // One CTA computes a 128 x BN tile of out over the K range of its split (blockIdx.z).
 // The `splits` CTAs of a tile form one thread-block cluster (z dimension); their fp32
 // partial tiles are summed through distributed shared memory in cluster-rank order, so
-// the result does not depend on timing.
+// the result does not depend on timing.  An unsplit tile whose output rows are whole 16-byte
+// units ends through TMA instead: C's tile is copied into the idle ring, the epilogue warps
+// subtract it in place from the accumulator rows they read out of TMEM, and the tile is
+// copied out (same arithmetic, same result as the thread loop).
 // Segmented mode (seg_blocks > 0, one CTA per tile over all of K): the K range is cut into
 // segments of seg_blocks stages, the same boundaries a K-split of the same problem uses; the
 // first segment accumulates into R (TMEM columns 0..BN-1), every later one into P (columns
@@ -363,15 +384,16 @@ template <class Md, int BN, int RK>
 __global__ void __launch_bounds__(THREADS, Cfg<Md, BN, RK>::CTAS_PER_SM)
 tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
                const int* __restrict__ a_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
-               int64_t k_per_split, int splits, int tile_base, int m_tiles, int skip_kblock, int seg_blocks) {
+               int64_t k_per_split, int splits, int tile_base, int m_tiles, int skip_kblock, int seg_blocks,
+               int epi_tma) {
   using L = Cfg<Md, BN, RK>;
   constexpr int STAGES = L::STAGES, BK = Md::BK, RED_STRIDE = L::RED_STRIDE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* aux = smem + L::RING;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], empty[S], accum, seg, fold
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (2 * STAGES + 3));
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (2 * STAGES + 3) + 8);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], empty[S], accum, seg, fold, c_load
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (2 * STAGES + 4));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (2 * STAGES + 4) + 8);
   float* red = reinterpret_cast<float*>(smem);  // [BM][RED_STRIDE] staged accumulator, after the mainloop
   float* col_scale = reinterpret_cast<float*>(aux + 1024);  // [BN] FP16X3: 2^-e of the tile's W rows
 
@@ -390,6 +412,9 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   const uint32_t accum_bar = bar_base + 8u * (2 * STAGES);
   const uint32_t seg_bar = bar_base + 8u * (2 * STAGES + 1);   // segmented: a later segment is in P
   const uint32_t fold_bar = bar_base + 8u * (2 * STAGES + 2);  // segmented: P folded into R
+  const uint32_t cload_bar = bar_base + 8u * (2 * STAGES + 3);  // TMA epilogue: the tile of C landed
+  // TMA epilogue: unsplit tiles whose output rows are whole 16-byte units (chosen by the host)
+  const bool tma_epi = epi_tma != 0 && splits == 1;
   const int seg_len = seg_blocks > 0 ? seg_blocks : nk + 1;    // stages per segment
   const int nseg = seg_blocks > 0 ? (int)ceil_div(nk, seg_blocks) : 1;
   const uint32_t tmem_cols = seg_blocks > 0 ? L::TMEM_COLS_SEG : L::TMEM_COLS;
@@ -402,6 +427,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     mbar_init(accum_bar, 1);
     mbar_init(seg_bar, 1);
     mbar_init(fold_bar, 4);  // one arrival per epilogue warp
+    mbar_init(cload_bar, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -558,7 +584,63 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     bool have = ok && (nk == 0 || mbar_wait(accum_bar, 0u, kWaitNs * 4, abort_flag));
     have = __all_sync(0xffffffffu, have) && !*abort_flag;
     pdl_trigger();
-    if (have) {
+    if (have && tma_epi) {
+      // The MMAs are done with the ring: C's tile comes in by TMA as BN / 32 chunks of 128 rows x
+      // 32 columns (128-byte swizzle: the 16-byte unit j of row r sits at unit j ^ (r & 7), so the
+      // eight rows a quarter-warp touches hit eight different bank groups); each thread takes its
+      // row from TMEM, scales it, subtracts C in place, and TMA stores the chunks (rows and columns
+      // past M and N are clipped by the copy).
+      tc_fence_after();
+      const int r = 32 * q + lane;
+      const float sr = pow2f(-e_row);
+      // chunks holding columns below N (the copies start inside the tensor)
+      const int nchunks = (int)std::min<int64_t>(BN / 32, ceil_div(N - n0, (int64_t)32));
+      if (C && t == 0) {
+        mbar_expect_tx(cload_bar, (uint32_t)nchunks * L::EPI_CHUNK);
+        const uint64_t pol_c = l2_evict_first();
+        for (int c = 0; c < nchunks; ++c)
+          tma_load_2d(smem_u32(smem + (size_t)c * L::EPI_CHUNK), &maps.c, cload_bar, (int)n0 + 32 * c, (int)m0, pol_c);
+      }
+      bool okc = !C || mbar_wait(cload_bar, 0u, kWaitNs, abort_flag);
+      okc = __all_sync(0xffffffffu, okc) && !*abort_flag;
+      if (okc) {
+#pragma unroll 1
+        for (int c = 0; c < nchunks; ++c) {
+          float v[32];
+          if (nk > 0) {
+            tmem_ld_32x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(32 * c), v);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+          }
+          if constexpr (Md::kF16) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = (v[i] * sr) * col_scale[32 * c + i];  // exact power-of-two scaling
+          }
+          float4* row = reinterpret_cast<float4*>(smem + (size_t)c * L::EPI_CHUNK + (size_t)r * 128);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float4 o = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+            float4* dst = row + (j ^ (r & 7));
+            if (C) {
+              const float4 cc = *dst;
+              o = make_float4(__fsub_rn(o.x, cc.x), __fsub_rn(o.y, cc.y), __fsub_rn(o.z, cc.z), __fsub_rn(o.w, cc.w));
+            }
+            *dst = o;
+          }
+        }
+        fence_proxy_async_smem();  // these writes before the copies that read them
+        epilogue_sync();
+        if (t == 0) {
+          for (int c = 0; c < nchunks; ++c)
+            tma_store_2d(&maps.y, smem_u32(smem + (size_t)c * L::EPI_CHUNK), (int)n0 + 32 * c, (int)m0);
+          tma_store_commit_wait();
+        }
+      } else if (lane == 0) {
+        *abort_flag = 1;
+        atomicOr(&g_device_status, kStatusTimeout);
+      }
+    } else if (have) {
       tc_fence_after();
       const int r = 32 * q + lane;
       float* row = red + (size_t)r * RED_STRIDE;
@@ -594,7 +676,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   } else {
     __syncthreads();
   }
-  {
+  if (!tma_epi) {
     const int rank = splits > 1 ? (int)cluster_rank() : 0;
     const int rows_per_rank = (BM + splits - 1) / splits;
     const int r0 = rank * rows_per_rank, r1 = (r0 + rows_per_rank < BM) ? r0 + rows_per_rank : BM;
@@ -676,7 +758,7 @@ bool set_smem_attr() {
 // (F: setup, pipeline fill and epilogue of a CTA; f: the cluster reduction per rank; b: the
 // mainloop per K element, relative to the 256-wide tile with the 192 KB ring), fitted to a sweep
 // of every variant, split and whole-wave form over the eight Llama and Qwen projections at 128,
-// 512, 1024, 2048 and 4096 rows on GB300: the shapes it picks are within 0.3% of the best
+// 512, 1024, 2048 and 4096 rows on GB300: the shapes it picks are within 0.35% of the best
 // measured, on average over the 40 cases.  A k-step of a narrower tile costs almost as much as
 // one of a 256-wide tile (b ~ 1 for every width), so the narrower tiles win only where they fill
 // a wave that the 256-wide tiles leave part empty (e.g. 512 x 3072 by 3072: 64 tiles of 192
@@ -686,9 +768,9 @@ struct Variant {
   double F, f, b;
 };
 constexpr int kVariants = 6;
-constexpr Variant kVariant[kVariants] = {{256, 192, 1, 600.0, 20.0, 1.0},   {128, 224, 1, 300.0, 20.0, 1.05},
-                                         {128, 96, 2, 300.0, 20.0, 1.05},   {160, 224, 1, 300.0, 20.0, 1.05},
-                                         {192, 224, 1, 450.0, 20.0, 0.95},  {224, 224, 1, 600.0, 20.0, 1.0}};
+constexpr Variant kVariant[kVariants] = {{256, 192, 1, 500.0, 20.0, 1.0},   {128, 224, 1, 300.0, 20.0, 1.05},
+                                         {128, 96, 2, 250.0, 20.0, 0.95},   {160, 224, 1, 250.0, 20.0, 1.05},
+                                         {192, 224, 1, 300.0, 20.0, 1.0},   {224, 224, 1, 500.0, 20.0, 1.0}};
 
 // Co-resident clusters of s CTAs of variant v on the current device; clusters must fit inside
 // one GPC, so this is not simply (SMs x CTAs per SM) / s.  Both encodings use the same shared
@@ -819,6 +901,13 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
       !make_map(&maps.w_hi, whi, f16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B) ||
       !make_map(&maps.w_lo, wlo, f16, a.N, a.K, Md::BK, BN, CU_TENSOR_MAP_SWIZZLE_64B))
     return SPL_ECUDA;
+  // TMA epilogue for unsplit tiles: needs output rows (and C's) of whole 16-byte units
+  int epi_tma = (a.N & 3) == 0 && aligned16(a.out) && (!a.c || aligned16(a.c)) ? 1 : 0;
+  if (epi_tma) {
+    if (!make_map(&maps.y, a.out, false, a.M, a.N, 32, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        (a.c && !make_map(&maps.c, a.c, false, a.M, a.N, 32, BM, CU_TENSOR_MAP_SWIZZLE_128B)))
+      return SPL_ECUDA;
+  }
   const int m_tiles = (int)ceil_div(a.M, BM);
   // The first launch follows the split of A under programmatic dependent launch: its CTAs start
   // (barriers, TMEM, weight tiles) while the split finishes.
@@ -844,7 +933,7 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
     first = false;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md, BN, RK>, maps, a.out, a.c, a_exp,
                                              (const int*)a.w_exp, a.M, a.K, a.N, kps, splits, (int)base, m_tiles,
-                                             skip_kblock, seg);
+                                             skip_kblock, seg, epi_tma);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   };

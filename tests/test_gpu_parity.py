@@ -403,6 +403,30 @@ def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path, draw
     assert spl.spl_get_device_status() == 0
 
 
+@pytest.mark.parametrize("tile_n,ring_kb", [(256, 192), (224, 224), (128, 96)])
+@pytest.mark.parametrize("N", [600, 601])
+def test_tc_unsplit_epilogue_on_ragged_rows(spl, tile_n, ring_kb, N):
+    """Unsplit tiles store through TMA when an output row is a whole number of 16-byte units
+    (N = 600) and through the thread loop otherwise (N = 601): in segmented mode (the K ranges of a
+    2-way split folded in order) both give the 2-way cluster-split product bit for bit, whose
+    reduction always stores through the thread loop; with and without C, ragged M and N."""
+    M, K = 131, 1040
+    W, Wt = _weights(spl, N, K, seed=53)
+    A = wl.activations(M, K, seed=54).numpy()
+    C = dev(wl.activations(M, N, seed=55).numpy())
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp16x3"))
+    for Cx in (C, None):
+        ref = torch.empty((M, N), device="cuda")
+        spl.spl_test_tc_product(ref, dev(A), Wt, Cx, tile_n=tile_n, ring_kb=ring_kb, splits=2, workspace=ws)
+        assert_product_close(f32(ref), A, W, "fp16x3", C=None if Cx is None else C.cpu().numpy(),
+                             what=f"N {N} split 2")
+        Y = torch.full((M, N), float("nan"), device="cuda")
+        spl.spl_test_tc_product(Y, dev(A), Wt, Cx, tile_n=tile_n, ring_kb=ring_kb, splits=1, seg_splits=2,
+                                workspace=ws)
+        assert torch.equal(Y, ref), float((Y - ref).abs().max())
+    assert spl.spl_get_device_status() == 0
+
+
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 @pytest.mark.parametrize("tile_n,ring_kb", TC_VARIANTS)
 def test_tc_segmented_equals_split_product(spl, path, tile_n, ring_kb):
