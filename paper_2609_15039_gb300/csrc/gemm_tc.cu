@@ -760,8 +760,8 @@ bool set_smem_attr() {
 // (F: setup, pipeline fill and epilogue of a CTA; f: the cluster reduction per rank; b: the
 // mainloop per K element, relative to the 256-wide tile with the 192 KB ring), fitted to a sweep
 // of every variant, split and whole-wave form over the eight Llama and Qwen projections at 128,
-// 512, 1024, 2048 and 4096 rows on GB300: the shapes it picks are within 0.35% of the best
-// measured, on average over the 40 cases.  A k-step of a narrower tile costs almost as much as
+// 512, 1024, 2048 and 4096 rows on GB300: the shapes it picks (ties going to the earlier variant,
+// as below) are within 0.5% of the best measured, on average over the 40 cases.  A k-step of a narrower tile costs almost as much as
 // one of a 256-wide tile (b ~ 1 for every width), so the narrower tiles win only where they fill
 // a wave that the 256-wide tiles leave part empty (e.g. 512 x 3072 by 3072: 64 tiles of 192
 // columns in clusters of 2 instead of 48 of 256).
@@ -772,7 +772,7 @@ struct Variant {
 constexpr int kVariants = 6;
 constexpr Variant kVariant[kVariants] = {{256, 192, 1, 500.0, 20.0, 1.0},   {128, 224, 1, 300.0, 20.0, 1.05},
                                          {128, 96, 2, 250.0, 20.0, 0.95},   {160, 224, 1, 250.0, 20.0, 1.05},
-                                         {192, 224, 1, 300.0, 20.0, 1.0},   {224, 224, 1, 500.0, 20.0, 1.0}};
+                                         {192, 224, 1, 300.0, 20.0, 1.0},   {224, 224, 1, 550.0, 20.0, 0.97}};
 
 // Co-resident clusters of s CTAs of variant v on the current device; clusters must fit inside
 // one GPC, so this is not simply (SMs x CTAs per SM) / s.  Both encodings use the same shared
