@@ -486,19 +486,22 @@ class MaskedStack:
         for layer in self.layers:
             layer.set_cycle(cycle)
 
-    def capture(self, inputs, eps, mech, path="auto", refill=True):
+    def capture(self, inputs, eps, mech, path="auto", refill=True, timer=None):
         """CUDA graphs of one bank cycle for the whole stack (see MaskedLayer.capture); graph 0
-        refills every layer's bank first unless ``refill`` is False."""
+        refills every layer's bank first unless ``refill`` is False.  ``timer(d, li, phase, kind,
+        group)``, when given, is called around every library call of the online steps (e.g. to put
+        CUDA events into the graphs)."""
         graphs, launches = [], []
         D = self.draws
         for d in range(D):
             graph = torch.cuda.CUDAGraph()
             n0 = spl.spl_launch_count()
             with torch.cuda.graph(graph):
-                for layer, x, seed in zip(self.layers, inputs, self.seeds):
+                for li, (layer, x, seed) in enumerate(zip(self.layers, inputs, self.seeds)):
                     if d == 0 and refill:
                         layer.refill(eps, mech, seed, 0, path=path, device_base=True, parallel=True)
-                    layer.online(x, eps, mech, seed, 0, d, path=path, device_base=True)
+                    t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) if timer else None
+                    layer.online(x, eps, mech, seed, 0, d, path=path, device_base=True, timer=t)
                 if d == D - 1:
                     for layer in self.layers:
                         for gi, g in enumerate(layer.groups):

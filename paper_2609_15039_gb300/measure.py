@@ -92,9 +92,12 @@ def _bound(stack, inputs, eps, mech, s, layers):
     return res
 
 
-def _prefill(stack, inputs, eps, mech, cycles=2):
+def _prefill(stack, inputs, eps, mech, cycles=2, product_times=False):
     """Graph-replayed prefill: online-only steps (draws 1..D-1) and the draw-0 step that also
-    refills every bank; returns ms per online pass and per refill."""
+    refills every bank; returns ms per online pass and per refill.  product_times: also the ms per
+    online pass spent in the masked products alone, from a second pass over the same steps whose
+    graphs hold a CUDA event pair around every product call (an event node keeps the next kernel
+    from starting early, so this slightly over-counts)."""
     stream = torch.cuda.current_stream()
     D = stack.draws
     stack.step(inputs, eps, mech, 0)  # sets up every library call before capture
@@ -109,7 +112,24 @@ def _prefill(stack, inputs, eps, mech, cycles=2):
     rf = sum(with_refill) / len(with_refill) - (on if online else 0.0)
     del graphs
     torch.cuda.synchronize()
-    return on, rf, launches
+    if not product_times:
+        return on, rf, launches
+    ev = {}
+
+    def timer(d, li, phase, kind, group):
+        if kind != "masked_linear_unmask":
+            return
+        e = torch.cuda.Event(enable_timing=True, external=True)
+        e.record()
+        ev.setdefault((d, li, group), [None, None])[0 if phase == "begin" else 1] = e
+
+    ev_graphs, _ = stack.capture(inputs, eps, mech, timer=timer)
+    stack.set_cycle(1)
+    _time_replays(ev_graphs, 0, D, stream)  # one cycle: each graph's events hold its last replay
+    prod = sum(b.elapsed_time(e) for (d, li, g), (b, e) in ev.items() if d != 0) / max(1, D - 1)
+    del ev_graphs
+    torch.cuda.synchronize()
+    return on, rf, launches, prod
 
 
 def llama_stack(layers=28, tokens=512, decode_steps=256, eps=1.0, mech="laplace", draws=8):
@@ -119,11 +139,16 @@ def llama_stack(layers=28, tokens=512, decode_steps=256, eps=1.0, mech="laplace"
     inputs = stack.inputs(11)
     _calibrate(stack, inputs, eps, mech)
     paths = _group_paths(stack, tokens)
-    on_ms, refill_ms, launches = _prefill(stack, inputs, eps, mech)
+    on_ms, refill_ms, launches, prod_ms = _prefill(stack, inputs, eps, mech, product_times=True)
     flops = 2 * tokens * model.weights_per_layer() * layers
     peak = flops / sum(2 * tokens * g.K * g.N * layers / _path_peak(paths[g.name], pk) for g in stack.layers[0].groups)
     prefill = {"ms_per_prefill": on_ms, "tflops": flops / (on_ms * 1e-3) / 1e12, "tokens_per_s": tokens / (on_ms * 1e-3),
                "roofline_peak_tflops": peak, "frac": flops / (on_ms * 1e-3) / 1e12 / peak,
+               "gemm": {"ms": prod_ms, "tflops": flops / (prod_ms * 1e-3) / 1e12,
+                        "frac": flops / (prod_ms * 1e-3) / 1e12 / peak,
+                        "timing": "the masked products alone (tensor-core kernels with fused unmask), CUDA event "
+                                  "pairs around each product call in a second pass over the same graph-replayed "
+                                  "steps; the mask + split kernels between them are the rest of ms_per_prefill"},
                "bank_refill_ms": refill_ms, "bank_refill_ms_per_draw": refill_ms / draws,
                "bank_refill_tflops": draws * flops / (refill_ms * 1e-3) / 1e12, "paths": paths,
                "kernels_per_online_step": launches[1] if len(launches) > 1 else launches[0]}
@@ -180,12 +205,14 @@ def qwen_stack(layers=36, tokens=2048, eps_list=(0.1, 1.0, 10.0), mech="gaussian
     for eps in eps_list:
         _calibrate(stack, inputs, eps, mech)
         paths = _group_paths(stack, tokens)
-        on_ms, refill_ms, _ = _prefill(stack, inputs, eps, mech, cycles=2)
+        on_ms, refill_ms, _, prod_ms = _prefill(stack, inputs, eps, mech, cycles=2, product_times=True)
         peak = flops / sum(2 * tokens * g.K * g.N * layers / _path_peak(paths[g.name], pk)
                            for g in stack.layers[0].groups)
         res[f"eps={eps}"] = {
             "ms_per_prefill": on_ms, "tflops": flops / (on_ms * 1e-3) / 1e12, "tokens_per_s": tokens / (on_ms * 1e-3),
             "roofline_peak_tflops": peak, "frac": flops / (on_ms * 1e-3) / 1e12 / peak,
+            "gemm": {"ms": prod_ms, "tflops": flops / (prod_ms * 1e-3) / 1e12,
+                     "frac": flops / (prod_ms * 1e-3) / 1e12 / peak},
             "bank_refill_ms_per_draw": refill_ms / draws, "paths": paths,
             "bound_check": _bound(stack, inputs, eps, mech, 5 * draws + 1, [0, layers - 1])}
     return {"workload": f"qwen3-4b-shaped stack, {layers} layers, prefill {tokens} tokens, {mech}, "
