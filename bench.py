@@ -50,6 +50,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-overlap", action="store_true",
                     help="compute each bank cycle's corrections before its steps instead of during the previous cycle")
+    ap.add_argument("--stored-noise", action="store_true",
+                    help="keep the bank's fp32 noise and mask each step with it instead of drawing it again")
     ap.add_argument("--workload", default="llama_layer",
                     choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep", "down_fp64", "slalom"],
                     help="llama_layer (default): the headline line; the others measure the stack and sweep "
@@ -265,7 +267,7 @@ def main():
                enumerate(model.projections())}
     layer = MaskedLayer.from_weights(model, weights, split=True, device=dev)
     layer.sensitivities()
-    layer.allocate(M, DRAWS, args.path)
+    layer.allocate(M, DRAWS, args.path, stored_noise=args.stored_noise)
     inputs = {g: wl.activations(M, K, seed=100 + gi, device=dev) for gi, (g, K, _n) in
               enumerate(model.input_groups())}
     if args.path == "auto":
@@ -528,6 +530,8 @@ def main():
                    "bank_schedule": ("each cycle's corrections computed during the previous cycle's steps, on "
                                      "lower-priority streams (whole-cycle graphs)") if use_ov else
                                     "each cycle's corrections computed before its first step",
+                   "online_noise": ("kept from the bank refill, read by each step's mask" if args.stored_noise
+                                    else "drawn again in each step's mask"),
                    "l2": "weights 1.2 GB per step > 129 MB L2 (no flush needed)",
                    "parallelism": "replicas" if world > 1 else "single"},
         "ms_per_prefill_28_layers": 28 * ms,

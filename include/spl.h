@@ -146,6 +146,19 @@ spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* 
                                 int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech,
                                 spl_rng rng, cudaStream_t stream);
 
+/* ---- a3 with a stored noise, fused with the fp16 split of X~ -------------
+ * Xt = fl32(X + N) elementwise (Sec. 3.3.1, the mask with a noise drawn earlier,
+ * e.g. written by spl_noise_mask_split with X NULL while a bank of corrections
+ * was precomputed), written to Xt unless it is NULL, and its FP16X3 split as
+ * spl_split_fp16 would write it: hi, lo [rows, cols] binary16 and row_exp
+ * [rows].  With N = the noise spl_noise_mask_split draws for the same rows, the
+ * outputs equal spl_noise_mask_split's bit for bit.  X, N [rows, cols] fp32,
+ * device, not aliasing the outputs.  One pass, one block per row.  Errors:
+ * EINVAL for negative sizes or NULL hi / lo / row_exp / X / N; EALIGN for
+ * cols % 8 != 0 or a pointer not 16-byte aligned; ESHAPE for cols > 16384. */
+spl_status spl_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,
+                          const float* N, int64_t rows, int64_t cols, cudaStream_t stream);
+
 /* ---- weight preparation for TF32X3 ------------------------------------
  * hi = src rounded to TF32 (10 explicit mantissa bits, ties away), lo = src - hi
  * (exact in fp32).  Done once per weight; hi and lo are [count] like src. */

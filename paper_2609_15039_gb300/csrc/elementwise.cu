@@ -272,8 +272,10 @@ __global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restri
 // thread, all loads issued before any is used, so a row costs one memory round trip.
 // MECH >= 0: the row is first masked (a2 + a3 fused into the split): xt = fl32(x + eta) with eta
 // drawn exactly as noise_mask_kernel draws it (element e: lane e % 4 of Philox block e / 4 +
-// offset), written to xt_out when it is not NULL, then split.
+// offset), written to xt_out when it is not NULL, then split.  MECH == kStored: eta is read
+// from `stored` (a noise drawn earlier, e.g. with a bank of corrections), xt = fl32(x + eta).
 constexpr int kNoMask = -1;
+constexpr int kStored = 3;
 
 template <int CH, int MECH>
 __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __restrict__ hi,
@@ -281,7 +283,8 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
                                                                    int* __restrict__ row_exp,
                                                                    const float* __restrict__ src, int64_t cols,
                                                                    float* __restrict__ xt_out, float b, const __grid_constant__ PhiloxKey key,
-                                                                   uint64_t offset_host, const uint64_t* offset_dev) {
+                                                                   uint64_t offset_host, const uint64_t* offset_dev,
+                                                                   const float* __restrict__ stored) {
   pdl_wait();
   pdl_trigger();
   __shared__ float warp_max[kThreads / 32];
@@ -300,7 +303,21 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
       v[2 * c] = v[2 * c + 1] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
-  if constexpr (MECH != kNoMask) {
+  if constexpr (MECH == kStored) {
+    const float4* nrow = reinterpret_cast<const float4*>(stored + r * cols);
+#pragma unroll
+    for (int c = 0; c < CH; ++c) {
+      const int64_t i = threadIdx.x + (int64_t)c * kThreads;
+      if (i >= n8) break;
+      v[2 * c] = add4(v[2 * c], __ldg(nrow + 2 * i));
+      v[2 * c + 1] = add4(v[2 * c + 1], __ldg(nrow + 2 * i + 1));
+      if (xt_out) {
+        float4* o = reinterpret_cast<float4*>(xt_out + r * cols);
+        __stcs(o + 2 * i, v[2 * c]);
+        __stcs(o + 2 * i + 1, v[2 * c + 1]);
+      }
+    }
+  } else if constexpr (MECH != kNoMask) {
     const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
     const uint64_t j0 = (uint64_t)((r * cols) >> 2) + offset;  // cols % 8 == 0: rows start on a block
 #pragma unroll
@@ -386,22 +403,23 @@ spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double
 // (more than 16384 entries) and no mask take the two-pass kernel.
 template <int MECH>
 spl_status launch_split_rows(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows,
-                             int64_t cols, float* xt_out, float b, const spl_rng& rng, cudaStream_t stream) {
+                             int64_t cols, float* xt_out, float b, const spl_rng& rng, cudaStream_t stream,
+                             const float* stored = nullptr) {
   const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
   const dim3 grid((unsigned)rows), block(kThreads);
   const PhiloxKey key = make_philox_key(rng.seed, rng.stream_id);
   if (per_thread <= 1)
     return launch_pdl(split_fp16_regs_kernel<1, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev, stored);
   if (per_thread <= 2)
     return launch_pdl(split_fp16_regs_kernel<2, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev, stored);
   if (per_thread <= 4)
     return launch_pdl(split_fp16_regs_kernel<4, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev, stored);
   if (per_thread <= 8)
     return launch_pdl(split_fp16_regs_kernel<8, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev);
+                      key, rng.offset, rng.offset_dev, stored);
   if (MECH != kNoMask) return SPL_ESHAPE;
   return launch_pdl(split_fp16_kernel, grid, block, 0, stream, hi, lo, row_exp, src, cols);
 }
@@ -526,6 +544,17 @@ extern "C" spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo
   if (b == 0.0f) return launch_split_rows<kZero>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
   if (mech == SPL_MECH_LAPLACE) return launch_split_rows<kLaplace>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
   return launch_split_rows<kGaussian>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
+}
+
+extern "C" spl_status spl_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,
+                                     const float* N, int64_t rows, int64_t cols, cudaStream_t stream) {
+  if (rows < 0 || cols < 0) return SPL_EINVAL;
+  if (rows == 0 || cols == 0) return SPL_OK;
+  if (!hi || !lo || !row_exp || !X || !N) return SPL_EINVAL;
+  if ((cols & 7) != 0) return SPL_EALIGN;
+  if (!aligned16(X) || !aligned16(N) || !aligned16(hi) || !aligned16(lo) || (Xt && !aligned16(Xt))) return SPL_EALIGN;
+  if (rows > 0x7fffffffLL) return SPL_ESHAPE;
+  return launch_split_rows<kStored>(hi, lo, row_exp, X, rows, cols, Xt, 0.0f, spl_rng{}, stream, N);
 }
 
 extern "C" spl_status spl_mask(float* Xt, const float* X, const float* N, int64_t rows, int64_t cols,

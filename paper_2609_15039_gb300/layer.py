@@ -144,9 +144,14 @@ class MaskedLayer:
                            spl.spl_f64_workspace_bytes(draws * M, g.K, g.N))
         return need
 
-    def allocate(self, M, draws, path="auto", workspace=None):
+    def allocate(self, M, draws, path="auto", workspace=None, stored_noise=False):
         """Buffers for M tokens and a bank of ``draws`` corrections per group.  ``workspace`` may be
-        shared with other layers whose calls run on the same stream."""
+        shared with other layers whose calls run on the same stream.  stored_noise: the FP16X3
+        groups keep the bank's fp32 noise, and each online step masks with its rows (spl_mask_split)
+        instead of drawing them again -- the same X~ bit for bit, the paper's precomputed noise.  Off
+        by default: on GB300 writing and reading the fp32 noise costs more than drawing it again
+        (Llama layer at 128 tokens: 267-268 against 271 TFLOP/s), since the split kernel that draws
+        it runs while the next product's CTAs start."""
         dev = self.groups[0].W.device
         need = self.workspace_bytes(M, draws, path)
         if workspace is not None:
@@ -155,12 +160,13 @@ class MaskedLayer:
         elif self.workspace is None or self.workspace.numel() < need:
             self.workspace = spl.workspace(need, dev)
         self.M, self.draws = M, draws
+        self.stored_noise = bool(stored_noise)
         self.rng_base = torch.zeros(len(self.groups), dtype=torch.int64, device=dev)
         self.bank = {}
         for g in self.groups:
             wide = torch.float64 if g.name in self.fp64 else torch.float32  # binary64 mask and correction
             self.bank[g.name] = {
-                "eta": torch.empty((draws * M, g.K), device=dev),  # transient: the draws being precomputed
+                "eta": torch.empty((draws * M, g.K), device=dev),  # the draws being precomputed (kept with stored noise)
                 "C": torch.empty((draws * M, g.N), device=dev, dtype=wide),
                 "xt": torch.empty((M, g.K), device=dev, dtype=wide),
                 "Y": torch.empty((M, g.N), device=dev),
@@ -175,16 +181,22 @@ class MaskedLayer:
                                      f16_exp=torch.empty(draws * M, dtype=torch.int32, device=dev))
 
     def enable_overlap(self):
-        """A second correction buffer per group, so that a bank cycle can run its online steps on one
-        while the next cycle's corrections are computed into the other (capture_overlapped)."""
+        """A second correction buffer per group (and noise buffer, for stored noise), so that a bank
+        cycle can run its online steps on one while the next cycle's are filled into the other
+        (capture_overlapped)."""
         for g in self.groups:
             b = self.bank[g.name]
             if "Cs" not in b:
                 b["Cs"] = [b["C"], torch.empty_like(b["C"])]
+                b["etas"] = [b["eta"], torch.empty_like(b["eta"])]
 
     def _C(self, g, parity):
         b = self.bank[g.name]
         return b["Cs"][parity] if "Cs" in b else b["C"]
+
+    def _eta(self, g, parity):
+        b = self.bank[g.name]
+        return b["etas"][parity] if "etas" in b else b["eta"]
 
     def _fused_split(self, g, path, M):
         """True when the online product of group g runs FP16X3: then the mask kernel also writes the
@@ -247,7 +259,9 @@ class MaskedLayer:
                     side.wait_stream(main)
                     forks.append(side)
                 with torch.cuda.stream(side):
-                    spl.spl_noise_mask_split(None, es.f16_hi, es.f16_lo, es.f16_exp, None, self.deltas[g.name], eps,
+                    # with stored noise, the fp32 draws are kept for the online steps' masks
+                    keep = self._eta(g, parity) if self.stored_noise else None
+                    spl.spl_noise_mask_split(keep, es.f16_hi, es.f16_lo, es.f16_exp, None, self.deltas[g.name], eps,
                                              mech, seed, stream_id=gi, offset=off, stream=side, offset_dev=off_dev)
                     if timer:
                         timer("begin", "precompute", g.name)
@@ -320,6 +334,9 @@ class MaskedLayer:
         if fp64:
             spl.spl_noise_mask_f64(b["xt"], inputs[g.name], self.deltas[g.name], eps, mech, seed, stream_id=gi,
                                    offset=off, stream=stream, offset_dev=off_dev)
+        elif xs is not None and self.stored_noise:  # the noise drawn with the bank: its rows for draw d
+            spl.spl_mask_split(None, xs.f16_hi, xs.f16_lo, xs.f16_exp, inputs[g.name],
+                               self._eta(g, parity)[d * M:(d + 1) * M], stream=stream)
         elif xs is not None:  # the FP16X3 product reads only the split: X~ itself is not written
             spl.spl_noise_mask_split(None, xs.f16_hi, xs.f16_lo, xs.f16_exp, inputs[g.name], self.deltas[g.name],
                                      eps, mech, seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)

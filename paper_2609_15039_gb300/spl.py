@@ -61,6 +61,7 @@ _SIGS = {
     "spl_noise_mask": (_I, [_P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_split_tf32": (_I, [_P, _P, _P, _I64, _P]),
     "spl_noise_mask_split": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
+    "spl_mask_split": (_I, [_P, _P, _P, _P, _P, _P, _I64, _I64, _P]),
     "spl_masked_linear_unmask_split": (_I, [_P, _PW, _PW, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_split_fp16": (_I, [_P, _P, _P, _P, _I64, _I64, _P]),
     "spl_resolve_path": (_I, [_I64, _I64, _I64, _I]),
@@ -251,6 +252,18 @@ def spl_noise_mask_split(Xt, hi, lo, row_exp, X, sensitivity, eps, mech, seed, s
                                       float(sensitivity), _eps(eps), _mech(mech),
                                       _rng(seed, stream_id, offset, offset_dev), _stream(stream)),
            "spl_noise_mask_split")
+
+
+def spl_mask_split(Xt, hi, lo, row_exp, X, N, stream=None):
+    """a3 with a stored noise N + the fp16 split of X~ in one pass (Xt may be None)."""
+    rows, cols = _rows_cols(X)
+    if (N.numel() != rows * cols or hi.numel() != rows * cols or lo.numel() != rows * cols
+            or row_exp.numel() != rows):
+        raise ValueError("spl_mask_split: shape mismatch")
+    _check(lib().spl_mask_split(_dev(Xt, "Xt"), _dev(hi, "hi", torch.int16), _dev(lo, "lo", torch.int16),
+                                _dev(row_exp, "row_exp", torch.int32), _dev(X, "X"), _dev(N, "N"), rows, cols,
+                                _stream(stream)),
+           "spl_mask_split")
 
 
 def spl_masked_linear_unmask_split(Y, Xt, W, C, path="auto", workspace=None, stream=None):

@@ -165,3 +165,26 @@ def test_stack_overlapped_decode_graphs_equal_eager_steps(spl):
     for layer in stack.layers:
         assert layer.rng_base.cpu().tolist() == [layer.block_offset(g, first + cycles, 0) for g in layer.groups]
     assert spl.spl_get_device_status() == 0
+
+
+@pytest.mark.parametrize("mech", ["laplace", "gaussian"])
+def test_stored_noise_steps_equal_drawn_noise_steps(spl, mech):
+    """Online steps that mask with the noise the refill kept give the results of steps that draw the
+    noise again, bit for bit, across two bank cycles."""
+    model = wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)
+    draws, eps, seed, M = 3, 1.0, 81, 128
+    res = []
+    for stored in (True, False):
+        layer, inputs = make_layer(model, M, draws)
+        layer.allocate(M, draws, stored_noise=stored)
+        outs = []
+        for s in range(2 * draws):
+            cycle, d = divmod(s, draws)
+            if d == 0:
+                layer.refill(eps, mech, seed, cycle)
+            outs.append({g: y.clone() for g, y in layer.online(inputs, eps, mech, seed, cycle, d).items()})
+        res.append(outs)
+    for a, b in zip(*res):
+        for g in a:
+            assert torch.equal(a[g], b[g]), g
+    assert spl.spl_get_device_status() == 0

@@ -481,6 +481,29 @@ def test_noise_mask_split_equals_separate_calls(spl, rows, cols, mech, eps):
     assert torch.equal(hi, hi_ref) and torch.equal(ex, ex_ref)
 
 
+@pytest.mark.parametrize("rows,cols,mech", [(5, 8, "laplace"), (130, 3072, "gaussian"), (3, 16384, "laplace")])
+def test_mask_split_with_stored_noise_equals_drawn(spl, rows, cols, mech):
+    """The mask with a noise drawn earlier (as a bank refill keeps it) gives the X~ and the fp16
+    split that drawing the noise in the same pass gives, bit for bit."""
+    X = dev(wl.activations(rows, cols, seed=rows + 7 * cols).numpy())
+    N = torch.empty_like(X)
+    spl.spl_noise(N, 825.3, 0.5, mech, seed=23, stream_id=1, offset=77)
+    ref_xt = torch.empty_like(X)
+    hi_ref = torch.empty(X.shape, dtype=torch.int16, device="cuda")
+    lo_ref, ex_ref = torch.empty_like(hi_ref), torch.empty(rows, dtype=torch.int32, device="cuda")
+    spl.spl_noise_mask_split(ref_xt, hi_ref, lo_ref, ex_ref, X, 825.3, 0.5, mech, seed=23, stream_id=1, offset=77)
+    xt = torch.empty_like(X)
+    hi, lo, ex = torch.empty_like(hi_ref), torch.empty_like(lo_ref), torch.empty_like(ex_ref)
+    spl.spl_mask_split(xt, hi, lo, ex, X, N)
+    assert torch.equal(xt, ref_xt) and torch.equal(hi, hi_ref) and torch.equal(lo, lo_ref) and torch.equal(ex, ex_ref)
+    spl.spl_mask_split(None, hi, lo, ex, X, N)  # no X~ out
+    assert torch.equal(hi, hi_ref) and torch.equal(ex, ex_ref)
+    # the noise a bank keeps: spl_noise_mask_split with X NULL writes it to Xt
+    keep = torch.empty_like(X)
+    spl.spl_noise_mask_split(keep, hi, lo, ex, None, 825.3, 0.5, mech, seed=23, stream_id=1, offset=77)
+    assert torch.equal(keep, N)
+
+
 @pytest.mark.parametrize("M,K,N,mech,eps", [(1, 3072, 3072, "laplace", 1.0), (2, 1028, 600, "gaussian", 0.5),
                                              (3, 8192, 520, "laplace", None), (4, 2560, 2056, "gaussian", 1.0),
                                              (5, 516, 300, "laplace", 1.0), (16, 3072, 512, "gaussian", 1.0)])
