@@ -79,13 +79,16 @@ def test_device_offset_equals_host_offset(spl):
     assert spl.lib().spl_rng_advance(base.data_ptr() + 4, 1, None) == spl.SPL_EALIGN
 
 
-def test_overlapped_cycle_graphs_equal_eager_steps(spl):
+@pytest.mark.parametrize("stored", [False, True])
+def test_overlapped_cycle_graphs_equal_eager_steps(spl, stored):
     """Whole-cycle graphs that compute the next cycle's corrections during this cycle's steps (on
     streams of their own) give, step by step, the eager results -- across three cycles, so both
-    correction buffers are filled by a graph and read by the other."""
+    correction buffers (and, with stored noise, both noise buffers) are filled by a graph and read
+    by the other."""
     model = wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)
     draws, eps, mech, seed, M = 3, 1.0, "gaussian", 78, 128
     layer, inputs = make_layer(model, M, draws)
+    layer.allocate(M, draws, stored_noise=stored)
     assert all(layer._fused_split(g, "auto", M) for g in layer.groups)
 
     def eager(s):
