@@ -53,7 +53,8 @@ def parse():
     ap.add_argument("--stored-noise", action="store_true",
                     help="keep the bank's fp32 noise and mask each step with it instead of drawing it again")
     ap.add_argument("--workload", default="llama_layer",
-                    choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep", "down_fp64", "slalom"],
+                    choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep", "down_fp64", "slalom",
+                             "lm_head"],
                     help="llama_layer (default): the headline line; the others measure the stack and sweep "
                          "workloads and print their own line")
     return ap.parse_args()
@@ -234,6 +235,9 @@ def run_workload(args):
     elif args.workload == "down_fp64":
         first = next(iter(res["down"].values()))["binary64"]
         value, unit, ms = first["mean_err"], "mean abs error of the recovered Down output", first["us_per_call"] / 1e3
+    elif args.workload == "lm_head":
+        first = next(iter(res["lm_head"].values()))
+        value, unit, ms = first["tflops"], UNIT, first["ms_per_step"]
     else:
         last = list(res["sweep"].values())[-1]
         value, unit, ms = last["tflops"], UNIT, last["online_ms"]

@@ -11,6 +11,7 @@ inputs are resident in HBM.  The workloads:
   the cancellation error of every output of the first and last layer checked against the bound.
 * qwen_sweep  -- one Qwen3-4B-shaped layer at M in {1, 4, 16, 64, 256, 1024} tokens, and the
   noise + mask kernel alone on 10^9 elements.
+* lm_head     -- the Llama LM head (3072 -> 128256) at 512 and 1 tokens with its bank.
 """
 
 import torch
@@ -377,5 +378,67 @@ def slalom_compare(tokens=(128, 1), eps=1.0, mech="gaussian", reps=10):
                         f"point) vs this path ({mech} eps={eps}), M in {list(tokens)}", "compare": out}
 
 
+def lm_head(tokens=(512, 1), eps=1.0, mech="gaussian", draws=8, cycles=3):
+    """The Llama LM head (3072 -> 128256 after the final RMSNorm, Delta from Thm. 1) at prefill and
+    decode sizes: per draw the noise + mask of X and the masked product with fused unmask, replayed
+    as CUDA graphs of one bank cycle; the bank (8 draws, summed in the online order) timed apart."""
+    model = wl.LLAMA_3_2_3B
+    pk = _peaks()
+    K, N = model.d_model, model.vocab
+    W = wl.weight(N, K, seed=9001, device="cuda")
+    Wt = spl.Weight.prepare(W)
+    delta = spl.spl_delta_layernorm(torch.ones(K))
+    stream = torch.cuda.current_stream()
+    out = {}
+    for M in tokens:
+        path = spl.PATH_NAMES[spl.spl_resolve_path(M, K, N, "auto")]
+        X = wl.activations(M, K, seed=9002, device="cuda")
+        Xt = torch.empty_like(X)
+        Y = torch.empty((M, N), device="cuda")
+        eta = torch.empty((draws * M, K), device="cuda")
+        C = torch.empty((draws * M, N), device="cuda")
+        ws = spl.workspace(max(spl.spl_precompute_matched_workspace_bytes(draws * M, K, N, M),
+                               spl.spl_linear_workspace_bytes(M, K, N)))
+        base = torch.zeros(1, dtype=torch.int64, device="cuda")
+
+        def refill():
+            spl.spl_noise(eta, delta, eps, mech, seed=606, offset_dev=base)
+            spl.spl_precompute_noise_product_matched(C, eta, Wt, M, workspace=ws)
+
+        def online(d):
+            spl.spl_noise_mask(Xt, None, X, delta, eps, mech, seed=606, offset=d * M * K // 4, offset_dev=base)
+            spl.spl_masked_linear_unmask(Y, Xt, Wt, C[d * M:(d + 1) * M], workspace=ws)
+
+        refill()
+        for d in range(draws):
+            online(d)
+        torch.cuda.synchronize()
+        g_on, g_rf = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_on):
+            for d in range(draws):
+                online(d)
+        with torch.cuda.graph(g_rf):
+            refill()
+        on_t = _time_replays([g_on], 0, cycles + 1, stream)[1:]
+        rf_t = _time_replays([g_rf], 0, cycles + 1, stream)[1:]
+        step_ms = sum(on_t) / (cycles * draws)
+        refill_ms = sum(rf_t) / cycles
+        flops = 2 * M * K * N
+        wbytes = 4 * K * N  # fp32 W (decode kernel) or its two fp16 halves: 4 bytes per weight either way
+        byts = wbytes + 4 * M * K + 8 * M * N
+        t_hbm = byts / (pk["hbm_gbs"] * 1e9)
+        t_tc = flops / (_path_peak(path, pk) * 1e12)
+        bound = "hbm" if t_hbm >= t_tc else "tensor"
+        out[f"M={M}"] = {"path": path, "ms_per_step": step_ms, "tflops": flops / (step_ms * 1e-3) / 1e12,
+                         "gbs": byts / (step_ms * 1e-3) / 1e9, "bound": bound,
+                         "frac": max(t_hbm, t_tc) * 1e3 / step_ms,
+                         "bank_refill_ms": refill_ms,
+                         "bank_refill_tflops": draws * flops / (refill_ms * 1e-3) / 1e12}
+        del g_on, g_rf, X, Xt, Y, eta, C, ws
+        torch.cuda.empty_cache()
+    return {"workload": f"llama-3.2-3b LM head (3072 -> 128256), {mech} eps={eps}, banks of {draws} draws, "
+                        f"tokens {list(tokens)}", "lm_head": out, "peak_source": pk["source"]}
+
+
 WORKLOADS = {"llama_stack": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep, "down_fp64": down_fp64,
-             "slalom": slalom_compare}
+             "slalom": slalom_compare, "lm_head": lm_head}
