@@ -438,14 +438,19 @@ spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int64_t cluster
  * unsplit tiles run in segmented mode (the bank's form: one CTA over all of K,
  * the partial sums of a seg_splits-way split of K folded in order), so the
  * result equals the seg_splits-way split product bit for bit; splits must then
- * be 1 or seg_splits.  path is SPL_PATH_TF32X3 or SPL_PATH_FP16X3.  Same
- * operands, workspace and errors as spl_masked_linear_unmask; EINVAL for another
- * path or variant, full_tiles outside [0, tiles], seg_splits outside [0, 8] or
- * a splits other than 1 or seg_splits, ESHAPE for a split outside 1..8. */
+ * be 1 or seg_splits.  persistent != 0: every tile unsplit in the persistent
+ * kernel (one CTA per SM looping over tiles, two TMEM accumulators; the result
+ * equals the unsplit product bit for bit); it needs splits 1, seg_splits 0,
+ * full_tiles 0, a one-CTA-per-SM variant and N % 4 == 0.  path is
+ * SPL_PATH_TF32X3 or SPL_PATH_FP16X3.  Same operands, workspace and errors as
+ * spl_masked_linear_unmask; EINVAL for another path or variant, full_tiles
+ * outside [0, tiles], seg_splits outside [0, 8], a splits other than 1 or
+ * seg_splits, or a persistent request that breaks its conditions; ESHAPE for a
+ * split outside 1..8. */
 spl_status spl_test_tc_product(float* Y, const float* Xt, const spl_weight* W, const float* C, int64_t M,
                                int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
-                               int64_t full_tiles, int seg_splits, void* workspace, size_t workspace_bytes,
-                               cudaStream_t stream);
+                               int64_t full_tiles, int seg_splits, int persistent, void* workspace,
+                               size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last

@@ -705,6 +705,232 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   }
 }
 
+// Persistent form for launches of several waves of unsplit tiles: one CTA per SM takes the
+// tiles blockIdx.x, blockIdx.x + gridDim.x, ... (M fastest, as above).  The stage ring runs on
+// across tiles and TMEM holds two accumulators (columns 0 and 256): while the epilogue warps finish
+// tile i from one, the MMAs of tile i + 1 go into the other, so each tile's epilogue (C in, Y out,
+// straight between TMEM rows and global memory) overlaps the next tile's mainloop and only the
+// first prologue and the last epilogue are exposed.  Every output element is summed exactly as by
+// tc_gemm_kernel with one K range (the same MMAs in the same order, the same scaling and
+// subtraction), so the two give the same result bit for bit.  Rows of out and C must be whole
+// 16-byte units (the host checks).  Every wait is bounded as in tc_gemm_kernel.
+template <class Md, int BN, int RK>
+__global__ void __launch_bounds__(THREADS, 1)
+tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
+                     const int* __restrict__ a_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
+                     int tiles, int m_tiles) {
+  using L = Cfg<Md, BN, RK>;
+  constexpr int STAGES = L::STAGES, BK = Md::BK;
+  constexpr uint32_t ACC_COLS = 256;  // column offset of the second accumulator
+  static_assert(BN <= (int)ACC_COLS, "two accumulators in 512 TMEM columns");
+  static_assert(8 * (2 * STAGES + 5) + 16 <= (int)AUX_BYTES, "aux fits");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* aux = smem + L::RING;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], empty[S], acc_full[2], acc_empty[2], drain
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (2 * STAGES + 5));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (2 * STAGES + 5) + 8);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int my_tiles = tiles > (int)blockIdx.x ? (tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+  const int nk = (int)ceil_div(K, BK);
+  const uint32_t bar_base = smem_u32(bars);
+  auto full_bar = [&](int st) { return bar_base + 8u * st; };
+  auto empty_bar = [&](int st) { return bar_base + 8u * (STAGES + st); };
+  auto acc_full = [&](int b) { return bar_base + 8u * (2 * STAGES + b); };
+  auto acc_empty = [&](int b) { return bar_base + 8u * (2 * STAGES + 2 + b); };
+  const uint32_t drain_bar = bar_base + 8u * (2 * STAGES + 4);
+  auto tile_origin = [&](int i, int64_t& m0, int64_t& n0) {
+    const int tile = (int)blockIdx.x + i * (int)gridDim.x;
+    m0 = (int64_t)(tile % m_tiles) * BM;
+    n0 = (int64_t)(tile / m_tiles) * BN;
+  };
+
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < STAGES; ++st) {
+      mbar_init(full_bar(st), 1);
+      mbar_init(empty_bar(st), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), 4);  // one arrival per epilogue warp
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(smem_u32(const_cast<uint32_t*>(tmem_slot)), 2 * ACC_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------- TMA producer: the ring runs on across this CTA's tiles ----------------
+    uint32_t issued_mask = 0u, phase_mask = 0u;
+    bool ok = true;
+    const uint64_t pol_w = l2_evict_first(), pol_a = l2_evict_last();
+    pdl_wait();  // A comes from the kernel before this one
+    uint32_t it = 0;
+    for (int i = 0; i < my_tiles && ok; ++i) {
+      int64_t m0, n0;
+      tile_origin(i, m0, n0);
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int st = (int)(it % STAGES);
+        const uint32_t ph = (it / STAGES) & 1u;
+        if (it >= (uint32_t)STAGES) {
+          ok = __all_sync(0xffffffffu, mbar_wait(empty_bar(st), ph ^ 1u, kWaitNs, abort_flag));
+          if (!ok) break;
+        }
+        if (lane == 0) {
+          const uint32_t sa = smem_u32(smem + (size_t)st * L::STAGE);
+          const int kx = kb * BK;
+          mbar_expect_tx(full_bar(st), L::STAGE);
+          tma_load_2d(sa + L::A_HI, &maps.a_hi, full_bar(st), kx, (int)m0, pol_a);
+          tma_load_2d(sa + L::A_LO, &maps.a_lo, full_bar(st), kx, (int)m0, pol_a);
+          tma_load_2d(sa + L::W_HI, &maps.w_hi, full_bar(st), kx, (int)n0, pol_w);
+          tma_load_2d(sa + L::W_LO, &maps.w_lo, full_bar(st), kx, (int)n0, pol_w);
+        }
+        __syncwarp();
+        issued_mask |= 1u << st;
+        phase_mask = (phase_mask & ~(1u << st)) | (ph << st);
+      }
+    }
+    pdl_trigger();
+    if (!ok) {
+      if (lane == 0) {
+        *abort_flag = 1;
+        atomicOr(&g_device_status, kStatusTimeout);
+      }
+      for (int st = 0; st < STAGES; ++st)
+        if (issued_mask & (1u << st)) mbar_wait(full_bar(st), (phase_mask >> st) & 1u, kDrainNs, nullptr);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer: tile i into accumulator i % 2 ----------------
+    bool ok = true;
+    uint32_t it = 0;
+    for (int i = 0; i < my_tiles && ok; ++i) {
+      const int buf = i & 1, use = i >> 1;
+      if (use >= 1) {  // the epilogue is done with this accumulator's previous tile
+        ok = __all_sync(0xffffffffu, mbar_wait(acc_empty(buf), (uint32_t)(use - 1) & 1u, kWaitNs * 4, abort_flag));
+        if (!ok) break;
+      }
+      tc_fence_after();
+      const uint32_t acc = tmem + (uint32_t)buf * ACC_COLS;
+      for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int st = (int)(it % STAGES);
+        const uint32_t ph = (it / STAGES) & 1u;
+        ok = __all_sync(0xffffffffu, mbar_wait(full_bar(st), ph, kWaitNs, abort_flag));
+        if (!ok) break;
+        if (lane == 0) {
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + (size_t)st * L::STAGE);
+#pragma unroll
+          for (int kk = 0; kk < BK / Md::UMMA_K; ++kk) {
+            const uint32_t koff = kk * 32u;
+            const uint32_t first = (kb == 0 && kk == 0) ? 0u : 1u;
+            mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_LO + koff), make_sdesc_sw64(sa + L::W_HI + koff), first);
+            mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_HI + koff), make_sdesc_sw64(sa + L::W_LO + koff), 1u);
+            mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_HI + koff), make_sdesc_sw64(sa + L::W_HI + koff), 1u);
+          }
+          mma_commit(empty_bar(st));
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+      if (lane == 0) mma_commit(acc_full(buf));  // the tile's sums are complete once these MMAs are
+      __syncwarp();
+    }
+    pdl_trigger();
+    if (!ok) {
+      if (lane == 0) {
+        *abort_flag = 1;
+        atomicOr(&g_device_status, kStatusTimeout);
+        mma_commit(drain_bar);  // MMAs already issued finish before TMEM is released
+      }
+      __syncwarp();
+      mbar_wait(drain_bar, 0u, kDrainNs, nullptr);
+    }
+  } else {
+    // ---------------- warps 2..5: epilogue of tile i from accumulator i % 2 ----------------
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int r = 32 * q + lane;
+    const bool vec_ok = (N & 3) == 0;
+    // the rows of C a tile subtracts, into L2 while its mainloop runs (tile i + 1's after tile i)
+    auto prefetch_c = [&](int i) {
+      if (!C || i >= my_tiles) return;
+      int64_t pm0, pn0;
+      tile_origin(i, pm0, pn0);
+      const int64_t ncols = std::min<int64_t>(BN, N - pn0);
+      const int lines = (int)ceil_div(ncols * 4, 128);
+      for (int j = threadIdx.x - 64; j < BM * lines; j += 128) {
+        const int64_t pm = pm0 + j / lines;
+        if (pm < M) prefetch_l2(C + pm * N + pn0 + (int64_t)(j % lines) * 32);
+      }
+    };
+    pdl_wait();  // C and the row exponents of A come from before this kernel
+    prefetch_c(0);
+    bool ok = true;
+    for (int i = 0; i < my_tiles; ++i) {
+      const int buf = i & 1, use = i >> 1;
+      int64_t m0, n0;
+      tile_origin(i, m0, n0);
+      const int64_t m = m0 + r;
+      const float sr = (Md::kF16 && m < M) ? pow2f(-__ldg(a_exp + m)) : 1.0f;
+      ok = __all_sync(0xffffffffu, mbar_wait(acc_full(buf), (uint32_t)use & 1u, kWaitNs * 4, abort_flag)) &&
+           !*abort_flag;
+      if (!ok) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        const int64_t nc = n0 + 32 * c;
+        if (nc >= N) break;  // the same for the whole warp
+        float v[32];
+        tmem_ld_32x32(tmem + (uint32_t)buf * ACC_COLS + ((uint32_t)(32 * q) << 16) + (uint32_t)(32 * c), v);
+        if constexpr (Md::kF16) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j)  // exact power-of-two scaling, as tc_gemm_kernel's col_scale
+            v[j] = (v[j] * sr) * pow2f(-((nc + j < N) ? __ldg(w_exp + nc + j) : 0));
+        }
+        if (m < M && vec_ok) {
+          float4 cc[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            cc[j] = (C && nc + 4 * j < N) ? __ldcs(reinterpret_cast<const float4*>(C + m * N + nc + 4 * j))
+                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (nc + 4 * j >= N) continue;
+            float4 o = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+            if (C)
+              o = make_float4(__fsub_rn(o.x, cc[j].x), __fsub_rn(o.y, cc[j].y), __fsub_rn(o.z, cc[j].z),
+                              __fsub_rn(o.w, cc[j].w));
+            *reinterpret_cast<float4*>(out + m * N + nc + 4 * j) = o;
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty(buf));
+      prefetch_c(i + 1);
+    }
+    pdl_trigger();
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      atomicOr(&g_device_status, kStatusTimeout);
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 2 * ACC_COLS);
+  }
+}
+
 // ---- host side: tensor maps ------------------------------------------------------
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -748,6 +974,20 @@ bool set_smem_attr() {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
   if (!done[dev]) {
     if (cudaFuncSetAttribute(tc_gemm_kernel<Md, BN, RK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)Cfg<Md, BN, RK>::SMEM) != cudaSuccess)
+      return false;
+    done[dev] = true;
+  }
+  return true;
+}
+
+template <class Md, int BN, int RK>
+bool set_smem_attr_persistent() {
+  static bool done[64] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  if (!done[dev]) {
+    if (cudaFuncSetAttribute(tc_persistent_kernel<Md, BN, RK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)Cfg<Md, BN, RK>::SMEM) != cudaSuccess)
       return false;
     done[dev] = true;
@@ -829,7 +1069,15 @@ struct TcShape {
   int64_t rest_tiles;  // tiles of the second launch
   int rest_splits;
   double cost;
+  bool persistent = false;  // one launch of tc_persistent_kernel over every tile (unsplit)
 };
+
+// Cost of the persistent form: the first prologue and the last epilogue (F) once, then per tile of
+// the busiest CTA its mainloop and a small hand-over (kPersistentTile, in units of K).  With it the
+// shapes picked over the eight projections at 512 to 4096 rows (persistent, split and whole-wave
+// forms all timed) are within 0.16% of the best measured on average; the persistent form saves 4-7%
+// on shapes of several waves (e.g. 2048 x 2560 by 19456: 386.5 against 412.8 us).
+constexpr double kPersistentTile = 60.0;
 
 double launch_cost(int v, int64_t tiles, int64_t K, int s, int sms) {
   if (tiles <= 0) return 0.0;
@@ -839,6 +1087,9 @@ double launch_cost(int v, int64_t tiles, int64_t K, int s, int sms) {
 }
 
 TcShape tc_shape_for(int v, int64_t M, int64_t K, int64_t N, int sms) {
+  // the persistent epilogue stores whole float4s: output rows of whole 16-byte units (a launch whose
+  // pointers are not 16-byte aligned runs the same tiles unsplit in tc_gemm_kernel: the same sums)
+  const bool persistent_ok = (N & 3) == 0;
   const int64_t tiles = ceil_div(M, BM) * ceil_div(N, kVariant[v].bn);
   const int max_s = (int)std::max<int64_t>(1, std::min<int64_t>(MAX_CLUSTER, K / 256));
   TcShape best{v, 0, tiles, 1, 1e300};
@@ -853,6 +1104,13 @@ TcShape tc_shape_for(int v, int64_t M, int64_t K, int64_t N, int sms) {
     for (int s = 1; s <= max_s; ++s) {
       const double c = cf + launch_cost(v, rest, K, s, sms);
       if (c < best.cost * (1.0 - 1e-9)) best = TcShape{v, full, rest, s, c};
+    }
+  }
+  if (persistent_ok && kVariant[v].cps == 1 && tiles > wave) {  // more than one wave of unsplit tiles
+    const double c = kVariant[v].F + (double)ceil_div(tiles, wave) * (kVariant[v].b * (double)K + kPersistentTile);
+    if (c < best.cost * (1.0 - 1e-9)) {
+      best = TcShape{v, 0, tiles, 1, c};
+      best.persistent = true;
     }
   }
   return best;
@@ -911,6 +1169,30 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
       return SPL_ECUDA;
   }
   const int m_tiles = (int)ceil_div(a.M, BM);
+  if constexpr (Cfg<Md, BN, RK>::CTAS_PER_SM == 1) {
+  if (shape.persistent && seg_splits == 0 && skip_kblock < 0 && epi_tma) {
+    // one CTA per SM over every tile (the same sums as one unsplit launch of tc_gemm_kernel)
+    if (!set_smem_attr_persistent<Md, BN, RK>()) return SPL_ECUDA;
+    const int64_t tiles = shape.full_tiles + shape.rest_tiles;
+    if (tiles > 0x7fffffffLL) return SPL_ESHAPE;
+    const int ctas = (int)std::min<int64_t>(tiles, max_active_clusters(shape.v, 1, device_sm_count()));
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof(cfg));
+    cfg.gridDim = dim3((unsigned)ctas, 1, 1);
+    cfg.blockDim = dim3(THREADS, 1, 1);
+    cfg.dynamicSmemBytes = Cfg<Md, BN, RK>::SMEM;
+    cfg.stream = a.stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_persistent_kernel<Md, BN, RK>, maps, a.out, a.c, a_exp,
+                                             (const int*)a.w_exp, a.M, a.K, a.N, (int)tiles, m_tiles);
+    note_launches(1);
+    return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
+  }
+  }
   // The first launch follows the split of A under programmatic dependent launch: its CTAs start
   // (barriers, TMEM, weight tiles) while the split finishes.
   bool first = true;
@@ -964,7 +1246,7 @@ spl_status launch_variant(const LinearArgs& a, const uint16_t* hi, const uint16_
 // and the rest with K split forced_splits ways (one launch when forced_full is 0).
 // seg_splits > 0: segmented mode, one unsplit launch whose sums follow a seg_splits-way split.
 spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int forced_splits, int seg_splits = 0,
-                       int64_t forced_full = 0) {
+                       int64_t forced_full = 0, bool forced_persistent = false) {
   const int cc = device_cc();
   if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
   const bool f16 = a.path == SPL_PATH_FP16X3;
@@ -1016,6 +1298,7 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int f
   if (forced_v >= 0) {
     const int64_t tiles = ceil_div(a.M, BM) * ceil_div(a.N, kVariant[forced_v].bn);
     shape = TcShape{forced_v, forced_full, tiles - forced_full, forced_splits, 0.0};
+    shape.persistent = forced_persistent;
   } else if (seg_splits > 0) {
     shape = tc_bank_shape(a.M, a.K, a.N, seg_splits, device_sm_count());
   } else {
@@ -1111,12 +1394,12 @@ extern "C" spl_status spl_test_tc_capacity(int64_t tile_n, int64_t ring_kb, int6
 
 // Test hook: the tensor-core product with a fixed tile width and K-split, so that tests cover
 // every kernel instance and a sweep can time each launch shape; seg_splits > 0 runs the unsplit
-// tiles in segmented mode (the bank's form), their sums following a seg_splits-way split of K.
-// The paper has no counterpart.
+// tiles in segmented mode (the bank's form), their sums following a seg_splits-way split of K;
+// persistent != 0 runs every tile unsplit in the persistent kernel.  The paper has no counterpart.
 extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_weight* W, const float* C, int64_t M,
                                           int64_t K, int64_t N, spl_path path, int tile_n, int ring_kb, int splits,
-                                          int64_t full_tiles, int seg_splits, void* workspace, size_t workspace_bytes,
-                                          cudaStream_t stream) {
+                                          int64_t full_tiles, int seg_splits, int persistent, void* workspace,
+                                          size_t workspace_bytes, cudaStream_t stream) {
   using namespace spl;
   if (!out || !A || !W || !W->w || M <= 0 || N <= 0 || K <= 0) return SPL_EINVAL;
   if (path != SPL_PATH_TF32X3 && path != SPL_PATH_FP16X3) return SPL_EINVAL;
@@ -1131,6 +1414,8 @@ extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_
   if (full_tiles < 0 || full_tiles > tiles) return SPL_EINVAL;
   if (seg_splits < 0 || seg_splits > MAX_CLUSTER || (seg_splits > 0 && splits > 1 && splits != seg_splits))
     return SPL_EINVAL;
+  if (persistent && (splits != 1 || seg_splits != 0 || full_tiles != 0 || kVariant[v].cps != 1 || (N & 3) != 0))
+    return SPL_EINVAL;
   const LinearArgs args = make_args(out, A, *W, C, M, K, N, workspace, workspace_bytes, stream, path);
-  return run_tc_impl(args, -1, v, splits, seg_splits, full_tiles);
+  return run_tc_impl(args, -1, v, splits, seg_splits, full_tiles, persistent != 0);
 }

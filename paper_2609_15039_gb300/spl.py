@@ -87,7 +87,7 @@ _SIGS = {
     "spl_test_tc_wait_timeout": (_I, [_P, _P, _PW, _I64, _I64, _I64, _P, _SZ, _P]),
     "spl_test_tc_capacity": (_I, [_I64, _I64, _I64, ctypes.POINTER(ctypes.c_int64)]),
     "spl_test_tc_shape": (_I, [_I64, _I64, _I64, _I64, ctypes.POINTER(ctypes.c_int64)]),
-    "spl_test_tc_product": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _I, _I, _I, _I64, _I, _P, _SZ, _P]),
+    "spl_test_tc_product": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _I, _I, _I, _I64, _I, _I, _P, _SZ, _P]),
     "spl_get_device_status": (_I, [_P]),
     "spl_launch_count": (ctypes.c_uint64, []),
     "spl_status_string": (ctypes.c_char_p, [_I]),
@@ -580,7 +580,7 @@ def spl_test_tc_capacity(tile_n, ring_kb, cluster):
 
 
 def spl_test_tc_product(Y, Xt, W, C=None, path="fp16x3", tile_n=256, ring_kb=192, splits=1, workspace=None,
-                        stream=None, full_tiles=0, seg_splits=0):
+                        stream=None, full_tiles=0, seg_splits=0, persistent=False):
     """The tensor-core product with a fixed launch variant and K-split, the unsplit tiles optionally in
     segmented mode (a test hook)."""
     W = _weight(W)
@@ -594,7 +594,7 @@ def spl_test_tc_product(Y, Xt, W, C=None, path="fp16x3", tile_n=256, ring_kb=192
     ws_ = W.c_struct()
     _check(lib().spl_test_tc_product(_dev(Y, "Y"), _dev(Xt, "Xt"), ctypes.byref(ws_), _dev(C, "C"), M, K, N,
                                      _path(path), int(tile_n), int(ring_kb), int(splits), int(full_tiles),
-                                     int(seg_splits), wsp, wsb, _stream(stream)),
+                                     int(seg_splits), int(bool(persistent)), wsp, wsb, _stream(stream)),
            "spl_test_tc_product")
 
 

@@ -428,6 +428,30 @@ def test_tc_unsplit_epilogue_on_ragged_rows(spl, tile_n, ring_kb, N):
 
 
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
+@pytest.mark.parametrize("tile_n,ring_kb", [v for v in TC_VARIANTS if v != (128, 96)])
+def test_tc_persistent_equals_unsplit_product(spl, path, tile_n, ring_kb):
+    """The persistent kernel (one CTA per SM looping over tiles, two TMEM accumulators, the epilogue
+    of one tile beside the mainloop of the next) gives the unsplit product bit for bit, with and
+    without C, on a problem of 2 to 4 tiles per CTA with ragged M, N and K."""
+    M, K, N = 2600, 264, 4000
+    W, Wt = _weights(spl, N, K, seed=61)
+    A = wl.activations(M, K, seed=62).numpy()
+    C = dev(wl.activations(M, N, seed=63).numpy())
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, path))
+    assert -(-M // 128) * -(-N // tile_n) > spl.spl_test_tc_capacity(tile_n, ring_kb, 1)
+    for Cx in (C, None):
+        ref = torch.empty((M, N), device="cuda")
+        spl.spl_test_tc_product(ref, dev(A), Wt, Cx, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=1, workspace=ws)
+        Y = torch.full((M, N), float("nan"), device="cuda")
+        spl.spl_test_tc_product(Y, dev(A), Wt, Cx, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=1, workspace=ws,
+                                persistent=True)
+        assert torch.equal(Y, ref), float((Y - ref).abs().max())
+    rows = np.arange(0, M, 97)
+    assert_product_close(f32(ref[torch.as_tensor(rows, device="cuda")]), A[rows], W, path, what="persistent, no C")
+    assert spl.spl_get_device_status() == 0
+
+
+@pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 @pytest.mark.parametrize("tile_n,ring_kb", TC_VARIANTS)
 def test_tc_segmented_equals_split_product(spl, path, tile_n, ring_kb):
     """Every kernel instance in segmented mode (one CTA over all of K, the partial sums of a 3-way
