@@ -414,9 +414,10 @@ spl_status spl_test_tc_wait_timeout(float* out, const float* A, const spl_weight
 
 /* Test hook (no counterpart in the paper): the launch shape the tensor-core
  * product of M x K by N x K takes (seg_splits = 0), or a correction whose sums
- * follow a seg_splits-way split of K (the bank, seg_splits >= 1).  out[5]
+ * follow a seg_splits-way split of K (the bank, seg_splits >= 1).  out[6]
  * (host) receives {tile width, ring KB, tiles of the unsplit launch, tiles of the
- * split launch, its K-split}.  EINVAL for non-positive sizes, seg_splits outside
+ * split launch, its K-split, 1 if the persistent kernel takes every tile (else
+ * 0)}.  EINVAL for non-positive sizes, seg_splits outside
  * [0, 8] or a NULL out.  No GPU work; needs a current CUDA device for the
  * occupancy queries. */
 spl_status spl_test_tc_shape(int64_t M, int64_t K, int64_t N, int64_t seg_splits, int64_t* out);

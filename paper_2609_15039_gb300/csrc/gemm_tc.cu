@@ -1364,7 +1364,8 @@ extern "C" spl_status spl_test_tc_wait_timeout(float* out, const float* A, const
 
 // Test hook: the launch shape the tensor-core product (seg_splits = 0) or a correction in the order
 // of a seg_splits-way split (seg_splits > 0) takes: out = {tile width, ring KB, tiles of the
-// unsplit launch, tiles of the split launch, its K-split}.  The paper has no counterpart.
+// unsplit launch, tiles of the split launch, its K-split, 1 if the persistent kernel takes every
+// tile}.  The paper has no counterpart.
 extern "C" spl_status spl_test_tc_shape(int64_t M, int64_t K, int64_t N, int64_t seg_splits, int64_t* out) {
   using namespace spl;
   if (!out || M <= 0 || K <= 0 || N <= 0 || seg_splits < 0 || seg_splits > MAX_CLUSTER) return SPL_EINVAL;
@@ -1375,6 +1376,7 @@ extern "C" spl_status spl_test_tc_shape(int64_t M, int64_t K, int64_t N, int64_t
   out[2] = t.full_tiles;
   out[3] = t.rest_tiles;
   out[4] = t.rest_splits;
+  out[5] = t.persistent ? 1 : 0;
   return SPL_OK;
 }
 

@@ -565,8 +565,8 @@ def spl_test_tc_wait_timeout(out, A, W, workspace=None, stream=None):
 
 def spl_test_tc_shape(M, K, N, seg_splits=0):
     """Launch shape of the tensor-core product (or of a correction in a seg_splits-way order):
-    (tile width, ring KB, unsplit tiles, split tiles, K-split)."""
-    out = (ctypes.c_int64 * 5)()
+    (tile width, ring KB, unsplit tiles, split tiles, K-split, persistent)."""
+    out = (ctypes.c_int64 * 6)()
     _check(lib().spl_test_tc_shape(int(M), int(K), int(N), int(seg_splits), out), "spl_test_tc_shape")
     return tuple(int(v) for v in out)
 

@@ -451,6 +451,28 @@ def test_tc_persistent_equals_unsplit_product(spl, path, tile_n, ring_kb):
     assert spl.spl_get_device_status() == 0
 
 
+def test_library_picks_persistent_for_many_waves(spl):
+    """The launch model takes the persistent kernel for a product of many waves of unsplit tiles
+    (Qwen Gate|Up at 2048 rows) and not for one wave (128 rows, cluster split); the product the
+    library runs equals the forced persistent launch bit for bit."""
+    M, K, N = 2048, 2560, 19456
+    shape = spl.spl_test_tc_shape(M, K, N)
+    assert shape[5] == 1 and shape[4] == 1 and shape[2] == 0
+    assert spl.spl_test_tc_shape(128, K, N)[5] == 0
+    W = wl.weight(N, K, seed=71, device="cuda")
+    Wt = spl.Weight.prepare(W)
+    X = wl.activations(M, K, seed=72, device="cuda")
+    C = wl.activations(M, N, seed=73, device="cuda")
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp16x3"))
+    Y = torch.empty((M, N), device="cuda")
+    spl.spl_masked_linear_unmask(Y, X, Wt, C, path="fp16x3", workspace=ws)
+    Yp = torch.full((M, N), float("nan"), device="cuda")
+    spl.spl_test_tc_product(Yp, X, Wt, C, path="fp16x3", tile_n=shape[0], ring_kb=shape[1], splits=1,
+                            workspace=ws, persistent=True)
+    assert torch.equal(Y, Yp)
+    assert spl.spl_get_device_status() == 0
+
+
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 @pytest.mark.parametrize("tile_n,ring_kb", TC_VARIANTS)
 def test_tc_segmented_equals_split_product(spl, path, tile_n, ring_kb):
