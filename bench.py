@@ -36,7 +36,7 @@ WORKLOAD = ("llama-3.2-3b-shaped layer (Q,K,V,O,gate,up,down), 128 tokens, fp32,
 DRAWS = 8
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=32)
@@ -57,7 +57,7 @@ def parse():
                              "lm_head"],
                     help="llama_layer (default): the headline line; the others measure the stack and sweep "
                          "workloads and print their own line")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def peaks():
@@ -144,6 +144,24 @@ def profiled_traffic():
     if not digest.startswith(fields.get("kernel_source_sha256_prefix", "-").strip()):
         return None, "kernel changed since the ncu capture"
     return float(fields["traffic_bytes_per_step"]), "ncu capture of the same kernel source (profiles/)"
+
+
+def max_over_ranks(x, device):
+    """The job's figure for a per-rank time: the largest over the ranks (one replica per GPU, so the
+    job is as slow as its slowest replica); x itself when the job has one rank."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_initialized() or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, units_per_step, ms):
+    """Whole-job rate of `world` replicas that each do units_per_step in ms per step (weak scaling:
+    the work per rank is fixed, the job's grows with the ranks)."""
+    return world * units_per_step / (ms * 1e-3)
 
 
 def dist_env():
@@ -422,16 +440,13 @@ def main():
     p_end.record(stream)
     torch.cuda.synchronize()
     ms_with_events = p_start.elapsed_time(p_end) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dev)
     st = spl.spl_get_device_status()
     if st != spl.SPL_OK:
         raise RuntimeError("device status " + spl.status_string(st))
 
     flops_step = layer.flops_per_step()
-    value = world * flops_step / (ms * 1e-3) / 1e12
+    value = job_rate(world, flops_step, ms) / 1e12
     group_paths = {g.name: spl.PATH_NAMES[spl.spl_resolve_path(M, g.K, g.N, layer.path_of(g, args.path, M))]
                    for g in layer.groups}
     path_name = "+".join(sorted(set(group_paths.values())))
@@ -515,11 +530,8 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = e0.elapsed_time(e1) / args.steps
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
-        e2e = {"value": world * flops_step / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        e2e_ms = max_over_ranks(e2e_ms, dev)
+        e2e = {"value": job_rate(world, flops_step, e2e_ms) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
                "copies": "pinned host memory, on a second stream inside each step's graph: the next "
                          "step's inputs copied in (double-buffered) while this one computes, each result "
