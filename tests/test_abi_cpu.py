@@ -96,6 +96,23 @@ def test_argument_validation_without_launch(spl):
     assert L.spl_slalom_quantize(None, None, -1, None) == spl.SPL_EINVAL
     assert L.spl_slalom_mask(None, None, None, 0, 3, rng, None) == spl.SPL_OK
     assert L.spl_slalom_linear_unmask(base, base, base, base, 1, 1 << 22, 1, None, 0, None) == spl.SPL_ESHAPE
+    # the mask fused with the fp16 split (drawn or stored noise)
+    assert L.spl_mask_split(None, base, base, base, base, base, -1, 8, None) == spl.SPL_EINVAL
+    assert L.spl_mask_split(None, None, None, None, None, None, 0, 8, None) == spl.SPL_OK
+    assert L.spl_mask_split(None, None, base, base, base, base, 2, 8, None) == spl.SPL_EINVAL  # NULL hi
+    assert L.spl_mask_split(None, base, base, base, base, None, 2, 8, None) == spl.SPL_EINVAL  # NULL noise
+    assert L.spl_mask_split(None, base, base, base, base, base, 2, 12, None) == spl.SPL_EALIGN  # cols % 8
+    assert L.spl_mask_split(None, base, base, base, base + 4, base, 2, 8, None) == spl.SPL_EALIGN
+    assert L.spl_mask_split(None, base, base, base, base, base, 1, 16392, None) == spl.SPL_ESHAPE  # row too long
+    assert L.spl_noise_mask_split(None, base, base, base, base, 2, 12, 1.0, 1.0, 0, rng, None) == spl.SPL_EALIGN
+    assert L.spl_noise_mask_split(None, None, base, base, base, 2, 8, 1.0, 1.0, 0, rng, None) == spl.SPL_EINVAL
+    # the tensor-core test hook refuses a persistent launch that breaks its conditions
+    w16 = spl.spl_weight(base, None, None, base, base, base)
+    for splits, seg, full in ((2, 0, 0), (1, 2, 0), (1, 0, 1)):
+        assert L.spl_test_tc_product(base, base, ctypes.byref(w16), None, 2, 8, 8, spl.SPL_PATH_FP16X3, 256, 192,
+                                     splits, full, seg, 1, None, 0, None) == spl.SPL_EINVAL
+    assert L.spl_test_tc_product(base, base, ctypes.byref(w16), None, 2, 8, 8, spl.SPL_PATH_FP16X3, 128, 96,
+                                 1, 0, 0, 1, None, 0, None) == spl.SPL_EINVAL  # two CTAs per SM: no persistent form
     stats = (ctypes.c_double * 27)()
     chosen = ctypes.c_int(5)
     assert L.spl_choose_path(ctypes.byref(chosen), stats, base, base, None, 4, 8, 8, None, 0, None) == spl.SPL_EINVAL
