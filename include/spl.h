@@ -336,9 +336,12 @@ spl_status spl_precompute_noise_product_matched_split(float* C, const spl_weight
  * library: 64 KiB of counters plus 4 MiB of partials, which every GPU that
  * loads the library holds until the process exits.  Nothing is allocated:
  * no cudaMalloc, cudaFree or allocating library routine is called.
- *  - The first call on a device (with that device current) looks up the
- *    array's device address and clears its counters; make that first call
- *    before any stream capture.
+ *  - Every call looks up the array's device address on the current device
+ *    (cudaGetSymbolAddress, which allocates nothing).  The first call on a
+ *    device, and the first after the library's module was loaded again (for
+ *    instance after cudaDeviceReset), also queues a clear of the counters on
+ *    `stream` ahead of its kernel; make that first call before any stream
+ *    capture, so that the clear runs when the call is made.
  *  - All calls share the one array, which keeps the last call's contents;
  *    each successful call leaves the counters at zero.  Calls that overlap on
  *    the GPU (on different streams or threads) race on it: serialise them.
@@ -466,6 +469,35 @@ uint64_t spl_launch_count(void);
 
 /* Static, NUL-terminated name of a status code. */
 const char* spl_status_string(spl_status status);
+
+/* ---- the boundary's call names as the problem statement lists them -------
+ * The calls of the masked-linear boundary follow the paper's statement of the
+ * problem (Sec. 3.3.1, Eq. add-and-then-subtract; the batched precompute of
+ * Sec. 5.2).  Most keep that name above; where the library's call is shaped
+ * differently, the listed name is kept as well:
+ *   spl_noise, spl_mask, spl_noise_mask, spl_unmask        -- as declared above
+ *   spl_masked_linear, spl_precompute_noise_product,
+ *   spl_masked_linear_unmask                                -- take the weight as a
+ *       const spl_weight* (W and its splits) instead of const float* W, plus a
+ *       workspace: a spl_weight with only `w` set is accepted and runs the
+ *       FP32 path (AUTO resolves to it; an explicit TF32X3 / FP16X3 reports
+ *       SPL_EUNSUPPORTED), so a caller holding only fp32 W passes {W}
+ *   spl_prepare_weight_split  -> spl_split_tf32 (the TF32X3 split, below) or
+ *       spl_split_fp16 (the FP16X3 split, the one the tensor-core products
+ *       prefer: 4 bytes per weight)
+ *   spl_get_last_device_status -> spl_get_device_status
+ *   spl_status_str             -> spl_status_string
+ * The three listed names are also exported with their listed signatures: */
+
+/* The TF32X3 split of a weight W[N, K] (fp32, device): W_hi = W rounded to
+ * TF32, W_lo = W - W_hi; spl_split_tf32 over the N K elements.  Errors as
+ * spl_split_tf32. */
+spl_status spl_prepare_weight_split(float* W_hi, float* W_lo, const float* W, int64_t N, int64_t K,
+                                    cudaStream_t stream);
+/* spl_get_device_status(stream). */
+spl_status spl_get_last_device_status(cudaStream_t stream);
+/* spl_status_string(status). */
+const char* spl_status_str(spl_status status);
 
 #ifdef __cplusplus
 }

@@ -596,3 +596,11 @@ extern "C" spl_status spl_split_tf32(float* hi, float* lo, const float* src, int
   if (!aligned16(hi) || !aligned16(lo) || !aligned16(src)) return SPL_EALIGN;
   return run_split_tf32(hi, lo, src, count, stream);
 }
+
+// The boundary's listed name for the TF32X3 weight split: spl_split_tf32 over the N x K weight.
+extern "C" spl_status spl_prepare_weight_split(float* W_hi, float* W_lo, const float* W, int64_t N, int64_t K,
+                                               cudaStream_t stream) {
+  if (N < 0 || K < 0) return SPL_EINVAL;
+  if (N > 0 && K > (int64_t(1) << 62) / N) return SPL_ESHAPE;
+  return spl_split_tf32(W_hi, W_lo, W, N * K, stream);
+}

@@ -550,20 +550,23 @@ constexpr int kMaxDev = 64;
 std::mutex g_static_mu;
 void* g_static_ptr[kMaxDev] = {nullptr};
 
-// Device address of g_static_scratch on the current device.  The first call on
-// a device looks it up (cudaGetSymbolAddress, with that device current) and
-// clears the counter region; later calls reuse the cached address.
-spl_status static_scratch(void** out) {
+// Device address of g_static_scratch on the current device, looked up on every call
+// (cudaGetSymbolAddress allocates nothing), so that an address from before a cudaDeviceReset is
+// never reused.  When the address is new for this device (its first call, or the module was
+// loaded again) a clear of the counter region is queued on the caller's stream, ahead of the
+// kernel that uses it; the array is zero when the module loads and every call that completes
+// leaves the counters at zero, so the clear is only a safeguard.
+spl_status static_scratch(void** out, cudaStream_t stream) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return SPL_ECUDA;
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) return SPL_ECUDA;
   std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_ptr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) return SPL_ECUDA;
-    if (cudaMemset(p, 0, kCounterBytes) != cudaSuccess) return SPL_ECUDA;
+  if (g_static_ptr[dev] != p) {
+    if (cudaMemsetAsync(p, 0, kCounterBytes, stream) != cudaSuccess) return SPL_ECUDA;
     g_static_ptr[dev] = p;
   }
-  *out = g_static_ptr[dev];
+  *out = p;
   return SPL_OK;
 }
 
@@ -588,7 +591,7 @@ extern "C" spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt
   if (plan.ws_partials > kStaticPartialBytes) return SPL_EWORKSPACE;  // beyond the built-in 4 MiB
   if (plan.splits > 1 && ceil_div(N, rows_per_block(padded_m(M))) > kMaxCounters) return SPL_EWORKSPACE;
   void* ws = nullptr;
-  spl_status st = static_scratch(&ws);
+  spl_status st = static_scratch(&ws, stream);
   if (st != SPL_OK) return st;
   LinearArgs args{};
   args.out = Y;

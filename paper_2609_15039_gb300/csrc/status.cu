@@ -67,3 +67,8 @@ extern "C" const char* spl_status_string(spl_status status) {
   }
   return "SPL_UNKNOWN";
 }
+
+// The boundary's listed names for the two status calls (the same calls as above).
+extern "C" spl_status spl_get_last_device_status(cudaStream_t stream) { return spl_get_device_status(stream); }
+
+extern "C" const char* spl_status_str(spl_status status) { return spl_status_string(status); }

@@ -91,6 +91,9 @@ _SIGS = {
     "spl_get_device_status": (_I, [_P]),
     "spl_launch_count": (ctypes.c_uint64, []),
     "spl_status_string": (ctypes.c_char_p, [_I]),
+    "spl_prepare_weight_split": (_I, [_P, _P, _P, _I64, _I64, _P]),
+    "spl_get_last_device_status": (_I, [_P]),
+    "spl_status_str": (ctypes.c_char_p, [_I]),
 }
 
 _lib = None
@@ -309,6 +312,15 @@ def spl_slalom_linear_unmask(Y, Xt_q, W_q, C, workspace=None, stream=None):
 def spl_split_tf32(hi, lo, src, stream=None):
     _check(lib().spl_split_tf32(_dev(hi, "hi"), _dev(lo, "lo"), _dev(src, "src"), src.numel(), _stream(stream)),
            "spl_split_tf32")
+
+
+def spl_prepare_weight_split(W_hi, W_lo, W, stream=None):
+    """The boundary's listed name for the TF32X3 weight split (spl_split_tf32 over W[N, K])."""
+    N, K = W.shape
+    if tuple(W_hi.shape) != (N, K) or tuple(W_lo.shape) != (N, K):
+        raise ValueError("spl_prepare_weight_split: shape mismatch")
+    _check(lib().spl_prepare_weight_split(_dev(W_hi, "W_hi"), _dev(W_lo, "W_lo"), _dev(W, "W"), N, K,
+                                          _stream(stream)), "spl_prepare_weight_split")
 
 
 def spl_split_fp16(hi, lo, row_exp, src, stream=None):
@@ -604,3 +616,13 @@ def spl_launch_count():
 
 def spl_get_device_status(stream=None):
     return lib().spl_get_device_status(_stream(stream))
+
+
+def spl_get_last_device_status(stream=None):
+    """The boundary's listed name for spl_get_device_status."""
+    return lib().spl_get_last_device_status(_stream(stream))
+
+
+def spl_status_str(status):
+    """The boundary's listed name for spl_status_string."""
+    return lib().spl_status_str(int(status)).decode()

@@ -119,6 +119,25 @@ def test_argument_validation_without_launch(spl):
     assert chosen.value == spl.SPL_PATH_FP32
 
 
+def test_listed_boundary_names(spl):
+    """The names the boundary's call list uses for the weight split and the status calls are exported
+    with their listed signatures and behave as the calls they stand for (no launch here)."""
+    names = declared_functions()
+    for listed in ("spl_prepare_weight_split", "spl_get_last_device_status", "spl_status_str"):
+        assert listed in names
+    L = spl.lib()
+    for st in range(9):
+        assert spl.spl_status_str(st) == spl.status_string(st)
+    buf = (ctypes.c_float * 64)()
+    p = ctypes.cast(buf, ctypes.c_void_p).value
+    base = p + (16 - p % 16) % 16
+    assert L.spl_prepare_weight_split(None, None, None, 0, 8, None) == spl.SPL_OK      # empty
+    assert L.spl_prepare_weight_split(None, None, None, -1, 8, None) == spl.SPL_EINVAL
+    assert L.spl_prepare_weight_split(None, base, base, 2, 8, None) == spl.SPL_EINVAL  # NULL W_hi
+    assert L.spl_prepare_weight_split(base + 4, base, base, 2, 8, None) == spl.SPL_EALIGN
+    assert L.spl_prepare_weight_split(base, base, base, 1 << 40, 1 << 40, None) == spl.SPL_ESHAPE
+
+
 def test_workspace_sizes_are_consistent(spl):
     # decode shapes need split-K partials after the 64 KiB counter region; the tensor-core
     # kernels reduce split-K in a cluster and keep only the split of the left operand there
