@@ -1,20 +1,30 @@
 #!/usr/bin/env python
 """Benchmark of the masked-linear hot path on one GB300.
 
-Workload (one step): one Llama-3.2-3B-shaped decoder layer's outsourced
-linears (Q, K, V, O, Gate, Up, Down) at 128 prompt tokens, fp32, Gaussian
-noise at eps = 1.  A step regenerates and adds the mask of each input group,
-then runs the masked product with the unmask fused into its epilogue
-(Y = X~ W^T - C).  Every 8 steps the correction bank is refilled: 8 masks
-per group are drawn and their corrections C = eta W^T computed as one
-product of 8 x 128 rows ("precomputed in a batch"), so each step carries an
-eighth of that work.  The weights (0.4 GB per layer in fp32, plus the TF32
-and fp16 splits) are larger than L2, so no step reuses L2-resident weights.
-The arithmetic path of each input group is chosen by the bound check on a
-masked sample (spl_choose_path) unless --path fixes it.
+Default workload (one step): one prefill of 512 tokens through a 28-layer
+Llama-3.2-3B-shaped linear stack (per layer Q|K|V 3072 -> 5120, O 3072 ->
+3072, Gate|Up 3072 -> 16384, Down 8192 -> 3072), fp32, Laplace noise at
+eps = 1, each layer seeded on its own.  A step draws and adds the mask of every
+input group of every layer (fused with the fp16 split the tensor-core product
+reads), runs the masked products with the unmask fused into their epilogues
+(Y = X~ W^T - C), and carries its share of the correction bank: the banks hold
+8 draws per group (C = eta W^T for 8 x 512 rows, summed in the online order),
+and each of the 8 steps of a cycle computes the next cycle's banks of an
+eighth of the layers on a lower-priority stream beside its own prefill.  So
+any number of steps times the whole method: prefill plus its correction.
+The weights (40 GB with their splits) are far larger than L2.
 
-Prints one JSON line.  ``--impl reference`` times the fp64 CPU oracle on a
-bounded sample of the same workload instead.
+Also reported on the same stack: the online prefill alone, the bank refill
+alone, the product kernels per launch (the roofline), decode at one token per
+step (tokens/s), the cancellation bound on every output of the first and last
+layer, Down on its own (its binary32 output is dominated by cancellation,
+which is why the paper keeps it in the enclave, and in binary64), the oracle
+on the host cores (cpu_baseline) and end to end through host memory (e2e).
+
+``--workload llama_layer`` is the one-layer, 128-token workload; the other
+``--workload`` values measure the Qwen workloads, the LM head and the
+comparators and print their own line.  ``--impl reference`` times the fp64
+CPU oracle on a bounded sample of the same workload instead.
 """
 
 import argparse
@@ -31,33 +41,50 @@ sys.path.insert(0, ROOT)
 METRIC = "masked-linear TFLOP/s & ms/prefill (Llama-3B shapes), % of roofline, oracle match"
 UNIT = "TFLOP/s"
 TF32_OVER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate on GB300
+DRAWS = 8
 WORKLOAD = ("llama-3.2-3b-shaped layer (Q,K,V,O,gate,up,down), 128 tokens, fp32, gaussian eps=1, "
             "corrections precomputed in banks of 8 draws")
-DRAWS = 8
+STACK_LAYERS, STACK_TOKENS, STACK_SEED, STACK_INPUT_SEED = 28, 512, 7, 11
+
+
+def stack_workload(layers, tokens, mech, eps):
+    return (f"llama-3.2-3b-shaped linear stack, {layers} layers (Q|K|V, O, Gate|Up, Down), prefill of {tokens} "
+            f"tokens, fp32, {mech} eps={eps:g}, per-layer seeds, corrections precomputed in banks of {DRAWS} "
+            f"draws (each step carries 1/{DRAWS} of the next cycle's banks)")
 
 
 def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=32)
+    ap.add_argument("--steps", type=int, default=24)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--eps", type=float, default=1.0)
     ap.add_argument("--path", default="auto")
-    ap.add_argument("--tokens", type=int, default=128)
+    ap.add_argument("--tokens", type=int, default=None, help="rows per step (stack: 512, llama_layer: 128)")
+    ap.add_argument("--layers", type=int, default=STACK_LAYERS, help="layers of the stack workload")
+    ap.add_argument("--mech", default=None, help="noise law (stack: laplace, llama_layer: gaussian)")
     ap.add_argument("--cpu-sample-rows", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-decode", action="store_true", help="stack: skip the one-token decode measurement")
+    ap.add_argument("--decode-steps", type=int, default=256)
     ap.add_argument("--no-overlap", action="store_true",
                     help="compute each bank cycle's corrections before its steps instead of during the previous cycle")
     ap.add_argument("--stored-noise", action="store_true",
-                    help="keep the bank's fp32 noise and mask each step with it instead of drawing it again")
-    ap.add_argument("--workload", default="llama_layer",
-                    choices=["llama_layer", "llama_stack", "qwen_stack", "qwen_sweep", "down_fp64", "slalom",
-                             "lm_head"],
-                    help="llama_layer (default): the headline line; the others measure the stack and sweep "
-                         "workloads and print their own line")
-    return ap.parse_args(argv)
+                    help="llama_layer: keep the bank's fp32 noise and mask each step with it instead of drawing it "
+                         "again")
+    ap.add_argument("--workload", default="llama_stack",
+                    choices=["llama_stack", "llama_layer", "llama_stack_detail", "qwen_stack", "qwen_sweep",
+                             "down_fp64", "slalom", "lm_head"],
+                    help="llama_stack (default): the headline line; llama_layer: one layer at 128 tokens; the "
+                         "others measure the other workloads and print their own line")
+    a = ap.parse_args(argv)
+    if a.tokens is None:
+        a.tokens = STACK_TOKENS if a.workload == "llama_stack" else 128
+    if a.mech is None:
+        a.mech = "laplace" if a.workload == "llama_stack" else "gaussian"
+    return a
 
 
 def peaks():
@@ -129,21 +156,23 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def profiled_traffic():
-    """DRAM bytes per step of the online product launches from the committed ncu summary, if it
-    was taken on the current tensor-core kernel source (else None)."""
+def profiled_traffic(profile="tc_gemm_fp16x3_llama_online_and_bank.md", field="traffic_bytes_per_step"):
+    """A DRAM byte count from a committed ncu summary, if it was taken on the current tensor-core
+    kernel source (else None)."""
     import hashlib
-    prof = os.path.join(ROOT, "profiles", "tc_gemm_fp16x3_llama_online_and_bank.md")
+    prof = os.path.join(ROOT, "profiles", profile)
     src = os.path.join(ROOT, "paper_2609_15039_gb300", "csrc", "gemm_tc.cu")
     try:
         fields = dict(line.split(":", 1) for line in open(prof).read().splitlines()
-                      if line.startswith(("traffic_bytes_per_step:", "kernel_source_sha256_prefix:")))
+                      if line.startswith((field + ":", "kernel_source_sha256_prefix:")))
         digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
     except (OSError, ValueError):
         return None, "no profile"
     if not digest.startswith(fields.get("kernel_source_sha256_prefix", "-").strip()):
         return None, "kernel changed since the ncu capture"
-    return float(fields["traffic_bytes_per_step"]), "ncu capture of the same kernel source (profiles/)"
+    if field not in fields:
+        return None, "no such figure in the profile"
+    return float(fields[field]), "ncu capture of the same kernel source (profiles/" + profile + ")"
 
 
 def max_over_ranks(x, device):
@@ -172,14 +201,16 @@ def dist_env():
 
 
 # ----------------------------------------------------------------------------- reference arm
-def oracle_sample(model, M, rows, eps, mech, seed, deltas, weights_cpu, inputs_cpu):
-    """The oracle on the first ``rows`` tokens of every group: noise, mask, products, unmask."""
+def oracle_sample(model, M, rows, eps, mech, seed, deltas, weights_cpu, inputs_cpu, offsets=None):
+    """The oracle on the first ``rows`` tokens of every group: noise, mask, products, unmask.
+    offsets: {group: first Philox block of the draw} (default 0)."""
     from oracle import linear, philox
     out = {}
     flops = 0
     for gi, (g, K, names) in enumerate(model.input_groups()):
         X = inputs_cpu[g][:rows]
-        eta = philox.noise((M, K), deltas[g], eps, mech, seed, stream_id=gi)[:rows]
+        off = (offsets or {}).get(g, 0)
+        eta = philox.noise((rows, K), deltas[g], eps, mech, seed, stream_id=gi, offset=off)
         Xt = linear.mask(X, eta)
         for name in names:
             W = weights_cpu[name]
@@ -190,12 +221,22 @@ def oracle_sample(model, M, rows, eps, mech, seed, deltas, weights_cpu, inputs_c
     return out, flops
 
 
-def cpu_setup(model, M):
+def cpu_setup(model, M, weight_seed=None, input_seed=None):
+    """Seeded inputs of one layer on the host (the stack's layer 0 when seeds are given, else the
+    one-layer workload's), and the noise scales of Thms. 1-3 from the oracle."""
     import numpy as np
     from oracle import sensitivity as osens
     from paper_2609_15039_gb300 import workloads as wl
-    weights = {name: wl.weight(N, K, seed=200 + pi).numpy() for pi, (name, K, N, g) in enumerate(model.projections())}
-    inputs = {g: wl.activations(M, K, seed=100 + gi).numpy() for gi, (g, K, _n) in enumerate(model.input_groups())}
+    if weight_seed is None:
+        weights = {name: wl.weight(N, K, seed=200 + pi).numpy() for pi, (name, K, N, g) in
+                   enumerate(model.projections())}
+        inputs = {g: wl.activations(M, K, seed=100 + gi).numpy() for gi, (g, K, _n) in
+                  enumerate(model.input_groups())}
+    else:
+        weights = {name: wl.weight(N, K, seed=wl.layer_seed(weight_seed, 0, pi)).numpy()
+                   for pi, (name, K, N, g) in enumerate(model.projections())}
+        inputs = {g: wl.activations(M, K, seed=wl.layer_seed(input_seed, 0, 50 + gi)).numpy()
+                  for gi, (g, K, _n) in enumerate(model.input_groups())}
     ones = np.ones(model.d_model)
     norms = {n: osens.spectral_norm(weights[n], iters=30) for n in ("v", "up", "gate")}
     deltas = {"qkv": osens.delta_layernorm(ones), "gateup": osens.delta_layernorm(ones),
@@ -205,28 +246,37 @@ def cpu_setup(model, M):
 
 
 def run_reference(args):
+    """The fp64 CPU oracle, as it stands, on a bounded sample of the workload's step: the first
+    rows of every input group of one layer per step (stack: its layer 0)."""
     world, rank, _ = dist_env()
     if rank != 0:
         return
     from paper_2609_15039_gb300 import workloads as wl
     model, M = wl.LLAMA_3_2_3B, args.tokens
-    weights, inputs, deltas = cpu_setup(model, M)
+    stack = args.workload == "llama_stack"
+    if stack:
+        weights, inputs, deltas = cpu_setup(model, M, STACK_SEED, STACK_INPUT_SEED)
+        workload = stack_workload(args.layers, M, args.mech, args.eps)
+    else:
+        weights, inputs, deltas = cpu_setup(model, M)
+        workload = WORKLOAD
     rows = args.cpu_sample_rows
     for w in range(args.warmup):
-        oracle_sample(model, M, rows, args.eps, "gaussian", 1000 + w, deltas, weights, inputs)
+        oracle_sample(model, M, rows, args.eps, args.mech, 1000 + w, deltas, weights, inputs)
     t0 = time.perf_counter()
     flops = 0
     for s in range(args.steps):
-        _, f = oracle_sample(model, M, rows, args.eps, "gaussian", 2000 + s, deltas, weights, inputs)
+        _, f = oracle_sample(model, M, rows, args.eps, args.mech, 2000 + s, deltas, weights, inputs)
         flops += f
     dt = time.perf_counter() - t0
     value = flops / dt / 1e12
-    sample = f"first {rows} of {M} tokens of every input group, all 7 projections, per step"
+    sample = (f"first {rows} of {M} tokens of every input group of one layer (all 7 projections: noise, mask, "
+              f"masked product, correction, unmask in fp64) per step")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "tokens": M, "eps": args.eps},
+        "config": {"workload": workload, "tokens": M, "eps": args.eps, "mech": args.mech},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
@@ -241,7 +291,7 @@ def run_workload(args):
     torch.cuda.set_device(local)
     with ClockSampler(local) as clocks:
         res = measure.WORKLOADS[args.workload]()
-    if args.workload == "llama_stack":
+    if args.workload == "llama_stack_detail":
         value, unit, ms = res["prefill"]["tflops"], UNIT, res["prefill"]["ms_per_prefill"]
     elif args.workload == "qwen_stack":
         first = next(iter(res["prefill"].values()))
@@ -270,8 +320,15 @@ def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "llama_stack":
+        return run_llama_stack(args)
     if args.workload != "llama_layer":
         return run_workload(args)
+    return run_llama_layer(args)
+
+
+def run_llama_layer(args):
+    """The one-layer workload: a Llama-3.2-3B-shaped layer at 128 tokens, banks of 8 draws."""
     import numpy as np
     import torch
     import torch.distributed as dist
@@ -283,7 +340,7 @@ def main():
         dist.init_process_group("nccl", init_method="env://")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    model, M, mech, seed = wl.LLAMA_3_2_3B, args.tokens, "gaussian", 4242
+    model, M, mech, seed = wl.LLAMA_3_2_3B, args.tokens, args.mech, 4242
 
     weights = {name: wl.weight(N, K, seed=200 + pi, device=dev) for pi, (name, K, N, g) in
                enumerate(model.projections())}
@@ -550,7 +607,6 @@ def main():
                                     else "drawn again in each step's mask"),
                    "l2": "weights 1.2 GB per step > 129 MB L2 (no flush needed)",
                    "parallelism": "replicas" if world > 1 else "single"},
-        "ms_per_prefill_28_layers": 28 * ms,
         "roofline": roofline,
         "gpu_launches": gpu_launches,
         "clocks": clocks.summary(),
@@ -609,6 +665,402 @@ def main():
                                   "sample": f"first {rows} of {M} tokens of every input group, {reps} repetitions"}
         result["oracle_match"] = {"rows_checked": rows, "max_err_over_hard_bound": worst, "pass": worst <= 1.0}
 
+    if rank == 0:
+        print(json.dumps(result))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def path_peaks(pk):
+    """Algorithmic flops per second at each path's instruction peak: FP16X3 = the measured
+    sustained bf16 rate (fp16 runs at the bf16 rate) / 3 products per term; TF32X3 = that x the
+    nominal TF32 : bf16 ratio; FP32 = 152 SMs x 128 lanes x 2 flops x 2.07 GHz (derived)."""
+    return {"fp16x3": pk["bf16_tflops_sustained"] / 3.0,
+            "tf32x3": pk["bf16_tflops_sustained"] * TF32_OVER_BF16 / 3.0,
+            "fp32": 152 * 128 * 2 * 2.07e9 / 1e12}
+
+
+PEAK_NOTE = ("fp16x3 = measured sustained bf16 (fp16 runs at the bf16 rate) / 3 products per term; tf32x3 = that x "
+             "the nominal tf32/bf16 ratio (1.1/2.25, not measured); fp32 FMA = 152 SMs x 128 lanes x 2 flop x "
+             "2.07 GHz (derived); hbm = measured copy bandwidth")
+
+
+def _time_graphs(graph_of, s0, n, stream):
+    """Replays graph_of(s) for s = s0 .. s0 + n - 1 with a CUDA event after each; per-step ms."""
+    import torch
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    ev[0].record(stream)
+    for i in range(n):
+        graph_of(s0 + i).replay()
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize()
+    return [ev[i].elapsed_time(ev[i + 1]) for i in range(n)]
+
+
+def run_llama_stack(args):
+    """The headline line: prefill of 512 tokens through the 28-layer Llama-3.2-3B-shaped stack, each
+    step carrying its share of the next bank cycle (see the module docstring)."""
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    from paper_2609_15039_gb300 import measure, spl, workloads as wl
+    from paper_2609_15039_gb300.layer import MaskedStack
+
+    world, rank, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    model, L, M, D, mech, eps, path = wl.LLAMA_3_2_3B, args.layers, args.tokens, DRAWS, args.mech, args.eps, args.path
+    pk = peaks()
+    ppk = path_peaks(pk)
+    t_build = time.perf_counter()
+    stack = MaskedStack.build(model, L, M, D, base_seed=STACK_SEED, device=dev, path=path)
+    inputs = stack.inputs(STACK_INPUT_SEED, device=dev)
+    if path == "auto":
+        # a8 is evaluated per (shape, eps): on layer 0's weights and a masked sample of its input, and
+        # the choice kept for every layer of the same shapes
+        l0 = stack.layers[0]
+        l0.calibrate(inputs[0], eps, mech, stack.seeds[0])
+        for layer in stack.layers[1:]:
+            layer.paths = dict(l0.paths)
+    layer0 = stack.layers[0]
+    groups = layer0.groups
+    group_paths = {g.name: spl.PATH_NAMES[spl.spl_resolve_path(M, g.K, g.N, layer0.path_of(g, path, M))]
+                   for g in groups}
+    bank_ws = spl.workspace(max(l.workspace_bytes(M, D, path) for l in stack.layers), dev)
+    stream = torch.cuda.current_stream(dev)
+    stack.step(inputs, eps, mech, 0, path=path)  # sets up every library call before capture
+    torch.cuda.synchronize()
+    build_s = time.perf_counter() - t_build
+
+    flops_layer = {g.name: 2 * M * g.K * g.N for g in groups}
+    flops_step = L * sum(flops_layer.values())  # the masked products of one prefill (algorithmic)
+
+    # ---- the timed steps: prefill + 1/D of the next cycle's banks per graph ----------------------
+    overlap = not args.no_overlap
+    if overlap:
+        graphs, glaunch = stack.capture_steps(inputs, eps, mech, bank_ws, path=path)
+        graph_of = lambda s: graphs[(s // D) % 2][s % D]
+        launches_of = lambda s: glaunch[(s // D) % 2][s % D]
+    else:
+        graphs, glaunch = stack.capture(inputs, eps, mech, path=path)
+        graph_of = lambda s: graphs[s % D]
+        launches_of = lambda s: glaunch[s % D]
+
+    def prime(cycle):
+        """Device-side Philox bases at ``cycle`` and, for the overlapped graphs, that cycle's banks."""
+        stack.set_cycle(cycle)
+        if overlap:
+            stack.refill_all(eps, mech, path, parity=cycle % 2, workspace=bank_ws)
+
+    s = D  # every pass starts at a bank cycle
+    prime(s // D)
+    for _ in range(args.warmup):
+        graph_of(s).replay()
+        s += 1
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s_timed = s
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_push("timed")
+        t_start.record(stream)
+        for _ in range(args.steps):
+            graph_of(s).replay()
+            s += 1
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
+    if world > 1:
+        dist.barrier()
+    ms = max_over_ranks(t_start.elapsed_time(t_end) / args.steps, dev)
+    gpu_launches = sum(launches_of(s_timed + i) for i in range(args.steps))
+    st = spl.spl_get_device_status()
+    if st != spl.SPL_OK:
+        raise RuntimeError("device status " + spl.status_string(st))
+    value = job_rate(world, flops_step, ms) / 1e12
+
+    # ---- the online prefill alone, and its product calls (event pairs around each) ---------------
+    on_graphs, on_launch = stack.capture(inputs, eps, mech, path=path, refill=False)
+    stack.set_cycle(1)
+    _time_graphs(lambda i: on_graphs[i % D], 0, D, stream)  # warm-up cycle
+    on_times = _time_graphs(lambda i: on_graphs[i % D], 0, 2 * D, stream)
+    ms_online = sum(on_times) / len(on_times)
+    del on_graphs
+    ev = {}
+
+    def timer(d, li, phase, kind, group):
+        if kind != "masked_linear_unmask":
+            return
+        e = torch.cuda.Event(enable_timing=True, external=True)
+        e.record()
+        ev.setdefault((d, li, group), [None, None])[0 if phase == "begin" else 1] = e
+
+    ev_graphs, _ = stack.capture(inputs, eps, mech, path=path, refill=False, timer=timer)
+    stack.set_cycle(1)
+    _time_graphs(lambda i: ev_graphs[i % D], 0, D, stream)  # each graph's events hold its last replay
+    per_group = {}
+    for (d, li, gname), (b, e) in ev.items():
+        per_group.setdefault(gname, []).append(b.elapsed_time(e))
+    del ev_graphs
+    prod = {}
+    for g in groups:
+        t = per_group[g.name]
+        avg = sum(t) / len(t)
+        prod[g.name] = {"calls": len(t), "avg_us": 1e3 * avg, "tflops": flops_layer[g.name] / (avg * 1e-3) / 1e12,
+                        "path": group_paths[g.name], "peak": ppk[group_paths[g.name]],
+                        "frac": flops_layer[g.name] / (avg * 1e-3) / 1e12 / ppk[group_paths[g.name]]}
+    prod_ms_layer = sum(p["avg_us"] for p in prod.values()) / 1e3
+    prod_flops_layer = sum(flops_layer.values())
+    prod_peak = prod_flops_layer / sum(flops_layer[n] / ppk[group_paths[n]] for n in flops_layer)
+    achieved = prod_flops_layer / (prod_ms_layer * 1e-3) / 1e12
+    traffic, traffic_note = profiled_traffic("tc_prefill_fp16x3_llama_512.md", "traffic_bytes_per_launch")
+    roofline = {
+        "bound": "tensor", "achieved": achieved, "peak": prod_peak, "unit": "TFLOP/s", "frac": achieved / prod_peak,
+        "traffic": traffic,
+        "kernel": (f"masked products with fused unmask at {M} rows (tc_persistent_kernel / tc_gemm_kernel, FP16X3 "
+                   f"on tcgen05): one call per input group, {len(groups)} per layer, {len(groups) * L} per prefill"),
+        "flops_per_launch": prod_flops_layer / len(groups), "avg_launch_us": 1e3 * prod_ms_layer / len(groups),
+        "per_group": prod, "share_of_online_prefill": L * prod_ms_layer / ms_online,
+        "timing": ("CUDA event pairs (external event nodes, on the launching stream) around every product call of "
+                   f"the 28 layers in graph-replayed online prefills (one bank cycle, {D} prefills); achieved = the "
+                   "calls' algorithmic flops / their summed durations"),
+        "traffic_note": traffic_note + "; DRAM bytes per call, averaged over the four calls of a layer",
+        "peak_source": pk["source"], "peak_note": "sustained peak (the calls run inside 8 ms prefills); " + PEAK_NOTE}
+
+    # ---- the bank refill alone: every layer's next cycle (D draws of M rows per group) ----------
+    bank_graph = torch.cuda.CUDAGraph()
+    n0 = spl.spl_launch_count()
+    with torch.cuda.graph(bank_graph):
+        stack.refill_all(eps, mech, path, parity=0, workspace=bank_ws)
+    bank_launches = spl.spl_launch_count() - n0
+    bank_times = _time_graphs(lambda i: bank_graph, 0, 3, stream)[1:]
+    bank_ms = sum(bank_times) / len(bank_times)
+    del bank_graph
+    bank_flops = D * flops_step
+    bank_peak = prod_peak
+    bank = {"ms_per_cycle": bank_ms, "ms_per_prefill": bank_ms / D, "tflops": bank_flops / (bank_ms * 1e-3) / 1e12,
+            "peak": bank_peak, "frac": bank_flops / (bank_ms * 1e-3) / 1e12 / bank_peak, "launches": bank_launches,
+            "what": (f"{D} noise draws per input group and layer (split as drawn) and their corrections as one "
+                     f"product of {D * M} rows per group, summed in the online product's order")}
+
+    # ---- end to end: the same steps with every layer's input copied in from pinned host memory
+    # and every output copied back, inside each step's graph, on two copy streams ----------------
+    e2e = None
+    if not args.no_e2e:
+        host_in = [{g: x.cpu().pin_memory() for g, x in inp.items()} for inp in inputs]
+        host_out = [{g.name: torch.empty((M, g.N)).pin_memory() for g in layer.groups} for layer in stack.layers]
+        h2d = sum(x.numel() * 4 for inp in host_in for x in inp.values())
+        d2h = sum(o.numel() * 4 for out in host_out for o in out.values())
+
+        def copy_in(li):
+            for g, x in inputs[li].items():
+                x.copy_(host_in[li][g], non_blocking=True)
+            e = torch.cuda.Event()
+            e.record()
+            return e
+
+        def copy_out(li):
+            layer = stack.layers[li]
+            for g in layer.groups:
+                host_out[li][g.name].copy_(layer.bank[g.name]["Y"], non_blocking=True)
+
+        if overlap:
+            e2e_graphs, _ = stack.capture_steps(inputs, eps, mech, bank_ws, path=path, copies=(copy_in, copy_out))
+            e2e_of = lambda s: e2e_graphs[(s // D) % 2][s % D]
+        else:
+            raise SystemExit("--no-overlap runs without --no-e2e are not supported on the stack workload")
+        s = -(-s // D) * D
+        prime(s // D)
+        for _ in range(2):
+            e2e_of(s).replay()
+            s += 1
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            e2e_of(s).replay()
+            s += 1
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, dev)
+        e2e = {"value": job_rate(world, flops_step, e2e_ms) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+               "copies": ("pinned host memory: each step's graph copies every layer's inputs in on one copy stream "
+                          "(layer l computes once its copy has landed) and every layer's outputs back on another, "
+                          "after the layer's products; the step ends when both are done")}
+        del e2e_graphs, host_in, host_out
+    st = spl.spl_get_device_status()
+    if st != spl.SPL_OK:
+        raise RuntimeError("device status " + spl.status_string(st))
+
+    # ---- the cancellation bound over every output of the first and last layer (an eager step) ---
+    bound = measure._bound(stack, inputs, eps, mech, 3 * D + 1, [0, L - 1])
+    for lk, groups_bc in bound.items():
+        for gname, v in groups_bc.items():
+            v.pop("mean_log_bound", None)
+
+    # ---- Down on its own path (Sec. 5.5): binary32 (the step's) and binary64, layer 0 -----------
+    down = {}
+    gd = layer0.group("down")
+    if gd is not None:
+        gi = [g.name for g in groups].index("down")
+        Xd = inputs[0]["down"]
+        delta = layer0.deltas["down"]
+        eta = torch.empty((M, gd.K), device=dev)
+        xt64 = torch.empty((M, gd.K), dtype=torch.float64, device=dev)
+        spl.spl_noise(eta, delta, eps, mech, stack.seeds[0], stream_id=gi, offset=0)
+        spl.spl_noise_mask_f64(xt64, Xd, delta, eps, mech, stack.seeds[0], stream_id=gi, offset=0)
+        ws64 = spl.workspace(spl.spl_f64_workspace_bytes(M, gd.K, gd.N), dev)
+        C64 = torch.empty((M, gd.N), dtype=torch.float64, device=dev)
+        spl.spl_precompute_noise_product_f64(C64, eta, gd.W, workspace=ws64)
+        Y64 = torch.empty((M, gd.N), device=dev)
+        spl.spl_masked_linear_unmask_f64(Y64, xt64, gd.W, C64, workspace=ws64)  # warm-up
+        torch.cuda.synchronize()
+        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        d0.record(stream)
+        spl.spl_masked_linear_unmask_f64(Y64, xt64, gd.W, C64, workspace=ws64)
+        d1.record(stream)
+        torch.cuda.synchronize()
+        bc64 = spl.spl_bound_check(Y64, Xd, xt64.float().contiguous(), eta, gd.W)
+        b32 = bound["layer0"]["down"]
+        down = {"note": ("the paper keeps Down in the enclave (Sec. 5.5): its Delta (Thm. 3) is ~3e8, so the "
+                         "binary32 recovered output is dominated by cancellation error, though inside the bound"),
+                "binary32": {"path": group_paths["down"], "us_per_call": prod["down"]["avg_us"],
+                             "tflops": prod["down"]["tflops"], "max_rel_err": b32["max_rel_err"],
+                             "mean_err": b32["mean_err"], "max_err_over_hard": b32["max_err_over_hard"]},
+                "binary64": {"ms_per_call": d0.elapsed_time(d1), "rows": M,
+                             "tflops": flops_layer["down"] / (d0.elapsed_time(d1) * 1e-3) / 1e12,
+                             "max_rel_err": bc64["max_err"] / bc64["max_abs_ref"] if bc64["max_abs_ref"] else 0.0,
+                             "mean_err": bc64["mean_err"]}}
+        del eta, xt64, C64, Y64, ws64
+    six = [n for n in prod if n != "down"]
+    six_flops = sum(flops_layer[n] for n in six)
+    six_ms = sum(prod[n]["avg_us"] for n in six) / 1e3
+    offloaded = {"projections": "Q, K, V, O, Gate, Up", "tflops": six_flops / (six_ms * 1e-3) / 1e12,
+                 "frac": six_flops / (six_ms * 1e-3) / 1e12 /
+                 (six_flops / sum(flops_layer[n] / ppk[group_paths[n]] for n in six)),
+                 "max_rel_err": max(bound[lk][n]["max_rel_err"] for lk in bound for n in six),
+                 "max_err_over_hard": max(bound[lk][n]["max_err_over_hard"] for lk in bound for n in six),
+                 "timing": "product calls alone, from the roofline's event pairs"}
+
+    # ---- cpu baseline + oracle match on the first rows of layer 0 (rank 0, N = 1 only) -----------
+    cpu = match = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from oracle import bounds, linear, philox
+        rows = args.cpu_sample_rows
+        cycle, d = 5, 3
+        seed0 = stack.seeds[0]
+        layer0.refill(eps, mech, seed0, cycle, path=path)
+        outs = layer0.online(inputs[0], eps, mech, seed0, cycle, d, path=path)
+        torch.cuda.synchronize()
+        gpu_rows = {g: outs[g][:rows].double().cpu().numpy() for g in outs}
+        w_cpu = {g.name: g.W.cpu().numpy() for g in groups}
+        x_cpu = {g: x[:rows].cpu().numpy() for g, x in inputs[0].items()}
+        t0, flops, reps, worst = time.perf_counter(), 0, 0, 0.0
+        while True:
+            for gi, g in enumerate(groups):
+                X = x_cpu[g.name]
+                eta = philox.noise((rows, g.K), layer0.deltas[g.name], eps, mech, seed0, stream_id=gi,
+                                   offset=layer0.block_offset(g, cycle, d))
+                Xt = linear.mask(X, eta)
+                r = linear.masked_linear(Xt, w_cpu[g.name])
+                C = linear.precompute_noise_product(eta, w_cpu[g.name])
+                linear.unmask(r.astype(np.float32), C.astype(np.float32))
+                flops += 2 * 2 * rows * g.K * g.N
+                if reps == 0:
+                    S = linear.abs_products(X, Xt, eta, w_cpu[g.name])
+                    err = np.abs(gpu_rows[g.name] - linear.reference_output(X, w_cpu[g.name]))
+                    worst = max(worst, float(np.max(err / bounds.hard_bound(*S, g.K))))
+            reps += 1
+            if time.perf_counter() - t0 > 10.0 or reps >= 50:
+                break
+        dt = time.perf_counter() - t0
+        cpu = {"value": flops / dt / 1e12, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "seconds": dt,
+               "sample": (f"first {rows} of {M} tokens of every input group of layer 0 (all 7 projections: noise, "
+                          f"mask, masked product, correction, unmask in fp64), {reps} repetitions; the rate is the "
+                          f"sample's flops over its time")}
+        match = {"rows_checked": rows, "layer": 0, "max_err_over_hard_bound": worst, "pass": worst <= 1.0}
+
+    # ---- decode at one token per step (the same layers, banks of D one-row draws) -----------------
+    decode = None
+    if not args.no_decode:
+        del graphs
+        torch.cuda.synchronize()
+        ws1 = spl.workspace(max(l.workspace_bytes(1, D) for l in stack.layers), dev)
+        for layer in stack.layers:
+            layer.allocate(1, D, workspace=ws1)
+        del bank_ws
+        torch.cuda.empty_cache()
+        inputs1 = stack.inputs(13, device=dev)
+        stack.step(inputs1, eps, mech, 0)
+        torch.cuda.synchronize()
+        bank_ws1 = spl.workspace(max(l.workspace_bytes(1, D) for l in stack.layers), dev)
+        ov_graphs, ol = stack.capture_overlapped(inputs1, eps, mech, bank_ws1)
+        cycles = max(1, -(-args.decode_steps // D))
+        stack.start_overlapped(1, eps, mech)
+        _time_graphs(lambda i: ov_graphs[(1 + i) % 2], 0, 2, stream)  # cycles 1 and 2
+        times = _time_graphs(lambda i: ov_graphs[(3 + i) % 2], 0, cycles, stream)
+        step_ms = sum(times) / (cycles * D)
+        dpaths = {g.name: spl.PATH_NAMES[spl.spl_resolve_path(1, g.K, g.N, layer0.path_of(g, "auto", 1))]
+                  for g in groups}
+        step_bytes = sum(4 * g.K * g.N + 4 * g.K + 8 * g.N for g in groups) * L * (1 + 1.0 / D)
+        decode = {"steps": cycles * D, "ms_per_token": step_ms, "tokens_per_s": 1e3 / step_ms,
+                  "gbs": step_bytes / (step_ms * 1e-3) / 1e9, "peak_gbs": pk["hbm_gbs"],
+                  "frac": step_bytes / (step_ms * 1e-3) / 1e9 / pk["hbm_gbs"], "bytes_per_step": step_bytes,
+                  "paths": dpaths, "kernels_per_step": sum(ol) / len(ol) / D,
+                  "schedule": ("whole-cycle graphs: each cycle's 8 one-token steps through every layer, and beside "
+                               "them on a lower-priority stream the next cycle's corrections (bytes per step: every "
+                               "weight once, x~, C and Y, plus 1/8 of the bank's weight reads)")}
+        del ov_graphs
+        st = spl.spl_get_device_status()
+        if st != spl.SPL_OK:
+            raise RuntimeError("device status " + spl.status_string(st))
+
+    path_name = "+".join(sorted(set(group_paths.values())))
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "path": path_name, "data": "synthetic",
+        "config": {"workload": stack_workload(L, M, mech, eps), "layers": L, "tokens": M, "eps": eps, "mech": mech,
+                   "bank_draws": D, "flops_per_step": flops_step,
+                   "value": ("algorithmic flops of the prefill's masked products (2 M K N per projection, 28 layers) "
+                             "per second of the whole step: online prefill plus its 1/8 share of the bank"),
+                   "bank_schedule": ("each step computes the next cycle's corrections of an eighth of the layers on a "
+                                     "lower-priority stream beside its prefill (per-step graphs)") if overlap else
+                                    "each cycle's corrections computed before its first step",
+                   "online_noise": "drawn again in each step's mask from the bank's Philox counters",
+                   "l2": "weights 40 GB per step (with their splits) >> 129 MB L2 (no flush needed)",
+                   "parallelism": "replicas" if world > 1 else "single", "setup_s": build_s},
+        "prefill": {"ms_per_prefill_with_correction": ms, "tokens_per_s": M / (ms * 1e-3),
+                    "online_only": {"ms_per_prefill": ms_online, "tflops": flops_step / (ms_online * 1e-3) / 1e12,
+                                    "frac": flops_step / (ms_online * 1e-3) / 1e12 / prod_peak,
+                                    "tokens_per_s": M / (ms_online * 1e-3), "kernels": on_launch[1]},
+                    "correction_serial_ms_per_prefill": bank_ms / D,
+                    "serial_sum_ms": ms_online + bank_ms / D},
+        "bank": bank,
+        "roofline": roofline,
+        "gpu_launches": gpu_launches,
+        "clocks": clocks.summary(),
+    }
+    if e2e is not None:
+        result["e2e"] = e2e
+    if decode is not None:
+        result["decode"] = decode
+    result["offloaded_six"] = offloaded
+    if down:
+        result["down"] = down
+    result["bound_check"] = bound
+    if layer0.calibration:
+        result["path_choice"] = {g: {"path": c["path"], **{f"{p}_max_err_over_hard": c[p]["max_err_over_hard"]
+                                                          for p in ("fp32", "tf32x3", "fp16x3")}}
+                                 for g, c in layer0.calibration.items()}
+    if cpu is not None:
+        result["cpu_baseline"] = cpu
+        result["oracle_match"] = match
     if rank == 0:
         print(json.dumps(result))
     if world > 1:

@@ -61,7 +61,11 @@ typedef enum spl_mech { SPL_MECH_LAPLACE = 0, SPL_MECH_GAUSSIAN = 1 } spl_mech;
  *  FP16X3 -- the same three products in fp16 (kind::f16, twice the TF32 rate)
  *            on rows scaled by powers of two, undone exactly in the epilogue;
  *            needs the weight split of spl_split_fp16 (4 bytes per weight)
- *            and K % 8 == 0.
+ *            and K % 8 == 0.  Per-term error about 2^-21 |a w| plus an
+ *            absolute 2^-39 max|a_row| |w| for entries that fall below fp16's
+ *            normal range after the row scaling (more than ~2^-28 under the
+ *            row's largest); spl_choose_path judges whether that stays inside
+ *            the bound for the data at hand.
  *  AUTO   -- the library's choice (spl_resolve_path). */
 typedef enum spl_path {
   SPL_PATH_AUTO = 0,

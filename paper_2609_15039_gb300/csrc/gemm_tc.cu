@@ -9,13 +9,18 @@
 //           kind::tf32, K = 8 per instruction, 8 bytes per element.
 //   FP16X3  each row is first scaled by a power of two so its largest entry lies in
 //           [2^14, 2^15); hi = fp16(a 2^e), lo = fp16(a 2^e - hi) (11 + 11 significant
-//           bits); per-term error ~2^-21 |a w|.  kind::f16 runs at twice the TF32 rate
-//           and the split is 4 bytes per element; the power-of-two scales are undone
-//           exactly in the epilogue.
-// Either way each term is within about 3 x 2^-21 of exact, below gamma_K = K 2^-24 for
-// K >= 64, so the masked product r = W x~ (Sec. 5.1) and the correction W eta (Sec. 5.2)
-// stay inside the binary32 error model the paper's Thm. 4 is built on while running on
-// the tensor pipe.  W is split once, offline; A is split by a pass before the product
+//           bits).  kind::f16 runs at twice the TF32 rate and the split is 4 bytes per
+//           element; the power-of-two scales are undone exactly in the epilogue.  Per-term
+//           error about 2^-21 |a w| + 2^-39 max|a_row| |w|: an entry more than ~2^-28
+//           below its row's largest falls into fp16's subnormal range, where hi + lo keeps
+//           an absolute (not relative) error of 2^-25 in the scaled units.
+// For rows of ordinary dynamic range each term is within about 3 x 2^-21 of exact, below
+// gamma_K = K 2^-24 for K >= 64, so the masked product r = W x~ (Sec. 5.1) and the
+// correction W eta (Sec. 5.2) stay inside the binary32 error model the paper's Thm. 4 is
+// built on while running on the tensor pipe.  Rows whose small entries carry the sum
+// while their large ones meet tiny weights can push the FP16X3 floor past that bound;
+// the bound-based path choice on sampled data (spl_choose_path) then takes TF32X3 (whose
+// split keeps fp32's exponent range) or FP32.  W is split once, offline; A is split by a pass before the product
 // into the workspace, so TMA lands every operand tile directly.
 //
 // Kernel shape (one CTA per 128 x BN output tile, 6 warps; BN = 256 with a 192 KB ring and

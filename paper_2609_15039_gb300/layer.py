@@ -188,7 +188,8 @@ class MaskedLayer:
             b = self.bank[g.name]
             if "Cs" not in b:
                 b["Cs"] = [b["C"], torch.empty_like(b["C"])]
-                b["etas"] = [b["eta"], torch.empty_like(b["eta"])]
+                # the fp32 noise is read again only with stored noise; otherwise one buffer serves
+                b["etas"] = [b["eta"], torch.empty_like(b["eta"]) if self.stored_noise else b["eta"]]
 
     def _C(self, g, parity):
         b = self.bank[g.name]
@@ -566,6 +567,83 @@ class MaskedStack:
             graphs.append(graph)
             launches.append(spl.spl_launch_count() - n0)
         return graphs, launches
+
+    def bank_slice(self, d):
+        """Layers whose next-cycle corrections step d of a cycle computes (capture_steps): the
+        layers split as evenly as whole layers allow over the ``draws`` steps."""
+        L, D = len(self.layers), self.draws
+        return range(d * L // D, (d + 1) * L // D)
+
+    def capture_steps(self, inputs, eps, mech, bank_workspace, path="auto", timer=None, copies=None):
+        """CUDA graphs of single steps, each carrying its share of the next bank cycle: graphs[p][d]
+        runs step d of a cycle through every layer on correction buffers p while, on a stream of
+        lower priority, the layers of bank_slice(d) compute their next-cycle corrections into buffers
+        1 - p (with ``bank_workspace``, at least max(layer.workspace_bytes(M, draws))); the graph ends
+        when both are done, and graph d = draws - 1 moves every Philox base on by one cycle.  After
+        start_overlapped(c), replay graphs[(s // draws) % 2][s % draws] for steps s = c draws, c
+        draws + 1, ... -- any number of them: every step holds its online pass and an equal share of
+        the refill, so a run of any length times the whole method.  ``timer(d, li, phase, kind,
+        group)`` as in capture.  ``copies``: (h2d, d2h) host-transfer hooks -- h2d(li) is called on
+        the host-to-device copy stream before the online steps, once per layer in order, and returns
+        an event that layer li's online work waits for; d2h(li) is called on the device-to-host copy
+        stream after layer li's online work (which that stream waits for first).  Returns the graphs
+        and their kernel counts."""
+        lo, hi = torch.cuda.Stream.priority_range()
+        if not hasattr(self, "_bank_stream"):
+            self._bank_stream = torch.cuda.Stream(priority=lo)
+            self._online_stream = torch.cuda.Stream(priority=hi)
+        if copies is not None and not hasattr(self, "_h2d_stream"):
+            self._h2d_stream = torch.cuda.Stream(priority=hi)
+            self._d2h_stream = torch.cuda.Stream(priority=hi)
+        for layer in self.layers:
+            layer.enable_overlap()
+        D = self.draws
+        graphs, launches = [[], []], [[], []]
+        for parity in range(2):
+            for d in range(D):
+                graph = torch.cuda.CUDAGraph()
+                n0 = spl.spl_launch_count()
+                with torch.cuda.graph(graph, stream=self._online_stream):
+                    main = torch.cuda.current_stream()
+                    self._bank_stream.wait_stream(main)
+                    with torch.cuda.stream(self._bank_stream):
+                        for li in self.bank_slice(d):
+                            self.layers[li].refill(eps, mech, self.seeds[li], 0, path=path, device_base=True,
+                                                   parity=1 - parity, ahead=1, workspace=bank_workspace)
+                    ready = []
+                    if copies is not None:
+                        self._h2d_stream.wait_stream(main)
+                        with torch.cuda.stream(self._h2d_stream):
+                            ready = [copies[0](li) for li in range(len(self.layers))]
+                        self._d2h_stream.wait_stream(main)
+                    for li, (layer, x, seed) in enumerate(zip(self.layers, inputs, self.seeds)):
+                        if ready:
+                            main.wait_event(ready[li])
+                        t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
+                            if timer else None
+                        layer.online(x, eps, mech, seed, 0, d, path=path, device_base=True, parity=parity, timer=t)
+                        if copies is not None:
+                            self._d2h_stream.wait_stream(main)
+                            with torch.cuda.stream(self._d2h_stream):
+                                copies[1](li)
+                    main.wait_stream(self._bank_stream)
+                    if copies is not None:
+                        main.wait_stream(self._h2d_stream)
+                        main.wait_stream(self._d2h_stream)
+                    if d == D - 1:
+                        for layer in self.layers:
+                            for gi, g in enumerate(layer.groups):
+                                spl.spl_rng_advance(layer.rng_base[gi:gi + 1], D * (layer.M * g.K // 4))
+                graphs[parity].append(graph)
+                launches[parity].append(spl.spl_launch_count() - n0)
+        return graphs, launches
+
+    def refill_all(self, eps, mech, path="auto", parity=0, ahead=0, workspace=None):
+        """Every layer's bank for the cycle at the device-side bases (+ ``ahead`` cycles), into
+        correction buffers ``parity``, on the current stream."""
+        for layer, seed in zip(self.layers, self.seeds):
+            layer.refill(eps, mech, seed, 0, path=path, device_base=True, parity=parity, ahead=ahead,
+                         workspace=workspace)
 
     def start_overlapped(self, cycle, eps, mech, path="auto"):
         """Before replaying the overlapped graphs from bank cycle ``cycle``: the device-side Philox

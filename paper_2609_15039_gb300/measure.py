@@ -88,7 +88,8 @@ def _bound(stack, inputs, eps, mech, s, layers):
         outs = layer.online(x, eps, mech, seed, cycle, d)
         bc = layer.bound_check(x, outs, eps, mech, seed, cycle, d)
         res[f"layer{li}"] = {g: {"max_err_over_hard": v["max_err_over_hard"], "log_violation_pct": v["violation_pct"],
-                                 "mean_err": v["mean_err"], "mean_log_bound": v["mean_log_bound"]}
+                                 "mean_err": v["mean_err"], "mean_log_bound": v["mean_log_bound"],
+                                 "max_rel_err": v["max_err"] / v["max_abs_ref"] if v["max_abs_ref"] else 0.0}
                              for g, v in bc.items()}
     return res
 
@@ -440,5 +441,5 @@ def lm_head(tokens=(512, 1), eps=1.0, mech="gaussian", draws=8, cycles=3):
                         f"tokens {list(tokens)}", "lm_head": out, "peak_source": pk["source"]}
 
 
-WORKLOADS = {"llama_stack": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep, "down_fp64": down_fp64,
+WORKLOADS = {"llama_stack_detail": llama_stack, "qwen_stack": qwen_stack, "qwen_sweep": qwen_sweep, "down_fp64": down_fp64,
              "slalom": slalom_compare, "lm_head": lm_head}
