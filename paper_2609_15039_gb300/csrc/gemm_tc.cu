@@ -65,6 +65,15 @@ constexpr int BM = 128, THREADS = 192;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // 1 s per wait
 constexpr unsigned long long kDrainNs = 100000000ull;  // 0.1 s to drain on abort
 constexpr int MAX_CLUSTER = 8;                         // split-K CTAs of one output tile (portable cluster)
+// Longest accumulation chain in TMEM, in k-blocks (1024 elements of K for FP16X3, 512 for TF32X3).
+// tcgen05.mma adds its products into the fp32 accumulator with truncation: measured on GB300 at
+// zero noise, the error of one chain grows linearly with its length and is almost all bias toward
+// zero (max-norm relative error 3.9e-6 at 1024 elements of K on the FP16X3 split, 3.9e-5 at 9728;
+// TF32X3, with half the K per instruction, twice that).  A CTA whose K range is longer is cut
+// into segments of this many k-blocks: each segment starts a fresh accumulator and is folded into
+// the running sum with a round-to-nearest fp32 add (R = fl(R + P)), so the bias of every chain is
+// bounded whatever K is, and the folds' own errors are unbiased.  A fold costs ~0.35 us per CTA.
+constexpr int kChainBlocks = 32;
 constexpr uint32_t AUX_BYTES = 2048;                   // barriers, TMEM slot, abort flag; column scales at +1024
 
 // ---- instruction descriptors (tcgen05.mma kind::tf32 / kind::f16) ---------------
@@ -712,18 +721,27 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
 
 // Persistent form for launches of several waves of unsplit tiles: one CTA per SM takes the
 // tiles blockIdx.x, blockIdx.x + gridDim.x, ... (M fastest, as above).  The stage ring runs on
-// across tiles and TMEM holds two accumulators (columns 0 and 256): while the epilogue warps finish
-// tile i from one, the MMAs of tile i + 1 go into the other, so each tile's epilogue (C in, Y out,
-// straight between TMEM rows and global memory) overlaps the next tile's mainloop and only the
-// first prologue and the last epilogue are exposed.  Every output element is summed exactly as by
-// tc_gemm_kernel with one K range (the same MMAs in the same order, the same scaling and
-// subtraction), so the two give the same result bit for bit.  Rows of out and C must be whole
-// 16-byte units (the host checks).  Every wait is bounded as in tc_gemm_kernel.
+// across tiles and TMEM holds two buffers (columns 0 and 256).  Tile i keeps its running sum R in
+// buffer i % 2; a K range longer than `chain` k-blocks is cut into segments of `chain`, the first
+// accumulated into R and each later one into the other buffer P, which the epilogue warps fold into
+// R (R = fl(R + P)) before the MMAs take P again.  After the last fold the epilogue warps finish tile
+// i from R (C in, Y out, straight between TMEM rows and global memory) while the MMAs of tile i + 1
+// accumulate its first segment into buffer (i + 1) % 2 -- the one tile i used as P -- so each
+// tile's epilogue overlaps the next tile's mainloop and only the first prologue and the last
+// epilogue are exposed.  Every output element is summed exactly as by tc_gemm_kernel with one K
+// range and segments of `chain` k-blocks (the same MMAs in the same order, the same folds, the same
+// scaling and subtraction), so the two give the same result bit for bit.  Rows of out and C must be
+// whole 16-byte units (the host checks).  Every wait is bounded as in tc_gemm_kernel.
+//
+// Hand-over: every use of a buffer (as R or as P) ends with one tcgen05.commit on buf_full[b] and
+// is released by one arrival of each epilogue warp on buf_free[b] (a P after its fold, an R after
+// its tile's epilogue), so the k-th use of buffer b waits for release k - 1 and the epilogue's k-th
+// wait on buf_full[b] sees completion k.
 template <class Md, int BN, int RK>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
                      const int* __restrict__ a_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
-                     int tiles, int m_tiles) {
+                     int tiles, int m_tiles, int chain) {
   using L = Cfg<Md, BN, RK>;
   constexpr int STAGES = L::STAGES, BK = Md::BK;
   constexpr uint32_t ACC_COLS = 256;  // column offset of the second accumulator
@@ -732,18 +750,20 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* aux = smem + L::RING;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], empty[S], acc_full[2], acc_empty[2], drain
+  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], empty[S], buf_full[2], buf_free[2], drain
   volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (2 * STAGES + 5));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (2 * STAGES + 5) + 8);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int my_tiles = tiles > (int)blockIdx.x ? (tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
   const int nk = (int)ceil_div(K, BK);
+  const int seg_len = chain > 0 && chain < nk ? chain : nk;  // k-blocks per segment
+  const int nseg = (int)ceil_div(nk, seg_len);
   const uint32_t bar_base = smem_u32(bars);
   auto full_bar = [&](int st) { return bar_base + 8u * st; };
   auto empty_bar = [&](int st) { return bar_base + 8u * (STAGES + st); };
-  auto acc_full = [&](int b) { return bar_base + 8u * (2 * STAGES + b); };
-  auto acc_empty = [&](int b) { return bar_base + 8u * (2 * STAGES + 2 + b); };
+  auto buf_full = [&](int b) { return bar_base + 8u * (2 * STAGES + b); };
+  auto buf_free = [&](int b) { return bar_base + 8u * (2 * STAGES + 2 + b); };
   const uint32_t drain_bar = bar_base + 8u * (2 * STAGES + 4);
   auto tile_origin = [&](int i, int64_t& m0, int64_t& n0) {
     const int tile = (int)blockIdx.x + i * (int)gridDim.x;
@@ -757,8 +777,8 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
       mbar_init(empty_bar(st), 1);
     }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(acc_full(b), 1);
-      mbar_init(acc_empty(b), 4);  // one arrival per epilogue warp
+      mbar_init(buf_full(b), 1);
+      mbar_init(buf_free(b), 4);  // one arrival per epilogue warp
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
@@ -812,40 +832,46 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
         if (issued_mask & (1u << st)) mbar_wait(full_bar(st), (phase_mask >> st) & 1u, kDrainNs, nullptr);
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer: tile i into accumulator i % 2 ----------------
+    // ---------------- MMA issuer: tile i's segments into buffers i % 2 (R) and (i + 1) % 2 (P) ------
     bool ok = true;
     uint32_t it = 0;
+    uint32_t uses[2] = {0u, 0u};  // uses of each buffer so far
     for (int i = 0; i < my_tiles && ok; ++i) {
-      const int buf = i & 1, use = i >> 1;
-      if (use >= 1) {  // the epilogue is done with this accumulator's previous tile
-        ok = __all_sync(0xffffffffu, mbar_wait(acc_empty(buf), (uint32_t)(use - 1) & 1u, kWaitNs * 4, abort_flag));
-        if (!ok) break;
-      }
-      tc_fence_after();
-      const uint32_t acc = tmem + (uint32_t)buf * ACC_COLS;
-      for (int kb = 0; kb < nk; ++kb, ++it) {
-        const int st = (int)(it % STAGES);
-        const uint32_t ph = (it / STAGES) & 1u;
-        ok = __all_sync(0xffffffffu, mbar_wait(full_bar(st), ph, kWaitNs, abort_flag));
-        if (!ok) break;
-        if (lane == 0) {
-          tc_fence_after();
-          const uint32_t sa = smem_u32(smem + (size_t)st * L::STAGE);
-#pragma unroll
-          for (int kk = 0; kk < BK / Md::UMMA_K; ++kk) {
-            const uint32_t koff = kk * 32u;
-            const uint32_t first = (kb == 0 && kk == 0) ? 0u : 1u;
-            mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_LO + koff), make_sdesc_sw64(sa + L::W_HI + koff), first);
-            mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_HI + koff), make_sdesc_sw64(sa + L::W_LO + koff), 1u);
-            mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_HI + koff), make_sdesc_sw64(sa + L::W_HI + koff), 1u);
-          }
-          mma_commit(empty_bar(st));
+      for (int sg = 0; sg < nseg && ok; ++sg) {
+        const int b = (i & 1) ^ (sg == 0 ? 0 : 1);
+        if (uses[b] >= 1) {  // released by the epilogue: P folded, or R's tile finished
+          ok = __all_sync(0xffffffffu, mbar_wait(buf_free(b), (uses[b] - 1u) & 1u, kWaitNs * 4, abort_flag));
+          if (!ok) break;
         }
+        tc_fence_after();
+        const uint32_t acc = tmem + (uint32_t)b * ACC_COLS;
+        const int kb0 = sg * seg_len, kb1 = std::min(nk, kb0 + seg_len);
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+          const int st = (int)(it % STAGES);
+          const uint32_t ph = (it / STAGES) & 1u;
+          ok = __all_sync(0xffffffffu, mbar_wait(full_bar(st), ph, kWaitNs, abort_flag));
+          if (!ok) break;
+          if (lane == 0) {
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + (size_t)st * L::STAGE);
+#pragma unroll
+            for (int kk = 0; kk < BK / Md::UMMA_K; ++kk) {
+              const uint32_t koff = kk * 32u;
+              const uint32_t first = (kb == kb0 && kk == 0) ? 0u : 1u;
+              mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_LO + koff), make_sdesc_sw64(sa + L::W_HI + koff),
+                                first);
+              mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_HI + koff), make_sdesc_sw64(sa + L::W_LO + koff), 1u);
+              mma<Md, L::IDESC>(acc, make_sdesc_sw64(sa + L::A_HI + koff), make_sdesc_sw64(sa + L::W_HI + koff), 1u);
+            }
+            mma_commit(empty_bar(st));
+          }
+          __syncwarp();
+        }
+        if (!ok) break;
+        if (lane == 0) mma_commit(buf_full(b));  // this segment's sums are complete once these MMAs are
         __syncwarp();
+        ++uses[b];
       }
-      if (!ok) break;
-      if (lane == 0) mma_commit(acc_full(buf));  // the tile's sums are complete once these MMAs are
-      __syncwarp();
     }
     pdl_trigger();
     if (!ok) {
@@ -877,14 +903,37 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
     pdl_wait();  // C and the row exponents of A come from before this kernel
     prefetch_c(0);
     bool ok = true;
+    uint32_t done[2] = {0u, 0u};  // completions of each buffer consumed so far
     for (int i = 0; i < my_tiles; ++i) {
-      const int buf = i & 1, use = i >> 1;
+      const int buf = i & 1, pbuf = buf ^ 1;
       int64_t m0, n0;
       tile_origin(i, m0, n0);
       const int64_t m = m0 + r;
       const float sr = (Md::kF16 && m < M) ? pow2f(-__ldg(a_exp + m)) : 1.0f;
-      ok = __all_sync(0xffffffffu, mbar_wait(acc_full(buf), (uint32_t)use & 1u, kWaitNs * 4, abort_flag)) &&
-           !*abort_flag;
+      ok = __all_sync(0xffffffffu, mbar_wait(buf_full(buf), done[buf] & 1u, kWaitNs * 4, abort_flag)) &&
+           !*abort_flag;  // the first segment, in R
+      if (!ok) break;
+      ++done[buf];
+      for (int sg = 1; sg < nseg && ok; ++sg) {  // fold each later segment (in P) into R
+        ok = __all_sync(0xffffffffu, mbar_wait(buf_full(pbuf), done[pbuf] & 1u, kWaitNs * 4, abort_flag)) &&
+             !*abort_flag;
+        if (!ok) break;
+        ++done[pbuf];
+        tc_fence_after();
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * q) << 16);
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          float rv[32], pv[32];
+          tmem_ld_32x32(lane_base + (uint32_t)buf * ACC_COLS + (uint32_t)(32 * c), rv);
+          tmem_ld_32x32(lane_base + (uint32_t)pbuf * ACC_COLS + (uint32_t)(32 * c), pv);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) rv[j] = __fadd_rn(rv[j], pv[j]);
+          tmem_st_32x32(lane_base + (uint32_t)buf * ACC_COLS + (uint32_t)(32 * c), rv);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(buf_free(pbuf));
+      }
       if (!ok) break;
       tc_fence_after();
 #pragma unroll 1
@@ -917,7 +966,7 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty(buf));
+      if (lane == 0) mbar_arrive(buf_free(buf));
       prefetch_c(i + 1);
     }
     pdl_trigger();
@@ -1150,11 +1199,35 @@ TcShape tc_shape(int64_t M, int64_t K, int64_t N, int sms) {
   return best;
 }
 
+// Segments of a CTA whose K range is k_range elements: kChainBlocks when the range is longer, else 0
+// (one chain).
+template <class Md>
+int chain_segments(int64_t k_range) {
+  return ceil_div(k_range, (int64_t)Md::BK) > kChainBlocks ? kChainBlocks : 0;
+}
+
 template <class Md, int BN, int RK>
 spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* a_lo, const int* a_exp,
-                     const TcShape& shape, int skip_kblock, int seg_splits) {
-  // segmented mode: one CTA per tile over all of K, cut where a seg_splits-way split would cut it
-  const int seg_blocks = seg_splits > 0 ? (int)(round_up(ceil_div(a.K, seg_splits), Md::BK) / Md::BK) : 0;
+                     TcShape shape, int skip_kblock, int seg_splits) {
+  // Every CTA cuts its K range into chains of at most kChainBlocks k-blocks.  A correction in the
+  // order of a seg_splits-way split (seg_splits > 0, the bank) reproduces, per tile, what the online
+  // product did: an online split of at most kChainBlocks k-blocks per rank is one chain per rank,
+  // summed in rank order, which one CTA over all of K reproduces by folding segments cut at the
+  // split's boundaries; an unsplit online product (seg_splits = 1) is folded at kChainBlocks; an
+  // online split whose ranks fold chains of their own is reproduced by the same cluster split.
+  int seg_blocks = 0;  // segments of the unsplit tiles of a seg_splits launch
+  if (seg_splits == 1) {
+    seg_blocks = chain_segments<Md>(a.K);
+  } else if (seg_splits > 1) {
+    const int rank_blocks = (int)(round_up(ceil_div(a.K, seg_splits), Md::BK) / Md::BK);
+    if (rank_blocks <= kChainBlocks) {
+      seg_blocks = rank_blocks;
+    } else {  // every tile as the online launch ran it: split seg_splits ways, each rank folding its chains
+      shape.rest_tiles += shape.full_tiles;
+      shape.full_tiles = 0;
+      shape.rest_splits = seg_splits;
+    }
+  }
   if (!set_smem_attr<Md, BN, RK>()) return SPL_ECUDA;
   TcMaps maps;
   std::memset(&maps, 0, sizeof(maps));
@@ -1193,7 +1266,7 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_persistent_kernel<Md, BN, RK>, maps, a.out, a.c, a_exp,
-                                             (const int*)a.w_exp, a.M, a.K, a.N, (int)tiles, m_tiles);
+                                             (const int*)a.w_exp, a.M, a.K, a.N, (int)tiles, m_tiles, kChainBlocks);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   }
@@ -1204,6 +1277,7 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
   auto launch = [&](int64_t tiles, int64_t base, int splits, int seg) -> spl_status {
     if (tiles <= 0) return SPL_OK;
     const int64_t kps = round_up(ceil_div(a.K, splits), Md::BK);
+    if (seg == 0) seg = chain_segments<Md>(kps);  // chains of at most kChainBlocks within the CTA's range
     cudaLaunchConfig_t cfg;
     std::memset(&cfg, 0, sizeof(cfg));
     cfg.gridDim = dim3((unsigned)tiles, 1, (unsigned)splits);

@@ -344,8 +344,8 @@ def test_empty_reduction(spl):
                                          (128, 3072, 3072, "fp16x3"), (128, 8192, 3072, "fp16x3")])
 def test_matched_correction_cancels_rounding(spl, M, K, N, path):
     """A bank of 8 corrections summed in the online product's order: the same values up to
-    rounding, and on the tensor-core path a much smaller recovered error than a correction
-    computed with its own plan for 8 x M rows."""
+    rounding, every recovered output inside the hard bound, and a recovered error no larger than
+    with a correction computed with its own plan for 8 x M rows."""
     draws, b = 8, 1443.0
     W, Wt = _weights(spl, N, K, seed=K + N)
     X = wl.activations(M, K, seed=21).numpy()
@@ -368,13 +368,12 @@ def test_matched_correction_cancels_rounding(spl, M, K, N, path):
         S = linear.abs_products(X, Xt, eta[d * M:(d + 1) * M], W)
         assert np.all(err <= bounds.hard_bound(*S, K)), name
         errs[name] = float(err.mean())
-    if path != "fp32":
-        # the tensor-core bank at 8x the rows uses another K split and cluster order; matched, the
-        # errors of fl(x~ W^T) and fl(eta W^T) cancel
-        assert errs["matched"] * 3 < errs["plain"], errs
-    else:
-        # FMA chains in ascending k already keep the two roundings correlated; matching never hurts
-        assert errs["matched"] <= errs["plain"] * 1.1, errs
+    # Matching never hurts.  How much it helps depends on how far the plain plan's order is from the
+    # online one: FMA chains in ascending k already keep the two roundings correlated, and on the
+    # tensor cores the dominant error -- the truncation bias of each accumulation chain -- is the same
+    # in both wherever their chains are cut at the same K boundaries (every chain of an unsplit tile
+    # starts at a multiple of 32 k-blocks), so only the round-to-nearest folds differ.
+    assert errs["matched"] <= errs["plain"] * 1.1, errs
 
 
 @pytest.mark.parametrize("M,K,N,path", [(128, 3072, 3072, "fp16x3"), (128, 3072, 5120, "fp16x3"),
@@ -429,11 +428,13 @@ def test_tc_unsplit_epilogue_on_ragged_rows(spl, tile_n, ring_kb, N):
 
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 @pytest.mark.parametrize("tile_n,ring_kb", [v for v in TC_VARIANTS if v != (128, 96)])
-def test_tc_persistent_equals_unsplit_product(spl, path, tile_n, ring_kb):
-    """The persistent kernel (one CTA per SM looping over tiles, two TMEM accumulators, the epilogue
-    of one tile beside the mainloop of the next) gives the unsplit product bit for bit, with and
-    without C, on a problem of 2 to 4 tiles per CTA with ragged M, N and K."""
-    M, K, N = 2600, 264, 4000
+@pytest.mark.parametrize("K", [264, 3080])
+def test_tc_persistent_equals_unsplit_product(spl, path, tile_n, ring_kb, K):
+    """The persistent kernel (one CTA per SM looping over tiles, two TMEM buffers, the epilogue of
+    one tile beside the mainloop of the next) gives the unsplit product bit for bit, with and
+    without C, on a problem of 2 to 4 tiles per CTA with ragged M, N and K -- at K = 3080 with every
+    tile's K range cut into accumulation chains that are folded in TMEM (4 for FP16X3, 7 for TF32X3)."""
+    M, N = 2600, 4000
     W, Wt = _weights(spl, N, K, seed=61)
     A = wl.activations(M, K, seed=62).numpy()
     C = dev(wl.activations(M, N, seed=63).numpy())
@@ -475,23 +476,27 @@ def test_library_picks_persistent_for_many_waves(spl):
 
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 @pytest.mark.parametrize("tile_n,ring_kb", TC_VARIANTS)
-def test_tc_segmented_equals_split_product(spl, path, tile_n, ring_kb):
-    """Every kernel instance in segmented mode (one CTA over all of K, the partial sums of a 3-way
-    split of K folded in TMEM in order) gives the 3-way cluster-split product bit for bit, alone
-    and with the tiles after the first half+1 split over a cluster; ragged M, N and K."""
-    M, K, N = 300, 2056, 700
+@pytest.mark.parametrize("K,s", [(2056, 3), (3080, 2), (3080, 1)])
+def test_tc_segmented_equals_split_product(spl, path, tile_n, ring_kb, K, s):
+    """Every kernel instance in the bank's form (seg_splits = s) gives the online product of the
+    same K-split bit for bit, alone and with the tiles after the first half+1 split over a cluster;
+    ragged M, N and K.  Where a rank's K range is one accumulation chain (2056 / 3 on FP16X3) one CTA
+    over all of K folds the ranks' partial sums in TMEM in rank order; where the ranks fold chains of
+    their own (3080 / 2, and 2056 / 3 on TF32X3) the tiles run as the same cluster split; an unsplit
+    product (s = 1) is folded at the same chain boundaries."""
+    M, N = 300, 700
     W, Wt = _weights(spl, N, K, seed=47)
     A = (wl.activations(M, K, seed=48).numpy() * 30).astype(np.float32)
     C = dev(wl.activations(M, N, seed=49).numpy())
     tiles = -(-M // 128) * -(-N // tile_n)
     ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, path))
     ref = torch.empty((M, N), device="cuda")
-    spl.spl_test_tc_product(ref, dev(A), Wt, C, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=3, workspace=ws)
-    assert_product_close(f32(ref), A, W, path, C=C.cpu().numpy(), what=f"{path} tile {tile_n} split 3")
-    for full, splits in ((0, 1), (tiles // 2 + 1, 3), (tiles, 1)):
+    spl.spl_test_tc_product(ref, dev(A), Wt, C, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=s, workspace=ws)
+    assert_product_close(f32(ref), A, W, path, C=C.cpu().numpy(), what=f"{path} tile {tile_n} split {s}")
+    for full, splits in ((0, 1), (tiles // 2 + 1, s), (tiles, 1)):
         Y = torch.full((M, N), float("nan"), device="cuda")
         spl.spl_test_tc_product(Y, dev(A), Wt, C, path=path, tile_n=tile_n, ring_kb=ring_kb, splits=splits,
-                                full_tiles=full, seg_splits=3, workspace=ws)
+                                full_tiles=full, seg_splits=s, workspace=ws)
         assert torch.equal(Y, ref), (full, splits, float((Y - ref).abs().max()))
     assert spl.spl_get_device_status() == 0
 

@@ -9,15 +9,15 @@ downgraded one.  With a = a_hi + a_lo (11 + 11 significant bits), dropping a cro
 leaves a per-term error uniform in +-2^-12 |a w|, whose sum over K terms has a standard deviation of
 2^-12/sqrt(3) tau = 296 x 2^-21 tau, tau = sqrt(sum_k (a_k w_k)^2) the root sum of squares of the
 terms; with random-signed terms |Y*| is of order tau too, so that is ~1.4e-4 relative -- fourteen times
-the tolerance -- and dropping all of a_lo is worse still.  A correct three-product split leaves
-~0.2 x 2^-21 tau per output, and fp32 accumulation (at most one rounding per product term) adds
-2^-24 tau sqrt(K/6) in standard deviation.  So the per-element check below,
+the tolerance -- and dropping all of a_lo is worse still.
 
-    mean over outputs of |Y - Y*| / (2^-21 tau)  <=  1 + sqrt(K) / 8,
-
-holds for the split at any K used here (at most 13.3 at K = 9728) and fails by more than 15x for a
-split that lost a cross product (mean ~236).  The same holds for the TF32X3 split (lo truncated to
-TF32: ~0.4 x 2^-21 tau) and for the FP32 FMA path (sequential accumulation only).
+The per-element check below is mean |Y - Y*| / (2^-21 tau) <= 16.  A correct three-product split
+contributes ~0.2; what dominates is the tensor core's accumulation, which truncates: on GB300 one
+unbroken chain of FP16X3 MMAs leaves a bias toward zero of 0.0059 per element of K in these units
+(TF32X3: 0.0117), which is why the kernels cut every chain at 1024 (FP16X3) or 512 (TF32X3) elements
+of K and fold the pieces with round-to-nearest adds -- at most ~6 whatever K is.  The FP32 FMA path
+(sequential round-to-nearest) stays near 0.5.  A split that lost a cross product reads ~236, fifteen
+times the limit.
 
 Launch forms covered: every tile width / ring of the tensor-core kernel, cluster K-splits 1..8, the
 two-launch shape (whole waves unsplit + the rest split), the persistent kernel, the segmented (bank)
@@ -41,8 +41,7 @@ TC_VARIANTS = [(256, 192), (128, 224), (128, 96), (160, 224), (192, 224), (224, 
 FULL_K = [2560, 3072, 8192, 9728]
 
 
-def stat_limit(K):
-    return 1.0 + np.sqrt(K) / 8.0
+STAT_LIMIT = 16.0
 
 
 @pytest.fixture(scope="module")
@@ -70,7 +69,7 @@ def zero_noise_errors(Y, A, W):
 def check(Y, A, W, K, what):
     rel, stat = zero_noise_errors(Y, A, W)
     assert rel <= REL_TOL, f"{what}: max-norm relative error {rel:.3g} > {REL_TOL}"
-    assert stat <= stat_limit(K), f"{what}: mean err / (2^-21 tau) = {stat:.3g} > {stat_limit(K):.3g}"
+    assert stat <= STAT_LIMIT, f"{what}: mean err / (2^-21 tau) = {stat:.3g} > {STAT_LIMIT}"
     return rel, stat
 
 
