@@ -460,6 +460,19 @@ spl_status spl_test_tc_product(float* Y, const float* Xt, const spl_weight* W, c
                                int64_t full_tiles, int seg_splits, int persistent, void* workspace,
                                size_t workspace_bytes, cudaStream_t stream);
 
+/* Test hook: the FP16X3 product on the swapped kernel the library takes for
+ * products of 9 to 64 rows (the weight in the MMA's 128 rows, the tokens in
+ * its N columns), forced to a token-tile width `tile_tokens` (16, 32, 64 or
+ * 128) and a K-split `splits` (1-8, a thread-block cluster summed in rank
+ * order) for any M.  Y[M, N] = fl32(Xt W^T - C) (C may be NULL), W with its
+ * fp16 split, workspace as spl_linear_workspace_bytes(M, K, N, FP16X3).
+ * Errors: EINVAL for a width not listed or NULL operands, ESHAPE for splits
+ * outside 1-8, EALIGN for K % 8 != 0 or unaligned pointers, as
+ * spl_masked_linear otherwise.  The paper has no counterpart. */
+spl_status spl_test_tc_swap_product(float* Y, const float* Xt, const spl_weight* W, const float* C, int64_t M,
+                                    int64_t K, int64_t N, int tile_tokens, int splits, void* workspace,
+                                    size_t workspace_bytes, cudaStream_t stream);
+
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last
  * call gave up a bounded wait (and clears the flag), else SPL_ECUDA if the

@@ -154,11 +154,12 @@ spl_status run_gemv_masked(const LinearArgs& a, const Plan& p, const MaskNoise& 
 // Argument check shared by the noise entries.
 spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech);
 int64_t gemv_max_ks(int64_t M);                           // largest K-slice the decode kernel stages for M rows
-// Launch variant and K-split of a one-launch tcgen05 call (false if the call makes two launches).
-bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, int* variant, int* splits);
-// One unsplit tcgen05 launch whose every output is summed in the order of a `splits`-way K-split
-// (partials of the K ranges added in rank order): the correction bank in the masked product's order.
-spl_status run_tc_segmented(const LinearArgs& a, int splits);
+// Launch variant and K-split of a one-launch tcgen05 call (false if the call makes two launches);
+// variant -1 is the swapped kernel of few rows.
+bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, spl_path path, int* variant, int* splits);
+// A tcgen05 product whose every output is summed in the order the masked product of `order_rows`
+// rows uses (the correction bank): the same K ranges, accumulation chains and cluster order.
+spl_status run_tc_matched(const LinearArgs& a, int64_t order_rows);
 size_t tc_asplit_bytes(int64_t M, int64_t K, spl_path path);  // FP16X3 split of A in the workspace (0 for TF32X3)
 spl_status run_simt(const LinearArgs& a, const Plan& p);
 spl_status run_tc(const LinearArgs& a, const Plan& p);

@@ -124,7 +124,7 @@ MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, sp
   mp.kernel = online.kernel;
   if (online.kernel == kKernelTc) {
     int variant = 0;  // the bank runs its own launch shape; only the K-split order carries over
-    if (!tc_uniform_shape(order_rows, K, N, &variant, &mp.splits)) return mp;
+    if (!tc_uniform_shape(order_rows, K, N, resolved, &variant, &mp.splits)) return mp;
     mp.ws = kCounterBytes + tc_asplit_bytes(M, K, resolved);
     mp.ok = true;
     return mp;
@@ -276,7 +276,7 @@ spl_status precompute_matched(float* C, const float* Nz, const spl_weight* A, co
     args.a_l16 = A->f16_lo;
     args.a_exp = A->f16_exp;
   }
-  if (mp.kernel == kKernelTc) return run_tc_segmented(args, mp.splits);
+  if (mp.kernel == kKernelTc) return run_tc_matched(args, order_rows);
   Plan p{};
   p.kernel = mp.kernel;
   p.splits = mp.splits;

@@ -88,6 +88,7 @@ _SIGS = {
     "spl_test_tc_capacity": (_I, [_I64, _I64, _I64, ctypes.POINTER(ctypes.c_int64)]),
     "spl_test_tc_shape": (_I, [_I64, _I64, _I64, _I64, ctypes.POINTER(ctypes.c_int64)]),
     "spl_test_tc_product": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _I, _I, _I, _I64, _I, _I, _P, _SZ, _P]),
+    "spl_test_tc_swap_product": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _I, _P, _SZ, _P]),
     "spl_get_device_status": (_I, [_P]),
     "spl_launch_count": (ctypes.c_uint64, []),
     "spl_status_string": (ctypes.c_char_p, [_I]),
@@ -608,6 +609,22 @@ def spl_test_tc_product(Y, Xt, W, C=None, path="fp16x3", tile_n=256, ring_kb=192
                                      _path(path), int(tile_n), int(ring_kb), int(splits), int(full_tiles),
                                      int(seg_splits), int(bool(persistent)), wsp, wsb, _stream(stream)),
            "spl_test_tc_product")
+
+
+def spl_test_tc_swap_product(Y, Xt, W, C=None, tile_tokens=16, splits=1, workspace=None, stream=None):
+    """The FP16X3 product on the swapped kernel with a fixed token-tile width and K-split (a test hook)."""
+    W = _weight(W)
+    M, K = _rows_cols(Xt)
+    N = W.shape[0]
+    if W.shape[-1] != K or Y.numel() != M * N or (C is not None and C.numel() != M * N):
+        raise ValueError("spl_test_tc_swap_product: shape mismatch")
+    if workspace is None:
+        workspace = globals()["workspace"](spl_linear_workspace_bytes(M, K, N, "fp16x3"), Xt.device)
+    wsp, wsb = _ws(workspace)
+    ws_ = W.c_struct()
+    _check(lib().spl_test_tc_swap_product(_dev(Y, "Y"), _dev(Xt, "Xt"), ctypes.byref(ws_), _dev(C, "C"), M, K, N,
+                                          int(tile_tokens), int(splits), wsp, wsb, _stream(stream)),
+           "spl_test_tc_swap_product")
 
 
 def spl_launch_count():

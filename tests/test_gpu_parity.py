@@ -260,6 +260,55 @@ def test_tc_every_launch_shape(spl, path, tile_n, ring_kb, splits):
     assert spl.spl_get_device_status() == 0
 
 
+SWAP_WIDTHS = [16, 32, 64, 128]
+
+
+@pytest.mark.parametrize("M", [9, 16, 33, 64])
+@pytest.mark.parametrize("splits", [1, 3, 8])
+def test_swap_every_width_and_split(spl, M, splits):
+    """The swapped kernel (weight rows in the MMA's 128 rows, tokens in its N) at every token-tile
+    width and cluster K-split, ragged M, K and N (tokens past M are the copy's zero rows): within the
+    product tolerance of the oracle, with and without C, and the same bits at every width -- an
+    output's sum does not depend on the other columns of its MMA, which the bank relies on."""
+    K, N = 1032, 600
+    W, Wt = _weights(spl, N, K, seed=81)
+    A = (wl.activations(M, K, seed=82 + M).numpy() * 300).astype(np.float32)
+    C = wl.activations(M, N, seed=83).numpy()
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp16x3"))
+    first = None
+    for tn in SWAP_WIDTHS:
+        Y = torch.full((M, N), float("nan"), device="cuda")
+        spl.spl_test_tc_swap_product(Y, dev(A), Wt, dev(C), tile_tokens=tn, splits=splits, workspace=ws)
+        assert_product_close(f32(Y), A, W, "fp16x3", C=C, what=f"swap {tn} split {splits}")
+        if first is None:
+            first = Y
+        assert torch.equal(Y, first), (tn, float((Y - first).abs().max()))
+    Y2 = torch.full((M, N), float("nan"), device="cuda")
+    spl.spl_test_tc_swap_product(Y2, dev(A), Wt, None, tile_tokens=16 if M <= 16 else 64, splits=splits, workspace=ws)
+    assert_product_close(f32(Y2), A, W, "fp16x3", what="swap without C")
+    assert spl.spl_get_device_status() == 0
+
+
+def test_library_takes_the_swapped_kernel_for_few_rows(spl):
+    """AUTO runs 9-32 rows on the swapped kernel: the library's product equals the swapped kernel's
+    bit for bit (at the width of the rows and the split the library picks)."""
+    K, N = 3072, 5120
+    W, Wt = _weights(spl, N, K, seed=91)
+    for M in (9, 16, 25, 32):
+        A = wl.activations(M, K, seed=92 + M).numpy()
+        ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N))
+        Y = torch.empty((M, N), device="cuda")
+        spl.spl_masked_linear(Y, dev(A), Wt, workspace=ws)
+        tn = next(t for t in SWAP_WIDTHS if M <= t)
+        hits = 0
+        for splits in range(1, 9):
+            Ys = torch.empty((M, N), device="cuda")
+            spl.spl_test_tc_swap_product(Ys, dev(A), Wt, None, tile_tokens=tn, splits=splits, workspace=ws)
+            hits += int(torch.equal(Y, Ys))
+        assert hits >= 1, M  # some split of the swapped kernel is exactly what the library ran
+    assert spl.spl_get_device_status() == 0
+
+
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 def test_products_with_extreme_row_scales(spl, path):
     """Rows of A and W spread over 60 orders of magnitude, zero rows included: the power-of-two
@@ -381,7 +430,9 @@ def test_matched_correction_cancels_rounding(spl, M, K, N, path):
                                          (128, 3072, 3072, "tf32x3"), (100, 1032, 600, "fp16x3"),
                                          (128, 3072, 3072, "fp32"), (1, 3072, 3072, "fp32"), (512, 3072, 3072, "fp16x3"),
                                          (1, 3072, 5120, "fp32"), (1, 3072, 16384, "fp32"), (1, 8192, 3072, "fp32"),
-                                         (4, 3072, 5120, "fp32"), (3, 1028, 600, "fp32")])
+                                         (4, 3072, 5120, "fp32"), (3, 1028, 600, "fp32"),
+                                         (16, 3072, 5120, "fp16x3"), (16, 9728, 2560, "fp16x3"),
+                                         (32, 2560, 19456, "fp16x3"), (12, 1032, 600, "fp16x3")])
 @pytest.mark.parametrize("draws", [4, 8])
 def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path, draws):
     """The bank's correction of draw d is, bit for bit, what the online product computes when

@@ -108,6 +108,18 @@ def test_every_tc_launch_form_at_full_k(spl, problems, K, path, tile_n, ring_kb)
 
 
 @pytest.mark.parametrize("K", FULL_K)
+@pytest.mark.parametrize("tn", [16, 64, 128])
+@pytest.mark.parametrize("splits", [1, 3, 8])
+def test_swap_forms_at_full_k(spl, problems, K, tn, splits):
+    """The swapped kernel of few rows (weight in the MMA's rows, tokens in its columns) at 40 tokens."""
+    A, W, Wt = problems[K]
+    A = np.ascontiguousarray(A[:40])
+    Y = torch.full((40, W.shape[0]), float("nan"), device="cuda")
+    spl.spl_test_tc_swap_product(Y, dev(A), Wt, None, tile_tokens=tn, splits=splits)
+    check(f32(Y), A, W, K, f"swap {tn} split {splits}")
+
+
+@pytest.mark.parametrize("K", FULL_K)
 @pytest.mark.parametrize("M", [1, 4, 16, 200])
 def test_fp32_paths_at_full_k(spl, problems, K, M):
     """The FP32 paths: the streaming decode kernel (M <= 16) and the FMA kernel (M = 200)."""
@@ -123,7 +135,7 @@ def test_fp32_paths_at_full_k(spl, problems, K, M):
     check(f32(Y2), A, W, K, f"fp32 masked_linear M={M}")
 
 
-@pytest.mark.parametrize("M", [1, 4, 16, 130])
+@pytest.mark.parametrize("M", [1, 4, 16, 64, 130])
 @pytest.mark.parametrize("K", FULL_K)
 def test_noise_free_call_chain(spl, problems, K, M):
     """eps = inf through the boundary's call chain: spl_noise_mask (zero noise, x~ = x bit for bit),
