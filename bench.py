@@ -28,6 +28,7 @@ CPU oracle on a bounded sample of the same workload instead.
 """
 
 import argparse
+import faulthandler
 import json
 import os
 import statistics
@@ -70,7 +71,11 @@ def parse(argv=None):
     ap.add_argument("--no-decode", action="store_true", help="stack: skip the one-token decode measurement")
     ap.add_argument("--decode-steps", type=int, default=256)
     ap.add_argument("--no-overlap", action="store_true",
-                    help="compute each bank cycle's corrections before its steps instead of during the previous cycle")
+                    help="llama_layer: compute each bank cycle's corrections before its steps instead of during the "
+                         "previous cycle")
+    ap.add_argument("--schedule", choices=["stacked", "banked"], default="stacked",
+                    help="stack workload: stacked (each product also computes the next cycle's correction of its "
+                         "draw) or banked (the next cycle's banks of 1/8 of the layers beside each step)")
     ap.add_argument("--stored-noise", action="store_true",
                     help="llama_layer: keep the bank's fp32 noise and mask each step with it instead of drawing it "
                          "again")
@@ -317,6 +322,7 @@ def run_workload(args):
 
 
 def main():
+    faulthandler.enable()  # a crash in native code prints the Python stack to stderr
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
@@ -671,6 +677,12 @@ def run_llama_layer(args):
         dist.destroy_process_group()
 
 
+def phase(msg):
+    """Progress of the run on stderr (the JSON line goes to stdout)."""
+    sys.stderr.write(f"[bench {time.strftime('%H:%M:%S')}] {msg}\n")
+    sys.stderr.flush()
+
+
 def path_peaks(pk):
     """Algorithmic flops per second at each path's instruction peak: FP16X3 = the measured
     sustained bf16 rate (fp16 runs at the bf16 rate) / 3 products per term; TF32X3 = that x the
@@ -712,49 +724,63 @@ def run_llama_stack(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     model, L, M, D, mech, eps, path = wl.LLAMA_3_2_3B, args.layers, args.tokens, DRAWS, args.mech, args.eps, args.path
+    stacked = args.schedule == "stacked"
     pk = peaks()
     ppk = path_peaks(pk)
     t_build = time.perf_counter()
-    stack = MaskedStack.build(model, L, M, D, base_seed=STACK_SEED, device=dev, path=path)
+    phase("building the stack")
+    stack = MaskedStack.build(model, L, M, D, base_seed=STACK_SEED, device=dev, path=path, stacked=stacked)
     inputs = stack.inputs(STACK_INPUT_SEED, device=dev)
+    layer0 = stack.layers[0]
+    groups = layer0.groups
     if path == "auto":
         # a8 is evaluated per (shape, eps): on layer 0's weights and a masked sample of its input, and
         # the choice kept for every layer of the same shapes
-        l0 = stack.layers[0]
-        l0.calibrate(inputs[0], eps, mech, stack.seeds[0])
+        layer0.calibrate(inputs[0], eps, mech, stack.seeds[0])
         for layer in stack.layers[1:]:
-            layer.paths = dict(l0.paths)
-    layer0 = stack.layers[0]
-    groups = layer0.groups
-    group_paths = {g.name: spl.PATH_NAMES[spl.spl_resolve_path(M, g.K, g.N, layer0.path_of(g, path, M))]
-                   for g in groups}
-    bank_ws = spl.workspace(max(l.workspace_bytes(M, D, path) for l in stack.layers), dev)
+            layer.paths = dict(layer0.paths)
+        if stacked:  # the buffers follow the chosen paths
+            for layer in stack.layers:
+                layer.allocate_stacked(M, D, path, workspace=layer.workspace)
+    rows = 2 * M if stacked else M  # rows of every product call
+    if stacked:
+        group_paths = {g.name: layer0.stacked[g.name]["path"] for g in groups}
+    else:
+        group_paths = {g.name: spl.PATH_NAMES[spl.spl_resolve_path(M, g.K, g.N, layer0.path_of(g, path, M))]
+                       for g in groups}
+    bank_ws = None if stacked else spl.workspace(max(l.workspace_bytes(M, D, path) for l in stack.layers), dev)
     stream = torch.cuda.current_stream(dev)
-    stack.step(inputs, eps, mech, 0, path=path)  # sets up every library call before capture
+    for li, layer in enumerate(stack.layers):  # sets up every library call before capture
+        if stacked:
+            layer.stacked_step(inputs[li], eps, mech, stack.seeds[li], 0, 0, path=path)
+        else:
+            layer.refill(eps, mech, stack.seeds[li], 0, path=path)
+            layer.online(inputs[li], eps, mech, stack.seeds[li], 0, 0, path=path)
     torch.cuda.synchronize()
     build_s = time.perf_counter() - t_build
 
-    flops_layer = {g.name: 2 * M * g.K * g.N for g in groups}
+    flops_layer = {g.name: 2 * M * g.K * g.N for g in groups}  # the masked product (online rows)
     flops_step = L * sum(flops_layer.values())  # the masked products of one prefill (algorithmic)
 
-    # ---- the timed steps: prefill + 1/D of the next cycle's banks per graph ----------------------
-    overlap = not args.no_overlap
-    if overlap:
-        graphs, glaunch = stack.capture_steps(inputs, eps, mech, bank_ws, path=path)
-        graph_of = lambda s: graphs[(s // D) % 2][s % D]
-        launches_of = lambda s: glaunch[(s // D) % 2][s % D]
+    # ---- the timed steps -----------------------------------------------------------------------
+    phase("capturing the step graphs")
+    if stacked:
+        graphs, glaunch = stack.capture_stacked(inputs, eps, mech, path=path)
     else:
-        graphs, glaunch = stack.capture(inputs, eps, mech, path=path)
-        graph_of = lambda s: graphs[s % D]
-        launches_of = lambda s: glaunch[s % D]
+        graphs, glaunch = stack.capture_steps(inputs, eps, mech, bank_ws, path=path)
+    graph_of = lambda s: graphs[(s // D) % 2][s % D]
+    launches_of = lambda s: glaunch[(s // D) % 2][s % D]
 
     def prime(cycle):
-        """Device-side Philox bases at ``cycle`` and, for the overlapped graphs, that cycle's banks."""
-        stack.set_cycle(cycle)
-        if overlap:
+        """Device-side Philox bases at ``cycle`` and that cycle's corrections in place."""
+        if stacked:
+            stack.start_stacked(cycle, graphs)
+        else:
+            stack.set_cycle(cycle)
             stack.refill_all(eps, mech, path, parity=cycle % 2, workspace=bank_ws)
 
-    s = D  # every pass starts at a bank cycle
+    s = 2 * D  # every pass starts at a bank cycle
+    phase("timed steps")
     prime(s // D)
     for _ in range(args.warmup):
         graph_of(s).replay()
@@ -783,74 +809,73 @@ def run_llama_stack(args):
         raise RuntimeError("device status " + spl.status_string(st))
     value = job_rate(world, flops_step, ms) / 1e12
 
-    # ---- the online prefill alone, and its product calls (event pairs around each) ---------------
-    on_graphs, on_launch = stack.capture(inputs, eps, mech, path=path, refill=False)
-    stack.set_cycle(1)
-    _time_graphs(lambda i: on_graphs[i % D], 0, D, stream)  # warm-up cycle
-    on_times = _time_graphs(lambda i: on_graphs[i % D], 0, 2 * D, stream)
-    ms_online = sum(on_times) / len(on_times)
-    del on_graphs
+    # ---- the product calls alone: CUDA event pairs around each, in graphs of the same steps ------
     ev = {}
+    ev_alive = []  # every event recorded into a graph lives as long as the graph (a graph of both parities
+                   # records its own events; the dict keeps the last captured ones)
 
-    def timer(d, li, phase, kind, group):
+    def timer(d, li, phase_, kind, group):
         if kind != "masked_linear_unmask":
             return
         e = torch.cuda.Event(enable_timing=True, external=True)
         e.record()
-        ev.setdefault((d, li, group), [None, None])[0 if phase == "begin" else 1] = e
+        ev_alive.append(e)
+        ev.setdefault((d, li, group), [None, None])[0 if phase_ == "begin" else 1] = e
 
-    ev_graphs, _ = stack.capture(inputs, eps, mech, path=path, refill=False, timer=timer)
-    stack.set_cycle(1)
-    _time_graphs(lambda i: ev_graphs[i % D], 0, D, stream)  # each graph's events hold its last replay
+    phase("per-call timing pass")
+    if stacked:
+        ev_graphs, _ = stack.capture_stacked(inputs, eps, mech, path=path, timer=timer)
+        c = -(-s // D) + 1
+        stack.start_stacked(c, ev_graphs)
+        for d in range(D):  # one cycle: each graph's events hold its last replay
+            ev_graphs[c % 2][d].replay()
+        torch.cuda.synchronize()
+        s = (c + 1) * D
+    else:
+        ev_graphs, _ = stack.capture(inputs, eps, mech, path=path, refill=False, timer=timer)
+        stack.set_cycle(1)
+        _time_graphs(lambda i: ev_graphs[i % D], 0, D, stream)
     per_group = {}
     for (d, li, gname), (b, e) in ev.items():
         per_group.setdefault(gname, []).append(b.elapsed_time(e))
     del ev_graphs
+    del ev_alive
     prod = {}
     for g in groups:
         t = per_group[g.name]
         avg = sum(t) / len(t)
-        prod[g.name] = {"calls": len(t), "avg_us": 1e3 * avg, "tflops": flops_layer[g.name] / (avg * 1e-3) / 1e12,
-                        "path": group_paths[g.name], "peak": ppk[group_paths[g.name]],
-                        "frac": flops_layer[g.name] / (avg * 1e-3) / 1e12 / ppk[group_paths[g.name]]}
+        f = 2 * rows * g.K * g.N
+        pp = ppk[group_paths[g.name]]
+        prod[g.name] = {"calls": len(t), "rows": rows, "avg_us": 1e3 * avg, "tflops": f / (avg * 1e-3) / 1e12,
+                        "path": group_paths[g.name], "peak": pp, "frac": f / (avg * 1e-3) / 1e12 / pp}
     prod_ms_layer = sum(p["avg_us"] for p in prod.values()) / 1e3
-    prod_flops_layer = sum(flops_layer.values())
-    prod_peak = prod_flops_layer / sum(flops_layer[n] / ppk[group_paths[n]] for n in flops_layer)
-    achieved = prod_flops_layer / (prod_ms_layer * 1e-3) / 1e12
-    traffic, traffic_note = profiled_traffic("tc_prefill_fp16x3_llama_512.md", "traffic_bytes_per_launch")
+    call_flops_layer = sum(2 * rows * g.K * g.N for g in groups)
+    prod_peak = call_flops_layer / sum(2 * rows * g.K * g.N / ppk[group_paths[g.name]] for g in groups)
+    achieved = call_flops_layer / (prod_ms_layer * 1e-3) / 1e12
+    traffic, traffic_note = (profiled_traffic("tc_stacked_fp16x3_llama_1024.md", "traffic_bytes_per_launch")
+                             if stacked else
+                             profiled_traffic("tc_prefill_fp16x3_llama_512.md", "traffic_bytes_per_launch"))
+    what = (f"one call per input group and layer: the {M} masked rows of the step and, in the same launch, the "
+            f"{M} noise rows of the next cycle's draw (their corrections), {rows} rows" if stacked else
+            f"one call per input group and layer, {M} rows")
     roofline = {
         "bound": "tensor", "achieved": achieved, "peak": prod_peak, "unit": "TFLOP/s", "frac": achieved / prod_peak,
         "traffic": traffic,
-        "kernel": (f"masked products with fused unmask at {M} rows (tc_persistent_kernel / tc_gemm_kernel, FP16X3 "
-                   f"on tcgen05): one call per input group, {len(groups)} per layer, {len(groups) * L} per prefill"),
-        "flops_per_launch": prod_flops_layer / len(groups), "avg_launch_us": 1e3 * prod_ms_layer / len(groups),
-        "per_group": prod, "share_of_online_prefill": L * prod_ms_layer / ms_online,
+        "kernel": ("tc_persistent_kernel / tc_gemm_kernel (FP16X3 on tcgen05) with the fused unmask: " + what +
+                   f"; {len(groups) * L} calls per step"),
+        "flops_per_launch": call_flops_layer / len(groups), "avg_launch_us": 1e3 * prod_ms_layer / len(groups),
+        "per_group": prod, "share_of_step": L * prod_ms_layer / ms,
         "timing": ("CUDA event pairs (external event nodes, on the launching stream) around every product call of "
-                   f"the 28 layers in graph-replayed online prefills (one bank cycle, {D} prefills); achieved = the "
-                   "calls' algorithmic flops / their summed durations"),
+                   f"the {L} layers in graph-replayed steps (one bank cycle, {D} steps); achieved = the calls' "
+                   "algorithmic flops (2 x rows x K x N) / their summed durations"),
         "traffic_note": traffic_note + "; DRAM bytes per call, averaged over the four calls of a layer",
-        "peak_source": pk["source"], "peak_note": "sustained peak (the calls run inside 8 ms prefills); " + PEAK_NOTE}
-
-    # ---- the bank refill alone: every layer's next cycle (D draws of M rows per group) ----------
-    bank_graph = torch.cuda.CUDAGraph()
-    n0 = spl.spl_launch_count()
-    with torch.cuda.graph(bank_graph):
-        stack.refill_all(eps, mech, path, parity=0, workspace=bank_ws)
-    bank_launches = spl.spl_launch_count() - n0
-    bank_times = _time_graphs(lambda i: bank_graph, 0, 3, stream)[1:]
-    bank_ms = sum(bank_times) / len(bank_times)
-    del bank_graph
-    bank_flops = D * flops_step
-    bank_peak = prod_peak
-    bank = {"ms_per_cycle": bank_ms, "ms_per_prefill": bank_ms / D, "tflops": bank_flops / (bank_ms * 1e-3) / 1e12,
-            "peak": bank_peak, "frac": bank_flops / (bank_ms * 1e-3) / 1e12 / bank_peak, "launches": bank_launches,
-            "what": (f"{D} noise draws per input group and layer (split as drawn) and their corrections as one "
-                     f"product of {D * M} rows per group, summed in the online product's order")}
+        "peak_source": pk["source"], "peak_note": "sustained peak (the calls run inside steps of ~13 ms); " + PEAK_NOTE}
 
     # ---- end to end: the same steps with every layer's input copied in from pinned host memory
     # and every output copied back, inside each step's graph, on two copy streams ----------------
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and stacked:
+        phase("end-to-end pass")
         host_in = [{g: x.cpu().pin_memory() for g, x in inp.items()} for inp in inputs]
         host_out = [{g.name: torch.empty((M, g.N)).pin_memory() for g in layer.groups} for layer in stack.layers]
         h2d = sum(x.numel() * 4 for inp in host_in for x in inp.values())
@@ -863,18 +888,14 @@ def run_llama_stack(args):
             e.record()
             return e
 
-        def copy_out(li):
-            layer = stack.layers[li]
-            for g in layer.groups:
-                host_out[li][g.name].copy_(layer.bank[g.name]["Y"], non_blocking=True)
+        def copy_out(li, outs):
+            for g, y in outs.items():
+                host_out[li][g].copy_(y, non_blocking=True)
 
-        if overlap:
-            e2e_graphs, _ = stack.capture_steps(inputs, eps, mech, bank_ws, path=path, copies=(copy_in, copy_out))
-            e2e_of = lambda s: e2e_graphs[(s // D) % 2][s % D]
-        else:
-            raise SystemExit("--no-overlap runs without --no-e2e are not supported on the stack workload")
-        s = -(-s // D) * D
-        prime(s // D)
+        e2e_graphs, _ = stack.capture_stacked(inputs, eps, mech, path=path, copies=(copy_in, copy_out))
+        e2e_of = lambda s: e2e_graphs[(s // D) % 2][s % D]
+        s = -(-s // D) * D + D
+        stack.start_stacked(s // D, e2e_graphs)
         for _ in range(2):
             e2e_of(s).replay()
             s += 1
@@ -898,51 +919,69 @@ def run_llama_stack(args):
         raise RuntimeError("device status " + spl.status_string(st))
 
     # ---- the cancellation bound over every output of the first and last layer (an eager step) ---
-    bound = measure._bound(stack, inputs, eps, mech, 3 * D + 1, [0, L - 1])
-    for lk, groups_bc in bound.items():
-        for gname, v in groups_bc.items():
-            v.pop("mean_log_bound", None)
+    phase("bound check")
+    check_cycle = -(-s // D) + 1
+    check_outs = {}
+    if stacked:
+        stack.start_stacked(check_cycle, graphs)  # this cycle's corrections in place
+        bound = {}
+        for li in sorted({0, L - 1}):
+            layer = stack.layers[li]
+            outs = layer.stacked_step(inputs[li], eps, mech, stack.seeds[li], 0, check_cycle % 2, cycle=check_cycle,
+                                      path=path)
+            check_outs[li] = outs
+            bc = layer.bound_check(inputs[li], outs, eps, mech, stack.seeds[li], check_cycle, 0)
+            bound[f"layer{li}"] = {g: {"max_err_over_hard": v["max_err_over_hard"],
+                                       "log_violation_pct": v["violation_pct"], "mean_err": v["mean_err"],
+                                       "max_rel_err": v["max_err"] / v["max_abs_ref"] if v["max_abs_ref"] else 0.0}
+                                   for g, v in bc.items()}
+    else:
+        bound = measure._bound(stack, inputs, eps, mech, 3 * D + 1, [0, L - 1])
+        for lk, groups_bc in bound.items():
+            for gname, v in groups_bc.items():
+                v.pop("mean_log_bound", None)
 
     # ---- Down on its own path (Sec. 5.5): binary32 (the step's) and binary64, layer 0 -----------
+    phase("binary64 Down")
     down = {}
     gd = layer0.group("down")
-    if gd is not None:
-        gi = [g.name for g in groups].index("down")
-        Xd = inputs[0]["down"]
-        delta = layer0.deltas["down"]
-        eta = torch.empty((M, gd.K), device=dev)
-        xt64 = torch.empty((M, gd.K), dtype=torch.float64, device=dev)
-        spl.spl_noise(eta, delta, eps, mech, stack.seeds[0], stream_id=gi, offset=0)
-        spl.spl_noise_mask_f64(xt64, Xd, delta, eps, mech, stack.seeds[0], stream_id=gi, offset=0)
-        ws64 = spl.workspace(spl.spl_f64_workspace_bytes(M, gd.K, gd.N), dev)
-        C64 = torch.empty((M, gd.N), dtype=torch.float64, device=dev)
-        spl.spl_precompute_noise_product_f64(C64, eta, gd.W, workspace=ws64)
-        Y64 = torch.empty((M, gd.N), device=dev)
-        spl.spl_masked_linear_unmask_f64(Y64, xt64, gd.W, C64, workspace=ws64)  # warm-up
-        torch.cuda.synchronize()
-        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        d0.record(stream)
-        spl.spl_masked_linear_unmask_f64(Y64, xt64, gd.W, C64, workspace=ws64)
-        d1.record(stream)
-        torch.cuda.synchronize()
-        bc64 = spl.spl_bound_check(Y64, Xd, xt64.float().contiguous(), eta, gd.W)
-        b32 = bound["layer0"]["down"]
-        down = {"note": ("the paper keeps Down in the enclave (Sec. 5.5): its Delta (Thm. 3) is ~3e8, so the "
-                         "binary32 recovered output is dominated by cancellation error, though inside the bound"),
-                "binary32": {"path": group_paths["down"], "us_per_call": prod["down"]["avg_us"],
-                             "tflops": prod["down"]["tflops"], "max_rel_err": b32["max_rel_err"],
-                             "mean_err": b32["mean_err"], "max_err_over_hard": b32["max_err_over_hard"]},
-                "binary64": {"ms_per_call": d0.elapsed_time(d1), "rows": M,
-                             "tflops": flops_layer["down"] / (d0.elapsed_time(d1) * 1e-3) / 1e12,
-                             "max_rel_err": bc64["max_err"] / bc64["max_abs_ref"] if bc64["max_abs_ref"] else 0.0,
-                             "mean_err": bc64["mean_err"]}}
-        del eta, xt64, C64, Y64, ws64
+    gi = [g.name for g in groups].index("down")
+    Xd = inputs[0]["down"]
+    delta = layer0.deltas["down"]
+    eta = torch.empty((M, gd.K), device=dev)
+    xt64 = torch.empty((M, gd.K), dtype=torch.float64, device=dev)
+    spl.spl_noise(eta, delta, eps, mech, stack.seeds[0], stream_id=gi, offset=0)
+    spl.spl_noise_mask_f64(xt64, Xd, delta, eps, mech, stack.seeds[0], stream_id=gi, offset=0)
+    ws64 = spl.workspace(spl.spl_f64_workspace_bytes(M, gd.K, gd.N), dev)
+    C64 = torch.empty((M, gd.N), dtype=torch.float64, device=dev)
+    spl.spl_precompute_noise_product_f64(C64, eta, gd.W, workspace=ws64)
+    Y64 = torch.empty((M, gd.N), device=dev)
+    spl.spl_masked_linear_unmask_f64(Y64, xt64, gd.W, C64, workspace=ws64)  # warm-up
+    torch.cuda.synchronize()
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record(stream)
+    spl.spl_masked_linear_unmask_f64(Y64, xt64, gd.W, C64, workspace=ws64)
+    d1.record(stream)
+    torch.cuda.synchronize()
+    bc64 = spl.spl_bound_check(Y64, Xd, xt64.float().contiguous(), eta, gd.W)
+    b32 = bound["layer0"]["down"]
+    down = {"note": ("the paper keeps Down in the enclave (Sec. 5.5): its Delta (Thm. 3) is ~3e8, so the "
+                     "binary32 recovered output is dominated by cancellation error, though inside the bound"),
+            "binary32": {"path": group_paths["down"], "us_per_call": prod["down"]["avg_us"],
+                         "rows_per_call": rows, "tflops": prod["down"]["tflops"], "max_rel_err": b32["max_rel_err"],
+                         "mean_err": b32["mean_err"], "max_err_over_hard": b32["max_err_over_hard"]},
+            "binary64": {"ms_per_call": d0.elapsed_time(d1), "rows": M,
+                         "tflops": flops_layer["down"] / (d0.elapsed_time(d1) * 1e-3) / 1e12,
+                         "max_rel_err": bc64["max_err"] / bc64["max_abs_ref"] if bc64["max_abs_ref"] else 0.0,
+                         "mean_err": bc64["mean_err"]}}
+    del eta, xt64, C64, Y64, ws64
     six = [n for n in prod if n != "down"]
-    six_flops = sum(flops_layer[n] for n in six)
+    six_flops = sum(2 * rows * gg.K * gg.N for gg in groups if gg.name in six)
     six_ms = sum(prod[n]["avg_us"] for n in six) / 1e3
     offloaded = {"projections": "Q, K, V, O, Gate, Up", "tflops": six_flops / (six_ms * 1e-3) / 1e12,
                  "frac": six_flops / (six_ms * 1e-3) / 1e12 /
-                 (six_flops / sum(flops_layer[n] / ppk[group_paths[n]] for n in six)),
+                 (six_flops / sum(2 * rows * gg.K * gg.N / ppk[group_paths[gg.name]] for gg in groups
+                                  if gg.name in six)),
                  "max_rel_err": max(bound[lk][n]["max_rel_err"] for lk in bound for n in six),
                  "max_err_over_hard": max(bound[lk][n]["max_err_over_hard"] for lk in bound for n in six),
                  "timing": "product calls alone, from the roofline's event pairs"}
@@ -950,27 +989,32 @@ def run_llama_stack(args):
     # ---- cpu baseline + oracle match on the first rows of layer 0 (rank 0, N = 1 only) -----------
     cpu = match = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        phase("oracle on the host cores")
         from oracle import bounds, linear, philox
-        rows = args.cpu_sample_rows
-        cycle, d = 5, 3
+        nrows = args.cpu_sample_rows
         seed0 = stack.seeds[0]
-        layer0.refill(eps, mech, seed0, cycle, path=path)
-        outs = layer0.online(inputs[0], eps, mech, seed0, cycle, d, path=path)
+        if stacked:
+            cycle, d = check_cycle, 0
+            outs = check_outs[0]
+        else:
+            cycle, d = 5, 3
+            layer0.refill(eps, mech, seed0, cycle, path=path)
+            outs = layer0.online(inputs[0], eps, mech, seed0, cycle, d, path=path)
         torch.cuda.synchronize()
-        gpu_rows = {g: outs[g][:rows].double().cpu().numpy() for g in outs}
+        gpu_rows = {g: outs[g][:nrows].double().cpu().numpy() for g in outs}
         w_cpu = {g.name: g.W.cpu().numpy() for g in groups}
-        x_cpu = {g: x[:rows].cpu().numpy() for g, x in inputs[0].items()}
+        x_cpu = {g: x[:nrows].cpu().numpy() for g, x in inputs[0].items()}
         t0, flops, reps, worst = time.perf_counter(), 0, 0, 0.0
         while True:
             for gi, g in enumerate(groups):
                 X = x_cpu[g.name]
-                eta = philox.noise((rows, g.K), layer0.deltas[g.name], eps, mech, seed0, stream_id=gi,
+                eta = philox.noise((nrows, g.K), layer0.deltas[g.name], eps, mech, seed0, stream_id=gi,
                                    offset=layer0.block_offset(g, cycle, d))
                 Xt = linear.mask(X, eta)
                 r = linear.masked_linear(Xt, w_cpu[g.name])
                 C = linear.precompute_noise_product(eta, w_cpu[g.name])
                 linear.unmask(r.astype(np.float32), C.astype(np.float32))
-                flops += 2 * 2 * rows * g.K * g.N
+                flops += 2 * 2 * nrows * g.K * g.N
                 if reps == 0:
                     S = linear.abs_products(X, Xt, eta, w_cpu[g.name])
                     err = np.abs(gpu_rows[g.name] - linear.reference_output(X, w_cpu[g.name]))
@@ -980,20 +1024,40 @@ def run_llama_stack(args):
                 break
         dt = time.perf_counter() - t0
         cpu = {"value": flops / dt / 1e12, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "seconds": dt,
-               "sample": (f"first {rows} of {M} tokens of every input group of layer 0 (all 7 projections: noise, "
-                          f"mask, masked product, correction, unmask in fp64), {reps} repetitions; the rate is the "
-                          f"sample's flops over its time")}
-        match = {"rows_checked": rows, "layer": 0, "max_err_over_hard_bound": worst, "pass": worst <= 1.0}
+               "sample": (f"first {nrows} of {M} tokens of every input group of layer 0 (all 7 projections: "
+                          f"noise, mask, masked product, correction, unmask in fp64), {reps} repetitions; the rate "
+                          f"is the sample's flops over its time")}
+        match = {"rows_checked": nrows, "layer": 0, "max_err_over_hard_bound": worst, "pass": worst <= 1.0}
+
+    # ---- the online prefill alone (masked products of 512 rows, no correction work) --------------
+    phase("online prefill alone")
+    del graphs
+    torch.cuda.synchronize()
+    for layer in stack.layers:
+        layer.stacked = None
+    torch.cuda.empty_cache()
+    ws_on = spl.workspace(max(l.workspace_bytes(M, 1, path) for l in stack.layers), dev)
+    for layer in stack.layers:
+        layer.allocate(M, 1, path, workspace=ws_on)
+    for li, layer in enumerate(stack.layers):
+        layer.online(inputs[li], eps, mech, stack.seeds[li], 0, 0, path=path)
+    torch.cuda.synchronize()
+    on_graphs, on_launch = stack.capture(inputs, eps, mech, path=path, refill=False)
+    stack.set_cycle(1)
+    _time_graphs(lambda i: on_graphs[0], 0, 3, stream)
+    on_times = _time_graphs(lambda i: on_graphs[0], 0, 8, stream)
+    ms_online = sum(on_times) / len(on_times)
+    del on_graphs
 
     # ---- decode at one token per step (the same layers, banks of D one-row draws) -----------------
     decode = None
     if not args.no_decode:
-        del graphs
+        phase("decode")
         torch.cuda.synchronize()
         ws1 = spl.workspace(max(l.workspace_bytes(1, D) for l in stack.layers), dev)
         for layer in stack.layers:
             layer.allocate(1, D, workspace=ws1)
-        del bank_ws
+        del ws_on
         torch.cuda.empty_cache()
         inputs1 = stack.inputs(13, device=dev)
         stack.step(inputs1, eps, mech, 0)
@@ -1021,27 +1085,30 @@ def run_llama_stack(args):
             raise RuntimeError("device status " + spl.status_string(st))
 
     path_name = "+".join(sorted(set(group_paths.values())))
+    schedule_note = (f"stacked: every product call multiplies the step's {M} masked rows and the {M} noise rows of "
+                     f"the next cycle's same draw in one launch of {2 * M} rows, so each step computes 1/{D} of the "
+                     "next cycle's corrections, summed exactly as the rows they will unmask"
+                     if stacked else
+                     f"banked: each step computes the next cycle's corrections of 1/{D} of the layers ({D} draws x "
+                     f"{M} rows per group) on a lower-priority stream beside its prefill")
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "path": path_name, "data": "synthetic",
         "config": {"workload": stack_workload(L, M, mech, eps), "layers": L, "tokens": M, "eps": eps, "mech": mech,
                    "bank_draws": D, "flops_per_step": flops_step,
-                   "value": ("algorithmic flops of the prefill's masked products (2 M K N per projection, 28 layers) "
-                             "per second of the whole step: online prefill plus its 1/8 share of the bank"),
-                   "bank_schedule": ("each step computes the next cycle's corrections of an eighth of the layers on a "
-                                     "lower-priority stream beside its prefill (per-step graphs)") if overlap else
-                                    "each cycle's corrections computed before its first step",
+                   "value": (f"algorithmic flops of the prefill's masked products (2 M K N per projection, {L} "
+                             "layers) per second of the whole step: the prefill with its correction work"),
+                   "bank_schedule": schedule_note,
                    "online_noise": "drawn again in each step's mask from the bank's Philox counters",
                    "l2": "weights 40 GB per step (with their splits) >> 129 MB L2 (no flush needed)",
                    "parallelism": "replicas" if world > 1 else "single", "setup_s": build_s},
         "prefill": {"ms_per_prefill_with_correction": ms, "tokens_per_s": M / (ms * 1e-3),
                     "online_only": {"ms_per_prefill": ms_online, "tflops": flops_step / (ms_online * 1e-3) / 1e12,
                                     "frac": flops_step / (ms_online * 1e-3) / 1e12 / prod_peak,
-                                    "tokens_per_s": M / (ms_online * 1e-3), "kernels": on_launch[1]},
-                    "correction_serial_ms_per_prefill": bank_ms / D,
-                    "serial_sum_ms": ms_online + bank_ms / D},
-        "bank": bank,
+                                    "tokens_per_s": M / (ms_online * 1e-3), "kernels": on_launch[0],
+                                    "what": f"the masked products of {M} rows with no correction work, timed alone"},
+                    "correction_ms_per_prefill": ms - ms_online},
         "roofline": roofline,
         "gpu_launches": gpu_launches,
         "clocks": clocks.summary(),
@@ -1051,8 +1118,7 @@ def run_llama_stack(args):
     if decode is not None:
         result["decode"] = decode
     result["offloaded_six"] = offloaded
-    if down:
-        result["down"] = down
+    result["down"] = down
     result["bound_check"] = bound
     if layer0.calibration:
         result["path_choice"] = {g: {"path": c["path"], **{f"{p}_max_err_over_hard": c[p]["max_err_over_hard"]

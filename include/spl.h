@@ -356,6 +356,27 @@ spl_status spl_precompute_noise_product_matched_split(float* C, const spl_weight
 spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt, const float* W, const float* C,
                                             int64_t M, int64_t K, int64_t N, cudaStream_t stream);
 
+/* ---- a4 + a5 + a6 in one launch: the online product beside a bank draw ------
+ * The masked product of M rows with its unmask (Eq. add-and-then-subtract) and
+ * the corrections W eta of M_bank noise rows (Sec. 5.2, the bank) as one
+ * product of M + M_bank rows, so that both run in the launch shape of the
+ * larger product.  A is the left operand [M + M_bank, K]: the M rows of X~
+ * first, then the M_bank noise rows, as fp32 (A->w) and/or its FP16X3 split
+ * (A->f16_hi, f16_lo, f16_exp, as spl_noise_mask_split writes it; the
+ * product then reads only the split).  C [M, N] is the correction of the M
+ * masked rows.  YC [M + M_bank, N]: rows 0..M-1 get Y = fl32(fl32(Xt W^T) - C),
+ * rows M.. the corrections fl32(eta W^T).  Every output row of a product is
+ * summed in the same order wherever it sits (launch forms are uniform over the
+ * rows of each column of tiles), so a correction computed here is summed
+ * exactly as the masked row that later meets it in a call with the same
+ * M + M_bank, K, N and path: their rounding errors cancel in the unmask.
+ * Tensor-core paths only (TF32X3 / FP16X3, resolved as for M + M_bank rows);
+ * EUNSUPPORTED for a path that resolves to FP32.  Workspace and other errors
+ * as spl_masked_linear_unmask for M + M_bank rows. */
+spl_status spl_masked_linear_unmask_precompute(float* YC, const spl_weight* A, const spl_weight* W, const float* C,
+                                               int64_t M, int64_t M_bank, int64_t K, int64_t N, spl_path path,
+                                               void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
 /* ---- a8: the cancellation bound on the GPU, and the path choice ----------
  * The paper judges a configuration by evaluating its floating-point bound on
  * sampled inputs and masks (Sec. 4.5 after Thm. 4; Sec. 6.3.2).

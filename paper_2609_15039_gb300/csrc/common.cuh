@@ -80,6 +80,7 @@ struct LinearArgs {
   const uint16_t* a_h16;    // [M, K]  fp16 split of a, made by the caller (FP16X3), or null
   const uint16_t* a_l16;
   const int32_t* a_exp;     // [M]
+  int64_t c_rows;           // rows of c: output rows from c_rows on subtract nothing (tensor-core kernels)
 };
 
 // Workspace layout shared by every product call: the first kCounterBytes hold
@@ -108,6 +109,7 @@ inline LinearArgs make_args(float* out, const float* a, const spl_weight& W, con
   r.ws_bytes = ws_bytes;
   r.stream = stream;
   r.path = path;
+  r.c_rows = M;
   return r;
 }
 

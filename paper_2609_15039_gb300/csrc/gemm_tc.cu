@@ -360,7 +360,8 @@ struct TcMaps {
 // flight per thread whatever S is, so the epilogue streams instead of waiting load by load.
 template <int S, int BN>
 __device__ __forceinline__ void reduce_store(const float* red, int r0, int r1, int64_t m0, int64_t n0, int64_t M,
-                                             int64_t N, const float* __restrict__ C, float* __restrict__ out) {
+                                             int64_t N, const float* __restrict__ C, float* __restrict__ out,
+                                             int64_t c_rows) {
   constexpr int RS = BN + 4;
   constexpr int P = S >= 8 ? 2 : (S >= 4 ? 4 : 8);
   const bool vec = (N & 3) == 0;
@@ -384,7 +385,7 @@ __device__ __forceinline__ void reduce_store(const float* red, int r0, int r1, i
 #pragma unroll
         for (int q = 0; q < S; ++q) part[u][q] = ld_cluster_f4(map_to_rank(off, (uint32_t)q));
       }
-      if (C && vec && n + 4 <= N) cc[u] = __ldcs(reinterpret_cast<const float4*>(C + m * N + n));
+      if (C && m < c_rows && vec && n + 4 <= N) cc[u] = __ldcs(reinterpret_cast<const float4*>(C + m * N + n));
     }
 #pragma unroll
     for (int u = 0; u < P; ++u) {
@@ -398,8 +399,9 @@ __device__ __forceinline__ void reduce_store(const float* red, int r0, int r1, i
         v = make_float4(__fadd_rn(v.x, part[u][q].x), __fadd_rn(v.y, part[u][q].y), __fadd_rn(v.z, part[u][q].z),
                         __fadd_rn(v.w, part[u][q].w));
       float* o = out + m * N + n;
+      const bool has_c = C && m < c_rows;
       if (vec && n + 4 <= N) {
-        if (C)
+        if (has_c)
           v = make_float4(__fsub_rn(v.x, cc[u].x), __fsub_rn(v.y, cc[u].y), __fsub_rn(v.z, cc[u].z),
                           __fsub_rn(v.w, cc[u].w));
         *reinterpret_cast<float4*>(o) = v;
@@ -407,7 +409,7 @@ __device__ __forceinline__ void reduce_store(const float* red, int r0, int r1, i
         const float vv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-          if (n + j < N) o[j] = C ? __fsub_rn(vv[j], C[m * N + n + j]) : vv[j];
+          if (n + j < N) o[j] = has_c ? __fsub_rn(vv[j], C[m * N + n + j]) : vv[j];
       }
     }
   }
@@ -431,7 +433,7 @@ __global__ void __launch_bounds__(THREADS, Cfg<Md, BN, RK>::CTAS_PER_SM)
 tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
                const int* __restrict__ a_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
                int64_t k_per_split, int splits, int tile_base, int m_tiles, int skip_kblock, int seg_blocks,
-               int epi_tma) {
+               int epi_tma, int64_t c_rows) {
   using L = Cfg<Md, BN, RK>;
   constexpr int STAGES = L::STAGES, BK = Md::BK, RED_STRIDE = L::RED_STRIDE;
   extern __shared__ uint8_t smem_raw[];
@@ -592,7 +594,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     const int t = threadIdx.x - 64;  // 0..127
     if constexpr (Md::kF16)
       for (int j = t; j < BN; j += 128) col_scale[j] = pow2f(-((n0 + j < N) ? __ldg(w_exp + n0 + j) : 0));
-    if (C && (N & 3) == 0) {
+    if (C && m0 < c_rows && (N & 3) == 0) {
       const int rows_per_rank = (BM + splits - 1) / splits;
       const int rank = splits > 1 ? (int)cluster_rank() : 0;
       const int r0 = rank * rows_per_rank, r1 = (r0 + rows_per_rank < BM) ? r0 + rows_per_rank : BM;
@@ -600,7 +602,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       const int lines = (int)ceil_div(ncols * 4, 128);
       for (int i = t; i < (r1 - r0) * lines; i += 128) {
         const int64_t m = m0 + r0 + i / lines;
-        if (m < M) prefetch_l2(C + m * N + n0 + (int64_t)(i % lines) * 32);
+        if (m < M && m < c_rows) prefetch_l2(C + m * N + n0 + (int64_t)(i % lines) * 32);
       }
     }
     pdl_wait();  // the row exponents of A come from the kernel before this one
@@ -641,13 +643,14 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       const float sr = pow2f(-e_row);
       // chunks holding columns below N (the copies start inside the tensor)
       const int nchunks = (int)std::min<int64_t>(BN / 32, ceil_div(N - n0, (int64_t)32));
-      if (C && t == 0) {
+      const bool c_tile = C && m0 < c_rows;  // rows past c_rows subtract nothing (the copy fills them with 0)
+      if (c_tile && t == 0) {
         mbar_expect_tx(cload_bar, (uint32_t)nchunks * L::EPI_CHUNK);
         const uint64_t pol_c = l2_evict_first();
         for (int c = 0; c < nchunks; ++c)
           tma_load_2d(smem_u32(smem + (size_t)c * L::EPI_CHUNK), &maps.c, cload_bar, (int)n0 + 32 * c, (int)m0, pol_c);
       }
-      bool okc = !C || mbar_wait(cload_bar, 0u, kWaitNs, abort_flag);
+      bool okc = !c_tile || mbar_wait(cload_bar, 0u, kWaitNs, abort_flag);
       okc = __all_sync(0xffffffffu, okc) && !*abort_flag;
       if (okc) {
 #pragma unroll 1
@@ -668,7 +671,7 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
           for (int j = 0; j < 8; ++j) {
             float4 o = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
             float4* dst = row + (j ^ (r & 7));
-            if (C) {
+            if (c_tile) {
               const float4 cc = *dst;
               o = make_float4(__fsub_rn(o.x, cc.x), __fsub_rn(o.y, cc.y), __fsub_rn(o.z, cc.z), __fsub_rn(o.w, cc.w));
             }
@@ -727,14 +730,14 @@ tc_gemm_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
     const int rows_per_rank = (BM + splits - 1) / splits;
     const int r0 = rank * rows_per_rank, r1 = (r0 + rows_per_rank < BM) ? r0 + rows_per_rank : BM;
     switch (splits) {
-      case 1: reduce_store<1, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
-      case 2: reduce_store<2, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
-      case 3: reduce_store<3, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
-      case 4: reduce_store<4, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
-      case 5: reduce_store<5, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
-      case 6: reduce_store<6, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
-      case 7: reduce_store<7, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
-      default: reduce_store<8, BN>(red, r0, r1, m0, n0, M, N, C, out); break;
+      case 1: reduce_store<1, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
+      case 2: reduce_store<2, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
+      case 3: reduce_store<3, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
+      case 4: reduce_store<4, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
+      case 5: reduce_store<5, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
+      case 6: reduce_store<6, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
+      case 7: reduce_store<7, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
+      default: reduce_store<8, BN>(red, r0, r1, m0, n0, M, N, C, out, c_rows); break;
     }
   }
   __syncwarp();
@@ -771,7 +774,7 @@ template <class Md, int BN, int RK>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
                      const int* __restrict__ a_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
-                     int tiles, int m_tiles, int chain) {
+                     int tiles, int m_tiles, int chain, int64_t c_rows) {
   using L = Cfg<Md, BN, RK>;
   constexpr int STAGES = L::STAGES, BK = Md::BK;
   constexpr uint32_t ACC_COLS = 256;  // column offset of the second accumulator
@@ -927,7 +930,7 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
       const int lines = (int)ceil_div(ncols * 4, 128);
       for (int j = threadIdx.x - 64; j < BM * lines; j += 128) {
         const int64_t pm = pm0 + j / lines;
-        if (pm < M) prefetch_l2(C + pm * N + pn0 + (int64_t)(j % lines) * 32);
+        if (pm < M && pm < c_rows) prefetch_l2(C + pm * N + pn0 + (int64_t)(j % lines) * 32);
       }
     };
     pdl_wait();  // C and the row exponents of A come from before this kernel
@@ -978,16 +981,17 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
             v[j] = (v[j] * sr) * pow2f(-((nc + j < N) ? __ldg(w_exp + nc + j) : 0));
         }
         if (m < M && vec_ok) {
+          const bool has_c = C && m < c_rows;
           float4 cc[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j)
-            cc[j] = (C && nc + 4 * j < N) ? __ldcs(reinterpret_cast<const float4*>(C + m * N + nc + 4 * j))
-                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+            cc[j] = (has_c && nc + 4 * j < N) ? __ldcs(reinterpret_cast<const float4*>(C + m * N + nc + 4 * j))
+                                              : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             if (nc + 4 * j >= N) continue;
             float4 o = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-            if (C)
+            if (has_c)
               o = make_float4(__fsub_rn(o.x, cc[j].x), __fsub_rn(o.y, cc[j].y), __fsub_rn(o.z, cc[j].z),
                               __fsub_rn(o.w, cc[j].w));
             *reinterpret_cast<float4*>(out + m * N + nc + 4 * j) = o;
@@ -1066,7 +1070,7 @@ template <int TN>
 __global__ void __launch_bounds__(THREADS, SwapCfg<TN>::CTAS_PER_SM)
 tc_swap_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
                const int* __restrict__ x_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
-               int64_t k_per_split, int splits, int m_tiles, int chain) {
+               int64_t k_per_split, int splits, int m_tiles, int chain, int64_t c_rows) {
   using L = SwapCfg<TN>;
   constexpr int STAGES = L::STAGES, BK = L::BK, RS = L::RED_STRIDE;
   extern __shared__ uint8_t smem_raw[];
@@ -1264,7 +1268,7 @@ tc_swap_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
               const int64_t m = m0 + 16 * c + i;
-              if (m < M) out[m * N + n] = C ? __fsub_rn(v[i], __ldcs(C + m * N + n)) : v[i];
+              if (m < M) out[m * N + n] = (C && m < c_rows) ? __fsub_rn(v[i], __ldcs(C + m * N + n)) : v[i];
             }
           }
         } else {
@@ -1295,7 +1299,7 @@ tc_swap_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
       const uint32_t off = red_base + (uint32_t)((rr * RS + j) * 4);
       float v = ld_cluster_f32(map_to_rank(off, 0u));
       for (int qq = 1; qq < splits; ++qq) v = __fadd_rn(v, ld_cluster_f32(map_to_rank(off, (uint32_t)qq)));
-      out[m * N + nn] = C ? __fsub_rn(v, __ldcs(C + m * N + nn)) : v;
+      out[m * N + nn] = (C && m < c_rows) ? __fsub_rn(v, __ldcs(C + m * N + nn)) : v;
     }
     __syncwarp();
     cluster_sync_all();  // no CTA leaves while others still read its shared memory
@@ -1525,7 +1529,10 @@ TcShape tc_shape_for(int v, int64_t M, int64_t K, int64_t N, int sms) {
     if (c < best.cost * (1.0 - 1e-9)) best = TcShape{v, 0, tiles, s, c};
   }
   const int64_t wave = max_active_clusters(v, 1, sms);
-  const int64_t full = (tiles / wave) * wave, rest = tiles - full;
+  // whole waves of unsplit tiles, cut at whole columns of tiles (M is the fast index), so that every
+  // output row of a column is summed the same way wherever it sits in M
+  const int64_t m_tiles = ceil_div(M, BM);
+  const int64_t full = (tiles / wave) * wave / m_tiles * m_tiles, rest = tiles - full;
   if (full > 0 && rest > 0) {
     const double cf = launch_cost(v, full, K, 1, sms);
     for (int s = 1; s <= max_s; ++s) {
@@ -1616,7 +1623,7 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
   int epi_tma = (a.N & 3) == 0 && aligned16(a.out) && (!a.c || aligned16(a.c)) ? 1 : 0;
   if (epi_tma) {
     if (!make_map(&maps.y, a.out, false, a.M, a.N, 32, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        (a.c && !make_map(&maps.c, a.c, false, a.M, a.N, 32, BM, CU_TENSOR_MAP_SWIZZLE_128B)))
+        (a.c && a.c_rows > 0 && !make_map(&maps.c, a.c, false, a.c_rows, a.N, 32, BM, CU_TENSOR_MAP_SWIZZLE_128B)))
       return SPL_ECUDA;
   }
   const int m_tiles = (int)ceil_div(a.M, BM);
@@ -1639,7 +1646,8 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_persistent_kernel<Md, BN, RK>, maps, a.out, a.c, a_exp,
-                                             (const int*)a.w_exp, a.M, a.K, a.N, (int)tiles, m_tiles, kChainBlocks);
+                                             (const int*)a.w_exp, a.M, a.K, a.N, (int)tiles, m_tiles, kChainBlocks,
+                                             a.c_rows);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   }
@@ -1669,7 +1677,7 @@ spl_status launch_tc(const LinearArgs& a, const uint16_t* a_hi, const uint16_t* 
     first = false;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_gemm_kernel<Md, BN, RK>, maps, a.out, a.c, a_exp,
                                              (const int*)a.w_exp, a.M, a.K, a.N, kps, splits, (int)base, m_tiles,
-                                             skip_kblock, seg, epi_tma);
+                                             skip_kblock, seg, epi_tma, a.c_rows);
     note_launches(1);
     return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
   };
@@ -1726,7 +1734,7 @@ spl_status launch_swap_tn(const LinearArgs& a, const uint16_t* x_hi, const uint1
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_swap_kernel<TN>, maps, a.out, a.c, x_exp, (const int*)a.w_exp,
-                                           a.M, a.K, a.N, kps, splits, m_tiles, chain);
+                                           a.M, a.K, a.N, kps, splits, m_tiles, chain, a.c_rows);
   note_launches(1);
   return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
 }

@@ -66,7 +66,7 @@ spl_status check_weight(const spl_weight* W, int64_t K) {
 
 spl_status run_linear(float* out, const float* a, const spl_weight* W, const float* C, bool need_c, int64_t M,
                       int64_t K, int64_t N, spl_path path, void* ws, size_t ws_bytes, cudaStream_t stream,
-                      const spl_weight* A = nullptr, const MaskNoise* noise = nullptr) {
+                      const spl_weight* A = nullptr, const MaskNoise* noise = nullptr, int64_t c_rows = -1) {
   if (M < 0 || K < 0 || N < 0) return SPL_EINVAL;
   if (!valid_path(path)) return SPL_EINVAL;
   if (M == 0 || N == 0) return SPL_OK;
@@ -93,6 +93,10 @@ spl_status run_linear(float* out, const float* a, const spl_weight* W, const flo
   if (!use_split && plan.total() > 0 && (!ws || ws_bytes < plan.total())) return SPL_EWORKSPACE;
   if (ws && !aligned16(ws)) return SPL_EALIGN;
   LinearArgs args = make_args(out, a, *W, C, M, K, N, ws, ws_bytes, stream, resolved);
+  if (c_rows >= 0) {  // only the first c_rows output rows subtract C (the tensor-core kernels)
+    if (plan.kernel != kKernelTc) return SPL_EUNSUPPORTED;
+    args.c_rows = c_rows;
+  }
   if (use_split) {
     args.a_h16 = A->f16_hi;
     args.a_l16 = A->f16_lo;
@@ -193,6 +197,22 @@ extern "C" spl_status spl_masked_linear_unmask_split(float* Y, const spl_weight*
                                                      void* workspace, size_t workspace_bytes, cudaStream_t stream) {
   if (!Xt) return SPL_EINVAL;
   return run_linear(Y, Xt->w, W, C, true, M, K, N, path, workspace, workspace_bytes, stream, Xt);
+}
+
+extern "C" spl_status spl_masked_linear_unmask_precompute(float* YC, const spl_weight* A, const spl_weight* W,
+                                                          const float* C, int64_t M, int64_t M_bank, int64_t K,
+                                                          int64_t N, spl_path path, void* workspace,
+                                                          size_t workspace_bytes, cudaStream_t stream) {
+  if (!A || M < 0 || M_bank < 0) return SPL_EINVAL;
+  if (M > 0 && !C) return SPL_EINVAL;
+  if (M + M_bank > (int64_t(1) << 31)) return SPL_ESHAPE;
+  if (M + M_bank == 0 || N == 0) return SPL_OK;
+  if (K > 0) {  // the tensor-core paths only: decide before anything runs
+    const spl_path resolved = resolve(M + M_bank, K, path, W && has_tf32(*W), W && has_f16(*W));
+    if (!is_tc(resolved)) return SPL_EUNSUPPORTED;
+  }
+  return run_linear(YC, A->w, W, C, M > 0, M + M_bank, K, N, path, workspace, workspace_bytes, stream, A, nullptr,
+                    M);
 }
 
 extern "C" spl_status spl_noise_mask_linear_unmask(float* Y, float* Xt, const float* X, const spl_weight* W,

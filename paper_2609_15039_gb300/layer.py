@@ -180,6 +180,75 @@ class MaskedLayer:
                                      f16_lo=torch.empty((draws * M, g.K), dtype=torch.int16, device=dev),
                                      f16_exp=torch.empty(draws * M, dtype=torch.int32, device=dev))
 
+    # ------------------------------------------------------------------ stacked schedule
+    def allocate_stacked(self, M, draws, path="auto", workspace=None):
+        """Buffers of the stacked schedule: step d of a bank cycle multiplies, in one product of 2M rows
+        (spl_masked_linear_unmask_precompute), the M rows of X~ for draw d of this cycle and the M noise
+        rows of draw d of the next cycle, so every step carries its share of the bank and the products
+        run in the launch shape of 2M rows.  Per group: the left operand [2M, K] (its fp16 split when
+        the product runs FP16X3, else fp32) and out[p][d] [2M, N] for parities p = 0, 1: a cycle of
+        parity p reads its corrections from out[p][d][M:] and writes [Y; the next cycle's corrections]
+        into out[1 - p][d].  A correction and the masked row that later meets it sit in products of
+        the same shape, which sum every row in the same order, so their roundings cancel."""
+        if M % 4:
+            raise ValueError("stacked schedule: M % 4 == 0 (the split's row exponents of each half are "
+                             "16-byte aligned)")
+        dev = self.groups[0].W.device
+        need = max(spl.spl_linear_workspace_bytes(2 * M, g.K, g.N, self.path_of(g, path, 2 * M)) for g in self.groups)
+        if workspace is not None:
+            assert workspace.numel() >= need, "shared workspace too small"
+            self.workspace = workspace
+        elif self.workspace is None or self.workspace.numel() < need:
+            self.workspace = spl.workspace(need, dev)
+        self.M, self.draws = M, draws
+        self.rng_base = torch.zeros(len(self.groups), dtype=torch.int64, device=dev)
+        self.stacked = {}
+        for g in self.groups:
+            if g.name in self.fp64:
+                raise ValueError("stacked schedule: the binary64 group keeps the separate bank")
+            fused = self._fused_split(g, path, 2 * M)
+            a = (spl.Weight(None, f16_hi=torch.empty((2 * M, g.K), dtype=torch.int16, device=dev),
+                            f16_lo=torch.empty((2 * M, g.K), dtype=torch.int16, device=dev),
+                            f16_exp=torch.empty(2 * M, dtype=torch.int32, device=dev))
+                 if fused else spl.Weight(torch.empty((2 * M, g.K), device=dev)))
+            out = [[torch.zeros((2 * M, g.N), device=dev) for _ in range(draws)] for _ in range(2)]
+            resolved = spl.PATH_NAMES[spl.spl_resolve_path(2 * M, g.K, g.N, self.path_of(g, path, 2 * M))]
+            self.stacked[g.name] = {"a": a, "out": out, "fused": fused, "path": resolved}
+
+    def stacked_step(self, inputs, eps, mech, seed, d, parity, cycle=0, path="auto", stream=None, timer=None,
+                     device_base=False):
+        """Step d of a cycle of parity ``parity`` in the stacked schedule (see allocate_stacked): the mask
+        of draw d of this cycle, the noise of draw d of the next cycle, and their product with W in one
+        call whose first M rows are unmasked with this cycle's correction.  The arithmetic path of each
+        group is the one resolved when the buffers were allocated.  Returns {group: Y [M, N]}."""
+        M, D = self.M, self.draws
+        out = {}
+        for gi, g in enumerate(self.groups):
+            st = self.stacked[g.name]
+            a = st["a"]
+            off, off_dev = self._offset(gi, g, cycle, d, device_base)
+            off_next = off + D * (M * g.K // 4)  # draw d of the next cycle
+            delta = self.deltas[g.name]
+            if st["fused"]:
+                spl.spl_noise_mask_split(None, a.f16_hi[:M], a.f16_lo[:M], a.f16_exp[:M], inputs[g.name], delta, eps,
+                                         mech, seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
+                spl.spl_noise_mask_split(None, a.f16_hi[M:], a.f16_lo[M:], a.f16_exp[M:], None, delta, eps, mech,
+                                         seed, stream_id=gi, offset=off_next, stream=stream, offset_dev=off_dev)
+            else:
+                spl.spl_noise_mask(a.w[:M], None, inputs[g.name], delta, eps, mech, seed, stream_id=gi, offset=off,
+                                   stream=stream, offset_dev=off_dev)
+                spl.spl_noise(a.w[M:], delta, eps, mech, seed, stream_id=gi, offset=off_next, stream=stream,
+                              offset_dev=off_dev)
+            res = st["out"][1 - parity][d]
+            if timer:
+                timer("begin", "masked_linear_unmask", g.name)
+            spl.spl_masked_linear_unmask_precompute(res, a, g.wt, st["out"][parity][d][M:], M, path=st["path"],
+                                                    workspace=self.workspace, stream=stream)
+            if timer:
+                timer("end", "masked_linear_unmask", g.name)
+            out[g.name] = res[:M]
+        return out
+
     def enable_overlap(self):
         """A second correction buffer per group (and noise buffer, for stored noise), so that a bank
         cycle can run its online steps on one while the next cycle's are filled into the other
@@ -464,8 +533,10 @@ class MaskedStack:
         self.layers, self.seeds = layers, seeds
 
     @classmethod
-    def build(cls, model, n_layers, M, draws, base_seed, device="cuda", split=True, power_iters=1000, path="auto"):
-        """Seeded synthetic weights per layer (workloads.layer_seed), Delta per layer (Thms. 1-3)."""
+    def build(cls, model, n_layers, M, draws, base_seed, device="cuda", split=True, power_iters=1000, path="auto",
+              stacked=False):
+        """Seeded synthetic weights per layer (workloads.layer_seed), Delta per layer (Thms. 1-3).
+        stacked: buffers of the stacked schedule (MaskedLayer.allocate_stacked) instead of a bank."""
         from . import workloads as wl
         layers = []
         for li in range(n_layers):
@@ -475,10 +546,16 @@ class MaskedStack:
             del weights
             layer.sensitivities(power_iters=power_iters)
             layers.append(layer)
-        need = max(l.workspace_bytes(M, draws, path) for l in layers)
-        ws = spl.workspace(need, device)
-        for layer in layers:
-            layer.allocate(M, draws, path, workspace=ws)
+        if stacked:
+            need = max(spl.spl_linear_workspace_bytes(2 * M, g.K, g.N, path) for l in layers for g in l.groups)
+            ws = spl.workspace(need, device)
+            for layer in layers:
+                layer.allocate_stacked(M, draws, path, workspace=ws)
+        else:
+            need = max(l.workspace_bytes(M, draws, path) for l in layers)
+            ws = spl.workspace(need, device)
+            for layer in layers:
+                layer.allocate(M, draws, path, workspace=ws)
         return cls(layers, [wl.layer_seed(base_seed, li, 99) for li in range(n_layers)])
 
     @property
@@ -637,6 +714,66 @@ class MaskedStack:
                 graphs[parity].append(graph)
                 launches[parity].append(spl.spl_launch_count() - n0)
         return graphs, launches
+
+    def capture_stacked(self, inputs, eps, mech, path="auto", timer=None, copies=None):
+        """CUDA graphs of the stacked schedule (MaskedLayer.allocate_stacked): graphs[p][d] runs step d of
+        a cycle of parity p through every layer -- each product also computing the next cycle's
+        correction of draw d -- and graph d = draws - 1 moves every Philox base on by one cycle.  After
+        start_stacked(c), replay graphs[(s // draws) % 2][s % draws] for steps s = c draws, ...: any
+        number of them, each one step of the method with its share of the bank.  ``timer(d, li, phase,
+        kind, group)`` as in capture.  ``copies``: (h2d, d2h) host-transfer hooks -- h2d(li) is called on
+        a host-to-device copy stream before the steps, once per layer in order, and returns an event
+        that layer li waits for; d2h(li, outs) on a device-to-host copy stream after layer li's calls
+        (which that stream waits for first), outs being the layer's {group: Y}.  Returns the graphs and
+        their kernel counts."""
+        if copies is not None and not hasattr(self, "_h2d_stream"):
+            _, hi = torch.cuda.Stream.priority_range()
+            self._h2d_stream = torch.cuda.Stream(priority=hi)
+            self._d2h_stream = torch.cuda.Stream(priority=hi)
+        D = self.draws
+        graphs, launches = [[], []], [[], []]
+        for parity in range(2):
+            for d in range(D):
+                graph = torch.cuda.CUDAGraph()
+                n0 = spl.spl_launch_count()
+                with torch.cuda.graph(graph):
+                    main = torch.cuda.current_stream()
+                    ready = []
+                    if copies is not None:
+                        self._h2d_stream.wait_stream(main)
+                        with torch.cuda.stream(self._h2d_stream):
+                            ready = [copies[0](li) for li in range(len(self.layers))]
+                        self._d2h_stream.wait_stream(main)
+                    for li, (layer, x, seed) in enumerate(zip(self.layers, inputs, self.seeds)):
+                        if ready:
+                            main.wait_event(ready[li])
+                        t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
+                            if timer else None
+                        outs = layer.stacked_step(x, eps, mech, seed, d, parity, path=path, timer=t, device_base=True)
+                        if copies is not None:
+                            self._d2h_stream.wait_stream(main)
+                            with torch.cuda.stream(self._d2h_stream):
+                                copies[1](li, outs)
+                    if copies is not None:
+                        main.wait_stream(self._h2d_stream)
+                        main.wait_stream(self._d2h_stream)
+                    if d == D - 1:
+                        for layer in self.layers:
+                            for gi, g in enumerate(layer.groups):
+                                spl.spl_rng_advance(layer.rng_base[gi:gi + 1], D * (layer.M * g.K // 4))
+                graphs[parity].append(graph)
+                launches[parity].append(spl.spl_launch_count() - n0)
+        return graphs, launches
+
+    def start_stacked(self, cycle, graphs):
+        """Before replaying the stacked graphs from cycle ``cycle``: run cycle ``cycle - 1``'s graphs once
+        (their outputs are discarded; their corrections, for cycle ``cycle``, are kept), leaving the
+        device-side Philox bases at ``cycle``."""
+        if cycle < 1:
+            raise ValueError("start_stacked: the cycle before must exist")
+        self.set_cycle(cycle - 1)
+        for g in graphs[(cycle - 1) % 2]:
+            g.replay()
 
     def refill_all(self, eps, mech, path="auto", parity=0, ahead=0, workspace=None):
         """Every layer's bank for the cycle at the device-side bases (+ ``ahead`` cycles), into

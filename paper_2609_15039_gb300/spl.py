@@ -74,6 +74,7 @@ _SIGS = {
     "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_masked_linear_unmask": (_I, [_P, _P, _PW, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_masked_linear_unmask_noalloc": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _P]),
+    "spl_masked_linear_unmask_precompute": (_I, [_P, _PW, _PW, _P, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_noise_mask_linear_unmask": (_I, [_P, _P, _P, _PW, _P, _I64, _I64, _I64, _D, _D, _I, spl_rng, _I, _P, _SZ,
                                           _P]),
     "spl_delta_layernorm": (_D, [_P, _I64]),
@@ -282,6 +283,23 @@ def spl_masked_linear_unmask_split(Y, Xt, W, C, path="auto", workspace=None, str
     _check(lib().spl_masked_linear_unmask_split(_dev(Y, "Y"), ctypes.byref(xs), ctypes.byref(ws_), _dev(C, "C"), M, K,
                                                 N, _path(path), wsp, wsb, _stream(stream)),
            "spl_masked_linear_unmask_split")
+
+
+def spl_masked_linear_unmask_precompute(YC, A, W, C, M, path="auto", workspace=None, stream=None):
+    """The masked product of the first M rows of A with its unmask and the corrections of A's other rows
+    in one launch: YC [M + M_bank, N], A a Weight over [M + M_bank, K] (fp32 and/or fp16 split),
+    C [M, N]."""
+    A, W = _weight(A), _weight(W)
+    rows, K = A.shape
+    N = W.shape[0]
+    M_bank = rows - int(M)
+    if W.shape[-1] != K or YC.numel() != rows * N or M_bank < 0 or (C is not None and C.numel() != int(M) * N):
+        raise ValueError("spl_masked_linear_unmask_precompute: shape mismatch")
+    wsp, wsb = _ws(workspace)
+    xs, ws_ = A.c_struct(), W.c_struct()
+    _check(lib().spl_masked_linear_unmask_precompute(_dev(YC, "YC"), ctypes.byref(xs), ctypes.byref(ws_),
+                                                     _dev(C, "C"), int(M), M_bank, K, N, _path(path), wsp, wsb,
+                                                     _stream(stream)), "spl_masked_linear_unmask_precompute")
 
 
 def spl_slalom_quantize(out, v, stream=None):

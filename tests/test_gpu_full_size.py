@@ -184,3 +184,22 @@ def test_llama_lm_head(spl, M):
     got = Y[torch.as_tensor(rows, device="cuda")][:, torch.as_tensor(cols, device="cuda")].double().cpu().numpy()
     err = np.abs(got - linear.reference_output(Xs, Ws))
     assert np.all(err <= bounds.hard_bound(*S, K) * (1 + 1e-5))
+
+
+def test_llama_stacked_prefill_512(spl):
+    """The bench's schedule at its own size: a Llama-3.2-3B-shaped layer at 512 tokens, each product of
+    1024 rows carrying the next cycle's correction of its draw; the recovered outputs of the second
+    cycle checked on sampled outputs against the hard bound (Laplace, eps = 1)."""
+    from paper_2609_15039_gb300.layer import MaskedLayer
+    model, M, draws, eps, mech = wl.LLAMA_3_2_3B, 512, 2, 1.0, "laplace"
+    layer, inputs = make_layer(model, 3, 7, draws, M)
+    stacked = MaskedLayer(model, layer.groups, deltas=layer.deltas)
+    stacked.allocate_stacked(M, draws)
+    seed = 1003
+    for cycle in range(2):
+        for d in range(draws):
+            outs = stacked.stacked_step(inputs, eps, mech, seed, d, cycle % 2, cycle=cycle)
+    torch.cuda.synchronize()
+    worst = check_sampled(stacked, inputs, outs, eps, mech, seed, 1, draws - 1)
+    assert worst < 0.05
+    assert spl.spl_get_device_status() == 0

@@ -191,3 +191,67 @@ def test_stored_noise_steps_equal_drawn_noise_steps(spl, mech):
         for g in a:
             assert torch.equal(a[g], b[g]), g
     assert spl.spl_get_device_status() == 0
+
+
+# ------------------------------------------------ the stacked schedule (online rows beside a bank draw)
+def make_stacked(model, M, draws, layers=1, zero_inputs=False):
+    from paper_2609_15039_gb300.layer import MaskedLayer, MaskedStack
+    stack_layers = []
+    for li in range(layers):
+        weights = {name: wl.weight(N, K, seed=500 + 10 * li + pi, device="cuda")
+                   for pi, (name, K, N, g) in enumerate(model.projections())}
+        layer = MaskedLayer.from_weights(model, weights)
+        layer.deltas = {"qkv": 90.0, "gateup": 90.0, "o": 45.0, "down": 700.0}
+        layer.allocate_stacked(M, draws)
+        stack_layers.append(layer)
+    stack = MaskedStack(stack_layers, [91 + li for li in range(layers)])
+    inputs = [{g: (torch.zeros((M, K), device="cuda") if zero_inputs else
+                   wl.activations(M, K, seed=600 + 10 * li + gi, device="cuda"))
+               for gi, (g, K, _n) in enumerate(model.input_groups())} for li in range(layers)]
+    return stack, inputs
+
+
+@pytest.mark.parametrize("M,model", [(128, wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)),
+                                     (512, wl.LLAMA_3_2_3B)])
+def test_stacked_correction_cancels_exactly(spl, M, model):
+    """With x = 0 the mask is the noise itself, so the recovered output is fl(eta W^T) - fl(eta W^T):
+    exactly zero when the correction (computed in the previous cycle in the bank half of a product of
+    2M rows) is summed in exactly the order of the online row that meets it (the masked half of a later
+    product of the same shape) -- every element, at the bench's own sizes too."""
+    draws, eps, mech = 2, 1.0, "laplace"
+    stack, inputs = make_stacked(model, M, draws, zero_inputs=True)
+    layer, seed = stack.layers[0], stack.seeds[0]
+    for cycle in range(3):
+        for d in range(draws):
+            outs = layer.stacked_step(inputs[0], eps, mech, seed, d, cycle % 2, cycle=cycle)
+            if cycle >= 1:  # cycle 0's corrections were never computed
+                for g, y in outs.items():
+                    assert not torch.any(y).item(), (cycle, d, g, float(y.abs().max()))
+    assert spl.spl_get_device_status() == 0
+
+
+def test_stacked_graphs_equal_eager_steps(spl):
+    """Replayed stacked graphs (two layers, device-side Philox bases, the last graph of a cycle moving
+    them on) give, bit for bit, the eager stacked steps of the same cycles; any number of steps."""
+    model = wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)
+    M, draws, eps, mech = 128, 3, 1.0, "gaussian"
+    stack, inputs = make_stacked(model, M, draws, layers=2)
+    expected = {}
+    for cycle in range(4):
+        for d in range(draws):
+            for li, layer in enumerate(stack.layers):
+                outs = layer.stacked_step(inputs[li], eps, mech, stack.seeds[li], d, cycle % 2, cycle=cycle)
+                expected[(cycle * draws + d, li)] = {g: y.clone() for g, y in outs.items()}
+    torch.cuda.synchronize()
+    graphs, launches = stack.capture_stacked(inputs, eps, mech)
+    assert all(n > 0 for p in launches for n in p)
+    stack.start_stacked(2, graphs)  # runs cycle 1's graphs: cycle 2's corrections, bases at cycle 2
+    for s in range(2 * draws, 4 * draws - 1):  # stop one short of a whole cycle: any step count works
+        graphs[(s // draws) % 2][s % draws].replay()
+        torch.cuda.synchronize()
+        cycle, d = divmod(s, draws)
+        for li, layer in enumerate(stack.layers):
+            for g in layer.groups:
+                y = layer.stacked[g.name]["out"][1 - cycle % 2][d][:M]
+                assert torch.equal(y, expected[(s, li)][g.name]), (s, li, g.name)
+    assert spl.spl_get_device_status() == 0
