@@ -150,6 +150,21 @@ spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* 
                                 int64_t rows, int64_t cols, double sensitivity, double eps, spl_mech mech,
                                 spl_rng rng, cudaStream_t stream);
 
+/* The left operand of spl_masked_linear_unmask_precompute in one pass: rows
+ * 0..x_rows-1 of hi / lo / row_exp get the split of fl32(X + eta), eta drawn
+ * as spl_noise_mask_split draws it for X (block offset rng.offset, rows from
+ * 0); rows x_rows..x_rows+noise_rows-1 get the split of noise alone, drawn as
+ * spl_noise_mask_split with X NULL would draw noise_rows rows at block offset
+ * rng.offset + noise_block_delta (e.g. the same draw of the next bank cycle).
+ * Bit for bit the two separate calls, in one launch.  X [x_rows, cols];
+ * hi, lo [x_rows + noise_rows, cols], row_exp [x_rows + noise_rows].  Errors
+ * as spl_noise_mask_split (EINVAL for NULL X with x_rows > 0 or negative
+ * counts). */
+spl_status spl_noise_mask_split_stacked(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,
+                                        int64_t x_rows, int64_t noise_rows, int64_t cols, double sensitivity,
+                                        double eps, spl_mech mech, spl_rng rng, uint64_t noise_block_delta,
+                                        cudaStream_t stream);
+
 /* ---- a3 with a stored noise, fused with the fp16 split of X~ -------------
  * Xt = fl32(X + N) elementwise (Sec. 3.3.1, the mask with a noise drawn earlier,
  * e.g. written by spl_noise_mask_split with X NULL while a bank of corrections

@@ -284,13 +284,16 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
                                                                    const float* __restrict__ src, int64_t cols,
                                                                    float* __restrict__ xt_out, float b, const __grid_constant__ PhiloxKey key,
                                                                    uint64_t offset_host, const uint64_t* offset_dev,
-                                                                   const float* __restrict__ stored) {
+                                                                   const float* __restrict__ stored, int64_t x_rows,
+                                                                   uint64_t noise_delta) {
   pdl_wait();
   pdl_trigger();
   __shared__ float warp_max[kThreads / 32];
   const int64_t r = blockIdx.x;
-  // src NULL (with a mechanism): the row is the noise alone
-  const float4* row = src ? reinterpret_cast<const float4*>(src + r * cols) : nullptr;
+  // rows from x_rows on (and every row when src is NULL, with a mechanism) are the noise alone,
+  // drawn noise_delta Philox blocks further on, their counters starting again at row x_rows
+  const bool own = r < x_rows;
+  const float4* row = (src && own) ? reinterpret_cast<const float4*>(src + r * cols) : nullptr;
   const int64_t n8 = cols >> 3;
   float4 v[2 * CH];
 #pragma unroll
@@ -318,8 +321,9 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
       }
     }
   } else if constexpr (MECH != kNoMask) {
-    const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull);
-    const uint64_t j0 = (uint64_t)((r * cols) >> 2) + offset;  // cols % 8 == 0: rows start on a block
+    const uint64_t offset = offset_host + (offset_dev ? *offset_dev : 0ull) + (own ? 0ull : noise_delta);
+    const int64_t rr = own ? r : r - x_rows;
+    const uint64_t j0 = (uint64_t)((rr * cols) >> 2) + offset;  // cols % 8 == 0: rows start on a block
 #pragma unroll
     for (int c = 0; c < CH; ++c) {
       const int64_t i = threadIdx.x + (int64_t)c * kThreads;
@@ -404,23 +408,24 @@ spl_status validate_noise(int64_t rows, int64_t cols, double sensitivity, double
 template <int MECH>
 spl_status launch_split_rows(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* src, int64_t rows,
                              int64_t cols, float* xt_out, float b, const spl_rng& rng, cudaStream_t stream,
-                             const float* stored = nullptr) {
+                             const float* stored = nullptr, int64_t x_rows = -1, uint64_t noise_delta = 0) {
+  if (x_rows < 0) x_rows = rows;
   const int64_t per_thread = ceil_div(cols >> 3, kThreads);  // chunks of 8 per thread
   const dim3 grid((unsigned)rows), block(kThreads);
   const PhiloxKey key = make_philox_key(rng.seed, rng.stream_id);
   if (per_thread <= 1)
     return launch_pdl(split_fp16_regs_kernel<1, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev, stored);
+                      key, rng.offset, rng.offset_dev, stored, x_rows, noise_delta);
   if (per_thread <= 2)
     return launch_pdl(split_fp16_regs_kernel<2, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev, stored);
+                      key, rng.offset, rng.offset_dev, stored, x_rows, noise_delta);
   if (per_thread <= 4)
     return launch_pdl(split_fp16_regs_kernel<4, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev, stored);
+                      key, rng.offset, rng.offset_dev, stored, x_rows, noise_delta);
   if (per_thread <= 8)
     return launch_pdl(split_fp16_regs_kernel<8, MECH>, grid, block, 0, stream, hi, lo, row_exp, src, cols, xt_out, b,
-                      key, rng.offset, rng.offset_dev, stored);
-  if (MECH != kNoMask) return SPL_ESHAPE;
+                      key, rng.offset, rng.offset_dev, stored, x_rows, noise_delta);
+  if (MECH != kNoMask || x_rows != rows) return SPL_ESHAPE;
   return launch_pdl(split_fp16_kernel, grid, block, 0, stream, hi, lo, row_exp, src, cols);
 }
 
@@ -544,6 +549,31 @@ extern "C" spl_status spl_noise_mask_split(float* Xt, uint16_t* hi, uint16_t* lo
   if (b == 0.0f) return launch_split_rows<kZero>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
   if (mech == SPL_MECH_LAPLACE) return launch_split_rows<kLaplace>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
   return launch_split_rows<kGaussian>(hi, lo, row_exp, X, rows, cols, Xt, b, rng, stream);
+}
+
+extern "C" spl_status spl_noise_mask_split_stacked(uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,
+                                                   int64_t x_rows, int64_t noise_rows, int64_t cols,
+                                                   double sensitivity, double eps, spl_mech mech, spl_rng rng,
+                                                   uint64_t noise_block_delta, cudaStream_t stream) {
+  spl_status st = validate_noise(x_rows, cols, sensitivity, eps, mech);
+  if (st != SPL_OK) return st;
+  if (noise_rows < 0) return SPL_EINVAL;
+  const int64_t rows = x_rows + noise_rows;
+  if (rows == 0 || cols == 0) return SPL_OK;
+  if (!hi || !lo || !row_exp || (x_rows > 0 && !X)) return SPL_EINVAL;
+  if ((cols & 7) != 0) return SPL_EALIGN;
+  if ((X && !aligned16(X)) || !aligned16(hi) || !aligned16(lo)) return SPL_EALIGN;
+  if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
+  if (rows > 0x7fffffffLL) return SPL_ESHAPE;
+  const float b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
+  if (b == 0.0f)
+    return launch_split_rows<kZero>(hi, lo, row_exp, X, rows, cols, nullptr, b, rng, stream, nullptr, x_rows,
+                                    noise_block_delta);
+  if (mech == SPL_MECH_LAPLACE)
+    return launch_split_rows<kLaplace>(hi, lo, row_exp, X, rows, cols, nullptr, b, rng, stream, nullptr, x_rows,
+                                       noise_block_delta);
+  return launch_split_rows<kGaussian>(hi, lo, row_exp, X, rows, cols, nullptr, b, rng, stream, nullptr, x_rows,
+                                      noise_block_delta);
 }
 
 extern "C" spl_status spl_mask_split(float* Xt, uint16_t* hi, uint16_t* lo, int32_t* row_exp, const float* X,

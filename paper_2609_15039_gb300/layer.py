@@ -229,11 +229,10 @@ class MaskedLayer:
             off, off_dev = self._offset(gi, g, cycle, d, device_base)
             off_next = off + D * (M * g.K // 4)  # draw d of the next cycle
             delta = self.deltas[g.name]
-            if st["fused"]:
-                spl.spl_noise_mask_split(None, a.f16_hi[:M], a.f16_lo[:M], a.f16_exp[:M], inputs[g.name], delta, eps,
-                                         mech, seed, stream_id=gi, offset=off, stream=stream, offset_dev=off_dev)
-                spl.spl_noise_mask_split(None, a.f16_hi[M:], a.f16_lo[M:], a.f16_exp[M:], None, delta, eps, mech,
-                                         seed, stream_id=gi, offset=off_next, stream=stream, offset_dev=off_dev)
+            if st["fused"]:  # both halves of the left operand in one launch
+                spl.spl_noise_mask_split_stacked(a.f16_hi, a.f16_lo, a.f16_exp, inputs[g.name], delta, eps, mech, seed,
+                                                 M, off_next - off, stream_id=gi, offset=off, stream=stream,
+                                                 offset_dev=off_dev)
             else:
                 spl.spl_noise_mask(a.w[:M], None, inputs[g.name], delta, eps, mech, seed, stream_id=gi, offset=off,
                                    stream=stream, offset_dev=off_dev)

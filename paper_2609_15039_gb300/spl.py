@@ -62,6 +62,8 @@ _SIGS = {
     "spl_split_tf32": (_I, [_P, _P, _P, _I64, _P]),
     "spl_noise_mask_split": (_I, [_P, _P, _P, _P, _P, _I64, _I64, _D, _D, _I, spl_rng, _P]),
     "spl_mask_split": (_I, [_P, _P, _P, _P, _P, _P, _I64, _I64, _P]),
+    "spl_noise_mask_split_stacked": (_I, [_P, _P, _P, _P, _I64, _I64, _I64, _D, _D, _I, spl_rng, ctypes.c_uint64,
+                                          _P]),
     "spl_masked_linear_unmask_split": (_I, [_P, _PW, _PW, _P, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_split_fp16": (_I, [_P, _P, _P, _P, _I64, _I64, _P]),
     "spl_resolve_path": (_I, [_I64, _I64, _I64, _I]),
@@ -257,6 +259,21 @@ def spl_noise_mask_split(Xt, hi, lo, row_exp, X, sensitivity, eps, mech, seed, s
                                       float(sensitivity), _eps(eps), _mech(mech),
                                       _rng(seed, stream_id, offset, offset_dev), _stream(stream)),
            "spl_noise_mask_split")
+
+
+def spl_noise_mask_split_stacked(hi, lo, row_exp, X, sensitivity, eps, mech, seed, noise_rows, noise_block_delta,
+                                 stream_id=0, offset=0, stream=None, offset_dev=None):
+    """Split of [X + eta; eta'] in one pass: rows of X masked and split, then noise_rows rows of noise
+    alone drawn noise_block_delta Philox blocks further on (see include/spl.h)."""
+    x_rows, cols = _rows_cols(X)
+    rows = x_rows + int(noise_rows)
+    if hi.numel() != rows * cols or lo.numel() != rows * cols or row_exp.numel() != rows:
+        raise ValueError("spl_noise_mask_split_stacked: shape mismatch")
+    _check(lib().spl_noise_mask_split_stacked(_dev(hi, "hi", torch.int16), _dev(lo, "lo", torch.int16),
+                                              _dev(row_exp, "row_exp", torch.int32), _dev(X, "X"), x_rows,
+                                              int(noise_rows), cols, float(sensitivity), _eps(eps), _mech(mech),
+                                              _rng(seed, stream_id, offset, offset_dev), int(noise_block_delta),
+                                              _stream(stream)), "spl_noise_mask_split_stacked")
 
 
 def spl_mask_split(Xt, hi, lo, row_exp, X, N, stream=None):

@@ -106,6 +106,11 @@ def test_argument_validation_without_launch(spl):
     assert L.spl_mask_split(None, base, base, base, base, base, 1, 16392, None) == spl.SPL_ESHAPE  # row too long
     assert L.spl_noise_mask_split(None, base, base, base, base, 2, 12, 1.0, 1.0, 0, rng, None) == spl.SPL_EALIGN
     assert L.spl_noise_mask_split(None, None, base, base, base, 2, 8, 1.0, 1.0, 0, rng, None) == spl.SPL_EINVAL
+    # the stacked split: negative counts, a missing X for masked rows, cols % 8
+    assert L.spl_noise_mask_split_stacked(base, base, base, base, 2, -1, 8, 1.0, 1.0, 0, rng, 0, None) == spl.SPL_EINVAL
+    assert L.spl_noise_mask_split_stacked(base, base, base, None, 2, 2, 8, 1.0, 1.0, 0, rng, 0, None) == spl.SPL_EINVAL
+    assert L.spl_noise_mask_split_stacked(base, base, base, base, 2, 2, 12, 1.0, 1.0, 0, rng, 0, None) == spl.SPL_EALIGN
+    assert L.spl_noise_mask_split_stacked(None, None, None, None, 0, 0, 8, 1.0, 1.0, 0, rng, 0, None) == spl.SPL_OK
     # the tensor-core test hook refuses a persistent launch that breaks its conditions
     w16 = spl.spl_weight(base, None, None, base, base, base)
     for splits, seg, full in ((2, 0, 0), (1, 2, 0), (1, 0, 1)):

@@ -583,6 +583,31 @@ def test_noise_mask_split_equals_separate_calls(spl, rows, cols, mech, eps):
     assert torch.equal(hi, hi_ref) and torch.equal(ex, ex_ref)
 
 
+@pytest.mark.parametrize("x_rows,noise_rows,cols,mech,eps", [(512, 512, 3072, "laplace", 1.0), (5, 3, 8, "gaussian", 0.5),
+                                                               (3, 7, 16384, "laplace", 2.0), (0, 4, 1032, "gaussian", 1.0),
+                                                               (6, 0, 1032, "laplace", None)])
+def test_stacked_split_equals_two_calls(spl, x_rows, noise_rows, cols, mech, eps):
+    """The left operand of the stacked product in one launch is, bit for bit, the mask + split of X's
+    rows and the split of the noise rows drawn further on, as two separate calls make them."""
+    eps = float("inf") if eps is None else eps
+    X = dev(wl.activations(x_rows, cols, seed=x_rows + cols + 1).numpy())
+    rows = x_rows + noise_rows
+    base = torch.tensor([777], dtype=torch.int64, device="cuda")
+    delta = 8 * 512 * cols // 4
+    hi_ref = torch.zeros((rows, cols), dtype=torch.int16, device="cuda")
+    lo_ref, ex_ref = torch.zeros_like(hi_ref), torch.zeros(rows, dtype=torch.int32, device="cuda")
+    if x_rows:
+        spl.spl_noise_mask_split(None, hi_ref[:x_rows], lo_ref[:x_rows], ex_ref[:x_rows], X, 825.3, eps, mech, seed=5,
+                                 stream_id=1, offset=13, offset_dev=base)
+    if noise_rows:
+        spl.spl_noise_mask_split(None, hi_ref[x_rows:], lo_ref[x_rows:], ex_ref[x_rows:], None, 825.3, eps, mech,
+                                 seed=5, stream_id=1, offset=13 + delta, offset_dev=base)
+    hi, lo, ex = torch.full_like(hi_ref, 7), torch.full_like(lo_ref, 7), torch.full_like(ex_ref, 7)
+    spl.spl_noise_mask_split_stacked(hi, lo, ex, X, 825.3, eps, mech, 5, noise_rows, delta, stream_id=1, offset=13,
+                                     offset_dev=base)
+    assert torch.equal(hi, hi_ref) and torch.equal(lo, lo_ref) and torch.equal(ex, ex_ref)
+
+
 @pytest.mark.parametrize("rows,cols,mech", [(5, 8, "laplace"), (130, 3072, "gaussian"), (3, 16384, "laplace")])
 def test_mask_split_with_stored_noise_equals_drawn(spl, rows, cols, mech):
     """The mask with a noise drawn earlier (as a bank refill keeps it) gives the X~ and the fp16
