@@ -748,7 +748,7 @@ def run_llama_stack(args):
                              "layers) per second of the whole step: the prefill with its correction work"),
                    "bank_schedule": schedule_note,
                    "online_noise": "drawn again in each step's mask from the bank's Philox counters",
-                   "l2": (f"weights {L * sum(g.K * g.N for g in groups) * 14 / 1e9:.1f} GB per step (fp32 + their "
+                   "l2": (f"weights {L * sum(g.K * g.N for g in groups) * 16 / 1e9:.1f} GB per step (fp32 + their "
                           "TF32 and fp16 splits) > 129 MB L2 (no flush needed)"),
                    "parallelism": "replicas" if world > 1 else "single", "setup_s": build_s},
         "prefill": {"ms_per_prefill_with_correction": ms, "tokens_per_s": M / (ms * 1e-3),
