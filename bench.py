@@ -12,7 +12,7 @@ reads), runs the masked products with the unmask fused into their epilogues
 and each of the 8 steps of a cycle computes the next cycle's banks of an
 eighth of the layers on a lower-priority stream beside its own prefill.  So
 any number of steps times the whole method: prefill plus its correction.
-The weights (40 GB with their splits) are far larger than L2.
+The weights (45 GB with their splits) are far larger than L2.
 
 Also reported on the same stack: the online prefill alone, the bank refill
 alone, the product kernels per launch (the roofline), decode at one token per
