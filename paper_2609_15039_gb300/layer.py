@@ -720,39 +720,37 @@ class MaskedStack:
         correction of draw d -- and graph d = draws - 1 moves every Philox base on by one cycle.  After
         start_stacked(c), replay graphs[(s // draws) % 2][s % draws] for steps s = c draws, ...: any
         number of them, each one step of the method with its share of the bank.  ``timer(d, li, phase,
-        kind, group)`` as in capture.  ``copies``: (h2d, d2h) host-transfer hooks -- h2d(li) is called on
-        a host-to-device copy stream before the steps, once per layer in order, and returns an event
-        that layer li waits for; d2h(li, outs) on a device-to-host copy stream after layer li's calls
-        (which that stream waits for first), outs being the layer's {group: Y}.  Returns the graphs and
-        their kernel counts."""
+        kind, group)`` as in capture.  ``inputs``: the per-layer input dicts, or a pair of them (step d
+        then reads inputs[d % 2]; draws is even, so consecutive steps alternate).  ``copies``:
+        (prefetch(d), drain(p, d)) host-transfer hooks called at the start of graph (p, d), each on a
+        copy stream of its own that the step joins at its end -- prefetch enqueues the next step's input
+        copies (into the other input set), drain the copies of the previous step's outputs (see
+        step_outputs).  Returns the graphs and their kernel counts."""
         if copies is not None and not hasattr(self, "_h2d_stream"):
             _, hi = torch.cuda.Stream.priority_range()
             self._h2d_stream = torch.cuda.Stream(priority=hi)
             self._d2h_stream = torch.cuda.Stream(priority=hi)
+        paired = isinstance(inputs, (list, tuple)) and len(inputs) == 2 and isinstance(inputs[0], (list, tuple))
         D = self.draws
         graphs, launches = [[], []], [[], []]
         for parity in range(2):
             for d in range(D):
                 graph = torch.cuda.CUDAGraph()
                 n0 = spl.spl_launch_count()
+                step_inputs = inputs[d % 2] if paired else inputs
                 with torch.cuda.graph(graph):
                     main = torch.cuda.current_stream()
-                    ready = []
                     if copies is not None:
                         self._h2d_stream.wait_stream(main)
                         with torch.cuda.stream(self._h2d_stream):
-                            ready = [copies[0](li) for li in range(len(self.layers))]
+                            copies[0](d)
                         self._d2h_stream.wait_stream(main)
-                    for li, (layer, x, seed) in enumerate(zip(self.layers, inputs, self.seeds)):
-                        if ready:
-                            main.wait_event(ready[li])
+                        with torch.cuda.stream(self._d2h_stream):
+                            copies[1](parity, d)
+                    for li, (layer, x, seed) in enumerate(zip(self.layers, step_inputs, self.seeds)):
                         t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
                             if timer else None
-                        outs = layer.stacked_step(x, eps, mech, seed, d, parity, path=path, timer=t, device_base=True)
-                        if copies is not None:
-                            self._d2h_stream.wait_stream(main)
-                            with torch.cuda.stream(self._d2h_stream):
-                                copies[1](li, outs)
+                        layer.stacked_step(x, eps, mech, seed, d, parity, path=path, timer=t, device_base=True)
                     if copies is not None:
                         main.wait_stream(self._h2d_stream)
                         main.wait_stream(self._d2h_stream)
@@ -763,6 +761,15 @@ class MaskedStack:
                 graphs[parity].append(graph)
                 launches[parity].append(spl.spl_launch_count() - n0)
         return graphs, launches
+
+    def step_outputs(self, parity, d):
+        """The outputs of step d of a cycle of parity ``parity`` (stacked schedule): per layer {group: Y}."""
+        return [{g.name: layer.stacked[g.name]["out"][1 - parity][d][:layer.M] for g in layer.groups}
+                for layer in self.layers]
+
+    def previous_step(self, parity, d):
+        """(parity, draw) of the step before step d of a cycle of parity ``parity``."""
+        return (parity, d - 1) if d > 0 else (1 - parity, self.draws - 1)
 
     def start_stacked(self, cycle, graphs):
         """Before replaying the stacked graphs from cycle ``cycle``: run cycle ``cycle - 1``'s graphs once

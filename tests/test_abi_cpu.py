@@ -143,6 +143,28 @@ def test_listed_boundary_names(spl):
     assert L.spl_prepare_weight_split(base, base, base, 1 << 40, 1 << 40, None) == spl.SPL_ESHAPE
 
 
+def test_precompute_and_swap_entries_validate_without_launch(spl):
+    """The stacked product entry and the swapped-kernel hook refuse bad arguments before launching."""
+    L = spl.lib()
+    buf = (ctypes.c_float * 64)()
+    p = ctypes.cast(buf, ctypes.c_void_p).value
+    base = p + (16 - p % 16) % 16
+    w = spl.spl_weight(base, None, None, None, None, None)
+    a = spl.spl_weight(base, None, None, None, None, None)
+    pre = L.spl_masked_linear_unmask_precompute
+    assert pre(base, None, ctypes.byref(w), base, 2, 2, 8, 4, 0, None, 0, None) == spl.SPL_EINVAL   # no A
+    assert pre(base, ctypes.byref(a), ctypes.byref(w), base, -1, 2, 8, 4, 0, None, 0, None) == spl.SPL_EINVAL
+    assert pre(base, ctypes.byref(a), ctypes.byref(w), None, 2, 2, 8, 4, 0, None, 0, None) == spl.SPL_EINVAL  # C
+    assert pre(base, ctypes.byref(a), ctypes.byref(w), None, 0, 0, 8, 4, 0, None, 0, None) == spl.SPL_OK      # empty
+    # no tensor-core device here, so AUTO resolves to FP32, which has no row limit on C
+    assert pre(base, ctypes.byref(a), ctypes.byref(w), base, 2, 2, 8, 4, 0, None, 0, None) == spl.SPL_EUNSUPPORTED
+    swap = L.spl_test_tc_swap_product
+    assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 24, 1, None, 0, None) == spl.SPL_EINVAL  # width
+    assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 16, 9, None, 0, None) == spl.SPL_ESHAPE  # splits
+    assert swap(base, base, ctypes.byref(w), None, 2, 12, 4, 16, 1, None, 0, None) == spl.SPL_EALIGN  # K % 8
+    assert swap(base, base, None, None, 2, 8, 4, 16, 1, None, 0, None) == spl.SPL_EINVAL
+
+
 def test_workspace_sizes_are_consistent(spl):
     # decode shapes need split-K partials after the 64 KiB counter region; the tensor-core
     # kernels reduce split-K in a cluster and keep only the split of the left operand there

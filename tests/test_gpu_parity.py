@@ -309,6 +309,35 @@ def test_library_takes_the_swapped_kernel_for_few_rows(spl):
     assert spl.spl_get_device_status() == 0
 
 
+@pytest.mark.parametrize("path", ["fp16x3", "tf32x3"])
+@pytest.mark.parametrize("M,M_bank,K,N", [(128, 128, 3072, 5120), (130, 70, 1032, 600), (0, 40, 264, 300),
+                                          (40, 0, 264, 300), (12, 12, 2056, 700)])
+def test_precompute_beside_masked_rows(spl, path, M, M_bank, K, N):
+    """spl_masked_linear_unmask_precompute: the first M output rows are the masked product with its unmask,
+    the others the corrections of the noise rows, each within the product tolerance of the oracle, and
+    every row summed as the same row of a plain product of M + M_bank rows (bit for bit: launch forms
+    are uniform over the rows)."""
+    W, Wt = _weights(spl, N, K, seed=K + N + 5)
+    rows = M + M_bank
+    A = (wl.activations(rows, K, seed=rows + 3).numpy() * 300).astype(np.float32)
+    C = wl.activations(M, N, seed=9).numpy()
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(rows, K, N, path))
+    YC = torch.full((rows, N), float("nan"), device="cuda")
+    spl.spl_masked_linear_unmask_precompute(YC, dev(A), Wt, dev(C) if M else None, M, path=path, workspace=ws)
+    if M:
+        assert_product_close(f32(YC[:M]), A[:M], W, path, C=C, what="masked rows")
+    if M_bank:
+        assert_product_close(f32(YC[M:]), A[M:], W, path, what="correction rows")
+    P = torch.empty((rows, N), device="cuda")
+    spl.spl_masked_linear(P, dev(A), Wt, path=path, workspace=ws)
+    assert torch.equal(YC[M:], P[M:])  # the correction rows: no C subtracted, the same sums
+    if M:
+        Yu = torch.empty((M, N), device="cuda")
+        spl.spl_unmask(Yu, P[:M].contiguous(), dev(C))
+        assert torch.equal(YC[:M], Yu)  # fused unmask = the plain product then one subtraction
+    assert spl.spl_get_device_status() == 0
+
+
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 def test_products_with_extreme_row_scales(spl, path):
     """Rows of A and W spread over 60 orders of magnitude, zero rows included: the power-of-two
