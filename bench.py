@@ -705,7 +705,38 @@ def run_llama_stack(args):
 
     # ---- decode at one token per step (the same layers, banks of D one-row draws) -----------------
     decode = None
-    if not args.no_decode:
+    if not args.no_decode and stacked:
+        phase("decode (stacked)")
+        torch.cuda.synchronize()
+        ws1 = spl.workspace(max(spl.spl_linear_workspace_bytes(2, g.K, g.N, "auto") for g in groups), dev)
+        for layer in stack.layers:
+            layer.allocate_stacked(1, D, workspace=ws1)
+        del ws_on
+        torch.cuda.empty_cache()
+        inputs1 = stack.inputs(13, device=dev)
+        dgraphs, dl = stack.capture_stacked(inputs1, eps, mech)
+        dgraph_of = lambda s: dgraphs[(s // D) % 2][s % D]
+        steps = max(D, args.decode_steps)
+        stack.start_stacked(1, dgraphs)
+        _time_graphs(dgraph_of, D, 2 * D, stream)  # cycles 1 and 2
+        times = _time_graphs(dgraph_of, 3 * D, steps, stream)
+        step_ms = sum(times) / steps
+        dpaths = {g.name: layer0.stacked[g.name]["path"] for g in groups}
+        step_bytes = sum(4 * g.K * g.N + 12 * g.K + 12 * g.N for g in groups) * L
+        decode = {"steps": steps, "ms_per_token": step_ms, "tokens_per_s": 1e3 / step_ms,
+                  "gbs": step_bytes / (step_ms * 1e-3) / 1e9, "peak_gbs": pk["hbm_gbs"],
+                  "frac": step_bytes / (step_ms * 1e-3) / 1e9 / pk["hbm_gbs"], "bytes_per_step": step_bytes,
+                  "paths": dpaths, "kernels_per_step": sum(sum(p) for p in dl) / (2 * D),
+                  "fused_one_launch": all(layer0.stacked[g.name]["fused_mask"] for g in groups),
+                  "schedule": ("stacked, one graph per token: every group's call draws the token's noise and the "
+                               "next cycle's same-draw noise row, masks and multiplies both rows in one launch "
+                               "of the decode kernel (bytes per step: every weight once, the token's x, C and Y, "
+                               "both rows of x~ and the new correction)")}
+        del dgraphs
+        st = spl.spl_get_device_status()
+        if st != spl.SPL_OK:
+            raise RuntimeError("device status " + spl.status_string(st))
+    elif not args.no_decode:
         phase("decode")
         torch.cuda.synchronize()
         ws1 = spl.workspace(max(l.workspace_bytes(1, D) for l in stack.layers), dev)

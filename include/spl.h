@@ -385,12 +385,34 @@ spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt, const flo
  * rows of each column of tiles), so a correction computed here is summed
  * exactly as the masked row that later meets it in a call with the same
  * M + M_bank, K, N and path: their rounding errors cancel in the unmask.
- * Tensor-core paths only (TF32X3 / FP16X3, resolved as for M + M_bank rows);
- * EUNSUPPORTED for a path that resolves to FP32.  Workspace and other errors
- * as spl_masked_linear_unmask for M + M_bank rows. */
+ * Runs on the tensor-core paths (TF32X3 / FP16X3, resolved as for M + M_bank
+ * rows) and, for M + M_bank <= 16 rows on FP32, on the decode kernel;
+ * EUNSUPPORTED for FP32 beyond 16 rows.  Workspace and other errors as
+ * spl_masked_linear_unmask for M + M_bank rows. */
 spl_status spl_masked_linear_unmask_precompute(float* YC, const spl_weight* A, const spl_weight* W, const float* C,
                                                int64_t M, int64_t M_bank, int64_t K, int64_t N, spl_path path,
                                                void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* ---- a2 + a3 + a4 + a5 + a6 in one decode launch: the stacked schedule ------
+ * spl_noise_mask_linear_unmask and spl_masked_linear_unmask_precompute in one:
+ * the left operand has M + M_bank rows, rows 0..M-1 being X~ = fl32(X + eta)
+ * with eta drawn as spl_noise_mask draws it for X (rows from 0, block offset
+ * rng.offset), rows M.. noise alone, drawn as spl_noise_mask with X NULL would
+ * draw M_bank rows at block offset rng.offset + noise_block_delta (the same
+ * draw of the next bank cycle, Sec. 5.2).  Xt [M + M_bank, K] receives that
+ * operand; YC [M + M_bank, N]: rows 0..M-1 get Y = fl32(fl32(Xt W^T) - C)
+ * with C [M, N] (Eq. add-and-then-subtract), rows M.. the corrections
+ * fl32(eta W^T).  Every row is summed in the same order, so a correction made
+ * here cancels the masked row that meets it in a later call of the same
+ * shape exactly as spl_masked_linear_unmask_precompute's do.  One launch of
+ * the FP32 decode kernel: 1 <= M + M_bank <= 4 and a path resolving to FP32
+ * (AUTO does there), else EUNSUPPORTED.  X may be NULL when M = 0 and must
+ * not overlap Xt (EINVAL).  Other errors as spl_noise_mask_linear_unmask. */
+spl_status spl_noise_mask_linear_unmask_precompute(float* YC, float* Xt, const float* X, const spl_weight* W,
+                                                   const float* C, int64_t M, int64_t M_bank, int64_t K, int64_t N,
+                                                   double sensitivity, double eps, spl_mech mech, spl_rng rng,
+                                                   uint64_t noise_block_delta, spl_path path, void* workspace,
+                                                   size_t workspace_bytes, cudaStream_t stream);
 
 /* ---- a8: the cancellation bound on the GPU, and the path choice ----------
  * The paper judges a configuration by evaluating its floating-point bound on

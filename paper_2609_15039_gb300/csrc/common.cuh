@@ -80,7 +80,7 @@ struct LinearArgs {
   const uint16_t* a_h16;    // [M, K]  fp16 split of a, made by the caller (FP16X3), or null
   const uint16_t* a_l16;
   const int32_t* a_exp;     // [M]
-  int64_t c_rows;           // rows of c: output rows from c_rows on subtract nothing (tensor-core kernels)
+  int64_t c_rows;           // rows of c: output rows from c_rows on subtract nothing (tensor-core and decode kernels)
 };
 
 // Workspace layout shared by every product call: the first kCounterBytes hold
@@ -150,6 +150,8 @@ struct MaskNoise {
   uint64_t seed, stream_id;    // Philox key, counter words 2-3
   uint64_t offset;             // Philox block offset (host part)
   const uint64_t* offset_dev;  // device part of the offset (may be null)
+  int64_t x_rows = -1;         // rows from x_rows on are noise alone (no X), drawn noise_delta blocks
+  uint64_t noise_delta = 0;    // further on with their counters starting again at row x_rows (-1: all rows X)
 };
 constexpr int kGemvMaskMaxM = 4;  // rows up to which every block draws its slice's noise itself
 spl_status run_gemv_masked(const LinearArgs& a, const Plan& p, const MaskNoise& nz);

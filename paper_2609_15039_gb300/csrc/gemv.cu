@@ -112,13 +112,16 @@ struct KernelNoise {
   PhiloxKey key;
   uint64_t offset;
   const uint64_t* offset_dev;
+  int x_rows;        // rows from x_rows on: noise alone, drawn delta blocks further on, counters from row x_rows
+  uint64_t delta;
 };
 
 template <int MT, int MASK>
 __global__ void __launch_bounds__(THREADS)
 gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* __restrict__ W,
             const float* __restrict__ C, float* __restrict__ part, unsigned int* __restrict__ counters, int M,
-            int64_t K, int64_t N, int ks, int splits, int prefetch_lines, const __grid_constant__ KernelNoise nz) {
+            int64_t K, int64_t N, int ks, int splits, int prefetch_lines, const __grid_constant__ KernelNoise nz,
+            int c_rows) {
   constexpr int RQ = rows_per_lane(MT), RB = rows_per_block(MT), U = unroll_steps(MT);
   constexpr int V = RQ * MT;
   extern __shared__ __align__(16) float4 xs[];  // [MT][ks / 4]
@@ -164,9 +167,11 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
   auto x4 = [&](int m, int q, float4* dst_out) -> float4 {
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
     if (m < M && q < q_len) {
-      v = __ldg(reinterpret_cast<const float4*>(X + (int64_t)m * K + k0) + q);
+      const bool own = MASK == kNoMask || m < nz.x_rows;  // a row of X (else noise alone)
+      if (own) v = __ldg(reinterpret_cast<const float4*>(X + (int64_t)m * K + k0) + q);
       if constexpr (MASK != kNoMask) {
-        const uint64_t j = (uint64_t)(((int64_t)m * K + k0) >> 2) + (uint64_t)q + nz.offset +
+        const int64_t mr = own ? m : m - nz.x_rows;
+        const uint64_t j = (uint64_t)((mr * K + k0) >> 2) + (uint64_t)q + nz.offset + (own ? 0ull : nz.delta) +
                            (nz.offset_dev ? *nz.offset_dev : 0ull);
         v = add4(v, draw_block<MASK>(j, nz.key, nz.b));
         if (dst_out) __stcs(dst_out, v);
@@ -203,13 +208,16 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
     const bool write_xt = blockIdx.x == 0;
 #pragma unroll
     for (int m = 0; m < MT; ++m) {
-      const float4* src = reinterpret_cast<const float4*>(X + (int64_t)m * K + k0);
+      const bool own = m < nz.x_rows;  // a row of X (else noise alone, delta blocks further on)
+      const float4* src = reinterpret_cast<const float4*>(X + (int64_t)(own ? m : 0) * K + k0);
       float4* dst = reinterpret_cast<float4*>(nz.xt + (int64_t)m * K + k0);
-      const uint64_t j0 = (uint64_t)(((int64_t)m * K + k0) >> 2) + off;
+      const int64_t mr = own ? m : m - nz.x_rows;
+      const uint64_t j0 = (uint64_t)((mr * K + k0) >> 2) + off + (own ? 0ull : nz.delta);
       for (int q = threadIdx.x; q < q_row; q += THREADS) {
         float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
         if (m < M && q < q_len) {
-          v = add4(__ldg(src + q), draw_block<MASK>(j0 + (uint64_t)q, nz.key, nz.b));
+          const float4 e = draw_block<MASK>(j0 + (uint64_t)q, nz.key, nz.b);
+          v = own ? add4(__ldg(src + q), e) : e;
           if (write_xt) __stcs(dst + q, v);
         }
         xs[m * q_row + q] = v;
@@ -328,7 +336,7 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
         const int64_t n = row0 + 4 * r;
         if (m < M && n < N) {
           const int64_t o = (int64_t)m * N + n;
-          out[o] = C ? __fsub_rn(acc[i], C[o]) : acc[i];
+          out[o] = (C && m < c_rows) ? __fsub_rn(acc[i], C[o]) : acc[i];
         }
       }
     }
@@ -361,7 +369,7 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
     const int64_t o = (int64_t)m * N + n;
     float s = __ldcg(part + o);
     for (int sp = 1; sp < splits; ++sp) s = __fadd_rn(s, __ldcg(part + (int64_t)sp * M * N + o));
-    out[o] = C ? __fsub_rn(s, C[o]) : s;
+    out[o] = (C && m < c_rows) ? __fsub_rn(s, C[o]) : s;
   }
   if (threadIdx.x == 0) counters[blockIdx.x] = 0u;
 }
@@ -413,7 +421,7 @@ spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int*
   const int64_t rows = (int64_t)grid.x * rows_per_block(MT) * p.splits;
   const int lines = (int)std::min<int64_t>(p.k_per_split / kStep, ((int64_t(32) << 20) / std::max<int64_t>(rows, 1)) >> 7);
   return launch_pdl(gemv_kernel<MT, MASK>, grid, dim3(THREADS), smem, a.stream, a.out, a.a, a.w, a.c, part, counters,
-                    (int)a.M, a.K, a.N, (int)p.k_per_split, p.splits, lines, nz);
+                    (int)a.M, a.K, a.N, (int)p.k_per_split, p.splits, lines, nz, (int)a.c_rows);
 }
 
 template <int MASK>
@@ -510,6 +518,8 @@ spl_status run_gemv_masked(const LinearArgs& a, const Plan& p, const MaskNoise& 
   kn.key = make_philox_key(nz.seed, nz.stream_id);
   kn.offset = nz.offset;
   kn.offset_dev = nz.offset_dev;
+  kn.x_rows = nz.x_rows < 0 ? (int)a.M : (int)nz.x_rows;
+  kn.delta = nz.noise_delta;
   if (nz.b == 0.0f) return launch_masked<kZero>(a, p, part, counters, kn);
   if (nz.mech == SPL_MECH_LAPLACE) return launch_masked<kLaplace>(a, p, part, counters, kn);
   return launch_masked<kGaussian>(a, p, part, counters, kn);
@@ -604,6 +614,7 @@ extern "C" spl_status spl_masked_linear_unmask_noalloc(float* Y, const float* Xt
   args.ws = ws;
   args.ws_bytes = kStaticScratchBytes;
   args.stream = stream;
+  args.c_rows = M;
   args.path = SPL_PATH_FP32;
   return run_gemv(args, plan);
 }

@@ -93,8 +93,8 @@ spl_status run_linear(float* out, const float* a, const spl_weight* W, const flo
   if (!use_split && plan.total() > 0 && (!ws || ws_bytes < plan.total())) return SPL_EWORKSPACE;
   if (ws && !aligned16(ws)) return SPL_EALIGN;
   LinearArgs args = make_args(out, a, *W, C, M, K, N, ws, ws_bytes, stream, resolved);
-  if (c_rows >= 0) {  // only the first c_rows output rows subtract C (the tensor-core kernels)
-    if (plan.kernel != kKernelTc) return SPL_EUNSUPPORTED;
+  if (c_rows >= 0) {  // only the first c_rows output rows subtract C (tensor-core and decode kernels)
+    if (plan.kernel != kKernelTc && plan.kernel != kKernelGemv) return SPL_EUNSUPPORTED;
     args.c_rows = c_rows;
   }
   if (use_split) {
@@ -207,11 +207,48 @@ extern "C" spl_status spl_masked_linear_unmask_precompute(float* YC, const spl_w
   if (M > 0 && !C) return SPL_EINVAL;
   if (M + M_bank > (int64_t(1) << 31)) return SPL_ESHAPE;
   if (M + M_bank == 0 || N == 0) return SPL_OK;
-  if (K > 0) {  // the tensor-core paths only: decide before anything runs
+  if (K > 0) {  // the tensor-core kernels and the decode kernel: decide before anything runs
     const spl_path resolved = resolve(M + M_bank, K, path, W && has_tf32(*W), W && has_f16(*W));
-    if (!is_tc(resolved)) return SPL_EUNSUPPORTED;
+    if (!is_tc(resolved) && M + M_bank > kGemvMaxM) return SPL_EUNSUPPORTED;
   }
   return run_linear(YC, A->w, W, C, M > 0, M + M_bank, K, N, path, workspace, workspace_bytes, stream, A, nullptr,
+                    M);
+}
+
+extern "C" spl_status spl_noise_mask_linear_unmask_precompute(float* YC, float* Xt, const float* X,
+                                                               const spl_weight* W, const float* C, int64_t M,
+                                                               int64_t M_bank, int64_t K, int64_t N,
+                                                               double sensitivity, double eps, spl_mech mech,
+                                                               spl_rng rng, uint64_t noise_block_delta,
+                                                               spl_path path, void* workspace, size_t workspace_bytes,
+                                                               cudaStream_t stream) {
+  spl_status st = validate_noise(M, K, sensitivity, eps, mech);
+  if (st != SPL_OK) return st;
+  if (M_bank < 0 || N < 0 || !valid_path(path)) return SPL_EINVAL;
+  const int64_t rows = M + M_bank;
+  if (rows == 0 || N == 0) return SPL_OK;
+  if (K > 0 && (!Xt || (M > 0 && !X) || !W)) return SPL_EINVAL;
+  if (M > 0 && !C) return SPL_EINVAL;
+  if ((Xt && !aligned16(Xt)) || (X && !aligned16(X))) return SPL_EALIGN;
+  if ((reinterpret_cast<uintptr_t>(rng.offset_dev) & 7u) != 0) return SPL_EALIGN;
+  if (K == 0 || rows > kGemvMaskMaxM || resolve(rows, K, path, has_tf32(*W), has_f16(*W)) != SPL_PATH_FP32)
+    return SPL_EUNSUPPORTED;  // one launch on the decode kernel only
+  if (X && M > 0) {  // X~ is written while other blocks still read X
+    const uintptr_t x0 = reinterpret_cast<uintptr_t>(X), t0 = reinterpret_cast<uintptr_t>(Xt);
+    const uintptr_t xb = (uintptr_t)(M * K) * sizeof(float), tb = (uintptr_t)(rows * K) * sizeof(float);
+    if (x0 < t0 + tb && t0 < x0 + xb) return SPL_EINVAL;
+  }
+  MaskNoise nz{};
+  nz.xt = Xt;
+  nz.b = std::isinf(eps) ? 0.0f : (float)(sensitivity / eps);
+  nz.mech = (int)mech;
+  nz.seed = rng.seed;
+  nz.stream_id = rng.stream_id;
+  nz.offset = rng.offset;
+  nz.offset_dev = rng.offset_dev;
+  nz.x_rows = M;
+  nz.noise_delta = noise_block_delta;
+  return run_linear(YC, X ? X : Xt, W, C, M > 0, rows, K, N, path, workspace, workspace_bytes, stream, nullptr, &nz,
                     M);
 }
 

@@ -189,10 +189,10 @@ class MaskedLayer:
         the product runs FP16X3, else fp32) and out[p][d] [2M, N] for parities p = 0, 1: a cycle of
         parity p reads its corrections from out[p][d][M:] and writes [Y; the next cycle's corrections]
         into out[1 - p][d].  A correction and the masked row that later meets it sit in products of
-        the same shape, which sum every row in the same order, so their roundings cancel."""
-        if M % 4:
-            raise ValueError("stacked schedule: M % 4 == 0 (the split's row exponents of each half are "
-                             "16-byte aligned)")
+        the same shape, which sum every row in the same order, so their roundings cancel.  When the
+        2M rows run on the FP32 decode kernel and fit its fused form (2M <= 4: decode), the noise
+        draw, the mask and the product of a step are one launch (spl_noise_mask_linear_unmask_precompute)
+        and the left operand is the fp32 X~ it writes."""
         dev = self.groups[0].W.device
         need = max(spl.spl_linear_workspace_bytes(2 * M, g.K, g.N, self.path_of(g, path, 2 * M)) for g in self.groups)
         if workspace is not None:
@@ -207,13 +207,17 @@ class MaskedLayer:
             if g.name in self.fp64:
                 raise ValueError("stacked schedule: the binary64 group keeps the separate bank")
             fused = self._fused_split(g, path, 2 * M)
+            if fused and M % 4:
+                raise ValueError("stacked schedule on FP16X3: M % 4 == 0 (the split's row exponents of each "
+                                 "half are 16-byte aligned)")
+            fused_mask = self._fused_mask(g, path, 2 * M)
             a = (spl.Weight(None, f16_hi=torch.empty((2 * M, g.K), dtype=torch.int16, device=dev),
                             f16_lo=torch.empty((2 * M, g.K), dtype=torch.int16, device=dev),
                             f16_exp=torch.empty(2 * M, dtype=torch.int32, device=dev))
                  if fused else spl.Weight(torch.empty((2 * M, g.K), device=dev)))
             out = [[torch.zeros((2 * M, g.N), device=dev) for _ in range(draws)] for _ in range(2)]
             resolved = spl.PATH_NAMES[spl.spl_resolve_path(2 * M, g.K, g.N, self.path_of(g, path, 2 * M))]
-            self.stacked[g.name] = {"a": a, "out": out, "fused": fused, "path": resolved}
+            self.stacked[g.name] = {"a": a, "out": out, "fused": fused, "fused_mask": fused_mask, "path": resolved}
 
     def stacked_step(self, inputs, eps, mech, seed, d, parity, cycle=0, path="auto", stream=None, timer=None,
                      device_base=False):
@@ -229,6 +233,18 @@ class MaskedLayer:
             off, off_dev = self._offset(gi, g, cycle, d, device_base)
             off_next = off + D * (M * g.K // 4)  # draw d of the next cycle
             delta = self.deltas[g.name]
+            res = st["out"][1 - parity][d]
+            if st["fused_mask"]:  # noise, mask and product of both halves in one decode launch
+                if timer:
+                    timer("begin", "masked_linear_unmask", g.name)
+                spl.spl_noise_mask_linear_unmask_precompute(
+                    res, a.w, inputs[g.name], g.wt, st["out"][parity][d][M:], delta, eps, mech, seed, M,
+                    off_next - off, stream_id=gi, offset=off, path=st["path"], workspace=self.workspace,
+                    stream=stream, offset_dev=off_dev)
+                if timer:
+                    timer("end", "masked_linear_unmask", g.name)
+                out[g.name] = res[:M]
+                continue
             if st["fused"]:  # both halves of the left operand in one launch
                 spl.spl_noise_mask_split_stacked(a.f16_hi, a.f16_lo, a.f16_exp, inputs[g.name], delta, eps, mech, seed,
                                                  M, off_next - off, stream_id=gi, offset=off, stream=stream,
@@ -238,7 +254,6 @@ class MaskedLayer:
                                    stream=stream, offset_dev=off_dev)
                 spl.spl_noise(a.w[M:], delta, eps, mech, seed, stream_id=gi, offset=off_next, stream=stream,
                               offset_dev=off_dev)
-            res = st["out"][1 - parity][d]
             if timer:
                 timer("begin", "masked_linear_unmask", g.name)
             spl.spl_masked_linear_unmask_precompute(res, a, g.wt, st["out"][parity][d][M:], M, path=st["path"],

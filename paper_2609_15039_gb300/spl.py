@@ -79,6 +79,8 @@ _SIGS = {
     "spl_masked_linear_unmask_precompute": (_I, [_P, _PW, _PW, _P, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_noise_mask_linear_unmask": (_I, [_P, _P, _P, _PW, _P, _I64, _I64, _I64, _D, _D, _I, spl_rng, _I, _P, _SZ,
                                           _P]),
+    "spl_noise_mask_linear_unmask_precompute": (_I, [_P, _P, _P, _PW, _P, _I64, _I64, _I64, _I64, _D, _D, _I,
+                                                     spl_rng, ctypes.c_uint64, _I, _P, _SZ, _P]),
     "spl_delta_layernorm": (_D, [_P, _I64]),
     "spl_delta_attention": (_D, [_P, _I64, _D]),
     "spl_delta_activation": (_D, [_P, _P, _I64, _I64, _D, _D]),
@@ -511,6 +513,30 @@ def spl_noise_mask_linear_unmask(Y, Xt, X, W, C, sensitivity, eps, mech, seed, s
                                               _rng(seed, stream_id, offset, offset_dev), _path(path), wsp, wsb,
                                               _stream(stream)),
            "spl_noise_mask_linear_unmask")
+
+
+def spl_noise_mask_linear_unmask_precompute(YC, Xt, X, W, C, sensitivity, eps, mech, seed, noise_rows,
+                                            noise_block_delta, stream_id=0, offset=0, path="auto", workspace=None,
+                                            stream=None, offset_dev=None):
+    """a2-a6 in one decode launch: rows of X masked and multiplied (unmasked with C), then noise_rows rows
+    of noise alone drawn noise_block_delta Philox blocks further on, multiplied (see include/spl.h)."""
+    W = _weight(W)
+    K = W.shape[-1]
+    if X is None:
+        M = 0
+    else:
+        M, K = _rows_cols(X)
+    rows = M + int(noise_rows)
+    N = W.shape[0]
+    if W.shape[-1] != K or Xt.numel() != rows * K or YC.numel() != rows * N or (
+            M > 0 and (C is None or C.numel() != M * N)):
+        raise ValueError("spl_noise_mask_linear_unmask_precompute: shape mismatch")
+    wsp, wsb = _ws(workspace)
+    ws_ = W.c_struct()
+    _check(lib().spl_noise_mask_linear_unmask_precompute(
+        _dev(YC, "YC"), _dev(Xt, "Xt"), _dev(X, "X"), ctypes.byref(ws_), _dev(C, "C") if M > 0 else None, M,
+        int(noise_rows), K, N, float(sensitivity), _eps(eps), _mech(mech), _rng(seed, stream_id, offset, offset_dev),
+        int(noise_block_delta), _path(path), wsp, wsb, _stream(stream)), "spl_noise_mask_linear_unmask_precompute")
 
 
 def spl_masked_linear_unmask_noalloc(Y, Xt, W, C, stream=None):

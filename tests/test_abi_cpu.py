@@ -156,8 +156,25 @@ def test_precompute_and_swap_entries_validate_without_launch(spl):
     assert pre(base, ctypes.byref(a), ctypes.byref(w), base, -1, 2, 8, 4, 0, None, 0, None) == spl.SPL_EINVAL
     assert pre(base, ctypes.byref(a), ctypes.byref(w), None, 2, 2, 8, 4, 0, None, 0, None) == spl.SPL_EINVAL  # C
     assert pre(base, ctypes.byref(a), ctypes.byref(w), None, 0, 0, 8, 4, 0, None, 0, None) == spl.SPL_OK      # empty
-    # no tensor-core device here, so AUTO resolves to FP32, which has no row limit on C
-    assert pre(base, ctypes.byref(a), ctypes.byref(w), base, 2, 2, 8, 4, 0, None, 0, None) == spl.SPL_EUNSUPPORTED
+    # no tensor-core device here, so AUTO resolves to FP32: beyond 16 rows that is the SIMT kernel,
+    # which has no row limit on C
+    assert pre(base, ctypes.byref(a), ctypes.byref(w), base, 9, 8, 8, 4, 0, None, 0, None) == spl.SPL_EUNSUPPORTED
+    fused = L.spl_noise_mask_linear_unmask_precompute
+    rng = spl._rng(1, 0, 0, None)
+    lap = spl._mech("laplace")
+
+    def call(Xt, X, C, M, M_bank, eps=1.0, path=0, rng_=rng):
+        return fused(base, Xt, X, ctypes.byref(w), C, M, M_bank, 8, 4, 1.0, eps, lap, rng_, 64, path, None, 0, None)
+
+    assert call(base, base + 128, base, 1, 1, eps=-1.0) == spl.SPL_EINVAL         # eps
+    assert call(base, base + 128, None, 1, 1) == spl.SPL_EINVAL                   # no C for the masked row
+    assert call(base, base + 128, base, 0, 0) == spl.SPL_OK                       # empty
+    assert call(base, base + 128, base, 2, 3) == spl.SPL_EUNSUPPORTED             # 5 rows: not one decode launch
+    assert call(base, base + 128, base, 1, 1, path=spl._path("fp16x3")) == spl.SPL_EUNSUPPORTED
+    assert call(base + 4, base + 128, base, 1, 1) == spl.SPL_EALIGN               # Xt
+    assert call(base, base + 16, base, 1, 1) == spl.SPL_EINVAL                    # X overlaps Xt's two rows
+    assert call(base, None, base, 1, 1) == spl.SPL_EINVAL                         # no X for the masked row
+    assert call(base, base + 128, base, 1, 1, rng_=spl.spl_rng(1, 0, 0, base + 4)) == spl.SPL_EALIGN  # offset_dev
     swap = L.spl_test_tc_swap_product
     assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 24, 1, None, 0, None) == spl.SPL_EINVAL  # width
     assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 16, 9, None, 0, None) == spl.SPL_ESHAPE  # splits

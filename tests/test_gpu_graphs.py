@@ -212,12 +212,16 @@ def make_stacked(model, M, draws, layers=1, zero_inputs=False):
 
 
 @pytest.mark.parametrize("M,model", [(128, wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)),
-                                     (512, wl.LLAMA_3_2_3B)])
+                                     (512, wl.LLAMA_3_2_3B), (1, wl.LLAMA_3_2_3B),
+                                     (2, wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)),
+                                     (4, wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000))])
 def test_stacked_correction_cancels_exactly(spl, M, model):
     """With x = 0 the mask is the noise itself, so the recovered output is fl(eta W^T) - fl(eta W^T):
     exactly zero when the correction (computed in the previous cycle in the bank half of a product of
     2M rows) is summed in exactly the order of the online row that meets it (the masked half of a later
-    product of the same shape) -- every element, at the bench's own sizes too."""
+    product of the same shape) -- every element, at the bench's own sizes too.  Decode sizes (2M <= 4)
+    take the one-launch form (noise, mask and product together); 2M = 8 the decode kernel after a
+    separate mask."""
     draws, eps, mech = 2, 1.0, "laplace"
     stack, inputs = make_stacked(model, M, draws, zero_inputs=True)
     layer, seed = stack.layers[0], stack.seeds[0]
@@ -230,11 +234,13 @@ def test_stacked_correction_cancels_exactly(spl, M, model):
     assert spl.spl_get_device_status() == 0
 
 
-def test_stacked_graphs_equal_eager_steps(spl):
+@pytest.mark.parametrize("M", [128, 1])
+def test_stacked_graphs_equal_eager_steps(spl, M):
     """Replayed stacked graphs (two layers, device-side Philox bases, the last graph of a cycle moving
-    them on) give, bit for bit, the eager stacked steps of the same cycles; any number of steps."""
+    them on) give, bit for bit, the eager stacked steps of the same cycles; any number of steps.  One
+    row: the decode form, one launch per group and step."""
     model = wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)
-    M, draws, eps, mech = 128, 3, 1.0, "gaussian"
+    draws, eps, mech = 3, 1.0, "gaussian"
     stack, inputs = make_stacked(model, M, draws, layers=2)
     expected = {}
     for cycle in range(4):

@@ -696,6 +696,87 @@ def test_noise_mask_linear_unmask_equals_separate_calls(spl, M, K, N, mech, eps)
     assert e.value.status == spl.SPL_EINVAL
 
 
+@pytest.mark.parametrize("M,M_bank,K,N,mech,eps", [(1, 1, 3072, 5120, "laplace", 1.0), (2, 2, 8192, 3072, "gaussian", 1.0),
+                                                  (1, 3, 1032, 600, "laplace", None), (0, 2, 3072, 1000, "gaussian", 0.5),
+                                                  (3, 0, 264, 300, "laplace", 0.5), (1, 1, 9728, 3072, "gaussian", 1.0)])
+def test_stacked_decode_call_equals_separate_calls(spl, M, M_bank, K, N, mech, eps):
+    """The stacked decode step in one launch: the X~ rows of spl_noise_mask, the noise rows of spl_noise
+    drawn noise_block_delta blocks further on, and the product of spl_masked_linear_unmask_precompute on
+    that operand, bit for bit; X~ and the noise against the oracle's draw, every output row within the
+    FP32 product bound of the operand the kernel wrote."""
+    W, Wt = _weights(spl, N, K, seed=N + K + 1)
+    rows = M + M_bank
+    X = wl.activations(max(M, 1), K, seed=M + 31).numpy()[:M]
+    C = dev(wl.activations(max(M, 1), N, seed=M + 32).numpy()[:M]) if M else None
+    base = torch.tensor([300], dtype=torch.int64, device="cuda")
+    delta = 8 * K // 4 + 5
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(rows, K, N, "fp32"))
+    xt_ref, YC_ref = torch.zeros((rows, K), device="cuda"), torch.empty((rows, N), device="cuda")
+    if M:
+        spl.spl_noise_mask(xt_ref[:M], None, dev(X), 825.3, eps, mech, seed=23, stream_id=2, offset=300 + 9)
+    if M_bank:
+        spl.spl_noise(xt_ref[M:], 825.3, eps, mech, seed=23, stream_id=2, offset=300 + 9 + delta)
+    spl.spl_masked_linear_unmask_precompute(YC_ref, spl.Weight(xt_ref), Wt, C, M, path="fp32", workspace=ws)
+    xt, YC = torch.full((rows, K), 7.0, device="cuda"), torch.full((rows, N), 7.0, device="cuda")
+    n0 = spl.spl_launch_count()
+    spl.spl_noise_mask_linear_unmask_precompute(YC, xt, dev(X) if M else None, Wt, C, 825.3, eps, mech, 23, M_bank,
+                                                delta, stream_id=2, offset=9, path="fp32", workspace=ws,
+                                                offset_dev=base)
+    torch.cuda.synchronize()
+    assert spl.spl_launch_count() - n0 == 1
+    assert torch.equal(xt, xt_ref) and torch.equal(YC, YC_ref)
+    e = math.inf if eps is None else eps
+    n_exp = np.zeros((rows, K))
+    if M:
+        n_exp[:M] = philox.noise((M, K), 825.3, e, mech, 23, 2, 309)
+    if M_bank:
+        n_exp[M:] = philox.noise((M_bank, K), 825.3, e, mech, 23, 2, 309 + delta)
+    xt_exp = n_exp.copy()
+    if M:
+        xt_exp[:M] = linear.mask(X, n_exp[:M].astype(np.float32))
+    tol = 2 * ulp32(xt_exp) + 8 * ulp32(n_exp)
+    if mech == "gaussian" and eps is not None:
+        r = np.zeros((rows, K))
+        if M:
+            r[:M] = philox.radius_fp64((M, K), 23, 2, 309)
+        if M_bank:
+            r[M:] = philox.radius_fp64((M_bank, K), 23, 2, 309 + delta)
+        tol = tol + 8 * U * float(np.float32(825.3 / eps)) * r
+    assert np.all(np.abs(f64(xt) - xt_exp) <= tol)
+    if M:
+        assert_product_close(f32(YC[:M]), f32(xt[:M]), W, "fp32", C=f32(C), what="masked rows")
+    if M_bank:
+        assert_product_close(f32(YC[M:]), f32(xt[M:]), W, "fp32", what="correction rows")
+    assert spl.spl_get_device_status() == 0
+
+
+@pytest.mark.parametrize("M,M_bank,K,N", [(1, 1, 3072, 5120), (8, 8, 8192, 3072), (0, 5, 1032, 600), (4, 0, 264, 300),
+                                          (3, 9, 9728, 3072)])
+def test_precompute_on_the_decode_kernel(spl, M, M_bank, K, N):
+    """spl_masked_linear_unmask_precompute at up to 16 rows on FP32 runs the decode kernel: every row
+    summed as the same row of a plain product of M + M_bank rows, C subtracted from the first M only."""
+    W, Wt = _weights(spl, N, K, seed=K + N + 7)
+    rows = M + M_bank
+    A = (wl.activations(rows, K, seed=rows + 5).numpy() * 300).astype(np.float32)
+    C = wl.activations(max(M, 1), N, seed=11).numpy()[:M]
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(rows, K, N, "fp32"))
+    YC = torch.full((rows, N), float("nan"), device="cuda")
+    spl.spl_masked_linear_unmask_precompute(YC, spl.Weight(dev(A)), Wt, dev(C) if M else None, M, path="fp32",
+                                            workspace=ws)
+    if M:
+        assert_product_close(f32(YC[:M]), A[:M], W, "fp32", C=C, what="masked rows")
+    if M_bank:
+        assert_product_close(f32(YC[M:]), A[M:], W, "fp32", what="correction rows")
+    P = torch.empty((rows, N), device="cuda")
+    spl.spl_masked_linear(P, dev(A), Wt, path="fp32", workspace=ws)
+    assert torch.equal(YC[M:], P[M:])
+    if M:
+        Yu = torch.empty((M, N), device="cuda")
+        spl.spl_unmask(Yu, P[:M].contiguous(), dev(C))
+        assert torch.equal(YC[:M], Yu)
+    assert spl.spl_get_device_status() == 0
+
+
 @pytest.mark.parametrize("rows,cols,mech,eps", [(1024, 3072, "gaussian", 1.0), (37, 1032, "laplace", 0.5),
                                                 (8, 8192, "laplace", None)])
 def test_noise_split_is_the_split_of_the_noise(spl, rows, cols, mech, eps):
