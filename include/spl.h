@@ -305,13 +305,25 @@ spl_status spl_slalom_mask(float* Xt_q, float* eta_out, const float* X, int64_t 
 spl_status spl_slalom_linear_unmask(float* Y, const float* Xt_q, const float* W_q, const double* C, int64_t M,
                                     int64_t K, int64_t N, void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
+/* Workspace bytes of a product (order_rows = M) or of a correction summed in
+ * the order of an online product of order_rows rows, of M rows, K, N on
+ * `path`, when its left operand comes split (FP16X3: the arrival counters and
+ * partial tiles the swapped kernel of 9-16 rows sums through; 0 for the
+ * kernels that reduce on chip) -- for AUTO the most over the paths, the
+ * others reading the fp32 operand as the plain calls do.  Calls whose
+ * workspaces are this small may run side by side on different streams only
+ * with separate workspaces when it is not 0.  0 for invalid arguments. */
+size_t spl_split_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows, spl_path path);
+
 /* ---- a5 + a6 with the left operand already split ---------------------------
  * As spl_masked_linear_unmask, with X~ given as a descriptor: Xt->w the fp32
  * X~ (may be NULL when the call runs FP16X3) and Xt->f16_hi / f16_lo / f16_exp
  * its fp16 split (from spl_noise_mask_split or spl_split_fp16).  On the FP16X3
- * path the product reads the split and skips its own split pass (no workspace
- * needed); other paths read Xt->w (EINVAL if it is NULL).  The result equals
- * spl_masked_linear_unmask's bit for bit. */
+ * path the product reads the split and skips its own split pass: the workspace
+ * then holds only what spl_split_workspace_bytes(M, K, N, M, path) asks (the
+ * swapped kernel's counters and partial tiles for 9-16 rows; none for the
+ * kernels that reduce on chip); other paths read Xt->w (EINVAL if it is NULL).
+ * The result equals spl_masked_linear_unmask's bit for bit. */
 spl_status spl_masked_linear_unmask_split(float* Y, const spl_weight* Xt, const spl_weight* W, const float* C,
                                           int64_t M, int64_t K, int64_t N, spl_path path, void* workspace,
                                           size_t workspace_bytes, cudaStream_t stream);
@@ -519,17 +531,23 @@ spl_status spl_test_tc_product(float* Y, const float* Xt, const spl_weight* W, c
                                size_t workspace_bytes, cudaStream_t stream);
 
 /* Test hook: the FP16X3 product on the swapped kernel the library takes for
- * products of 9 to 64 rows (the weight in the MMA's 128 rows, the tokens in
+ * products of 9 to 16 rows (the weight in the MMA's 128 rows, the tokens in
  * its N columns), forced to a token-tile width `tile_tokens` (16, 32, 64 or
- * 128) and a K-split `splits` (1-8, a thread-block cluster summed in rank
- * order) for any M.  Y[M, N] = fl32(Xt W^T - C) (C may be NULL), W with its
- * fp16 split, workspace as spl_linear_workspace_bytes(M, K, N, FP16X3).
- * Errors: EINVAL for a width not listed or NULL operands, ESHAPE for splits
- * outside 1-8, EALIGN for K % 8 != 0 or unaligned pointers, as
- * spl_masked_linear otherwise.  The paper has no counterpart. */
+ * 128) and `ctas` CTAs per token tile (0: the library's count) for any M: the
+ * (128-row weight tile, 64-element k-block) units of each token tile dealt out
+ * in `ctas` equal contiguous runs, the pieces of a tile summed in K order by
+ * the CTA that finishes the tile last, through the workspace.  Y[M, N] =
+ * fl32(Xt W^T - C) (C may be NULL), W with its fp16 split; the workspace holds
+ * at least spl_test_tc_swap_workspace_bytes(M, K, N, tile_tokens, ctas) bytes,
+ * its first 64 KiB zero (each call leaves them zero).  Errors: EINVAL for a
+ * width not listed, NULL operands or ctas < 0, EALIGN for K % 8 != 0 or
+ * unaligned pointers, EWORKSPACE for a short workspace, ESHAPE for more than
+ * 16384 tiles, as spl_masked_linear otherwise.  The paper has no
+ * counterpart. */
 spl_status spl_test_tc_swap_product(float* Y, const float* Xt, const spl_weight* W, const float* C, int64_t M,
-                                    int64_t K, int64_t N, int tile_tokens, int splits, void* workspace,
+                                    int64_t K, int64_t N, int tile_tokens, int ctas, void* workspace,
                                     size_t workspace_bytes, cudaStream_t stream);
+size_t spl_test_tc_swap_workspace_bytes(int64_t M, int64_t K, int64_t N, int tile_tokens, int ctas);
 
 /* ---- status -------------------------------------------------------------
  * Synchronises `stream`, returns SPL_ETIMEOUT if any kernel since the last

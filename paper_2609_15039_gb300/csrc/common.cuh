@@ -165,6 +165,9 @@ bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, spl_path path, int* varia
 // rows uses (the correction bank): the same K ranges, accumulation chains and cluster order.
 spl_status run_tc_matched(const LinearArgs& a, int64_t order_rows);
 size_t tc_asplit_bytes(int64_t M, int64_t K, spl_path path);  // FP16X3 split of A in the workspace (0 for TF32X3)
+// Workspace for the partial tiles of a tcgen05 product of M rows summed in the order of `order_rows`
+// (the swapped kernel's runs; 0 for the cluster-reduced kernels), after the split of A.
+size_t tc_partial_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows, spl_path path);
 spl_status run_simt(const LinearArgs& a, const Plan& p);
 spl_status run_tc(const LinearArgs& a, const Plan& p);
 

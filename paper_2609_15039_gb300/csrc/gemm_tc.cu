@@ -144,6 +144,17 @@ __device__ __forceinline__ uint64_t make_sdesc_sw64(uint32_t saddr) {
   return d;
 }
 
+// The same for the 128-byte swizzle: 128-byte rows, 8-row (1024-byte) atoms, SWIZZLE_128B = 2.
+__device__ __forceinline__ uint64_t make_sdesc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1u << 16;
+  d |= (uint64_t)(1024u >> 4) << 32;
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)2u << 61;
+  return d;
+}
+
 // ---- PTX wrappers ----------------------------------------------------------------
 __device__ __forceinline__ float pow2f(int e) { return __int_as_float((e + 127) << 23); }  // e in [-126, 127]
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -293,7 +304,7 @@ __device__ __forceinline__ void tmem_st_32x32(uint32_t taddr, const float (&v)[3
       : "memory");
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
-// 32 lanes x 16 columns of 32-bit words (thread t gets lane base + t), and back.
+// 32 lanes x 16 columns of 32-bit words (thread t gets lane base + t).
 __device__ __forceinline__ void tmem_ld_32x16(uint32_t taddr, float (&v)[16]) {
   uint32_t r[16];
   asm volatile(
@@ -305,23 +316,6 @@ __device__ __forceinline__ void tmem_ld_32x16(uint32_t taddr, float (&v)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-__device__ __forceinline__ void tmem_st_32x16(uint32_t taddr, const float (&v)[16]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-          taddr),
-      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
-      "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
-      "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
-      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
-      "r"(__float_as_uint(v[15]))
-      : "memory");
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
-  return v;
 }
 __device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 __device__ __forceinline__ void prefetch_l2(const void* p) {
@@ -1020,93 +1014,113 @@ tc_persistent_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ ou
 }
 
 // ---- few rows: the weight in the MMA's 128 rows, the tokens in its N ------------------------------
-// out[M, N] = A[M, K] W[N, K]^T (- C) on FP16X3 for a few tokens (9 to 32 rows: from 33 rows on the
+// out[M, N] = A[M, K] W[N, K]^T (- C) on FP16X3 for a few tokens (9 to 16 rows: from 17 rows on the
 // 128-row tiles of tc_gemm_kernel were as fast on GB300, and up to 8 rows the FP32 decode kernel is
-// the library's choice): D = W A^T, so the
-// weight fills the 128 rows of the MMA and the tokens its N columns (TN per tile, a multiple of 16;
-// tokens past M are the zero rows the copy fills in).  A tile of 128 weight rows streams its rows of
-// W once per token tile -- 4 bytes per weight, the same as the fp32 weight the decode kernel reads --
-// while the MMAs do a small fraction of a full tile's work, so the kernel runs near HBM rate where a
-// 128-row tile of tokens would be tensor-bound on mostly empty rows.  With so little work per MMA
-// the instructions themselves cost time, so the three products of a term take two: the tokens' lo
-// and hi rows sit next to each other in shared memory, and one MMA of N = 2 TN multiplies W_hi by
-// both (columns 0..TN-1: hi*lo; TN..2TN-1: hi*hi), a second multiplies W_lo by the tokens' hi rows
-// into columns 0..TN-1 (every accumulator starts on a 32-column boundary).  The large hi*hi sums and the small cross terms thus accumulate apart (the
-// cross terms' truncation error is ~2^-11 smaller) and are added with round-to-nearest in the
-// epilogue.  As in tc_gemm_kernel: row exponents undone exactly (the weight's per MMA row, the
-// tokens' per column), accumulation chains of at most kChainBlocks k-blocks folded in TMEM, a cluster
-// K-split summed in rank order.  TMEM lane r holds weight row n0 + r, so a warp's 32 lanes store 32
-// consecutive outputs of one token (128 bytes).  An element's sum does not depend on the other
-// columns of its MMA, so a bank of corrections for several draws of tokens, run with a wider TN and
-// the same K-split, reproduces the online product bit for bit.  Narrow tiles keep a 96 KB ring so
-// that two CTAs share an SM (one streaming while the other starts or finishes).
-constexpr int64_t kSwapMaxM = 32;
+// the library's choice): D = W A^T, so the weight fills the 128 rows of the MMA and the tokens its N
+// columns (TN per token tile, a multiple of 16; tokens past M are the zero rows the copy fills in).
+// The weight streams once per token tile -- 4 bytes per weight, the same as the fp32 weight the
+// decode kernel reads -- while the MMAs do a small fraction of a full tile's work, so the kernel runs
+// near HBM rate where a 128-row tile of tokens would be tensor-bound on mostly empty rows.  With so
+// little work per MMA the instructions themselves cost time, so the three products of a term take
+// two: the tokens' lo and hi rows sit next to each other in shared memory, one MMA of N = 2 TN
+// multiplies W_hi by both (columns 0..TN-1: hi*lo; TN..2TN-1: hi*hi) and a second multiplies W_lo
+// by the tokens' hi rows into columns 0..TN-1.  The large hi*hi sums and the small cross terms thus
+// accumulate apart (the cross terms' truncation error is ~2^-11 smaller) and are added with
+// round-to-nearest when a chain is read out.  Row exponents are undone exactly (the weight's per
+// MMA row, the tokens' per column).  K-blocks are 64 elements (128-byte rows, 128-byte swizzle):
+// measured on GB300, half as many ring round trips per byte made the 64-byte form 10-30% slower.
+//
+// Work split (stream-K): the (weight tile, k-block) units of one token tile, tile-major, are dealt
+// out in `ctas` contiguous runs of equal length (CTA c takes units [c U / ctas, (c + 1) U / ctas)
+// of U), so every CTA streams the same number of weight bytes whatever the number of tiles: no
+// partly empty wave and no clusters.  A run crosses tile boundaries: its part of one tile (a piece)
+// is summed in chains of at most 1024 elements of K (kChainBlocks of the 32-element unit),
+// alternating between two TMEM accumulators so that the epilogue reads one chain while the MMAs
+// fill the other; the chains of a piece are added in order with round-to-nearest.  A piece that is
+// a whole tile goes straight out.  Otherwise its partial tile (8-64 KB) goes to the workspace and
+// the CTA bumps the tile's arrival counter; the CTA that arrives last sums the tile's pieces in K
+// order (every CTA's slot, its own included), undoes the row scales, subtracts C, stores, and puts
+// the counter back to zero for the next call.  No CTA waits on another.  The decomposition depends
+// only on N, K and `ctas`, the same for every token tile and every token column, and an element's
+// sum does not depend on the other columns of its MMA, so a bank run with the online product's
+// `ctas` at any token-tile width reproduces its sums bit for bit.
+constexpr int64_t kSwapMaxM = 16;
+
+// Units of CTA c of `ctas` over `total` units: [run_begin(c), run_begin(c + 1)).
+__host__ __device__ __forceinline__ int64_t run_begin(int64_t c, int64_t total, int64_t ctas) {
+  return c * total / ctas;
+}
+// The CTA whose run holds unit u (the largest c with run_begin(c) <= u; ctas <= total).
+__host__ __device__ __forceinline__ int64_t run_of(int64_t u, int64_t total, int64_t ctas) {
+  return ((u + 1) * ctas - 1) / total;
+}
 
 template <int TN>
 struct SwapCfg {
   static_assert(TN % 16 == 0 && TN >= 16 && TN <= 128, "MMA N of 2 TN: a multiple of 32 up to 256");
-  static constexpr int BK = 32;  // fp16 elements of K per 64-byte row
+  static constexpr int BK = 64;  // fp16 elements of K per 128-byte swizzled row
   static constexpr uint32_t W_HALF = BM * BK * 2, X_HALF = TN * BK * 2;
   static constexpr uint32_t W_HI = 0, W_LO = W_HALF, X_LO = 2 * W_HALF, X_HI = X_LO + X_HALF;
   static constexpr uint32_t STAGE = X_HI + X_HALF;  // bytes TMA brings per stage
-  static constexpr int CTAS_PER_SM = TN <= 64 ? 2 : 1;
-  static constexpr uint32_t RING = (TN <= 64 ? 96u : 192u) * 1024u;
+  static constexpr uint32_t RING = 192u * 1024u;    // one CTA per SM
   static constexpr int STAGES = (int)(RING / STAGE) > 12 ? 12 : (int)(RING / STAGE);
   static constexpr uint32_t SMEM = RING + AUX_BYTES + 1024;
-  static constexpr int RED_STRIDE = TN + 1;  // floats per weight row of the staged partial tile
   static constexpr uint32_t IDESC_HI = make_idesc(0, BM, 2 * TN);  // W_hi x [x_lo; x_hi]
   static constexpr uint32_t IDESC_LO = make_idesc(0, BM, TN);      // W_lo x x_hi
-  // TMEM: R (cross terms at 0, hi*hi at TN) and, for a later accumulation chain, P at P_OFF
-  static constexpr uint32_t ACC = 2 * TN, P_OFF = ACC;
-  static constexpr uint32_t TMEM_COLS = 4 * TN < 64 ? 64u : (uint32_t)(4 * TN);
+  static constexpr uint32_t BUF = 2 * TN;                          // columns of one accumulator
+  static constexpr uint32_t TMEM_COLS = 4 * TN < 64 ? 64u : (uint32_t)(4 * TN);  // two of them
+  static constexpr uint32_t AUX_BARS = 8 * (2 * STAGES + 5);  // full[S], empty[S], buf_full[2], buf_free[2], drain
+  static constexpr int64_t CHAIN = kChainBlocks * 32 / BK;    // k-blocks per chain: 1024 elements of K
   static_assert(X_HALF % 1024 == 0 && STAGE % 1024 == 0 && X_LO % 1024 == 0, "swizzle atoms aligned");
   static_assert(STAGES >= 3, "ring depth");
-  static_assert(8 * (2 * STAGES + 4) + 16 <= 1024, "barriers fit");
-  static_assert((size_t)BM * RED_STRIDE * 4 <= RING, "staging fits in the stage ring");
-  static_assert(CTAS_PER_SM * (SMEM + 1024) <= 233472, "CTAs per SM fit in shared memory");
+  static_assert(AUX_BARS + 16 <= 1024, "barriers fit");
+  static_assert(TMEM_COLS <= 512, "TMEM of the CTA");
+  static_assert(SMEM + 1024 <= 233472, "shared memory of the CTA");
 };
 
 template <int TN>
-__global__ void __launch_bounds__(THREADS, SwapCfg<TN>::CTAS_PER_SM)
+__global__ void __launch_bounds__(THREADS, 1)
 tc_swap_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, const float* __restrict__ C,
-               const int* __restrict__ x_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N,
-               int64_t k_per_split, int splits, int m_tiles, int chain, int64_t c_rows) {
+               const int* __restrict__ x_exp, const int* __restrict__ w_exp, int64_t M, int64_t K, int64_t N, int ctas,
+               int64_t c_rows, float* __restrict__ part, unsigned int* __restrict__ counters) {
   using L = SwapCfg<TN>;
-  constexpr int STAGES = L::STAGES, BK = L::BK, RS = L::RED_STRIDE;
+  constexpr int STAGES = L::STAGES, BK = L::BK;
+  constexpr int64_t CH = L::CHAIN;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* aux = smem + L::RING;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);  // full[S], empty[S], accum, seg, fold, spare
-  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + 8 * (2 * STAGES + 4));
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + 8 * (2 * STAGES + 4) + 8);
-  float* red = reinterpret_cast<float*>(smem);  // [BM][RS] staged partial tile, after the mainloop
+  uint64_t* bars = reinterpret_cast<uint64_t*>(aux);
+  volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(aux + L::AUX_BARS);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(aux + L::AUX_BARS + 8);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(aux + L::AUX_BARS + 12);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // token tiles of one weight tile side by side, so they share its rows in L2
-  const int tile = (int)blockIdx.x;
-  const int64_t m0 = (int64_t)(tile % m_tiles) * TN, n0 = (int64_t)(tile / m_tiles) * BM;
-  const int64_t kbeg = (int64_t)blockIdx.z * k_per_split;
-  const int64_t kend = std::min<int64_t>(K, kbeg + k_per_split);
-  const int nk = kend > kbeg ? (int)ceil_div(kend - kbeg, BK) : 0;
-  const int seg_len = chain > 0 && chain < nk ? chain : nk + 1;
-  const int nseg = chain > 0 && chain < nk ? (int)ceil_div(nk, chain) : 1;
+  const int64_t nkb = ceil_div(K, (int64_t)BK);
+  const int64_t w_tiles = ceil_div(N, (int64_t)BM);
+  const int64_t total = w_tiles * nkb;
+  const int64_t c = blockIdx.x, tt = blockIdx.y;
+  const int64_t m0 = tt * TN;
+  const int64_t u0 = run_begin(c, total, ctas), u1 = run_begin(c + 1, total, ctas);
 
   const uint32_t bar_base = smem_u32(bars);
   auto full_bar = [&](int st) { return bar_base + 8u * st; };
   auto empty_bar = [&](int st) { return bar_base + 8u * (STAGES + st); };
-  const uint32_t accum_bar = bar_base + 8u * (2 * STAGES);
-  const uint32_t seg_bar = bar_base + 8u * (2 * STAGES + 1);   // a later segment is in P
-  const uint32_t fold_bar = bar_base + 8u * (2 * STAGES + 2);  // P folded into R
+  auto buf_full = [&](int b) { return bar_base + 8u * (2 * STAGES + b); };      // a chain is in buffer b
+  auto buf_free = [&](int b) { return bar_base + 8u * (2 * STAGES + 2 + b); };  // buffer b has been read
+  const uint32_t drain_bar = bar_base + 8u * (2 * STAGES + 4);
 
   if (threadIdx.x == 0) {
     for (int st = 0; st < STAGES; ++st) {
       mbar_init(full_bar(st), 1);
       mbar_init(empty_bar(st), 1);
     }
-    mbar_init(accum_bar, 1);
-    mbar_init(seg_bar, 1);
-    mbar_init(fold_bar, 4);  // one arrival per epilogue warp
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(buf_full(b), 1);
+      mbar_init(buf_free(b), 4);  // one arrival per epilogue warp
+    }
+    mbar_init(drain_bar, 1);
     *abort_flag = 0;
+    *last_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -1115,46 +1129,46 @@ tc_swap_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  const int n_units = (int)(u1 - u0);
 
   if (warp == 0) {
-    // ---------------- TMA producer: W_hi, W_lo (128 rows), X_hi, X_lo (TN rows) ----------------
-    // The weight does not depend on the kernel before this one: the first stages' weight tiles go
-    // out before waiting for it.
+    // ---------------- TMA producer: the run's units in order, W_hi, W_lo, X_hi, X_lo ----------------
     uint32_t issued_mask = 0u, phase_mask = 0u;
     bool ok = true;
     const uint64_t pol_w = l2_evict_first(), pol_x = l2_evict_last();
-    const int pre = nk < STAGES ? nk : STAGES;
-    for (int kb = 0; kb < pre; ++kb) {
+    const int pre = n_units < STAGES ? n_units : STAGES;
+    for (int j = 0; j < pre; ++j) {  // the weight does not depend on the kernel before this one
       if (lane == 0) {
-        const uint32_t st = smem_u32(smem + (size_t)kb * L::STAGE);
-        const int kx = (int)(kbeg + (int64_t)kb * BK);
-        mbar_expect_tx(full_bar(kb), L::STAGE);
-        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(kb), kx, (int)n0, pol_w);
-        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(kb), kx, (int)n0, pol_w);
+        const int64_t u = u0 + j;
+        const uint32_t st = smem_u32(smem + (size_t)j * L::STAGE);
+        mbar_expect_tx(full_bar(j), L::STAGE);
+        tma_load_2d(st + L::W_HI, &maps.w_hi, full_bar(j), (int)((u % nkb) * BK), (int)((u / nkb) * BM), pol_w);
+        tma_load_2d(st + L::W_LO, &maps.w_lo, full_bar(j), (int)((u % nkb) * BK), (int)((u / nkb) * BM), pol_w);
       }
-      issued_mask |= 1u << kb;
+      issued_mask |= 1u << j;
     }
     pdl_wait();
-    for (int kb = 0; kb < pre; ++kb) {
+    for (int j = 0; j < pre; ++j) {
       if (lane == 0) {
-        const uint32_t st = smem_u32(smem + (size_t)kb * L::STAGE);
-        const int kx = (int)(kbeg + (int64_t)kb * BK);
-        tma_load_2d(st + L::X_HI, &maps.a_hi, full_bar(kb), kx, (int)m0, pol_x);
-        tma_load_2d(st + L::X_LO, &maps.a_lo, full_bar(kb), kx, (int)m0, pol_x);
+        const int64_t u = u0 + j;
+        const uint32_t st = smem_u32(smem + (size_t)j * L::STAGE);
+        tma_load_2d(st + L::X_HI, &maps.a_hi, full_bar(j), (int)((u % nkb) * BK), (int)m0, pol_x);
+        tma_load_2d(st + L::X_LO, &maps.a_lo, full_bar(j), (int)((u % nkb) * BK), (int)m0, pol_x);
       }
     }
     __syncwarp();
-    for (int kb = pre; kb < nk; ++kb) {
-      const int st = kb % STAGES;
-      const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+    for (int j = pre; j < n_units; ++j) {
+      const int st = j % STAGES;
+      const uint32_t ph = (uint32_t)(j / STAGES) & 1u;
       ok = __all_sync(0xffffffffu, mbar_wait(empty_bar(st), ph ^ 1u, kWaitNs, abort_flag));
       if (!ok) break;
       if (lane == 0) {
+        const int64_t u = u0 + j;
+        const int kx = (int)((u % nkb) * BK), ny = (int)((u / nkb) * BM);
         const uint32_t sa = smem_u32(smem + (size_t)st * L::STAGE);
-        const int kx = (int)(kbeg + (int64_t)kb * BK);
         mbar_expect_tx(full_bar(st), L::STAGE);
-        tma_load_2d(sa + L::W_HI, &maps.w_hi, full_bar(st), kx, (int)n0, pol_w);
-        tma_load_2d(sa + L::W_LO, &maps.w_lo, full_bar(st), kx, (int)n0, pol_w);
+        tma_load_2d(sa + L::W_HI, &maps.w_hi, full_bar(st), kx, ny, pol_w);
+        tma_load_2d(sa + L::W_LO, &maps.w_lo, full_bar(st), kx, ny, pol_w);
         tma_load_2d(sa + L::X_HI, &maps.a_hi, full_bar(st), kx, (int)m0, pol_x);
         tma_load_2d(sa + L::X_LO, &maps.a_lo, full_bar(st), kx, (int)m0, pol_x);
       }
@@ -1172,36 +1186,46 @@ tc_swap_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
         if (issued_mask & (1u << st)) mbar_wait(full_bar(st), (phase_mask >> st) & 1u, kDrainNs, nullptr);
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer: D[w row, token] += W x^T, three products per term ----------------
+    // ---------------- MMA issuer: chains of at most CH units, buffers alternating ----------------
     bool ok = true;
-    for (int kb = 0; kb < nk; ++kb) {
-      const int st = kb % STAGES;
-      const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-      const int sg = kb / seg_len, in_seg = kb % seg_len;
-      if (in_seg == 0 && sg >= 2) {  // P is free once the previous segment has been folded into R
-        ok = __all_sync(0xffffffffu, mbar_wait(fold_bar, (uint32_t)(sg - 2) & 1u, kWaitNs, abort_flag));
-        if (!ok) break;
-      }
-      ok = __all_sync(0xffffffffu, mbar_wait(full_bar(st), ph, kWaitNs, abort_flag));
-      if (!ok) break;
-      if (lane == 0) {
-        tc_fence_after();
-        const uint32_t sa = smem_u32(smem + (size_t)st * L::STAGE);
-        const uint32_t acc = tmem + (sg >= 1 ? L::P_OFF : 0u);
-#pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk) {
-          const uint32_t koff = kk * 32u;  // one instruction's K is 32 bytes of the 64-byte swizzled row
-          const uint32_t first = (in_seg == 0 && kk == 0) ? 0u : 1u;
-          // W_hi x [x_lo; x_hi] (2 TN columns: hi*lo, then hi*hi), then W_lo x x_hi into the cross columns
-          mma<Fp16x3, L::IDESC_HI>(acc, make_sdesc_sw64(sa + L::W_HI + koff), make_sdesc_sw64(sa + L::X_LO + koff),
-                                   first);
-          mma<Fp16x3, L::IDESC_LO>(acc, make_sdesc_sw64(sa + L::W_LO + koff), make_sdesc_sw64(sa + L::X_HI + koff),
-                                   1u);
+    int j = 0, it = 0;  // unit of the run, chain of the run
+    for (int64_t u = u0; u < u1 && ok;) {
+      const int64_t pe = std::min<int64_t>(u1, (u / nkb + 1) * nkb);  // end of the piece
+      for (int64_t s = u; s < pe && ok;) {
+        const int64_t se = std::min<int64_t>(pe, s + CH);
+        const int b = it & 1;
+        if (it >= 2) {  // the epilogue has read this buffer's previous chain
+          ok = __all_sync(0xffffffffu, mbar_wait(buf_free(b), (uint32_t)((it >> 1) - 1) & 1u, kWaitNs, abort_flag));
+          if (!ok) break;
         }
-        mma_commit(empty_bar(st));  // stage reusable once these MMAs have read it
-        if (sg >= 1 && (in_seg == seg_len - 1 || kb == nk - 1)) mma_commit(seg_bar);  // P complete
+        const uint32_t acc = tmem + (uint32_t)b * L::BUF;
+        for (int64_t v = s; v < se; ++v, ++j) {
+          const int st = j % STAGES;
+          const uint32_t ph = (uint32_t)(j / STAGES) & 1u;
+          ok = __all_sync(0xffffffffu, mbar_wait(full_bar(st), ph, kWaitNs, abort_flag));
+          if (!ok) break;
+          if (lane == 0) {
+            tc_fence_after();
+            const uint32_t sa = smem_u32(smem + (size_t)st * L::STAGE);
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+              const uint32_t koff = kk * 32u;  // one instruction's K is 32 bytes of the swizzled row
+              const uint32_t first = (v == s && kk == 0) ? 0u : 1u;
+              // W_hi x [x_lo; x_hi] (2 TN columns: hi*lo, then hi*hi), then W_lo x x_hi into the cross columns
+              mma<Fp16x3, L::IDESC_HI>(acc, make_sdesc_sw128(sa + L::W_HI + koff),
+                                       make_sdesc_sw128(sa + L::X_LO + koff), first);
+              mma<Fp16x3, L::IDESC_LO>(acc, make_sdesc_sw128(sa + L::W_LO + koff),
+                                       make_sdesc_sw128(sa + L::X_HI + koff), 1u);
+            }
+            mma_commit(empty_bar(st));
+            if (v == se - 1) mma_commit(buf_full(b));
+          }
+          __syncwarp();
+        }
+        ++it;
+        s = se;
       }
-      __syncwarp();
+      u = pe;
     }
     pdl_trigger();
     if (lane == 0) {
@@ -1209,103 +1233,148 @@ tc_swap_kernel(const __grid_constant__ TcMaps maps, float* __restrict__ out, con
         *abort_flag = 1;
         atomicOr(&g_device_status, kStatusTimeout);
       }
-      mma_commit(accum_bar);  // MMAs already issued must finish before TMEM is read or released
+      mma_commit(drain_bar);  // issued MMAs finish before TMEM is released
     }
     __syncwarp();
-    if (!ok) mbar_wait(accum_bar, 0u, kDrainNs, nullptr);
+    if (!ok) mbar_wait(drain_bar, 0u, kDrainNs, nullptr);
   } else {
-    // ---------------- warps 2..5: folds, then the tile out (or staged for the cluster) --------------
+    // ---------------- warps 2..5: chains summed per piece; pieces out or through the workspace -------
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int r = 32 * q + lane;
-    const int64_t n = n0 + r;
     const uint32_t lane_base = tmem + ((uint32_t)(32 * q) << 16);
-    pdl_wait();  // the tokens' row exponents and C come from before this kernel
-    const float sw = n < N ? pow2f(-__ldg(w_exp + n)) : 1.0f;
+    pdl_wait();  // the tokens' row exponents, C and the counters come from before this kernel
     bool ok = true;
-    for (int f = 0; f + 1 < nseg; ++f) {  // fold segment f + 1 (in P) into R
-      ok = __all_sync(0xffffffffu, mbar_wait(seg_bar, (uint32_t)f & 1u, kWaitNs * 4, abort_flag));
-      if (!ok) break;
-      tc_fence_after();
-#pragma unroll 1
-      for (int c = 0; c < 2 * TN / 16; ++c) {  // both halves: the cross terms and hi*hi
-        float rv[16], pv[16];
-        tmem_ld_32x16(lane_base + (uint32_t)(16 * c), rv);
-        tmem_ld_32x16(lane_base + L::P_OFF + (uint32_t)(16 * c), pv);
+    int it = 0;
+    float run[TN];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) rv[i] = __fadd_rn(rv[i], pv[i]);
-        tmem_st_32x16(lane_base + (uint32_t)(16 * c), rv);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(fold_bar);
-    }
-    bool have = ok && (nk == 0 || mbar_wait(accum_bar, 0u, kWaitNs * 4, abort_flag));
-    have = __all_sync(0xffffffffu, have) && !*abort_flag;
-    pdl_trigger();
-    if (have) {
-      tc_fence_after();
-#pragma unroll 1
-      for (int c = 0; c < TN / 16; ++c) {
-        float v[16];
-        if (nk > 0) {
-          float cross[16];
-          tmem_ld_32x16(lane_base + (uint32_t)(TN + 16 * c), v);  // hi*hi
-          tmem_ld_32x16(lane_base + (uint32_t)(16 * c), cross);
+    for (int i = 0; i < TN; ++i) run[i] = 0.f;
+    for (int64_t u = u0; u < u1;) {
+      const int64_t t = u / nkb;
+      const int64_t pe = std::min<int64_t>(u1, (t + 1) * nkb);
+      for (int64_t s = u; s < pe;) {
+        const int64_t se = std::min<int64_t>(pe, s + CH);
+        const int b = it & 1;
+        ok = ok && __all_sync(0xffffffffu, mbar_wait(buf_full(b), (uint32_t)(it >> 1) & 1u, kWaitNs * 4, abort_flag));
+        if (ok) {
+          tc_fence_after();
+          const uint32_t base = lane_base + (uint32_t)b * L::BUF;
 #pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] = __fadd_rn(v[i], cross[i]);
-        } else {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] = 0.f;
-        }
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int64_t m = m0 + 16 * c + i;
-          // exact power-of-two scaling: the weight row's exponent, then the token's
-          v[i] = (v[i] * sw) * (m < M ? pow2f(-__ldg(x_exp + m)) : 1.0f);
-        }
-        if (splits == 1) {
-          if (n < N) {
+          for (int cc = 0; cc < TN / 16; ++cc) {
+            float hh[16], cr[16];
+            tmem_ld_32x16(base + (uint32_t)(TN + 16 * cc), hh);  // hi*hi
+            tmem_ld_32x16(base + (uint32_t)(16 * cc), cr);       // the cross terms
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              const int64_t m = m0 + 16 * c + i;
-              if (m < M) out[m * N + n] = (C && m < c_rows) ? __fsub_rn(v[i], __ldcs(C + m * N + n)) : v[i];
+              const float v = __fadd_rn(hh[i], cr[i]);
+              run[16 * cc + i] = s == u ? v : __fadd_rn(run[16 * cc + i], v);
             }
           }
-        } else {
+          tc_fence_before();
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(buf_free(b));
+        ++it;
+        s = se;
+      }
+      // the piece [u, pe) of weight tile t is in run[] (row r of the tile, tokens m0 ..)
+      const int64_t n = t * BM + r;
+      const bool whole = u == t * nkb && pe == (t + 1) * nkb;
+      bool store = whole;
+      if (!whole) {
+        // partial tiles [BM][TN]: a row's TN sums contiguous, moved as float4
+        const int slot = u == u0 ? 0 : 1;  // a run's first piece, or its last
+        float4* dst = reinterpret_cast<float4*>(part + ((tt * ctas + c) * 2 + slot) * (int64_t)(TN * BM)) +
+                      r * (TN / 4);
+        if (ok) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) red[r * RS + 16 * c + i] = v[i];
+          for (int i = 0; i < TN / 4; ++i)
+            __stcg(dst + i, make_float4(run[4 * i], run[4 * i + 1], run[4 * i + 2], run[4 * i + 3]));
+        }
+        // the epilogue's stores, then one gpu-scope fence and the arrival (release); the last
+        // arrival fences again before the epilogue reads the other pieces (acquire)
+        epilogue_sync();
+        if (threadIdx.x == 64) {
+          const int64_t c_first = run_of(t * nkb, total, ctas), c_last = run_of((t + 1) * nkb - 1, total, ctas);
+          unsigned int* cnt = counters + tt * w_tiles + t;
+          __threadfence();
+          const unsigned int prev = atomicAdd(cnt, 1u);
+          const int last = prev == (unsigned int)(c_last - c_first);
+          if (last) {
+            *cnt = 0u;  // every piece has arrived: ready for the next call
+            __threadfence();
+          }
+          *last_flag = last;
+        }
+        epilogue_sync();
+        store = *last_flag != 0;
+        if (store) {
+          // the tile's pieces in K order; PB pieces' loads in flight at a time
+          constexpr int PB = TN <= 16 ? 8 : (TN <= 32 ? 4 : (TN <= 64 ? 2 : 1));
+          const int64_t c_first = run_of(t * nkb, total, ctas), c_last = run_of((t + 1) * nkb - 1, total, ctas);
+          for (int64_t cq = c_first; cq <= c_last; cq += PB) {
+            float4 buf[PB][TN / 4];
+#pragma unroll
+            for (int bq = 0; bq < PB; ++bq) {
+              if (cq + bq <= c_last) {
+                const int sq = run_begin(cq + bq, total, ctas) / nkb == t ? 0 : 1;
+                const float4* src =
+                    reinterpret_cast<const float4*>(part + ((tt * ctas + cq + bq) * 2 + sq) * (int64_t)(TN * BM)) +
+                    r * (TN / 4);
+#pragma unroll
+                for (int i = 0; i < TN / 4; ++i) buf[bq][i] = __ldcg(src + i);
+              }
+            }
+#pragma unroll
+            for (int bq = 0; bq < PB; ++bq) {
+              if (cq + bq <= c_last) {
+                const bool first = cq + bq == c_first;
+#pragma unroll
+                for (int i = 0; i < TN / 4; ++i) {
+                  run[4 * i] = first ? buf[bq][i].x : __fadd_rn(run[4 * i], buf[bq][i].x);
+                  run[4 * i + 1] = first ? buf[bq][i].y : __fadd_rn(run[4 * i + 1], buf[bq][i].y);
+                  run[4 * i + 2] = first ? buf[bq][i].z : __fadd_rn(run[4 * i + 2], buf[bq][i].z);
+                  run[4 * i + 3] = first ? buf[bq][i].w : __fadd_rn(run[4 * i + 3], buf[bq][i].w);
+                }
+              }
+            }
+          }
+        }
+        epilogue_sync();  // last_flag is read before the next piece may set it
+      }
+      if (store && ok && n < N) {
+        const float sw = pow2f(-__ldg(w_exp + n));
+#pragma unroll
+        for (int cc = 0; cc < TN / 16; ++cc) {  // 16 tokens at a time: their loads in flight together
+          float cv[16];
+          int ex[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int64_t m = m0 + 16 * cc + i;
+            cv[i] = (C && m < c_rows && m < M) ? __ldcs(C + m * N + n) : 0.f;
+            ex[i] = m < M ? __ldg(x_exp + m) : 0;
+          }
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int64_t m = m0 + 16 * cc + i;
+            if (m < M) {
+              // exact power-of-two scaling: the weight row's exponent, then the token's
+              const float v = (run[16 * cc + i] * sw) * pow2f(-ex[i]);
+              out[m * N + n] = (C && m < c_rows) ? __fsub_rn(v, cv[i]) : v;
+            }
+          }
         }
       }
-    } else if (lane == 0) {
+      u = pe;
+    }
+    if (!ok && lane == 0) {
       *abort_flag = 1;
       atomicOr(&g_device_status, kStatusTimeout);
     }
   }
 
-  // ---- split K: the cluster's partial tiles summed in rank order, minus C, stored ----
   __syncwarp();
   tc_fence_before();
-  if (splits > 1) {
-    cluster_sync_all();  // every rank's partial tile is staged
-    const int rank = (int)cluster_rank();
-    const int tn_eff = (int)std::min<int64_t>(TN, M - m0);
-    const int per = (tn_eff + splits - 1) / splits;
-    const int t0 = std::min(tn_eff, rank * per), t1 = std::min(tn_eff, t0 + per);
-    const uint32_t red_base = smem_u32(red);
-    for (int idx = threadIdx.x; idx < (t1 - t0) * BM; idx += THREADS) {
-      const int rr = idx % BM, j = t0 + idx / BM;
-      const int64_t nn = n0 + rr, m = m0 + j;
-      if (nn >= N) continue;
-      const uint32_t off = red_base + (uint32_t)((rr * RS + j) * 4);
-      float v = ld_cluster_f32(map_to_rank(off, 0u));
-      for (int qq = 1; qq < splits; ++qq) v = __fadd_rn(v, ld_cluster_f32(map_to_rank(off, (uint32_t)qq)));
-      out[m * N + nn] = (C && m < c_rows) ? __fsub_rn(v, __ldcs(C + m * N + nn)) : v;
-    }
-    __syncwarp();
-    cluster_sync_all();  // no CTA leaves while others still read its shared memory
-  } else {
-    __syncthreads();
-  }
+  __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, L::TMEM_COLS);
@@ -1399,31 +1468,6 @@ int swap_width_index(int64_t tokens) {
   for (int i = 0; i < kSwapWidths; ++i)
     if (tokens <= kSwapTn[i]) return i;
   return kSwapWidths - 1;
-}
-
-// K-split of the swapped kernel for an online product of `tokens` rows.  The kernel streams W, and
-// on GB300 it streams fastest with about 1.6 CTAs per SM in flight (two fit on an SM): measured on
-// the eight Llama and Qwen projections at 16 rows, the best split put 120-304 CTAs on the 152 SMs
-// (0.50-0.79 of the HBM copy rate against 0.24-0.62 at one split per tile).  So s is the split
-// whose CTA count (weight tiles x token tiles x s) is nearest that in ratio, with at least 320 of K
-// per CTA; ties go to fewer splits.
-constexpr double kSwapCtasPerSm = 1.6;
-
-int swap_splits(int64_t tokens, int64_t K, int64_t N, int sms) {
-  const int w = swap_width_index(tokens);
-  const int64_t tiles = ceil_div(N, BM) * ceil_div(tokens, (int64_t)kSwapTn[w]);
-  const int max_s = (int)std::max<int64_t>(1, std::min<int64_t>(MAX_CLUSTER, K / 320));
-  const double target = kSwapCtasPerSm * (double)sms;
-  int best_s = 1;
-  double best = 1e300;
-  for (int s = 1; s <= max_s; ++s) {
-    const double c = std::fabs(std::log((double)(tiles * s) / target));
-    if (c < best - 1e-9) {
-      best = c;
-      best_s = s;
-    }
-  }
-  return best_s;
 }
 
 // The launch variants: tile width, ring size, CTAs per SM, and the cost constants of the
@@ -1702,64 +1746,80 @@ spl_status launch_variant(const LinearArgs& a, const uint16_t* hi, const uint16_
   }
 }
 
+// CTAs per token tile of the swapped kernel.  Measured on GB300 (the eight Llama and Qwen
+// projections at 8 and 16 rows): runs of whole tiles are fastest where the weight tiles number
+// between 3/4 of the SMs and all of them (one tile per CTA, no partial tiles: Qwen Gate|Up, 152
+// tiles); otherwise 3/4 of the SMs beat all of them by 0.3-1.5 us, fewer partial tiles to sum
+// outweighing the longer runs, and 1/2 of them lost 1-4 us.  More tiles than SMs: one CTA per SM.
+int swap_ctas(int64_t K, int64_t N, int sms) {
+  const int64_t w_tiles = ceil_div(N, BM);
+  const int64_t total = w_tiles * ceil_div(K, (int64_t)SwapCfg<16>::BK);
+  int64_t c = 3 * (int64_t)sms / 4;
+  if (w_tiles > sms) c = sms;
+  else if (4 * w_tiles >= 3 * (int64_t)sms) c = w_tiles;
+  return (int)std::max<int64_t>(1, std::min<int64_t>(c, total));
+}
+
+// Workspace of the swapped kernel's partial tiles: two slots per CTA and token tile of width tn.
+size_t swap_partial_bytes(int64_t rows, int tn, int ctas) {
+  return (size_t)round_up(ceil_div(rows, (int64_t)tn) * ctas * 2 * tn * BM * 4, 256);
+}
+
 template <int TN>
-spl_status launch_swap_tn(const LinearArgs& a, const uint16_t* x_hi, const uint16_t* x_lo, const int* x_exp,
-                          int splits) {
+spl_status launch_swap_tn(const LinearArgs& a, const uint16_t* x_hi, const uint16_t* x_lo, const int* x_exp, int ctas,
+                          float* part, size_t part_bytes) {
+  using L = SwapCfg<TN>;
   if (!set_smem_attr_swap<TN>()) return SPL_ECUDA;
+  const int64_t t_tiles = ceil_div(a.M, (int64_t)TN), w_tiles = ceil_div(a.N, BM);
+  const int64_t total = w_tiles * ceil_div(a.K, (int64_t)L::BK);
+  if (t_tiles * w_tiles > kMaxCounters || t_tiles > 65535) return SPL_ESHAPE;
+  if (ctas < 1) return SPL_EINVAL;
+  if (ctas > total) ctas = (int)total;  // every CTA at least one unit
+  if (!a.ws || !part || part_bytes < swap_partial_bytes(a.M, TN, ctas)) return SPL_EWORKSPACE;
   TcMaps maps;
   std::memset(&maps, 0, sizeof(maps));
-  if (!make_map(&maps.a_hi, x_hi, true, a.M, a.K, SwapCfg<TN>::BK, TN, CU_TENSOR_MAP_SWIZZLE_64B) ||
-      !make_map(&maps.a_lo, x_lo, true, a.M, a.K, SwapCfg<TN>::BK, TN, CU_TENSOR_MAP_SWIZZLE_64B) ||
-      !make_map(&maps.w_hi, a.w_h16, true, a.N, a.K, SwapCfg<TN>::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B) ||
-      !make_map(&maps.w_lo, a.w_l16, true, a.N, a.K, SwapCfg<TN>::BK, BM, CU_TENSOR_MAP_SWIZZLE_64B))
+  if (!make_map(&maps.a_hi, x_hi, true, a.M, a.K, L::BK, TN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&maps.a_lo, x_lo, true, a.M, a.K, L::BK, TN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&maps.w_hi, a.w_h16, true, a.N, a.K, L::BK, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map(&maps.w_lo, a.w_l16, true, a.N, a.K, L::BK, BM, CU_TENSOR_MAP_SWIZZLE_128B))
     return SPL_ECUDA;
-  const int m_tiles = (int)ceil_div(a.M, (int64_t)TN);
-  const int64_t tiles = (int64_t)m_tiles * ceil_div(a.N, BM);
-  if (tiles > 0x7fffffffLL) return SPL_ESHAPE;
-  const int64_t kps = round_up(ceil_div(a.K, splits), SwapCfg<TN>::BK);
-  const int chain = chain_segments<Fp16x3>(kps);
   cudaLaunchConfig_t cfg;
   std::memset(&cfg, 0, sizeof(cfg));
-  cfg.gridDim = dim3((unsigned)tiles, 1, (unsigned)splits);
+  cfg.gridDim = dim3((unsigned)ctas, (unsigned)t_tiles, 1);
   cfg.blockDim = dim3(THREADS, 1, 1);
-  cfg.dynamicSmemBytes = SwapCfg<TN>::SMEM;
+  cfg.dynamicSmemBytes = L::SMEM;
   cfg.stream = a.stream;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 1;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = (unsigned)splits;
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_swap_kernel<TN>, maps, a.out, a.c, x_exp, (const int*)a.w_exp,
-                                           a.M, a.K, a.N, kps, splits, m_tiles, chain, a.c_rows);
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, tc_swap_kernel<TN>, maps, a.out, a.c, x_exp, (const int*)a.w_exp, a.M,
+                                           a.K, a.N, ctas, a.c_rows, part, static_cast<unsigned int*>(a.ws));
   note_launches(1);
   return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
 }
 
-// The swapped kernel with token-tile width index w and a K-split of `splits` (FP16X3, split of the
-// tokens given).
+// The swapped kernel with token-tile width index w and `ctas` CTAs per token tile (FP16X3, split
+// of the tokens given); part: the workspace after the counters (and the split of A).
 spl_status launch_swap(const LinearArgs& a, const uint16_t* x_hi, const uint16_t* x_lo, const int* x_exp, int w,
-                       int splits) {
-  if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
+                       int ctas, float* part, size_t part_bytes) {
   switch (w) {
-    case 0: return launch_swap_tn<16>(a, x_hi, x_lo, x_exp, splits);
-    case 1: return launch_swap_tn<32>(a, x_hi, x_lo, x_exp, splits);
-    case 2: return launch_swap_tn<64>(a, x_hi, x_lo, x_exp, splits);
-    default: return launch_swap_tn<128>(a, x_hi, x_lo, x_exp, splits);
+    case 0: return launch_swap_tn<16>(a, x_hi, x_lo, x_exp, ctas, part, part_bytes);
+    case 1: return launch_swap_tn<32>(a, x_hi, x_lo, x_exp, ctas, part, part_bytes);
+    case 2: return launch_swap_tn<64>(a, x_hi, x_lo, x_exp, ctas, part, part_bytes);
+    default: return launch_swap_tn<128>(a, x_hi, x_lo, x_exp, ctas, part, part_bytes);
   }
 }
 
 // forced_v >= 0: every tile with that variant, the first forced_full tiles unsplit in a launch of their own
 // and the rest with K split forced_splits ways (one launch when forced_full is 0).
 // seg_splits > 0: segmented mode, one unsplit launch whose sums follow a seg_splits-way split.
-// swap_w >= 0: the swapped kernel with that token-tile width index and a K-split of swap_s (0: the
-// online product's split for a.M tokens, or for swap_order tokens when swap_order > 0 -- the bank).
+// swap_w >= 0: the swapped kernel with that token-tile width index and swap_s CTAs per token tile
+// (0: the library's count, which depends on K and N only, so a bank of any width meets the online
+// product's runs).
 spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int forced_splits, int seg_splits = 0,
-                       int64_t forced_full = 0, bool forced_persistent = false, int swap_w = -1, int swap_s = 0,
-                       int64_t swap_order = 0) {
+                       int64_t forced_full = 0, bool forced_persistent = false, int swap_w = -1, int swap_s = 0) {
   const int cc = device_cc();
   if (cc != 100 && cc != 103) return SPL_EUNSUPPORTED;
   const bool f16 = a.path == SPL_PATH_FP16X3;
@@ -1807,11 +1867,13 @@ spl_status run_tc_impl(const LinearArgs& a, int skip_kblock, int forced_v, int f
     a_hi = hi_;
     a_lo = lo_;
   }
-  if (swap_w >= 0) {
+  if (swap_w >= 0) {  // the swapped kernel; its partial tiles after the counters (and the split of A)
     if (!f16) return SPL_EUNSUPPORTED;
-    int sp = swap_s;
-    if (sp <= 0) sp = swap_splits(swap_order > 0 ? swap_order : a.M, a.K, a.N, device_sm_count());
-    return launch_swap(a, static_cast<const uint16_t*>(a_hi), static_cast<const uint16_t*>(a_lo), a_exp, swap_w, sp);
+    const int ctas = swap_s > 0 ? swap_s : swap_ctas(a.K, a.N, device_sm_count());
+    const size_t off = kCounterBytes + (presplit ? 0 : tc_asplit_bytes(a.M, a.K, a.path));
+    if (!a.ws || a.ws_bytes < off) return SPL_EWORKSPACE;
+    return launch_swap(a, static_cast<const uint16_t*>(a_hi), static_cast<const uint16_t*>(a_lo), a_exp, swap_w, ctas,
+                       reinterpret_cast<float*>(static_cast<char*>(a.ws) + off), a.ws_bytes - off);
   }
   TcShape shape;
   if (forced_v >= 0) {
@@ -1843,14 +1905,22 @@ Plan plan_tc(int64_t M, int64_t K, int64_t N, int sms, spl_path path) {
   Plan p{};
   p.kernel = kKernelTc;
   if (tc_swapped(M, path)) {
-    p.splits = swap_splits(M, K, N, sms);
+    p.splits = 1;  // runs of k-blocks, partial tiles summed through the workspace
+    p.ws_partials = tc_partial_bytes(M, K, N, M, path);
   } else {
     const TcShape t = tc_shape(M, K, N, sms);
-    p.splits = t.rest_splits;
+    p.splits = t.rest_splits;  // partials are reduced through distributed shared memory
   }
   p.k_per_split = ceil_div(K, p.splits);
-  p.ws_asplit = tc_asplit_bytes(M, K, path);  // partials are reduced through distributed shared memory
+  p.ws_asplit = tc_asplit_bytes(M, K, path);
   return p;
+}
+
+size_t tc_partial_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows, spl_path path) {
+  if (!tc_swapped(order_rows, path) || M <= 0 || K <= 0 || N <= 0) return 0;
+  const int64_t total = ceil_div(N, BM) * ceil_div(K, (int64_t)SwapCfg<16>::BK);
+  const int ctas = (int)std::min<int64_t>(swap_ctas(K, N, device_sm_count()), total);
+  return swap_partial_bytes(M, kSwapTn[swap_width_index(M)], ctas);
 }
 
 spl_status run_tc(const LinearArgs& a, const Plan& p) {
@@ -1862,7 +1932,7 @@ spl_status run_tc(const LinearArgs& a, const Plan& p) {
 bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, spl_path path, int* variant, int* splits) {
   if (tc_swapped(M, path)) {  // one launch of the swapped kernel
     *variant = -1;
-    *splits = swap_splits(M, K, N, device_sm_count());
+    *splits = 1;
     return true;
   }
   const TcShape t = tc_shape(M, K, N, device_sm_count());
@@ -1873,8 +1943,8 @@ bool tc_uniform_shape(int64_t M, int64_t K, int64_t N, spl_path path, int* varia
 }
 
 spl_status run_tc_matched(const LinearArgs& a, int64_t order_rows) {
-  if (tc_swapped(order_rows, a.path))  // the swapped kernel with the online split; a width for all of M
-    return run_tc_impl(a, -1, -1, 0, 0, 0, false, swap_width_index(a.M), 0, order_rows);
+  if (tc_swapped(order_rows, a.path))  // the swapped kernel with the online runs; a width for all of M
+    return run_tc_impl(a, -1, -1, 0, 0, 0, false, swap_width_index(a.M), 0);
   int variant = 0, splits = 1;
   if (!tc_uniform_shape(order_rows, a.K, a.N, a.path, &variant, &splits)) return SPL_EINVAL;
   if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
@@ -1958,21 +2028,33 @@ extern "C" spl_status spl_test_tc_product(float* out, const float* A, const spl_
 }
 
 // Test hook: the swapped tensor-core product (FP16X3, the weight in the MMA's rows, the tokens in its
-// columns) with a fixed token-tile width (16, 32, 64 or 128) and K-split (1-8), whatever M is,
-// so that tests cover every kernel instance and compare widths bit for bit.  The paper has no
-// counterpart.
+// columns) with a fixed token-tile width (16, 32, 64 or 128) and `ctas` CTAs per token tile (0: the
+// library's count), whatever M is, so that tests cover every kernel instance and compare widths and
+// run lengths.  The paper has no counterpart.
 extern "C" spl_status spl_test_tc_swap_product(float* out, const float* A, const spl_weight* W, const float* C,
-                                               int64_t M, int64_t K, int64_t N, int tile_tokens, int splits,
+                                               int64_t M, int64_t K, int64_t N, int tile_tokens, int ctas,
                                                void* workspace, size_t workspace_bytes, cudaStream_t stream) {
   using namespace spl;
-  if (!out || !A || !W || !W->w || M <= 0 || N <= 0 || K <= 0) return SPL_EINVAL;
+  if (!out || !A || !W || !W->w || M <= 0 || N <= 0 || K <= 0 || ctas < 0) return SPL_EINVAL;
   int w = -1;
   for (int i = 0; i < kSwapWidths; ++i)
     if (kSwapTn[i] == tile_tokens) w = i;
   if (w < 0) return SPL_EINVAL;
-  if (splits < 1 || splits > MAX_CLUSTER) return SPL_ESHAPE;
   if ((K & 7) != 0) return SPL_EALIGN;
   if (!aligned16(out) || !aligned16(A) || (C && !aligned16(C))) return SPL_EALIGN;
   const LinearArgs args = make_args(out, A, *W, C, M, K, N, workspace, workspace_bytes, stream, SPL_PATH_FP16X3);
-  return run_tc_impl(args, -1, -1, 0, 0, 0, false, w, splits);
+  return run_tc_impl(args, -1, -1, 0, 0, 0, false, w, ctas);
+}
+
+// Workspace bytes spl_test_tc_swap_product needs for these arguments: the counters, the split of A
+// and the partial tiles.  0 for arguments it refuses.
+extern "C" size_t spl_test_tc_swap_workspace_bytes(int64_t M, int64_t K, int64_t N, int tile_tokens, int ctas) {
+  using namespace spl;
+  if (M <= 0 || K <= 0 || N <= 0 || ctas < 0) return 0;
+  bool listed = false;
+  for (int i = 0; i < kSwapWidths; ++i) listed = listed || kSwapTn[i] == tile_tokens;
+  if (!listed) return 0;
+  const int64_t total = ceil_div(N, BM) * ceil_div(K, (int64_t)SwapCfg<16>::BK);
+  const int p = (int)std::min<int64_t>(total, ctas > 0 ? ctas : swap_ctas(K, N, device_sm_count()));
+  return kCounterBytes + tc_asplit_bytes(M, K, SPL_PATH_FP16X3) + swap_partial_bytes(M, tile_tokens, p);
 }

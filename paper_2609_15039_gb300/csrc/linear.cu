@@ -90,7 +90,9 @@ spl_status run_linear(float* out, const float* a, const spl_weight* W, const flo
   if (!a && resolved != SPL_PATH_FP16X3) return SPL_EINVAL;  // only FP16X3 reads the split alone
   const bool use_split = a_split && resolved == SPL_PATH_FP16X3;
   const Plan plan = make_plan(M, K, N, resolved);
-  if (!use_split && plan.total() > 0 && (!ws || ws_bytes < plan.total())) return SPL_EWORKSPACE;
+  // a pre-split operand needs only the counters and partial tiles (the split of A is not written)
+  const size_t need = use_split ? (plan.ws_partials ? kCounterBytes + plan.ws_partials : 0) : plan.total();
+  if (need > 0 && (!ws || ws_bytes < need)) return SPL_EWORKSPACE;
   if (ws && !aligned16(ws)) return SPL_EALIGN;
   LinearArgs args = make_args(out, a, *W, C, M, K, N, ws, ws_bytes, stream, resolved);
   if (c_rows >= 0) {  // only the first c_rows output rows subtract C (tensor-core and decode kernels)
@@ -129,7 +131,7 @@ MatchedPlan matched_plan(int64_t M, int64_t K, int64_t N, int64_t order_rows, sp
   if (online.kernel == kKernelTc) {
     int variant = 0;  // the bank runs its own launch shape; only the K-split order carries over
     if (!tc_uniform_shape(order_rows, K, N, resolved, &variant, &mp.splits)) return mp;
-    mp.ws = kCounterBytes + tc_asplit_bytes(M, K, resolved);
+    mp.ws = kCounterBytes + tc_asplit_bytes(M, K, resolved) + tc_partial_bytes(M, K, N, order_rows, resolved);
     mp.ok = true;
     return mp;
   }
@@ -284,6 +286,23 @@ extern "C" spl_status spl_noise_mask_linear_unmask(float* Y, float* Xt, const fl
   nz.offset = rng.offset;
   nz.offset_dev = rng.offset_dev;
   return run_linear(Y, X, W, C, true, M, K, N, path, workspace, workspace_bytes, stream, nullptr, &nz);
+}
+
+extern "C" size_t spl_split_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows, spl_path path) {
+  if (M <= 0 || K <= 0 || N <= 0 || order_rows <= 0 || !valid_path(path)) return 0;
+  size_t need = 0;
+  const spl_path paths[3] = {SPL_PATH_FP32, SPL_PATH_TF32X3, SPL_PATH_FP16X3};
+  for (spl_path p : paths) {
+    if (path != SPL_PATH_AUTO && path != p) continue;
+    if (p == SPL_PATH_FP16X3) {  // the split is read as given: counters and partial tiles only
+      const size_t part = tc_partial_bytes(M, K, N, order_rows, p);
+      need = std::max(need, part ? kCounterBytes + part : (size_t)0);
+    } else {  // these paths read the fp32 operand
+      const MatchedPlan mp = matched_plan(M, K, N, order_rows, p);
+      need = std::max(need, order_rows == M ? make_plan(M, K, N, p).total() : (mp.ok ? mp.ws : make_plan(M, K, N, p).total()));
+    }
+  }
+  return need;
 }
 
 extern "C" size_t spl_precompute_matched_workspace_bytes(int64_t M, int64_t K, int64_t N, int64_t order_rows,

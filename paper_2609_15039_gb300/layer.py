@@ -319,9 +319,11 @@ class MaskedLayer:
                parallel=False, parity=0, ahead=0, workspace=None):
         """a2 + a4: draw ``draws`` masks per group and precompute their corrections in one product.
 
-        parallel: the FP16X3 groups' corrections (which use no workspace: the noise comes split and
-        the tensor-core kernel reduces on chip) run side by side on streams of their own, so the
-        tiles of one fill the SMs another leaves idle; the current stream waits for all of them.
+        parallel: the FP16X3 groups' corrections that need no workspace (the noise comes split and
+        the tensor-core kernel reduces on chip: spl_split_workspace_bytes is 0) run side by side on
+        streams of their own, so the tiles of one fill the SMs another leaves idle; the others (the
+        swapped kernel of few rows, which sums partial tiles through the workspace) run in order on
+        the current stream.  The current stream waits for all of them.
         parity: the correction buffer to fill (see enable_overlap); ahead: the draws of cycle
         ``cycle + ahead`` (with device_base: that many cycles past the device-side base).
         workspace: the workspace of the corrections that take one (default: the layer's), e.g. a
@@ -338,7 +340,7 @@ class MaskedLayer:
             es = b.get("es") if self._fused_split(g, path, self.M) else None
             if es is not None:  # the FP16X3 correction reads only the split: the noise is split as drawn
                 side = main
-                if parallel:
+                if parallel and spl.spl_split_workspace_bytes(self.draws * self.M, g.K, g.N, self.M, "fp16x3") == 0:
                     side = self._side_stream(gi)
                     side.wait_stream(main)
                     forks.append(side)
@@ -351,7 +353,7 @@ class MaskedLayer:
                         timer("begin", "precompute", g.name)
                     spl.spl_precompute_noise_product_matched_split(C, es, g.wt, self.M,
                                                                    path=self.path_of(g, path, self.M),
-                                                                   workspace=self.workspace, stream=side)
+                                                                   workspace=ws, stream=side)
                     if timer:
                         timer("end", "precompute", g.name)
                 continue
@@ -482,11 +484,12 @@ class MaskedLayer:
         graphs[c % 2] for cycle c after set_cycle(c) and a refill of buffer c % 2 for cycle c.
         ``before(d)`` / ``after(d)`` / ``group_hooks`` as in capture; ``inputs`` may be a list
         (step d reads inputs[d % len(inputs)]).  Returns the graphs and their kernel counts."""
-        # the two sides must not share the workspace: every group's online product and correction
-        # take the fp16 split (on-chip reductions, no workspace)
+        # the two sides must not share the workspace: the corrections take a workspace of their own
         if not all(self._fused_split(g, path, self.M) for g in self.groups):
             raise ValueError("capture_overlapped needs every group on FP16X3 with the fused split")
         self.enable_overlap()
+        if not hasattr(self, "_bank_ws"):
+            self._bank_ws = spl.workspace(self.workspace_bytes(self.M, self.draws), self.groups[0].W.device)
         lo, hi = torch.cuda.Stream.priority_range()
         if not hasattr(self, "_bank_stream"):
             self._bank_stream = torch.cuda.Stream(priority=lo)
@@ -500,7 +503,7 @@ class MaskedLayer:
                 self._bank_stream.wait_stream(main)
                 with torch.cuda.stream(self._bank_stream):
                     self.refill(eps, mech, seed, 0, path=path, device_base=True, parallel=True, parity=1 - parity,
-                                ahead=1)
+                                ahead=1, workspace=self._bank_ws)
                 for d in range(self.draws):
                     if before:
                         before(d)

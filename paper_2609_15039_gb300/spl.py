@@ -71,6 +71,7 @@ _SIGS = {
     "spl_masked_linear": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_precompute_noise_product": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_precompute_matched_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I64, _I]),
+    "spl_split_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I64, _I]),
     "spl_precompute_noise_product_matched": (_I, [_P, _P, _PW, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_precompute_noise_product_matched_split": (_I, [_P, _PW, _PW, _I64, _I64, _I64, _I64, _I, _P, _SZ, _P]),
     "spl_unmask": (_I, [_P, _P, _P, _I64, _I64, _P]),
@@ -81,6 +82,7 @@ _SIGS = {
                                           _P]),
     "spl_noise_mask_linear_unmask_precompute": (_I, [_P, _P, _P, _PW, _P, _I64, _I64, _I64, _I64, _D, _D, _I,
                                                      spl_rng, ctypes.c_uint64, _I, _P, _SZ, _P]),
+    "spl_test_tc_swap_workspace_bytes": (_SZ, [_I64, _I64, _I64, _I, _I]),
     "spl_delta_layernorm": (_D, [_P, _I64]),
     "spl_delta_attention": (_D, [_P, _I64, _D]),
     "spl_delta_activation": (_D, [_P, _P, _I64, _I64, _D, _D]),
@@ -458,6 +460,13 @@ def spl_precompute_noise_product(C, Nz, W, path="auto", workspace=None, stream=N
             stream)
 
 
+def spl_split_workspace_bytes(M, K, N, order_rows=None, path="auto"):
+    """Workspace bytes of a product (or a correction in the order of order_rows rows) whose left
+    operand comes split; 0 when the kernel reduces on chip (see include/spl.h)."""
+    return int(lib().spl_split_workspace_bytes(int(M), int(K), int(N), int(M if order_rows is None else order_rows),
+                                               _path(path)))
+
+
 def spl_precompute_matched_workspace_bytes(M, K, N, order_rows, path="auto"):
     return int(lib().spl_precompute_matched_workspace_bytes(M, K, N, order_rows, _path(path)))
 
@@ -672,19 +681,24 @@ def spl_test_tc_product(Y, Xt, W, C=None, path="fp16x3", tile_n=256, ring_kb=192
            "spl_test_tc_product")
 
 
-def spl_test_tc_swap_product(Y, Xt, W, C=None, tile_tokens=16, splits=1, workspace=None, stream=None):
-    """The FP16X3 product on the swapped kernel with a fixed token-tile width and K-split (a test hook)."""
+def spl_test_tc_swap_workspace_bytes(M, K, N, tile_tokens=16, ctas=0):
+    return int(lib().spl_test_tc_swap_workspace_bytes(int(M), int(K), int(N), int(tile_tokens), int(ctas)))
+
+
+def spl_test_tc_swap_product(Y, Xt, W, C=None, tile_tokens=16, ctas=0, workspace=None, stream=None):
+    """The FP16X3 product on the swapped kernel with a fixed token-tile width and CTA count per token
+    tile (0: the library's), a test hook."""
     W = _weight(W)
     M, K = _rows_cols(Xt)
     N = W.shape[0]
     if W.shape[-1] != K or Y.numel() != M * N or (C is not None and C.numel() != M * N):
         raise ValueError("spl_test_tc_swap_product: shape mismatch")
     if workspace is None:
-        workspace = globals()["workspace"](spl_linear_workspace_bytes(M, K, N, "fp16x3"), Xt.device)
+        workspace = globals()["workspace"](spl_test_tc_swap_workspace_bytes(M, K, N, tile_tokens, ctas), Xt.device)
     wsp, wsb = _ws(workspace)
     ws_ = W.c_struct()
     _check(lib().spl_test_tc_swap_product(_dev(Y, "Y"), _dev(Xt, "Xt"), ctypes.byref(ws_), _dev(C, "C"), M, K, N,
-                                          int(tile_tokens), int(splits), wsp, wsb, _stream(stream)),
+                                          int(tile_tokens), int(ctas), wsp, wsb, _stream(stream)),
            "spl_test_tc_swap_product")
 
 

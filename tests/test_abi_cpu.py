@@ -177,7 +177,11 @@ def test_precompute_and_swap_entries_validate_without_launch(spl):
     assert call(base, base + 128, base, 1, 1, rng_=spl.spl_rng(1, 0, 0, base + 4)) == spl.SPL_EALIGN  # offset_dev
     swap = L.spl_test_tc_swap_product
     assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 24, 1, None, 0, None) == spl.SPL_EINVAL  # width
-    assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 16, 9, None, 0, None) == spl.SPL_ESHAPE  # splits
+    assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 16, -1, None, 0, None) == spl.SPL_EINVAL  # ctas
+    # valid arguments reach the device check: no tensor-core device here
+    assert swap(base, base, ctypes.byref(w), None, 2, 8, 4, 16, 0, None, 0, None) == spl.SPL_EUNSUPPORTED
+    assert L.spl_test_tc_swap_workspace_bytes(2, 8, 4, 24, 0) == 0  # width not listed
+    assert L.spl_test_tc_swap_workspace_bytes(2, 64, 256, 16, 3) >= 64 * 1024 + 2 * 2 * 16 * 128 * 4
     assert swap(base, base, ctypes.byref(w), None, 2, 12, 4, 16, 1, None, 0, None) == spl.SPL_EALIGN  # K % 8
     assert swap(base, base, None, None, 2, 8, 4, 16, 1, None, 0, None) == spl.SPL_EINVAL
 

@@ -264,48 +264,57 @@ SWAP_WIDTHS = [16, 32, 64, 128]
 
 
 @pytest.mark.parametrize("M", [9, 16, 33, 64])
-@pytest.mark.parametrize("splits", [1, 3, 8])
-def test_swap_every_width_and_split(spl, M, splits):
+@pytest.mark.parametrize("ctas", [0, 1, 7, 40])
+def test_swap_every_width_and_run_length(spl, M, ctas):
     """The swapped kernel (weight rows in the MMA's 128 rows, tokens in its N) at every token-tile
-    width and cluster K-split, ragged M, K and N (tokens past M are the copy's zero rows): within the
-    product tolerance of the oracle, with and without C, and the same bits at every width -- an
-    output's sum does not depend on the other columns of its MMA, which the bank relies on."""
+    width and run length (1 CTA: one run over every tile, whole tiles straight out; 7 and 40: runs
+    that cut tiles into pieces summed through the workspace), ragged M, K and N (tokens past M are
+    the copy's zero rows): within the product tolerance of the oracle, with and without C, and the
+    same bits at every width -- an output's sum does not depend on the other columns of its MMA,
+    which the bank relies on."""
     K, N = 1032, 600
     W, Wt = _weights(spl, N, K, seed=81)
     A = (wl.activations(M, K, seed=82 + M).numpy() * 300).astype(np.float32)
     C = wl.activations(M, N, seed=83).numpy()
-    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp16x3"))
+    ws = spl.workspace(max(spl.spl_test_tc_swap_workspace_bytes(M, K, N, tn, ctas) for tn in SWAP_WIDTHS))
     first = None
     for tn in SWAP_WIDTHS:
         Y = torch.full((M, N), float("nan"), device="cuda")
-        spl.spl_test_tc_swap_product(Y, dev(A), Wt, dev(C), tile_tokens=tn, splits=splits, workspace=ws)
-        assert_product_close(f32(Y), A, W, "fp16x3", C=C, what=f"swap {tn} split {splits}")
+        spl.spl_test_tc_swap_product(Y, dev(A), Wt, dev(C), tile_tokens=tn, ctas=ctas, workspace=ws)
+        assert_product_close(f32(Y), A, W, "fp16x3", C=C, what=f"swap {tn} ctas {ctas}")
         if first is None:
             first = Y
         assert torch.equal(Y, first), (tn, float((Y - first).abs().max()))
     Y2 = torch.full((M, N), float("nan"), device="cuda")
-    spl.spl_test_tc_swap_product(Y2, dev(A), Wt, None, tile_tokens=16 if M <= 16 else 64, splits=splits, workspace=ws)
+    spl.spl_test_tc_swap_product(Y2, dev(A), Wt, None, tile_tokens=16 if M <= 16 else 64, ctas=ctas, workspace=ws)
     assert_product_close(f32(Y2), A, W, "fp16x3", what="swap without C")
     assert spl.spl_get_device_status() == 0
 
 
 def test_library_takes_the_swapped_kernel_for_few_rows(spl):
-    """AUTO runs 9-32 rows on the swapped kernel: the library's product equals the swapped kernel's
-    bit for bit (at the width of the rows and the split the library picks)."""
+    """AUTO runs 9-16 rows on the swapped kernel: the library's product equals the swapped kernel's
+    bit for bit (at the width of the rows and the library's run length), also on the operand split
+    beforehand (the layers' form); from 17 rows on it takes the 128-row tiles."""
     K, N = 3072, 5120
     W, Wt = _weights(spl, N, K, seed=91)
-    for M in (9, 16, 25, 32):
+    for M in (9, 16, 17):
         A = wl.activations(M, K, seed=92 + M).numpy()
         ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N))
         Y = torch.empty((M, N), device="cuda")
         spl.spl_masked_linear(Y, dev(A), Wt, workspace=ws)
         tn = next(t for t in SWAP_WIDTHS if M <= t)
-        hits = 0
-        for splits in range(1, 9):
-            Ys = torch.empty((M, N), device="cuda")
-            spl.spl_test_tc_swap_product(Ys, dev(A), Wt, None, tile_tokens=tn, splits=splits, workspace=ws)
-            hits += int(torch.equal(Y, Ys))
-        assert hits >= 1, M  # some split of the swapped kernel is exactly what the library ran
+        Ys = torch.empty((M, N), device="cuda")
+        spl.spl_test_tc_swap_product(Ys, dev(A), Wt, None, tile_tokens=tn, ctas=0,
+                                     workspace=spl.workspace(spl.spl_test_tc_swap_workspace_bytes(M, K, N, tn, 0)))
+        assert torch.equal(Y, Ys) == (M <= 16), M
+        if M <= 16:  # the pre-split operand
+            hi = torch.empty((M, K), dtype=torch.int16, device="cuda")
+            lo, ex = torch.empty_like(hi), torch.empty(M, dtype=torch.int32, device="cuda")
+            spl.spl_split_fp16(hi, lo, ex, dev(A))
+            Yp = torch.empty((M, N), device="cuda")
+            spl.spl_masked_linear_unmask_split(Yp, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt,
+                                               torch.zeros((M, N), device="cuda"), workspace=ws)
+            assert torch.equal(Yp, Y)
     assert spl.spl_get_device_status() == 0
 
 
@@ -839,9 +848,19 @@ def test_presplit_product_equals_plain(spl, M, K, N):
     spl.spl_masked_linear_unmask(Y_plain, xt, Wt, C, path="fp16x3", workspace=ws)
     spl.spl_masked_linear_unmask_split(Y_split, spl.Weight(xt, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, C,
                                        path="fp16x3", workspace=ws)
+    # the split operand needs no room for its split: the kernels that reduce on chip take no workspace,
+    # the swapped kernel of 9-16 rows only its counters and partial tiles
+    need = spl.spl_split_workspace_bytes(M, K, N, path="fp16x3")
+    assert (need > 0) == (M <= 16)
+    assert need < spl.spl_linear_workspace_bytes(M, K, N, "fp16x3") or need == 0
     spl.spl_masked_linear_unmask_split(Y_none, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, C,
-                                       path="fp16x3", workspace=None)
+                                       path="fp16x3", workspace=spl.workspace(need) if need else None)
     assert torch.equal(Y_plain, Y_split) and torch.equal(Y_plain, Y_none)
+    if need:
+        with pytest.raises(spl.SplError) as e:  # the partial tiles need their room
+            spl.spl_masked_linear_unmask_split(Y_none, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, C,
+                                               path="fp16x3", workspace=None)
+        assert e.value.status == spl.SPL_EWORKSPACE
     with pytest.raises(spl.SplError) as e:  # FP32 reads the fp32 X~, which is absent
         spl.spl_masked_linear_unmask_split(Y_none, spl.Weight(None, f16_hi=hi, f16_lo=lo, f16_exp=ex), Wt, C,
                                            path="fp32", workspace=ws)

@@ -109,14 +109,16 @@ def test_every_tc_launch_form_at_full_k(spl, problems, K, path, tile_n, ring_kb)
 
 @pytest.mark.parametrize("K", FULL_K)
 @pytest.mark.parametrize("tn", [16, 64, 128])
-@pytest.mark.parametrize("splits", [1, 3, 8])
-def test_swap_forms_at_full_k(spl, problems, K, tn, splits):
-    """The swapped kernel of few rows (weight in the MMA's rows, tokens in its columns) at 40 tokens."""
+@pytest.mark.parametrize("ctas", [0, 1, 57])
+def test_swap_forms_at_full_k(spl, problems, K, tn, ctas):
+    """The swapped kernel of few rows (weight in the MMA's rows, tokens in its columns) at 40 tokens:
+    the library's run length, one run over all of K (chains folded over whole tiles), and runs
+    cutting tiles into pieces summed through the workspace."""
     A, W, Wt = problems[K]
     A = np.ascontiguousarray(A[:40])
     Y = torch.full((40, W.shape[0]), float("nan"), device="cuda")
-    spl.spl_test_tc_swap_product(Y, dev(A), Wt, None, tile_tokens=tn, splits=splits)
-    check(f32(Y), A, W, K, f"swap {tn} split {splits}")
+    spl.spl_test_tc_swap_product(Y, dev(A), Wt, None, tile_tokens=tn, ctas=ctas)
+    check(f32(Y), A, W, K, f"swap {tn} ctas {ctas}")
 
 
 @pytest.mark.parametrize("K", FULL_K)
