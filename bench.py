@@ -70,6 +70,9 @@ def parse(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-decode", action="store_true", help="stack: skip the one-token decode measurement")
     ap.add_argument("--decode-steps", type=int, default=256)
+    ap.add_argument("--rows", type=str, default=None,
+                    help="qwen_sweep: comma-separated row counts (default 1,4,16,64,256,1024; the mask measured "
+                         "on 10^9 elements only with the default)")
     ap.add_argument("--schedule", choices=["stacked", "banked"], default="stacked",
                     help="stack workload: stacked (each product also computes the next cycle's correction of its "
                          "draw) or banked (the next cycle's banks of 1/8 of the layers beside each step)")
@@ -287,7 +290,10 @@ def run_workload(args):
     world, rank, local = dist_env()
     torch.cuda.set_device(local)
     with ClockSampler(local) as clocks:
-        res = measure.WORKLOADS[args.workload]()
+        if args.workload == "qwen_sweep" and args.rows:
+            res = measure.qwen_sweep(Ms=tuple(int(m) for m in args.rows.split(",")), mask_elements=10 ** 6)
+        else:
+            res = measure.WORKLOADS[args.workload]()
     if args.workload == "llama_stack_detail":
         value, unit, ms = res["prefill"]["tflops"], UNIT, res["prefill"]["ms_per_prefill"]
     elif args.workload == "qwen_stack":
@@ -719,7 +725,9 @@ def run_llama_stack(args):
         steps = max(D, args.decode_steps)
         stack.start_stacked(1, dgraphs)
         _time_graphs(dgraph_of, D, 2 * D, stream)  # cycles 1 and 2
+        torch.cuda.nvtx.range_push("decode")
         times = _time_graphs(dgraph_of, 3 * D, steps, stream)
+        torch.cuda.nvtx.range_pop()
         step_ms = sum(times) / steps
         dpaths = {g.name: layer0.stacked[g.name]["path"] for g in groups}
         step_bytes = sum(4 * g.K * g.N + 12 * g.K + 12 * g.N for g in groups) * L
