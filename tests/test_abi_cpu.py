@@ -186,6 +186,21 @@ def test_precompute_and_swap_entries_validate_without_launch(spl):
     assert swap(base, base, None, None, 2, 8, 4, 16, 1, None, 0, None) == spl.SPL_EINVAL
 
 
+def test_split_operand_workspace(spl):
+    """A product given its left operand split needs only the swapped kernel's counters and partial
+    tiles (9-16 rows on FP16X3) and nothing for the kernels that reduce on chip; invalid arguments
+    ask for nothing."""
+    few = spl.spl_split_workspace_bytes(16, 3072, 5120, path="fp16x3")
+    assert few >= 64 * 1024 + 2 * 16 * 128 * 4
+    assert few < spl.spl_linear_workspace_bytes(16, 3072, 5120, "fp16x3")  # no room for the split itself
+    assert spl.spl_split_workspace_bytes(128, 3072, 5120, path="fp16x3") == 0
+    assert spl.spl_split_workspace_bytes(1024, 3072, 5120, 512, path="fp16x3") == 0
+    # a bank of 8 draws in the order of 16-row products: the wider token tile's partial tiles
+    assert spl.spl_split_workspace_bytes(128, 3072, 5120, 16, path="fp16x3") > few
+    assert spl.spl_split_workspace_bytes(0, 3072, 5120, path="fp16x3") == 0
+    assert spl.spl_split_workspace_bytes(16, 3072, 5120, path=9) == 0
+
+
 def test_workspace_sizes_are_consistent(spl):
     # decode shapes need split-K partials after the 64 KiB counter region; the tensor-core
     # kernels reduce split-K in a cluster and keep only the split of the left operand there
