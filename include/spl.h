@@ -199,14 +199,18 @@ spl_path spl_resolve_path(int64_t M, int64_t K, int64_t N, spl_path path);
 
 /* Bytes of device workspace the three product calls below need for this
  * problem on the current device (0 if none; for AUTO the largest over the
- * paths).  Layout: the first 64 KiB hold the decode kernel's arrival
- * counters, then either split-K partial sums (FP32 kernels) or the split of
- * the left operand for the tensor-core paths (TF32X3: hi and lo in fp32;
- * FP16X3: one power-of-two exponent per row, hi and lo in fp16).  It must be
- * zero-filled before its first use; every call that
+ * paths).  Layout: the first 64 KiB hold the arrival counters of the decode
+ * kernel and of the swapped few-row kernel, then either split-K partial sums
+ * (FP32 kernels) or the split of the left operand for the tensor-core paths
+ * (TF32X3: hi and lo in fp32; FP16X3: one power-of-two exponent per row, hi
+ * and lo in fp16), followed for 9-16 rows on FP16X3 by the swapped kernel's
+ * partial tiles.  It must be zero-filled before its first use; every call that
  * returns SPL_OK leaves the counters at zero again, so one workspace (sized
- * for the largest call) serves calls of any shape and path.  Calls that can
- * run concurrently must not share a workspace. */
+ * for the largest call) serves calls of any shape and path.  After a call
+ * whose kernels gave up a bounded wait (spl_get_device_status returns
+ * SPL_ETIMEOUT) the counters may not be zero: zero the first 64 KiB again
+ * before the workspace is reused.  Calls that can run concurrently must not
+ * share a workspace. */
 size_t spl_linear_workspace_bytes(int64_t M, int64_t K, int64_t N, spl_path path);
 
 /* ---- a5: masked product -----------------------------------------------
