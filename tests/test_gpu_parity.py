@@ -470,7 +470,8 @@ def test_matched_correction_cancels_rounding(spl, M, K, N, path):
                                          (1, 3072, 5120, "fp32"), (1, 3072, 16384, "fp32"), (1, 8192, 3072, "fp32"),
                                          (4, 3072, 5120, "fp32"), (3, 1028, 600, "fp32"),
                                          (16, 3072, 5120, "fp16x3"), (16, 9728, 2560, "fp16x3"),
-                                         (32, 2560, 19456, "fp16x3"), (12, 1032, 600, "fp16x3")])
+                                         (16, 3072, 16384, "fp16x3"), (32, 2560, 19456, "fp16x3"),
+                                         (12, 1032, 600, "fp16x3")])
 @pytest.mark.parametrize("draws", [4, 8])
 def test_matched_correction_is_the_online_order_bitwise(spl, M, K, N, path, draws):
     """The bank's correction of draw d is, bit for bit, what the online product computes when
