@@ -194,6 +194,40 @@ def test_layer_production_paths_noise_free(spl, model_name, M):
     assert spl.spl_get_device_status() == 0
 
 
+@pytest.mark.parametrize("model_name,M", [("llama", 512), ("qwen", 8), ("llama", 1), ("qwen", 1)])
+def test_stacked_production_paths_noise_free(spl, model_name, M):
+    """The stacked schedule the bench times, eps = inf: every call multiplies the step's M rows and the
+    next cycle's M noise rows (here zero) -- 1024-row tensor-core calls (Llama 512), the swapped kernel
+    at 16 rows (Qwen 8), the one-launch decode kernel at 2 rows (M = 1) -- and the noise rows' outputs,
+    the next cycle's corrections, are exactly zero; sampled outputs of every projection within 1e-5."""
+    from paper_2609_15039_gb300.layer import MaskedLayer
+    model = wl.LLAMA_3_2_3B if model_name == "llama" else wl.QWEN3_4B
+    weights = {name: wl.weight(N, K, seed=wl.layer_seed(19, 0, pi), device="cuda")
+               for pi, (name, K, N, g) in enumerate(model.projections())}
+    layer = MaskedLayer.from_weights(model, weights)
+    layer.deltas = {g: 825.3 for g, _k, _n in model.input_groups()}
+    layer.allocate_stacked(M, 2)
+    inputs = {g: wl.activations(M, K, seed=wl.layer_seed(19, 0, 50 + gi), device="cuda")
+              for gi, (g, K, _n) in enumerate(model.input_groups())}
+    eps, mech, seed = float("inf"), "gaussian", 7
+    for cycle in range(2):
+        for d in range(2):
+            outs = layer.stacked_step(inputs, eps, mech, seed, d, cycle % 2, cycle=cycle)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(M + 3)
+    rows = np.sort(rng.choice(M, size=min(16, M), replace=False))
+    ri = torch.as_tensor(rows, device="cuda")
+    for g in layer.groups:
+        full = layer.stacked[g.name]["out"][0][1]  # the last step (cycle 1, draw 1) wrote parity 0's buffer
+        assert not torch.any(full[M:]).item(), g.name  # zero noise: zero corrections
+        X = inputs[g.name][ri].cpu().numpy()
+        Yg = outs[g.name][ri].cpu().numpy()
+        cols = np.sort(rng.choice(g.N, size=min(512, g.N), replace=False))
+        W = g.W[torch.as_tensor(cols, device="cuda")].cpu().numpy()
+        check(Yg[:, cols], X, W, g.K, f"stacked {model_name} M={M} {g.name} ({layer.stacked[g.name]['path']})")
+    assert spl.spl_get_device_status() == 0
+
+
 def test_fp16x3_range_limit_is_caught_by_the_path_choice(spl):
     """The FP16X3 split scales each row by one power of two, so entries far below the row's largest
     fall under fp16's normal range and keep an absolute error of about 2^-39 max|a_row| |w| instead
