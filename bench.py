@@ -525,13 +525,14 @@ def run_llama_stack(args):
                                                   "steps); " + PEAK_NOTE}
 
     # ---- end to end: the same steps with every layer's input copied in from pinned host memory
-    # and every output copied back, inside each step's graph, on two copy streams ----------------
+    # and every output copied back, beside each step's graph, on a copy stream ------------------
     e2e = None
     if not args.no_e2e and stacked:
         phase("end-to-end pass")
-        # inputs double-buffered: step s computes on set s % 2 while its graph copies step s + 1's
-        # inputs into the other set and the previous step's outputs back, each on a copy stream of
-        # its own; the last step's outputs are copied after the loop, inside the timed region
+        # inputs double-buffered: step s computes on set s % 2 while a copy stream beside its graph
+        # copies step s + 1's inputs into the other set, then the previous step's outputs back
+        # (MaskedStack.replay_stacked); the last step's outputs are copied after the loop, inside the
+        # timed region
         host_in = [{g: x.cpu().pin_memory() for g, x in inp.items()} for inp in inputs]
         host_out = [{g.name: torch.empty((M, g.N)).pin_memory() for g in layer.groups} for layer in stack.layers]
         sets = [inputs, [{g: torch.empty_like(x) for g, x in inp.items()} for inp in inputs]]
@@ -548,18 +549,17 @@ def run_llama_stack(args):
                 for g, y in outs.items():
                     host_out[li][g].copy_(y, non_blocking=True)
 
-        e2e_graphs, _ = stack.capture_stacked(sets, eps, mech, path=path, copies=(prefetch, drain))
-        e2e_of = lambda s: e2e_graphs[(s // D) % 2][s % D]
+        e2e_graphs, _ = stack.capture_stacked(sets, eps, mech, path=path)
         s = -(-s // D) * D + D
         stack.start_stacked(s // D, e2e_graphs)  # also leaves step s's inputs in place (set s % 2 = 0)
         for _ in range(2):
-            e2e_of(s).replay()
+            stack.replay_stacked(e2e_graphs, s, copies=(prefetch, drain))
             s += 1
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(args.steps):
-            e2e_of(s).replay()
+            stack.replay_stacked(e2e_graphs, s, copies=(prefetch, drain))
             s += 1
         last = ((s - 1) // D) % 2, (s - 1) % D
         for li, outs in enumerate(stack.step_outputs(*last)):  # the last step's results
@@ -570,9 +570,9 @@ def run_llama_stack(args):
         e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, dev)
         e2e = {"value": job_rate(world, flops_step, e2e_ms) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
-               "copies": ("pinned host memory, inputs double-buffered: each step's graph copies the next step's inputs "
-                          "of every layer in and the previous step's outputs back, on two copy streams beside its "
-                          "compute; the last step's outputs are copied inside the timed region")}
+               "copies": ("pinned host memory, inputs double-buffered: beside each step's graph a copy stream copies "
+                          "the next step's inputs of every layer in, then the previous step's outputs back; the last "
+                          "step's outputs are copied inside the timed region")}
         del e2e_graphs, host_in, host_out, sets
     st = spl.spl_get_device_status()
     if st != spl.SPL_OK:

@@ -668,7 +668,7 @@ class MaskedStack:
         L, D = len(self.layers), self.draws
         return range(d * L // D, (d + 1) * L // D)
 
-    def capture_steps(self, inputs, eps, mech, bank_workspace, path="auto", timer=None, copies=None):
+    def capture_steps(self, inputs, eps, mech, bank_workspace, path="auto", timer=None):
         """CUDA graphs of single steps, each carrying its share of the next bank cycle: graphs[p][d]
         runs step d of a cycle through every layer on correction buffers p while, on a stream of
         lower priority, the layers of bank_slice(d) compute their next-cycle corrections into buffers
@@ -677,18 +677,11 @@ class MaskedStack:
         start_overlapped(c), replay graphs[(s // draws) % 2][s % draws] for steps s = c draws, c
         draws + 1, ... -- any number of them: every step holds its online pass and an equal share of
         the refill, so a run of any length times the whole method.  ``timer(d, li, phase, kind,
-        group)`` as in capture.  ``copies``: (h2d, d2h) host-transfer hooks -- h2d(li) is called on
-        the host-to-device copy stream before the online steps, once per layer in order, and returns
-        an event that layer li's online work waits for; d2h(li) is called on the device-to-host copy
-        stream after layer li's online work (which that stream waits for first).  Returns the graphs
-        and their kernel counts."""
+        group)`` as in capture.  Returns the graphs and their kernel counts."""
         lo, hi = torch.cuda.Stream.priority_range()
         if not hasattr(self, "_bank_stream"):
             self._bank_stream = torch.cuda.Stream(priority=lo)
             self._online_stream = torch.cuda.Stream(priority=hi)
-        if copies is not None and not hasattr(self, "_h2d_stream"):
-            self._h2d_stream = torch.cuda.Stream(priority=hi)
-            self._d2h_stream = torch.cuda.Stream(priority=hi)
         for layer in self.layers:
             layer.enable_overlap()
         D = self.draws
@@ -704,26 +697,11 @@ class MaskedStack:
                         for li in self.bank_slice(d):
                             self.layers[li].refill(eps, mech, self.seeds[li], 0, path=path, device_base=True,
                                                    parity=1 - parity, ahead=1, workspace=bank_workspace)
-                    ready = []
-                    if copies is not None:
-                        self._h2d_stream.wait_stream(main)
-                        with torch.cuda.stream(self._h2d_stream):
-                            ready = [copies[0](li) for li in range(len(self.layers))]
-                        self._d2h_stream.wait_stream(main)
                     for li, (layer, x, seed) in enumerate(zip(self.layers, inputs, self.seeds)):
-                        if ready:
-                            main.wait_event(ready[li])
                         t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
                             if timer else None
                         layer.online(x, eps, mech, seed, 0, d, path=path, device_base=True, parity=parity, timer=t)
-                        if copies is not None:
-                            self._d2h_stream.wait_stream(main)
-                            with torch.cuda.stream(self._d2h_stream):
-                                copies[1](li)
                     main.wait_stream(self._bank_stream)
-                    if copies is not None:
-                        main.wait_stream(self._h2d_stream)
-                        main.wait_stream(self._d2h_stream)
                     if d == D - 1:
                         for layer in self.layers:
                             for gi, g in enumerate(layer.groups):
@@ -732,22 +710,15 @@ class MaskedStack:
                 launches[parity].append(spl.spl_launch_count() - n0)
         return graphs, launches
 
-    def capture_stacked(self, inputs, eps, mech, path="auto", timer=None, copies=None):
+    def capture_stacked(self, inputs, eps, mech, path="auto", timer=None):
         """CUDA graphs of the stacked schedule (MaskedLayer.allocate_stacked): graphs[p][d] runs step d of
         a cycle of parity p through every layer -- each product also computing the next cycle's
         correction of draw d -- and graph d = draws - 1 moves every Philox base on by one cycle.  After
         start_stacked(c), replay graphs[(s // draws) % 2][s % draws] for steps s = c draws, ...: any
         number of them, each one step of the method with its share of the bank.  ``timer(d, li, phase,
         kind, group)`` as in capture.  ``inputs``: the per-layer input dicts, or a pair of them (step d
-        then reads inputs[d % 2]; draws is even, so consecutive steps alternate).  ``copies``:
-        (prefetch(d), drain(p, d)) host-transfer hooks called at the start of graph (p, d), each on a
-        copy stream of its own that the step joins at its end -- prefetch enqueues the next step's input
-        copies (into the other input set), drain the copies of the previous step's outputs (see
-        step_outputs).  Returns the graphs and their kernel counts."""
-        if copies is not None and not hasattr(self, "_h2d_stream"):
-            _, hi = torch.cuda.Stream.priority_range()
-            self._h2d_stream = torch.cuda.Stream(priority=hi)
-            self._d2h_stream = torch.cuda.Stream(priority=hi)
+        then reads inputs[d % 2]; draws is even, so consecutive steps alternate).  Host transfers go
+        beside the replays (replay_stacked).  Returns the graphs and their kernel counts."""
         paired = isinstance(inputs, (list, tuple)) and len(inputs) == 2 and isinstance(inputs[0], (list, tuple))
         D = self.draws
         graphs, launches = [[], []], [[], []]
@@ -757,21 +728,10 @@ class MaskedStack:
                 n0 = spl.spl_launch_count()
                 step_inputs = inputs[d % 2] if paired else inputs
                 with torch.cuda.graph(graph):
-                    main = torch.cuda.current_stream()
-                    if copies is not None:
-                        self._h2d_stream.wait_stream(main)
-                        with torch.cuda.stream(self._h2d_stream):
-                            copies[0](d)
-                        self._d2h_stream.wait_stream(main)
-                        with torch.cuda.stream(self._d2h_stream):
-                            copies[1](parity, d)
                     for li, (layer, x, seed) in enumerate(zip(self.layers, step_inputs, self.seeds)):
                         t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
                             if timer else None
                         layer.stacked_step(x, eps, mech, seed, d, parity, path=path, timer=t, device_base=True)
-                    if copies is not None:
-                        main.wait_stream(self._h2d_stream)
-                        main.wait_stream(self._d2h_stream)
                     if d == D - 1:
                         for layer in self.layers:
                             for gi, g in enumerate(layer.groups):
@@ -788,6 +748,31 @@ class MaskedStack:
     def previous_step(self, parity, d):
         """(parity, draw) of the step before step d of a cycle of parity ``parity``."""
         return (parity, d - 1) if d > 0 else (1 - parity, self.draws - 1)
+
+    def replay_stacked(self, graphs, s, copies=None):
+        """Step s of the stacked schedule: replays graphs[(s // draws) % 2][s % draws] (capture_stacked).
+        ``copies``: (prefetch(d), drain(p, d)) host-transfer hooks, enqueued on a copy stream beside the
+        replay once the previous step is done -- the next step's input copies (into the other input
+        set), then the copies of the previous step's outputs (step_outputs) -- which the current stream
+        waits for before the next step.  Issued here rather than captured into the graphs: measured on
+        GB300 (28-layer Llama stack, 1.0 GB in and 1.6 GB out per step), copies captured as graph nodes
+        hid under the step in one instantiation out of five (15.3 ms) and slowed it to 21.6-22.2 ms in
+        the others, while the same copies issued beside the replays hid every time (15.2 against 15.1
+        ms without copies); inputs then outputs, the two directions side by side having cost 19 ms."""
+        D = self.draws
+        p, d = (s // D) % 2, s % D
+        if copies is not None:
+            main = torch.cuda.current_stream()
+            if not hasattr(self, "_copy_stream"):
+                _, hi = torch.cuda.Stream.priority_range()
+                self._copy_stream = torch.cuda.Stream(priority=hi)
+            self._copy_stream.wait_stream(main)
+            with torch.cuda.stream(self._copy_stream):
+                copies[0](d)
+                copies[1](p, d)
+        graphs[p][d].replay()
+        if copies is not None:
+            main.wait_stream(self._copy_stream)
 
     def start_stacked(self, cycle, graphs):
         """Before replaying the stacked graphs from cycle ``cycle``: run cycle ``cycle - 1``'s graphs once
