@@ -33,8 +33,12 @@ inline spl_status launch_status() {
 // Programmatic dependent launch.  A kernel launched with launch_pdl may start while the kernel
 // before it in the stream is still running; it calls pdl_wait() before it touches memory that
 // kernel writes (or any memory at all, when in doubt), and pdl_trigger() once it has waited, so
-// that the next kernel can be scheduled early in turn (a chain never runs more than one kernel
-// ahead, and no kernel holds SM resources while waiting on a kernel that is not yet resident).
+// that the next kernel can be scheduled early in turn.  A dependent is scheduled only once every
+// CTA of its predecessor has triggered or exited, so every CTA it could wait on has started: no
+// kernel holds SM resources while waiting on one that is not yet resident, and every tensor-core
+// kernel has its tensor memory before it triggers.  The fp16 split kernels therefore trigger before
+// they wait: the product after a split (at most two kernels ahead) may start loading its weight
+// while the kernel before the split finishes.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 

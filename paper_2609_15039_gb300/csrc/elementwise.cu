@@ -226,6 +226,8 @@ __global__ void __launch_bounds__(kThreads) split_tf32_kernel(float* __restrict_
 __global__ void __launch_bounds__(kThreads) split_fp16_kernel(uint16_t* __restrict__ hi, uint16_t* __restrict__ lo,
                                                               int* __restrict__ row_exp, const float* __restrict__ src,
                                                               int64_t cols) {
+  pdl_trigger();  // before waiting: see the split kernel below
+  pdl_wait();  // src may come from the kernel before this one, which may still read hi and lo
   __shared__ float warp_max[kThreads / 32];
   const int64_t r = blockIdx.x;
   const float4* row = reinterpret_cast<const float4*>(src + r * cols);
@@ -286,8 +288,12 @@ __global__ void __launch_bounds__(kThreads) split_fp16_regs_kernel(uint16_t* __r
                                                                    uint64_t offset_host, const uint64_t* offset_dev,
                                                                    const float* __restrict__ stored, int64_t x_rows,
                                                                    uint64_t noise_delta) {
-  pdl_wait();
+  // The product after this split may be scheduled before the split waits: every block of this
+  // grid has started by then, and so has every CTA of the kernel it waits for, so the product's
+  // CTAs (which read only the weight before they wait, an L2 prefetch of C aside) take SMs that
+  // nothing before them still needs; they stream the weight while the kernel before this split ends.
   pdl_trigger();
+  pdl_wait();
   __shared__ float warp_max[kThreads / 32];
   const int64_t r = blockIdx.x;
   // rows from x_rows on (and every row when src is NULL, with a mechanism) are the noise alone,

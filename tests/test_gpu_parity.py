@@ -171,9 +171,10 @@ def _fp16_bits(x):
     return np.asarray(x, dtype=np.float16).view(np.int16)
 
 
-def test_split_fp16_properties(spl):
+@pytest.mark.parametrize("cols", [1032, 16448])  # rows held in registers; longer rows take the two-pass kernel
+def test_split_fp16_properties(spl, cols):
     """hi = fp16(w 2^e), lo = fp16(w 2^e - hi) per row; e puts the row's largest |w| in [2^14, 2^15)."""
-    W = wl.weight(37, 1032, seed=6).numpy()
+    W = wl.weight(37, cols, seed=6).numpy()
     W[1] = 0.0                                  # all-zero row: e = 0, hi = lo = 0
     W[2] *= np.float32(1e-30)                   # tiny row (residuals below fp16's normal range)
     W[3] *= np.float32(1e30)                    # huge row
@@ -235,9 +236,37 @@ def test_products_match_oracle(spl, M, K, N, path):
 TC_VARIANTS = [(256, 192), (128, 224), (128, 96), (160, 224), (192, 224), (224, 224)]
 
 
+def test_long_row_products_back_to_back_share_a_workspace(spl):
+    """FP16X3 products with K > 16384 (the left operand split by the two-pass kernel) issued back to
+    back on one stream with one workspace: each split waits for the product before it, which may
+    still be reading the previous split, so every result equals the same call made alone."""
+    M, K, N = 130, 16448, 384
+    Ws = [spl.Weight.prepare(wl.weight(N, K, seed=60 + i, device="cuda")) for i in range(2)]
+    Xs = [wl.activations(M, K, seed=70 + i, device="cuda") * (1 + 40 * i) for i in range(2)]
+    Cs = [wl.activations(M, N, seed=80 + i, device="cuda") for i in range(2)]
+    refs = []
+    for X, W, C in zip(Xs, Ws, Cs):
+        Y = torch.empty((M, N), device="cuda")
+        spl.spl_masked_linear_unmask(Y, X, W, C, path="fp16x3",
+                                     workspace=spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp16x3")))
+        torch.cuda.synchronize()
+        refs.append(Y)
+    ws = spl.workspace(spl.spl_linear_workspace_bytes(M, K, N, "fp16x3"))
+    outs = [[torch.empty((M, N), device="cuda") for _ in range(2)] for _ in range(4)]
+    for rep in range(4):
+        for i in range(2):
+            spl.spl_masked_linear_unmask(outs[rep][i], Xs[i], Ws[i], Cs[i], path="fp16x3", workspace=ws)
+    torch.cuda.synchronize()
+    for rep in range(4):
+        for i in range(2):
+            assert torch.equal(outs[rep][i], refs[i]), (rep, i)
+    ref64 = Xs[0].double() @ Ws[0].w.double().T - Cs[0].double()
+    assert float((refs[0].double() - ref64).abs().max()) <= 1e-5 * float(ref64.abs().max())
+
+
+@pytest.mark.parametrize("splits", [1, 3, 8])
 @pytest.mark.parametrize("path", ["tf32x3", "fp16x3"])
 @pytest.mark.parametrize("tile_n,ring_kb", TC_VARIANTS)
-@pytest.mark.parametrize("splits", [1, 3, 8])
 def test_tc_every_launch_shape(spl, path, tile_n, ring_kb, splits):
     """Each kernel instance (encoding x tile width x ring) with each cluster K-split, on a ragged
     problem: M, N and K not multiples of the tile, and at 8 splits an empty last K range."""
