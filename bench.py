@@ -368,7 +368,7 @@ def run_llama_stack(args):
     import torch
     import torch.distributed as dist
     from paper_2609_15039_gb300 import measure, spl, workloads as wl
-    from paper_2609_15039_gb300.layer import MaskedStack
+    from paper_2609_15039_gb300.layer import MaskedStack, StackIO
 
     world, rank, local = dist_env()
     if world > 1:
@@ -529,51 +529,38 @@ def run_llama_stack(args):
     e2e = None
     if not args.no_e2e and stacked:
         phase("end-to-end pass")
-        # inputs double-buffered: step s computes on set s % 2 while a copy stream beside its graph
-        # copies step s + 1's inputs into the other set, then the previous step's outputs back
-        # (MaskedStack.replay_stacked); the last step's outputs are copied after the loop, inside the
-        # timed region
-        host_in = [{g: x.cpu().pin_memory() for g, x in inp.items()} for inp in inputs]
-        host_out = [{g.name: torch.empty((M, g.N)).pin_memory() for g in layer.groups} for layer in stack.layers]
-        sets = [inputs, [{g: torch.empty_like(x) for g, x in inp.items()} for inp in inputs]]
-        h2d = sum(x.numel() * 4 for inp in host_in for x in inp.values())
-        d2h = sum(o.numel() * 4 for out in host_out for o in out.values())
-
-        def prefetch(d):
-            for li, inp in enumerate(sets[(d + 1) % 2]):
-                for g, x in inp.items():
-                    x.copy_(host_in[li][g], non_blocking=True)
-
-        def drain(parity, d):
-            for li, outs in enumerate(stack.step_outputs(*stack.previous_step(parity, d))):
-                for g, y in outs.items():
-                    host_out[li][g].copy_(y, non_blocking=True)
-
-        e2e_graphs, _ = stack.capture_stacked(sets, eps, mech, path=path)
+        # every step copies its inputs of every layer in from page-locked host memory and its outputs
+        # of every layer back (StackIO: one copy per input group in, one strided copy per group out,
+        # the two directions on their own streams beside the graph replays); the last step's outputs
+        # reach the host inside the timed region
+        host_in = {g: torch.stack([inp[g] for inp in inputs]).cpu().pin_memory() for g in inputs[0]}
+        io = StackIO(stack, host_in)
+        h2d, d2h = io.bytes_per_step()
+        e2e_graphs, _ = stack.capture_stacked(io.layer_inputs(), eps, mech, path=path)
         s = -(-s // D) * D + D
-        stack.start_stacked(s // D, e2e_graphs)  # also leaves step s's inputs in place (set s % 2 = 0)
-        for _ in range(2):
-            stack.replay_stacked(e2e_graphs, s, copies=(prefetch, drain))
+        stack.start_stacked(s // D, e2e_graphs)
+        s_timed = s + max(2, args.warmup)
+        while s < s_timed:  # no warm-up step copies in a timed step's inputs
+            io.step(e2e_graphs, s, stop=s_timed)
             s += 1
+        io.finish()
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for _ in range(args.steps):
-            stack.replay_stacked(e2e_graphs, s, copies=(prefetch, drain))
+        for _ in range(args.steps):  # each timed step's inputs in and outputs out inside the region
+            io.step(e2e_graphs, s, stop=s_timed + args.steps)
             s += 1
-        last = ((s - 1) // D) % 2, (s - 1) % D
-        for li, outs in enumerate(stack.step_outputs(*last)):  # the last step's results
-            for g, y in outs.items():
-                host_out[li][g].copy_(y, non_blocking=True)
+        io.finish()
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, dev)
         e2e = {"value": job_rate(world, flops_step, e2e_ms) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
-               "copies": ("pinned host memory, inputs double-buffered: beside each step's graph a copy stream copies "
-                          "the next step's inputs of every layer in, then the previous step's outputs back; the last "
-                          "step's outputs are copied inside the timed region")}
-        del e2e_graphs, host_in, host_out, sets
+               "copies": ("page-locked host memory; per step one copy in per input group (every layer's rows) and "
+                          "one strided copy out per group (every layer's Y rows), inputs and outputs on their own "
+                          f"streams beside the graph replays, inputs up to {io.sets - 1} steps ahead (StackIO); "
+                          "every timed step's inputs go in and its outputs reach the host inside the timed region")}
+        del e2e_graphs, io, host_in
     st = spl.spl_get_device_status()
     if st != spl.SPL_OK:
         raise RuntimeError("device status " + spl.status_string(st))

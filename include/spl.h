@@ -567,6 +567,20 @@ uint64_t spl_launch_count(void);
 /* Static, NUL-terminated name of a status code. */
 const char* spl_status_string(spl_status status);
 
+/* ---- host-link transfers (plumbing, not a step of the method) -----------
+ * Copies `rows` rows of `width_bytes` bytes each from src to dst, source rows
+ * src_pitch bytes apart and destination rows dst_pitch bytes apart, queued on
+ * `stream` (cudaMemcpy2DAsync; device or page-locked host memory on either
+ * side, the direction taken from the pointers).  It moves a step's outputs
+ * of every layer, which sit at a fixed pitch in a pooled output buffer, to
+ * or from the host in one copy instead of one per layer.  No kernel runs.
+ * rows == 0 or width_bytes == 0: nothing to do, SPL_OK.  SPL_EINVAL: a null
+ * pointer, or width_bytes above either pitch; SPL_ECUDA: the copy could not
+ * be queued.  The caller keeps both buffers alive and unchanged until the
+ * stream has passed the copy. */
+spl_status spl_copy_2d(void* dst, size_t dst_pitch, const void* src, size_t src_pitch, size_t width_bytes,
+                       size_t rows, cudaStream_t stream);
+
 /* ---- the boundary's call names as the problem statement lists them -------
  * The calls of the masked-linear boundary follow the paper's statement of the
  * problem (Sec. 3.3.1, Eq. add-and-then-subtract; the batched precompute of

@@ -72,3 +72,11 @@ extern "C" const char* spl_status_string(spl_status status) {
 extern "C" spl_status spl_get_last_device_status(cudaStream_t stream) { return spl_get_device_status(stream); }
 
 extern "C" const char* spl_status_str(spl_status status) { return spl_status_string(status); }
+
+extern "C" spl_status spl_copy_2d(void* dst, size_t dst_pitch, const void* src, size_t src_pitch, size_t width_bytes,
+                                  size_t rows, cudaStream_t stream) {
+  if (rows == 0 || width_bytes == 0) return SPL_OK;
+  if (!dst || !src || width_bytes > dst_pitch || width_bytes > src_pitch) return SPL_EINVAL;
+  const cudaError_t e = cudaMemcpy2DAsync(dst, dst_pitch, src, src_pitch, width_bytes, rows, cudaMemcpyDefault, stream);
+  return e == cudaSuccess ? SPL_OK : SPL_ECUDA;
+}

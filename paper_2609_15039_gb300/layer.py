@@ -181,7 +181,7 @@ class MaskedLayer:
                                      f16_exp=torch.empty(draws * M, dtype=torch.int32, device=dev))
 
     # ------------------------------------------------------------------ stacked schedule
-    def allocate_stacked(self, M, draws, path="auto", workspace=None):
+    def allocate_stacked(self, M, draws, path="auto", workspace=None, out=None):
         """Buffers of the stacked schedule: step d of a bank cycle multiplies, in one product of 2M rows
         (spl_masked_linear_unmask_precompute), the M rows of X~ for draw d of this cycle and the M noise
         rows of draw d of the next cycle, so every step carries its share of the bank and the products
@@ -192,7 +192,8 @@ class MaskedLayer:
         the same shape, which sum every row in the same order, so their roundings cancel.  When the
         2M rows run on the FP32 decode kernel and fit its fused form (2M <= 4: decode), the noise
         draw, the mask and the product of a step are one launch (spl_noise_mask_linear_unmask_precompute)
-        and the left operand is the fp32 X~ it writes."""
+        and the left operand is the fp32 X~ it writes.  ``out(name)``, if given, supplies a group's
+        out[p][d] (contiguous [2M, N] tensors, e.g. views of a buffer pooled over layers)."""
         dev = self.groups[0].W.device
         need = max(spl.spl_linear_workspace_bytes(2 * M, g.K, g.N, self.path_of(g, path, 2 * M)) for g in self.groups)
         if workspace is not None:
@@ -215,9 +216,13 @@ class MaskedLayer:
                             f16_lo=torch.empty((2 * M, g.K), dtype=torch.int16, device=dev),
                             f16_exp=torch.empty(2 * M, dtype=torch.int32, device=dev))
                  if fused else spl.Weight(torch.empty((2 * M, g.K), device=dev)))
-            out = [[torch.zeros((2 * M, g.N), device=dev) for _ in range(draws)] for _ in range(2)]
+            if out is not None:
+                bufs = out(g.name)
+                assert all(b.shape == (2 * M, g.N) and b.is_contiguous() for row in bufs for b in row)
+            else:
+                bufs = [[torch.zeros((2 * M, g.N), device=dev) for _ in range(draws)] for _ in range(2)]
             resolved = spl.PATH_NAMES[spl.spl_resolve_path(2 * M, g.K, g.N, self.path_of(g, path, 2 * M))]
-            self.stacked[g.name] = {"a": a, "out": out, "fused": fused, "fused_mask": fused_mask, "path": resolved}
+            self.stacked[g.name] = {"a": a, "out": bufs, "fused": fused, "fused_mask": fused_mask, "path": resolved}
 
     def stacked_step(self, inputs, eps, mech, seed, d, parity, cycle=0, path="auto", stream=None, timer=None,
                      device_base=False):
@@ -548,6 +553,7 @@ class MaskedStack:
 
     def __init__(self, layers, seeds):
         self.layers, self.seeds = layers, seeds
+        self.out_pool = None  # stacked schedule built by build(): {group: [2, draws, layers, 2M, N]}
 
     @classmethod
     def build(cls, model, n_layers, M, draws, base_seed, device="cuda", split=True, power_iters=1000, path="auto",
@@ -563,17 +569,25 @@ class MaskedStack:
             del weights
             layer.sensitivities(power_iters=power_iters)
             layers.append(layer)
+        pool = None
         if stacked:
             need = max(spl.spl_linear_workspace_bytes(2 * M, g.K, g.N, path) for l in layers for g in l.groups)
             ws = spl.workspace(need, device)
-            for layer in layers:
-                layer.allocate_stacked(M, draws, path, workspace=ws)
+            # each group's outputs pooled over the layers, [parity, draw, layer, 2M, N]: the Y rows of one
+            # step of every layer then sit at one pitch (StackIO moves them with one copy per group)
+            pool = {g.name: torch.zeros((2, draws, n_layers, 2 * M, g.N), device=device) for g in layers[0].groups}
+            for li, layer in enumerate(layers):
+                layer.allocate_stacked(M, draws, path, workspace=ws,
+                                       out=lambda name, li=li: [[pool[name][p, d, li] for d in range(draws)]
+                                                                for p in range(2)])
         else:
             need = max(l.workspace_bytes(M, draws, path) for l in layers)
             ws = spl.workspace(need, device)
             for layer in layers:
                 layer.allocate(M, draws, path, workspace=ws)
-        return cls(layers, [wl.layer_seed(base_seed, li, 99) for li in range(n_layers)])
+        stack = cls(layers, [wl.layer_seed(base_seed, li, 99) for li in range(n_layers)])
+        stack.out_pool = pool
+        return stack
 
     @property
     def draws(self):
@@ -716,17 +730,19 @@ class MaskedStack:
         correction of draw d -- and graph d = draws - 1 moves every Philox base on by one cycle.  After
         start_stacked(c), replay graphs[(s // draws) % 2][s % draws] for steps s = c draws, ...: any
         number of them, each one step of the method with its share of the bank.  ``timer(d, li, phase,
-        kind, group)`` as in capture.  ``inputs``: the per-layer input dicts, or a pair of them (step d
-        then reads inputs[d % 2]; draws is even, so consecutive steps alternate).  Host transfers go
-        beside the replays (replay_stacked).  Returns the graphs and their kernel counts."""
-        paired = isinstance(inputs, (list, tuple)) and len(inputs) == 2 and isinstance(inputs[0], (list, tuple))
+        kind, group)`` as in capture.  ``inputs``: the per-layer input dicts, or n sets of them with n
+        dividing draws (step d then reads inputs[d % n], so step s reads set s % n).  Host transfers go
+        beside the replays (StackIO).  Returns the graphs and their kernel counts."""
+        sets = isinstance(inputs, (list, tuple)) and len(inputs) > 0 and isinstance(inputs[0], (list, tuple))
         D = self.draws
+        if sets and D % len(inputs):
+            raise ValueError("capture_stacked: the number of input sets must divide draws")
         graphs, launches = [[], []], [[], []]
         for parity in range(2):
             for d in range(D):
                 graph = torch.cuda.CUDAGraph()
                 n0 = spl.spl_launch_count()
-                step_inputs = inputs[d % 2] if paired else inputs
+                step_inputs = inputs[d % len(inputs)] if sets else inputs
                 with torch.cuda.graph(graph):
                     for li, (layer, x, seed) in enumerate(zip(self.layers, step_inputs, self.seeds)):
                         t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
@@ -749,30 +765,11 @@ class MaskedStack:
         """(parity, draw) of the step before step d of a cycle of parity ``parity``."""
         return (parity, d - 1) if d > 0 else (1 - parity, self.draws - 1)
 
-    def replay_stacked(self, graphs, s, copies=None):
+    def replay_stacked(self, graphs, s):
         """Step s of the stacked schedule: replays graphs[(s // draws) % 2][s % draws] (capture_stacked).
-        ``copies``: (prefetch(d), drain(p, d)) host-transfer hooks, enqueued on a copy stream beside the
-        replay once the previous step is done -- the next step's input copies (into the other input
-        set), then the copies of the previous step's outputs (step_outputs) -- which the current stream
-        waits for before the next step.  Issued here rather than captured into the graphs: measured on
-        GB300 (28-layer Llama stack, 1.0 GB in and 1.6 GB out per step), copies captured as graph nodes
-        hid under the step in one instantiation out of five (15.3 ms) and slowed it to 21.6-22.2 ms in
-        the others, while the same copies issued beside the replays hid every time (15.2 against 15.1
-        ms without copies); inputs then outputs, the two directions side by side having cost 19 ms."""
+        Host transfers beside the replays: StackIO."""
         D = self.draws
-        p, d = (s // D) % 2, s % D
-        if copies is not None:
-            main = torch.cuda.current_stream()
-            if not hasattr(self, "_copy_stream"):
-                _, hi = torch.cuda.Stream.priority_range()
-                self._copy_stream = torch.cuda.Stream(priority=hi)
-            self._copy_stream.wait_stream(main)
-            with torch.cuda.stream(self._copy_stream):
-                copies[0](d)
-                copies[1](p, d)
-        graphs[p][d].replay()
-        if copies is not None:
-            main.wait_stream(self._copy_stream)
+        graphs[(s // D) % 2][s % D].replay()
 
     def start_stacked(self, cycle, graphs):
         """Before replaying the stacked graphs from cycle ``cycle``: run cycle ``cycle - 1``'s graphs once
@@ -810,3 +807,118 @@ def split_outputs(layer, outs):
             a, b = g.columns(p)
             res[p] = outs[g.name][:, a:b]
     return res
+
+
+class StackIO:
+    """Host transfers of the stacked schedule beside its graph replays, few and large.
+
+    Each input group of every layer sits in one page-locked host buffer ``host_in[group]`` and in
+    ``sets`` device sets ([layers, M, K]; step s reads set s % sets, as capture_stacked does with the
+    sets from ``layer_inputs()``), and the Y rows of one step of every layer lie at one pitch in the
+    stack's pooled output buffer (MaskedStack.build), so a step moves each group in with one copy
+    and out with one strided copy (spl_copy_2d): a handful of host calls per step, which lets the
+    host run far ahead of the device.  Inputs go in on one stream and outputs out on another, the
+    two directions of the host link at once.  Inputs go in up to sets - 1 steps ahead (never past
+    ``stop``) and step s waits only for its own; its outputs go to host slot s % ring once it is
+    done, and only have to be out before step s + 2 draws rewrites the same device buffer, so a copy
+    that stalls holds the steps up only once it has fallen that far behind.
+
+    Measured on GB300 (28-layer Llama stack, 1.0 GB in and 1.6 GB out per step): a step's inputs
+    take 4.8 ms and its outputs 8.2 ms, beside the 14.5-15 ms of compute.  On some boxes the host
+    side stalls now and then (one direction's copies 50-250 ms at a time, the host thread too): the
+    earlier schedule -- a copy per layer and group, inputs then outputs on one stream that each step
+    waited for, the host a step or two ahead -- put every stall on the step time (20.4 ms per step
+    on average); here the host is hundreds of steps ahead and a stall holds the steps up only once
+    the copies have fallen sets - 1 steps (inputs) or 2 draws steps (outputs) behind, but a timed
+    run still ends only when its last outputs are on the host.  ``streams=1`` puts both directions
+    on one copy stream."""
+
+    def __init__(self, stack, host_in, ring=2, sets=None, streams=2):
+        if stack.out_pool is None:
+            raise ValueError("StackIO: a stack built with stacked=True (pooled outputs)")
+        D = stack.draws
+        if sets is None:  # the most sets up to 8 that divide the draws
+            sets = max([n for n in range(2, min(D, 8) + 1) if D % n == 0], default=0)
+        if sets < 2 or D % sets:
+            raise ValueError("StackIO: at least two input sets, a divisor of draws")
+        self.stack, self.sets = stack, sets
+        L, M = len(stack.layers), stack.layers[0].M
+        dev = stack.layers[0].groups[0].W.device
+        self.host_in = host_in
+        for g, x in host_in.items():
+            if not x.is_pinned() or x.shape[:2] != (L, M):
+                raise ValueError("StackIO: host_in[group] is page-locked [layers, M, K]")
+        self.dev_in = [{g: torch.zeros(x.shape, device=dev) for g, x in host_in.items()} for _ in range(sets)]
+        self.host_out = [{g: torch.empty((L, M, p.shape[-1])).pin_memory() for g, p in stack.out_pool.items()}
+                         for _ in range(ring)]
+        if streams not in (1, 2):
+            raise ValueError("StackIO: one copy stream or one per direction")
+        self.h2d = torch.cuda.Stream()
+        self.d2h = self.h2d if streams == 1 else torch.cuda.Stream()
+        self._in, self._done, self._out = {}, {}, {}
+
+    def layer_inputs(self):
+        """The device sets as capture_stacked takes them: per set, per layer {group: [M, K] view}."""
+        L = len(self.stack.layers)
+        return [[{g: x[li] for g, x in dset.items()} for li in range(L)] for dset in self.dev_in]
+
+    def bytes_per_step(self):
+        """(bytes in, bytes out) per step."""
+        return (sum(x.numel() * x.element_size() for x in self.host_in.values()),
+                sum(y.numel() * y.element_size() for y in self.host_out[0].values()))
+
+    @staticmethod
+    def _event(stream):
+        e = torch.cuda.Event()
+        e.record(stream)
+        return e
+
+    def _prefetch(self, s):
+        done = self._done.pop(s - self.sets, None)  # set s % sets was last read by step s - sets
+        if done is not None:
+            self.h2d.wait_event(done)
+        dst = self.dev_in[s % self.sets]
+        with torch.cuda.stream(self.h2d):
+            for g, x in self.host_in.items():
+                dst[g].copy_(x, non_blocking=True)
+        self._in[s] = self._event(self.h2d)
+
+    def step(self, graphs, s, stop=None):
+        """Step s with graphs from capture_stacked(layer_inputs(), ...): the inputs of steps s to
+        s + sets - 1 in (those not already there, none from step ``stop`` on), the replay, then this
+        step's outputs out to host slot s % ring."""
+        D, M = self.stack.draws, self.stack.layers[0].M
+        if stop is not None and s >= stop:
+            raise ValueError("StackIO.step: s is past stop")
+        main = torch.cuda.current_stream()
+        if not self._in and not self._done:  # first step: the sets may still be read by earlier work
+            self.h2d.wait_stream(main)
+        hi = s + self.sets if stop is None else min(s + self.sets, stop)
+        for t in range(s, hi):  # set t % sets was last read by step t - sets < s
+            if t not in self._in:
+                self._prefetch(t)
+        main.wait_event(self._in.pop(s))
+        out_back = self._out.pop(s - 2 * D, None)  # the last copy out of the device buffer step s rewrites
+        if out_back is not None:
+            main.wait_event(out_back)
+        p, d = (s // D) % 2, s % D
+        graphs[p][d].replay()
+        done = self._event(main)
+        self._done[s] = done
+        self.d2h.wait_event(done)
+        dst = self.host_out[s % len(self.host_out)]
+        with torch.cuda.stream(self.d2h):
+            for g, y in dst.items():
+                src = self.stack.out_pool[g][1 - p, d]  # [layers, 2M, N]: rows [0, M) of each layer are Y
+                row = M * src.shape[-1] * src.element_size()
+                spl.spl_copy_2d(y, src, src.shape[0], row, row, 2 * row, stream=self.d2h)
+        self._out[s] = self._event(self.d2h)
+
+    def outputs(self, s):
+        """Host slot of step s ({group: [layers, M, N]}) and the event after which it holds step s's
+        outputs (until step s + ring is copied out into the same slot)."""
+        return self.host_out[s % len(self.host_out)], self._out.get(s)
+
+    def finish(self):
+        """The current stream waits until every output issued so far is on the host."""
+        torch.cuda.current_stream().wait_stream(self.d2h)

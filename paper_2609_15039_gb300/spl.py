@@ -102,6 +102,7 @@ _SIGS = {
     "spl_prepare_weight_split": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "spl_get_last_device_status": (_I, [_P]),
     "spl_status_str": (ctypes.c_char_p, [_I]),
+    "spl_copy_2d": (_I, [_P, _SZ, _P, _SZ, _SZ, _SZ, _P]),
 }
 
 _lib = None
@@ -700,6 +701,19 @@ def spl_test_tc_swap_product(Y, Xt, W, C=None, tile_tokens=16, ctas=0, workspace
     _check(lib().spl_test_tc_swap_product(_dev(Y, "Y"), _dev(Xt, "Xt"), ctypes.byref(ws_), _dev(C, "C"), M, K, N,
                                           int(tile_tokens), int(ctas), wsp, wsb, _stream(stream)),
            "spl_test_tc_swap_product")
+
+
+def spl_copy_2d(dst, src, rows, width_bytes, dst_pitch, src_pitch, stream=None):
+    """``rows`` rows of ``width_bytes`` bytes from src to dst, rows ``src_pitch`` / ``dst_pitch`` bytes
+    apart (host-link plumbing, not a step of the method).  Each tensor is contiguous and on the GPU
+    or in page-locked host memory; the copied extent lies inside both."""
+    for t, name, pitch in ((dst, "dst", dst_pitch), (src, "src", src_pitch)):
+        if not t.is_contiguous() or not (t.is_cuda or t.is_pinned()):
+            raise ValueError(f"spl_copy_2d: {name} must be contiguous, on the GPU or page-locked")
+        if rows and width_bytes and (rows - 1) * pitch + width_bytes > t.numel() * t.element_size():
+            raise ValueError(f"spl_copy_2d: the copied extent does not fit {name}")
+    _check(lib().spl_copy_2d(dst.data_ptr(), int(dst_pitch), src.data_ptr(), int(src_pitch), int(width_bytes),
+                             int(rows), _stream(stream)), "spl_copy_2d")
 
 
 def spl_launch_count():

@@ -201,6 +201,23 @@ def test_split_operand_workspace(spl):
     assert spl.spl_split_workspace_bytes(16, 3072, 5120, path=9) == 0
 
 
+def test_copy_2d_validates_without_a_copy(spl):
+    """The host-link copy refuses null pointers and rows wider than a pitch before it queues anything;
+    nothing to copy is a no-op."""
+    L = spl.lib()
+    buf = ctypes.create_string_buffer(64)
+    p = ctypes.addressof(buf)
+    assert L.spl_copy_2d(None, 16, p, 16, 8, 2, None) == spl.SPL_EINVAL
+    assert L.spl_copy_2d(p, 16, None, 16, 8, 2, None) == spl.SPL_EINVAL
+    assert L.spl_copy_2d(p, 8, p, 16, 16, 2, None) == spl.SPL_EINVAL  # wider than the destination pitch
+    assert L.spl_copy_2d(p, 16, p, 8, 16, 2, None) == spl.SPL_EINVAL  # wider than the source pitch
+    assert L.spl_copy_2d(None, 0, None, 0, 8, 0, None) == spl.SPL_OK
+    assert L.spl_copy_2d(None, 0, None, 0, 0, 3, None) == spl.SPL_OK
+    import torch
+    with pytest.raises(ValueError):  # the binding checks the extent against the tensors
+        spl.spl_copy_2d(torch.zeros(4), torch.zeros(8), 2, 16, 16, 16)
+
+
 def test_workspace_sizes_are_consistent(spl):
     # decode shapes need split-K partials after the 64 KiB counter region; the tensor-core
     # kernels reduce split-K in a cluster and keep only the split of the left operand there

@@ -261,3 +261,44 @@ def test_stacked_graphs_equal_eager_steps(spl, M):
                 y = layer.stacked[g.name]["out"][1 - cycle % 2][d][:M]
                 assert torch.equal(y, expected[(s, li)][g.name]), (s, li, g.name)
     assert spl.spl_get_device_status() == 0
+
+
+@pytest.mark.parametrize("M,draws,streams", [(128, 2, 2), (1, 2, 2), (128, 4, 2), (128, 4, 1)])
+def test_stack_io_moves_every_step_exactly(spl, M, draws, streams):
+    """StackIO: every layer's inputs copied in from page-locked host memory one step ahead and every
+    layer's outputs copied back with one strided copy per group, on their own streams, with no host
+    synchronisation between steps and the device output buffers rewritten while earlier copies may
+    still be in flight: each step's host outputs equal, bit for bit, the device outputs of the same
+    steps replayed one at a time with the inputs already in place."""
+    from paper_2609_15039_gb300.layer import MaskedStack, StackIO
+    model = wl.ModelShape("small", 1, 512, 1024, 512, 256, 1000)
+    eps, mech = 1.0, "laplace"
+    stack = MaskedStack.build(model, 3, M, draws, base_seed=5, power_iters=50, stacked=True)
+    inputs = stack.inputs(17)
+    host_in = {g: torch.stack([inp[g] for inp in inputs]).cpu().pin_memory() for g in inputs[0]}
+    steps = list(range(2 * draws, 2 * draws + 4 * draws + 1))
+    io = StackIO(stack, host_in, ring=len(steps), streams=streams)  # a host slot per step
+    assert io.sets == draws  # inputs go in up to draws - 1 steps ahead
+    assert io.bytes_per_step() == (sum(x.numel() * 4 for x in host_in.values()),
+                                   sum(3 * M * g.N * 4 for g in stack.layers[0].groups))
+    graphs, _ = stack.capture_stacked(io.layer_inputs(), eps, mech)
+    stack.start_stacked(2, graphs)
+    for s in steps:
+        io.step(graphs, s, stop=steps[-1] + 1)
+    assert not io._in  # nothing copied in for a step past the last
+    io.finish()
+    torch.cuda.synchronize()
+    got = {s: {g: y.clone() for g, y in io.outputs(s)[0].items()} for s in steps}
+    for dset in io.dev_in:  # the reference: both input sets in place beforehand, one step at a time
+        for g, x in host_in.items():
+            dset[g].copy_(x)
+    stack.start_stacked(2, graphs)
+    for s in steps:
+        stack.replay_stacked(graphs, s)
+        torch.cuda.synchronize()
+        p, d = (s // draws) % 2, s % draws
+        for g, pool in stack.out_pool.items():
+            assert torch.equal(got[s][g], pool[1 - p, d, :, :M].cpu()), (s, g)
+            for li, layer in enumerate(stack.layers):  # the pool is the layers' own output buffers
+                assert layer.stacked[g]["out"][1 - p][d].data_ptr() == pool[1 - p, d, li].data_ptr()
+    assert spl.spl_get_device_status() == 0
