@@ -230,43 +230,57 @@ class MaskedLayer:
         of draw d of this cycle, the noise of draw d of the next cycle, and their product with W in one
         call whose first M rows are unmasked with this cycle's correction.  The arithmetic path of each
         group is the one resolved when the buffers were allocated.  Returns {group: Y [M, N]}."""
-        M, D = self.M, self.draws
-        out = {}
         for gi, g in enumerate(self.groups):
-            st = self.stacked[g.name]
-            a = st["a"]
+            self._stacked_prepare(gi, g, inputs, eps, mech, seed, d, cycle, device_base, stream)
+        return {g.name: self._stacked_product(gi, g, inputs, eps, mech, seed, d, parity, cycle, device_base, stream,
+                                              timer)
+                for gi, g in enumerate(self.groups)}
+
+    def _stacked_prepare(self, gi, g, inputs, eps, mech, seed, d, cycle, device_base, stream):
+        """The left operand of group g for step d where the product takes it ready-made (the noise of
+        both halves, the mask and, on FP16X3, the split); False where the product draws it itself
+        (the one-launch decode form).  Reads only the inputs and the Philox bases, writes only the
+        group's operand buffer, so it may run beside other groups' products."""
+        M, D = self.M, self.draws
+        st = self.stacked[g.name]
+        if st["fused_mask"]:
+            return False
+        a = st["a"]
+        off, off_dev = self._offset(gi, g, cycle, d, device_base)
+        off_next = off + D * (M * g.K // 4)  # draw d of the next cycle
+        delta = self.deltas[g.name]
+        if st["fused"]:  # both halves of the left operand in one launch
+            spl.spl_noise_mask_split_stacked(a.f16_hi, a.f16_lo, a.f16_exp, inputs[g.name], delta, eps, mech, seed,
+                                             M, off_next - off, stream_id=gi, offset=off, stream=stream,
+                                             offset_dev=off_dev)
+        else:
+            spl.spl_noise_mask(a.w[:M], None, inputs[g.name], delta, eps, mech, seed, stream_id=gi, offset=off,
+                               stream=stream, offset_dev=off_dev)
+            spl.spl_noise(a.w[M:], delta, eps, mech, seed, stream_id=gi, offset=off_next, stream=stream,
+                          offset_dev=off_dev)
+        return True
+
+    def _stacked_product(self, gi, g, inputs, eps, mech, seed, d, parity, cycle, device_base, stream, timer):
+        """The product call of group g for step d (after _stacked_prepare); returns Y [M, N]."""
+        M, D = self.M, self.draws
+        st = self.stacked[g.name]
+        a = st["a"]
+        res = st["out"][1 - parity][d]
+        if timer:
+            timer("begin", "masked_linear_unmask", g.name)
+        if st["fused_mask"]:  # noise, mask and product of both halves in one decode launch
             off, off_dev = self._offset(gi, g, cycle, d, device_base)
-            off_next = off + D * (M * g.K // 4)  # draw d of the next cycle
-            delta = self.deltas[g.name]
-            res = st["out"][1 - parity][d]
-            if st["fused_mask"]:  # noise, mask and product of both halves in one decode launch
-                if timer:
-                    timer("begin", "masked_linear_unmask", g.name)
-                spl.spl_noise_mask_linear_unmask_precompute(
-                    res, a.w, inputs[g.name], g.wt, st["out"][parity][d][M:], delta, eps, mech, seed, M,
-                    off_next - off, stream_id=gi, offset=off, path=st["path"], workspace=self.workspace,
-                    stream=stream, offset_dev=off_dev)
-                if timer:
-                    timer("end", "masked_linear_unmask", g.name)
-                out[g.name] = res[:M]
-                continue
-            if st["fused"]:  # both halves of the left operand in one launch
-                spl.spl_noise_mask_split_stacked(a.f16_hi, a.f16_lo, a.f16_exp, inputs[g.name], delta, eps, mech, seed,
-                                                 M, off_next - off, stream_id=gi, offset=off, stream=stream,
-                                                 offset_dev=off_dev)
-            else:
-                spl.spl_noise_mask(a.w[:M], None, inputs[g.name], delta, eps, mech, seed, stream_id=gi, offset=off,
-                                   stream=stream, offset_dev=off_dev)
-                spl.spl_noise(a.w[M:], delta, eps, mech, seed, stream_id=gi, offset=off_next, stream=stream,
-                              offset_dev=off_dev)
-            if timer:
-                timer("begin", "masked_linear_unmask", g.name)
+            off_next = off + D * (M * g.K // 4)
+            spl.spl_noise_mask_linear_unmask_precompute(
+                res, a.w, inputs[g.name], g.wt, st["out"][parity][d][M:], self.deltas[g.name], eps, mech, seed, M,
+                off_next - off, stream_id=gi, offset=off, path=st["path"], workspace=self.workspace,
+                stream=stream, offset_dev=off_dev)
+        else:
             spl.spl_masked_linear_unmask_precompute(res, a, g.wt, st["out"][parity][d][M:], M, path=st["path"],
                                                     workspace=self.workspace, stream=stream)
-            if timer:
-                timer("end", "masked_linear_unmask", g.name)
-            out[g.name] = res[:M]
-        return out
+        if timer:
+            timer("end", "masked_linear_unmask", g.name)
+        return res[:M]
 
     def enable_overlap(self):
         """A second correction buffer per group (and noise buffer, for stored noise), so that a bank
@@ -737,6 +751,8 @@ class MaskedStack:
         D = self.draws
         if sets and D % len(inputs):
             raise ValueError("capture_stacked: the number of input sets must divide draws")
+        side = torch.cuda.Stream()
+        forked = any(not l.stacked[g.name]["fused_mask"] for l in self.layers for g in l.groups)
         graphs, launches = [[], []], [[], []]
         for parity in range(2):
             for d in range(D):
@@ -744,10 +760,28 @@ class MaskedStack:
                 n0 = spl.spl_launch_count()
                 step_inputs = inputs[d % len(inputs)] if sets else inputs
                 with torch.cuda.graph(graph):
+                    # every group's left operand on a side stream, the products in order on this one, each
+                    # waiting only for its own operand: the operands (issue-bound on the noise) run beside
+                    # the products (tensor-bound) instead of between them
+                    main = torch.cuda.current_stream()
+                    ready = {}
+                    if forked:
+                        side.wait_stream(main)
+                        with torch.cuda.stream(side):
+                            for li, (layer, x, seed) in enumerate(zip(self.layers, step_inputs, self.seeds)):
+                                for gi, g in enumerate(layer.groups):
+                                    if layer._stacked_prepare(gi, g, x, eps, mech, seed, d, 0, True, side):
+                                        ready[(li, g.name)] = torch.cuda.Event()
+                                        ready[(li, g.name)].record(side)
                     for li, (layer, x, seed) in enumerate(zip(self.layers, step_inputs, self.seeds)):
                         t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
                             if timer else None
-                        layer.stacked_step(x, eps, mech, seed, d, parity, path=path, timer=t, device_base=True)
+                        for gi, g in enumerate(layer.groups):
+                            if (li, g.name) in ready:
+                                main.wait_event(ready[(li, g.name)])
+                            layer._stacked_product(gi, g, x, eps, mech, seed, d, parity, 0, True, main, t)
+                    if forked:
+                        main.wait_stream(side)
                     if d == D - 1:
                         for layer in self.layers:
                             for gi, g in enumerate(layer.groups):
