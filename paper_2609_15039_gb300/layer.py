@@ -230,21 +230,21 @@ class MaskedLayer:
         of draw d of this cycle, the noise of draw d of the next cycle, and their product with W in one
         call whose first M rows are unmasked with this cycle's correction.  The arithmetic path of each
         group is the one resolved when the buffers were allocated.  Returns {group: Y [M, N]}."""
+        out = {}
         for gi, g in enumerate(self.groups):
             self._stacked_prepare(gi, g, inputs, eps, mech, seed, d, cycle, device_base, stream)
-        return {g.name: self._stacked_product(gi, g, inputs, eps, mech, seed, d, parity, cycle, device_base, stream,
-                                              timer)
-                for gi, g in enumerate(self.groups)}
+            out[g.name] = self._stacked_product(gi, g, inputs, eps, mech, seed, d, parity, cycle, device_base,
+                                                stream, timer)
+        return out
 
     def _stacked_prepare(self, gi, g, inputs, eps, mech, seed, d, cycle, device_base, stream):
         """The left operand of group g for step d where the product takes it ready-made (the noise of
-        both halves, the mask and, on FP16X3, the split); False where the product draws it itself
-        (the one-launch decode form).  Reads only the inputs and the Philox bases, writes only the
-        group's operand buffer, so it may run beside other groups' products."""
+        both halves, the mask and, on FP16X3, the split, in one launch there); nothing where the
+        product draws it itself (the one-launch decode form)."""
         M, D = self.M, self.draws
         st = self.stacked[g.name]
         if st["fused_mask"]:
-            return False
+            return
         a = st["a"]
         off, off_dev = self._offset(gi, g, cycle, d, device_base)
         off_next = off + D * (M * g.K // 4)  # draw d of the next cycle
@@ -258,7 +258,6 @@ class MaskedLayer:
                                stream=stream, offset_dev=off_dev)
             spl.spl_noise(a.w[M:], delta, eps, mech, seed, stream_id=gi, offset=off_next, stream=stream,
                           offset_dev=off_dev)
-        return True
 
     def _stacked_product(self, gi, g, inputs, eps, mech, seed, d, parity, cycle, device_base, stream, timer):
         """The product call of group g for step d (after _stacked_prepare); returns Y [M, N]."""
@@ -751,8 +750,6 @@ class MaskedStack:
         D = self.draws
         if sets and D % len(inputs):
             raise ValueError("capture_stacked: the number of input sets must divide draws")
-        side = torch.cuda.Stream()
-        forked = any(not l.stacked[g.name]["fused_mask"] for l in self.layers for g in l.groups)
         graphs, launches = [[], []], [[], []]
         for parity in range(2):
             for d in range(D):
@@ -760,28 +757,10 @@ class MaskedStack:
                 n0 = spl.spl_launch_count()
                 step_inputs = inputs[d % len(inputs)] if sets else inputs
                 with torch.cuda.graph(graph):
-                    # every group's left operand on a side stream, the products in order on this one, each
-                    # waiting only for its own operand: the operands (issue-bound on the noise) run beside
-                    # the products (tensor-bound) instead of between them
-                    main = torch.cuda.current_stream()
-                    ready = {}
-                    if forked:
-                        side.wait_stream(main)
-                        with torch.cuda.stream(side):
-                            for li, (layer, x, seed) in enumerate(zip(self.layers, step_inputs, self.seeds)):
-                                for gi, g in enumerate(layer.groups):
-                                    if layer._stacked_prepare(gi, g, x, eps, mech, seed, d, 0, True, side):
-                                        ready[(li, g.name)] = torch.cuda.Event()
-                                        ready[(li, g.name)].record(side)
                     for li, (layer, x, seed) in enumerate(zip(self.layers, step_inputs, self.seeds)):
                         t = (lambda phase, kind, group, _d=d, _li=li: timer(_d, _li, phase, kind, group)) \
                             if timer else None
-                        for gi, g in enumerate(layer.groups):
-                            if (li, g.name) in ready:
-                                main.wait_event(ready[(li, g.name)])
-                            layer._stacked_product(gi, g, x, eps, mech, seed, d, parity, 0, True, main, t)
-                    if forked:
-                        main.wait_stream(side)
+                        layer.stacked_step(x, eps, mech, seed, d, parity, timer=t, device_base=True)
                     if d == D - 1:
                         for layer in self.layers:
                             for gi, g in enumerate(layer.groups):
