@@ -7,12 +7,14 @@ Llama-3.2-3B-shaped linear stack (per layer Q|K|V 3072 -> 5120, O 3072 ->
 eps = 1, each layer seeded on its own.  A step draws and adds the mask of every
 input group of every layer (fused with the fp16 split the tensor-core product
 reads), runs the masked products with the unmask fused into their epilogues
-(Y = X~ W^T - C), and carries its share of the correction bank: the banks hold
-8 draws per group (C = eta W^T for 8 x 512 rows, summed in the online order),
-and each of the 8 steps of a cycle computes the next cycle's banks of an
-eighth of the layers on a lower-priority stream beside its own prefill.  So
-any number of steps times the whole method: prefill plus its correction.
-The weights (45 GB with their splits) are far larger than L2.
+(Y = X~ W^T - C), and carries its share of the correction bank: each product
+call multiplies the step's 512 masked rows together with the 512 noise rows of
+the same draw of the next bank cycle (8 draws per cycle), whose products are
+the corrections that cycle's step subtracts.  So any number of steps times the
+whole method: prefill plus its correction.  ``--schedule banked`` runs the
+separate bank instead (8 draws of corrections per group refilled beside the
+steps on a lower-priority stream).  The weights (45 GB with their splits) are
+far larger than L2.
 
 Also reported on the same stack: the online prefill alone, the bank refill
 alone, the product kernels per launch (the roofline), decode at one token per
