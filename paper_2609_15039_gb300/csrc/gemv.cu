@@ -36,7 +36,8 @@ namespace {
 
 constexpr int THREADS = 256, WARPS = 8;
 constexpr int kStep = 32;                    // K elements a quarter-warp covers per step
-constexpr int kSliceAlign = 128;             // K-slices are multiples of this
+constexpr int kSliceAlign = 64;              // K-slices are multiples of this (staged_ks pads the
+                                             // staged slice to the iteration step)
 constexpr int kXsBytes = 96 * 1024;          // largest X~ slice a block stages (two blocks per SM)
 constexpr int kMaxKs = kXsBytes / (4 * kGemvMaxM) / kSliceAlign * kSliceAlign;  // 1536: every MT fits it
 
@@ -46,6 +47,12 @@ __host__ __device__ constexpr int rows_per_block(int mt) { return WARPS * 4 * ro
 // Steps of 32 per unrolled iteration: 8 float4 loads of W in flight per lane per buffer, but 4 at 8
 // rows (then 80 registers give 3 blocks per SM instead of 2; measured faster at 8 rows, slower at 16).
 __host__ __device__ constexpr int unroll_steps(int mt) { return mt == 8 ? 2 : 8 / rows_per_lane(mt); }
+// Columns of the staged X~ slice: ks rounded up to the columns one unrolled iteration reads (64 or
+// 128), so a slice that is a multiple of kSliceAlign but not of that step is staged with zero
+// columns after it and no iteration reads past the staged rows.
+__host__ __device__ constexpr int staged_ks(int mt, int ks) {
+  return (ks + unroll_steps(mt) * kStep - 1) / (unroll_steps(mt) * kStep) * (unroll_steps(mt) * kStep);
+}
 
 // Rows of X~ are summed in packed pairs (p2 / fma2 / up2 of noise.cuh): one fma.rn.f32x2 does the
 // two round-to-nearest FMAs the scalar loop would, so the sums are the same bit for bit with half
@@ -124,7 +131,7 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
             int c_rows) {
   constexpr int RQ = rows_per_lane(MT), RB = rows_per_block(MT), U = unroll_steps(MT);
   constexpr int V = RQ * MT;
-  extern __shared__ __align__(16) float4 xs[];  // [MT][ks / 4]
+  extern __shared__ __align__(16) float4 xs[];  // [MT][staged_ks(MT, ks) / 4]
   __shared__ int s_last;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quarter = lane >> 3, kl = (lane & 7) * 4;
@@ -163,8 +170,9 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
   // fetch their first weight lines while this one streams (decode 2.28 -> 2.24 ms per token)
   pdl_trigger();
 
-  // stage X~[:, k0:k0+ks] (rows >= M and columns >= klen are zero)
-  const int q_row = ks >> 2, q_len = klen >> 2;
+  // stage X~[:, k0:k0+ks] (rows >= M and columns >= klen are zero), rows ksp columns apart
+  const int ksp = staged_ks(MT, ks);
+  const int q_row = ksp >> 2, q_len = klen >> 2;
   float* xsf = reinterpret_cast<float*>(xs);
   // X~ of rows m, columns 4q..4q+3 (stored as given, or with the noise drawn here)
   auto x4 = [&](int m, int q, float4* dst_out) -> float4 {
@@ -192,8 +200,8 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
         float4* d0 = write_xt && 2 * p < M && q < q_len ? reinterpret_cast<float4*>(nz.xt + (int64_t)(2 * p) * K + k0) + q : nullptr;
         float4* d1 = write_xt && 2 * p + 1 < M && q < q_len ? reinterpret_cast<float4*>(nz.xt + (int64_t)(2 * p + 1) * K + k0) + q : nullptr;
         const float4 a = x4(2 * p, q, d0), b = x4(2 * p + 1, q, d1);
-        *reinterpret_cast<float4*>(xsf + pair_off(p, ks, q, 0)) = make_float4(a.x, b.x, a.y, b.y);
-        *reinterpret_cast<float4*>(xsf + pair_off(p, ks, q, 1)) = make_float4(a.z, b.z, a.w, b.w);
+        *reinterpret_cast<float4*>(xsf + pair_off(p, ksp, q, 0)) = make_float4(a.x, b.x, a.y, b.y);
+        *reinterpret_cast<float4*>(xsf + pair_off(p, ksp, q, 1)) = make_float4(a.z, b.z, a.w, b.w);
       }
     if constexpr (MASK != kNoMask) load_first();
   } else if constexpr (MASK == kNoMask) {
@@ -266,8 +274,8 @@ gemv_kernel(float* __restrict__ out, const float* __restrict__ X, const float* _
 #pragma unroll
         for (int p = 0; p < MT / 2; ++p) {
           unsigned long long x0, x1, x2, x3;  // columns k, k+1, k+2, k+3 of rows 2p, 2p+1
-          lds_v2b64(xbase + 4u * (uint32_t)pair_off(p, ks, q, 0), x0, x1);
-          lds_v2b64(xbase + 4u * (uint32_t)pair_off(p, ks, q, 1), x2, x3);
+          lds_v2b64(xbase + 4u * (uint32_t)pair_off(p, ksp, q, 0), x0, x1);
+          lds_v2b64(xbase + 4u * (uint32_t)pair_off(p, ksp, q, 1), x2, x3);
 #pragma unroll
           for (int r = 0; r < RQ; ++r) {
             unsigned long long a = acc2[r][p];
@@ -417,7 +425,7 @@ spl_status launch(const LinearArgs& a, const Plan& p, float* part, unsigned int*
                   const KernelNoise& nz = KernelNoise{}) {
   if (!smem_attr_set()) return SPL_ECUDA;
   dim3 grid((unsigned)ceil_div(a.N, rows_per_block(MT)), (unsigned)p.splits);
-  const size_t smem = (size_t)MT * p.k_per_split * sizeof(float);
+  const size_t smem = (size_t)MT * staged_ks(MT, (int)p.k_per_split) * sizeof(float);
   // L2 budget of the early prefetch: about 32 MB over the whole grid, in 128-byte lines per row
   const int64_t rows = (int64_t)grid.x * rows_per_block(MT) * p.splits;
   const int lines = (int)std::min<int64_t>(p.k_per_split / kStep, ((int64_t(32) << 20) / std::max<int64_t>(rows, 1)) >> 7);
@@ -438,7 +446,7 @@ spl_status launch_masked(const LinearArgs& a, const Plan& p, float* part, unsign
 // Resident blocks per SM of the decode kernel for MT rows and a K-slice of ks (cached).
 int blocks_per_sm(int mt, int64_t ks) {
   static std::mutex mu;
-  static int cache[64][5][kMaxKs / kSliceAlign + 1] = {{{0}}};  // device, log2(mt), ks / 128
+  static int cache[64][5][kMaxKs / kSliceAlign + 1] = {{{0}}};  // device, log2(mt), ks / kSliceAlign
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
   if (!smem_attr_set()) return 1;
@@ -449,7 +457,7 @@ int blocks_per_sm(int mt, int64_t ks) {
   if (v == 0) {
     int n = 0;
     const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel_for(mt), THREADS,
-                                                                         (size_t)mt * ks * sizeof(float));
+                                                                         (size_t)mt * staged_ks(mt, (int)ks) * sizeof(float));
     if (e != cudaSuccess) cudaGetLastError();
     v = (e == cudaSuccess && n > 0) ? n : 1;
   }
@@ -463,7 +471,7 @@ int64_t gemv_max_ks(int64_t M) {
 }
 
 // K-split of the decode kernel: the number of splits s minimises waves(s) x (K/s + F), waves
-// counting the resident block slots of all SMs, with K/s a multiple of 128 no larger than 1536
+// counting the resident block slots of all SMs, with K/s a multiple of 64 no larger than 1536
 // (the slice 16 rows can stage, so a correction of up to 16 rows per launch reproduces the
 // online order); F (the fixed cost of a block -- staging X~, the warp reduction, the split-K
 // reduction -- in units of K) measured on GB300.
@@ -476,7 +484,7 @@ Plan plan_gemv(int64_t M, int64_t K, int64_t N, int sms) {
   const int64_t ks_max = kMaxKs;
   const int64_t groups = ceil_div(N, rows_per_block(mt));
   const int64_t s_min = ceil_div(K, ks_max);
-  const int64_t s_max = std::max<int64_t>(s_min, std::min<int64_t>(64, K / 256));
+  const int64_t s_max = std::max<int64_t>(s_min, std::min<int64_t>(64, K / 128));
   double best = 1e300;
   for (int64_t s = s_min; s <= s_max; ++s) {
     const int64_t ks = std::min<int64_t>(round_up(ceil_div(K, s), kSliceAlign), ks_max);
