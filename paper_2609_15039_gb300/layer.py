@@ -849,6 +849,8 @@ class StackIO:
     def __init__(self, stack, host_in, ring=2, sets=None, streams=2):
         if stack.out_pool is None:
             raise ValueError("StackIO: a stack built with stacked=True (pooled outputs)")
+        if streams not in (1, 2):
+            raise ValueError("StackIO: one copy stream or one per direction")
         D = stack.draws
         if sets is None:  # the most sets up to 8 that divide the draws
             sets = max([n for n in range(2, min(D, 8) + 1) if D % n == 0], default=0)
@@ -864,8 +866,6 @@ class StackIO:
         self.dev_in = [{g: torch.zeros(x.shape, device=dev) for g, x in host_in.items()} for _ in range(sets)]
         self.host_out = [{g: torch.empty((L, M, p.shape[-1])).pin_memory() for g, p in stack.out_pool.items()}
                          for _ in range(ring)]
-        if streams not in (1, 2):
-            raise ValueError("StackIO: one copy stream or one per direction")
         self.h2d = torch.cuda.Stream()
         self.d2h = self.h2d if streams == 1 else torch.cuda.Stream()
         self._in, self._done, self._out = {}, {}, {}
